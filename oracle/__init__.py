@@ -1,0 +1,158 @@
+"""fp64 CPU oracle for the MoT KV-cache translation pass (ctypes wrapper).
+
+TEST INFRASTRUCTURE. Only the tests, ``__graft_entry__.smoke()`` and the
+CPU-baseline / reference legs of ``bench.py`` may import this package. The
+product path (the ``paper_2607_28979_gb300`` package and its CUDA library)
+never imports, links or runs it, and this package imports nothing from there.
+
+The arithmetic lives in ``mot_oracle.c``; its header states what is computed
+(Def. 3.1 / Eq. mot_definition, the App. C.2 translator read as the configs'
+Linear-GELU-Linear MLP, the App. C.3 depth-ratio map) and how each part is pinned.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+from typing import Optional, Sequence
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "mot_oracle.c")
+_LIB = os.path.join(_HERE, "libmot_oracle.so")
+
+
+class OracleDims(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in
+                ("L_s", "H_s", "d_s", "L_t", "H_t", "d_t", "E", "top_k", "H", "B", "S", "dtype")]
+
+
+def build(force: bool = False) -> str:
+    """Compile ``libmot_oracle.so`` next to its source if missing or stale."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".{os.getpid()}.tmp"
+        subprocess.check_call(["gcc", "-O2", "-fopenmp", "-shared", "-fPIC", "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+_lib = None
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        lib.oracle_depth_ratio_map.restype = ctypes.c_int
+        lib.oracle_depth_ratio_map.argtypes = [ctypes.c_int32, ctypes.c_int32, P]
+        lib.oracle_gelu.restype = ctypes.c_double
+        lib.oracle_gelu.argtypes = [ctypes.c_double]
+        lib.oracle_bf16_to_double.restype = ctypes.c_double
+        lib.oracle_bf16_to_double.argtypes = [ctypes.c_uint16]
+        lib.oracle_gate_from_logits.restype = None
+        lib.oracle_gate_from_logits.argtypes = [P, ctypes.c_int, ctypes.c_int, P]
+        lib.oracle_translate_tokens.restype = ctypes.c_int
+        lib.oracle_translate_tokens.argtypes = [ctypes.POINTER(OracleDims), P, P, P, P,
+                                                ctypes.c_int64, P, P, P, P, P]
+        lib.oracle_translate_full.restype = ctypes.c_int
+        lib.oracle_translate_full.argtypes = [ctypes.POINTER(OracleDims), P, P, P, P,
+                                              ctypes.c_int32, P, P, P]
+        _lib = lib
+    return _lib
+
+
+def _ptr(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data
+
+
+def dims_of(wl) -> OracleDims:
+    """OracleDims for a ``synth.Workload``-like object."""
+    return OracleDims(wl.n_layers_src, wl.src_kv_heads, wl.src_head_dim,
+                      wl.n_layers_tgt, wl.tgt_kv_heads, wl.tgt_head_dim,
+                      wl.n_translators, wl.top_k, wl.hidden, wl.max_batch, wl.max_seq,
+                      0 if wl.dtype == "bf16" else 1)
+
+
+def depth_ratio_map(L_s: int, L_t: int) -> list:
+    out = np.zeros(L_t, dtype=np.int32)
+    if _load().oracle_depth_ratio_map(L_s, L_t, out.ctypes.data) != 0:
+        raise ValueError("invalid layer counts")
+    return out.tolist()
+
+
+def gelu(x: float) -> float:
+    return float(_load().oracle_gelu(float(x)))
+
+
+def bf16_to_double(bits: int) -> float:
+    return float(_load().oracle_bf16_to_double(bits))
+
+
+def gate_from_logits(logits: Sequence[float], top_k: int = 0) -> np.ndarray:
+    lg = np.ascontiguousarray(logits, dtype=np.float64)
+    g = np.empty_like(lg)
+    _load().oracle_gate_from_logits(lg.ctypes.data, lg.size, top_k, g.ctypes.data)
+    return g
+
+
+def _map_arr(layer_map):
+    return None if layer_map is None else np.ascontiguousarray(layer_map, dtype=np.int32)
+
+
+def translate_tokens(wl, src_k, src_v, blob, tok_b, tok_s, gate_fixed=None, want_gate=False):
+    """Translate sampled tokens. Returns out[L_t][2][n][D_t] (NaN for untranslated
+    layers) and, if ``want_gate``, the kept renormalised gate [L_t][2][n][E]."""
+    tb = np.ascontiguousarray(tok_b, dtype=np.int32)
+    ts = np.ascontiguousarray(tok_s, dtype=np.int32)
+    n = tb.size
+    out = np.full((wl.n_layers_tgt, 2, n, wl.d_tgt), np.nan, dtype=np.float64)
+    gate = np.full((wl.n_layers_tgt, 2, n, wl.n_translators), np.nan) if want_gate else None
+    gf = None if gate_fixed is None else np.ascontiguousarray(gate_fixed, dtype=np.float64)
+    lm = _map_arr(wl.layer_map)
+    d = dims_of(wl)
+    rc = _load().oracle_translate_tokens(ctypes.byref(d), _ptr(lm), _ptr(np.ascontiguousarray(src_k)),
+                                         _ptr(np.ascontiguousarray(src_v)),
+                                         _ptr(np.ascontiguousarray(blob)), n, _ptr(tb), _ptr(ts),
+                                         _ptr(gf), _ptr(out), _ptr(gate))
+    if rc != 0:
+        raise ValueError("oracle_translate_tokens: invalid arguments")
+    return (out, gate) if want_gate else out
+
+
+def translate_full(wl, src_k, src_v, blob, seq_lens, fill=np.nan):
+    """Full translation into double caches shaped like the target cache."""
+    sl = np.ascontiguousarray(seq_lens, dtype=np.int32)
+    dk = np.full(wl.dst_shape(), fill, dtype=np.float64)
+    dv = np.full(wl.dst_shape(), fill, dtype=np.float64)
+    lm = _map_arr(wl.layer_map)
+    d = dims_of(wl)
+    rc = _load().oracle_translate_full(ctypes.byref(d), _ptr(lm), _ptr(np.ascontiguousarray(src_k)),
+                                       _ptr(np.ascontiguousarray(src_v)),
+                                       _ptr(np.ascontiguousarray(blob)), sl.size, _ptr(sl),
+                                       _ptr(dk), _ptr(dv))
+    if rc != 0:
+        raise ValueError("oracle_translate_full: invalid arguments")
+    return dk, dv
+
+
+def sample_tokens(seq_lens, n_per_seq: int, seed: int = 1, tile: int = 128):
+    """A fixed token sample that always includes each sequence's first and last
+    position and the positions on either side of every ``tile`` boundary (the
+    sample layout is test bookkeeping, not method arithmetic)."""
+    rng = np.random.default_rng(seed)
+    tb, ts = [], []
+    for b, L in enumerate(seq_lens):
+        if L <= 0:
+            continue
+        pos = {0, L - 1}
+        for k in range(tile, L, tile * max(1, (L // tile) // 4 or 1)):
+            pos.update({k - 1, k})
+        extra = max(0, n_per_seq - len(pos))
+        if extra:
+            pos.update(rng.integers(0, L, size=extra).tolist())
+        for s in sorted(pos):
+            tb.append(b)
+            ts.append(s)
+    return np.asarray(tb, dtype=np.int32), np.asarray(ts, dtype=np.int32)

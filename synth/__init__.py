@@ -1,0 +1,227 @@
+"""Seeded synthetic workloads for the MoT KV-cache translation pass.
+
+This package draws the inputs that both the fp64 oracle and the CUDA path
+consume: source K/V caches, the packed translator weight blob and the ragged
+sequence lengths. It holds none of the translation method's arithmetic (no
+gate, GELU, layer mapping or combine) -- only random draws, storage rounding
+and the blob's byte layout, which is part of the library interface.
+
+Value recipe (stands in for real model caches and trained translators, which
+are not available):
+  * K, V = s_c * N(0, 1), with a per-channel scale s_c ~ LogNormal(0, 0.5)
+    drawn once per (source layer, K/V, channel c = h*d + i);
+  * every weight and bias ~ N(0, 1/fan_in): fan_in = D_s for the gate and the
+    first translator layer, H for the second;
+  * fp64 draws rounded to fp32, then (bf16 workloads) to bf16 with
+    round-to-nearest-even.
+
+The generator itself (SplitMix64 + Box-Muller) is implemented in ``synth.c``.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+import subprocess
+from typing import Optional, Sequence, Tuple
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "synth.c")
+_LIB = os.path.join(_HERE, "libsynth.so")
+
+# Blob tensor ids, in blob order within one (target layer, K/V) group.
+T_WG, T_BG, T_W1, T_B1, T_W2, T_B2 = range(6)
+
+
+def build(force: bool = False) -> str:
+    """Compile ``libsynth.so`` next to its source if it is missing or stale."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".{os.getpid()}.tmp"
+        subprocess.check_call(
+            ["gcc", "-O2", "-fopenmp", "-shared", "-fPIC", "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+_lib = None
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(build())
+        lib.synth_stream_key.restype = ctypes.c_uint64
+        lib.synth_stream_key.argtypes = [ctypes.c_uint64, ctypes.c_uint64]
+        lib.synth_splitmix64.restype = ctypes.c_uint64
+        lib.synth_splitmix64.argtypes = [ctypes.c_uint64, ctypes.c_uint64]
+        lib.synth_normal_at.restype = ctypes.c_double
+        lib.synth_normal_at.argtypes = [ctypes.c_uint64, ctypes.c_uint64]
+        lib.synth_fill_normal.restype = None
+        lib.synth_fill_normal.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int64,
+                                          ctypes.c_double, ctypes.c_int, ctypes.c_void_p]
+        lib.synth_fill_cache_layer.restype = None
+        lib.synth_fill_cache_layer.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64,
+                                               ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                               ctypes.c_int, ctypes.c_int, ctypes.c_void_p]
+        _lib = lib
+    return _lib
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    """Shapes of one translation workload (mirrors the C ``mot_config``)."""
+    name: str
+    n_layers_src: int
+    src_kv_heads: int
+    src_head_dim: int
+    n_layers_tgt: int
+    tgt_kv_heads: int
+    tgt_head_dim: int
+    n_translators: int
+    hidden: int
+    max_batch: int
+    max_seq: int
+    dtype: str                      # "bf16" or "fp32"
+    seq_lens: Tuple[int, ...]
+    top_k: int = 0                  # 0 (or E) = dense softmax gate
+    layer_map: Optional[Tuple[int, ...]] = None   # None = depth-ratio default; -1 = untranslated
+
+    @property
+    def d_src(self) -> int:
+        return self.src_kv_heads * self.src_head_dim
+
+    @property
+    def d_tgt(self) -> int:
+        return self.tgt_kv_heads * self.tgt_head_dim
+
+    @property
+    def batch(self) -> int:
+        return len(self.seq_lens)
+
+    @property
+    def tokens(self) -> int:
+        return int(sum(self.seq_lens))
+
+    @property
+    def np_dtype(self):
+        return np.uint16 if self.dtype == "bf16" else np.float32
+
+    @property
+    def esize(self) -> int:
+        return 2 if self.dtype == "bf16" else 4
+
+    def translated_layers(self) -> list:
+        """Target layers that receive a translation (all, unless the map says -1)."""
+        if self.layer_map is None:
+            return list(range(self.n_layers_tgt))
+        return [l for l, s in enumerate(self.layer_map) if s >= 0]
+
+    def src_shape(self):
+        return (self.n_layers_src, self.max_batch, self.src_kv_heads, self.max_seq, self.src_head_dim)
+
+    def dst_shape(self):
+        return (self.n_layers_tgt, self.max_batch, self.tgt_kv_heads, self.max_seq, self.tgt_head_dim)
+
+    def group_elems(self) -> int:
+        """Elements of one (target layer, K/V) block of the weight blob."""
+        E, Ds, Dt, H = self.n_translators, self.d_src, self.d_tgt, self.hidden
+        return E * Ds + E + E * (H * Ds + H + Dt * H + Dt)
+
+    def blob_elems(self) -> int:
+        return 2 * len(self.translated_layers()) * self.group_elems()
+
+    def replace(self, **kw) -> "Workload":
+        return dataclasses.replace(self, **kw)
+
+
+# The five workloads: shapes of the paper's model pairs.
+WORKLOADS = {
+    # GPT-2-small (first 4 layers, 12x64) -> OPT-125m-shaped (4 layers, 12x64), fp32.
+    "tiny_fp32": Workload("tiny_fp32", 4, 12, 64, 4, 12, 64, 2, 768, 1, 64, "fp32", (64,)),
+    # GPT-2-small -> OPT-125m, 12 layers each, E=4, MLP 768->1536->768.
+    "gpt2s_opt125m": Workload("gpt2s_opt125m", 12, 12, 64, 12, 12, 64, 4, 1536, 8, 1024, "bf16",
+                              (1024,) * 8),
+    # Qwen2.5-0.5B (24L, 2x64) -> Qwen2.5-1.5B (28L, 2x128), E=4, MLP 128->1024->256.
+    "qwen05_qwen15": Workload("qwen05_qwen15", 24, 2, 64, 28, 2, 128, 4, 1024, 4, 4096, "bf16",
+                              (4096,) * 4),
+    # GPT-2-medium (24L, 16x64) -> Qwen2.5-7B (28L, 4x128), E=8, MLP 1024->2048->512.
+    "gpt2m_qwen7": Workload("gpt2m_qwen7", 24, 16, 64, 28, 4, 128, 8, 2048, 2, 8192, "bf16",
+                            (8192,) * 2),
+    # Qwen2.5-7B -> Qwen2.5-7B (28L, 4x128), ragged batch of 4 long sequences.
+    "qwen7_long": Workload("qwen7_long", 28, 4, 128, 28, 4, 128, 4, 2048, 4, 32768, "bf16",
+                           (32768, 16384, 8192, 4096)),
+}
+
+# Order in which the workloads are listed in the build's benchmark configuration.
+WORKLOAD_ORDER = ["tiny_fp32", "gpt2s_opt125m", "qwen05_qwen15", "gpt2m_qwen7", "qwen7_long"]
+
+
+def _stream_cache(kind: int, x: int, layer: int) -> int:
+    return (kind << 56) | (x << 48) | layer
+
+
+def _stream_weight(layer: int, x: int, expert: int, tensor: int) -> int:
+    return (3 << 56) | (x << 48) | (layer << 24) | (expert << 8) | tensor
+
+
+def gen_cache(wl: Workload, x: int, seed: int = 0) -> np.ndarray:
+    """Source cache for K (x=0) or V (x=1): [L_s][B][H_s][S_max][d_s] in storage dtype."""
+    lib = _load()
+    shape = wl.src_shape()
+    out = np.empty(shape, dtype=wl.np_dtype)
+    dt = 0 if wl.dtype == "bf16" else 1
+    for l in range(wl.n_layers_src):
+        view = out[l]
+        lib.synth_fill_cache_layer(seed, _stream_cache(1, x, l), _stream_cache(2, x, l),
+                                   wl.max_batch, wl.src_kv_heads, wl.max_seq, wl.src_head_dim,
+                                   dt, view.ctypes.data)
+    return out
+
+
+def blob_offsets(wl: Workload):
+    """Yield (target layer, x, tensor id, expert, offset, numel, fan_in) for every blob tensor."""
+    E, Ds, Dt, H = wl.n_translators, wl.d_src, wl.d_tgt, wl.hidden
+    off = 0
+    for l in wl.translated_layers():
+        for x in (0, 1):
+            yield (l, x, T_WG, 0, off, E * Ds, Ds); off += E * Ds
+            yield (l, x, T_BG, 0, off, E, Ds); off += E
+            for m in range(E):
+                yield (l, x, T_W1, m, off, H * Ds, Ds); off += H * Ds
+                yield (l, x, T_B1, m, off, H, Ds); off += H
+                yield (l, x, T_W2, m, off, Dt * H, H); off += Dt * H
+                yield (l, x, T_B2, m, off, Dt, H); off += Dt
+
+
+def gen_weights(wl: Workload, seed: int = 0) -> np.ndarray:
+    """Packed weight blob (flat, storage dtype) in the library's documented order."""
+    lib = _load()
+    out = np.empty(wl.blob_elems(), dtype=wl.np_dtype)
+    dt = 0 if wl.dtype == "bf16" else 1
+    base = out.ctypes.data
+    for (l, x, t, m, off, n, fan_in) in blob_offsets(wl):
+        lib.synth_fill_normal(seed, _stream_weight(l, x, m, t), n, 1.0 / np.sqrt(fan_in), dt,
+                              base + off * wl.esize)
+    assert off + n == out.size
+    return out
+
+
+def seq_lens_array(wl: Workload) -> np.ndarray:
+    return np.asarray(wl.seq_lens, dtype=np.int32)
+
+
+def normal(seed: int, stream: int, n: int) -> np.ndarray:
+    """n fp64 standard-normal draws of one stream (for tests of the generator)."""
+    out = np.empty(n, dtype=np.float64)
+    _load().synth_fill_normal(seed, stream, n, 1.0, 2, out.ctypes.data)
+    return out
+
+
+def splitmix64(key: int, n: int) -> int:
+    return int(_load().synth_splitmix64(key, n))
+
+
+def stream_key(seed: int, stream: int) -> int:
+    return int(_load().synth_stream_key(seed, stream))

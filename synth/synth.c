@@ -1,0 +1,106 @@
+/*
+ * Seeded synthetic inputs for the MoT KV-cache translation pass.
+ *
+ * This module holds NO arithmetic of the translation method. It only draws
+ * random numbers and rounds them to the storage type. Both the fp64 oracle
+ * and the CUDA path consume what it writes, which is why it lives in a module
+ * of its own.
+ *
+ * Generator (published definitions, restated):
+ *   - SplitMix64 (Steele, Lea & Flood, "Fast splittable pseudorandom number
+ *     generators", OOPSLA 2014): output n of a stream with state s0 is
+ *     mix(s0 + (n+1)*GAMMA), GAMMA = 0x9E3779B97F4A7C15, where mix is the
+ *     variant-13 finaliser (shifts 30/27/31, multipliers 0xBF58476D1CE4E5B9,
+ *     0x94D049BB133111EB).
+ *   - Stream key: s0 = mix(seed ^ mix(stream + GAMMA)).
+ *   - Normal draw i of a stream: Box-Muller (1958) on outputs 2i and 2i+1:
+ *     u1 = ((o_{2i} >> 11) + 1) * 2^-53 in (0,1], u2 = (o_{2i+1} >> 11) * 2^-53,
+ *     n = sqrt(-2 ln u1) * cos(2 pi u2).
+ *   - Storage rounding: fp64 -> fp32 (C cast, round-to-nearest-even), then for
+ *     bf16 the fp32 bit pattern is rounded to its top 16 bits with
+ *     round-to-nearest-even.
+ *
+ * Every element depends only on (seed, stream, index), so generation is
+ * parallel (OpenMP) and reproducible.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <string.h>
+
+#define SYNTH_GAMMA 0x9E3779B97F4A7C15ULL
+
+static inline uint64_t synth_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+  return z ^ (z >> 31);
+}
+
+uint64_t synth_stream_key(uint64_t seed, uint64_t stream) {
+  return synth_mix(seed ^ synth_mix(stream + SYNTH_GAMMA));
+}
+
+uint64_t synth_splitmix64(uint64_t key, uint64_t n) {
+  return synth_mix(key + (n + 1) * SYNTH_GAMMA);
+}
+
+double synth_normal_at(uint64_t key, uint64_t i) {
+  const double two_m53 = 1.0 / 9007199254740992.0;
+  uint64_t o1 = synth_splitmix64(key, 2 * i);
+  uint64_t o2 = synth_splitmix64(key, 2 * i + 1);
+  double u1 = (double)((o1 >> 11) + 1) * two_m53;
+  double u2 = (double)(o2 >> 11) * two_m53;
+  return sqrt(-2.0 * log(u1)) * cos(6.283185307179586476925 * u2);
+}
+
+static inline uint16_t f32_to_bf16_rne(float f) {
+  uint32_t u;
+  memcpy(&u, &f, 4);
+  uint32_t lsb = (u >> 16) & 1u;
+  u += 0x7FFFu + lsb;
+  return (uint16_t)(u >> 16);
+}
+
+static inline void store_val(void* out, int64_t idx, double v, int dtype) {
+  float f = (float)v;
+  if (dtype == 0)
+    ((uint16_t*)out)[idx] = f32_to_bf16_rne(f);
+  else
+    ((float*)out)[idx] = f;
+}
+
+/* out[i] = stddev * N_i for i in [0, n); dtype 0 = bf16 bits, 1 = fp32, 2 = fp64. */
+void synth_fill_normal(uint64_t seed, uint64_t stream, int64_t n, double stddev,
+                       int dtype, void* out) {
+  uint64_t key = synth_stream_key(seed, stream);
+#pragma omp parallel for schedule(static)
+  for (int64_t i = 0; i < n; ++i) {
+    double v = stddev * synth_normal_at(key, (uint64_t)i);
+    if (dtype == 2)
+      ((double*)out)[i] = v;
+    else
+      store_val(out, i, v, dtype);
+  }
+}
+
+/*
+ * One layer of a KV cache laid out [B][H][S][d]: value = s_c * N, where the
+ * per-channel scale s_c = exp(0.5 * n_c) ~ LogNormal(0, 0.5) is drawn once per
+ * (layer, K/V, channel c = h*d + i) from `scale_stream` and the values from
+ * `value_stream`.
+ */
+void synth_fill_cache_layer(uint64_t seed, uint64_t scale_stream, uint64_t value_stream,
+                            int B, int H, int S, int d, int dtype, void* out) {
+  uint64_t kscale = synth_stream_key(seed, scale_stream);
+  uint64_t kval = synth_stream_key(seed, value_stream);
+  const int64_t per_b = (int64_t)H * S * d;
+  const int64_t n = (int64_t)B * per_b;
+#pragma omp parallel for schedule(static)
+  for (int64_t idx = 0; idx < n; ++idx) {
+    int64_t r = idx % per_b;
+    int h = (int)(r / ((int64_t)S * d));
+    int i = (int)(r % d);
+    double sc = exp(0.5 * synth_normal_at(kscale, (uint64_t)(h * d + i)));
+    double v = sc * synth_normal_at(kval, (uint64_t)idx);
+    store_val(out, idx, v, dtype);
+  }
+}

@@ -1,0 +1,430 @@
+#!/usr/bin/env python3
+"""Benchmark of the MoT KV-cache translation pass on GB300.
+
+Metric: source-context tokens translated per second into the full target
+cache (sum of seq_lens per mot_translate call, all translated layers, K and V).
+
+One step = one mot_translate call over one synthetic batch of the workload
+(default: the GPT-2-small -> OPT-125m-shaped pair, 12 layers, 12x64 heads,
+E=4 translators 768->1536->768, batch 8 x 1024 tokens), with inputs resident
+in HBM. Every step reads 1.06 GB (source caches, weights, target caches), far
+more than the 129 MB L2, so no flush is needed between steps.
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl mot|reference]
+
+With N > 1 (torchrun) every rank runs an independent replica of the workload
+(the translation shards by token and by layer with no exchange step); value is
+all ranks' tokens over the slowest rank's time. ``--impl reference`` times the
+fp64 CPU oracle on bounded token samples of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np   # noqa: E402
+
+import synth   # noqa: E402
+
+METRIC = "source-context tokens translated/sec into full target cache (1×GB300); % of roofline"
+UNIT = "tokens/s"
+DEFAULT_WORKLOAD = "gpt2s_opt125m"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def workload_desc(wl) -> str:
+    return (f"{wl.name}: {wl.n_layers_src}L {wl.src_kv_heads}x{wl.src_head_dim} -> "
+            f"{wl.n_layers_tgt}L {wl.tgt_kv_heads}x{wl.tgt_head_dim}, E={wl.n_translators} MLP "
+            f"{wl.d_src}-{wl.hidden}-{wl.d_tgt} GELU, dense softmax gate, {wl.dtype}, "
+            f"batch {wl.batch} seq_lens {list(wl.seq_lens)}")
+
+
+def algorithmic(wl, layer_map):
+    """FLOPs and bytes the method needs per step (no intermediate traffic).
+    ``layer_map``: the channel map in use (source layer per target layer, -1 = none)."""
+    T, E, Ds, Dt, Hh = wl.tokens, wl.n_translators, wl.d_src, wl.d_tgt, wl.hidden
+    n_tl = len(wl.translated_layers())
+    groups = 2 * n_tl
+    f_gate = 2 * Ds * E
+    f_g1 = E * 2 * Ds * Hh
+    f_g2 = E * 2 * Hh * Dt + 2 * E * Dt
+    src_layers = {s for s in layer_map if s >= 0}
+    es = wl.esize
+    bytes_src = 2 * len(src_layers) * T * Ds * es
+    bytes_dst = groups * T * Dt * es
+    bytes_w = wl.blob_elems() * es
+    return dict(flops=groups * T * (f_gate + f_g1 + f_g2), flops_gemm1=groups * T * f_g1,
+                flops_gemm2=groups * T * f_g2, bytes=bytes_src + bytes_dst + bytes_w,
+                bytes_src=bytes_src, bytes_dst=bytes_dst, bytes_w=bytes_w)
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+def kernel_source_sha() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2607_28979_gb300", "csrc")
+    for n in sorted(os.listdir(csrc)):
+        if n.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, n), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current kernel sources; else None."""
+    p = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    if not os.path.exists(p):
+        return None
+    sha = kernel_source_sha()
+    for line in open(p):
+        f = dict(kv.split("=", 1) for kv in line.split() if "=" in kv)
+        if f.get("kernel") == kernel and f.get("workload") == workload and f.get("source_sha") == sha:
+            return float(f["bytes_per_launch"])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi samples (every 200 ms) during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="mot_clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        self.proc.wait(timeout=10)
+        rows = []
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 9:
+                rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        smax = [num(r[2]) for r in rows if num(r[2]) is not None]
+        pw = [num(r[3]) for r in rows if num(r[3]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        # samples under load: power above the midpoint of the observed range
+        if pw:
+            thr = (min(pw) + max(pw)) / 2
+            loaded = [num(r[1]) for r in rows if num(r[3]) is not None and num(r[3]) >= thr
+                      and num(r[1]) is not None]
+        else:
+            loaded = sm
+        return {"sm_mhz": statistics.median(loaded or sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None, "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(pw) if pw else None}
+
+
+def dist_setup(gpus: int):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != gpus and world > 1:
+        raise SystemExit(f"--gpus {gpus} but WORLD_SIZE={world}")
+    return world, rank, local
+
+
+def cpu_oracle_rate(wl, sk, sv, blob, budget_s: float, seed: int = 3):
+    """Tokens/s of the fp64 oracle on a bounded token sample (about budget_s)."""
+    import oracle
+    rng = np.random.default_rng(seed)
+
+    def sample(n):
+        b = rng.integers(0, wl.batch, size=n)
+        s = np.array([rng.integers(0, wl.seq_lens[i]) for i in b])
+        return b.astype(np.int32), s.astype(np.int32)
+    c = omp_cores()
+    tb, ts = sample(c)   # one token per thread: measures the parallel throughput
+    t0 = time.perf_counter()
+    oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
+    per_tok = max((time.perf_counter() - t0) / c, 1e-6)
+    n = int(max(c, min(100000, budget_s / per_tok)))
+    tb, ts = sample(n)
+    t0 = time.perf_counter()
+    oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
+    dt = time.perf_counter() - t0
+    return n / dt, n, dt
+
+
+def omp_cores() -> int:
+    v = os.environ.get("OMP_NUM_THREADS")
+    if v and v.isdigit():
+        return int(v)
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def run_reference(args, wl):
+    """The fp64 oracle as the reference arm: each step is a bounded token sample."""
+    world, rank, _ = dist_setup(args.gpus)
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    sk, sv, blob = synth.gen_cache(wl, 0), synth.gen_cache(wl, 1), synth.gen_weights(wl)
+    rng = np.random.default_rng(11)
+    # size the per-step sample to about 2 s of CPU work
+    c = omp_cores()
+    tb = np.zeros(c, np.int32)
+    ts = (np.arange(c) % wl.seq_lens[0]).astype(np.int32)
+    t0 = time.perf_counter()
+    oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
+    per_tok = (time.perf_counter() - t0) / c
+    n = int(max(c, min(4096, 2.0 / max(per_tok, 1e-6))))
+
+    def step():
+        b = rng.integers(0, wl.batch, size=n).astype(np.int32)
+        s = np.array([rng.integers(0, wl.seq_lens[i]) for i in b], dtype=np.int32)
+        t = time.perf_counter()
+        oracle.translate_tokens(wl, sk, sv, blob, b, s)
+        return time.perf_counter() - t
+    for _ in range(args.warmup):
+        step()
+    times = [step() for _ in range(args.steps)]
+    total = sum(times)
+    value = n * args.steps / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * total / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded SplitMix64/Box-Muller caches and weights)",
+        "config": {"workload": workload_desc(wl), "tokens_per_step": n,
+                   "sample": f"{n} random tokens of the workload per step, all {2 * len(wl.translated_layers())} (layer, K/V) groups"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": omp_cores(), "kind": "oracle",
+                         "sample": f"{n} tokens per step x {args.steps} steps"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_mot(args, wl):
+    world, rank, local = dist_setup(args.gpus)
+    import torch
+    import torch.distributed as dist
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2607_28979_gb300 import build as mot_build
+    if rank == 0 or world == 1:
+        mot_build.build()
+    if world > 1:
+        dist.barrier()
+    import paper_2607_28979_gb300.mot as M
+
+    sk_h, sv_h, blob = synth.gen_cache(wl, 0), synth.gen_cache(wl, 1), synth.gen_weights(wl)
+    h = M.mot_create(M.config_from(wl))
+    M.mot_load_weights(h, blob)
+    path = M.mot_get_path(h)
+    bf = wl.dtype == "bf16"
+    tdt = torch.bfloat16 if bf else torch.float32
+
+    def dev(a):
+        t = torch.from_numpy(a.view(np.int16) if bf else a).cuda()
+        return t.view(torch.bfloat16) if bf else t
+    sk, sv = dev(sk_h), dev(sv_h)
+    dk = torch.zeros(wl.dst_shape(), dtype=tdt, device="cuda")
+    dv = torch.zeros(wl.dst_shape(), dtype=tdt, device="cuda")
+    lens = torch.tensor(wl.seq_lens, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.Stream()
+    B = wl.batch
+
+    def step():
+        M.mot_translate(h, sk, sv, lens, B, dk, dv, stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    stream.synchronize()
+    if M.mot_get_device_status(h, stream) != M.MOT_OK:
+        raise SystemExit("device status not OK after warm-up")
+
+    sampler = ClockSampler(local) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    M.mot_profile_enable(h, True)
+    M.mot_profile_read(h)
+    launches0 = M.mot_get_launch_count(h)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    elapsed_ms = e0.elapsed_time(e1)
+    launches = M.mot_get_launch_count(h) - launches0
+    kstats = M.mot_profile_read(h)
+    M.mot_profile_enable(h, False)
+    clocks = sampler.stop() if sampler else None
+    status = M.mot_get_device_status(h, stream)
+    if status != M.MOT_OK:
+        raise SystemExit(f"device status {M.mot_status_string(status)}")
+
+    # ---- end to end through the host-buffer entry point (pinned memory)
+    hk = torch.from_numpy(sk_h.view(np.int16) if bf else sk_h).pin_memory()
+    hv = torch.from_numpy(sv_h.view(np.int16) if bf else sv_h).pin_memory()
+    odt = torch.int16 if bf else torch.float32
+    ok = torch.empty(wl.dst_shape(), dtype=odt).pin_memory()
+    ov = torch.empty(wl.dst_shape(), dtype=odt).pin_memory()
+    lens_h = np.asarray(wl.seq_lens, dtype=np.int32)
+    e2e_steps = max(3, min(args.steps, 50))
+    for _ in range(2):
+        M.mot_translate_host(h, hk, hv, lens_h, B, ok, ov, stream)
+    stream.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        M.mot_translate_host(h, hk, hv, lens_h, B, ok, ov, stream)
+    stream.synchronize()
+    e2e_s = time.perf_counter() - t0
+    es = wl.esize
+    tl = len(wl.translated_layers())
+    h2d = 2 * wl.n_layers_src * wl.tokens * wl.d_src * es + 4 * B
+    d2h = 2 * tl * wl.tokens * wl.d_tgt * es
+
+    # ---- aggregate over ranks: max time
+    t_step = elapsed_ms / args.steps
+    if world > 1:
+        t = torch.tensor([t_step, e2e_s], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        t_step, e2e_s = float(t[0]), float(t[1])
+    tokens = wl.tokens
+    value = world * tokens / (t_step / 1000.0)
+    e2e_value = world * tokens * e2e_steps / e2e_s
+
+    if rank == 0:
+        alg = algorithmic(wl, M.mot_get_layer_map(h))
+        peaks, peak_kind = load_peaks()
+        # dominant kernel: the largest share of device time
+        name, (n_launch, tot_ms) = max(kstats.items(), key=lambda kv: kv[1][1])
+        gp_groups = 2 * tl
+        per_launch_flops = {"umma_gemm1_gelu_gate": alg["flops_gemm1"],
+                            "simt_gemm1_gelu_gate": alg["flops_gemm1"],
+                            "umma_gemm2_combine_store": alg["flops_gemm2"],
+                            "simt_gemm2_combine_store": alg["flops_gemm2"]}
+        launches_per_step = max(1, n_launch // args.steps)
+        if name in per_launch_flops:
+            work = per_launch_flops[name] / launches_per_step
+            avg_s = tot_ms / n_launch / 1000.0
+            achieved = work / avg_s / 1e12
+            peak = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+            roof = {"kernel": name, "bound": "tensor", "achieved": round(achieved, 1),
+                    "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
+                    "peak_kind": f"bf16 dense sustained, {peak_kind}",
+                    "traffic": recorded_traffic(name, wl.name),
+                    "algorithmic_per_launch": work, "avg_launch_ms": tot_ms / n_launch}
+        else:
+            roof = {"kernel": name, "bound": "hbm", "achieved": None, "peak": peaks["hbm_gbs"],
+                    "unit": "GB/s", "frac": None, "traffic": None}
+        # whole-step roofline (the slower of FLOPs at tensor peak and bytes at HBM peak)
+        t_roof = max(alg["flops"] / (peaks["bf16_tflops"] * 1e12), alg["bytes"] / (peaks["hbm_gbs"] * 1e9))
+        cpu = None
+        if world == 1 and not args.no_cpu_baseline:
+            rate, n, dt = cpu_oracle_rate(wl, sk_h, sv_h, blob, budget_s=15.0)
+            cpu = {"value": rate, "unit": UNIT, "cores": omp_cores(), "kind": "oracle",
+                   "sample": f"{n} random tokens x all {2 * tl} (layer, K/V) groups, {dt:.1f} s"}
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": t_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
+            "data": "synthetic (seeded SplitMix64/Box-Muller caches, N(0,1/fan_in) weights)",
+            "config": {"workload": workload_desc(wl), "tokens_per_step": tokens,
+                       "parallelism": "replicas" if world > 1 else "single GPU",
+                       "path": "tcgen05" if path == 1 else "simt",
+                       "l2": "inputs larger than L2 (%.2f GB read+written per step)" % (alg["bytes"] / 1e9)},
+            "roofline": roof,
+            "step_roofline": {"flops": alg["flops"], "bytes": alg["bytes"],
+                              "roofline_ms": 1000 * t_roof,
+                              "frac": round(1000 * t_roof / t_step, 4),
+                              "peaks": f"bf16 {peaks['bf16_tflops']} TFLOP/s burst, HBM {peaks['hbm_gbs']} GB/s ({peak_kind})"},
+            "kernels": {k: {"launches": v[0], "total_ms": round(v[1], 3),
+                            "share": round(v[1] / sum(x[1] for x in kstats.values()), 4)}
+                        for k, v in kstats.items()},
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+                    "api": "mot_translate_host (pinned host buffers)"},
+            "gpu_launches": launches,
+            "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+    M.mot_destroy(h)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=500)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["mot", "reference"], default="mot")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "mot":
+        args.warmup = 3
+    wl = synth.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        return run_reference(args, wl)
+    return run_mot(args, wl)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,176 @@
+/*
+ * mot.h -- C ABI of the GB300 (sm_103a) Mixture-of-Translators KV-cache
+ * translation library (libmot.so).
+ *
+ * The library maps a source LLM's per-layer context KV cache into a target
+ * LLM's cache space (Sec. 2.1, "Translation": KV^{Src,Ctx} -> KV^{Tgt,Ctx}).
+ * For every translated target layer l it reads source layer pi(l) (a channel
+ * (pi(l), l), Sec. 2.1 "Communication"; depth-ratio default, App. C.3), and
+ * for every token u and X in {K, V} (translated independently, App. C.2):
+ *
+ *   g(z_u)         = softmax(Wg z_u + bg)                          (Def. 3.1)
+ *   gtilde         = g renormalised over its Top-K entries         (Def. 3.1)
+ *   Tr_m(z_u)      = W2_m GELU(W1_m z_u + b1_m) + b2_m
+ *   Tr_MoT(z_u)    = sum_{m in Top-K} gtilde_m Tr_m(z_u)            (Eq. mot_definition)
+ *
+ * and writes the result into the target cache in the target's head layout,
+ * with no positional re-encoding (the paper prescribes none).
+ *
+ * Layouts (all row-major, contiguous, caller-owned device memory):
+ *   source cache  src_X[L_s][max_batch][H_s][max_seq][d_s]
+ *   target cache  dst_X[L_t][max_batch][H_t][max_seq][d_t]
+ *   A token vector is its heads concatenated: channel c = h*d + i.
+ *   Element type: bf16 (MOT_BF16) or fp32 (MOT_FP32), the same for caches
+ *   and weights.
+ *
+ * Every call returns a mot_status. Nothing in this library traps, asserts on
+ * the device or spins without a bound: device-side anomalies (a sequence
+ * length outside [0, max_seq], a pipeline wait that exceeded its limit) set a
+ * sticky status word that mot_get_device_status reports.
+ */
+#ifndef MOT_H_
+#define MOT_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+struct CUstream_st;
+typedef struct CUstream_st* mot_stream_t;
+
+typedef enum {
+  MOT_OK = 0,
+  MOT_ERR_INVALID_ARG = 1,   /* NULL / misaligned pointer, bad size or config value */
+  MOT_ERR_UNSUPPORTED = 2,   /* valid but outside what this build implements */
+  MOT_ERR_NO_WEIGHTS = 3,    /* mot_translate before mot_load_weights */
+  MOT_ERR_WEIGHTS_SIZE = 4,  /* blob byte count differs from the config's */
+  MOT_ERR_OOM = 5,           /* device allocation failed */
+  MOT_ERR_CUDA = 6,          /* a CUDA runtime/driver call failed (incl. no GPU) */
+  MOT_ERR_SEQ_LEN = 7,       /* a sequence length was outside [0, max_seq] */
+  MOT_ERR_TIMEOUT = 8        /* a bounded device-side pipeline wait gave up */
+} mot_status;
+
+typedef enum { MOT_BF16 = 0, MOT_FP32 = 1 } mot_dtype;
+
+/*
+ * Shapes of one translation (source model -> target model).
+ * D_s = src_kv_heads * src_head_dim, D_t = tgt_kv_heads * tgt_head_dim.
+ */
+typedef struct {
+  int32_t n_layers_src, src_kv_heads, src_head_dim;
+  int32_t n_layers_tgt, tgt_kv_heads, tgt_head_dim;
+  int32_t n_translators;     /* E = N_Tr, 1..16 (Def. 3.1) */
+  int32_t top_k;             /* 0 or E: dense softmax gate; 1..E-1: Top-K (Def. 3.1) */
+  int32_t hidden;            /* H, translator MLP width */
+  int32_t max_batch;         /* B: batch capacity of the caches, 1..4096 */
+  int32_t max_seq;           /* S_max: sequence capacity of the caches */
+  mot_dtype dtype;           /* caches and weights */
+  const int32_t* layer_map;  /* host [n_layers_tgt]: source layer of each target layer,
+                                -1 = not translated; NULL = depth-ratio map (App. C.3)
+                                pi(l) = round(l*(L_s-1)/(L_t-1)), halves up. Copied. */
+} mot_config;
+
+typedef struct mot_ctx* mot_handle;
+
+/*
+ * Validate `cfg` and create a handle on the CURRENT CUDA device. Allocates the
+ * device weight storage and the translation workspace (the translate calls
+ * allocate nothing). Config errors are reported before any CUDA call.
+ * Errors: MOT_ERR_INVALID_ARG (cfg/out NULL, non-positive sizes, top_k outside
+ * [0, E], a layer_map entry outside [-1, L_s)), MOT_ERR_UNSUPPORTED (E > 16,
+ * max_batch > 4096), MOT_ERR_CUDA (no usable device), MOT_ERR_OOM.
+ * On error *out is set to NULL.
+ */
+mot_status mot_create(const mot_config* cfg, mot_handle* out);
+
+/*
+ * Upload the translator weights from a host blob (synchronous; the blob may
+ * be freed on return). Blob layout, all elements in cfg.dtype, for every
+ * translated target layer l in ascending order, then X = K, V:
+ *   Wg[E][D_s], bg[E],
+ *   then for m = 0..E-1:  W1[H][D_s], b1[H], W2[D_t][H], b2[D_t]
+ * (nn.Linear (out, in) convention). `bytes` must equal that size exactly.
+ * The library repacks the weights into its own device layout.
+ * Errors: MOT_ERR_INVALID_ARG, MOT_ERR_WEIGHTS_SIZE, MOT_ERR_CUDA.
+ */
+mot_status mot_load_weights(mot_handle h, const void* host_blob, size_t bytes);
+
+/*
+ * Translate (Eq. mot_definition) the source caches into the target caches.
+ * src_k, src_v, dst_k, dst_v: device pointers, 16-byte aligned, in the layouts
+ * above. seq_lens: DEVICE int32[batch], batch <= max_batch; token (b, s) is
+ * translated for s < seq_lens[b]. Only those positions of translated layers
+ * are written; padding positions, batch entries >= batch and untranslated
+ * layers keep their contents. A length outside [0, max_seq] is clamped into
+ * that range and reported later by mot_get_device_status (MOT_ERR_SEQ_LEN).
+ * Asynchronous on `stream`: no host synchronisation, no allocation. One
+ * handle must not run two translations concurrently (shared workspace).
+ * Errors: MOT_ERR_INVALID_ARG (NULL/misaligned pointers, batch outside
+ * [0, max_batch], dst aliasing src), MOT_ERR_NO_WEIGHTS, MOT_ERR_CUDA.
+ */
+mot_status mot_translate(mot_handle h, const void* src_k, const void* src_v,
+                         const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
+                         mot_stream_t stream);
+
+/*
+ * The same translation with HOST buffers (pinned memory recommended): copies
+ * the real tokens of src_k/src_v and seq_lens (host int32[batch]) to
+ * library-owned device staging, translates, and copies the translated
+ * positions back into dst_k/dst_v, all enqueued on `stream`. The call returns
+ * once the work is enqueued; synchronise `stream` before reading dst. The
+ * staging buffers are allocated on the first call and freed by mot_destroy.
+ * Errors: as mot_translate, plus MOT_ERR_SEQ_LEN for a host length outside
+ * [0, max_seq] (nothing is enqueued then) and MOT_ERR_OOM.
+ */
+mot_status mot_translate_host(mot_handle h, const void* src_k, const void* src_v,
+                              const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
+                              mot_stream_t stream);
+
+/*
+ * Synchronise `stream`, then report and clear the sticky device status word:
+ * MOT_ERR_SEQ_LEN, MOT_ERR_TIMEOUT, or MOT_OK. MOT_ERR_CUDA if the stream
+ * reports an error.
+ */
+mot_status mot_get_device_status(mot_handle h, mot_stream_t stream);
+
+/* Free every device resource of the handle (synchronises the device first). */
+mot_status mot_destroy(mot_handle h);
+
+/* Static, human-readable name of a status code. */
+const char* mot_status_string(mot_status s);
+
+/* ---- introspection (no method counterpart; for tests and benchmarks) ------ */
+
+/* The channel map in use: out[n_layers_tgt] (n must equal n_layers_tgt). */
+mot_status mot_get_layer_map(mot_handle h, int32_t* out, int32_t n);
+
+/* Which kernel path translate uses: 1 = tcgen05/TMA bf16 GEMMs, 0 = SIMT. */
+mot_status mot_get_path(mot_handle h, int32_t* path);
+
+/*
+ * Per-kernel timing. While enabled, every kernel that translate launches is
+ * bracketed by CUDA events on the launching stream. mot_profile_read
+ * synchronises those events, writes up to `cap` records (one per kernel
+ * name, in first-launch order) and clears the collected events.
+ */
+typedef struct {
+  char name[32];
+  int64_t launches;
+  double total_ms;
+} mot_kernel_stat;
+
+mot_status mot_profile_enable(mot_handle h, int32_t enable);
+mot_status mot_profile_read(mot_handle h, mot_kernel_stat* out, int32_t cap, int32_t* n);
+
+/* Number of kernels this handle has launched since it was created. */
+mot_status mot_get_launch_count(mot_handle h, int64_t* count);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MOT_H_ */

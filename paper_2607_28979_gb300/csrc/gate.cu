@@ -1,0 +1,213 @@
+// Ragged token-tile list and the per-token gate (Def. 3.1).
+#include <cuda_bf16.h>
+
+#include "mot_internal.h"
+
+namespace mot {
+
+// ---------------------------------------------------------------- tile list
+
+// One block. Clamps every length into [0, S] (flagging kStatusSeqLen), then
+// lays the 128-token tiles of all batch entries out contiguously: tile i
+// covers rows [i*128, i*128+128) of the gate / A2 workspaces.
+__global__ void prep_tiles_kernel(const int32_t* __restrict__ seq_lens, int32_t batch, int32_t S,
+                                  TileInfo* __restrict__ tiles, int32_t* __restrict__ n_tiles,
+                                  int32_t* __restrict__ status) {
+  __shared__ int32_t s_len[4096];
+  __shared__ int32_t s_off[4096];
+  for (int b = threadIdx.x; b < batch; b += blockDim.x) {
+    int32_t L = seq_lens[b];
+    if (L < 0 || L > S) {
+      atomicOr(status, kStatusSeqLen);
+      L = L < 0 ? 0 : S;
+    }
+    s_len[b] = L;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int32_t acc = 0;
+    for (int b = 0; b < batch; ++b) {
+      s_off[b] = acc;
+      acc += (s_len[b] + kTileM - 1) / kTileM;
+    }
+    *n_tiles = acc;
+  }
+  __syncthreads();
+  for (int b = threadIdx.x; b < batch; b += blockDim.x) {
+    const int32_t L = s_len[b];
+    const int32_t nt = (L + kTileM - 1) / kTileM;
+    for (int t = 0; t < nt; ++t) {
+      TileInfo ti;
+      ti.b = b;
+      ti.s0 = t * kTileM;
+      ti.rows = min(kTileM, L - t * kTileM);
+      ti.pad = 0;
+      tiles[s_off[b] + t] = ti;
+    }
+  }
+}
+
+cudaError_t launch_prep(const int32_t* seq_lens, int32_t batch, const Dims& d, TileInfo* tiles,
+                        int32_t* n_tiles, int32_t* status, cudaStream_t st) {
+  prep_tiles_kernel<<<1, 256, 0, st>>>(seq_lens, batch, d.S, tiles, n_tiles, status);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- gate
+
+template <typename T>
+struct Vec;
+template <>
+struct Vec<__nv_bfloat16> {
+  static constexpr int N = 8;   // 16-byte loads
+  __device__ static void load(const __nv_bfloat16* p, float (&v)[8]) {
+    const uint4 u = *reinterpret_cast<const uint4*>(p);
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 f = __bfloat1622float2(h[k]);
+      v[2 * k] = f.x;
+      v[2 * k + 1] = f.y;
+    }
+  }
+};
+template <>
+struct Vec<float> {
+  static constexpr int N = 4;
+  __device__ static void load(const float* p, float (&v)[4]) {
+    const float4 u = *reinterpret_cast<const float4*>(p);
+    v[0] = u.x; v[1] = u.y; v[2] = u.z; v[3] = u.w;
+  }
+};
+
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+// Grid (tiles_max, G), 256 threads: each warp produces the gate of 16 token
+// rows of one tile for one (layer, K/V) group. Lanes split the D_s channels
+// (VEC-wide vectors when the head dim allows it), reduce the E logits with
+// warp shuffles, and lane 0 applies the max-subtracted softmax and the Top-K
+// renormalisation. Rows past the tile's length get a zero gate.
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(256) gate_kernel(PathArgs a) {
+  const Dims& d = a.d;
+  const int m = blockIdx.x;
+  const int grp = blockIdx.y;
+  if (m >= *a.n_tiles) return;
+  const TileInfo ti = a.tiles[m];
+  const GroupInfo gi = a.groups[grp];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int E = d.E;
+  const T* __restrict__ src = static_cast<const T*>(a.src[gi.x]);
+  const T* __restrict__ wg = static_cast<const T*>(a.wg) + static_cast<size_t>(grp) * E * d.Ds;
+  const float* __restrict__ bg = a.bg + static_cast<size_t>(grp) * E;
+  constexpr int NV = VEC ? Vec<T>::N : 1;
+
+  for (int r = warp; r < kTileM; r += 8) {
+    float* __restrict__ gout = a.gate + (static_cast<size_t>(grp) * d.tpad + static_cast<size_t>(m) * kTileM + r) * E;
+    if (r >= ti.rows) {
+      if (lane < E) gout[lane] = 0.f;
+      continue;
+    }
+    const int s = ti.s0 + r;
+    float acc[kMaxE];
+#pragma unroll
+    for (int e = 0; e < kMaxE; ++e) acc[e] = 0.f;
+    for (int c = lane * NV; c < d.Ds; c += 32 * NV) {
+      const int h = c / d.d_s, i = c - h * d.d_s;
+      const T* zp = src + ((((static_cast<size_t>(gi.src_layer) * d.B + ti.b) * d.H_s + h) * d.S + s) * d.d_s + i);
+      float z[NV];
+      if constexpr (VEC) {
+        Vec<T>::load(zp, z);
+      } else {
+        z[0] = to_f(*zp);
+      }
+#pragma unroll
+      for (int e = 0; e < kMaxE; ++e) {
+        if (e < E) {
+          float w[NV];
+          if constexpr (VEC) {
+            Vec<T>::load(wg + static_cast<size_t>(e) * d.Ds + c, w);
+          } else {
+            w[0] = to_f(wg[static_cast<size_t>(e) * d.Ds + c]);
+          }
+#pragma unroll
+          for (int k = 0; k < NV; ++k) acc[e] = fmaf(w[k], z[k], acc[e]);
+        }
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < kMaxE; ++e) {
+      if (e < E) {
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) acc[e] += __shfl_xor_sync(0xffffffffu, acc[e], off);
+      }
+    }
+    if (lane == 0) {
+      float g[kMaxE];
+      float mx = -INFINITY;
+#pragma unroll
+      for (int e = 0; e < kMaxE; ++e)
+        if (e < E) {
+          g[e] = acc[e] + bg[e];
+          mx = fmaxf(mx, g[e]);
+        }
+      float sum = 0.f;
+#pragma unroll
+      for (int e = 0; e < kMaxE; ++e)
+        if (e < E) {
+          g[e] = expf(g[e] - mx);
+          sum += g[e];
+        }
+      const float inv = 1.f / sum;
+#pragma unroll
+      for (int e = 0; e < kMaxE; ++e)
+        if (e < E) g[e] *= inv;
+      if (d.top_k > 0 && d.top_k < E) {
+        // keep the top_k largest scores (equal scores: lower index first)
+        uint32_t keep = 0;
+        for (int k = 0; k < d.top_k; ++k) {
+          int best = -1;
+          float bv = 0.f;
+#pragma unroll
+          for (int e = 0; e < kMaxE; ++e)
+            if (e < E && !((keep >> e) & 1u) && (best < 0 || g[e] > bv)) {
+              best = e;
+              bv = g[e];
+            }
+          keep |= 1u << best;
+        }
+        float ks = 0.f;
+#pragma unroll
+        for (int e = 0; e < kMaxE; ++e)
+          if (e < E && ((keep >> e) & 1u)) ks += g[e];
+        const float kinv = 1.f / ks;
+#pragma unroll
+        for (int e = 0; e < kMaxE; ++e)
+          if (e < E) g[e] = ((keep >> e) & 1u) ? g[e] * kinv : 0.f;
+      }
+#pragma unroll
+      for (int e = 0; e < kMaxE; ++e)
+        if (e < E) gout[e] = g[e];
+    }
+  }
+}
+
+cudaError_t launch_gate(const PathArgs& a, cudaStream_t st) {
+  const Dims& d = a.d;
+  dim3 grid(d.tiles_max, d.G);
+  if (d.dtype == 0) {
+    if (d.d_s % 8 == 0)
+      gate_kernel<__nv_bfloat16, true><<<grid, 256, 0, st>>>(a);
+    else
+      gate_kernel<__nv_bfloat16, false><<<grid, 256, 0, st>>>(a);
+  } else {
+    if (d.d_s % 4 == 0)
+      gate_kernel<float, true><<<grid, 256, 0, st>>>(a);
+    else
+      gate_kernel<float, false><<<grid, 256, 0, st>>>(a);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace mot

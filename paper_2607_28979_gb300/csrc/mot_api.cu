@@ -1,0 +1,627 @@
+// C ABI of libmot.so: handle lifetime, weight repacking, argument checking and
+// the launch sequence of one translation (see include/mot.h).
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <algorithm>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "mot_internal.h"
+
+using namespace mot;
+
+namespace {
+
+// Upper bound on the A2 workspace; groups are translated in passes of `gp`
+// groups so that gp * tpad * E*H elements fit in it.
+constexpr size_t kA2Budget = size_t(8) << 30;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static bool tried = false;
+  if (!tried) {
+    tried = true;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// bf16 tensor map with 128-byte swizzle; dims[0] is the contiguous one.
+bool encode_bf16(CUtensorMap* map, const void* base, int rank, const uint64_t* dims,
+                 const uint64_t* strides_bytes, const uint32_t* box) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t gd[5], gs[4];
+  cuuint32_t bx[5], es[5];
+  for (int i = 0; i < rank; ++i) {
+    gd[i] = dims[i];
+    bx[i] = box[i];
+    es[i] = 1;
+  }
+  for (int i = 0; i < rank - 1; ++i) gs[i] = strides_bytes[i];
+  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), gd, gs, bx,
+                  es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+struct Ev {
+  cudaEvent_t a, b;
+  int kind;
+};
+
+}  // namespace
+
+struct mot_ctx {
+  mot_config cfg{};
+  std::vector<int32_t> layer_map;
+  Dims d{};
+  int device = 0;
+  int num_sms = 0;
+  bool use_umma = false;
+  bool weights_loaded = false;
+  int gp_max = 1;
+  std::vector<GroupInfo> groups_h;
+
+  // weights (library layout, see PathArgs)
+  void* wg = nullptr;
+  float* bg = nullptr;
+  void* w1 = nullptr;
+  float* b1 = nullptr;
+  void* w2 = nullptr;
+  float* b2 = nullptr;
+  GroupInfo* groups = nullptr;
+  // workspace
+  float* gate = nullptr;
+  void* a2 = nullptr;
+  TileInfo* tiles = nullptr;
+  int32_t* n_tiles = nullptr;
+  int32_t* status = nullptr;
+  // tensor maps that do not depend on the caller's buffers
+  CUtensorMap tm_w1{}, tm_w2{}, tm_a2{};
+  // host-buffer staging for mot_translate_host (allocated on first use)
+  void* st_src[2] = {nullptr, nullptr};
+  void* st_dst[2] = {nullptr, nullptr};
+  int32_t* st_len = nullptr;
+  // profiling
+  bool profile = false;
+  std::vector<Ev> ev_used, ev_free;
+  std::vector<std::string> kind_names;
+  int64_t launches = 0;
+};
+
+namespace {
+
+size_t esize(const Dims& d) { return d.dtype == 0 ? 2 : 4; }
+size_t src_bytes(const Dims& d) {
+  return size_t(d.L_s) * d.B * d.H_s * size_t(d.S) * d.d_s * esize(d);
+}
+size_t dst_bytes(const Dims& d) {
+  return size_t(d.L_t) * d.B * d.H_t * size_t(d.S) * d.d_t * esize(d);
+}
+size_t group_elems(const Dims& d) {
+  const size_t E = d.E, Ds = d.Ds, Dt = d.Dt, H = d.H;
+  return E * Ds + E + E * (H * Ds + H + Dt * H + Dt);
+}
+
+void free_all(mot_ctx* h) {
+  void* ptrs[] = {h->wg, h->bg, h->w1, h->b1, h->w2, h->b2, h->groups, h->gate, h->a2, h->tiles,
+                  h->n_tiles, h->status, h->st_src[0], h->st_src[1], h->st_dst[0], h->st_dst[1],
+                  h->st_len};
+  for (void* p : ptrs)
+    if (p) cudaFree(p);
+  for (auto& e : h->ev_used) { cudaEventDestroy(e.a); cudaEventDestroy(e.b); }
+  for (auto& e : h->ev_free) { cudaEventDestroy(e.a); cudaEventDestroy(e.b); }
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool overlap(const void* a, size_t na, const void* b, size_t nb) {
+  const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+  return x < y + nb && y < x + na;
+}
+
+int kind_id(mot_ctx* h, const char* name) {
+  for (size_t i = 0; i < h->kind_names.size(); ++i)
+    if (h->kind_names[i] == name) return static_cast<int>(i);
+  h->kind_names.emplace_back(name);
+  return static_cast<int>(h->kind_names.size() - 1);
+}
+
+// Launch wrapper: counts the launch and, when profiling, brackets it with events.
+template <class F>
+cudaError_t timed(mot_ctx* h, const char* name, cudaStream_t st, F&& launch) {
+  Ev ev{};
+  if (h->profile) {
+    if (!h->ev_free.empty()) {
+      ev = h->ev_free.back();
+      h->ev_free.pop_back();
+    } else {
+      if (cudaEventCreate(&ev.a) != cudaSuccess || cudaEventCreate(&ev.b) != cudaSuccess)
+        return cudaErrorMemoryAllocation;
+    }
+    ev.kind = kind_id(h, name);
+    cudaEventRecord(ev.a, st);
+  }
+  cudaError_t e = launch();
+  ++h->launches;
+  if (h->profile) {
+    cudaEventRecord(ev.b, st);
+    h->ev_used.push_back(ev);
+  }
+  return e;
+}
+
+mot_status validate(const mot_config* c) {
+  if (c->n_layers_src <= 0 || c->src_kv_heads <= 0 || c->src_head_dim <= 0 ||
+      c->n_layers_tgt <= 0 || c->tgt_kv_heads <= 0 || c->tgt_head_dim <= 0 ||
+      c->n_translators <= 0 || c->hidden <= 0 || c->max_batch <= 0 || c->max_seq <= 0)
+    return MOT_ERR_INVALID_ARG;
+  if (c->top_k < 0 || c->top_k > c->n_translators) return MOT_ERR_INVALID_ARG;
+  if (c->dtype != MOT_BF16 && c->dtype != MOT_FP32) return MOT_ERR_INVALID_ARG;
+  if (c->layer_map)
+    for (int l = 0; l < c->n_layers_tgt; ++l)
+      if (c->layer_map[l] < -1 || c->layer_map[l] >= c->n_layers_src) return MOT_ERR_INVALID_ARG;
+  if (c->n_translators > kMaxE || c->max_batch > 4096) return MOT_ERR_UNSUPPORTED;
+  // index arithmetic inside the kernels uses 32-bit tile and row counts
+  const long long tiles = (long long)c->max_batch * ((c->max_seq + kTileM - 1) / kTileM);
+  if (tiles * kTileM > INT32_MAX / 2) return MOT_ERR_UNSUPPORTED;
+  if ((long long)c->n_translators * c->hidden > (1 << 24)) return MOT_ERR_UNSUPPORTED;
+  return MOT_OK;
+}
+
+// Depth-ratio channel map (App. C.3): round(l*(L_s-1)/(L_t-1)), halves up.
+void depth_ratio(int L_s, int L_t, std::vector<int32_t>& out) {
+  out.resize(L_t);
+  for (int l = 0; l < L_t; ++l) {
+    if (L_t == 1) { out[l] = 0; continue; }
+    const long long num = (long long)l * (L_s - 1), den = L_t - 1;
+    out[l] = static_cast<int32_t>((2 * num + den) / (2 * den));
+  }
+}
+
+PathArgs path_args(mot_ctx* h) {
+  PathArgs a{};
+  a.d = h->d;
+  a.tiles = h->tiles;
+  a.n_tiles = h->n_tiles;
+  a.groups = h->groups;
+  a.wg = h->wg;
+  a.bg = h->bg;
+  a.w1 = h->w1;
+  a.b1 = h->b1;
+  a.w2 = h->w2;
+  a.b2 = h->b2;
+  a.gate = h->gate;
+  a.a2 = h->a2;
+  a.status = h->status;
+  return a;
+}
+
+#define MOT_CUDA_TRY(x)                 \
+  do {                                  \
+    if ((x) != cudaSuccess) {           \
+      cudaGetLastError();               \
+      return MOT_ERR_CUDA;              \
+    }                                   \
+  } while (0)
+
+mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const int32_t* seq_lens,
+                         int32_t batch, void* dst_k, void* dst_v, cudaStream_t st) {
+  const Dims& d = h->d;
+  if (batch == 0 || d.G == 0) return MOT_OK;
+  PathArgs a = path_args(h);
+  a.src[0] = src_k;
+  a.src[1] = src_v;
+  a.dst[0] = dst_k;
+  a.dst[1] = dst_v;
+
+  CUtensorMap tmK{}, tmV{};
+  if (h->use_umma) {
+    const uint64_t dims[5] = {uint64_t(d.d_s), uint64_t(d.S), uint64_t(d.H_s), uint64_t(d.B),
+                              uint64_t(d.L_s)};
+    const uint64_t st_b[4] = {uint64_t(d.d_s) * 2, uint64_t(d.S) * d.d_s * 2,
+                              uint64_t(d.H_s) * d.S * d.d_s * 2,
+                              uint64_t(d.B) * d.H_s * d.S * d.d_s * 2};
+    const uint32_t box[5] = {uint32_t(kUmmaK), uint32_t(kTileM), 1, 1, 1};
+    if (!encode_bf16(&tmK, src_k, 5, dims, st_b, box) ||
+        !encode_bf16(&tmV, src_v, 5, dims, st_b, box))
+      return MOT_ERR_CUDA;
+  }
+
+  MOT_CUDA_TRY(timed(h, "prep_tiles", st, [&] {
+    return launch_prep(seq_lens, batch, d, h->tiles, h->n_tiles, h->status, st);
+  }));
+  MOT_CUDA_TRY(timed(h, "gate", st, [&] { return launch_gate(a, st); }));
+  for (int g0 = 0; g0 < d.G; g0 += h->gp_max) {
+    a.g0 = g0;
+    a.gp = std::min(h->gp_max, d.G - g0);
+    if (h->use_umma) {
+      MOT_CUDA_TRY(timed(h, "umma_gemm1_gelu_gate", st, [&] {
+        return launch_umma_gemm1(a, tmK, tmV, h->tm_w1, h->num_sms, st);
+      }));
+      MOT_CUDA_TRY(timed(h, "umma_gemm2_combine_store", st, [&] {
+        return launch_umma_gemm2(a, h->tm_a2, h->tm_w2, h->num_sms, st);
+      }));
+    } else {
+      MOT_CUDA_TRY(timed(h, "simt_gemm1_gelu_gate", st, [&] { return launch_simt_gemm1(a, st); }));
+      MOT_CUDA_TRY(timed(h, "simt_gemm2_combine_store", st, [&] { return launch_simt_gemm2(a, st); }));
+    }
+  }
+  return MOT_OK;
+}
+
+mot_status check_translate_args(mot_ctx* h, const void* src_k, const void* src_v,
+                                const int32_t* seq_lens, int32_t batch, const void* dst_k,
+                                const void* dst_v) {
+  if (!h) return MOT_ERR_INVALID_ARG;
+  if (batch < 0 || batch > h->d.B) return MOT_ERR_INVALID_ARG;
+  if (!src_k || !src_v || !dst_k || !dst_v || (batch > 0 && !seq_lens)) return MOT_ERR_INVALID_ARG;
+  if (!aligned16(src_k) || !aligned16(src_v) || !aligned16(dst_k) || !aligned16(dst_v))
+    return MOT_ERR_INVALID_ARG;
+  const size_t sb = src_bytes(h->d), db = dst_bytes(h->d);
+  if (overlap(dst_k, db, dst_v, db) || overlap(dst_k, db, src_k, sb) ||
+      overlap(dst_k, db, src_v, sb) || overlap(dst_v, db, src_k, sb) ||
+      overlap(dst_v, db, src_v, sb))
+    return MOT_ERR_INVALID_ARG;
+  if (!h->weights_loaded) return MOT_ERR_NO_WEIGHTS;
+  return MOT_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* mot_status_string(mot_status s) {
+  switch (s) {
+    case MOT_OK: return "MOT_OK";
+    case MOT_ERR_INVALID_ARG: return "MOT_ERR_INVALID_ARG";
+    case MOT_ERR_UNSUPPORTED: return "MOT_ERR_UNSUPPORTED";
+    case MOT_ERR_NO_WEIGHTS: return "MOT_ERR_NO_WEIGHTS";
+    case MOT_ERR_WEIGHTS_SIZE: return "MOT_ERR_WEIGHTS_SIZE";
+    case MOT_ERR_OOM: return "MOT_ERR_OOM";
+    case MOT_ERR_CUDA: return "MOT_ERR_CUDA";
+    case MOT_ERR_SEQ_LEN: return "MOT_ERR_SEQ_LEN";
+    case MOT_ERR_TIMEOUT: return "MOT_ERR_TIMEOUT";
+  }
+  return "MOT_ERR_UNKNOWN";
+}
+
+mot_status mot_create(const mot_config* cfg, mot_handle* out) {
+  if (!out) return MOT_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg) return MOT_ERR_INVALID_ARG;
+  mot_status vs = validate(cfg);
+  if (vs != MOT_OK) return vs;
+
+  mot_ctx* h = new (std::nothrow) mot_ctx();
+  if (!h) return MOT_ERR_OOM;
+  h->cfg = *cfg;
+  if (cfg->layer_map)
+    h->layer_map.assign(cfg->layer_map, cfg->layer_map + cfg->n_layers_tgt);
+  else
+    depth_ratio(cfg->n_layers_src, cfg->n_layers_tgt, h->layer_map);
+  h->cfg.layer_map = nullptr;
+
+  Dims& d = h->d;
+  d.L_s = cfg->n_layers_src; d.H_s = cfg->src_kv_heads; d.d_s = cfg->src_head_dim;
+  d.L_t = cfg->n_layers_tgt; d.H_t = cfg->tgt_kv_heads; d.d_t = cfg->tgt_head_dim;
+  d.E = cfg->n_translators; d.top_k = cfg->top_k; d.H = cfg->hidden;
+  d.B = cfg->max_batch; d.S = cfg->max_seq;
+  d.Ds = d.H_s * d.d_s; d.Dt = d.H_t * d.d_t; d.EH = d.E * d.H;
+  d.dtype = cfg->dtype == MOT_BF16 ? 0 : 1;
+  d.tiles_max = d.B * ((d.S + kTileM - 1) / kTileM);
+  d.tpad = d.tiles_max * kTileM;
+  for (int l = 0; l < d.L_t; ++l)
+    if (h->layer_map[l] >= 0)
+      for (int x = 0; x < 2; ++x) h->groups_h.push_back(GroupInfo{l, h->layer_map[l], x, 0});
+  d.G = static_cast<int32_t>(h->groups_h.size());
+
+  int dev = 0, cc_major = 0, cc_minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&cc_major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&cc_minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess) {
+    cudaGetLastError();
+    delete h;
+    return MOT_ERR_CUDA;
+  }
+  h->device = dev;
+  if (cc_major != 10 || cc_minor != 3) {   // the kernels are built for sm_103a only
+    delete h;
+    return MOT_ERR_UNSUPPORTED;
+  }
+  h->use_umma = umma_supported(d) && encode_fn() != nullptr;
+
+  const size_t es = esize(d), G = d.G, E = d.E, EH = d.EH;
+  const size_t a2_row = EH * (h->use_umma ? 2 : 4);
+  const size_t per_group_a2 = size_t(d.tpad) * a2_row;
+  h->gp_max = static_cast<int>(std::max<size_t>(1, std::min<size_t>(G ? G : 1, kA2Budget / per_group_a2)));
+  if (G) {   // balance the passes
+    const int passes = (d.G + h->gp_max - 1) / h->gp_max;
+    h->gp_max = (d.G + passes - 1) / passes;
+  }
+  struct A { void** p; size_t n; } allocs[] = {
+      {&h->wg, G * E * d.Ds * es}, {(void**)&h->bg, G * E * 4},
+      {&h->w1, G * EH * d.Ds * es}, {(void**)&h->b1, G * EH * 4},
+      {&h->w2, G * d.Dt * EH * es}, {(void**)&h->b2, G * E * d.Dt * 4},
+      {(void**)&h->groups, std::max<size_t>(G, 1) * sizeof(GroupInfo)},
+      {(void**)&h->gate, G * size_t(d.tpad) * E * 4},
+      {&h->a2, size_t(h->gp_max) * per_group_a2},
+      {(void**)&h->tiles, size_t(d.tiles_max) * sizeof(TileInfo)},
+      {(void**)&h->n_tiles, 16}, {(void**)&h->status, 16}};
+  for (auto& a : allocs) {
+    if (cudaMalloc(a.p, std::max<size_t>(a.n, 16)) != cudaSuccess) {
+      cudaGetLastError();
+      free_all(h);
+      delete h;
+      return MOT_ERR_OOM;
+    }
+  }
+  if (cudaMemset(h->status, 0, 16) != cudaSuccess || cudaMemset(h->n_tiles, 0, 16) != cudaSuccess ||
+      (G && cudaMemcpy(h->groups, h->groups_h.data(), G * sizeof(GroupInfo),
+                       cudaMemcpyHostToDevice) != cudaSuccess)) {
+    cudaGetLastError();
+    free_all(h);
+    delete h;
+    return MOT_ERR_CUDA;
+  }
+  if (h->use_umma && G) {
+    bool ok = true;
+    {  // W1cat: [G*EH rows][Ds], box 64 x 256
+      const uint64_t dims[2] = {uint64_t(d.Ds), uint64_t(G * EH)};
+      const uint64_t st_b[1] = {uint64_t(d.Ds) * 2};
+      const uint32_t box[2] = {uint32_t(kUmmaK), uint32_t(kUmmaN)};
+      ok = ok && encode_bf16(&h->tm_w1, h->w1, 2, dims, st_b, box);
+    }
+    {  // W2cat: [G*Dt rows][EH], box 64 x 256
+      const uint64_t dims[2] = {uint64_t(EH), uint64_t(G * d.Dt)};
+      const uint64_t st_b[1] = {uint64_t(EH) * 2};
+      const uint32_t box[2] = {uint32_t(kUmmaK), uint32_t(kUmmaN)};
+      ok = ok && encode_bf16(&h->tm_w2, h->w2, 2, dims, st_b, box);
+    }
+    {  // A2: [gp][tpad][EH], box 64 x 128 x 1
+      const uint64_t dims[3] = {uint64_t(EH), uint64_t(d.tpad), uint64_t(h->gp_max)};
+      const uint64_t st_b[2] = {uint64_t(EH) * 2, uint64_t(d.tpad) * EH * 2};
+      const uint32_t box[3] = {uint32_t(kUmmaK), uint32_t(kTileM), 1};
+      ok = ok && encode_bf16(&h->tm_a2, h->a2, 3, dims, st_b, box);
+    }
+    if (!ok) {
+      free_all(h);
+      delete h;
+      return MOT_ERR_CUDA;
+    }
+  }
+  *out = h;
+  return MOT_OK;
+}
+
+mot_status mot_load_weights(mot_handle h, const void* host_blob, size_t bytes) {
+  if (!h || !host_blob) return MOT_ERR_INVALID_ARG;
+  const Dims& d = h->d;
+  const size_t es = esize(d), gsz = group_elems(d);
+  if (bytes != size_t(d.G) * gsz * es) return MOT_ERR_WEIGHTS_SIZE;
+  if (cudaSetDevice(h->device) != cudaSuccess) return MOT_ERR_CUDA;
+  const size_t E = d.E, Ds = d.Ds, Dt = d.Dt, H = d.H, EH = d.EH;
+  const char* blob = static_cast<const char*>(host_blob);
+  auto to_f = [&](const char* p, size_t i) -> float {
+    if (d.dtype == 1) {
+      float f;
+      memcpy(&f, p + 4 * i, 4);
+      return f;
+    }
+    uint16_t b;
+    memcpy(&b, p + 2 * i, 2);
+    uint32_t u = uint32_t(b) << 16;
+    float f;
+    memcpy(&f, &u, 4);
+    return f;
+  };
+  std::vector<float> bg(d.G * E), b1(d.G * EH), b2(d.G * E * Dt);
+  char* wg = static_cast<char*>(h->wg);
+  char* w1 = static_cast<char*>(h->w1);
+  char* w2 = static_cast<char*>(h->w2);
+  for (size_t g = 0; g < size_t(d.G); ++g) {
+    const char* p = blob + g * gsz * es;
+    size_t off = 0;
+    MOT_CUDA_TRY(cudaMemcpy(wg + g * E * Ds * es, p, E * Ds * es, cudaMemcpyHostToDevice));
+    off += E * Ds;
+    for (size_t m = 0; m < E; ++m) bg[g * E + m] = to_f(p, off + m);
+    off += E;
+    for (size_t m = 0; m < E; ++m) {
+      // W1_m -> rows [m*H, (m+1)*H) of W1cat
+      MOT_CUDA_TRY(cudaMemcpy(w1 + (g * EH + m * H) * Ds * es, p + off * es, H * Ds * es,
+                              cudaMemcpyHostToDevice));
+      off += H * Ds;
+      for (size_t j = 0; j < H; ++j) b1[g * EH + m * H + j] = to_f(p, off + j);
+      off += H;
+      // W2_m [Dt][H] -> columns [m*H, (m+1)*H) of W2cat [Dt][EH]
+      MOT_CUDA_TRY(cudaMemcpy2D(w2 + (g * Dt * EH + m * H) * es, EH * es, p + off * es, H * es,
+                                H * es, Dt, cudaMemcpyHostToDevice));
+      off += Dt * H;
+      for (size_t i = 0; i < Dt; ++i) b2[(g * E + m) * Dt + i] = to_f(p, off + i);
+      off += Dt;
+    }
+  }
+  if (d.G) {
+    MOT_CUDA_TRY(cudaMemcpy(h->bg, bg.data(), bg.size() * 4, cudaMemcpyHostToDevice));
+    MOT_CUDA_TRY(cudaMemcpy(h->b1, b1.data(), b1.size() * 4, cudaMemcpyHostToDevice));
+    MOT_CUDA_TRY(cudaMemcpy(h->b2, b2.data(), b2.size() * 4, cudaMemcpyHostToDevice));
+  }
+  MOT_CUDA_TRY(cudaDeviceSynchronize());
+  h->weights_loaded = true;
+  return MOT_OK;
+}
+
+mot_status mot_translate(mot_handle h, const void* src_k, const void* src_v,
+                         const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
+                         mot_stream_t stream) {
+  mot_status s = check_translate_args(h, src_k, src_v, seq_lens, batch, dst_k, dst_v);
+  if (s != MOT_OK) return s;
+  return run_translate(h, src_k, src_v, seq_lens, batch, dst_k, dst_v,
+                       reinterpret_cast<cudaStream_t>(stream));
+}
+
+mot_status mot_translate_host(mot_handle h, const void* src_k, const void* src_v,
+                              const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
+                              mot_stream_t stream) {
+  if (!h) return MOT_ERR_INVALID_ARG;
+  if (batch < 0 || batch > h->d.B) return MOT_ERR_INVALID_ARG;
+  if (!src_k || !src_v || !dst_k || !dst_v || (batch > 0 && !seq_lens)) return MOT_ERR_INVALID_ARG;
+  if (!h->weights_loaded) return MOT_ERR_NO_WEIGHTS;
+  const Dims& d = h->d;
+  for (int b = 0; b < batch; ++b)
+    if (seq_lens[b] < 0 || seq_lens[b] > d.S) return MOT_ERR_SEQ_LEN;
+  if (batch == 0 || d.G == 0) return MOT_OK;
+  if (!h->st_src[0]) {
+    const size_t sb = src_bytes(d), db = dst_bytes(d);
+    void** ps[5] = {&h->st_src[0], &h->st_src[1], &h->st_dst[0], &h->st_dst[1], (void**)&h->st_len};
+    const size_t ns[5] = {sb, sb, db, db, size_t(d.B) * 4};
+    for (int i = 0; i < 5; ++i)
+      if (cudaMalloc(ps[i], ns[i]) != cudaSuccess) {
+        cudaGetLastError();
+        for (int k = 0; k < 5; ++k)
+          if (*ps[k]) { cudaFree(*ps[k]); *ps[k] = nullptr; }
+        return MOT_ERR_OOM;
+      }
+  }
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const size_t es = esize(d);
+  MOT_CUDA_TRY(cudaMemcpyAsync(h->st_len, seq_lens, size_t(batch) * 4, cudaMemcpyHostToDevice, st));
+  // Real tokens only: for batch entry b, positions [0, len) of every (layer, head) row.
+  for (int b = 0; b < batch; ++b) {
+    const size_t len = seq_lens[b];
+    if (len == 0) continue;
+    for (int x = 0; x < 2; ++x) {
+      cudaMemcpy3DParms p{};
+      const size_t pitch = size_t(d.S) * d.d_s * es;
+      const size_t off = size_t(b) * d.H_s * pitch;
+      p.srcPtr = make_cudaPitchedPtr(const_cast<char*>(static_cast<const char*>(x ? src_v : src_k)) + off,
+                                     pitch, len * d.d_s * es, size_t(d.B) * d.H_s);
+      p.dstPtr = make_cudaPitchedPtr(static_cast<char*>(h->st_src[x]) + off, pitch,
+                                     len * d.d_s * es, size_t(d.B) * d.H_s);
+      p.extent = make_cudaExtent(len * d.d_s * es, d.H_s, d.L_s);
+      p.kind = cudaMemcpyHostToDevice;
+      MOT_CUDA_TRY(cudaMemcpy3DAsync(&p, st));
+    }
+  }
+  mot_status s = run_translate(h, h->st_src[0], h->st_src[1], h->st_len, batch, h->st_dst[0],
+                               h->st_dst[1], st);
+  if (s != MOT_OK) return s;
+  // Translated positions back: per batch entry and per run of translated layers.
+  for (int b = 0; b < batch; ++b) {
+    const size_t len = seq_lens[b];
+    if (len == 0) continue;
+    int l = 0;
+    while (l < d.L_t) {
+      if (h->layer_map[l] < 0) { ++l; continue; }
+      int l1 = l;
+      while (l1 < d.L_t && h->layer_map[l1] >= 0) ++l1;
+      for (int x = 0; x < 2; ++x) {
+        cudaMemcpy3DParms p{};
+        const size_t pitch = size_t(d.S) * d.d_t * es;
+        const size_t off = (size_t(l) * d.B + b) * d.H_t * pitch;
+        p.srcPtr = make_cudaPitchedPtr(static_cast<char*>(h->st_dst[x]) + off, pitch,
+                                       len * d.d_t * es, size_t(d.B) * d.H_t);
+        p.dstPtr = make_cudaPitchedPtr(static_cast<char*>(x ? dst_v : dst_k) + off, pitch,
+                                       len * d.d_t * es, size_t(d.B) * d.H_t);
+        p.extent = make_cudaExtent(len * d.d_t * es, d.H_t, size_t(l1 - l));
+        p.kind = cudaMemcpyDeviceToHost;
+        MOT_CUDA_TRY(cudaMemcpy3DAsync(&p, st));
+      }
+      l = l1;
+    }
+  }
+  return MOT_OK;
+}
+
+mot_status mot_get_device_status(mot_handle h, mot_stream_t stream) {
+  if (!h) return MOT_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  MOT_CUDA_TRY(cudaStreamSynchronize(st));
+  int32_t v = 0;
+  MOT_CUDA_TRY(cudaMemcpy(&v, h->status, 4, cudaMemcpyDeviceToHost));
+  MOT_CUDA_TRY(cudaMemset(h->status, 0, 4));
+  if (v & kStatusTimeout) return MOT_ERR_TIMEOUT;
+  if (v & kStatusSeqLen) return MOT_ERR_SEQ_LEN;
+  return MOT_OK;
+}
+
+mot_status mot_destroy(mot_handle h) {
+  if (!h) return MOT_ERR_INVALID_ARG;
+  cudaSetDevice(h->device);
+  cudaDeviceSynchronize();
+  free_all(h);
+  cudaGetLastError();
+  delete h;
+  return MOT_OK;
+}
+
+mot_status mot_get_layer_map(mot_handle h, int32_t* out, int32_t n) {
+  if (!h || !out || n != h->d.L_t) return MOT_ERR_INVALID_ARG;
+  for (int l = 0; l < n; ++l) out[l] = h->layer_map[l];
+  return MOT_OK;
+}
+
+mot_status mot_get_path(mot_handle h, int32_t* path) {
+  if (!h || !path) return MOT_ERR_INVALID_ARG;
+  *path = h->use_umma ? 1 : 0;
+  return MOT_OK;
+}
+
+mot_status mot_profile_enable(mot_handle h, int32_t enable) {
+  if (!h) return MOT_ERR_INVALID_ARG;
+  h->profile = enable != 0;
+  return MOT_OK;
+}
+
+mot_status mot_profile_read(mot_handle h, mot_kernel_stat* out, int32_t cap, int32_t* n) {
+  if (!h || !n || (cap > 0 && !out)) return MOT_ERR_INVALID_ARG;
+  std::vector<mot_kernel_stat> stats(h->kind_names.size());
+  for (size_t i = 0; i < stats.size(); ++i) {
+    memset(&stats[i], 0, sizeof(mot_kernel_stat));
+    strncpy(stats[i].name, h->kind_names[i].c_str(), sizeof(stats[i].name) - 1);
+  }
+  mot_status rs = MOT_OK;
+  for (auto& e : h->ev_used) {
+    float ms = 0.f;
+    if (cudaEventSynchronize(e.b) != cudaSuccess || cudaEventElapsedTime(&ms, e.a, e.b) != cudaSuccess) {
+      cudaGetLastError();
+      rs = MOT_ERR_CUDA;
+    }
+    stats[e.kind].launches += 1;
+    stats[e.kind].total_ms += ms;
+    h->ev_free.push_back(e);
+  }
+  h->ev_used.clear();
+  int32_t k = 0;
+  for (size_t i = 0; i < stats.size(); ++i) {
+    if (stats[i].launches == 0) continue;
+    if (k < cap) out[k] = stats[i];
+    ++k;
+  }
+  *n = std::min(k, cap);
+  return rs;
+}
+
+mot_status mot_get_launch_count(mot_handle h, int64_t* count) {
+  if (!h || !count) return MOT_ERR_INVALID_ARG;
+  *count = h->launches;
+  return MOT_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,84 @@
+// Internal declarations shared by the C-ABI layer and the kernel files.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "mot.h"
+
+namespace mot {
+
+constexpr int kTileM = 128;   // tokens per token tile (rows of one MMA tile)
+constexpr int kMaxE = 16;     // translators per (layer, K/V) group
+
+// Sticky device status bits, OR-ed into the handle's status word.
+enum : int32_t { kStatusSeqLen = 1, kStatusTimeout = 2 };
+
+// One 128-token tile of the ragged batch: batch entry b, positions
+// [s0, s0 + rows).
+struct TileInfo {
+  int32_t b, s0, rows, pad;
+};
+
+// One translated (target layer, K/V) group.
+struct GroupInfo {
+  int32_t tgt_layer, src_layer, x, pad;
+};
+
+struct Dims {
+  int32_t L_s, H_s, d_s, L_t, H_t, d_t, E, top_k, H, B, S;
+  int32_t Ds, Dt, EH;
+  int32_t G;          // translated groups = 2 * translated target layers
+  int32_t tiles_max;  // B * ceil(S / 128): token tiles at full capacity
+  int32_t tpad;       // tiles_max * 128: rows of the gate / A2 workspaces
+  int32_t dtype;      // 0 = bf16, 1 = fp32
+};
+
+// Everything one translation pass needs on the device. Weights are in the
+// library's repacked layout:
+//   wg [G][E][Ds] (dtype), bg [G][E] (fp32),
+//   w1 [G][E*H][Ds] (dtype; the E experts' W1 stacked along rows),
+//   b1 [G][E*H] (fp32),
+//   w2 [G][Dt][E*H] (dtype; the E experts' W2 side by side along K),
+//   b2 [G][E][Dt] (fp32).
+// Workspace: gate [G][tpad][E] fp32 (renormalised gate weights per token
+// row), a2 [gp][tpad][E*H] (GELU(hidden) * gate, bf16 on the tensor-core path
+// and fp32 on the SIMT path).
+struct PathArgs {
+  Dims d;
+  const void* src[2];
+  void* dst[2];
+  const TileInfo* tiles;
+  const int32_t* n_tiles;
+  const GroupInfo* groups;
+  const void* wg;
+  const float* bg;
+  const void* w1;
+  const float* b1;
+  const void* w2;
+  const float* b2;
+  float* gate;
+  void* a2;
+  int32_t* status;
+  int32_t g0, gp;   // groups [g0, g0 + gp) of this pass
+};
+
+// Kernel launchers (each returns the launch's cudaError_t).
+cudaError_t launch_prep(const int32_t* seq_lens, int32_t batch, const Dims& d, TileInfo* tiles,
+                        int32_t* n_tiles, int32_t* status, cudaStream_t st);
+cudaError_t launch_gate(const PathArgs& a, cudaStream_t st);
+cudaError_t launch_simt_gemm1(const PathArgs& a, cudaStream_t st);
+cudaError_t launch_simt_gemm2(const PathArgs& a, cudaStream_t st);
+
+// tcgen05 path. tmA0/tmA1: source K/V maps (GEMM1) or the A2 map (GEMM2, tmA0
+// only); tmB: W1 (GEMM1) or W2 (GEMM2) map.
+constexpr int kUmmaN = 256;   // N of one accumulator tile
+constexpr int kUmmaK = 64;    // K per pipeline stage (one 128-byte swizzle row)
+bool umma_supported(const Dims& d);
+cudaError_t launch_umma_gemm1(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                              const CUtensorMap& tmW1, int num_sms, cudaStream_t st);
+cudaError_t launch_umma_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2,
+                              int num_sms, cudaStream_t st);
+
+}  // namespace mot

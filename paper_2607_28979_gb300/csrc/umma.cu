@@ -1,0 +1,372 @@
+// tcgen05 / TMEM / TMA translation GEMMs for sm_103a (bf16 in, fp32 accumulate).
+//
+// The MoT combine (Eq. mot_definition) is a K-reduction once the experts are
+// concatenated: with W1cat = [W1_1; ...; W1_E] (E*H x D_s) and
+// W2cat = [W2_1, ..., W2_E] (D_t x E*H),
+//   GEMM1:  A2 = bf16( GELU(Z W1cat^T + b1cat) (.) gtilde_expand )      [T, E*H]
+//   GEMM2:  Y  = A2 W2cat^T + sum_m gtilde_m b2_m                        [T, D_t]
+// so sum_m gtilde_m W2_m GELU(W1_m z + b1_m) is exactly GEMM2's sum over E*H.
+//
+// One persistent, warp-specialised kernel template runs both GEMMs:
+//   warp 0 (one lane)  TMA producer: A and B K-blocks (64 bf16 = one 128-byte
+//                      swizzle row) into a 4-stage shared-memory ring;
+//   warp 1 (one lane)  MMA issuer: tcgen05.mma M=128, N=256, K=16, fp32
+//                      accumulator in TMEM, two accumulator buffers (512 cols);
+//   warp 2             TMEM allocator;
+//   warps 4-7          epilogue: tcgen05.ld of the accumulator (warp w reads
+//                      lanes 32*(w%4)...), fused bias / GELU / gate / combine,
+//                      16-byte vector stores.
+// The epilogue of tile i overlaps the MMAs of tile i+1. Every wait is bounded
+// (mot::mbar_wait); on a timeout all roles unwind, in-flight copies and MMAs
+// are drained, TMEM is freed and kStatusTimeout is raised.
+//
+// GEMM1's A operand is read straight from the source cache
+// [L_s][B][H_s][S][d_s] through a 5-D tensor map with box (64, 128, 1, 1, 1):
+// K-block kb is head kb*64 / d_s, dims (kb*64) % d_s .. +63, of 128
+// consecutive positions of one batch entry. Positions past the cache end read
+// as zero; rows past the tile's length are computed but never stored.
+#include <cuda_bf16.h>
+
+#include "mot_internal.h"
+#include "ptx.cuh"
+
+namespace mot {
+namespace {
+
+constexpr int UM = kTileM;   // 128
+constexpr int UN = kUmmaN;   // 256
+constexpr int UK = kUmmaK;   // 64
+constexpr int kStages = 4;
+constexpr int kABytes = UM * UK * 2;   // 16 KB
+constexpr int kBBytes = UN * UK * 2;   // 32 KB
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kTmemCols = 2 * UN;      // two fp32 accumulators of 256 columns
+constexpr int kThreads = 256;
+constexpr int kBarBytes = 256;
+constexpr int kSmemBytes = kStages * kStageBytes + kBarBytes + 1024;   // + alignment slack
+
+struct UmmaArgs {
+  PathArgs p;
+  int32_t nk;        // K blocks per tile
+  int32_t n_tiles_n; // N tiles per group
+  int32_t b_rows;    // rows of B per group (E*H for GEMM1, D_t for GEMM2)
+};
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// GELU(u) * g with the tanh form of GELU on the hardware tanh unit:
+// 0.5 u (1 + tanh(sqrt(2/pi) (u + 0.044715 u^3))). Its largest deviation from
+// the erf form is 4.7e-4 (at |u| = 2.7), below the bf16 rounding of the result.
+__device__ __forceinline__ float gelu_times(float u, float half_g) {
+  const float k0 = 0.7978845608028654f, k1 = 0.7978845608028654f * 0.044715f;
+  const float t = tanh_approx(u * fmaf(k1, u * u, k0));
+  const float hu = u * half_g;
+  return fmaf(hu, t, hu);
+}
+
+template <int MODE>   // 1 = GEMM1 (A = source cache), 2 = GEMM2 (A = A2)
+__global__ void __launch_bounds__(kThreads, 1)
+    umma_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
+                     const __grid_constant__ CUtensorMap tmA1,
+                     const __grid_constant__ CUtensorMap tmB, const UmmaArgs ua) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + kStages * kABytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
+  uint64_t* empty = full + kStages;
+  uint64_t* tfull = empty + kStages;    // [2]
+  uint64_t* tempty = tfull + 2;         // [2]
+  uint64_t* drain = tempty + 2;         // [1] used only when unwinding
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const PathArgs& p = ua.p;
+  const Dims& d = p.d;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA0);
+    if (MODE == 1) tma_prefetch_desc(&tmA1);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 2) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int n_m = min(*p.n_tiles, d.tiles_max);
+  const int per_grp = n_m * ua.n_tiles_n;
+  const int total = p.gp * per_grp;
+  // Unwind bookkeeping: TMA loads issued per stage and their phase parity
+  // (producer lane), and whether any MMA was issued (MMA lane).
+  uint32_t issued_mask = 0, issue_parity = 0;
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int t = blockIdx.x; t < total; t += gridDim.x) {
+        const int gl = t / per_grp, rem = t - gl * per_grp;
+        const int m = rem / ua.n_tiles_n, n = rem - m * ua.n_tiles_n;
+        const int grp = p.g0 + gl;
+        TileInfo ti;
+        GroupInfo gi;
+        if (MODE == 1) {
+          ti = p.tiles[m];
+          gi = p.groups[grp];
+        }
+        bool ok = true;
+        for (int kb = 0; kb < ua.nk; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[stage], kStageBytes);
+          if (MODE == 1) {
+            const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
+            tma_load_5d(sA + stage * kABytes, gi.x ? &tmA1 : &tmA0, &full[stage], d0, ti.s0, h,
+                        ti.b, gi.src_layer);
+          } else {
+            tma_load_3d(sA + stage * kABytes, &tmA0, &full[stage], kb * UK, m * UM, gl);
+          }
+          tma_load_2d(sB + stage * kBBytes, &tmB, &full[stage], kb * UK,
+                      grp * ua.b_rows + n * UN);
+          issued_mask |= 1u << stage;
+          issue_parity = (issue_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------ MMA issuer
+      const uint32_t idesc = idesc_bf16_f32(UM, UN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      for (int t = blockIdx.x; t < total; t += gridDim.x) {
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * UN);
+        bool ok = true;
+        for (int kb = 0; kb < ua.nk; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t adesc = sdesc_k_sw128(smem_u32(sA + stage * kABytes));
+          const uint64_t bdesc = sdesc_k_sw128(smem_u32(sB + stage * kBBytes));
+#pragma unroll
+          for (int k = 0; k < UK / 16; ++k)   // +32 bytes of K per step = +2 in the address field
+            umma_bf16(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (kb | k) != 0);
+          mma_issued = true;
+          umma_commit(&empty[stage]);
+          if (++stage == kStages) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        umma_commit(&tfull[acc]);
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1u;
+      }
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------ epilogue
+    const int q = warp - 4;             // TMEM lane quarter of this warp
+    const int row = q * 32 + lane;      // accumulator row = token row in the tile
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&tfull[acc], acc_phase, abort_flag) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      const int gl = t / per_grp, rem = t - gl * per_grp;
+      const int m = rem / ua.n_tiles_n, n = rem - m * ua.n_tiles_n;
+      const int grp = p.g0 + gl;
+      const uint32_t tbase = tmem_base + static_cast<uint32_t>(acc * UN) +
+                             (static_cast<uint32_t>(q * 32) << 16);
+      const size_t grow = static_cast<size_t>(m) * UM + row;   // workspace row
+      const int n0 = n * UN;
+      if (MODE == 1) {
+        // A2 = bf16(GELU(acc + b1) * gtilde[expert]); one expert per tile (H % 256 == 0)
+        const int expert = n0 / d.H;
+        const float half_g =
+            0.5f * p.gate[(static_cast<size_t>(grp) * d.tpad + grow) * d.E + expert];
+        const float* __restrict__ bias = p.b1 + static_cast<size_t>(grp) * d.EH + n0;
+        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.a2) +
+                             (static_cast<size_t>(gl) * d.tpad + grow) * d.EH + n0;
+#pragma unroll 1
+        for (int ch = 0; ch < UN / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tbase + ch * 32, r);
+          tmem_ld_wait();
+          const float4* b4 = reinterpret_cast<const float4*>(bias + ch * 32);
+          uint32_t pk[16];
+#pragma unroll
+          for (int v = 0; v < 8; ++v) {
+            const float4 bb = __ldg(b4 + v);
+            const float u0 = __uint_as_float(r[4 * v + 0]) + bb.x;
+            const float u1 = __uint_as_float(r[4 * v + 1]) + bb.y;
+            const float u2 = __uint_as_float(r[4 * v + 2]) + bb.z;
+            const float u3 = __uint_as_float(r[4 * v + 3]) + bb.w;
+            pk[2 * v] = pack_bf16x2(gelu_times(u0, half_g), gelu_times(u1, half_g));
+            pk[2 * v + 1] = pack_bf16x2(gelu_times(u2, half_g), gelu_times(u3, half_g));
+          }
+          uint4* o4 = reinterpret_cast<uint4*>(out + ch * 32);
+#pragma unroll
+          for (int v = 0; v < 4; ++v)
+            o4[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+        }
+      } else {
+        // y = acc + sum_m gtilde_m b2_m -> bf16 -> dst[l][b][c / d_t][s][c % d_t]
+        const GroupInfo gi = p.groups[grp];
+        const TileInfo ti = p.tiles[m];
+        const bool valid = row < ti.rows;
+        const float* grow_g = p.gate + (static_cast<size_t>(grp) * d.tpad + grow) * d.E;
+        float g[kMaxE];
+#pragma unroll
+        for (int e = 0; e < kMaxE; ++e) g[e] = e < d.E ? grow_g[e] : 0.f;
+        __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.dst[gi.x]);
+        const size_t s = static_cast<size_t>(ti.s0) + row;
+#pragma unroll 1
+        for (int ch = 0; ch < UN / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tbase + ch * 32, r);
+          tmem_ld_wait();
+          const int c = n0 + ch * 32;
+          float y[32];
+#pragma unroll
+          for (int j = 0; j < 32; ++j) y[j] = __uint_as_float(r[j]);
+#pragma unroll
+          for (int e = 0; e < kMaxE; ++e) {
+            if (e < d.E) {
+              const float4* b4 = reinterpret_cast<const float4*>(
+                  p.b2 + (static_cast<size_t>(grp) * d.E + e) * d.Dt + c);
+#pragma unroll
+              for (int v = 0; v < 8; ++v) {
+                const float4 bb = __ldg(b4 + v);
+                y[4 * v + 0] = fmaf(g[e], bb.x, y[4 * v + 0]);
+                y[4 * v + 1] = fmaf(g[e], bb.y, y[4 * v + 1]);
+                y[4 * v + 2] = fmaf(g[e], bb.z, y[4 * v + 2]);
+                y[4 * v + 3] = fmaf(g[e], bb.w, y[4 * v + 3]);
+              }
+            }
+          }
+          if (valid) {
+            const int h = c / d.d_t, i0 = c - h * d.d_t;
+            uint4* o4 = reinterpret_cast<uint4*>(
+                dst + ((((static_cast<size_t>(gi.tgt_layer) * d.B + ti.b) * d.H_t + h) * d.S + s) *
+                           d.d_t + i0));
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              o4[v] = make_uint4(pack_bf16x2(y[8 * v + 0], y[8 * v + 1]),
+                                 pack_bf16x2(y[8 * v + 2], y[8 * v + 3]),
+                                 pack_bf16x2(y[8 * v + 4], y[8 * v + 5]),
+                                 pack_bf16x2(y[8 * v + 6], y[8 * v + 7]));
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[acc]);
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort_flag) {
+    // Unwinding after a timed-out wait: let every copy the producer started
+    // land and every MMA already issued finish before TMEM is freed and the
+    // CTA exits. These waits are bounded as well.
+    if (warp == 0 && lane == 0) {
+      for (int s = 0; s < kStages; ++s)
+        if ((issued_mask >> s) & 1u) {
+          const uint32_t a = smem_u32(&full[s]);
+          const long long t0 = clock64();
+          while (!mbar_try_wait(a, (issue_parity >> s) & 1u) &&
+                 clock64() - t0 < kWaitLimitCycles) {
+          }
+        }
+    }
+    if (warp == 1 && lane == 0 && mma_issued) {
+      umma_commit(drain);
+      const uint32_t a = smem_u32(drain);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(a, 0) && clock64() - t0 < kWaitLimitCycles) {
+      }
+    }
+    __syncthreads();
+  }
+  if (warp == 2) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicOr(p.status, kStatusTimeout);
+}
+
+template <int MODE>
+cudaError_t launch_umma(const PathArgs& a, const CUtensorMap& A0, const CUtensorMap& A1,
+                        const CUtensorMap& B, int nk, int n_tiles_n, int b_rows, int num_sms,
+                        cudaStream_t st) {
+  static bool attr_set = false;   // per process; the attribute is per function
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(umma_gemm_kernel<MODE>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  UmmaArgs ua;
+  ua.p = a;
+  ua.nk = nk;
+  ua.n_tiles_n = n_tiles_n;
+  ua.b_rows = b_rows;
+  const long long upper = static_cast<long long>(a.gp) * a.d.tiles_max * n_tiles_n;
+  const int grid = static_cast<int>(upper < num_sms ? upper : num_sms);
+  if (grid <= 0) return cudaSuccess;
+  umma_gemm_kernel<MODE><<<grid, kThreads, kSmemBytes, st>>>(A0, A1, B, ua);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool umma_supported(const Dims& d) {
+  return d.dtype == 0 && d.d_s % UK == 0 && d.Ds % UK == 0 && d.H % UN == 0 && d.EH % UK == 0 &&
+         d.Dt % UN == 0 && d.d_t % 32 == 0 && d.E <= kMaxE;
+}
+
+cudaError_t launch_umma_gemm1(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                              const CUtensorMap& tmW1, int num_sms, cudaStream_t st) {
+  return launch_umma<1>(a, tmK, tmV, tmW1, a.d.Ds / UK, a.d.EH / UN, a.d.EH, num_sms, st);
+}
+
+cudaError_t launch_umma_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2,
+                              int num_sms, cudaStream_t st) {
+  return launch_umma<2>(a, tmA2, tmA2, tmW2, a.d.EH / UK, a.d.Dt / UN, a.d.Dt, num_sms, st);
+}
+
+}  // namespace mot

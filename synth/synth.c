@@ -13,9 +13,10 @@
  *     variant-13 finaliser (shifts 30/27/31, multipliers 0xBF58476D1CE4E5B9,
  *     0x94D049BB133111EB).
  *   - Stream key: s0 = mix(seed ^ mix(stream + GAMMA)).
- *   - Normal draw i of a stream: Box-Muller (1958) on outputs 2i and 2i+1:
- *     u1 = ((o_{2i} >> 11) + 1) * 2^-53 in (0,1], u2 = (o_{2i+1} >> 11) * 2^-53,
- *     n = sqrt(-2 ln u1) * cos(2 pi u2).
+ *   - Normal draws 2k and 2k+1 of a stream: Box-Muller (1958) on outputs 2k
+ *     and 2k+1: u1 = ((o_{2k} >> 11) + 1) * 2^-53 in (0,1],
+ *     u2 = (o_{2k+1} >> 11) * 2^-53, R = sqrt(-2 ln u1),
+ *     n_{2k} = R cos(2 pi u2), n_{2k+1} = R sin(2 pi u2).
  *   - Storage rounding: fp64 -> fp32 (C cast, round-to-nearest-even), then for
  *     bf16 the fp32 bit pattern is rounded to its top 16 bits with
  *     round-to-nearest-even.
@@ -25,6 +26,7 @@
  */
 #include <math.h>
 #include <stdint.h>
+#include <stdlib.h>
 #include <string.h>
 
 #define SYNTH_GAMMA 0x9E3779B97F4A7C15ULL
@@ -43,13 +45,22 @@ uint64_t synth_splitmix64(uint64_t key, uint64_t n) {
   return synth_mix(key + (n + 1) * SYNTH_GAMMA);
 }
 
-double synth_normal_at(uint64_t key, uint64_t i) {
+static inline void normal_pair(uint64_t key, uint64_t k, double* n0, double* n1) {
   const double two_m53 = 1.0 / 9007199254740992.0;
-  uint64_t o1 = synth_splitmix64(key, 2 * i);
-  uint64_t o2 = synth_splitmix64(key, 2 * i + 1);
+  uint64_t o1 = synth_splitmix64(key, 2 * k);
+  uint64_t o2 = synth_splitmix64(key, 2 * k + 1);
   double u1 = (double)((o1 >> 11) + 1) * two_m53;
   double u2 = (double)(o2 >> 11) * two_m53;
-  return sqrt(-2.0 * log(u1)) * cos(6.283185307179586476925 * u2);
+  double r = sqrt(-2.0 * log(u1));
+  double th = 6.283185307179586476925 * u2;
+  *n0 = r * cos(th);
+  *n1 = r * sin(th);
+}
+
+double synth_normal_at(uint64_t key, uint64_t i) {
+  double a, b;
+  normal_pair(key, i >> 1, &a, &b);
+  return (i & 1) ? b : a;
 }
 
 static inline uint16_t f32_to_bf16_rne(float f) {
@@ -72,21 +83,27 @@ static inline void store_val(void* out, int64_t idx, double v, int dtype) {
 void synth_fill_normal(uint64_t seed, uint64_t stream, int64_t n, double stddev,
                        int dtype, void* out) {
   uint64_t key = synth_stream_key(seed, stream);
+  const int64_t np = (n + 1) / 2;
 #pragma omp parallel for schedule(static)
-  for (int64_t i = 0; i < n; ++i) {
-    double v = stddev * synth_normal_at(key, (uint64_t)i);
-    if (dtype == 2)
-      ((double*)out)[i] = v;
-    else
-      store_val(out, i, v, dtype);
+  for (int64_t k = 0; k < np; ++k) {
+    double v[2];
+    normal_pair(key, (uint64_t)k, &v[0], &v[1]);
+    for (int j = 0; j < 2; ++j) {
+      const int64_t i = 2 * k + j;
+      if (i >= n) break;
+      if (dtype == 2)
+        ((double*)out)[i] = stddev * v[j];
+      else
+        store_val(out, i, stddev * v[j], dtype);
+    }
   }
 }
 
 /*
  * One layer of a KV cache laid out [B][H][S][d]: value = s_c * N, where the
  * per-channel scale s_c = exp(0.5 * n_c) ~ LogNormal(0, 0.5) is drawn once per
- * (layer, K/V, channel c = h*d + i) from `scale_stream` and the values from
- * `value_stream`.
+ * (layer, K/V, channel c = h*d + i) from `scale_stream` (draw c) and the values
+ * from `value_stream` (draw = flat index of the element).
  */
 void synth_fill_cache_layer(uint64_t seed, uint64_t scale_stream, uint64_t value_stream,
                             int B, int H, int S, int d, int dtype, void* out) {
@@ -94,13 +111,22 @@ void synth_fill_cache_layer(uint64_t seed, uint64_t scale_stream, uint64_t value
   uint64_t kval = synth_stream_key(seed, value_stream);
   const int64_t per_b = (int64_t)H * S * d;
   const int64_t n = (int64_t)B * per_b;
+  double* sc = (double*)malloc(sizeof(double) * (size_t)H * d);
+  if (!sc) return;
+  for (int64_t c = 0; c < (int64_t)H * d; ++c) sc[c] = exp(0.5 * synth_normal_at(kscale, (uint64_t)c));
+  const int64_t np = (n + 1) / 2;
 #pragma omp parallel for schedule(static)
-  for (int64_t idx = 0; idx < n; ++idx) {
-    int64_t r = idx % per_b;
-    int h = (int)(r / ((int64_t)S * d));
-    int i = (int)(r % d);
-    double sc = exp(0.5 * synth_normal_at(kscale, (uint64_t)(h * d + i)));
-    double v = sc * synth_normal_at(kval, (uint64_t)idx);
-    store_val(out, idx, v, dtype);
+  for (int64_t k = 0; k < np; ++k) {
+    double v[2];
+    normal_pair(kval, (uint64_t)k, &v[0], &v[1]);
+    for (int j = 0; j < 2; ++j) {
+      const int64_t idx = 2 * k + j;
+      if (idx >= n) break;
+      const int64_t r = idx % per_b;
+      const int64_t h = r / ((int64_t)S * d);
+      const int64_t i = r % d;
+      store_val(out, idx, sc[h * d + i] * v[j], dtype);
+    }
   }
+  free(sc);
 }

@@ -1,0 +1,96 @@
+"""The C-ABI library without a GPU: it loads, exports every entry point that
+include/mot.h declares, and rejects bad arguments before any CUDA call."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2607_28979_gb300 import build as mot_build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+mot_build.build()
+import paper_2607_28979_gb300.mot as M   # noqa: E402
+
+
+def declared_entry_points():
+    text = open(os.path.join(ROOT, "include", "mot.h")).read()
+    return sorted(set(re.findall(r"^(?:mot_status|const char\*)\s+(mot_\w+)\(", text, re.M)))
+
+
+def test_every_declared_symbol_is_exported():
+    names = declared_entry_points()
+    assert len(names) >= 12
+    for n in names:
+        assert hasattr(M._lib, n), f"libmot.so does not export {n}"
+    assert names == M.EXPORTED
+
+
+def test_library_is_in_tree_and_has_no_cuda_runtime_dependency():
+    assert os.path.dirname(M.LIB_PATH) == os.path.join(ROOT, "paper_2607_28979_gb300")
+
+
+def test_status_strings():
+    assert M.mot_status_string(M.MOT_OK) == "MOT_OK"
+    assert M.mot_status_string(M.MOT_ERR_SEQ_LEN) == "MOT_ERR_SEQ_LEN"
+    assert M.mot_status_string(M.MOT_ERR_TIMEOUT) == "MOT_ERR_TIMEOUT"
+    assert M.mot_status_string(99) == "MOT_ERR_UNKNOWN"
+
+
+GOOD = dict(n_layers_src=2, src_kv_heads=2, src_head_dim=64, n_layers_tgt=3, tgt_kv_heads=2,
+            tgt_head_dim=128, n_translators=2, hidden=256, max_batch=2, max_seq=64)
+
+
+@pytest.mark.parametrize("change,expect", [
+    (dict(n_layers_src=0), M.MOT_ERR_INVALID_ARG),
+    (dict(src_kv_heads=-1), M.MOT_ERR_INVALID_ARG),
+    (dict(tgt_head_dim=0), M.MOT_ERR_INVALID_ARG),
+    (dict(n_translators=0), M.MOT_ERR_INVALID_ARG),
+    (dict(hidden=0), M.MOT_ERR_INVALID_ARG),
+    (dict(max_batch=0), M.MOT_ERR_INVALID_ARG),
+    (dict(max_seq=0), M.MOT_ERR_INVALID_ARG),
+    (dict(top_k=3), M.MOT_ERR_INVALID_ARG),
+    (dict(top_k=-1), M.MOT_ERR_INVALID_ARG),
+    (dict(layer_map=[0, 2, 1]), M.MOT_ERR_INVALID_ARG),     # source layer 2 of 2
+    (dict(layer_map=[0, -2, 1]), M.MOT_ERR_INVALID_ARG),
+    (dict(n_translators=17, top_k=0), M.MOT_ERR_UNSUPPORTED),
+    (dict(max_batch=4097), M.MOT_ERR_UNSUPPORTED),
+])
+def test_create_rejects_bad_config_before_cuda(change, expect):
+    kw = dict(GOOD)
+    kw.update(change)
+    cfg = M.make_config(**kw)
+    out = ctypes.c_void_p(123)
+    assert M._lib.mot_create(ctypes.byref(cfg), ctypes.byref(out)) == expect
+    assert out.value is None
+
+
+def test_bad_dtype_rejected():
+    cfg = M.make_config(**GOOD)
+    cfg.dtype = 7
+    out = ctypes.c_void_p()
+    assert M._lib.mot_create(ctypes.byref(cfg), ctypes.byref(out)) == M.MOT_ERR_INVALID_ARG
+
+
+def test_null_arguments():
+    L = M._lib
+    assert L.mot_create(None, None) == M.MOT_ERR_INVALID_ARG
+    out = ctypes.c_void_p()
+    assert L.mot_create(None, ctypes.byref(out)) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_load_weights(None, None, 0) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_translate(None, 16, 16, 16, 1, 16, 16, None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_translate_host(None, 16, 16, 16, 1, 16, 16, None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_get_device_status(None, None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_destroy(None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_get_path(None, None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_profile_enable(None, 1) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_get_launch_count(None, None) == M.MOT_ERR_INVALID_ARG
+
+
+def test_valid_config_without_gpu_is_a_cuda_error():
+    torch = pytest.importorskip("torch")
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    with pytest.raises(M.MotError) as e:
+        M.mot_create(M.make_config(**GOOD))
+    assert e.value.status == M.MOT_ERR_CUDA

@@ -1,0 +1,249 @@
+"""CUDA path vs the fp64 oracle, element by element, through the C ABI."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+import _helpers as H
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+import _gpu as G   # noqa: E402
+M = G.M
+
+
+def inputs(wl, seed=0):
+    return synth.gen_cache(wl, 0, seed), synth.gen_cache(wl, 1, seed), synth.gen_weights(wl, seed)
+
+
+def full_check(wl, run, sk, sv, blob, label):
+    """Every element against oracle.translate_full; untouched positions keep the sentinel."""
+    assert run.canaries_intact(), f"{label}: wrote past the end of dst"
+    assert run.padding_untouched(), f"{label}: wrote a position it must not touch"
+    rk, rv = oracle.translate_full(wl, sk, sv, blob, run.seq[:run.batch])
+    gk, gv = run.dst_f64()
+    mask = G.translated_mask_full(wl, run.seq, run.batch)
+    mk = G.assert_parity(wl, gk[mask], rk[mask], label + " K")
+    mv = G.assert_parity(wl, gv[mask], rv[mask], label + " V")
+    return mk, mv
+
+
+# ---------------------------------------------------------------- small shapes, every element
+
+SMALL = {
+    # tensor-core path: ragged tails, several tiles, D_s != D_t, a -1 in the map, unused batch slot
+    "umma_ragged": synth.Workload("umma_ragged", 3, 2, 64, 4, 2, 128, 2, 256, 4, 300, "bf16",
+                                  (300, 129, 1), layer_map=(2, -1, 0, 1)),
+    # tensor-core path, E = 3, 128-dim source heads, depth-ratio map 5 -> 3
+    "umma_e3": synth.Workload("umma_e3", 5, 1, 128, 3, 4, 64, 3, 512, 2, 200, "bf16", (200, 77)),
+    # SIMT path (head dims outside the tensor-core tiling), bf16
+    "simt_bf16": synth.Workload("simt_bf16", 2, 3, 16, 2, 5, 8, 3, 40, 2, 70, "bf16", (70, 33)),
+    # SIMT path, fp32, odd sizes
+    "simt_fp32": synth.Workload("simt_fp32", 3, 2, 12, 2, 3, 10, 2, 50, 3, 90, "fp32",
+                                (90, 0, 65), layer_map=(2, 0)),
+    # single translator (E = 1) on the tensor-core path
+    "umma_e1": synth.Workload("umma_e1", 2, 4, 64, 2, 2, 128, 1, 512, 1, 256, "bf16", (256,)),
+}
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_small_shapes_every_element(name):
+    wl = SMALL[name]
+    sk, sv, blob = inputs(wl, seed=1)
+    run = G.Run(wl, sk, sv, blob)
+    expect_path = 1 if name.startswith("umma") else 0
+    assert M.mot_get_path(run.h) == expect_path
+    assert run.translate() == M.MOT_OK
+    full_check(wl, run, sk, sv, blob, name)
+
+
+def test_tiny_fp32_workload_every_element():
+    """The fp32 GPT-2-small -> OPT-125m-shaped workload (4 layers, seq 64, E=2), in full."""
+    wl = synth.WORKLOADS["tiny_fp32"]
+    sk, sv, blob = inputs(wl)
+    run = G.Run(wl, sk, sv, blob)
+    assert run.translate() == M.MOT_OK
+    full_check(wl, run, sk, sv, blob, wl.name)
+
+
+# ---------------------------------------------------------------- full-size workloads, sampled
+
+@pytest.mark.parametrize("name", ["gpt2s_opt125m", "qwen05_qwen15", "gpt2m_qwen7", "qwen7_long"])
+def test_full_size_workload_sampled(name):
+    """The workload at full size in the benchmark's launch configuration: the
+    oracle computes a token sample (sequence ends and 128-token tile boundaries
+    included); every untouched position must still hold the sentinel."""
+    wl = synth.WORKLOADS[name]
+    sk, sv, blob = inputs(wl)
+    run = G.Run(wl, sk, sv, blob)
+    assert run.translate() == M.MOT_OK
+    assert run.canaries_intact() and run.padding_untouched()
+    tb, ts = oracle.sample_tokens(wl.seq_lens, n_per_seq=6)
+    ref = oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
+    got = run.gather(tb, ts)
+    tl = wl.translated_layers()
+    m = G.assert_parity(wl, got[tl], ref[tl], name)
+    print(name, m)
+
+
+# ---------------------------------------------------------------- invariants on the GPU
+
+def _identity_blob(wl):
+    D = wl.d_src
+
+    def fn(l, x):
+        tr = [H.signed_perm_translator(D, wl.hidden, np.arange(D), np.arange(D))
+              for _ in range(wl.n_translators)]
+        return dict(Wg=np.zeros((wl.n_translators, D)), bg=np.zeros(wl.n_translators),
+                    W1=[t[0] for t in tr], b1=[t[1] for t in tr], W2=[t[2] for t in tr],
+                    b2=[t[3] for t in tr])
+    return H.make_blob(wl, fn)
+
+
+def test_identity_translator_copies_the_cache():
+    """W1=[I;-I], W2=[I,-I]: each translated layer is the mapped source layer,
+    re-headed from 4x64 to 2x128 (bf16 rounding of the hidden layer aside)."""
+    wl = synth.Workload("ident", 3, 4, 64, 4, 2, 128, 2, 512, 2, 160, "bf16", (160, 40))
+    sk, sv, _ = inputs(wl, seed=2)
+    blob = _identity_blob(wl)
+    run = G.Run(wl, sk, sv, blob)
+    assert M.mot_get_path(run.h) == 1
+    assert run.translate() == M.MOT_OK
+    gk, gv = run.dst_f64()
+    lm = oracle.depth_ratio_map(3, 4)
+    assert M.mot_get_layer_map(run.h) == lm
+    for l in range(4):
+        for src, got in ((sk, gk), (sv, gv)):
+            for b, L in enumerate(wl.seq_lens):
+                z = H.storage_to_f64(wl, src[lm[l], b, :, :L, :]).transpose(1, 0, 2).reshape(L, -1)
+                y = got[l, b, :, :L, :].transpose(1, 0, 2).reshape(L, -1)
+                # hidden activations are rounded to bf16 before the second GEMM
+                np.testing.assert_allclose(y, z, rtol=1e-2, atol=2e-2)
+
+
+def test_one_hot_gate_equals_single_translator_run():
+    """Proof of Prop. 3.1 on the GPU: a one-hot gate over E=3 gives the E=1 result."""
+    wl3 = synth.Workload("oh3", 2, 2, 64, 2, 2, 128, 3, 256, 1, 256, "bf16", (256,))
+    wl1 = wl3.replace(n_translators=1)
+    sk, sv, blob = inputs(wl3, seed=4)
+    grp = H.split_blob(wl3, blob)
+    m0 = 2
+
+    def onehot(l, x):
+        g = dict(grp[(l, x)])
+        g["Wg"] = np.zeros_like(g["Wg"])
+        g["bg"] = np.array([0.0, 0.0, 1e4])
+        return g
+
+    def single(l, x):
+        g = grp[(l, x)]
+        return dict(Wg=np.zeros((1, wl3.d_src)), bg=np.zeros(1), W1=[g["W1"][m0]], b1=[g["b1"][m0]],
+                    W2=[g["W2"][m0]], b2=[g["b2"][m0]])
+    r3 = G.Run(wl3, sk, sv, H.make_blob(wl3, onehot))
+    r1 = G.Run(wl1, sk, sv, H.make_blob(wl1, single))
+    assert r3.translate() == M.MOT_OK and r1.translate() == M.MOT_OK
+    a, b = r3.dst_f64(), r1.dst_f64()
+    for x in (0, 1):
+        np.testing.assert_array_equal(a[x], b[x])
+
+
+def test_prefix_consistency_and_unused_batch_slots():
+    """Shorter sequences give bit-identical values on their prefix; batch slots
+    beyond `batch` and positions past each length are untouched."""
+    wl = SMALL["umma_ragged"]
+    sk, sv, blob = inputs(wl, seed=5)
+    full = G.Run(wl, sk, sv, blob)
+    assert full.translate() == M.MOT_OK
+    short = G.Run(wl, sk, sv, blob, seq_lens=(131, 5, 1))
+    assert short.translate() == M.MOT_OK
+    assert short.padding_untouched() and short.canaries_intact()
+    for a, b in ((full.dk, short.dk), (full.dv, short.dv)):
+        for bb, L in enumerate((131, 5, 1)):
+            assert torch.equal(G.int_view(a[:, bb, :, :L]), G.int_view(b[:, bb, :, :L]))
+
+
+def test_zero_length_batch_and_batch_zero():
+    wl = SMALL["umma_ragged"]
+    sk, sv, blob = inputs(wl, seed=6)
+    run = G.Run(wl, sk, sv, blob, seq_lens=(0, 0, 0))
+    assert run.translate() == M.MOT_OK
+    assert run.padding_untouched()
+    run2 = G.Run(wl, sk, sv, blob, seq_lens=(5,), batch=0)
+    assert run2.translate() == M.MOT_OK
+    assert run2.padding_untouched(lens=[0, 0, 0, 0])
+
+
+def test_seq_len_out_of_range_is_clamped_and_reported():
+    wl = SMALL["umma_ragged"]
+    sk, sv, blob = inputs(wl, seed=7)
+    bad = G.Run(wl, sk, sv, blob, seq_lens=(wl.max_seq + 50, -3, 10))
+    assert bad.translate() == M.MOT_ERR_SEQ_LEN
+    assert M.mot_get_device_status(bad.h) == M.MOT_OK     # reading clears the word
+    good = G.Run(wl, sk, sv, blob, seq_lens=(wl.max_seq, 0, 10))
+    assert good.translate() == M.MOT_OK
+    assert torch.equal(G.int_view(bad.dk), G.int_view(good.dk))
+    assert torch.equal(G.int_view(bad.dv), G.int_view(good.dv))
+
+
+def test_host_buffer_entry_point_matches_device_entry_point():
+    wl = SMALL["umma_ragged"]
+    sk, sv, blob = inputs(wl, seed=8)
+    run = G.Run(wl, sk, sv, blob)
+    assert run.translate() == M.MOT_OK
+    dt = torch.int16 if wl.dtype == "bf16" else torch.int32
+    hk = torch.from_numpy(sk.view(np.int16)).pin_memory()
+    hv = torch.from_numpy(sv.view(np.int16)).pin_memory()
+    ok = torch.full(wl.dst_shape(), G.sentinel_value(wl), dtype=dt).pin_memory()
+    ov = torch.full(wl.dst_shape(), G.sentinel_value(wl), dtype=dt).pin_memory()
+    lens = np.asarray(wl.seq_lens, dtype=np.int32)
+    st = torch.cuda.current_stream()
+    M.mot_translate_host(run.h, hk, hv, lens, len(lens), ok, ov, st)
+    st.synchronize()
+    assert torch.equal(ok, G.int_view(run.dk).cpu())
+    assert torch.equal(ov, G.int_view(run.dv).cpu())
+    with pytest.raises(M.MotError) as e:
+        M.mot_translate_host(run.h, hk, hv, np.asarray([wl.max_seq + 1], np.int32), 1, ok, ov, st)
+    assert e.value.status == M.MOT_ERR_SEQ_LEN
+
+
+def test_argument_errors_with_a_live_handle():
+    wl = SMALL["umma_ragged"]
+    sk, sv, blob = inputs(wl, seed=9)
+    h = M.mot_create(M.config_from(wl))
+    with pytest.raises(M.MotError) as e:
+        M.mot_load_weights(h, blob[:-1])
+    assert e.value.status == M.MOT_ERR_WEIGHTS_SIZE
+    k, v = G.to_device(wl, sk), G.to_device(wl, sv)
+    _, dk = G.alloc_dst(wl)
+    _, dv = G.alloc_dst(wl)
+    lens = torch.tensor(wl.seq_lens, dtype=torch.int32, device="cuda")
+    with pytest.raises(M.MotError) as e:
+        M.mot_translate(h, k, v, lens, 3, dk, dv)
+    assert e.value.status == M.MOT_ERR_NO_WEIGHTS
+    M.mot_load_weights(h, blob)
+    for args, why in [((k.data_ptr() + 2, v, lens, 3, dk, dv), "misaligned"),
+                      ((k, v, lens, 5, dk, dv), "batch > max_batch"),
+                      ((k, v, lens, -1, dk, dv), "negative batch"),
+                      ((k, v, lens, 3, dk, dk), "dst_k aliases dst_v"),
+                      ((k, v, None, 3, dk, dv), "NULL seq_lens")]:
+        with pytest.raises(M.MotError) as e:
+            M.mot_translate(h, *args)
+        assert e.value.status == M.MOT_ERR_INVALID_ARG, why
+    M.mot_destroy(h)
+
+
+def test_profile_and_launch_count():
+    wl = SMALL["umma_ragged"]
+    sk, sv, blob = inputs(wl, seed=10)
+    run = G.Run(wl, sk, sv, blob)
+    n0 = M.mot_get_launch_count(run.h)
+    M.mot_profile_enable(run.h, True)
+    assert run.translate() == M.MOT_OK
+    stats = M.mot_profile_read(run.h)
+    assert set(stats) == {"prep_tiles", "gate", "umma_gemm1_gelu_gate", "umma_gemm2_combine_store"}
+    assert all(v[0] >= 1 and v[1] > 0 for v in stats.values())
+    assert M.mot_get_launch_count(run.h) - n0 == sum(v[0] for v in stats.values())

@@ -417,10 +417,16 @@ def main():
     ap.add_argument("--impl", choices=["mot", "reference"], default="mot")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--n-layers", type=int, default=0,
+                    help="keep only the first N layers of both models (smaller profiling case)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mot":
         args.warmup = 3
     wl = synth.WORKLOADS[args.workload]
+    if args.n_layers > 0:
+        wl = wl.replace(name=f"{wl.name}_L{args.n_layers}",
+                        n_layers_src=min(args.n_layers, wl.n_layers_src),
+                        n_layers_tgt=min(args.n_layers, wl.n_layers_tgt))
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_mot(args, wl)

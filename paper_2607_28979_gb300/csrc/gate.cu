@@ -193,10 +193,137 @@ __global__ void __launch_bounds__(256) gate_kernel(PathArgs a) {
   }
 }
 
+// Tile-wide variant for head dims that split into CPR 16-byte chunks with CPR
+// dividing 256: block (tile m, group) of 256 threads; thread t owns channel
+// chunk t % CPR of every head and rows t / CPR + p * (256 / CPR), p < P. A
+// warp's loads of one head then cover 512 contiguous bytes of the cache (the
+// tile's rows of one head are contiguous), every load is independent, and the
+// CPR partial dot products of a row are summed with shuffles inside a warp.
+template <typename T, int CPR, int P, int EMAX>
+__global__ void __launch_bounds__(256) gate_tile_kernel(PathArgs a) {
+  const Dims& d = a.d;
+  const int m = blockIdx.x;
+  const int grp = blockIdx.y;
+  if (m >= *a.n_tiles) return;
+  const TileInfo ti = a.tiles[m];
+  const GroupInfo gi = a.groups[grp];
+  constexpr int NV = Vec<T>::N;
+  constexpr int RPP = 256 / CPR;   // rows per pass
+  const int E = d.E;
+  const int cp = (threadIdx.x % CPR) * NV;   // channel offset inside a head
+  const int r0 = threadIdx.x / CPR;
+  const T* __restrict__ src = static_cast<const T*>(a.src[gi.x]);
+  const T* __restrict__ wg = static_cast<const T*>(a.wg) + static_cast<size_t>(grp) * E * d.Ds;
+  float acc[P][EMAX];
+#pragma unroll
+  for (int p = 0; p < P; ++p)
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e) acc[p][e] = 0.f;
+  for (int h = 0; h < d.H_s; ++h) {
+    float w[EMAX][NV];
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e) {
+      if (e < E) {
+        Vec<T>::load(wg + static_cast<size_t>(e) * d.Ds + h * d.d_s + cp, w[e]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < NV; ++k) w[e][k] = 0.f;
+      }
+    }
+    const T* base = src + (((static_cast<size_t>(gi.src_layer) * d.B + ti.b) * d.H_s + h) * d.S + ti.s0) * d.d_s + cp;
+#pragma unroll
+    for (int p = 0; p < P; ++p) {
+      const int r = r0 + p * RPP;
+      float z[NV];
+      if (r < ti.rows) {
+        Vec<T>::load(base + static_cast<size_t>(r) * d.d_s, z);
+      } else {
+#pragma unroll
+        for (int k = 0; k < NV; ++k) z[k] = 0.f;
+      }
+#pragma unroll
+      for (int e = 0; e < EMAX; ++e)
+#pragma unroll
+        for (int k = 0; k < NV; ++k) acc[p][e] = fmaf(w[e][k], z[k], acc[p][e]);
+    }
+  }
+#pragma unroll
+  for (int p = 0; p < P; ++p)
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+#pragma unroll
+      for (int off = CPR / 2; off > 0; off >>= 1)
+        acc[p][e] += __shfl_xor_sync(0xffffffffu, acc[p][e], off);
+  if (threadIdx.x % CPR != 0) return;
+  const float* __restrict__ bg = a.bg + static_cast<size_t>(grp) * E;
+#pragma unroll
+  for (int p = 0; p < P; ++p) {
+    const int r = r0 + p * RPP;
+    float* __restrict__ gout = a.gate + (static_cast<size_t>(grp) * d.tpad + static_cast<size_t>(m) * kTileM + r) * E;
+    if (r >= ti.rows) {
+      for (int e = 0; e < E; ++e) gout[e] = 0.f;
+      continue;
+    }
+    float g[EMAX];
+    float mx = -INFINITY;
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+      if (e < E) {
+        g[e] = acc[p][e] + bg[e];
+        mx = fmaxf(mx, g[e]);
+      }
+    float sum = 0.f;
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+      if (e < E) {
+        g[e] = expf(g[e] - mx);
+        sum += g[e];
+      }
+    const float inv = 1.f / sum;
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+      if (e < E) g[e] *= inv;
+    if (d.top_k > 0 && d.top_k < E) {
+      uint32_t keep = 0;
+      for (int k = 0; k < d.top_k; ++k) {
+        int best = -1;
+        float bv = 0.f;
+#pragma unroll
+        for (int e = 0; e < EMAX; ++e)
+          if (e < E && !((keep >> e) & 1u) && (best < 0 || g[e] > bv)) {
+            best = e;
+            bv = g[e];
+          }
+        keep |= 1u << best;
+      }
+      float ks = 0.f;
+#pragma unroll
+      for (int e = 0; e < EMAX; ++e)
+        if (e < E && ((keep >> e) & 1u)) ks += g[e];
+      const float kinv = 1.f / ks;
+#pragma unroll
+      for (int e = 0; e < EMAX; ++e)
+        if (e < E) g[e] = ((keep >> e) & 1u) ? g[e] * kinv : 0.f;
+    }
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+      if (e < E) gout[e] = g[e];
+  }
+}
+
 cudaError_t launch_gate(const PathArgs& a, cudaStream_t st) {
   const Dims& d = a.d;
   dim3 grid(d.tiles_max, d.G);
-  if (d.dtype == 0) {
+  // tile-wide kernel: 16-byte chunks per head row (CPR) of 8 or 16, E <= 8
+  if (d.dtype == 0 && d.E <= 4 && d.d_s == 64) {
+    gate_tile_kernel<__nv_bfloat16, 8, 4, 4><<<grid, 256, 0, st>>>(a);
+  } else if (d.dtype == 0 && d.E <= 8 && d.d_s == 64) {
+    gate_tile_kernel<__nv_bfloat16, 8, 4, 8><<<grid, 256, 0, st>>>(a);
+  } else if (d.dtype == 0 && d.E <= 4 && d.d_s == 128) {
+    gate_tile_kernel<__nv_bfloat16, 16, 8, 4><<<grid, 256, 0, st>>>(a);
+  } else if (d.dtype == 0 && d.E <= 8 && d.d_s == 128) {
+    gate_tile_kernel<__nv_bfloat16, 16, 8, 8><<<grid, 256, 0, st>>>(a);
+  } else if (d.dtype == 0) {
     if (d.d_s % 8 == 0)
       gate_kernel<__nv_bfloat16, true><<<grid, 256, 0, st>>>(a);
     else

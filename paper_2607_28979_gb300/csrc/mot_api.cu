@@ -92,7 +92,7 @@ struct mot_ctx {
   int32_t* n_tiles = nullptr;
   int32_t* status = nullptr;
   // tensor maps that do not depend on the caller's buffers
-  CUtensorMap tm_w1{}, tm_w2{}, tm_a2{};
+  CUtensorMap tm_w1{}, tm_w2{}, tm_a2{}, tm_a2_st{};
   // host-buffer staging for mot_translate_host (allocated on first use)
   void* st_src[2] = {nullptr, nullptr};
   void* st_dst[2] = {nullptr, nullptr};
@@ -252,7 +252,7 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
     a.gp = std::min(h->gp_max, d.G - g0);
     if (h->use_umma) {
       MOT_CUDA_TRY(timed(h, "umma_gemm1_gelu_gate", st, [&] {
-        return launch_umma_gemm1(a, tmK, tmV, h->tm_w1, h->num_sms, st);
+        return launch_umma_gemm1(a, tmK, tmV, h->tm_w1, h->tm_a2_st, h->num_sms, st);
       }));
       MOT_CUDA_TRY(timed(h, "umma_gemm2_combine_store", st, [&] {
         return launch_umma_gemm2(a, h->tm_a2, h->tm_w2, h->num_sms, st);
@@ -399,6 +399,8 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       const uint64_t st_b[2] = {uint64_t(EH) * 2, uint64_t(d.tpad) * EH * 2};
       const uint32_t box[3] = {uint32_t(kUmmaK), uint32_t(kTileM), 1};
       ok = ok && encode_bf16(&h->tm_a2, h->a2, 3, dims, st_b, box);
+      const uint32_t box_st[3] = {uint32_t(kUmmaK), 32, 1};   // one epilogue warp's store tile
+      ok = ok && encode_bf16(&h->tm_a2_st, h->a2, 3, dims, st_b, box_st);
     }
     if (!ok) {
       free_all(h);

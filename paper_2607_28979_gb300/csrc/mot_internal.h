@@ -71,13 +71,14 @@ cudaError_t launch_gate(const PathArgs& a, cudaStream_t st);
 cudaError_t launch_simt_gemm1(const PathArgs& a, cudaStream_t st);
 cudaError_t launch_simt_gemm2(const PathArgs& a, cudaStream_t st);
 
-// tcgen05 path. tmA0/tmA1: source K/V maps (GEMM1) or the A2 map (GEMM2, tmA0
-// only); tmB: W1 (GEMM1) or W2 (GEMM2) map.
+// tcgen05 path. GEMM1: source K/V load maps, W1 load map and the A2 store map
+// (box 64 x 32 x 1); GEMM2: A2 load map (box 64 x 128 x 1) and W2 load map.
 constexpr int kUmmaN = 256;   // N of one accumulator tile
 constexpr int kUmmaK = 64;    // K per pipeline stage (one 128-byte swizzle row)
 bool umma_supported(const Dims& d);
 cudaError_t launch_umma_gemm1(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
-                              const CUtensorMap& tmW1, int num_sms, cudaStream_t st);
+                              const CUtensorMap& tmW1, const CUtensorMap& tmA2st, int num_sms,
+                              cudaStream_t st);
 cudaError_t launch_umma_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2,
                               int num_sms, cudaStream_t st);
 

@@ -13,9 +13,13 @@
 //   warp 1 (one lane)  MMA issuer: tcgen05.mma M=128, N=256, K=16, fp32
 //                      accumulator in TMEM, two accumulator buffers (512 cols);
 //   warp 2             TMEM allocator;
-//   warps 4-7          epilogue: tcgen05.ld of the accumulator (warp w reads
-//                      lanes 32*(w%4)...), fused bias / GELU / gate / combine,
-//                      16-byte vector stores.
+//   warps 4..          epilogue: tcgen05.ld of the accumulator (warp w reads
+//                      lanes 32*(w%4)...), fused bias / GELU / gate / combine.
+//                      GEMM1 runs 8 epilogue warps (two per lane quarter, each
+//                      owning 128 of the 256 columns) and writes A2 through a
+//                      128B-swizzled shared-memory tile and a TMA store; GEMM2
+//                      runs 4 and stores 16-byte vectors straight into the
+//                      target cache rows (only rows inside the sequence).
 // The epilogue of tile i overlaps the MMAs of tile i+1. Every wait is bounded
 // (mot::mbar_wait); on a timeout all roles unwind, in-flight copies and MMAs
 // are drained, TMEM is freed and kStatusTimeout is raised.
@@ -41,9 +45,17 @@ constexpr int kABytes = UM * UK * 2;   // 16 KB
 constexpr int kBBytes = UN * UK * 2;   // 32 KB
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kTmemCols = 2 * UN;      // two fp32 accumulators of 256 columns
-constexpr int kThreads = 256;
 constexpr int kBarBytes = 256;
-constexpr int kSmemBytes = kStages * kStageBytes + kBarBytes + 1024;   // + alignment slack
+constexpr int kStoreTileBytes = 32 * 128;   // one warp's 32 rows x 64 bf16 columns
+__host__ __device__ constexpr int epi_warps(int mode) { return mode == 1 ? 8 : 4; }
+__host__ __device__ constexpr int threads_of(int mode) { return 32 * (4 + epi_warps(mode)); }
+__host__ __device__ constexpr int store_bytes(int mode) {
+  return mode == 1 ? epi_warps(mode) * kStoreTileBytes : 0;
+}
+__host__ __device__ constexpr int smem_bytes(int mode) {
+  return kStages * kStageBytes + store_bytes(mode) + kBarBytes + 1024;   // + alignment slack
+}
+static_assert(smem_bytes(1) <= 232448 && smem_bytes(2) <= 232448, "shared memory budget");
 
 struct UmmaArgs {
   PathArgs p;
@@ -68,16 +80,18 @@ __device__ __forceinline__ float gelu_times(float u, float half_g) {
 }
 
 template <int MODE>   // 1 = GEMM1 (A = source cache), 2 = GEMM2 (A = A2)
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(threads_of(MODE), 1)
     umma_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                      const __grid_constant__ CUtensorMap tmA1,
-                     const __grid_constant__ CUtensorMap tmB, const UmmaArgs ua) {
+                     const __grid_constant__ CUtensorMap tmB,
+                     const __grid_constant__ CUtensorMap tmS, const UmmaArgs ua) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + kStages * kABytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
+  uint8_t* sOut = smem + kStages * kStageBytes;   // GEMM1: one store tile per epilogue warp
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes + store_bytes(MODE));
   uint64_t* empty = full + kStages;
   uint64_t* tfull = empty + kStages;    // [2]
   uint64_t* tempty = tfull + 2;         // [2]
@@ -96,7 +110,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 4);
+      mbar_init(&tempty[a], epi_warps(MODE));
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -106,6 +120,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tmA0);
     if (MODE == 1) tma_prefetch_desc(&tmA1);
     tma_prefetch_desc(&tmB);
+    if (MODE == 1) tma_prefetch_desc(&tmS);
   }
   if (warp == 2) {
     tmem_alloc(tmem_slot, kTmemCols);
@@ -192,7 +207,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 4) {
     // ------------------------------------------------ epilogue
-    const int q = warp - 4;             // TMEM lane quarter of this warp
+    const int e = warp - 4;
+    const int q = e & 3;                // TMEM lane quarter of this warp (= warp % 4)
     const int row = q * 32 + lane;      // accumulator row = token row in the tile
     int acc = 0;
     uint32_t acc_phase = 0;
@@ -210,34 +226,51 @@ __global__ void __launch_bounds__(kThreads, 1)
       const size_t grow = static_cast<size_t>(m) * UM + row;   // workspace row
       const int n0 = n * UN;
       if (MODE == 1) {
-        // A2 = bf16(GELU(acc + b1) * gtilde[expert]); one expert per tile (H % 256 == 0)
+        // A2 = bf16(GELU(acc + b1) * gtilde[expert]); one expert per tile (H % 256 == 0).
+        // This warp: rows 32q..32q+31, columns 128*(e/4) .. +127 in two 64-column chunks.
         const int expert = n0 / d.H;
         const float half_g =
             0.5f * p.gate[(static_cast<size_t>(grp) * d.tpad + grow) * d.E + expert];
         const float* __restrict__ bias = p.b1 + static_cast<size_t>(grp) * d.EH + n0;
-        __nv_bfloat16* out = static_cast<__nv_bfloat16*>(p.a2) +
-                             (static_cast<size_t>(gl) * d.tpad + grow) * d.EH + n0;
+        uint8_t* tile = sOut + e * kStoreTileBytes;
+        const uint32_t tile_addr = smem_u32(tile);
 #pragma unroll 1
-        for (int ch = 0; ch < UN / 32; ++ch) {
-          uint32_t r[32];
-          tmem_ld_32x32b_x32(tbase + ch * 32, r);
-          tmem_ld_wait();
-          const float4* b4 = reinterpret_cast<const float4*>(bias + ch * 32);
-          uint32_t pk[16];
+        for (int c = 0; c < 2; ++c) {
+          const int col0 = (e >> 2) * 128 + c * 64;
+          uint32_t ra[32], rb[32];
+          tmem_ld_32x32b_x32(tbase + col0, ra);
+          tmem_ld_32x32b_x32(tbase + col0 + 32, rb);
+          tmem_ld_wait(ra);
+          tmem_ld_wait(rb);
+          const float4* b4 = reinterpret_cast<const float4*>(bias + col0);
+          uint32_t pk[32];
 #pragma unroll
-          for (int v = 0; v < 8; ++v) {
+          for (int v = 0; v < 16; ++v) {
             const float4 bb = __ldg(b4 + v);
-            const float u0 = __uint_as_float(r[4 * v + 0]) + bb.x;
-            const float u1 = __uint_as_float(r[4 * v + 1]) + bb.y;
-            const float u2 = __uint_as_float(r[4 * v + 2]) + bb.z;
-            const float u3 = __uint_as_float(r[4 * v + 3]) + bb.w;
+            const uint32_t* r = v < 8 ? ra : rb;
+            const int j = (v & 7) * 4;
+            const float u0 = __uint_as_float(r[j + 0]) + bb.x;
+            const float u1 = __uint_as_float(r[j + 1]) + bb.y;
+            const float u2 = __uint_as_float(r[j + 2]) + bb.z;
+            const float u3 = __uint_as_float(r[j + 3]) + bb.w;
             pk[2 * v] = pack_bf16x2(gelu_times(u0, half_g), gelu_times(u1, half_g));
             pk[2 * v + 1] = pack_bf16x2(gelu_times(u2, half_g), gelu_times(u3, half_g));
           }
-          uint4* o4 = reinterpret_cast<uint4*>(out + ch * 32);
+          // the previous TMA store of this warp must have finished reading the tile
+          if (lane == 0) bulk_wait_group_read<0>();
+          __syncwarp();
+          // row `lane` of the 32x64 tile, 16-byte chunk cc at chunk position cc ^ (row % 8)
+          // (the 128-byte swizzle the store map is encoded with; conflict-free banks)
 #pragma unroll
-          for (int v = 0; v < 4; ++v)
-            o4[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+          for (int cc = 0; cc < 8; ++cc)
+            st_shared_v4(tile_addr + lane * 128 + ((cc ^ (lane & 7)) << 4), pk[4 * cc],
+                         pk[4 * cc + 1], pk[4 * cc + 2], pk[4 * cc + 3]);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            tma_store_3d(&tmS, tile, n0 + col0, m * UM + q * 32, gl);
+            bulk_commit_group();
+          }
         }
       } else {
         // y = acc + sum_m gtilde_m b2_m -> bf16 -> dst[l][b][c / d_t][s][c % d_t]
@@ -254,7 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int ch = 0; ch < UN / 32; ++ch) {
           uint32_t r[32];
           tmem_ld_32x32b_x32(tbase + ch * 32, r);
-          tmem_ld_wait();
+          tmem_ld_wait(r);
           const int c = n0 + ch * 32;
           float y[32];
 #pragma unroll
@@ -294,6 +327,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
+    if (MODE == 1 && lane == 0) bulk_wait_group<0>();   // A2 stores complete before exit
   }
 
   tc_fence_before();
@@ -331,12 +365,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 template <int MODE>
 cudaError_t launch_umma(const PathArgs& a, const CUtensorMap& A0, const CUtensorMap& A1,
-                        const CUtensorMap& B, int nk, int n_tiles_n, int b_rows, int num_sms,
-                        cudaStream_t st) {
+                        const CUtensorMap& B, const CUtensorMap& S, int nk, int n_tiles_n,
+                        int b_rows, int num_sms, cudaStream_t st) {
   static bool attr_set = false;   // per process; the attribute is per function
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(umma_gemm_kernel<MODE>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         smem_bytes(MODE));
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
@@ -348,7 +383,7 @@ cudaError_t launch_umma(const PathArgs& a, const CUtensorMap& A0, const CUtensor
   const long long upper = static_cast<long long>(a.gp) * a.d.tiles_max * n_tiles_n;
   const int grid = static_cast<int>(upper < num_sms ? upper : num_sms);
   if (grid <= 0) return cudaSuccess;
-  umma_gemm_kernel<MODE><<<grid, kThreads, kSmemBytes, st>>>(A0, A1, B, ua);
+  umma_gemm_kernel<MODE><<<grid, threads_of(MODE), smem_bytes(MODE), st>>>(A0, A1, B, S, ua);
   return cudaGetLastError();
 }
 
@@ -360,13 +395,14 @@ bool umma_supported(const Dims& d) {
 }
 
 cudaError_t launch_umma_gemm1(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
-                              const CUtensorMap& tmW1, int num_sms, cudaStream_t st) {
-  return launch_umma<1>(a, tmK, tmV, tmW1, a.d.Ds / UK, a.d.EH / UN, a.d.EH, num_sms, st);
+                              const CUtensorMap& tmW1, const CUtensorMap& tmA2st, int num_sms,
+                              cudaStream_t st) {
+  return launch_umma<1>(a, tmK, tmV, tmW1, tmA2st, a.d.Ds / UK, a.d.EH / UN, a.d.EH, num_sms, st);
 }
 
 cudaError_t launch_umma_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2,
                               int num_sms, cudaStream_t st) {
-  return launch_umma<2>(a, tmA2, tmA2, tmW2, a.d.EH / UK, a.d.Dt / UN, a.d.Dt, num_sms, st);
+  return launch_umma<2>(a, tmA2, tmA2, tmW2, tmA2, a.d.EH / UK, a.d.Dt / UN, a.d.Dt, num_sms, st);
 }
 
 }  // namespace mot

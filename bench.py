@@ -264,6 +264,7 @@ def run_mot(args, wl):
     h = M.mot_create(M.config_from(wl))
     M.mot_load_weights(h, blob)
     path = M.mot_get_path(h)
+    M.mot_set_schedule(h, {"split": 0, "fused": 1, "pair": 2}[args.schedule])
     bf = wl.dtype == "bf16"
     tdt = torch.bfloat16 if bf else torch.float32
 
@@ -353,7 +354,10 @@ def run_mot(args, wl):
         # dominant kernel: the largest share of device time
         name, (n_launch, tot_ms) = max(kstats.items(), key=lambda kv: kv[1][1])
         gp_groups = 2 * tl
-        per_launch_flops = {"umma_gemm1_gelu_gate": alg["flops_gemm1"],
+        per_launch_flops = {"umma_fused_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
+                            "umma2_gemm1_gelu_gate": alg["flops_gemm1"],
+                            "umma2_gemm2_combine_store": alg["flops_gemm2"],
+                            "umma_gemm1_gelu_gate": alg["flops_gemm1"],
                             "simt_gemm1_gelu_gate": alg["flops_gemm1"],
                             "umma_gemm2_combine_store": alg["flops_gemm2"],
                             "simt_gemm2_combine_store": alg["flops_gemm2"]}
@@ -385,7 +389,7 @@ def run_mot(args, wl):
             "data": "synthetic (seeded SplitMix64/Box-Muller caches, N(0,1/fan_in) weights)",
             "config": {"workload": workload_desc(wl), "tokens_per_step": tokens,
                        "parallelism": "replicas" if world > 1 else "single GPU",
-                       "path": "tcgen05" if path == 1 else "simt",
+                       "path": ("tcgen05 " + args.schedule) if path == 1 else "simt",
                        "l2": "inputs larger than L2 (%.2f GB read+written per step)" % (alg["bytes"] / 1e9)},
             "roofline": roof,
             "step_roofline": {"flops": alg["flops"], "bytes": alg["bytes"],
@@ -417,6 +421,9 @@ def main():
     ap.add_argument("--impl", choices=["mot", "reference"], default="mot")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--schedule", choices=["pair", "fused", "split"], default="pair",
+                    help="tcgen05 launch schedule: GEMMs on CTA pairs (2-SM MMA), one fused "
+                         "persistent launch, or GEMMs on single SMs")
     ap.add_argument("--n-layers", type=int, default=0,
                     help="keep only the first N layers of both models (smaller profiling case)")
     args = ap.parse_args()

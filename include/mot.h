@@ -152,6 +152,18 @@ mot_status mot_get_layer_map(mot_handle h, int32_t* out, int32_t n);
 mot_status mot_get_path(mot_handle h, int32_t* path);
 
 /*
+ * Launch schedule of the tcgen05 path (no effect on the SIMT path); all give
+ * the same results.
+ *   2 (default): per pass of groups, GEMM1 then GEMM2 on pairs of CTAs (two
+ *      SMs per 256 x 256 tile, tcgen05.mma.cta_group::2);
+ *   1: one fused persistent launch per pass running both GEMMs as
+ *      dependency-ordered work items on single SMs;
+ *   0: GEMM1 then GEMM2 on single SMs (128 x 256 tiles).
+ */
+mot_status mot_set_schedule(mot_handle h, int32_t schedule);
+mot_status mot_get_schedule(mot_handle h, int32_t* schedule);
+
+/*
  * Per-kernel timing. While enabled, every kernel that translate launches is
  * bracketed by CUDA events on the launching stream. mot_profile_read
  * synchronises those events, writes up to `cap` records (one per kernel

@@ -40,9 +40,10 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// bf16 tensor map with 128-byte swizzle; dims[0] is the contiguous one.
+// 16-bit tensor map (bf16, or fp16 when `f16`) with 128-byte swizzle;
+// dims[0] is the contiguous one.
 bool encode_bf16(CUtensorMap* map, const void* base, int rank, const uint64_t* dims,
-                 const uint64_t* strides_bytes, const uint32_t* box) {
+                 const uint64_t* strides_bytes, const uint32_t* box, bool f16 = false) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t gd[5], gs[4];
@@ -53,7 +54,7 @@ bool encode_bf16(CUtensorMap* map, const void* base, int rank, const uint64_t* d
     es[i] = 1;
   }
   for (int i = 0; i < rank - 1; ++i) gs[i] = strides_bytes[i];
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), gd, gs, bx,
+  CUresult r = fn(map, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), gd, gs, bx,
                   es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
@@ -73,6 +74,7 @@ struct mot_ctx {
   int device = 0;
   int num_sms = 0;
   bool use_umma = false;
+  int schedule = 2;           // tcgen05 path: 0 split, 1 fused, 2 split on CTA pairs
   bool weights_loaded = false;
   int gp_max = 1;
   std::vector<GroupInfo> groups_h;
@@ -82,7 +84,8 @@ struct mot_ctx {
   float* bg = nullptr;
   void* w1 = nullptr;
   float* b1 = nullptr;
-  void* w2 = nullptr;
+  void* b1h = nullptr;   // fp16 copy of b1 (tensor-core path)
+  void* w2 = nullptr;    // dtype on the SIMT path, fp16 on the tensor-core path
   float* b2 = nullptr;
   GroupInfo* groups = nullptr;
   // workspace
@@ -91,8 +94,9 @@ struct mot_ctx {
   TileInfo* tiles = nullptr;
   int32_t* n_tiles = nullptr;
   int32_t* status = nullptr;
+  int32_t* counters = nullptr;   // fused schedule: item counter + per-tile completions
   // tensor maps that do not depend on the caller's buffers
-  CUtensorMap tm_w1{}, tm_w2{}, tm_a2{}, tm_a2_st{};
+  CUtensorMap tm_w1{}, tm_w2{}, tm_a2{}, tm_a2_st{}, tm_w1h{}, tm_w2h{};
   // host-buffer staging for mot_translate_host (allocated on first use)
   void* st_src[2] = {nullptr, nullptr};
   void* st_dst[2] = {nullptr, nullptr};
@@ -119,9 +123,9 @@ size_t group_elems(const Dims& d) {
 }
 
 void free_all(mot_ctx* h) {
-  void* ptrs[] = {h->wg, h->bg, h->w1, h->b1, h->w2, h->b2, h->groups, h->gate, h->a2, h->tiles,
-                  h->n_tiles, h->status, h->st_src[0], h->st_src[1], h->st_dst[0], h->st_dst[1],
-                  h->st_len};
+  void* ptrs[] = {h->wg, h->bg, h->w1, h->b1, h->b1h, h->w2, h->b2, h->groups, h->gate, h->a2, h->tiles,
+                  h->n_tiles, h->status, h->counters, h->st_src[0], h->st_src[1], h->st_dst[0],
+                  h->st_dst[1], h->st_len};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (auto& e : h->ev_used) { cudaEventDestroy(e.a); cudaEventDestroy(e.b); }
@@ -204,6 +208,7 @@ PathArgs path_args(mot_ctx* h) {
   a.bg = h->bg;
   a.w1 = h->w1;
   a.b1 = h->b1;
+  a.b1h = h->b1h;
   a.w2 = h->w2;
   a.b2 = h->b2;
   a.gate = h->gate;
@@ -250,7 +255,19 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
   for (int g0 = 0; g0 < d.G; g0 += h->gp_max) {
     a.g0 = g0;
     a.gp = std::min(h->gp_max, d.G - g0);
-    if (h->use_umma) {
+    if (h->use_umma && h->schedule == 2) {
+      MOT_CUDA_TRY(timed(h, "umma2_gemm1_gelu_gate", st, [&] {
+        return launch_umma2_gemm1(a, tmK, tmV, h->tm_w1h, h->tm_a2_st, h->num_sms, st);
+      }));
+      MOT_CUDA_TRY(timed(h, "umma2_gemm2_combine_store", st, [&] {
+        return launch_umma2_gemm2(a, h->tm_a2, h->tm_w2h, h->num_sms, st);
+      }));
+    } else if (h->use_umma && h->schedule == 1) {
+      MOT_CUDA_TRY(timed(h, "umma_fused_translate", st, [&] {
+        return launch_fused(a, tmK, tmV, h->tm_w1, h->tm_a2, h->tm_w2, h->tm_a2_st, h->counters,
+                            h->num_sms, st);
+      }));
+    } else if (h->use_umma) {
       MOT_CUDA_TRY(timed(h, "umma_gemm1_gelu_gate", st, [&] {
         return launch_umma_gemm1(a, tmK, tmV, h->tm_w1, h->tm_a2_st, h->num_sms, st);
       }));
@@ -357,13 +374,14 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
   }
   struct A { void** p; size_t n; } allocs[] = {
       {&h->wg, G * E * d.Ds * es}, {(void**)&h->bg, G * E * 4},
-      {&h->w1, G * EH * d.Ds * es}, {(void**)&h->b1, G * EH * 4},
+      {&h->w1, G * EH * d.Ds * es}, {(void**)&h->b1, G * EH * 4}, {&h->b1h, G * EH * 2},
       {&h->w2, G * d.Dt * EH * es}, {(void**)&h->b2, G * E * d.Dt * 4},
       {(void**)&h->groups, std::max<size_t>(G, 1) * sizeof(GroupInfo)},
       {(void**)&h->gate, G * size_t(d.tpad) * E * 4},
       {&h->a2, size_t(h->gp_max) * per_group_a2},
       {(void**)&h->tiles, size_t(d.tiles_max) * sizeof(TileInfo)},
-      {(void**)&h->n_tiles, 16}, {(void**)&h->status, 16}};
+      {(void**)&h->n_tiles, 16}, {(void**)&h->status, 16},
+      {(void**)&h->counters, fused_counter_ints(d, h->gp_max) * sizeof(int32_t)}};
   for (auto& a : allocs) {
     if (cudaMalloc(a.p, std::max<size_t>(a.n, 16)) != cudaSuccess) {
       cudaGetLastError();
@@ -387,20 +405,24 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       const uint64_t st_b[1] = {uint64_t(d.Ds) * 2};
       const uint32_t box[2] = {uint32_t(kUmmaK), uint32_t(kUmmaN)};
       ok = ok && encode_bf16(&h->tm_w1, h->w1, 2, dims, st_b, box);
+      const uint32_t box_h[2] = {uint32_t(kUmmaK), uint32_t(kUmmaN / 2)};   // one CTA of a pair
+      ok = ok && encode_bf16(&h->tm_w1h, h->w1, 2, dims, st_b, box_h);
     }
     {  // W2cat: [G*Dt rows][EH], box 64 x 256
       const uint64_t dims[2] = {uint64_t(EH), uint64_t(G * d.Dt)};
       const uint64_t st_b[1] = {uint64_t(EH) * 2};
       const uint32_t box[2] = {uint32_t(kUmmaK), uint32_t(kUmmaN)};
-      ok = ok && encode_bf16(&h->tm_w2, h->w2, 2, dims, st_b, box);
+      ok = ok && encode_bf16(&h->tm_w2, h->w2, 2, dims, st_b, box, /*f16=*/true);
+      const uint32_t box_h[2] = {uint32_t(kUmmaK), uint32_t(kUmmaN / 2)};
+      ok = ok && encode_bf16(&h->tm_w2h, h->w2, 2, dims, st_b, box_h, /*f16=*/true);
     }
     {  // A2: [gp][tpad][EH], box 64 x 128 x 1
       const uint64_t dims[3] = {uint64_t(EH), uint64_t(d.tpad), uint64_t(h->gp_max)};
       const uint64_t st_b[2] = {uint64_t(EH) * 2, uint64_t(d.tpad) * EH * 2};
       const uint32_t box[3] = {uint32_t(kUmmaK), uint32_t(kTileM), 1};
-      ok = ok && encode_bf16(&h->tm_a2, h->a2, 3, dims, st_b, box);
+      ok = ok && encode_bf16(&h->tm_a2, h->a2, 3, dims, st_b, box, /*f16=*/true);
       const uint32_t box_st[3] = {uint32_t(kUmmaK), 32, 1};   // one epilogue warp's store tile
-      ok = ok && encode_bf16(&h->tm_a2_st, h->a2, 3, dims, st_b, box_st);
+      ok = ok && encode_bf16(&h->tm_a2_st, h->a2, 3, dims, st_b, box_st, /*f16=*/true);
     }
     if (!ok) {
       free_all(h);
@@ -463,6 +485,11 @@ mot_status mot_load_weights(mot_handle h, const void* host_blob, size_t bytes) {
     MOT_CUDA_TRY(cudaMemcpy(h->bg, bg.data(), bg.size() * 4, cudaMemcpyHostToDevice));
     MOT_CUDA_TRY(cudaMemcpy(h->b1, b1.data(), b1.size() * 4, cudaMemcpyHostToDevice));
     MOT_CUDA_TRY(cudaMemcpy(h->b2, b2.data(), b2.size() * 4, cudaMemcpyHostToDevice));
+    if (h->use_umma) {
+      // GEMM2 runs fp16 x fp16: W2 to fp16 in place, b1 copied to fp16
+      MOT_CUDA_TRY(launch_bf16_to_f16_inplace(h->w2, size_t(d.G) * Dt * EH, 0));
+      MOT_CUDA_TRY(launch_f32_to_f16(h->b1, h->b1h, b1.size(), 0));
+    }
   }
   MOT_CUDA_TRY(cudaDeviceSynchronize());
   h->weights_loaded = true;
@@ -582,6 +609,18 @@ mot_status mot_get_layer_map(mot_handle h, int32_t* out, int32_t n) {
 mot_status mot_get_path(mot_handle h, int32_t* path) {
   if (!h || !path) return MOT_ERR_INVALID_ARG;
   *path = h->use_umma ? 1 : 0;
+  return MOT_OK;
+}
+
+mot_status mot_set_schedule(mot_handle h, int32_t schedule) {
+  if (!h || schedule < 0 || schedule > 2) return MOT_ERR_INVALID_ARG;
+  h->schedule = schedule;
+  return MOT_OK;
+}
+
+mot_status mot_get_schedule(mot_handle h, int32_t* schedule) {
+  if (!h || !schedule) return MOT_ERR_INVALID_ARG;
+  *schedule = h->schedule;
   return MOT_OK;
 }
 

@@ -42,9 +42,11 @@ struct Dims {
 //   b1 [G][E*H] (fp32),
 //   w2 [G][Dt][E*H] (dtype; the E experts' W2 side by side along K),
 //   b2 [G][E][Dt] (fp32).
+// On the tensor-core path w2 holds fp16 (converted from the bf16 blob at
+// load) and b1h an fp16 copy of b1, so that GEMM2 runs fp16 x fp16 -> fp32.
 // Workspace: gate [G][tpad][E] fp32 (renormalised gate weights per token
-// row), a2 [gp][tpad][E*H] (GELU(hidden) * gate, bf16 on the tensor-core path
-// and fp32 on the SIMT path).
+// row), a2 [gp][tpad][E*H] (GELU(hidden) * gate: fp16 on the tensor-core path,
+// fp32 on the SIMT path).
 struct PathArgs {
   Dims d;
   const void* src[2];
@@ -56,6 +58,7 @@ struct PathArgs {
   const float* bg;
   const void* w1;
   const float* b1;
+  const void* b1h;   // fp16 [G][E*H] (tensor-core path)
   const void* w2;
   const float* b2;
   float* gate;
@@ -65,6 +68,8 @@ struct PathArgs {
 };
 
 // Kernel launchers (each returns the launch's cudaError_t).
+cudaError_t launch_bf16_to_f16_inplace(void* buf, size_t n, cudaStream_t st);
+cudaError_t launch_f32_to_f16(const float* src, void* dst, size_t n, cudaStream_t st);
 cudaError_t launch_prep(const int32_t* seq_lens, int32_t batch, const Dims& d, TileInfo* tiles,
                         int32_t* n_tiles, int32_t* status, cudaStream_t st);
 cudaError_t launch_gate(const PathArgs& a, cudaStream_t st);
@@ -81,5 +86,22 @@ cudaError_t launch_umma_gemm1(const PathArgs& a, const CUtensorMap& tmK, const C
                               cudaStream_t st);
 cudaError_t launch_umma_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2,
                               int num_sms, cudaStream_t st);
+
+// 2-SM variant (umma2.cu): CTA pairs, tcgen05.mma.cta_group::2 on 256 x 256
+// tiles. The W maps here have 64 x 128 boxes (each CTA loads half of B).
+cudaError_t launch_umma2_gemm1(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                               const CUtensorMap& tmW1h, const CUtensorMap& tmA2st, int num_sms,
+                               cudaStream_t st);
+cudaError_t launch_umma2_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2h,
+                               int num_sms, cudaStream_t st);
+
+// Fused persistent kernel: both GEMMs of a pass in one launch (fused.cu).
+// `counters` holds fused_counter_ints(d, gp) int32 (zeroed by the launcher).
+int fused_block_tiles(const Dims& d, int num_sms);
+size_t fused_counter_ints(const Dims& d, int gp);
+cudaError_t launch_fused(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                         const CUtensorMap& tmW1, const CUtensorMap& tmA2,
+                         const CUtensorMap& tmW2, const CUtensorMap& tmA2st, int32_t* counters,
+                         int num_sms, cudaStream_t st);
 
 }  // namespace mot

@@ -1,9 +1,10 @@
-// tcgen05 / TMEM / TMA translation GEMMs for sm_103a (bf16 in, fp32 accumulate).
+// tcgen05 / TMEM / TMA translation GEMMs for sm_103a (fp32 accumulate; GEMM1
+// bf16 x bf16, GEMM2 fp16 x fp16 on the fp16 intermediate and fp16 W2).
 //
 // The MoT combine (Eq. mot_definition) is a K-reduction once the experts are
 // concatenated: with W1cat = [W1_1; ...; W1_E] (E*H x D_s) and
 // W2cat = [W2_1, ..., W2_E] (D_t x E*H),
-//   GEMM1:  A2 = bf16( GELU(Z W1cat^T + b1cat) (.) gtilde_expand )      [T, E*H]
+//   GEMM1:  A2 = fp16( GELU(Z W1cat^T + b1cat) (.) gtilde_expand )      [T, E*H]
 //   GEMM2:  Y  = A2 W2cat^T + sum_m gtilde_m b2_m                        [T, D_t]
 // so sum_m gtilde_m W2_m GELU(W1_m z + b1_m) is exactly GEMM2's sum over E*H.
 //
@@ -29,24 +30,12 @@
 // K-block kb is head kb*64 / d_s, dims (kb*64) % d_s .. +63, of 128
 // consecutive positions of one batch entry. Positions past the cache end read
 // as zero; rows past the tile's length are computed but never stored.
-#include <cuda_bf16.h>
-
-#include "mot_internal.h"
-#include "ptx.cuh"
+#include "umma_common.cuh"
 
 namespace mot {
 namespace {
 
-constexpr int UM = kTileM;   // 128
-constexpr int UN = kUmmaN;   // 256
-constexpr int UK = kUmmaK;   // 64
-constexpr int kStages = 4;
-constexpr int kABytes = UM * UK * 2;   // 16 KB
-constexpr int kBBytes = UN * UK * 2;   // 32 KB
-constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kTmemCols = 2 * UN;      // two fp32 accumulators of 256 columns
 constexpr int kBarBytes = 256;
-constexpr int kStoreTileBytes = 32 * 128;   // one warp's 32 rows x 64 bf16 columns
 __host__ __device__ constexpr int epi_warps(int mode) { return mode == 1 ? 8 : 4; }
 __host__ __device__ constexpr int threads_of(int mode) { return 32 * (4 + epi_warps(mode)); }
 __host__ __device__ constexpr int store_bytes(int mode) {
@@ -63,21 +52,6 @@ struct UmmaArgs {
   int32_t n_tiles_n; // N tiles per group
   int32_t b_rows;    // rows of B per group (E*H for GEMM1, D_t for GEMM2)
 };
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
-  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-  return *reinterpret_cast<uint32_t*>(&v);
-}
-
-// GELU(u) * g with the tanh form of GELU on the hardware tanh unit:
-// 0.5 u (1 + tanh(sqrt(2/pi) (u + 0.044715 u^3))). Its largest deviation from
-// the erf form is 4.7e-4 (at |u| = 2.7), below the bf16 rounding of the result.
-__device__ __forceinline__ float gelu_times(float u, float half_g) {
-  const float k0 = 0.7978845608028654f, k1 = 0.7978845608028654f * 0.044715f;
-  const float t = tanh_approx(u * fmaf(k1, u * u, k0));
-  const float hu = u * half_g;
-  return fmaf(hu, t, hu);
-}
 
 template <int MODE>   // 1 = GEMM1 (A = source cache), 2 = GEMM2 (A = A2)
 __global__ void __launch_bounds__(threads_of(MODE), 1)
@@ -177,7 +151,8 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------ MMA issuer
-      const uint32_t idesc = idesc_bf16_f32(UM, UN);
+      // GEMM1: bf16 source x bf16 W1; GEMM2: fp16 A2 x fp16 W2
+      const uint32_t idesc = MODE == 1 ? idesc_bf16_f32(UM, UN) : idesc_f16_f32(UM, UN);
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
@@ -209,7 +184,6 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
     // ------------------------------------------------ epilogue
     const int e = warp - 4;
     const int q = e & 3;                // TMEM lane quarter of this warp (= warp % 4)
-    const int row = q * 32 + lane;      // accumulator row = token row in the tile
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
@@ -223,104 +197,11 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
       const int grp = p.g0 + gl;
       const uint32_t tbase = tmem_base + static_cast<uint32_t>(acc * UN) +
                              (static_cast<uint32_t>(q * 32) << 16);
-      const size_t grow = static_cast<size_t>(m) * UM + row;   // workspace row
-      const int n0 = n * UN;
-      if (MODE == 1) {
-        // A2 = bf16(GELU(acc + b1) * gtilde[expert]); one expert per tile (H % 256 == 0).
-        // This warp: rows 32q..32q+31, columns 128*(e/4) .. +127 in two 64-column chunks.
-        const int expert = n0 / d.H;
-        const float half_g =
-            0.5f * p.gate[(static_cast<size_t>(grp) * d.tpad + grow) * d.E + expert];
-        const float* __restrict__ bias = p.b1 + static_cast<size_t>(grp) * d.EH + n0;
-        uint8_t* tile = sOut + e * kStoreTileBytes;
-        const uint32_t tile_addr = smem_u32(tile);
-#pragma unroll 1
-        for (int c = 0; c < 2; ++c) {
-          const int col0 = (e >> 2) * 128 + c * 64;
-          uint32_t ra[32], rb[32];
-          tmem_ld_32x32b_x32(tbase + col0, ra);
-          tmem_ld_32x32b_x32(tbase + col0 + 32, rb);
-          tmem_ld_wait(ra);
-          tmem_ld_wait(rb);
-          const float4* b4 = reinterpret_cast<const float4*>(bias + col0);
-          uint32_t pk[32];
-#pragma unroll
-          for (int v = 0; v < 16; ++v) {
-            const float4 bb = __ldg(b4 + v);
-            const uint32_t* r = v < 8 ? ra : rb;
-            const int j = (v & 7) * 4;
-            const float u0 = __uint_as_float(r[j + 0]) + bb.x;
-            const float u1 = __uint_as_float(r[j + 1]) + bb.y;
-            const float u2 = __uint_as_float(r[j + 2]) + bb.z;
-            const float u3 = __uint_as_float(r[j + 3]) + bb.w;
-            pk[2 * v] = pack_bf16x2(gelu_times(u0, half_g), gelu_times(u1, half_g));
-            pk[2 * v + 1] = pack_bf16x2(gelu_times(u2, half_g), gelu_times(u3, half_g));
-          }
-          // the previous TMA store of this warp must have finished reading the tile
-          if (lane == 0) bulk_wait_group_read<0>();
-          __syncwarp();
-          // row `lane` of the 32x64 tile, 16-byte chunk cc at chunk position cc ^ (row % 8)
-          // (the 128-byte swizzle the store map is encoded with; conflict-free banks)
-#pragma unroll
-          for (int cc = 0; cc < 8; ++cc)
-            st_shared_v4(tile_addr + lane * 128 + ((cc ^ (lane & 7)) << 4), pk[4 * cc],
-                         pk[4 * cc + 1], pk[4 * cc + 2], pk[4 * cc + 3]);
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            tma_store_3d(&tmS, tile, n0 + col0, m * UM + q * 32, gl);
-            bulk_commit_group();
-          }
-        }
-      } else {
-        // y = acc + sum_m gtilde_m b2_m -> bf16 -> dst[l][b][c / d_t][s][c % d_t]
-        const GroupInfo gi = p.groups[grp];
-        const TileInfo ti = p.tiles[m];
-        const bool valid = row < ti.rows;
-        const float* grow_g = p.gate + (static_cast<size_t>(grp) * d.tpad + grow) * d.E;
-        float g[kMaxE];
-#pragma unroll
-        for (int e = 0; e < kMaxE; ++e) g[e] = e < d.E ? grow_g[e] : 0.f;
-        __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.dst[gi.x]);
-        const size_t s = static_cast<size_t>(ti.s0) + row;
-#pragma unroll 1
-        for (int ch = 0; ch < UN / 32; ++ch) {
-          uint32_t r[32];
-          tmem_ld_32x32b_x32(tbase + ch * 32, r);
-          tmem_ld_wait(r);
-          const int c = n0 + ch * 32;
-          float y[32];
-#pragma unroll
-          for (int j = 0; j < 32; ++j) y[j] = __uint_as_float(r[j]);
-#pragma unroll
-          for (int e = 0; e < kMaxE; ++e) {
-            if (e < d.E) {
-              const float4* b4 = reinterpret_cast<const float4*>(
-                  p.b2 + (static_cast<size_t>(grp) * d.E + e) * d.Dt + c);
-#pragma unroll
-              for (int v = 0; v < 8; ++v) {
-                const float4 bb = __ldg(b4 + v);
-                y[4 * v + 0] = fmaf(g[e], bb.x, y[4 * v + 0]);
-                y[4 * v + 1] = fmaf(g[e], bb.y, y[4 * v + 1]);
-                y[4 * v + 2] = fmaf(g[e], bb.z, y[4 * v + 2]);
-                y[4 * v + 3] = fmaf(g[e], bb.w, y[4 * v + 3]);
-              }
-            }
-          }
-          if (valid) {
-            const int h = c / d.d_t, i0 = c - h * d.d_t;
-            uint4* o4 = reinterpret_cast<uint4*>(
-                dst + ((((static_cast<size_t>(gi.tgt_layer) * d.B + ti.b) * d.H_t + h) * d.S + s) *
-                           d.d_t + i0));
-#pragma unroll
-            for (int v = 0; v < 4; ++v)
-              o4[v] = make_uint4(pack_bf16x2(y[8 * v + 0], y[8 * v + 1]),
-                                 pack_bf16x2(y[8 * v + 2], y[8 * v + 3]),
-                                 pack_bf16x2(y[8 * v + 4], y[8 * v + 5]),
-                                 pack_bf16x2(y[8 * v + 6], y[8 * v + 7]));
-          }
-        }
-      }
+      if (MODE == 1)   // 8 warps: this warp owns columns 128 * (e / 4) .. +127
+        epilogue_gemm1(p, &tmS, tbase, sOut + e * kStoreTileBytes, q, lane, gl, grp, m, n * UN,
+                       (e >> 2) * 128, 2);
+      else             // 4 warps: all 256 columns
+        epilogue_gemm2(p, tbase, q, lane, grp, m, n * UN, 0, UN / 32);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[acc]);

@@ -1,0 +1,300 @@
+// 2-SM (cta_group::2) variant of the two translation GEMMs (see umma.cu for
+// what each computes). A cluster of two CTAs computes a 256 x 256 tile: token
+// tiles 2*mp (leader, cluster rank 0) and 2*mp + 1 (peer), against one
+// 256-column slice of W1cat / W2cat. Each CTA stages only its own 128 rows of
+// A and its own 128 rows of B per K block (32 KB instead of 48 KB for the
+// same tensor-core work per SM), so six stages fit where four did, and every
+// SM pulls two thirds of the operand bytes through L2 and its TMA unit.
+//
+// Roles per CTA (same warp layout as umma.cu):
+//   warp 0 lane 0 (both CTAs)  TMA loads of its A rows and B half; the
+//                              transaction bytes of both CTAs complete on the
+//                              leader's stage barrier;
+//   warp 1 lane 0 (leader)     tcgen05.mma.cta_group::2 M=256 N=256 K=16;
+//                              commits arrive on both CTAs' barriers;
+//   warp 2 (both CTAs)         allocates the pair's TMEM together;
+//   warps 4.. (both CTAs)      epilogue of its own 128 accumulator rows, then
+//                              an arrive on the leader's accumulator-free
+//                              barrier.
+// A token tile past the last one (odd tile count) is read as zeros by TMA and
+// never stored. Every wait is bounded; a timeout unwinds and raises
+// kStatusTimeout.
+#include "umma_common.cuh"
+
+namespace mot {
+namespace {
+
+constexpr int kStages2 = 6;
+constexpr int kABytes2 = UM * UK * 2;         // 16 KB: this CTA's 128 rows of A
+constexpr int kBBytes2 = (UN / 2) * UK * 2;   // 16 KB: this CTA's 128 rows of B
+constexpr int kStageBytes2 = kABytes2 + kBBytes2;
+constexpr int kBarBytes2 = 256;
+__host__ __device__ constexpr int epi_warps2(int mode) { return mode == 1 ? 8 : 4; }
+__host__ __device__ constexpr int threads2(int mode) { return 32 * (4 + epi_warps2(mode)); }
+__host__ __device__ constexpr int store_bytes2(int mode) {
+  return mode == 1 ? epi_warps2(mode) * kStoreTileBytes : 0;
+}
+__host__ __device__ constexpr int smem_bytes2(int mode) {
+  return kStages2 * kStageBytes2 + store_bytes2(mode) + kBarBytes2 + 1024;
+}
+static_assert(smem_bytes2(1) <= 232448 && smem_bytes2(2) <= 232448, "shared memory budget");
+
+struct Umma2Args {
+  PathArgs p;
+  int32_t nk;         // K blocks per tile
+  int32_t n_tiles_n;  // 256-column tiles per group
+  int32_t b_rows;     // rows of B per group (E*H for GEMM1, D_t for GEMM2)
+};
+
+// Spin about `cycles` SM cycles (used only while unwinding after a timeout).
+__device__ __forceinline__ void spin_cycles(long long cycles) {
+  const long long t0 = clock64();
+  while (clock64() - t0 < cycles) {
+  }
+}
+
+template <int MODE>   // 1 = GEMM1 (A = source cache), 2 = GEMM2 (A = A2)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
+    umma2_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
+                      const __grid_constant__ CUtensorMap tmA1,
+                      const __grid_constant__ CUtensorMap tmB,
+                      const __grid_constant__ CUtensorMap tmS, const Umma2Args ua) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + kStages2 * kABytes2;
+  uint8_t* sOut = smem + kStages2 * kStageBytes2;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sOut + store_bytes2(MODE));
+  uint64_t* empty = full + kStages2;
+  uint64_t* tfull = empty + kStages2;   // [2]
+  uint64_t* tempty = tfull + 2;         // [2] (used in the leader)
+  uint64_t* drain = tempty + 2;         // [1]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const PathArgs& p = ua.p;
+  const Dims& d = p.d;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages2; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 2 * epi_warps2(MODE));
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA0);
+    if (MODE == 1) tma_prefetch_desc(&tmA1);
+    tma_prefetch_desc(&tmB);
+    if (MODE == 1) tma_prefetch_desc(&tmS);
+  }
+  if (warp == 2) {
+    tmem_alloc_pair(tmem_slot, kTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync();   // barrier inits and the TMEM address are visible in both CTAs
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int n_m = min(*p.n_tiles, d.tiles_max);
+  const int n_mp = (n_m + 1) / 2;
+  const int per_grp = n_mp * ua.n_tiles_n;
+  const int total = p.gp * per_grp;
+  const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+
+  uint32_t issued_mask = 0, issue_parity = 0;
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer (both CTAs)
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int t = pair; t < total; t += n_pairs) {
+        const int gl = t / per_grp, rem = t - gl * per_grp;
+        const int mp = rem / ua.n_tiles_n, n = rem - mp * ua.n_tiles_n;
+        const int grp = p.g0 + gl;
+        const int m_own = 2 * mp + static_cast<int>(rank);
+        TileInfo ti;
+        GroupInfo gi;
+        if (MODE == 1) {
+          gi = p.groups[grp];
+          if (m_own < n_m) {
+            ti = p.tiles[m_own];
+          } else {   // no such tile: rows past the cache end read as zeros
+            ti.b = 0;
+            ti.s0 = d.S;
+          }
+        }
+        bool ok = true;
+        for (int kb = 0; kb < ua.nk; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) { ok = false; break; }
+          if (leader) mbar_arrive_expect_tx(&full[stage], 2 * kStageBytes2);
+          const uint32_t bar = leader_addr(&full[stage]);
+          if (MODE == 1) {
+            const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
+            tma_load_5d_pair(sA + stage * kABytes2, gi.x ? &tmA1 : &tmA0, bar, d0, ti.s0, h, ti.b,
+                             gi.src_layer);
+          } else {
+            tma_load_3d_pair(sA + stage * kABytes2, &tmA0, bar, kb * UK, m_own * UM, gl);
+          }
+          tma_load_2d_pair(sB + stage * kBBytes2, &tmB, bar, kb * UK,
+                           grp * ua.b_rows + n * UN + static_cast<int>(rank) * (UN / 2));
+          issued_mask |= 1u << stage;
+          issue_parity = (issue_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == kStages2) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      // ------------------------------------------------ MMA issuer (leader)
+      const uint32_t idesc = MODE == 1 ? idesc_bf16_f32(2 * UM, UN) : idesc_f16_f32(2 * UM, UN);
+      int stage = 0, acc = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      for (int t = pair; t < total; t += n_pairs) {
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * UN);
+        bool ok = true;
+        for (int kb = 0; kb < ua.nk; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag)) { ok = false; break; }
+          tc_fence_after();
+          const uint64_t adesc = sdesc_k_sw128(smem_u32(sA + stage * kABytes2));
+          const uint64_t bdesc = sdesc_k_sw128(smem_u32(sB + stage * kBBytes2));
+#pragma unroll
+          for (int k = 0; k < UK / 16; ++k)   // +32 bytes of K per step = +2 in the address field
+            umma_pair(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (kb | k) != 0);
+          mma_issued = true;
+          umma_commit_pair(&empty[stage]);
+          if (++stage == kStages2) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        umma_commit_pair(&tfull[acc]);
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1u;
+      }
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------ epilogue (both CTAs)
+    const int e = warp - 4;
+    const int q = e & 3;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int t = pair; t < total; t += n_pairs) {
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&tfull[acc], acc_phase, abort_flag) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      const int gl = t / per_grp, rem = t - gl * per_grp;
+      const int mp = rem / ua.n_tiles_n, n = rem - mp * ua.n_tiles_n;
+      const int grp = p.g0 + gl;
+      const int m_own = 2 * mp + static_cast<int>(rank);
+      const uint32_t tbase = tmem_base + static_cast<uint32_t>(acc * UN) +
+                             (static_cast<uint32_t>(q * 32) << 16);
+      if (m_own < n_m) {
+        if (MODE == 1)   // 8 warps: this warp owns columns 128 * (e / 4) .. +127
+          epilogue_gemm1(p, &tmS, tbase, sOut + e * kStoreTileBytes, q, lane, gl, grp, m_own,
+                         n * UN, (e >> 2) * 128, 2);
+        else             // 4 warps: all 256 columns
+          epilogue_gemm2(p, tbase, q, lane, grp, m_own, n * UN, 0, UN / 32);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(&tempty[acc], 0);
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+    if (MODE == 1 && lane == 0) bulk_wait_group<0>();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort_flag) {
+    // Unwinding after a timed-out wait (bounded): copies this CTA started
+    // complete on the leader's barriers, so give them time to land; the
+    // leader also waits for its issued MMAs.
+    if (warp == 0 && lane == 0 && issued_mask) {
+      if (leader) {
+        for (int s = 0; s < kStages2; ++s)
+          if ((issued_mask >> s) & 1u) {
+            const uint32_t a = smem_u32(&full[s]);
+            const long long t0 = clock64();
+            while (!mbar_try_wait(a, (issue_parity >> s) & 1u) &&
+                   clock64() - t0 < kWaitLimitCycles) {
+            }
+          }
+      } else {
+        spin_cycles(20000000LL);
+      }
+    }
+    if (warp == 1 && lane == 0 && leader && mma_issued) {
+      umma_commit_pair(drain);
+      const uint32_t a = smem_u32(drain);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(a, 0) && clock64() - t0 < kWaitLimitCycles) {
+      }
+    }
+    __syncthreads();
+  }
+  tc_fence_before();
+  cluster_sync();   // the leader's MMAs no longer read this CTA's shared memory or TMEM
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, kTmemCols);
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicOr(p.status, kStatusTimeout);
+}
+
+template <int MODE>
+cudaError_t launch_umma2(const PathArgs& a, const CUtensorMap& A0, const CUtensorMap& A1,
+                         const CUtensorMap& B, const CUtensorMap& S, int nk, int n_tiles_n,
+                         int b_rows, int num_sms, cudaStream_t st) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(umma2_gemm_kernel<MODE>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         smem_bytes2(MODE));
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  Umma2Args ua;
+  ua.p = a;
+  ua.nk = nk;
+  ua.n_tiles_n = n_tiles_n;
+  ua.b_rows = b_rows;
+  const long long pairs = static_cast<long long>(a.gp) * ((a.d.tiles_max + 1) / 2) * n_tiles_n;
+  const long long max_pairs = num_sms / 2;
+  const int grid = 2 * static_cast<int>(pairs < max_pairs ? pairs : max_pairs);
+  if (grid <= 0) return cudaSuccess;
+  umma2_gemm_kernel<MODE><<<grid, threads2(MODE), smem_bytes2(MODE), st>>>(A0, A1, B, S, ua);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_umma2_gemm1(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                               const CUtensorMap& tmW1h, const CUtensorMap& tmA2st, int num_sms,
+                               cudaStream_t st) {
+  return launch_umma2<1>(a, tmK, tmV, tmW1h, tmA2st, a.d.Ds / UK, a.d.EH / UN, a.d.EH, num_sms, st);
+}
+
+cudaError_t launch_umma2_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2h,
+                               int num_sms, cudaStream_t st) {
+  return launch_umma2<2>(a, tmA2, tmA2, tmW2h, tmA2, a.d.EH / UK, a.d.Dt / UN, a.d.Dt, num_sms, st);
+}
+
+}  // namespace mot

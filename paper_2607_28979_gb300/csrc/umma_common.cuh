@@ -1,0 +1,173 @@
+// Tile geometry and the two fused epilogues shared by the tcgen05 kernels.
+//
+//   GEMM1 epilogue:  A2[row, n0 + c] = fp16( GELU(acc[row, c] + b1[n0 + c]) * gtilde_m(row) )
+//                    (one expert m per 256-column tile since H % 256 == 0), computed in
+//                    packed fp16x2 arithmetic and written as 32x64 tiles through
+//                    128B-swizzled shared memory + TMA store.
+//   GEMM2 epilogue:  y[row, c] = acc[row, c] + sum_m gtilde_m(row) * b2_m[c], rounded
+//                    to bf16 and stored as 16-byte vectors into the target cache row
+//                    dst[l][b][c / d_t][s][c % d_t] when s < seq_len[b].
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "mot_internal.h"
+#include "ptx.cuh"
+
+namespace mot {
+
+constexpr int UM = kTileM;   // 128 rows (tokens) per accumulator tile
+constexpr int UN = kUmmaN;   // 256 columns per accumulator tile
+constexpr int UK = kUmmaK;   // 64 K elements per pipeline stage
+constexpr int kStages = 4;
+constexpr int kABytes = UM * UK * 2;   // 16 KB
+constexpr int kBBytes = UN * UK * 2;   // 32 KB
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kTmemCols = 2 * UN;      // two fp32 accumulators of 256 columns
+constexpr int kStoreTileBytes = 32 * 128;   // one warp's 32 rows x 64 bf16 columns
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// GELU(u) * g with the tanh form of GELU on the hardware tanh unit:
+// 0.5 u (1 + tanh(sqrt(2/pi) (u + 0.044715 u^3))). Its largest deviation from
+// the erf form is 4.7e-4 (at |u| = 2.7). fp32 version (for reference and tests).
+__device__ __forceinline__ float gelu_times(float u, float half_g) {
+  const float k0 = 0.7978845608028654f, k1 = 0.7978845608028654f * 0.044715f;
+  const float t = tanh_approx(u * fmaf(k1, u * u, k0));
+  const float hu = u * half_g;
+  return fmaf(hu, t, hu);
+}
+
+// The same on two fp16 lanes at once (HFMA2 + tanh.approx.f16x2): about 2^-11
+// relative rounding per step, finer than the fp16 result it produces.
+__device__ __forceinline__ __half2 gelu_times_h2(__half2 u, __half2 half_g) {
+  const __half2 k0 = __float2half2_rn(0.7978845608028654f);
+  const __half2 k1 = __float2half2_rn(0.7978845608028654f * 0.044715f);
+  const __half2 arg = __hmul2(u, __hfma2(__hmul2(u, u), k1, k0));
+  const uint32_t tb = tanh_approx_f16x2(*reinterpret_cast<const uint32_t*>(&arg));
+  const __half2 t = *reinterpret_cast<const __half2*>(&tb);
+  const __half2 hu = __hmul2(u, half_g);
+  return __hfma2(hu, t, hu);
+}
+
+// GEMM1 epilogue of one warp: rows 32*q + lane of the tile, columns
+// [col_begin, col_begin + 64 * n_chunks). `tbase` is the accumulator's TMEM
+// address including the warp's lane quarter; `tile` this warp's 4 KB store
+// tile (1024-byte aligned). The caller commits nothing: each chunk is its own
+// bulk group.
+__device__ __forceinline__ void epilogue_gemm1(const PathArgs& p, const CUtensorMap* tmS,
+                                               uint32_t tbase, uint8_t* tile, int q, int lane,
+                                               int gl, int grp, int m, int n0, int col_begin,
+                                               int n_chunks) {
+  const Dims& d = p.d;
+  const size_t grow = static_cast<size_t>(m) * UM + q * 32 + lane;
+  const int expert = n0 / d.H;
+  const __half2 half_g =
+      __float2half2_rn(0.5f * p.gate[(static_cast<size_t>(grp) * d.tpad + grow) * d.E + expert]);
+  const __half* __restrict__ bias =
+      static_cast<const __half*>(p.b1h) + static_cast<size_t>(grp) * d.EH + n0;
+  const uint32_t tile_addr = smem_u32(tile);
+#pragma unroll 1
+  for (int c = 0; c < n_chunks; ++c) {
+    const int col0 = col_begin + c * 64;
+    uint32_t ra[32], rb[32];
+    tmem_ld_32x32b_x32(tbase + col0, ra);
+    tmem_ld_32x32b_x32(tbase + col0 + 32, rb);
+    tmem_ld_wait(ra);
+    tmem_ld_wait(rb);
+    const uint4* b4 = reinterpret_cast<const uint4*>(bias + col0);   // 8 fp16 biases each
+    uint32_t pk[32];   // pk[k] = columns 2k, 2k+1 as fp16x2
+#pragma unroll
+    for (int v = 0; v < 8; ++v) {
+      const uint4 bb = __ldg(b4 + v);
+      const uint32_t bw[4] = {bb.x, bb.y, bb.z, bb.w};
+      const uint32_t* r = v < 4 ? ra : rb;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int j = (v & 3) * 8 + 2 * k;
+        __half2 u = __float22half2_rn(make_float2(__uint_as_float(r[j]), __uint_as_float(r[j + 1])));
+        u = __hadd2(u, *reinterpret_cast<const __half2*>(&bw[k]));
+        const __half2 o = gelu_times_h2(u, half_g);
+        pk[4 * v + k] = *reinterpret_cast<const uint32_t*>(&o);
+      }
+    }
+    // the previous TMA store of this warp must have finished reading the tile
+    if (lane == 0) bulk_wait_group_read<0>();
+    __syncwarp();
+    // row `lane` of the 32x64 tile; 16-byte chunk cc sits at chunk position
+    // cc ^ (row % 8), the 128-byte swizzle of the store map (bank-conflict free)
+#pragma unroll
+    for (int cc = 0; cc < 8; ++cc)
+      st_shared_v4(tile_addr + lane * 128 + ((cc ^ (lane & 7)) << 4), pk[4 * cc], pk[4 * cc + 1],
+                   pk[4 * cc + 2], pk[4 * cc + 3]);
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_3d(tmS, tile, n0 + col0, m * UM + q * 32, gl);
+      bulk_commit_group();
+    }
+  }
+}
+
+// GEMM2 epilogue of one warp: row 32*q + lane of the tile, columns
+// [col_begin, col_begin + 32 * n_chunks) of output tile n0.
+__device__ __forceinline__ void epilogue_gemm2(const PathArgs& p, uint32_t tbase, int q, int lane,
+                                               int grp, int m, int n0, int col_begin,
+                                               int n_chunks) {
+  const Dims& d = p.d;
+  const int row = q * 32 + lane;
+  const size_t grow = static_cast<size_t>(m) * UM + row;
+  const GroupInfo gi = p.groups[grp];
+  const TileInfo ti = p.tiles[m];
+  const bool valid = row < ti.rows;
+  const float* grow_g = p.gate + (static_cast<size_t>(grp) * d.tpad + grow) * d.E;
+  float g[kMaxE];
+#pragma unroll
+  for (int e = 0; e < kMaxE; ++e) g[e] = e < d.E ? grow_g[e] : 0.f;
+  __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.dst[gi.x]);
+  const size_t s = static_cast<size_t>(ti.s0) + row;
+#pragma unroll 1
+  for (int ch = 0; ch < n_chunks; ++ch) {
+    const int cl = col_begin + ch * 32;
+    uint32_t r[32];
+    tmem_ld_32x32b_x32(tbase + cl, r);
+    tmem_ld_wait(r);
+    const int c = n0 + cl;
+    float y[32];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) y[j] = __uint_as_float(r[j]);
+#pragma unroll
+    for (int e = 0; e < kMaxE; ++e) {
+      if (e < d.E) {
+        const float4* b4 =
+            reinterpret_cast<const float4*>(p.b2 + (static_cast<size_t>(grp) * d.E + e) * d.Dt + c);
+#pragma unroll
+        for (int v = 0; v < 8; ++v) {
+          const float4 bb = __ldg(b4 + v);
+          y[4 * v + 0] = fmaf(g[e], bb.x, y[4 * v + 0]);
+          y[4 * v + 1] = fmaf(g[e], bb.y, y[4 * v + 1]);
+          y[4 * v + 2] = fmaf(g[e], bb.z, y[4 * v + 2]);
+          y[4 * v + 3] = fmaf(g[e], bb.w, y[4 * v + 3]);
+        }
+      }
+    }
+    if (valid) {
+      const int h = c / d.d_t, i0 = c - h * d.d_t;
+      uint4* o4 = reinterpret_cast<uint4*>(
+          dst + ((((static_cast<size_t>(gi.tgt_layer) * d.B + ti.b) * d.H_t + h) * d.S + s) * d.d_t +
+                 i0));
+#pragma unroll
+      for (int v = 0; v < 4; ++v)
+        o4[v] = make_uint4(pack_bf16x2(y[8 * v + 0], y[8 * v + 1]),
+                           pack_bf16x2(y[8 * v + 2], y[8 * v + 3]),
+                           pack_bf16x2(y[8 * v + 4], y[8 * v + 5]),
+                           pack_bf16x2(y[8 * v + 6], y[8 * v + 7]));
+    }
+  }
+}
+
+}  // namespace mot

@@ -62,6 +62,8 @@ _SIGS = {
     "mot_destroy": [_H],
     "mot_get_layer_map": [_H, _P, ctypes.c_int32],
     "mot_get_path": [_H, ctypes.POINTER(ctypes.c_int32)],
+    "mot_set_schedule": [_H, ctypes.c_int32],
+    "mot_get_schedule": [_H, ctypes.POINTER(ctypes.c_int32)],
     "mot_profile_enable": [_H, ctypes.c_int32],
     "mot_profile_read": [_H, ctypes.POINTER(mot_kernel_stat), ctypes.c_int32,
                          ctypes.POINTER(ctypes.c_int32)],
@@ -204,6 +206,19 @@ def mot_get_path(h: Handle) -> int:
     p = ctypes.c_int32()
     _check(_lib.mot_get_path(h.ptr, ctypes.byref(p)), "mot_get_path")
     return p.value
+
+
+SCHEDULE_SPLIT, SCHEDULE_FUSED, SCHEDULE_PAIR = 0, 1, 2
+
+
+def mot_set_schedule(h: Handle, schedule: int) -> None:
+    _check(_lib.mot_set_schedule(h.ptr, int(schedule)), "mot_set_schedule")
+
+
+def mot_get_schedule(h: Handle) -> int:
+    v = ctypes.c_int32()
+    _check(_lib.mot_get_schedule(h.ptr, ctypes.byref(v)), "mot_get_schedule")
+    return v.value
 
 
 def mot_profile_enable(h: Handle, enable: bool = True) -> None:

@@ -50,15 +50,34 @@ SMALL = {
 }
 
 
+@pytest.mark.parametrize("schedule", [2, 1, 0])
 @pytest.mark.parametrize("name", sorted(SMALL))
-def test_small_shapes_every_element(name):
+def test_small_shapes_every_element(name, schedule):
     wl = SMALL[name]
+    if schedule != 2 and not name.startswith("umma"):
+        pytest.skip("the schedule only applies to the tensor-core path")
     sk, sv, blob = inputs(wl, seed=1)
     run = G.Run(wl, sk, sv, blob)
     expect_path = 1 if name.startswith("umma") else 0
     assert M.mot_get_path(run.h) == expect_path
+    M.mot_set_schedule(run.h, schedule)
     assert run.translate() == M.MOT_OK
     full_check(wl, run, sk, sv, blob, name)
+
+
+@pytest.mark.parametrize("other", [1, 2])
+@pytest.mark.parametrize("name", ["umma_ragged", "umma_e3", "gpt2s_opt125m", "qwen7_long"])
+def test_launch_schedules_are_bit_identical(name, other):
+    """Every launch schedule runs the same per-tile arithmetic in the same order."""
+    wl = SMALL.get(name) or synth.WORKLOADS[name]
+    sk, sv, blob = inputs(wl, seed=3)
+    a = G.Run(wl, sk, sv, blob)
+    b = G.Run(wl, sk, sv, blob)
+    M.mot_set_schedule(a.h, 0)
+    M.mot_set_schedule(b.h, other)
+    assert a.translate() == M.MOT_OK and b.translate() == M.MOT_OK
+    assert torch.equal(G.int_view(a.dk), G.int_view(b.dk))
+    assert torch.equal(G.int_view(a.dv), G.int_view(b.dv))
 
 
 def test_tiny_fp32_workload_every_element():
@@ -236,14 +255,20 @@ def test_argument_errors_with_a_live_handle():
     M.mot_destroy(h)
 
 
-def test_profile_and_launch_count():
+@pytest.mark.parametrize("schedule,kernels", [
+    (2, {"prep_tiles", "gate", "umma2_gemm1_gelu_gate", "umma2_gemm2_combine_store"}),
+    (1, {"prep_tiles", "gate", "umma_fused_translate"}),
+    (0, {"prep_tiles", "gate", "umma_gemm1_gelu_gate", "umma_gemm2_combine_store"})])
+def test_profile_and_launch_count(schedule, kernels):
     wl = SMALL["umma_ragged"]
     sk, sv, blob = inputs(wl, seed=10)
     run = G.Run(wl, sk, sv, blob)
+    assert M.mot_get_schedule(run.h) == 2
+    M.mot_set_schedule(run.h, schedule)
     n0 = M.mot_get_launch_count(run.h)
     M.mot_profile_enable(run.h, True)
     assert run.translate() == M.MOT_OK
     stats = M.mot_profile_read(run.h)
-    assert set(stats) == {"prep_tiles", "gate", "umma_gemm1_gelu_gate", "umma_gemm2_combine_store"}
+    assert set(stats) == kernels
     assert all(v[0] >= 1 and v[1] > 0 for v in stats.values())
     assert M.mot_get_launch_count(run.h) - n0 == sum(v[0] for v in stats.values())

@@ -143,6 +143,37 @@ mot_status mot_destroy(mot_handle h);
 /* Static, human-readable name of a status code. */
 const char* mot_status_string(mot_status s);
 
+/*
+ * Allocation-free translation (the paper has no counterpart: this is a service
+ * for callers that cannot call cudaMalloc, such as a process whose device
+ * memory is divided up front by its own pool allocator and forbids further
+ * allocations, or a host that must not grow its device footprint per call).
+ * No handle: `cfg` is as for mot_create (layer_map NULL = depth-ratio map),
+ * `weights` is the packed blob of mot_load_weights already in the caller's
+ * DEVICE memory (16-byte aligned, cfg.dtype), and the caches and device
+ * seq_lens are as for mot_translate. Nothing is allocated: the per-call
+ * intermediates live in one 64 MiB __device__ scratch array
+ * (MOT_STATIC_SCRATCH_BYTES) that every GPU which loads this library holds
+ * until the process exits. A call needs
+ *   256-rounded(batch * S_pad * E * 4) + batch * S_pad * E * H * 4 bytes,
+ *   S_pad = max_seq rounded up to 64,
+ * and returns MOT_ERR_UNSUPPORTED, before any CUDA call, when that exceeds the
+ * array. The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current); make that first call
+ * before any stream capture. All calls share the array and it keeps the last
+ * call's contents (nothing in it needs to start at zero): calls that overlap
+ * on the GPU, on any streams, race with each other. Lengths outside
+ * [0, max_seq] are clamped; there is no status word to report them. The
+ * arithmetic is fp32 FFMA throughout (exact-erf GELU), so bf16 results match
+ * mot_translate's within the bf16 tolerance and fp32 results to ~1e-6.
+ * Asynchronous on `stream`. Errors: MOT_ERR_INVALID_ARG, MOT_ERR_UNSUPPORTED,
+ * MOT_ERR_CUDA.
+ */
+#define MOT_STATIC_SCRATCH_BYTES ((size_t)64 << 20)
+mot_status mot_translate_static(const mot_config* cfg, const void* weights, const void* src_k,
+                                const void* src_v, const int32_t* seq_lens, int32_t batch,
+                                void* dst_k, void* dst_v, mot_stream_t stream);
+
 /* ---- introspection (no method counterpart; for tests and benchmarks) ------ */
 
 /* The channel map in use: out[n_layers_tgt] (n must equal n_layers_tgt). */

@@ -68,6 +68,8 @@ _SIGS = {
     "mot_profile_read": [_H, ctypes.POINTER(mot_kernel_stat), ctypes.c_int32,
                          ctypes.POINTER(ctypes.c_int32)],
     "mot_get_launch_count": [_H, ctypes.POINTER(ctypes.c_int64)],
+    "mot_translate_static": [ctypes.POINTER(mot_config), _P, _P, _P, _P, ctypes.c_int32, _P, _P,
+                             _P],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -183,6 +185,17 @@ def mot_translate_host(h: Handle, src_k, src_v, seq_lens, batch: int, dst_k, dst
     _check(_lib.mot_translate_host(h.ptr, _addr(src_k), _addr(src_v), _addr(seq_lens), int(batch),
                                    _addr(dst_k), _addr(dst_v), _stream(stream)),
            "mot_translate_host")
+
+
+MOT_STATIC_SCRATCH_BYTES = 64 << 20
+
+
+def mot_translate_static(cfg: mot_config, weights, src_k, src_v, seq_lens, batch: int, dst_k,
+                         dst_v, stream=None) -> None:
+    """Allocation-free translation: no handle, weights (packed blob) in device memory."""
+    _check(_lib.mot_translate_static(ctypes.byref(cfg), _addr(weights), _addr(src_k),
+                                     _addr(src_v), _addr(seq_lens), int(batch), _addr(dst_k),
+                                     _addr(dst_v), _stream(stream)), "mot_translate_static")
 
 
 def mot_get_device_status(h: Handle, stream=None) -> int:

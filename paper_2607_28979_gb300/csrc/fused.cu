@@ -184,8 +184,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive_expect_tx(&full[stage], kStageBytes);
           if (it.type == 1) {
             const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
-            tma_load_5d(sA + stage * kABytes, gi.x ? &tmV : &tmK, &full[stage], d0, ti.s0, h, ti.b,
-                        gi.src_layer);
+            tma_load_2d(sA + stage * kABytes, gi.x ? &tmV : &tmK, &full[stage], d0,
+                        ((gi.src_layer * d.B + ti.b) * d.H_s + h) * d.S + ti.s0);
             tma_load_2d(sB + stage * kBBytes, &tmW1, &full[stage], kb * UK,
                         grp * d.EH + it.n * UN);
           } else {

@@ -185,6 +185,9 @@ mot_status validate(const mot_config* c) {
   const long long tiles = (long long)c->max_batch * ((c->max_seq + kTileM - 1) / kTileM);
   if (tiles * kTileM > INT32_MAX / 2) return MOT_ERR_UNSUPPORTED;
   if ((long long)c->n_translators * c->hidden > (1 << 24)) return MOT_ERR_UNSUPPORTED;
+  // TMA row coordinates of the caches are 32-bit
+  if ((long long)c->n_layers_src * c->max_batch * c->src_kv_heads * c->max_seq > INT32_MAX / 2)
+    return MOT_ERR_UNSUPPORTED;
   return MOT_OK;
 }
 
@@ -237,14 +240,12 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
 
   CUtensorMap tmK{}, tmV{};
   if (h->use_umma) {
-    const uint64_t dims[5] = {uint64_t(d.d_s), uint64_t(d.S), uint64_t(d.H_s), uint64_t(d.B),
-                              uint64_t(d.L_s)};
-    const uint64_t st_b[4] = {uint64_t(d.d_s) * 2, uint64_t(d.S) * d.d_s * 2,
-                              uint64_t(d.H_s) * d.S * d.d_s * 2,
-                              uint64_t(d.B) * d.H_s * d.S * d.d_s * 2};
-    const uint32_t box[5] = {uint32_t(kUmmaK), uint32_t(kTileM), 1, 1, 1};
-    if (!encode_bf16(&tmK, src_k, 5, dims, st_b, box) ||
-        !encode_bf16(&tmV, src_v, 5, dims, st_b, box))
+    // the source cache as rows of d_s elements: row ((l * B + b) * H_s + h) * S + s
+    const uint64_t dims[2] = {uint64_t(d.d_s), uint64_t(d.L_s) * d.B * d.H_s * d.S};
+    const uint64_t st_b[1] = {uint64_t(d.d_s) * 2};
+    const uint32_t box[2] = {uint32_t(kUmmaK), uint32_t(kTileM)};
+    if (!encode_bf16(&tmK, src_k, 2, dims, st_b, box) ||
+        !encode_bf16(&tmV, src_v, 2, dims, st_b, box))
       return MOT_ERR_CUDA;
   }
 

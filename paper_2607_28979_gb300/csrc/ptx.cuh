@@ -343,12 +343,14 @@ __device__ __forceinline__ void umma_commit_pair(uint64_t* bar) {
       : "memory");
 }
 
-// Arrive on the barrier at `bar`'s offset in cluster CTA `cta`.
+// Arrive on the barrier at `bar`'s offset in cluster CTA `cta` (default
+// semantics: release at CTA scope; callers order their tcgen05 reads with
+// tcgen05.wait::ld and tcgen05.fence before arriving).
 __device__ __forceinline__ void mbar_arrive_cluster(uint64_t* bar, uint32_t cta) {
   asm volatile(
       "{\n\t.reg .b32 ra;\n\t"
       "mapa.shared::cluster.u32 ra, %0, %1;\n\t"
-      "mbarrier.arrive.release.cluster.shared::cluster.b64 _, [ra];\n\t}" ::"r"(smem_u32(bar)),
+      "mbarrier.arrive.shared::cluster.b64 _, [ra];\n\t}" ::"r"(smem_u32(bar)),
       "r"(cta)
       : "memory");
 }

@@ -25,11 +25,13 @@
 // (mot::mbar_wait); on a timeout all roles unwind, in-flight copies and MMAs
 // are drained, TMEM is freed and kStatusTimeout is raised.
 //
-// GEMM1's A operand is read straight from the source cache
-// [L_s][B][H_s][S][d_s] through a 5-D tensor map with box (64, 128, 1, 1, 1):
-// K-block kb is head kb*64 / d_s, dims (kb*64) % d_s .. +63, of 128
-// consecutive positions of one batch entry. Positions past the cache end read
-// as zero; rows past the tile's length are computed but never stored.
+// GEMM1's A operand is read straight from the source cache [L_s][B][H_s][S][d_s]
+// through a 2-D tensor map over its rows (inner dim d_s, row
+// ((l * B + b) * H_s + h) * S + s) with box (64, 128): K-block kb is head
+// kb*64 / d_s, dims (kb*64) % d_s .. +63, of 128 consecutive positions of one
+// batch entry. In a short last tile the rows past S are the next head's (or,
+// at the end of the cache, zeros); rows past the tile's length are computed
+// but never stored.
 #include "umma_common.cuh"
 
 namespace mot {
@@ -134,8 +136,8 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
           mbar_arrive_expect_tx(&full[stage], kStageBytes);
           if (MODE == 1) {
             const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
-            tma_load_5d(sA + stage * kABytes, gi.x ? &tmA1 : &tmA0, &full[stage], d0, ti.s0, h,
-                        ti.b, gi.src_layer);
+            tma_load_2d(sA + stage * kABytes, gi.x ? &tmA1 : &tmA0, &full[stage], d0,
+                        ((gi.src_layer * d.B + ti.b) * d.H_s + h) * d.S + ti.s0);
           } else {
             tma_load_3d(sA + stage * kABytes, &tmA0, &full[stage], kb * UK, m * UM, gl);
           }

@@ -16,8 +16,8 @@
 //   warps 4.. (both CTAs)      epilogue of its own 128 accumulator rows, then
 //                              an arrive on the leader's accumulator-free
 //                              barrier.
-// A token tile past the last one (odd tile count) is read as zeros by TMA and
-// never stored. Every wait is bounded; a timeout unwinds and raises
+// A token tile past the last one (odd tile count) is computed from arbitrary
+// in-bounds rows and never stored. Every wait is bounded; a timeout unwinds and raises
 // kStatusTimeout.
 #include "umma_common.cuh"
 
@@ -132,9 +132,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
           gi = p.groups[grp];
           if (m_own < n_m) {
             ti = p.tiles[m_own];
-          } else {   // no such tile: rows past the cache end read as zeros
+          } else {   // no such tile: load any in-bounds rows; they are never stored
             ti.b = 0;
-            ti.s0 = d.S;
+            ti.s0 = 0;
           }
         }
         bool ok = true;
@@ -144,8 +144,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
           const uint32_t bar = leader_addr(&full[stage]);
           if (MODE == 1) {
             const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
-            tma_load_5d_pair(sA + stage * kABytes2, gi.x ? &tmA1 : &tmA0, bar, d0, ti.s0, h, ti.b,
-                             gi.src_layer);
+            tma_load_2d_pair(sA + stage * kABytes2, gi.x ? &tmA1 : &tmA0, bar, d0,
+                             ((gi.src_layer * d.B + ti.b) * d.H_s + h) * d.S + ti.s0);
           } else {
             tma_load_3d_pair(sA + stage * kABytes2, &tmA0, bar, kb * UK, m_own * UM, gl);
           }

@@ -161,6 +161,22 @@ class ClockSampler:
                 "samples": len(rows), "power_w_max": max(pw) if pw else None}
 
 
+def reduce_max(values, world: int, device):
+    """Element-wise max over all ranks of a list of floats (identity on one rank)."""
+    if world == 1:
+        return [float(v) for v in values]
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def aggregate_throughput(tokens_per_rank: int, world: int, seconds_max: float) -> float:
+    """Whole-job throughput: every rank's tokens over the slowest rank's time."""
+    return world * tokens_per_rank / seconds_max
+
+
 def dist_setup(gpus: int):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -339,14 +355,10 @@ def run_mot(args, wl):
     d2h = 2 * tl * wl.tokens * wl.d_tgt * es
 
     # ---- aggregate over ranks: max time
-    t_step = elapsed_ms / args.steps
-    if world > 1:
-        t = torch.tensor([t_step, e2e_s], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        t_step, e2e_s = float(t[0]), float(t[1])
+    t_step, e2e_s = reduce_max([elapsed_ms / args.steps, e2e_s], world, "cuda")
     tokens = wl.tokens
-    value = world * tokens / (t_step / 1000.0)
-    e2e_value = world * tokens * e2e_steps / e2e_s
+    value = aggregate_throughput(tokens, world, t_step / 1000.0)
+    e2e_value = aggregate_throughput(tokens * e2e_steps, world, e2e_s)
 
     if rank == 0:
         alg = algorithmic(wl, M.mot_get_layer_map(h))

@@ -209,6 +209,17 @@ typedef struct {
 mot_status mot_profile_enable(mot_handle h, int32_t enable);
 mot_status mot_profile_read(mot_handle h, mot_kernel_stat* out, int32_t cap, int32_t* n);
 
+/*
+ * Failure-detection test hook. Every device pipeline wait of this handle's
+ * kernels gives up after `wait_limit_cycles` SM cycles (0 = the default, about
+ * two seconds), sets MOT_ERR_TIMEOUT in the status word and unwinds (copies
+ * and MMAs in flight are drained, TMEM is freed). With stall_test = 1, the
+ * first CTA of the single-SM GEMM1 kernel (schedule 0) never fills its first
+ * pipeline stage, so a wait on it runs out: translations then report
+ * MOT_ERR_TIMEOUT through mot_get_device_status and the context stays usable.
+ */
+mot_status mot_debug_set(mot_handle h, int32_t stall_test, int64_t wait_limit_cycles);
+
 /* Number of kernels this handle has launched since it was created. */
 mot_status mot_get_launch_count(mot_handle h, int64_t* count);
 

@@ -65,7 +65,7 @@ __device__ __forceinline__ void signal_done(int32_t* ctr) {
 
 // Bounded acquire-spin until *ctr >= target; then order the async proxy.
 __device__ __forceinline__ bool wait_done(const int32_t* ctr, int target,
-                                          volatile int* abort_flag) {
+                                          volatile int* abort_flag, long long limit) {
   const long long t0 = clock64();
   for (;;) {
     if (ld_acquire(ctr) >= target) {
@@ -73,7 +73,7 @@ __device__ __forceinline__ bool wait_done(const int32_t* ctr, int target,
       return true;
     }
     if (*abort_flag) return false;
-    if (clock64() - t0 > kWaitLimitCycles) {
+    if (clock64() - t0 > limit) {
       *abort_flag = 1;
       return false;
     }
@@ -161,7 +161,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0, slot = 0;
       uint32_t phase = 0, sphase = 0;
       for (;;) {
-        if (!mbar_wait(&iempty[slot], sphase ^ 1u, abort_flag)) break;
+        if (!mbar_wait(&iempty[slot], sphase ^ 1u, abort_flag, p.wait_limit)) break;
         int i = atomicAdd(fa.counters, 1);
         if (i >= total) i = -1;
         ring[slot] = i;
@@ -170,7 +170,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (i < 0) break;
         const Item it = schedule_item(sch, i);
         const int gl = it.f / n_m, m = it.f - gl * n_m, grp = p.g0 + gl;
-        if (it.type == 2 && !wait_done(done + it.f, done_target, abort_flag)) break;
+        if (it.type == 2 && !wait_done(done + it.f, done_target, abort_flag, p.wait_limit)) break;
         TileInfo ti;
         GroupInfo gi;
         if (it.type == 1) {
@@ -180,7 +180,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int nk = it.type == 1 ? fa.nk1 : fa.nk2;
         bool ok = true;
         for (int kb = 0; kb < nk; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[stage], kStageBytes);
           if (it.type == 1) {
             const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
@@ -208,7 +208,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0, slot = 0, acc = 0;
       uint32_t phase = 0, sphase = 0, acc_phase = 0;
       for (;;) {
-        if (!mbar_wait(&ifull[slot], sphase, abort_flag)) break;
+        if (!mbar_wait(&ifull[slot], sphase, abort_flag, p.wait_limit)) break;
         const int i = ring[slot];
         mbar_arrive(&iempty[slot]);
         if (++slot == kRing) { slot = 0; sphase ^= 1u; }
@@ -216,12 +216,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         const Item it = schedule_item(sch, i);
         const int nk = it.type == 1 ? fa.nk1 : fa.nk2;
         const uint32_t idesc = it.type == 1 ? idesc1 : idesc2;
-        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag)) break;
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, p.wait_limit)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * UN);
         bool ok = true;
         for (int kb = 0; kb < nk; ++kb) {
-          if (!mbar_wait(&full[stage], phase, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(&full[stage], phase, abort_flag, p.wait_limit)) { ok = false; break; }
           tc_fence_after();
           const uint64_t adesc = sdesc_k_sw128(smem_u32(sA + stage * kABytes));
           const uint64_t bdesc = sdesc_k_sw128(smem_u32(sB + stage * kBBytes));
@@ -248,7 +248,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (;;) {
       int ok = 1, i = 0;
       if (lane == 0) {
-        ok = mbar_wait(&ifull[slot], sphase, abort_flag) ? 1 : 0;
+        ok = mbar_wait(&ifull[slot], sphase, abort_flag, p.wait_limit) ? 1 : 0;
         if (ok) i = ring[slot];
       }
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -263,7 +263,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (i < 0) break;
       const Item it = schedule_item(sch, i);
       const int gl = it.f / n_m, m = it.f - gl * n_m, grp = p.g0 + gl;
-      if (lane == 0) ok = mbar_wait(&tfull[acc], acc_phase, abort_flag) ? 1 : 0;
+      if (lane == 0) ok = mbar_wait(&tfull[acc], acc_phase, abort_flag, p.wait_limit) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
@@ -294,7 +294,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if ((issued_mask >> s) & 1u) {
           const uint32_t a = smem_u32(&full[s]);
           const long long t0 = clock64();
-          while (!mbar_try_wait(a, (issue_parity >> s) & 1u) && clock64() - t0 < kWaitLimitCycles) {
+          while (!mbar_try_wait(a, (issue_parity >> s) & 1u) && clock64() - t0 < p.wait_limit) {
           }
         }
     }
@@ -302,7 +302,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       umma_commit(drain);
       const uint32_t a = smem_u32(drain);
       const long long t0 = clock64();
-      while (!mbar_try_wait(a, 0) && clock64() - t0 < kWaitLimitCycles) {
+      while (!mbar_try_wait(a, 0) && clock64() - t0 < p.wait_limit) {
       }
     }
     __syncthreads();

@@ -75,6 +75,8 @@ struct mot_ctx {
   int num_sms = 0;
   bool use_umma = false;
   int schedule = 2;           // tcgen05 path: 0 split, 1 fused, 2 split on CTA pairs
+  long long wait_limit = 4000000000LL;   // bound of every pipeline wait (SM cycles)
+  int stall_test = 0;                    // test hook, see mot_debug_set
   bool weights_loaded = false;
   int gp_max = 1;
   std::vector<GroupInfo> groups_h;
@@ -217,6 +219,8 @@ PathArgs path_args(mot_ctx* h) {
   a.gate = h->gate;
   a.a2 = h->a2;
   a.status = h->status;
+  a.wait_limit = h->wait_limit;
+  a.stall_test = h->stall_test;
   return a;
 }
 
@@ -622,6 +626,13 @@ mot_status mot_set_schedule(mot_handle h, int32_t schedule) {
 mot_status mot_get_schedule(mot_handle h, int32_t* schedule) {
   if (!h || !schedule) return MOT_ERR_INVALID_ARG;
   *schedule = h->schedule;
+  return MOT_OK;
+}
+
+mot_status mot_debug_set(mot_handle h, int32_t stall_test, int64_t wait_limit_cycles) {
+  if (!h || stall_test < 0 || stall_test > 1 || wait_limit_cycles < 0) return MOT_ERR_INVALID_ARG;
+  h->stall_test = stall_test;
+  h->wait_limit = wait_limit_cycles > 0 ? wait_limit_cycles : 4000000000LL;
   return MOT_OK;
 }
 

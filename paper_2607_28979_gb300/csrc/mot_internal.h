@@ -64,7 +64,9 @@ struct PathArgs {
   float* gate;
   void* a2;
   int32_t* status;
-  int32_t g0, gp;   // groups [g0, g0 + gp) of this pass
+  int32_t g0, gp;         // groups [g0, g0 + gp) of this pass
+  long long wait_limit;   // bound of every pipeline wait, in SM cycles
+  int32_t stall_test;     // test hook (single-SM GEMM1): CTA 0 withholds its first stage
 };
 
 // Kernel launchers (each returns the launch's cudaError_t).

@@ -53,9 +53,10 @@ constexpr long long kWaitLimitCycles = 4000000000LL;
 
 // Wait for phase `parity` of `bar` to complete. Returns false (without
 // completing) once `abort_flag` is set by any thread of the CTA, or after
-// kWaitLimitCycles, in which case this thread sets `abort_flag` itself.
+// `limit` cycles, in which case this thread sets `abort_flag` itself.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
-                                          volatile int* abort_flag) {
+                                          volatile int* abort_flag,
+                                          long long limit = kWaitLimitCycles) {
   const uint32_t a = smem_u32(bar);
   if (mbar_try_wait(a, parity)) return true;
   const long long t0 = clock64();
@@ -63,7 +64,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
     if (mbar_try_wait(a, parity)) return true;
     if ((it & 63u) == 0) {
       if (*abort_flag) return false;
-      if (clock64() - t0 > kWaitLimitCycles) {
+      if (clock64() - t0 > limit) {
         *abort_flag = 1;
         return false;
       }

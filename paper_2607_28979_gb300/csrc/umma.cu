@@ -132,7 +132,12 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
         }
         bool ok = true;
         for (int kb = 0; kb < ua.nk; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit)) { ok = false; break; }
+          if (MODE == 1 && p.stall_test && blockIdx.x == 0 && t == 0 && kb == 0) {
+            // test hook: this stage is never filled, so the MMA wait on it runs out
+            if (++stage == kStages) { stage = 0; phase ^= 1u; }
+            continue;
+          }
           mbar_arrive_expect_tx(&full[stage], kStageBytes);
           if (MODE == 1) {
             const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
@@ -160,12 +165,12 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       for (int t = blockIdx.x; t < total; t += gridDim.x) {
-        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag)) break;
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, p.wait_limit)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * UN);
         bool ok = true;
         for (int kb = 0; kb < ua.nk; ++kb) {
-          if (!mbar_wait(&full[stage], phase, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(&full[stage], phase, abort_flag, p.wait_limit)) { ok = false; break; }
           tc_fence_after();
           const uint64_t adesc = sdesc_k_sw128(smem_u32(sA + stage * kABytes));
           const uint64_t bdesc = sdesc_k_sw128(smem_u32(sB + stage * kBBytes));
@@ -190,7 +195,7 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
     uint32_t acc_phase = 0;
     for (int t = blockIdx.x; t < total; t += gridDim.x) {
       int ok = 1;
-      if (lane == 0) ok = mbar_wait(&tfull[acc], acc_phase, abort_flag) ? 1 : 0;
+      if (lane == 0) ok = mbar_wait(&tfull[acc], acc_phase, abort_flag, p.wait_limit) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
@@ -225,7 +230,7 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
           const uint32_t a = smem_u32(&full[s]);
           const long long t0 = clock64();
           while (!mbar_try_wait(a, (issue_parity >> s) & 1u) &&
-                 clock64() - t0 < kWaitLimitCycles) {
+                 clock64() - t0 < p.wait_limit) {
           }
         }
     }
@@ -233,7 +238,7 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
       umma_commit(drain);
       const uint32_t a = smem_u32(drain);
       const long long t0 = clock64();
-      while (!mbar_try_wait(a, 0) && clock64() - t0 < kWaitLimitCycles) {
+      while (!mbar_try_wait(a, 0) && clock64() - t0 < p.wait_limit) {
       }
     }
     __syncthreads();

@@ -139,7 +139,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
         }
         bool ok = true;
         for (int kb = 0; kb < ua.nk; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit)) { ok = false; break; }
           if (leader) mbar_arrive_expect_tx(&full[stage], 2 * kStageBytes2);
           const uint32_t bar = leader_addr(&full[stage]);
           if (MODE == 1) {
@@ -165,12 +165,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
       for (int t = pair; t < total; t += n_pairs) {
-        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag)) break;
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, p.wait_limit)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * UN);
         bool ok = true;
         for (int kb = 0; kb < ua.nk; ++kb) {
-          if (!mbar_wait(&full[stage], phase, abort_flag)) { ok = false; break; }
+          if (!mbar_wait(&full[stage], phase, abort_flag, p.wait_limit)) { ok = false; break; }
           tc_fence_after();
           const uint64_t adesc = sdesc_k_sw128(smem_u32(sA + stage * kABytes2));
           const uint64_t bdesc = sdesc_k_sw128(smem_u32(sB + stage * kBBytes2));
@@ -195,7 +195,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
     uint32_t acc_phase = 0;
     for (int t = pair; t < total; t += n_pairs) {
       int ok = 1;
-      if (lane == 0) ok = mbar_wait(&tfull[acc], acc_phase, abort_flag) ? 1 : 0;
+      if (lane == 0) ok = mbar_wait(&tfull[acc], acc_phase, abort_flag, p.wait_limit) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
@@ -234,7 +234,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
             const uint32_t a = smem_u32(&full[s]);
             const long long t0 = clock64();
             while (!mbar_try_wait(a, (issue_parity >> s) & 1u) &&
-                   clock64() - t0 < kWaitLimitCycles) {
+                   clock64() - t0 < p.wait_limit) {
             }
           }
       } else {
@@ -245,7 +245,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
       umma_commit_pair(drain);
       const uint32_t a = smem_u32(drain);
       const long long t0 = clock64();
-      while (!mbar_try_wait(a, 0) && clock64() - t0 < kWaitLimitCycles) {
+      while (!mbar_try_wait(a, 0) && clock64() - t0 < p.wait_limit) {
       }
     }
     __syncthreads();

@@ -68,6 +68,7 @@ _SIGS = {
     "mot_profile_read": [_H, ctypes.POINTER(mot_kernel_stat), ctypes.c_int32,
                          ctypes.POINTER(ctypes.c_int32)],
     "mot_get_launch_count": [_H, ctypes.POINTER(ctypes.c_int64)],
+    "mot_debug_set": [_H, ctypes.c_int32, ctypes.c_int64],
     "mot_translate_static": [ctypes.POINTER(mot_config), _P, _P, _P, _P, ctypes.c_int32, _P, _P,
                              _P],
 }
@@ -232,6 +233,10 @@ def mot_get_schedule(h: Handle) -> int:
     v = ctypes.c_int32()
     _check(_lib.mot_get_schedule(h.ptr, ctypes.byref(v)), "mot_get_schedule")
     return v.value
+
+
+def mot_debug_set(h: Handle, stall_test: bool, wait_limit_cycles: int = 0) -> None:
+    _check(_lib.mot_debug_set(h.ptr, int(bool(stall_test)), int(wait_limit_cycles)), "mot_debug_set")
 
 
 def mot_profile_enable(h: Handle, enable: bool = True) -> None:

@@ -272,3 +272,62 @@ def test_profile_and_launch_count(schedule, kernels):
     assert set(stats) == kernels
     assert all(v[0] >= 1 and v[1] > 0 for v in stats.values())
     assert M.mot_get_launch_count(run.h) - n0 == sum(v[0] for v in stats.values())
+
+
+# ---------------------------------------------------------------- Top-K routing (Def. 3.1)
+
+TOPK = {
+    # the paper's default (Top-K, N_Tr) = (1, 2), tensor-core path
+    "umma_top1_of2": synth.Workload("umma_top1_of2", 2, 2, 64, 3, 2, 128, 2, 256, 2, 200, "bf16",
+                                    (200, 61), top_k=1),
+    # (2, 4), tensor-core path
+    "umma_top2_of4": synth.Workload("umma_top2_of4", 2, 2, 64, 2, 2, 128, 4, 256, 2, 160, "bf16",
+                                    (160, 33), top_k=2),
+    # SIMT fp32 path, Top-3 of 5
+    "simt_fp32_top3_of5": synth.Workload("simt_fp32_top3_of5", 2, 2, 12, 2, 3, 10, 5, 30, 2, 50,
+                                         "fp32", (50, 17), top_k=3),
+}
+
+
+@pytest.mark.parametrize("name", sorted(TOPK))
+def test_topk_routing_against_oracle(name):
+    """Top-K keeps the K largest gate scores and renormalises over them. Where
+    the K-th and (K+1)-th scores are within 1e-4, fp32 and fp64 may keep
+    different experts (both valid): such tokens are excluded, and must be rare."""
+    wl = TOPK[name]
+    sk, sv, blob = inputs(wl, seed=12)
+    run = G.Run(wl, sk, sv, blob)
+    assert run.translate() == M.MOT_OK
+    assert run.canaries_intact() and run.padding_untouched()
+    tb = np.concatenate([np.full(L, b) for b, L in enumerate(wl.seq_lens)]).astype(np.int32)
+    ts = np.concatenate([np.arange(L) for L in wl.seq_lens]).astype(np.int32)
+    ref, _ = oracle.translate_tokens(wl, sk, sv, blob, tb, ts, want_gate=True)
+    _, dense = oracle.translate_tokens(wl.replace(top_k=0), sk, sv, blob, tb, ts, want_gate=True)
+    srt = -np.sort(-dense, axis=-1)                       # [L_t][2][n][E], descending
+    margin = srt[..., wl.top_k - 1] - srt[..., wl.top_k]  # [L_t][2][n]
+    ok = margin >= 1e-4
+    tl = wl.translated_layers()
+    assert ok[tl].mean() > 0.99
+    got = run.gather(tb, ts)
+    keep = np.broadcast_to(ok[..., None], got.shape)
+    G.assert_parity(wl, got[tl][keep[tl]], ref[tl][keep[tl]], name)
+
+
+# ---------------------------------------------------------------- failure detection
+
+def test_bounded_wait_reports_timeout_and_the_context_survives():
+    """A pipeline stage that is never filled makes a bounded wait run out: the
+    kernels unwind, the status word reports MOT_ERR_TIMEOUT, and the next
+    translation on the same context is correct."""
+    wl = SMALL["umma_ragged"]
+    sk, sv, blob = inputs(wl, seed=11)
+    run = G.Run(wl, sk, sv, blob)
+    M.mot_set_schedule(run.h, 0)
+    M.mot_debug_set(run.h, True, 20_000_000)      # about 10 ms of SM cycles
+    assert run.translate() == M.MOT_ERR_TIMEOUT
+    assert M.mot_get_device_status(run.h) == M.MOT_OK   # reading cleared it
+    M.mot_debug_set(run.h, False, 0)
+    run.buf_k, run.dk = G.alloc_dst(wl)
+    run.buf_v, run.dv = G.alloc_dst(wl)
+    assert run.translate() == M.MOT_OK
+    full_check(wl, run, sk, sv, blob, "after a timeout")

@@ -23,7 +23,26 @@ __global__ void f32_to_f16_kernel(const float* src, uint16_t* dst, size_t n) {
     dst[i] = __half_as_ushort(__float2half_rn(src[i]));
 }
 
+// b2t[g][c][m] = fp16(b2[g][m][c]) for m < E, 0 for E <= m < 64.
+__global__ void build_b2t_kernel(const float* b2, uint16_t* b2t, int G, int E, int Dt) {
+  const size_t n = size_t(G) * Dt * 64;
+  for (size_t i = blockIdx.x * size_t(blockDim.x) + threadIdx.x; i < n;
+       i += size_t(gridDim.x) * blockDim.x) {
+    const int m = static_cast<int>(i % 64);
+    const size_t gc = i / 64;
+    const int c = static_cast<int>(gc % Dt), g = static_cast<int>(gc / Dt);
+    const float v = m < E ? b2[(size_t(g) * E + m) * Dt + c] : 0.f;
+    b2t[i] = __half_as_ushort(__float2half_rn(v));
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_build_b2t(const float* b2, void* b2t, int G, int E, int Dt, cudaStream_t st) {
+  if (G == 0) return cudaSuccess;
+  build_b2t_kernel<<<1024, 256, 0, st>>>(b2, static_cast<uint16_t*>(b2t), G, E, Dt);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_bf16_to_f16_inplace(void* buf, size_t n, cudaStream_t st) {
   if (n == 0) return cudaSuccess;

@@ -41,7 +41,7 @@ static_assert(kSmemBytes <= 232448, "shared memory budget");
 struct FusedArgs {
   PathArgs p;
   int32_t n1, n2;     // 256-column tiles of E*H and of D_t
-  int32_t nk1, nk2;   // 64-element K blocks of D_s and of E*H
+  int32_t nk1, nk2;   // 64-element K blocks of D_s and of E*H (+1: the bias block)
   int32_t mb;         // token tiles per schedule block
   int32_t* counters;  // [0] item counter, [1 + f] GEMM1 completions of flat tile f
 };
@@ -86,7 +86,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                      const __grid_constant__ CUtensorMap tmW1,
                      const __grid_constant__ CUtensorMap tmA2,
                      const __grid_constant__ CUtensorMap tmW2,
-                     const __grid_constant__ CUtensorMap tmS, const FusedArgs fa) {
+                     const __grid_constant__ CUtensorMap tmS,
+                     const __grid_constant__ CUtensorMap tmG16,
+                     const __grid_constant__ CUtensorMap tmB2t, const FusedArgs fa) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -132,6 +134,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tmA2);
     tma_prefetch_desc(&tmW2);
     tma_prefetch_desc(&tmS);
+    tma_prefetch_desc(&tmG16);
+    tma_prefetch_desc(&tmB2t);
   }
   if (warp == 2) {
     tmem_alloc(tmem_slot, kTmemCols);
@@ -188,10 +192,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                         ((gi.src_layer * d.B + ti.b) * d.H_s + h) * d.S + ti.s0);
             tma_load_2d(sB + stage * kBBytes, &tmW1, &full[stage], kb * UK,
                         grp * d.EH + it.n * UN);
-          } else {
+          } else if (kb < nk - 1) {   // A2 x W2cat
             tma_load_3d(sA + stage * kABytes, &tmA2, &full[stage], kb * UK, m * UM, gl);
             tma_load_2d(sB + stage * kBBytes, &tmW2, &full[stage], kb * UK,
                         grp * d.Dt + it.n * UN);
+          } else {                    // last K block: gate16 x b2t (the combine biases)
+            tma_load_3d(sA + stage * kABytes, &tmG16, &full[stage], 0, m * UM, grp);
+            tma_load_2d(sB + stage * kBBytes, &tmB2t, &full[stage], 0, grp * d.Dt + it.n * UN);
           }
           issued_mask |= 1u << stage;
           issue_parity = (issue_parity & ~(1u << stage)) | (phase << stage);
@@ -328,7 +335,8 @@ size_t fused_counter_ints(const Dims& d, int gp) { return 1 + size_t(gp) * d.til
 
 cudaError_t launch_fused(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
                          const CUtensorMap& tmW1, const CUtensorMap& tmA2,
-                         const CUtensorMap& tmW2, const CUtensorMap& tmA2st, int32_t* counters,
+                         const CUtensorMap& tmW2, const CUtensorMap& tmA2st,
+                         const CUtensorMap& tmG16, const CUtensorMap& tmB2t, int32_t* counters,
                          int num_sms, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
@@ -344,13 +352,14 @@ cudaError_t launch_fused(const PathArgs& a, const CUtensorMap& tmK, const CUtens
   fa.n1 = a.d.EH / UN;
   fa.n2 = a.d.Dt / UN;
   fa.nk1 = a.d.Ds / UK;
-  fa.nk2 = a.d.EH / UK;
+  fa.nk2 = a.d.EH / UK + 1;   // + the combine-bias K block
   fa.mb = fused_block_tiles(a.d, num_sms);
   fa.counters = counters;
   const long long upper = static_cast<long long>(a.gp) * a.d.tiles_max * (fa.n1 + fa.n2);
   const int grid = static_cast<int>(upper < num_sms ? upper : num_sms);
   if (grid <= 0) return cudaSuccess;
-  mot_fused_kernel<<<grid, kThreads, kSmemBytes, st>>>(tmK, tmV, tmW1, tmA2, tmW2, tmA2st, fa);
+  mot_fused_kernel<<<grid, kThreads, kSmemBytes, st>>>(tmK, tmV, tmW1, tmA2, tmW2, tmA2st, tmG16,
+                                                       tmB2t, fa);
   return cudaGetLastError();
 }
 

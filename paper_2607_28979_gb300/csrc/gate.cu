@@ -1,5 +1,6 @@
 // Ragged token-tile list and the per-token gate (Def. 3.1).
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include "mot_internal.h"
 
@@ -80,6 +81,27 @@ struct Vec<float> {
   }
 };
 
+// The fp16 gate row of the tensor-core path: gtilde in columns [0, E), zeros up
+// to 64 (one K block of GEMM2's bias step). `g` may be null (all zeros).
+__device__ __forceinline__ void write_gate16(const PathArgs& a, int grp, size_t row, const float* g,
+                                             int E) {
+  if (!a.gate16) return;
+  uint4* out = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.gate16) +
+                                        (static_cast<size_t>(grp) * a.d.tpad + row) * 64);
+#pragma unroll
+  for (int v = 0; v < 8; ++v) {
+    uint32_t w[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int e0 = v * 8 + 2 * k;
+      const float lo = (g && e0 < E) ? g[e0] : 0.f, hi = (g && e0 + 1 < E) ? g[e0 + 1] : 0.f;
+      const __half2 h = __floats2half2_rn(lo, hi);
+      w[k] = *reinterpret_cast<const uint32_t*>(&h);
+    }
+    out[v] = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
 __device__ __forceinline__ float to_f(float x) { return x; }
 __device__ __forceinline__ float to_f(__nv_bfloat16 x) { return __bfloat162float(x); }
 
@@ -107,6 +129,7 @@ __global__ void __launch_bounds__(256) gate_kernel(PathArgs a) {
     float* __restrict__ gout = a.gate + (static_cast<size_t>(grp) * d.tpad + static_cast<size_t>(m) * kTileM + r) * E;
     if (r >= ti.rows) {
       if (lane < E) gout[lane] = 0.f;
+      if (lane == 0) write_gate16(a, grp, static_cast<size_t>(m) * kTileM + r, nullptr, E);
       continue;
     }
     const int s = ti.s0 + r;
@@ -189,6 +212,7 @@ __global__ void __launch_bounds__(256) gate_kernel(PathArgs a) {
 #pragma unroll
       for (int e = 0; e < kMaxE; ++e)
         if (e < E) gout[e] = g[e];
+      write_gate16(a, grp, static_cast<size_t>(m) * kTileM + r, g, E);
     }
   }
 }
@@ -219,7 +243,28 @@ __global__ void __launch_bounds__(256) gate_tile_kernel(PathArgs a) {
   for (int p = 0; p < P; ++p)
 #pragma unroll
     for (int e = 0; e < EMAX; ++e) acc[p][e] = 0.f;
+  // Software pipeline over heads: the raw 16-byte loads of head h + 1 are in
+  // flight while head h is multiplied, so each thread keeps 2 * P loads
+  // outstanding instead of P.
+  const size_t head_stride = static_cast<size_t>(d.S) * d.d_s;
+  const T* base0 = src + ((static_cast<size_t>(gi.src_layer) * d.B + ti.b) * d.H_s * d.S + ti.s0) * d.d_s + cp;
+  uint4 raw_cur[P], raw_nxt[P];
+#pragma unroll
+  for (int p = 0; p < P; ++p) {
+    const int r = r0 + p * RPP;
+    raw_cur[p] = r < ti.rows ? *reinterpret_cast<const uint4*>(base0 + static_cast<size_t>(r) * d.d_s)
+                             : make_uint4(0, 0, 0, 0);
+  }
   for (int h = 0; h < d.H_s; ++h) {
+    if (h + 1 < d.H_s) {
+      const T* bn = base0 + (h + 1) * head_stride;
+#pragma unroll
+      for (int p = 0; p < P; ++p) {
+        const int r = r0 + p * RPP;
+        raw_nxt[p] = r < ti.rows ? *reinterpret_cast<const uint4*>(bn + static_cast<size_t>(r) * d.d_s)
+                                 : make_uint4(0, 0, 0, 0);
+      }
+    }
     float w[EMAX][NV];
 #pragma unroll
     for (int e = 0; e < EMAX; ++e) {
@@ -230,22 +275,17 @@ __global__ void __launch_bounds__(256) gate_tile_kernel(PathArgs a) {
         for (int k = 0; k < NV; ++k) w[e][k] = 0.f;
       }
     }
-    const T* base = src + (((static_cast<size_t>(gi.src_layer) * d.B + ti.b) * d.H_s + h) * d.S + ti.s0) * d.d_s + cp;
 #pragma unroll
     for (int p = 0; p < P; ++p) {
-      const int r = r0 + p * RPP;
       float z[NV];
-      if (r < ti.rows) {
-        Vec<T>::load(base + static_cast<size_t>(r) * d.d_s, z);
-      } else {
-#pragma unroll
-        for (int k = 0; k < NV; ++k) z[k] = 0.f;
-      }
+      Vec<T>::load(reinterpret_cast<const T*>(&raw_cur[p]), z);
 #pragma unroll
       for (int e = 0; e < EMAX; ++e)
 #pragma unroll
         for (int k = 0; k < NV; ++k) acc[p][e] = fmaf(w[e][k], z[k], acc[p][e]);
     }
+#pragma unroll
+    for (int p = 0; p < P; ++p) raw_cur[p] = raw_nxt[p];
   }
 #pragma unroll
   for (int p = 0; p < P; ++p)
@@ -254,60 +294,87 @@ __global__ void __launch_bounds__(256) gate_tile_kernel(PathArgs a) {
 #pragma unroll
       for (int off = CPR / 2; off > 0; off >>= 1)
         acc[p][e] += __shfl_xor_sync(0xffffffffu, acc[p][e], off);
-  if (threadIdx.x % CPR != 0) return;
+  // Every thread of a row's CPR group now holds the row's logits: each one
+  // evaluates the softmax (cheap, E values) and writes its slice of the fp16
+  // gate row; the group's first thread also writes the fp32 gate.
+  const int j = threadIdx.x % CPR;
+  constexpr int kSlice = 64 / CPR;   // fp16 gate16 elements per thread (8 or 4)
   const float* __restrict__ bg = a.bg + static_cast<size_t>(grp) * E;
 #pragma unroll
   for (int p = 0; p < P; ++p) {
     const int r = r0 + p * RPP;
-    float* __restrict__ gout = a.gate + (static_cast<size_t>(grp) * d.tpad + static_cast<size_t>(m) * kTileM + r) * E;
-    if (r >= ti.rows) {
-      for (int e = 0; e < E; ++e) gout[e] = 0.f;
-      continue;
-    }
+    const size_t row = static_cast<size_t>(m) * kTileM + r;
+    float* __restrict__ gout = a.gate + (static_cast<size_t>(grp) * d.tpad + row) * E;
     float g[EMAX];
-    float mx = -INFINITY;
+    if (r >= ti.rows) {
 #pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e < E) {
-        g[e] = acc[p][e] + bg[e];
-        mx = fmaxf(mx, g[e]);
-      }
-    float sum = 0.f;
+      for (int e = 0; e < EMAX; ++e) g[e] = 0.f;
+    } else {
+      float mx = -INFINITY;
 #pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e < E) {
-        g[e] = expf(g[e] - mx);
-        sum += g[e];
-      }
-    const float inv = 1.f / sum;
+      for (int e = 0; e < EMAX; ++e)
+        if (e < E) {
+          g[e] = acc[p][e] + bg[e];
+          mx = fmaxf(mx, g[e]);
+        }
+      float sum = 0.f;
 #pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e < E) g[e] *= inv;
-    if (d.top_k > 0 && d.top_k < E) {
-      uint32_t keep = 0;
-      for (int k = 0; k < d.top_k; ++k) {
-        int best = -1;
-        float bv = 0.f;
+      for (int e = 0; e < EMAX; ++e)
+        if (e < E) {
+          g[e] = expf(g[e] - mx);
+          sum += g[e];
+        }
+      const float inv = 1.f / sum;
+#pragma unroll
+      for (int e = 0; e < EMAX; ++e) g[e] = e < E ? g[e] * inv : 0.f;
+      if (d.top_k > 0 && d.top_k < E) {
+        uint32_t keep = 0;
+        for (int k = 0; k < d.top_k; ++k) {
+          int best = -1;
+          float bv = 0.f;
+#pragma unroll
+          for (int e = 0; e < EMAX; ++e)
+            if (e < E && !((keep >> e) & 1u) && (best < 0 || g[e] > bv)) {
+              best = e;
+              bv = g[e];
+            }
+          keep |= 1u << best;
+        }
+        float ks = 0.f;
 #pragma unroll
         for (int e = 0; e < EMAX; ++e)
-          if (e < E && !((keep >> e) & 1u) && (best < 0 || g[e] > bv)) {
-            best = e;
-            bv = g[e];
-          }
-        keep |= 1u << best;
+          if (e < E && ((keep >> e) & 1u)) ks += g[e];
+        const float kinv = 1.f / ks;
+#pragma unroll
+        for (int e = 0; e < EMAX; ++e) g[e] = (e < E && ((keep >> e) & 1u)) ? g[e] * kinv : 0.f;
       }
-      float ks = 0.f;
-#pragma unroll
-      for (int e = 0; e < EMAX; ++e)
-        if (e < E && ((keep >> e) & 1u)) ks += g[e];
-      const float kinv = 1.f / ks;
-#pragma unroll
-      for (int e = 0; e < EMAX; ++e)
-        if (e < E) g[e] = ((keep >> e) & 1u) ? g[e] * kinv : 0.f;
     }
+    if (j == 0) {
 #pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e < E) gout[e] = g[e];
+      for (int e = 0; e < EMAX; ++e)
+        if (e < E) gout[e] = g[e];
+    }
+    if (a.gate16) {
+      uint16_t* out = static_cast<uint16_t*>(a.gate16) +
+                      (static_cast<size_t>(grp) * d.tpad + row) * 64 + j * kSlice;
+      uint32_t w[kSlice / 2];
+#pragma unroll
+      for (int k = 0; k < kSlice / 2; ++k) {
+        const int e0 = j * kSlice + 2 * k;   // this thread's columns e0, e0 + 1
+        float lo = 0.f, hi = 0.f;
+#pragma unroll
+        for (int e = 0; e < EMAX; ++e) {   // register selects, no indexed access
+          lo = e == e0 ? g[e] : lo;
+          hi = e == e0 + 1 ? g[e] : hi;
+        }
+        const __half2 hv = __floats2half2_rn(lo, hi);
+        w[k] = *reinterpret_cast<const uint32_t*>(&hv);
+      }
+      if constexpr (kSlice == 8)
+        *reinterpret_cast<uint4*>(out) = make_uint4(w[0], w[1], w[2], w[3]);
+      else
+        *reinterpret_cast<uint2*>(out) = make_uint2(w[0], w[1]);
+    }
   }
 }
 

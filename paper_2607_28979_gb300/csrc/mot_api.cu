@@ -92,6 +92,8 @@ struct mot_ctx {
   GroupInfo* groups = nullptr;
   // workspace
   float* gate = nullptr;
+  void* gate16 = nullptr;   // fp16 gate rows padded to 64 (tensor-core path)
+  void* b2t = nullptr;      // fp16 b2 transposed, padded to 64 (tensor-core path)
   void* a2 = nullptr;
   TileInfo* tiles = nullptr;
   int32_t* n_tiles = nullptr;
@@ -99,6 +101,7 @@ struct mot_ctx {
   int32_t* counters = nullptr;   // fused schedule: item counter + per-tile completions
   // tensor maps that do not depend on the caller's buffers
   CUtensorMap tm_w1{}, tm_w2{}, tm_a2{}, tm_a2_st{}, tm_w1h{}, tm_w2h{};
+  CUtensorMap tm_g16{}, tm_b2t{}, tm_b2th{};
   // host-buffer staging for mot_translate_host (allocated on first use)
   void* st_src[2] = {nullptr, nullptr};
   void* st_dst[2] = {nullptr, nullptr};
@@ -125,7 +128,8 @@ size_t group_elems(const Dims& d) {
 }
 
 void free_all(mot_ctx* h) {
-  void* ptrs[] = {h->wg, h->bg, h->w1, h->b1, h->b1h, h->w2, h->b2, h->groups, h->gate, h->a2, h->tiles,
+  void* ptrs[] = {h->wg, h->bg, h->w1, h->b1, h->b1h, h->w2, h->b2, h->groups, h->gate, h->gate16,
+                  h->b2t, h->a2, h->tiles,
                   h->n_tiles, h->status, h->counters, h->st_src[0], h->st_src[1], h->st_dst[0],
                   h->st_dst[1], h->st_len};
   for (void* p : ptrs)
@@ -217,6 +221,8 @@ PathArgs path_args(mot_ctx* h) {
   a.w2 = h->w2;
   a.b2 = h->b2;
   a.gate = h->gate;
+  a.gate16 = h->use_umma ? h->gate16 : nullptr;
+  a.b2t = h->b2t;
   a.a2 = h->a2;
   a.status = h->status;
   a.wait_limit = h->wait_limit;
@@ -265,19 +271,19 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
         return launch_umma2_gemm1(a, tmK, tmV, h->tm_w1h, h->tm_a2_st, h->num_sms, st);
       }));
       MOT_CUDA_TRY(timed(h, "umma2_gemm2_combine_store", st, [&] {
-        return launch_umma2_gemm2(a, h->tm_a2, h->tm_w2h, h->num_sms, st);
+        return launch_umma2_gemm2(a, h->tm_a2, h->tm_w2h, h->tm_g16, h->tm_b2th, h->num_sms, st);
       }));
     } else if (h->use_umma && h->schedule == 1) {
       MOT_CUDA_TRY(timed(h, "umma_fused_translate", st, [&] {
-        return launch_fused(a, tmK, tmV, h->tm_w1, h->tm_a2, h->tm_w2, h->tm_a2_st, h->counters,
-                            h->num_sms, st);
+        return launch_fused(a, tmK, tmV, h->tm_w1, h->tm_a2, h->tm_w2, h->tm_a2_st, h->tm_g16,
+                            h->tm_b2t, h->counters, h->num_sms, st);
       }));
     } else if (h->use_umma) {
       MOT_CUDA_TRY(timed(h, "umma_gemm1_gelu_gate", st, [&] {
         return launch_umma_gemm1(a, tmK, tmV, h->tm_w1, h->tm_a2_st, h->num_sms, st);
       }));
       MOT_CUDA_TRY(timed(h, "umma_gemm2_combine_store", st, [&] {
-        return launch_umma_gemm2(a, h->tm_a2, h->tm_w2, h->num_sms, st);
+        return launch_umma_gemm2(a, h->tm_a2, h->tm_w2, h->tm_g16, h->tm_b2t, h->num_sms, st);
       }));
     } else {
       MOT_CUDA_TRY(timed(h, "simt_gemm1_gelu_gate", st, [&] { return launch_simt_gemm1(a, st); }));
@@ -383,6 +389,8 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       {&h->w2, G * d.Dt * EH * es}, {(void**)&h->b2, G * E * d.Dt * 4},
       {(void**)&h->groups, std::max<size_t>(G, 1) * sizeof(GroupInfo)},
       {(void**)&h->gate, G * size_t(d.tpad) * E * 4},
+      {&h->gate16, h->use_umma ? G * size_t(d.tpad) * 64 * 2 : 16},
+      {&h->b2t, h->use_umma ? G * size_t(d.Dt) * 64 * 2 : 16},
       {&h->a2, size_t(h->gp_max) * per_group_a2},
       {(void**)&h->tiles, size_t(d.tiles_max) * sizeof(TileInfo)},
       {(void**)&h->n_tiles, 16}, {(void**)&h->status, 16},
@@ -428,6 +436,19 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       ok = ok && encode_bf16(&h->tm_a2, h->a2, 3, dims, st_b, box, /*f16=*/true);
       const uint32_t box_st[3] = {uint32_t(kUmmaK), 32, 1};   // one epilogue warp's store tile
       ok = ok && encode_bf16(&h->tm_a2_st, h->a2, 3, dims, st_b, box_st, /*f16=*/true);
+    }
+    {  // gate16: [G][tpad][64], box 64 x 128 x 1 (GEMM2's bias K block, A side)
+      const uint64_t dims[3] = {64, uint64_t(d.tpad), uint64_t(G)};
+      const uint64_t st_b[2] = {128, uint64_t(d.tpad) * 128};
+      const uint32_t box[3] = {64, uint32_t(kTileM), 1};
+      ok = ok && encode_bf16(&h->tm_g16, h->gate16, 3, dims, st_b, box, /*f16=*/true);
+    }
+    {  // b2t: [G * Dt][64], boxes 64 x 256 and 64 x 128 (B side)
+      const uint64_t dims[2] = {64, uint64_t(G * d.Dt)};
+      const uint64_t st_b[1] = {128};
+      const uint32_t box[2] = {64, uint32_t(kUmmaN)}, box_h[2] = {64, uint32_t(kUmmaN / 2)};
+      ok = ok && encode_bf16(&h->tm_b2t, h->b2t, 2, dims, st_b, box, /*f16=*/true);
+      ok = ok && encode_bf16(&h->tm_b2th, h->b2t, 2, dims, st_b, box_h, /*f16=*/true);
     }
     if (!ok) {
       free_all(h);
@@ -494,6 +515,7 @@ mot_status mot_load_weights(mot_handle h, const void* host_blob, size_t bytes) {
       // GEMM2 runs fp16 x fp16: W2 to fp16 in place, b1 copied to fp16
       MOT_CUDA_TRY(launch_bf16_to_f16_inplace(h->w2, size_t(d.G) * Dt * EH, 0));
       MOT_CUDA_TRY(launch_f32_to_f16(h->b1, h->b1h, b1.size(), 0));
+      MOT_CUDA_TRY(launch_build_b2t(h->b2, h->b2t, d.G, d.E, d.Dt, 0));
     }
   }
   MOT_CUDA_TRY(cudaDeviceSynchronize());

@@ -44,6 +44,8 @@ struct Dims {
 //   b2 [G][E][Dt] (fp32).
 // On the tensor-core path w2 holds fp16 (converted from the bf16 blob at
 // load) and b1h an fp16 copy of b1, so that GEMM2 runs fp16 x fp16 -> fp32.
+// The gate-weighted bias sum_m gtilde_m b2_m is one more K block of GEMM2:
+// A = gate16 (the token's gtilde in its first E columns), B = b2t.
 // Workspace: gate [G][tpad][E] fp32 (renormalised gate weights per token
 // row), a2 [gp][tpad][E*H] (GELU(hidden) * gate: fp16 on the tensor-core path,
 // fp32 on the SIMT path).
@@ -62,6 +64,8 @@ struct PathArgs {
   const void* w2;
   const float* b2;
   float* gate;
+  void* gate16;      // fp16 [G][tpad][64]: gtilde padded with zeros (tensor-core path, else null)
+  const void* b2t;   // fp16 [G][D_t][64]: b2 transposed, zero-padded (tensor-core path)
   void* a2;
   int32_t* status;
   int32_t g0, gp;         // groups [g0, g0 + gp) of this pass
@@ -71,6 +75,7 @@ struct PathArgs {
 
 // Kernel launchers (each returns the launch's cudaError_t).
 cudaError_t launch_bf16_to_f16_inplace(void* buf, size_t n, cudaStream_t st);
+cudaError_t launch_build_b2t(const float* b2, void* b2t, int G, int E, int Dt, cudaStream_t st);
 cudaError_t launch_f32_to_f16(const float* src, void* dst, size_t n, cudaStream_t st);
 cudaError_t launch_prep(const int32_t* seq_lens, int32_t batch, const Dims& d, TileInfo* tiles,
                         int32_t* n_tiles, int32_t* status, cudaStream_t st);
@@ -87,7 +92,8 @@ cudaError_t launch_umma_gemm1(const PathArgs& a, const CUtensorMap& tmK, const C
                               const CUtensorMap& tmW1, const CUtensorMap& tmA2st, int num_sms,
                               cudaStream_t st);
 cudaError_t launch_umma_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2,
-                              int num_sms, cudaStream_t st);
+                              const CUtensorMap& tmG16, const CUtensorMap& tmB2t, int num_sms,
+                              cudaStream_t st);
 
 // 2-SM variant (umma2.cu): CTA pairs, tcgen05.mma.cta_group::2 on 256 x 256
 // tiles. The W maps here have 64 x 128 boxes (each CTA loads half of B).
@@ -95,7 +101,8 @@ cudaError_t launch_umma2_gemm1(const PathArgs& a, const CUtensorMap& tmK, const 
                                const CUtensorMap& tmW1h, const CUtensorMap& tmA2st, int num_sms,
                                cudaStream_t st);
 cudaError_t launch_umma2_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2h,
-                               int num_sms, cudaStream_t st);
+                               const CUtensorMap& tmG16, const CUtensorMap& tmB2th, int num_sms,
+                               cudaStream_t st);
 
 // Fused persistent kernel: both GEMMs of a pass in one launch (fused.cu).
 // `counters` holds fused_counter_ints(d, gp) int32 (zeroed by the launcher).
@@ -103,7 +110,8 @@ int fused_block_tiles(const Dims& d, int num_sms);
 size_t fused_counter_ints(const Dims& d, int gp);
 cudaError_t launch_fused(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
                          const CUtensorMap& tmW1, const CUtensorMap& tmA2,
-                         const CUtensorMap& tmW2, const CUtensorMap& tmA2st, int32_t* counters,
+                         const CUtensorMap& tmW2, const CUtensorMap& tmA2st,
+                         const CUtensorMap& tmG16, const CUtensorMap& tmB2t, int32_t* counters,
                          int num_sms, cudaStream_t st);
 
 }  // namespace mot

@@ -5,7 +5,8 @@
 // concatenated: with W1cat = [W1_1; ...; W1_E] (E*H x D_s) and
 // W2cat = [W2_1, ..., W2_E] (D_t x E*H),
 //   GEMM1:  A2 = fp16( GELU(Z W1cat^T + b1cat) (.) gtilde_expand )      [T, E*H]
-//   GEMM2:  Y  = A2 W2cat^T + sum_m gtilde_m b2_m                        [T, D_t]
+//   GEMM2:  Y  = A2 W2cat^T + gate16 b2t^T                                [T, D_t]
+//           (the last K block adds sum_m gtilde_m b2_m: gate16 holds gtilde, b2t = b2^T)
 // so sum_m gtilde_m W2_m GELU(W1_m z + b1_m) is exactly GEMM2's sum over E*H.
 //
 // One persistent, warp-specialised kernel template runs both GEMMs:
@@ -94,9 +95,9 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
   }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA0);
-    if (MODE == 1) tma_prefetch_desc(&tmA1);
+    tma_prefetch_desc(&tmA1);
     tma_prefetch_desc(&tmB);
-    if (MODE == 1) tma_prefetch_desc(&tmS);
+    tma_prefetch_desc(&tmS);
   }
   if (warp == 2) {
     tmem_alloc(tmem_slot, kTmemCols);
@@ -143,11 +144,16 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
             const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
             tma_load_2d(sA + stage * kABytes, gi.x ? &tmA1 : &tmA0, &full[stage], d0,
                         ((gi.src_layer * d.B + ti.b) * d.H_s + h) * d.S + ti.s0);
-          } else {
+            tma_load_2d(sB + stage * kBBytes, &tmB, &full[stage], kb * UK,
+                        grp * ua.b_rows + n * UN);
+          } else if (kb < ua.nk - 1) {   // A2 x W2cat
             tma_load_3d(sA + stage * kABytes, &tmA0, &full[stage], kb * UK, m * UM, gl);
+            tma_load_2d(sB + stage * kBBytes, &tmB, &full[stage], kb * UK,
+                        grp * ua.b_rows + n * UN);
+          } else {                       // last K block: gate16 x b2t (the combine biases)
+            tma_load_3d(sA + stage * kABytes, &tmA1, &full[stage], 0, m * UM, grp);
+            tma_load_2d(sB + stage * kBBytes, &tmS, &full[stage], 0, grp * ua.b_rows + n * UN);
           }
-          tma_load_2d(sB + stage * kBBytes, &tmB, &full[stage], kb * UK,
-                      grp * ua.b_rows + n * UN);
           issued_mask |= 1u << stage;
           issue_parity = (issue_parity & ~(1u << stage)) | (phase << stage);
           if (++stage == kStages) { stage = 0; phase ^= 1u; }
@@ -288,9 +294,12 @@ cudaError_t launch_umma_gemm1(const PathArgs& a, const CUtensorMap& tmK, const C
   return launch_umma<1>(a, tmK, tmV, tmW1, tmA2st, a.d.Ds / UK, a.d.EH / UN, a.d.EH, num_sms, st);
 }
 
+// GEMM2's map slots: A0 = A2, A1 = gate16, B = W2cat, S = b2t (last K block).
 cudaError_t launch_umma_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2,
-                              int num_sms, cudaStream_t st) {
-  return launch_umma<2>(a, tmA2, tmA2, tmW2, tmA2, a.d.EH / UK, a.d.Dt / UN, a.d.Dt, num_sms, st);
+                              const CUtensorMap& tmG16, const CUtensorMap& tmB2t, int num_sms,
+                              cudaStream_t st) {
+  return launch_umma<2>(a, tmA2, tmG16, tmW2, tmB2t, a.d.EH / UK + 1, a.d.Dt / UN, a.d.Dt, num_sms,
+                        st);
 }
 
 }  // namespace mot

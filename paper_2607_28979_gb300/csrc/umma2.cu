@@ -94,9 +94,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
   }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA0);
-    if (MODE == 1) tma_prefetch_desc(&tmA1);
+    tma_prefetch_desc(&tmA1);
     tma_prefetch_desc(&tmB);
-    if (MODE == 1) tma_prefetch_desc(&tmS);
+    tma_prefetch_desc(&tmS);
   }
   if (warp == 2) {
     tmem_alloc_pair(tmem_slot, kTmemCols);
@@ -142,15 +142,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit)) { ok = false; break; }
           if (leader) mbar_arrive_expect_tx(&full[stage], 2 * kStageBytes2);
           const uint32_t bar = leader_addr(&full[stage]);
+          const int b_row = grp * ua.b_rows + n * UN + static_cast<int>(rank) * (UN / 2);
           if (MODE == 1) {
             const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
             tma_load_2d_pair(sA + stage * kABytes2, gi.x ? &tmA1 : &tmA0, bar, d0,
                              ((gi.src_layer * d.B + ti.b) * d.H_s + h) * d.S + ti.s0);
-          } else {
+            tma_load_2d_pair(sB + stage * kBBytes2, &tmB, bar, kb * UK, b_row);
+          } else if (kb < ua.nk - 1) {   // A2 x W2cat
             tma_load_3d_pair(sA + stage * kABytes2, &tmA0, bar, kb * UK, m_own * UM, gl);
+            tma_load_2d_pair(sB + stage * kBBytes2, &tmB, bar, kb * UK, b_row);
+          } else {                       // last K block: gate16 x b2t (the combine biases)
+            tma_load_3d_pair(sA + stage * kABytes2, &tmA1, bar, 0, m_own * UM, grp);
+            tma_load_2d_pair(sB + stage * kBBytes2, &tmS, bar, 0, b_row);
           }
-          tma_load_2d_pair(sB + stage * kBBytes2, &tmB, bar, kb * UK,
-                           grp * ua.b_rows + n * UN + static_cast<int>(rank) * (UN / 2));
           issued_mask |= 1u << stage;
           issue_parity = (issue_parity & ~(1u << stage)) | (phase << stage);
           if (++stage == kStages2) { stage = 0; phase ^= 1u; }
@@ -292,9 +296,12 @@ cudaError_t launch_umma2_gemm1(const PathArgs& a, const CUtensorMap& tmK, const 
   return launch_umma2<1>(a, tmK, tmV, tmW1h, tmA2st, a.d.Ds / UK, a.d.EH / UN, a.d.EH, num_sms, st);
 }
 
+// GEMM2's map slots: A0 = A2, A1 = gate16, B = W2cat half, S = b2t half (last K block).
 cudaError_t launch_umma2_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2h,
-                               int num_sms, cudaStream_t st) {
-  return launch_umma2<2>(a, tmA2, tmA2, tmW2h, tmA2, a.d.EH / UK, a.d.Dt / UN, a.d.Dt, num_sms, st);
+                               const CUtensorMap& tmG16, const CUtensorMap& tmB2th, int num_sms,
+                               cudaStream_t st) {
+  return launch_umma2<2>(a, tmA2, tmG16, tmW2h, tmB2th, a.d.EH / UK + 1, a.d.Dt / UN, a.d.Dt,
+                         num_sms, st);
 }
 
 }  // namespace mot

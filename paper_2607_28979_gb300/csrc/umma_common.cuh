@@ -4,8 +4,9 @@
 //                    (one expert m per 256-column tile since H % 256 == 0), computed in
 //                    packed fp16x2 arithmetic and written as 32x64 tiles through
 //                    128B-swizzled shared memory + TMA store.
-//   GEMM2 epilogue:  y[row, c] = acc[row, c] + sum_m gtilde_m(row) * b2_m[c], rounded
-//                    to bf16 and stored as 16-byte vectors into the target cache row
+//   GEMM2 epilogue:  y[row, c] = acc[row, c] (the gate-weighted biases
+//                    sum_m gtilde_m(row) * b2_m[c] are GEMM2's last K block), rounded to
+//                    bf16 and stored as 16-byte vectors into the target cache row
 //                    dst[l][b][c / d_t][s][c % d_t] when s < seq_len[b].
 #pragma once
 
@@ -114,20 +115,16 @@ __device__ __forceinline__ void epilogue_gemm1(const PathArgs& p, const CUtensor
 }
 
 // GEMM2 epilogue of one warp: row 32*q + lane of the tile, columns
-// [col_begin, col_begin + 32 * n_chunks) of output tile n0.
+// [col_begin, col_begin + 32 * n_chunks) of output tile n0. The gate-weighted
+// biases are already in the accumulator (GEMM2's last K block).
 __device__ __forceinline__ void epilogue_gemm2(const PathArgs& p, uint32_t tbase, int q, int lane,
                                                int grp, int m, int n0, int col_begin,
                                                int n_chunks) {
   const Dims& d = p.d;
   const int row = q * 32 + lane;
-  const size_t grow = static_cast<size_t>(m) * UM + row;
   const GroupInfo gi = p.groups[grp];
   const TileInfo ti = p.tiles[m];
   const bool valid = row < ti.rows;
-  const float* grow_g = p.gate + (static_cast<size_t>(grp) * d.tpad + grow) * d.E;
-  float g[kMaxE];
-#pragma unroll
-  for (int e = 0; e < kMaxE; ++e) g[e] = e < d.E ? grow_g[e] : 0.f;
   __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.dst[gi.x]);
   const size_t s = static_cast<size_t>(ti.s0) + row;
 #pragma unroll 1
@@ -137,24 +134,6 @@ __device__ __forceinline__ void epilogue_gemm2(const PathArgs& p, uint32_t tbase
     tmem_ld_32x32b_x32(tbase + cl, r);
     tmem_ld_wait(r);
     const int c = n0 + cl;
-    float y[32];
-#pragma unroll
-    for (int j = 0; j < 32; ++j) y[j] = __uint_as_float(r[j]);
-#pragma unroll
-    for (int e = 0; e < kMaxE; ++e) {
-      if (e < d.E) {
-        const float4* b4 =
-            reinterpret_cast<const float4*>(p.b2 + (static_cast<size_t>(grp) * d.E + e) * d.Dt + c);
-#pragma unroll
-        for (int v = 0; v < 8; ++v) {
-          const float4 bb = __ldg(b4 + v);
-          y[4 * v + 0] = fmaf(g[e], bb.x, y[4 * v + 0]);
-          y[4 * v + 1] = fmaf(g[e], bb.y, y[4 * v + 1]);
-          y[4 * v + 2] = fmaf(g[e], bb.z, y[4 * v + 2]);
-          y[4 * v + 3] = fmaf(g[e], bb.w, y[4 * v + 3]);
-        }
-      }
-    }
     if (valid) {
       const int h = c / d.d_t, i0 = c - h * d.d_t;
       uint4* o4 = reinterpret_cast<uint4*>(
@@ -162,10 +141,10 @@ __device__ __forceinline__ void epilogue_gemm2(const PathArgs& p, uint32_t tbase
                  i0));
 #pragma unroll
       for (int v = 0; v < 4; ++v)
-        o4[v] = make_uint4(pack_bf16x2(y[8 * v + 0], y[8 * v + 1]),
-                           pack_bf16x2(y[8 * v + 2], y[8 * v + 3]),
-                           pack_bf16x2(y[8 * v + 4], y[8 * v + 5]),
-                           pack_bf16x2(y[8 * v + 6], y[8 * v + 7]));
+        o4[v] = make_uint4(pack_bf16x2(__uint_as_float(r[8 * v + 0]), __uint_as_float(r[8 * v + 1])),
+                           pack_bf16x2(__uint_as_float(r[8 * v + 2]), __uint_as_float(r[8 * v + 3])),
+                           pack_bf16x2(__uint_as_float(r[8 * v + 4]), __uint_as_float(r[8 * v + 5])),
+                           pack_bf16x2(__uint_as_float(r[8 * v + 6]), __uint_as_float(r[8 * v + 7])));
     }
   }
 }

@@ -351,7 +351,8 @@ def run_mot(args, wl):
     e2e_s = time.perf_counter() - t0
     es = wl.esize
     tl = len(wl.translated_layers())
-    h2d = 2 * wl.n_layers_src * wl.tokens * wl.d_src * es + 4 * B
+    used_src = len({s for s in M.mot_get_layer_map(h) if s >= 0})   # source layers copied
+    h2d = 2 * used_src * wl.tokens * wl.d_src * es + 4 * B
     d2h = 2 * tl * wl.tokens * wl.d_tgt * es
 
     # ---- aggregate over ranks: max time

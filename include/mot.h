@@ -120,9 +120,12 @@ mot_status mot_translate(mot_handle h, const void* src_k, const void* src_v,
  * The same translation with HOST buffers (pinned memory recommended): copies
  * the real tokens of src_k/src_v and seq_lens (host int32[batch]) to
  * library-owned device staging, translates, and copies the translated
- * positions back into dst_k/dst_v, all enqueued on `stream`. The call returns
- * once the work is enqueued; synchronise `stream` before reading dst. The
- * staging buffers are allocated on the first call and freed by mot_destroy.
+ * positions back into dst_k/dst_v. The work is pipelined over chunks of target
+ * layers on `stream` and two library-owned copy streams, so the copies of one
+ * chunk overlap the translation of its neighbours; `stream` is made to wait
+ * for the last copy back. The call returns once the work is enqueued;
+ * synchronise `stream` before reading dst. The staging buffers, copy streams
+ * and events are created on the first call and freed by mot_destroy.
  * Errors: as mot_translate, plus MOT_ERR_SEQ_LEN for a host length outside
  * [0, max_seq] (nothing is enqueued then) and MOT_ERR_OOM.
  */

@@ -105,7 +105,7 @@ __device__ __forceinline__ void write_gate16(const PathArgs& a, int grp, size_t 
 __device__ __forceinline__ float to_f(float x) { return x; }
 __device__ __forceinline__ float to_f(__nv_bfloat16 x) { return __bfloat162float(x); }
 
-// Grid (tiles_max, G), 256 threads: each warp produces the gate of 16 token
+// Grid (tiles_max, gp), 256 threads: each warp produces the gate of 16 token
 // rows of one tile for one (layer, K/V) group. Lanes split the D_s channels
 // (VEC-wide vectors when the head dim allows it), reduce the E logits with
 // warp shuffles, and lane 0 applies the max-subtracted softmax and the Top-K
@@ -114,7 +114,7 @@ template <typename T, bool VEC>
 __global__ void __launch_bounds__(256) gate_kernel(PathArgs a) {
   const Dims& d = a.d;
   const int m = blockIdx.x;
-  const int grp = blockIdx.y;
+  const int grp = a.g0 + blockIdx.y;
   if (m >= *a.n_tiles) return;
   const TileInfo ti = a.tiles[m];
   const GroupInfo gi = a.groups[grp];
@@ -227,7 +227,7 @@ template <typename T, int CPR, int P, int EMAX>
 __global__ void __launch_bounds__(256) gate_tile_kernel(PathArgs a) {
   const Dims& d = a.d;
   const int m = blockIdx.x;
-  const int grp = blockIdx.y;
+  const int grp = a.g0 + blockIdx.y;
   if (m >= *a.n_tiles) return;
   const TileInfo ti = a.tiles[m];
   const GroupInfo gi = a.groups[grp];
@@ -378,9 +378,11 @@ __global__ void __launch_bounds__(256) gate_tile_kernel(PathArgs a) {
   }
 }
 
+// Gate of groups [a.g0, a.g0 + a.gp).
 cudaError_t launch_gate(const PathArgs& a, cudaStream_t st) {
   const Dims& d = a.d;
-  dim3 grid(d.tiles_max, d.G);
+  if (a.gp <= 0) return cudaSuccess;
+  dim3 grid(d.tiles_max, a.gp);
   // tile-wide kernel: 16-byte chunks per head row (CPR) of 8 or 16, E <= 8
   if (d.dtype == 0 && d.E <= 4 && d.d_s == 64) {
     gate_tile_kernel<__nv_bfloat16, 8, 4, 4><<<grid, 256, 0, st>>>(a);

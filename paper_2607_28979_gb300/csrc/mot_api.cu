@@ -20,6 +20,9 @@ namespace {
 // groups so that gp * tpad * E*H elements fit in it.
 constexpr size_t kA2Budget = size_t(8) << 30;
 
+// Chunks of target layers the host-buffer entry point pipelines over.
+constexpr int kHostChunks = 4;
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
@@ -106,6 +109,9 @@ struct mot_ctx {
   void* st_src[2] = {nullptr, nullptr};
   void* st_dst[2] = {nullptr, nullptr};
   int32_t* st_len = nullptr;
+  cudaStream_t copy_h2d = nullptr, copy_d2h = nullptr;   // created on first use
+  cudaEvent_t ev_h2d[kHostChunks] = {}, ev_comp[kHostChunks] = {};
+  cudaEvent_t ev_prev_compute = nullptr, ev_prev_d2h = nullptr;
   // profiling
   bool profile = false;
   std::vector<Ev> ev_used, ev_free;
@@ -135,6 +141,14 @@ void free_all(mot_ctx* h) {
   for (void* p : ptrs)
     if (p) cudaFree(p);
   for (auto& e : h->ev_used) { cudaEventDestroy(e.a); cudaEventDestroy(e.b); }
+  for (int c = 0; c < kHostChunks; ++c) {
+    if (h->ev_h2d[c]) cudaEventDestroy(h->ev_h2d[c]);
+    if (h->ev_comp[c]) cudaEventDestroy(h->ev_comp[c]);
+  }
+  if (h->ev_prev_compute) cudaEventDestroy(h->ev_prev_compute);
+  if (h->ev_prev_d2h) cudaEventDestroy(h->ev_prev_d2h);
+  if (h->copy_h2d) cudaStreamDestroy(h->copy_h2d);
+  if (h->copy_d2h) cudaStreamDestroy(h->copy_d2h);
   for (auto& e : h->ev_free) { cudaEventDestroy(e.a); cudaEventDestroy(e.b); }
 }
 
@@ -238,10 +252,13 @@ PathArgs path_args(mot_ctx* h) {
     }                                   \
   } while (0)
 
+// Translate groups [g_begin, g_end) (group 2r + x: r-th translated target
+// layer, x = K/V) on `st`; `do_prep` builds the tile list from seq_lens first.
 mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const int32_t* seq_lens,
-                         int32_t batch, void* dst_k, void* dst_v, cudaStream_t st) {
+                         int32_t batch, void* dst_k, void* dst_v, cudaStream_t st, int g_begin,
+                         int g_end, bool do_prep) {
   const Dims& d = h->d;
-  if (batch == 0 || d.G == 0) return MOT_OK;
+  if (batch == 0 || g_end <= g_begin) return MOT_OK;
   PathArgs a = path_args(h);
   a.src[0] = src_k;
   a.src[1] = src_v;
@@ -259,13 +276,16 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
       return MOT_ERR_CUDA;
   }
 
-  MOT_CUDA_TRY(timed(h, "prep_tiles", st, [&] {
-    return launch_prep(seq_lens, batch, d, h->tiles, h->n_tiles, h->status, st);
-  }));
+  if (do_prep)
+    MOT_CUDA_TRY(timed(h, "prep_tiles", st, [&] {
+      return launch_prep(seq_lens, batch, d, h->tiles, h->n_tiles, h->status, st);
+    }));
+  a.g0 = g_begin;
+  a.gp = g_end - g_begin;
   MOT_CUDA_TRY(timed(h, "gate", st, [&] { return launch_gate(a, st); }));
-  for (int g0 = 0; g0 < d.G; g0 += h->gp_max) {
+  for (int g0 = g_begin; g0 < g_end; g0 += h->gp_max) {
     a.g0 = g0;
-    a.gp = std::min(h->gp_max, d.G - g0);
+    a.gp = std::min(h->gp_max, g_end - g0);
     if (h->use_umma && h->schedule == 2) {
       MOT_CUDA_TRY(timed(h, "umma2_gemm1_gelu_gate", st, [&] {
         return launch_umma2_gemm1(a, tmK, tmV, h->tm_w1h, h->tm_a2_st, h->num_sms, st);
@@ -529,7 +549,7 @@ mot_status mot_translate(mot_handle h, const void* src_k, const void* src_v,
   mot_status s = check_translate_args(h, src_k, src_v, seq_lens, batch, dst_k, dst_v);
   if (s != MOT_OK) return s;
   return run_translate(h, src_k, src_v, seq_lens, batch, dst_k, dst_v,
-                       reinterpret_cast<cudaStream_t>(stream));
+                       reinterpret_cast<cudaStream_t>(stream), 0, h->d.G, true);
 }
 
 mot_status mot_translate_host(mot_handle h, const void* src_k, const void* src_v,
@@ -555,53 +575,80 @@ mot_status mot_translate_host(mot_handle h, const void* src_k, const void* src_v
         return MOT_ERR_OOM;
       }
   }
+  if (!h->copy_h2d) {
+    if (cudaStreamCreateWithFlags(&h->copy_h2d, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaStreamCreateWithFlags(&h->copy_d2h, cudaStreamNonBlocking) != cudaSuccess) {
+      cudaGetLastError();
+      return MOT_ERR_CUDA;
+    }
+    for (auto* e : {&h->ev_prev_compute, &h->ev_prev_d2h})
+      if (cudaEventCreateWithFlags(e, cudaEventDisableTiming) != cudaSuccess) return MOT_ERR_CUDA;
+    for (int c = 0; c < kHostChunks; ++c)
+      if (cudaEventCreateWithFlags(&h->ev_h2d[c], cudaEventDisableTiming) != cudaSuccess ||
+          cudaEventCreateWithFlags(&h->ev_comp[c], cudaEventDisableTiming) != cudaSuccess)
+        return MOT_ERR_CUDA;
+    MOT_CUDA_TRY(cudaEventRecord(h->ev_prev_compute, h->copy_h2d));
+    MOT_CUDA_TRY(cudaEventRecord(h->ev_prev_d2h, h->copy_d2h));
+  }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const size_t es = esize(d);
+  // Pipeline over chunks of translated target layers: the copies of chunk c's
+  // source layers (stream copy_h2d), the translation of chunk c (`stream`) and
+  // the copies of chunk c's target layers back (stream copy_d2h) overlap with
+  // the neighbouring chunks. Only real tokens (s < seq_len[b]) are copied.
+  std::vector<int> tl;   // translated target layers, ascending (group 2r + x)
+  for (int l = 0; l < d.L_t; ++l)
+    if (h->layer_map[l] >= 0) tl.push_back(l);
+  const int n_tl = static_cast<int>(tl.size());
+  const int nc = std::min(kHostChunks, n_tl);
+  // the previous call's translation read the source staging and its copies
+  // read the target staging: order this call after both
+  MOT_CUDA_TRY(cudaStreamWaitEvent(h->copy_h2d, h->ev_prev_compute, 0));
+  MOT_CUDA_TRY(cudaStreamWaitEvent(st, h->ev_prev_d2h, 0));
   MOT_CUDA_TRY(cudaMemcpyAsync(h->st_len, seq_lens, size_t(batch) * 4, cudaMemcpyHostToDevice, st));
-  // Real tokens only: for batch entry b, positions [0, len) of every (layer, head) row.
-  for (int b = 0; b < batch; ++b) {
-    const size_t len = seq_lens[b];
-    if (len == 0) continue;
-    for (int x = 0; x < 2; ++x) {
-      cudaMemcpy3DParms p{};
-      const size_t pitch = size_t(d.S) * d.d_s * es;
-      const size_t off = size_t(b) * d.H_s * pitch;
-      p.srcPtr = make_cudaPitchedPtr(const_cast<char*>(static_cast<const char*>(x ? src_v : src_k)) + off,
-                                     pitch, len * d.d_s * es, size_t(d.B) * d.H_s);
-      p.dstPtr = make_cudaPitchedPtr(static_cast<char*>(h->st_src[x]) + off, pitch,
-                                     len * d.d_s * es, size_t(d.B) * d.H_s);
-      p.extent = make_cudaExtent(len * d.d_s * es, d.H_s, d.L_s);
-      p.kind = cudaMemcpyHostToDevice;
-      MOT_CUDA_TRY(cudaMemcpy3DAsync(&p, st));
+  std::vector<char> copied(d.L_s, 0);
+  for (int c = 0; c < nc; ++c) {
+    const int r0 = c * n_tl / nc, r1 = (c + 1) * n_tl / nc;
+    for (int r = r0; r < r1; ++r) {
+      const int ls = h->layer_map[tl[r]];
+      if (copied[ls]) continue;
+      copied[ls] = 1;
+      for (int x = 0; x < 2; ++x)
+        for (int b = 0; b < batch; ++b) {
+          const size_t len = seq_lens[b];
+          if (len == 0) continue;
+          const size_t pitch = size_t(d.S) * d.d_s * es;
+          const size_t off = (size_t(ls) * d.B + b) * d.H_s * pitch;
+          MOT_CUDA_TRY(cudaMemcpy2DAsync(static_cast<char*>(h->st_src[x]) + off, pitch,
+                                         static_cast<const char*>(x ? src_v : src_k) + off, pitch,
+                                         len * d.d_s * es, d.H_s, cudaMemcpyHostToDevice,
+                                         h->copy_h2d));
+        }
     }
+    MOT_CUDA_TRY(cudaEventRecord(h->ev_h2d[c], h->copy_h2d));
+    MOT_CUDA_TRY(cudaStreamWaitEvent(st, h->ev_h2d[c], 0));
+    mot_status s = run_translate(h, h->st_src[0], h->st_src[1], h->st_len, batch, h->st_dst[0],
+                                 h->st_dst[1], st, 2 * r0, 2 * r1, c == 0);
+    if (s != MOT_OK) return s;
+    MOT_CUDA_TRY(cudaEventRecord(h->ev_comp[c], st));
+    MOT_CUDA_TRY(cudaStreamWaitEvent(h->copy_d2h, h->ev_comp[c], 0));
+    for (int r = r0; r < r1; ++r)
+      for (int x = 0; x < 2; ++x)
+        for (int b = 0; b < batch; ++b) {
+          const size_t len = seq_lens[b];
+          if (len == 0) continue;
+          const size_t pitch = size_t(d.S) * d.d_t * es;
+          const size_t off = (size_t(tl[r]) * d.B + b) * d.H_t * pitch;
+          MOT_CUDA_TRY(cudaMemcpy2DAsync(static_cast<char*>(x ? dst_v : dst_k) + off, pitch,
+                                         static_cast<const char*>(h->st_dst[x]) + off, pitch,
+                                         len * d.d_t * es, d.H_t, cudaMemcpyDeviceToHost,
+                                         h->copy_d2h));
+        }
   }
-  mot_status s = run_translate(h, h->st_src[0], h->st_src[1], h->st_len, batch, h->st_dst[0],
-                               h->st_dst[1], st);
-  if (s != MOT_OK) return s;
-  // Translated positions back: per batch entry and per run of translated layers.
-  for (int b = 0; b < batch; ++b) {
-    const size_t len = seq_lens[b];
-    if (len == 0) continue;
-    int l = 0;
-    while (l < d.L_t) {
-      if (h->layer_map[l] < 0) { ++l; continue; }
-      int l1 = l;
-      while (l1 < d.L_t && h->layer_map[l1] >= 0) ++l1;
-      for (int x = 0; x < 2; ++x) {
-        cudaMemcpy3DParms p{};
-        const size_t pitch = size_t(d.S) * d.d_t * es;
-        const size_t off = (size_t(l) * d.B + b) * d.H_t * pitch;
-        p.srcPtr = make_cudaPitchedPtr(static_cast<char*>(h->st_dst[x]) + off, pitch,
-                                       len * d.d_t * es, size_t(d.B) * d.H_t);
-        p.dstPtr = make_cudaPitchedPtr(static_cast<char*>(x ? dst_v : dst_k) + off, pitch,
-                                       len * d.d_t * es, size_t(d.B) * d.H_t);
-        p.extent = make_cudaExtent(len * d.d_t * es, d.H_t, size_t(l1 - l));
-        p.kind = cudaMemcpyDeviceToHost;
-        MOT_CUDA_TRY(cudaMemcpy3DAsync(&p, st));
-      }
-      l = l1;
-    }
-  }
+  MOT_CUDA_TRY(cudaEventRecord(h->ev_prev_compute, st));
+  MOT_CUDA_TRY(cudaEventRecord(h->ev_prev_d2h, h->copy_d2h));
+  // `stream` completes only after the last copy back
+  MOT_CUDA_TRY(cudaStreamWaitEvent(st, h->ev_prev_d2h, 0));
   return MOT_OK;
 }
 

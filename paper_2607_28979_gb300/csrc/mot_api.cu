@@ -21,7 +21,7 @@ namespace {
 constexpr size_t kA2Budget = size_t(8) << 30;
 
 // Chunks of target layers the host-buffer entry point pipelines over.
-constexpr int kHostChunks = 4;
+constexpr int kHostChunks = 6;
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
@@ -311,6 +311,45 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
     }
   }
   return MOT_OK;
+}
+
+// Copy the real-token rows (s < lens[b], every head, batch entries b < batch)
+// of layers [l0, l1) of a cache laid out [L][B][H][S][d] between host and
+// device staging. Equal lengths make each layer (and, with the whole batch, a
+// run of layers) one strided 2-D copy; ragged lengths copy per batch entry.
+cudaError_t copy_real_rows(void* dst, const void* src, int l0, int l1, int B, int H, int S, int dd,
+                           size_t es, const int32_t* lens, int batch, cudaMemcpyKind kind,
+                           cudaStream_t st) {
+  bool uniform = true;
+  for (int b = 1; b < batch; ++b) uniform = uniform && lens[b] == lens[0];
+  const size_t pitch = size_t(S) * dd * es;
+  char* dp = static_cast<char*>(dst);
+  const char* sp = static_cast<const char*>(src);
+  if (uniform) {
+    const size_t width = size_t(lens[0]) * dd * es;
+    if (width == 0) return cudaSuccess;
+    if (batch == B) {
+      const size_t off = size_t(l0) * B * H * pitch;
+      return cudaMemcpy2DAsync(dp + off, pitch, sp + off, pitch, width,
+                               size_t(l1 - l0) * B * H, kind, st);
+    }
+    for (int l = l0; l < l1; ++l) {
+      const size_t off = size_t(l) * B * H * pitch;
+      cudaError_t e = cudaMemcpy2DAsync(dp + off, pitch, sp + off, pitch, width, size_t(batch) * H,
+                                        kind, st);
+      if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+  }
+  for (int l = l0; l < l1; ++l)
+    for (int b = 0; b < batch; ++b) {
+      const size_t width = size_t(lens[b]) * dd * es;
+      if (width == 0) continue;
+      const size_t off = (size_t(l) * B + b) * H * pitch;
+      cudaError_t e = cudaMemcpy2DAsync(dp + off, pitch, sp + off, pitch, width, H, kind, st);
+      if (e != cudaSuccess) return e;
+    }
+  return cudaSuccess;
 }
 
 mot_status check_translate_args(mot_ctx* h, const void* src_k, const void* src_v,
@@ -609,21 +648,20 @@ mot_status mot_translate_host(mot_handle h, const void* src_k, const void* src_v
   std::vector<char> copied(d.L_s, 0);
   for (int c = 0; c < nc; ++c) {
     const int r0 = c * n_tl / nc, r1 = (c + 1) * n_tl / nc;
+    // source layers first needed by this chunk, copied in runs of consecutive layers
+    std::vector<char> need(d.L_s, 0);
     for (int r = r0; r < r1; ++r) {
       const int ls = h->layer_map[tl[r]];
-      if (copied[ls]) continue;
-      copied[ls] = 1;
+      if (!copied[ls]) need[ls] = copied[ls] = 1;
+    }
+    for (int l0 = 0; l0 < d.L_s;) {
+      if (!need[l0]) { ++l0; continue; }
+      int l1 = l0;
+      while (l1 < d.L_s && need[l1]) ++l1;
       for (int x = 0; x < 2; ++x)
-        for (int b = 0; b < batch; ++b) {
-          const size_t len = seq_lens[b];
-          if (len == 0) continue;
-          const size_t pitch = size_t(d.S) * d.d_s * es;
-          const size_t off = (size_t(ls) * d.B + b) * d.H_s * pitch;
-          MOT_CUDA_TRY(cudaMemcpy2DAsync(static_cast<char*>(h->st_src[x]) + off, pitch,
-                                         static_cast<const char*>(x ? src_v : src_k) + off, pitch,
-                                         len * d.d_s * es, d.H_s, cudaMemcpyHostToDevice,
-                                         h->copy_h2d));
-        }
+        MOT_CUDA_TRY(copy_real_rows(h->st_src[x], x ? src_v : src_k, l0, l1, d.B, d.H_s, d.S, d.d_s,
+                                    es, seq_lens, batch, cudaMemcpyHostToDevice, h->copy_h2d));
+      l0 = l1;
     }
     MOT_CUDA_TRY(cudaEventRecord(h->ev_h2d[c], h->copy_h2d));
     MOT_CUDA_TRY(cudaStreamWaitEvent(st, h->ev_h2d[c], 0));
@@ -632,18 +670,16 @@ mot_status mot_translate_host(mot_handle h, const void* src_k, const void* src_v
     if (s != MOT_OK) return s;
     MOT_CUDA_TRY(cudaEventRecord(h->ev_comp[c], st));
     MOT_CUDA_TRY(cudaStreamWaitEvent(h->copy_d2h, h->ev_comp[c], 0));
-    for (int r = r0; r < r1; ++r)
+    // this chunk's target layers back, in runs of consecutive layers
+    for (int r = r0; r < r1;) {
+      int r2 = r + 1;
+      while (r2 < r1 && tl[r2] == tl[r2 - 1] + 1) ++r2;
       for (int x = 0; x < 2; ++x)
-        for (int b = 0; b < batch; ++b) {
-          const size_t len = seq_lens[b];
-          if (len == 0) continue;
-          const size_t pitch = size_t(d.S) * d.d_t * es;
-          const size_t off = (size_t(tl[r]) * d.B + b) * d.H_t * pitch;
-          MOT_CUDA_TRY(cudaMemcpy2DAsync(static_cast<char*>(x ? dst_v : dst_k) + off, pitch,
-                                         static_cast<const char*>(h->st_dst[x]) + off, pitch,
-                                         len * d.d_t * es, d.H_t, cudaMemcpyDeviceToHost,
-                                         h->copy_d2h));
-        }
+        MOT_CUDA_TRY(copy_real_rows(x ? dst_v : dst_k, h->st_dst[x], tl[r], tl[r2 - 1] + 1, d.B,
+                                    d.H_t, d.S, d.d_t, es, seq_lens, batch,
+                                    cudaMemcpyDeviceToHost, h->copy_d2h));
+      r = r2;
+    }
   }
   MOT_CUDA_TRY(cudaEventRecord(h->ev_prev_compute, st));
   MOT_CUDA_TRY(cudaEventRecord(h->ev_prev_d2h, h->copy_d2h));

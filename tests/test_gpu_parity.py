@@ -208,8 +208,19 @@ def test_seq_len_out_of_range_is_clamped_and_reported():
     assert torch.equal(G.int_view(bad.dv), G.int_view(good.dv))
 
 
-def test_host_buffer_entry_point_matches_device_entry_point():
-    wl = SMALL["umma_ragged"]
+HOST_CASES = {
+    "ragged": (SMALL["umma_ragged"], None),
+    "uniform_partial_batch": (SMALL["umma_ragged"].replace(seq_lens=(200, 200)), None),
+    "uniform_full_batch": (SMALL["umma_e3"].replace(seq_lens=(200, 200)), None),
+}
+
+
+@pytest.mark.parametrize("case", sorted(HOST_CASES))
+def test_host_buffer_entry_point_matches_device_entry_point(case):
+    """The pipelined host-buffer path copies only real tokens (one strided copy per
+    run of layers when lengths are equal, per batch entry when ragged) and must
+    give the device entry point's bytes exactly, leaving every other position."""
+    wl, _ = HOST_CASES[case]
     sk, sv, blob = inputs(wl, seed=8)
     run = G.Run(wl, sk, sv, blob)
     assert run.translate() == M.MOT_OK

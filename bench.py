@@ -77,10 +77,18 @@ def load_peaks():
     return FALLBACK_PEAKS, "fallback"
 
 
-def kernel_source_sha() -> str:
+# Source files each profiled kernel is built from (its traffic figure is stale
+# once any of them changes).
+KERNEL_SOURCES = {
+    "umma2_gemm1_gelu_gate": ["umma2.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
+    "umma2_gemm2_combine_store": ["umma2.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
+}
+
+
+def kernel_source_sha(kernel: str) -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2607_28979_gb300", "csrc")
-    for n in sorted(os.listdir(csrc)):
+    for n in KERNEL_SOURCES.get(kernel, sorted(os.listdir(csrc))):
         if n.endswith((".cu", ".cuh", ".h")):
             with open(os.path.join(csrc, n), "rb") as f:
                 h.update(f.read())
@@ -93,7 +101,7 @@ def recorded_traffic(kernel: str, workload: str):
     p = os.path.join(ROOT, "profiles", "dram_traffic.txt")
     if not os.path.exists(p):
         return None
-    sha = kernel_source_sha()
+    sha = kernel_source_sha(kernel)
     for line in open(p):
         f = dict(kv.split("=", 1) for kv in line.split() if "=" in kv)
         if f.get("kernel") == kernel and f.get("workload") == workload and f.get("source_sha") == sha:

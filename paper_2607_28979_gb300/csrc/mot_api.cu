@@ -43,10 +43,11 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 16-bit tensor map (bf16, or fp16 when `f16`) with 128-byte swizzle;
-// dims[0] is the contiguous one.
+// 16-bit tensor map (bf16, or fp16 when `f16`) with 128-byte swizzle (64-byte
+// when `swizzle64`); dims[0] is the contiguous one.
 bool encode_bf16(CUtensorMap* map, const void* base, int rank, const uint64_t* dims,
-                 const uint64_t* strides_bytes, const uint32_t* box, bool f16 = false) {
+                 const uint64_t* strides_bytes, const uint32_t* box, bool f16 = false,
+                 bool swizzle64 = false) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t gd[5], gs[4];
@@ -58,7 +59,8 @@ bool encode_bf16(CUtensorMap* map, const void* base, int rank, const uint64_t* d
   }
   for (int i = 0; i < rank - 1; ++i) gs[i] = strides_bytes[i];
   CUresult r = fn(map, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), gd, gs, bx,
-                  es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  swizzle64 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
@@ -493,8 +495,9 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       const uint64_t st_b[2] = {uint64_t(EH) * 2, uint64_t(d.tpad) * EH * 2};
       const uint32_t box[3] = {uint32_t(kUmmaK), uint32_t(kTileM), 1};
       ok = ok && encode_bf16(&h->tm_a2, h->a2, 3, dims, st_b, box, /*f16=*/true);
-      const uint32_t box_st[3] = {uint32_t(kUmmaK), 32, 1};   // one epilogue warp's store tile
-      ok = ok && encode_bf16(&h->tm_a2_st, h->a2, 3, dims, st_b, box_st, /*f16=*/true);
+      const uint32_t box_st[3] = {32, 32, 1};   // one epilogue warp's 32 x 32 store tile
+      ok = ok && encode_bf16(&h->tm_a2_st, h->a2, 3, dims, st_b, box_st, /*f16=*/true,
+                             /*swizzle64=*/true);
     }
     {  // gate16: [G][tpad][64], box 64 x 128 x 1 (GEMM2's bias K block, A side)
       const uint64_t dims[3] = {64, uint64_t(d.tpad), uint64_t(G)};

@@ -212,7 +212,8 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
                              (static_cast<uint32_t>(q * 32) << 16);
       if (MODE == 1)   // 8 warps: this warp owns columns 128 * (e / 4) .. +127
         epilogue_gemm1(p, &tmS, tbase, sOut + e * kStoreTileBytes, q, lane, gl, grp, m, n * UN,
-                       (e >> 2) * 128, 2);
+                       (e >> 2) * 128, 2,
+                       gemm1_prefetch(p, q, lane, grp, m, n * UN, (e >> 2) * 128));
       else             // 4 warps: all 256 columns
         epilogue_gemm2(p, tbase, q, lane, grp, m, n * UN, 0, UN / 32);
       tc_fence_before();

@@ -197,7 +197,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
     const int q = e & 3;
     int acc = 0;
     uint32_t acc_phase = 0;
+    // GEMM1: the gate value of this thread's row for the next tile, fetched ahead
+    auto tile_coords = [&](int tt, int& gl, int& grp, int& m_own, int& n) {
+      gl = tt / per_grp;
+      const int rem = tt - gl * per_grp;
+      const int mp = rem / ua.n_tiles_n;
+      n = rem - mp * ua.n_tiles_n;
+      grp = p.g0 + gl;
+      m_own = 2 * mp + static_cast<int>(rank);
+    };
+    float gate_next = 0.f;
+    if (MODE == 1 && pair < total) {
+      int gl, grp, m_own, n;
+      tile_coords(pair, gl, grp, m_own, n);
+      if (m_own < n_m) gate_next = gemm1_prefetch(p, q, lane, grp, m_own, n * UN, (e >> 2) * 128);
+    }
     for (int t = pair; t < total; t += n_pairs) {
+      const float gate_cur = gate_next;
+      if (MODE == 1 && t + n_pairs < total) {
+        int gl, grp, m_own, n;
+        tile_coords(t + n_pairs, gl, grp, m_own, n);
+        if (m_own < n_m) gate_next = gemm1_prefetch(p, q, lane, grp, m_own, n * UN, (e >> 2) * 128);
+      }
       int ok = 1;
       if (lane == 0) ok = mbar_wait(&tfull[acc], acc_phase, abort_flag, p.wait_limit) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
@@ -212,7 +233,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
       if (m_own < n_m) {
         if (MODE == 1)   // 8 warps: this warp owns columns 128 * (e / 4) .. +127
           epilogue_gemm1(p, &tmS, tbase, sOut + e * kStoreTileBytes, q, lane, gl, grp, m_own,
-                         n * UN, (e >> 2) * 128, 2);
+                         n * UN, (e >> 2) * 128, 2, gate_cur);
         else             // 4 warps: all 256 columns
           epilogue_gemm2(p, tbase, q, lane, grp, m_own, n * UN, 0, UN / 32);
       }

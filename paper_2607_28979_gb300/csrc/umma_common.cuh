@@ -2,8 +2,8 @@
 //
 //   GEMM1 epilogue:  A2[row, n0 + c] = fp16( GELU(acc[row, c] + b1[n0 + c]) * gtilde_m(row) )
 //                    (one expert m per 256-column tile since H % 256 == 0), computed in
-//                    packed fp16x2 arithmetic and written as 32x64 tiles through
-//                    128B-swizzled shared memory + TMA store.
+//                    packed fp16x2 arithmetic and written as 32x32 tiles through
+//                    64B-swizzled, double-buffered shared memory + TMA store.
 //   GEMM2 epilogue:  y[row, c] = acc[row, c] (the gate-weighted biases
 //                    sum_m gtilde_m(row) * b2_m[c] are GEMM2's last K block), rounded to
 //                    bf16 and stored as 16-byte vectors into the target cache row
@@ -26,7 +26,7 @@ constexpr int kABytes = UM * UK * 2;   // 16 KB
 constexpr int kBBytes = UN * UK * 2;   // 32 KB
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kTmemCols = 2 * UN;      // two fp32 accumulators of 256 columns
-constexpr int kStoreTileBytes = 32 * 128;   // one warp's 32 rows x 64 bf16 columns
+constexpr int kStoreTileBytes = 2 * 32 * 64;   // one warp's two 32 x 32 fp16 store tiles
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
@@ -57,59 +57,89 @@ __device__ __forceinline__ __half2 gelu_times_h2(__half2 u, __half2 half_g) {
 
 // GEMM1 epilogue of one warp: rows 32*q + lane of the tile, columns
 // [col_begin, col_begin + 64 * n_chunks). `tbase` is the accumulator's TMEM
-// address including the warp's lane quarter; `tile` this warp's 4 KB store
-// tile (1024-byte aligned). The caller commits nothing: each chunk is its own
-// bulk group.
+// address including the warp's lane quarter; `tile` this warp's 4 KB of
+// shared memory (two 2 KB store tiles). The columns are processed in 32-wide
+// sub-chunks: the TMEM load of sub-chunk i+1 is in flight while sub-chunk i is
+// evaluated, and each 32x32 fp16 result goes out by TMA store from one of the
+// two tiles while the other is refilled.
+__device__ __forceinline__ void gemm1_sub(const uint32_t (&r)[32], const uint4* b4, __half2 half_g,
+                                          uint32_t (&pk)[16]) {
+#pragma unroll
+  for (int v = 0; v < 4; ++v) {
+    const uint4 bb = __ldg(b4 + v);
+    const uint32_t bw[4] = {bb.x, bb.y, bb.z, bb.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int j = v * 8 + 2 * k;
+      __half2 u = __float22half2_rn(make_float2(__uint_as_float(r[j]), __uint_as_float(r[j + 1])));
+      u = __hadd2(u, *reinterpret_cast<const __half2*>(&bw[k]));
+      const __half2 o = gelu_times_h2(u, half_g);
+      pk[4 * v + k] = *reinterpret_cast<const uint32_t*>(&o);
+    }
+  }
+}
+
+// Gate value of this thread's row for GEMM1 tile (grp, m, n0), and an L1
+// prefetch of the warp's bias columns: issued one tile ahead by the caller so
+// that neither round trip sits at the start of the tile's epilogue.
+__device__ __forceinline__ float gemm1_prefetch(const PathArgs& p, int q, int lane, int grp, int m,
+                                                int n0, int col_begin) {
+  const Dims& d = p.d;
+  const size_t grow = static_cast<size_t>(m) * UM + q * 32 + lane;
+  const float g = p.gate[(static_cast<size_t>(grp) * d.tpad + grow) * d.E + n0 / d.H];
+  if (lane < 2) {
+    const __half* b = static_cast<const __half*>(p.b1h) + static_cast<size_t>(grp) * d.EH + n0 +
+                      col_begin + lane * 64;
+    asm volatile("prefetch.global.L1 [%0];" ::"l"(b));
+  }
+  return g;
+}
+
 __device__ __forceinline__ void epilogue_gemm1(const PathArgs& p, const CUtensorMap* tmS,
                                                uint32_t tbase, uint8_t* tile, int q, int lane,
                                                int gl, int grp, int m, int n0, int col_begin,
-                                               int n_chunks) {
+                                               int n_chunks, float gate) {
   const Dims& d = p.d;
-  const size_t grow = static_cast<size_t>(m) * UM + q * 32 + lane;
-  const int expert = n0 / d.H;
-  const __half2 half_g =
-      __float2half2_rn(0.5f * p.gate[(static_cast<size_t>(grp) * d.tpad + grow) * d.E + expert]);
+  const __half2 half_g = __float2half2_rn(0.5f * gate);
   const __half* __restrict__ bias =
       static_cast<const __half*>(p.b1h) + static_cast<size_t>(grp) * d.EH + n0;
   const uint32_t tile_addr = smem_u32(tile);
+  const int n_sub = 2 * n_chunks;
+  uint32_t ra[32], rb[32];
+  tmem_ld_32x32b_x32(tbase + col_begin, ra);
 #pragma unroll 1
-  for (int c = 0; c < n_chunks; ++c) {
-    const int col0 = col_begin + c * 64;
-    uint32_t ra[32], rb[32];
-    tmem_ld_32x32b_x32(tbase + col0, ra);
-    tmem_ld_32x32b_x32(tbase + col0 + 32, rb);
+  for (int sc = 0; sc < n_sub; sc += 2) {
+    // ---- sub-chunk sc (in ra); load sc + 1 into rb meanwhile
     tmem_ld_wait(ra);
-    tmem_ld_wait(rb);
-    const uint4* b4 = reinterpret_cast<const uint4*>(bias + col0);   // 8 fp16 biases each
-    uint32_t pk[32];   // pk[k] = columns 2k, 2k+1 as fp16x2
+    tmem_ld_32x32b_x32(tbase + col_begin + (sc + 1) * 32, rb);
 #pragma unroll
-    for (int v = 0; v < 8; ++v) {
-      const uint4 bb = __ldg(b4 + v);
-      const uint32_t bw[4] = {bb.x, bb.y, bb.z, bb.w};
-      const uint32_t* r = v < 4 ? ra : rb;
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const int j = (v & 3) * 8 + 2 * k;
-        __half2 u = __float22half2_rn(make_float2(__uint_as_float(r[j]), __uint_as_float(r[j + 1])));
-        u = __hadd2(u, *reinterpret_cast<const __half2*>(&bw[k]));
-        const __half2 o = gelu_times_h2(u, half_g);
-        pk[4 * v + k] = *reinterpret_cast<const uint32_t*>(&o);
+    for (int half = 0; half < 2; ++half) {
+      const int s = sc + half;
+      const int col0 = col_begin + s * 32;
+      uint32_t pk[16];   // columns col0 + 2k, +1 of this row as fp16x2
+      if (half == 0) {
+        gemm1_sub(ra, reinterpret_cast<const uint4*>(bias + col0), half_g, pk);
+      } else {
+        tmem_ld_wait(rb);
+        if (s + 1 < n_sub) tmem_ld_32x32b_x32(tbase + col_begin + (s + 1) * 32, ra);
+        gemm1_sub(rb, reinterpret_cast<const uint4*>(bias + col0), half_g, pk);
       }
-    }
-    // the previous TMA store of this warp must have finished reading the tile
-    if (lane == 0) bulk_wait_group_read<0>();
-    __syncwarp();
-    // row `lane` of the 32x64 tile; 16-byte chunk cc sits at chunk position
-    // cc ^ (row % 8), the 128-byte swizzle of the store map (bank-conflict free)
+      // the store that last used this half's tile must have finished reading it
+      if (lane == 0) bulk_wait_group_read<1>();
+      __syncwarp();
+      // row `lane` of the 32x32 tile (64 bytes); 16-byte chunk cc sits at chunk
+      // position cc ^ ((row / 2) % 4), the 64-byte swizzle of the store map
+      const uint32_t t_addr = tile_addr + half * 2048;
 #pragma unroll
-    for (int cc = 0; cc < 8; ++cc)
-      st_shared_v4(tile_addr + lane * 128 + ((cc ^ (lane & 7)) << 4), pk[4 * cc], pk[4 * cc + 1],
-                   pk[4 * cc + 2], pk[4 * cc + 3]);
-    fence_proxy_async_smem();
-    __syncwarp();
-    if (lane == 0) {
-      tma_store_3d(tmS, tile, n0 + col0, m * UM + q * 32, gl);
-      bulk_commit_group();
+      for (int cc = 0; cc < 4; ++cc)
+        st_shared_v4(t_addr + lane * 64 + ((cc ^ ((lane >> 1) & 3)) << 4), pk[4 * cc],
+                     pk[4 * cc + 1], pk[4 * cc + 2], pk[4 * cc + 3]);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        tma_store_3d(tmS, tile + half * 2048, n0 + col0, m * UM + q * 32, gl);
+        bulk_commit_group();
+      }
     }
   }
 }

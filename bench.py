@@ -82,6 +82,7 @@ def load_peaks():
 KERNEL_SOURCES = {
     "umma2_gemm1_gelu_gate": ["umma2.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
     "umma2_gemm2_combine_store": ["umma2.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
+    "umma2_onchip_translate": ["onchip.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
 }
 
 
@@ -288,7 +289,10 @@ def run_mot(args, wl):
     h = M.mot_create(M.config_from(wl))
     M.mot_load_weights(h, blob)
     path = M.mot_get_path(h)
-    M.mot_set_schedule(h, {"split": 0, "fused": 1, "pair": 2}[args.schedule])
+    names = {0: "split", 1: "fused", 2: "pair", 3: "onchip"}
+    if args.schedule != "auto":
+        M.mot_set_schedule(h, {v: k for k, v in names.items()}[args.schedule])
+    schedule = names[M.mot_get_schedule(h)]
     bf = wl.dtype == "bf16"
     tdt = torch.bfloat16 if bf else torch.float32
 
@@ -376,6 +380,7 @@ def run_mot(args, wl):
         name, (n_launch, tot_ms) = max(kstats.items(), key=lambda kv: kv[1][1])
         gp_groups = 2 * tl
         per_launch_flops = {"umma_fused_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
+                            "umma2_onchip_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
                             "umma2_gemm1_gelu_gate": alg["flops_gemm1"],
                             "umma2_gemm2_combine_store": alg["flops_gemm2"],
                             "umma_gemm1_gelu_gate": alg["flops_gemm1"],
@@ -410,7 +415,7 @@ def run_mot(args, wl):
             "data": "synthetic (seeded SplitMix64/Box-Muller caches, N(0,1/fan_in) weights)",
             "config": {"workload": workload_desc(wl), "tokens_per_step": tokens,
                        "parallelism": "replicas" if world > 1 else "single GPU",
-                       "path": ("tcgen05 " + args.schedule) if path == 1 else "simt",
+                       "path": ("tcgen05 " + schedule) if path == 1 else "simt",
                        "l2": "inputs larger than L2 (%.2f GB read+written per step)" % (alg["bytes"] / 1e9)},
             "roofline": roof,
             "step_roofline": {"flops": alg["flops"], "bytes": alg["bytes"],
@@ -442,9 +447,11 @@ def main():
     ap.add_argument("--impl", choices=["mot", "reference"], default="mot")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--schedule", choices=["pair", "fused", "split"], default="pair",
-                    help="tcgen05 launch schedule: GEMMs on CTA pairs (2-SM MMA), one fused "
-                         "persistent launch, or GEMMs on single SMs")
+    ap.add_argument("--schedule", choices=["auto", "onchip", "pair", "fused", "split"],
+                    default="auto",
+                    help="tcgen05 launch schedule: the library's default for the shape, the "
+                         "on-chip GEMM1-GELU-GEMM2 kernel (D_s <= 128, D_t = 256), GEMMs on CTA "
+                         "pairs (2-SM MMA), one fused persistent launch, or GEMMs on single SMs")
     ap.add_argument("--n-layers", type=int, default=0,
                     help="keep only the first N layers of both models (smaller profiling case)")
     args = ap.parse_args()

@@ -186,10 +186,16 @@ mot_status mot_get_layer_map(mot_handle h, int32_t* out, int32_t n);
 mot_status mot_get_path(mot_handle h, int32_t* path);
 
 /*
- * Launch schedule of the tcgen05 path (no effect on the SIMT path); all give
- * the same results.
- *   2 (default): per pass of groups, GEMM1 then GEMM2 on pairs of CTAs (two
- *      SMs per 256 x 256 tile, tcgen05.mma.cta_group::2);
+ * Launch schedule of the tcgen05 path (schedules 0-2 have no effect on the
+ * SIMT path); all give the same results.
+ *   3 (default where supported): one persistent launch on pairs of CTAs that
+ *      keeps each token tile's hidden activations GELU(W1 z + b1) * gtilde in
+ *      shared memory and TMEM between the two GEMMs, so they never reach HBM.
+ *      Supported when D_s <= 128, D_t = 256 and H % 256 == 0 (bf16);
+ *      otherwise setting it returns MOT_ERR_UNSUPPORTED.
+ *   2 (default otherwise): per pass of groups, GEMM1 then GEMM2 on pairs of
+ *      CTAs (two SMs per 256 x 256 tile, tcgen05.mma.cta_group::2), with the
+ *      hidden activations in an HBM workspace;
  *   1: one fused persistent launch per pass running both GEMMs as
  *      dependency-ordered work items on single SMs;
  *   0: GEMM1 then GEMM2 on single SMs (128 x 256 tiles).

@@ -79,7 +79,7 @@ struct mot_ctx {
   int device = 0;
   int num_sms = 0;
   bool use_umma = false;
-  int schedule = 2;           // tcgen05 path: 0 split, 1 fused, 2 split on CTA pairs
+  int schedule = 2;           // tcgen05 path: 0 split, 1 fused, 2 split on CTA pairs, 3 on-chip
   long long wait_limit = 4000000000LL;   // bound of every pipeline wait (SM cycles)
   int stall_test = 0;                    // test hook, see mot_debug_set
   bool weights_loaded = false;
@@ -105,7 +105,7 @@ struct mot_ctx {
   int32_t* status = nullptr;
   int32_t* counters = nullptr;   // fused schedule: item counter + per-tile completions
   // tensor maps that do not depend on the caller's buffers
-  CUtensorMap tm_w1{}, tm_w2{}, tm_a2{}, tm_a2_st{}, tm_w1h{}, tm_w2h{};
+  CUtensorMap tm_w1{}, tm_w2{}, tm_a2{}, tm_a2_st{}, tm_w1h{}, tm_w2h{}, tm_w1q{};
   CUtensorMap tm_g16{}, tm_b2t{}, tm_b2th{};
   // host-buffer staging for mot_translate_host (allocated on first use)
   void* st_src[2] = {nullptr, nullptr};
@@ -285,6 +285,13 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
   a.g0 = g_begin;
   a.gp = g_end - g_begin;
   MOT_CUDA_TRY(timed(h, "gate", st, [&] { return launch_gate(a, st); }));
+  if (h->use_umma && h->schedule == 3) {   // one launch; no A2 workspace, so no passes
+    MOT_CUDA_TRY(timed(h, "umma2_onchip_translate", st, [&] {
+      return launch_onchip(a, tmK, tmV, h->tm_w1q, h->tm_w2h, h->tm_g16, h->tm_b2th, h->num_sms,
+                           st);
+    }));
+    return MOT_OK;
+  }
   for (int g0 = g_begin; g0 < g_end; g0 += h->gp_max) {
     a.g0 = g0;
     a.gp = std::min(h->gp_max, g_end - g0);
@@ -435,6 +442,7 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
     return MOT_ERR_UNSUPPORTED;
   }
   h->use_umma = umma_supported(d) && encode_fn() != nullptr;
+  if (h->use_umma && onchip_supported(d)) h->schedule = 3;
 
   const size_t es = esize(d), G = d.G, E = d.E, EH = d.EH;
   const size_t a2_row = EH * (h->use_umma ? 2 : 4);
@@ -481,6 +489,8 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       ok = ok && encode_bf16(&h->tm_w1, h->w1, 2, dims, st_b, box);
       const uint32_t box_h[2] = {uint32_t(kUmmaK), uint32_t(kUmmaN / 2)};   // one CTA of a pair
       ok = ok && encode_bf16(&h->tm_w1h, h->w1, 2, dims, st_b, box_h);
+      const uint32_t box_q[2] = {uint32_t(kUmmaK), 64};   // one CTA's half of a 128-row chunk
+      ok = ok && encode_bf16(&h->tm_w1q, h->w1, 2, dims, st_b, box_q);
     }
     {  // W2cat: [G*Dt rows][EH], box 64 x 256
       const uint64_t dims[2] = {uint64_t(EH), uint64_t(G * d.Dt)};
@@ -726,7 +736,8 @@ mot_status mot_get_path(mot_handle h, int32_t* path) {
 }
 
 mot_status mot_set_schedule(mot_handle h, int32_t schedule) {
-  if (!h || schedule < 0 || schedule > 2) return MOT_ERR_INVALID_ARG;
+  if (!h || schedule < 0 || schedule > 3) return MOT_ERR_INVALID_ARG;
+  if (schedule == 3 && !(h->use_umma && onchip_supported(h->d))) return MOT_ERR_UNSUPPORTED;
   h->schedule = schedule;
   return MOT_OK;
 }

@@ -104,6 +104,16 @@ cudaError_t launch_umma2_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const
                                const CUtensorMap& tmG16, const CUtensorMap& tmB2th, int num_sms,
                                cudaStream_t st);
 
+// On-chip translation on CTA pairs for D_s <= 128, D_t = 256 (onchip.cu):
+// GEMM1, GELU * gate and GEMM2 in one persistent launch over all groups, the
+// hidden activations kept in shared memory. W1 map: box 64 x 64 (half of a
+// 128-row chunk); W2 and b2t maps: box 64 x 128; gate16: box 64 x 128 x 1.
+bool onchip_supported(const Dims& d);
+cudaError_t launch_onchip(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                          const CUtensorMap& tmW1q, const CUtensorMap& tmW2h,
+                          const CUtensorMap& tmG16, const CUtensorMap& tmB2th, int num_sms,
+                          cudaStream_t st);
+
 // Fused persistent kernel: both GEMMs of a pass in one launch (fused.cu).
 // `counters` holds fused_counter_ints(d, gp) int32 (zeroed by the launcher).
 int fused_block_tiles(const Dims& d, int num_sms);

@@ -1,0 +1,441 @@
+// On-chip translation for narrow translators (D_s <= 128, D_t = 256) on CTA
+// pairs: GEMM1 -> GELU * gate -> GEMM2 with the hidden activations kept in
+// shared memory and TMEM, so the A2 intermediate (E*H fp16 values per token
+// row, 7.5 GB for the Qwen2.5-0.5B -> 1.5B shapes) never goes through HBM.
+//
+// A cluster of two CTAs owns a 256-row pair tile (token tiles 2*mp, 2*mp + 1
+// of one (target layer, K/V) group) and walks the concatenated hidden
+// dimension E*H in chunks of 128 columns. For chunk j:
+//   U_j  = Z * W1cat[128 j .. 128 j + 127]^T       tcgen05 M=256 N=128 K=D_s -> TMEM acc1[c % 2]
+//   A2_j = fp16( GELU(U_j + b1) * gtilde_m )        epilogue warps, into shared memory in the
+//                                                  K-major 128B-swizzled operand layout
+//   Y   += A2_j * W2cat[:, 128 j .. 128 j + 127]^T  tcgen05 M=256 N=256 K=128 -> TMEM acc2
+// (c counts chunks across tiles; m = 128 j / H is the chunk's expert, as
+// H % 128 == 0). After the last chunk Y += gate16 * b2t adds the
+// gate-weighted biases sum_m gtilde_m b2_m (Def. 3.1), and the epilogue
+// stores Y as bf16 into the target cache.
+//
+// TMEM per CTA (512 columns): acc2 in [0, 256), acc1[0] in [256, 384),
+// acc1[1] in [384, 512). Shared memory per CTA: Z 2 x 32 KB (the next tile's
+// rows load during the current tile), W1 ring 2 x 16 KB, W2 ring 2 x 32 KB
+// (the last stage of a tile holds b2t and gate16), A2 2 x 32 KB.
+//
+// Roles per CTA:
+//   warp 0 lane 0 (both)    TMA loads of its Z rows and its halves of W1 / W2;
+//                           transaction bytes complete on the leader's barriers;
+//   warp 1 lane 0 (leader)  MMA issue, in the order G1(0) G1(1) | G2(j) G1(j+2) ... | bias;
+//   warp 2 (both)           TMEM allocation of the pair;
+//   warps 4..11 (both)      epilogue: warp 4 + 4 p + q owns rows 32 q .. 32 q + 31 and
+//                           the chunks with c % 2 == p; at the end of a tile it stores
+//                           output columns 128 p .. 128 p + 127.
+// Every wait is bounded; a timeout unwinds and raises kStatusTimeout.
+#include "umma_common.cuh"
+
+namespace mot {
+namespace {
+
+constexpr int kChunk = 128;                              // hidden columns per chunk
+constexpr int kBlk16 = UM * UK * 2;                      // 16 KB: 128 rows x 64 K, 16-bit
+constexpr int kZBytes = 2 * kBlk16;                      // Z: 128 rows x D_s (<= 128)
+constexpr int kW1Blk = (kChunk / 2) * UK * 2;            // 8 KB: 64 rows x 64 K
+constexpr int kW1Bytes = 2 * kW1Blk;
+constexpr int kW2Bytes = 2 * kBlk16;                     // 128 rows x 128 K
+constexpr int kA2Bytes = 2 * kBlk16;                     // 128 rows x 128 K
+constexpr int kOffW1 = 2 * kZBytes;
+constexpr int kOffW2 = kOffW1 + 2 * kW1Bytes;
+constexpr int kOffA2 = kOffW2 + 2 * kW2Bytes;
+constexpr int kOffBar = kOffA2 + 2 * kA2Bytes;
+constexpr int kEpiWarps = 8;
+constexpr int kThreads = 32 * (4 + kEpiWarps);
+constexpr int kSmemBytes = kOffBar + 256 + 1024;
+static_assert(kSmemBytes <= 232448, "shared memory budget");
+constexpr uint32_t kAcc1Col = UN;   // acc1[b] at column 256 + 128 b
+constexpr uint32_t kTmemAlloc = 512;
+
+struct Bars {
+  uint64_t zfull[2], zempty[2], w1full[2], w1empty[2], w2full[2], w2empty[2];
+  uint64_t a1full[2];   // GEMM1 of a chunk done (commit, both CTAs)
+  uint64_t a2full[2];   // chunk's A2 written and acc1 read (leader; 2 x 4 warp arrivals)
+  uint64_t acc2full;    // a tile's GEMM2 + bias done (commit, both CTAs)
+  uint64_t acc2empty;   // acc2 read out (leader; 2 x 8 warp arrivals)
+  uint64_t drain;
+  uint32_t tmem_slot;
+  int abort_flag;
+};
+static_assert(sizeof(Bars) <= 256, "barrier block");
+
+struct OnchipArgs {
+  PathArgs p;
+  int32_t nk1;   // 64-wide K blocks of GEMM1 (D_s / 64)
+  int32_t nc;    // chunks per tile (E*H / 128)
+};
+
+__device__ __forceinline__ void spin_cycles(long long cycles) {
+  const long long t0 = clock64();
+  while (clock64() - t0 < cycles) {
+  }
+}
+
+// Row r's 32 columns of sub-chunk s (columns 32 s .. 32 s + 31 of the chunk)
+// into the A2 buffer at `a2`: K block s / 2, 16-byte chunks 4 (s % 2) .. + 3,
+// each at chunk position (index ^ (r % 8)) of its 128-byte row (128B swizzle).
+__device__ __forceinline__ void store_a2_sub(uint32_t a2, int r, int s, const uint32_t (&pk)[16]) {
+  const uint32_t row = a2 + static_cast<uint32_t>((s >> 1) * kBlk16 + r * 128);
+  const int c0 = (s & 1) * 4;
+#pragma unroll
+  for (int v = 0; v < 4; ++v)
+    st_shared_v4(row + static_cast<uint32_t>(((c0 + v) ^ (r & 7)) << 4), pk[4 * v],
+                 pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+}
+
+// GEMM1 epilogue of one warp for one chunk: TMEM acc1 (32 rows x 128 columns
+// at `tb`) -> GELU(u + b1) * g -> fp16 into the A2 buffer at `a2`.
+__device__ __forceinline__ void epi_chunk(uint32_t tb, const __half* bias, float gate, uint32_t a2,
+                                          int r) {
+  const __half2 half_g = __float2half2_rn(0.5f * gate);
+  uint32_t ra[32], rb[32], pk[16];
+  tmem_ld_32x32b_x32(tb, ra);
+#pragma unroll 1
+  for (int s = 0; s < 4; s += 2) {
+    tmem_ld_wait(ra);
+    tmem_ld_32x32b_x32(tb + (s + 1) * 32, rb);
+    gemm1_sub(ra, reinterpret_cast<const uint4*>(bias + s * 32), half_g, pk);
+    store_a2_sub(a2, r, s, pk);
+    tmem_ld_wait(rb);
+    if (s + 2 < 4) tmem_ld_32x32b_x32(tb + (s + 2) * 32, ra);
+    gemm1_sub(rb, reinterpret_cast<const uint4*>(bias + (s + 1) * 32), half_g, pk);
+    store_a2_sub(a2, r, s + 1, pk);
+  }
+}
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+    onchip_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                  const __grid_constant__ CUtensorMap tmW1q,
+                  const __grid_constant__ CUtensorMap tmW2h,
+                  const __grid_constant__ CUtensorMap tmG16,
+                  const __grid_constant__ CUtensorMap tmB2th, const OnchipArgs oa) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sZ = smem;
+  uint8_t* sW1 = smem + kOffW1;
+  uint8_t* sW2 = smem + kOffW2;
+  uint8_t* sA2 = smem + kOffA2;
+  Bars* bars = reinterpret_cast<Bars*>(smem + kOffBar);
+  volatile int* abort_flag = &bars->abort_flag;
+
+  const PathArgs& p = oa.p;
+  const Dims& d = p.d;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int nc = oa.nc, nk1 = oa.nk1;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars->zfull[i], 1);
+      mbar_init(&bars->zempty[i], 1);
+      mbar_init(&bars->w1full[i], 1);
+      mbar_init(&bars->w1empty[i], 1);
+      mbar_init(&bars->w2full[i], 1);
+      mbar_init(&bars->w2empty[i], 1);
+      mbar_init(&bars->a1full[i], 1);
+      mbar_init(&bars->a2full[i], 2 * (kEpiWarps / 2));
+    }
+    mbar_init(&bars->acc2full, 1);
+    mbar_init(&bars->acc2empty, 2 * kEpiWarps);
+    mbar_init(&bars->drain, 1);
+    bars->abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmV);
+    tma_prefetch_desc(&tmW1q);
+    tma_prefetch_desc(&tmW2h);
+    tma_prefetch_desc(&tmG16);
+    tma_prefetch_desc(&tmB2th);
+  }
+  if (warp == 2) {
+    tmem_alloc_pair(&bars->tmem_slot, kTmemAlloc);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync();
+  tc_fence_after();
+  const uint32_t tmem_base = bars->tmem_slot;
+
+  const int n_m = min(*p.n_tiles, d.tiles_max);
+  const int n_mp = (n_m + 1) / 2;
+  const int total = p.gp * n_mp;
+  const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+
+  // unwinding state: full barriers with loads in flight (bit i: zfull 0-1,
+  // w1full 2-3, w2full 4-5) and the parity of each one's last phase
+  uint32_t pend_mask = 0, pend_par = 0;
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer (both CTAs)
+      uint32_t i1 = 0, i2 = 0;
+      auto note = [&](int bit, uint32_t ph) {
+        pend_mask |= 1u << bit;
+        pend_par = (pend_par & ~(1u << bit)) | (ph << bit);
+      };
+      auto load_z = [&](int t, uint32_t k) -> bool {
+        const int zb = k & 1;
+        const uint32_t ph = (k >> 1) & 1u;
+        if (!mbar_wait(&bars->zempty[zb], ph ^ 1u, abort_flag, p.wait_limit)) return false;
+        const int gl = t / n_mp, mp = t - gl * n_mp;
+        const GroupInfo gi = p.groups[p.g0 + gl];
+        const int m_own = 2 * mp + static_cast<int>(rank);
+        TileInfo ti;
+        if (m_own < n_m) {
+          ti = p.tiles[m_own];
+        } else {   // no such tile: any in-bounds rows; they are never stored
+          ti.b = 0;
+          ti.s0 = 0;
+        }
+        if (leader) mbar_arrive_expect_tx(&bars->zfull[zb], 2 * nk1 * kBlk16);
+        const uint32_t bar = leader_addr(&bars->zfull[zb]);
+        for (int kb = 0; kb < nk1; ++kb) {
+          const int kk = kb * UK, h = kk / d.d_s, d0 = kk - h * d.d_s;
+          tma_load_2d_pair(sZ + zb * kZBytes + kb * kBlk16, gi.x ? &tmV : &tmK, bar, d0,
+                           ((gi.src_layer * d.B + ti.b) * d.H_s + h) * d.S + ti.s0);
+        }
+        note(zb, ph);
+        return true;
+      };
+      auto load_w1 = [&](int grp, int j) -> bool {
+        const int s = i1 & 1;
+        const uint32_t ph = (i1 >> 1) & 1u;
+        if (!mbar_wait(&bars->w1empty[s], ph ^ 1u, abort_flag, p.wait_limit)) return false;
+        if (leader) mbar_arrive_expect_tx(&bars->w1full[s], 2 * nk1 * kW1Blk);
+        const uint32_t bar = leader_addr(&bars->w1full[s]);
+        const int row = grp * d.EH + j * kChunk + static_cast<int>(rank) * (kChunk / 2);
+        for (int kb = 0; kb < nk1; ++kb)
+          tma_load_2d_pair(sW1 + s * kW1Bytes + kb * kW1Blk, &tmW1q, bar, kb * UK, row);
+        note(2 + s, ph);
+        ++i1;
+        return true;
+      };
+      auto load_w2 = [&](int grp, int m_own, int j) -> bool {   // j == nc: the bias stage
+        const int s = i2 & 1;
+        const uint32_t ph = (i2 >> 1) & 1u;
+        if (!mbar_wait(&bars->w2empty[s], ph ^ 1u, abort_flag, p.wait_limit)) return false;
+        if (leader) mbar_arrive_expect_tx(&bars->w2full[s], 2 * kW2Bytes);
+        const uint32_t bar = leader_addr(&bars->w2full[s]);
+        const int row = grp * d.Dt + static_cast<int>(rank) * (UN / 2);
+        uint8_t* dst = sW2 + s * kW2Bytes;
+        if (j < nc) {
+          tma_load_2d_pair(dst, &tmW2h, bar, j * kChunk, row);
+          tma_load_2d_pair(dst + kBlk16, &tmW2h, bar, j * kChunk + UK, row);
+        } else {   // B = b2t half, A = gate16 rows of this CTA's token tile
+          tma_load_2d_pair(dst, &tmB2th, bar, 0, row);
+          tma_load_3d_pair(dst + kBlk16, &tmG16, bar, 0, m_own * UM, grp);
+        }
+        note(4 + s, ph);
+        ++i2;
+        return true;
+      };
+      uint32_t k = 0;
+      for (int t = pair; t < total; t += n_pairs, ++k) {
+        const int gl = t / n_mp, mp = t - gl * n_mp;
+        const int grp = p.g0 + gl;
+        const int m_own = 2 * mp + static_cast<int>(rank);
+        bool ok = true;
+        if (k == 0) ok = load_z(t, 0);
+        ok = ok && load_w1(grp, 0);
+        if (nc > 1) ok = ok && load_w1(grp, 1);
+        if (t + n_pairs < total) ok = ok && load_z(t + n_pairs, k + 1);
+        for (int j = 0; ok && j < nc; ++j) {
+          ok = load_w2(grp, m_own, j);
+          if (j + 2 < nc) ok = ok && load_w1(grp, j + 2);
+        }
+        ok = ok && load_w2(grp, m_own, nc);
+        if (!ok) break;
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      // ------------------------------------------------ MMA issuer (leader)
+      constexpr uint32_t idesc1 = idesc_bf16_f32(2 * UM, kChunk);
+      constexpr uint32_t idesc2 = idesc_f16_f32(2 * UM, UN);
+      uint32_t i1 = 0, i2 = 0, c0 = 0, k = 0;
+      bool ok = true;
+      for (int t = pair; ok && t < total; t += n_pairs, ++k) {
+        const int zb = k & 1;
+        if (!mbar_wait(&bars->zfull[zb], (k >> 1) & 1u, abort_flag, p.wait_limit)) break;
+        tc_fence_after();
+        auto g1 = [&](int j) -> bool {
+          const int s = i1 & 1;
+          if (!mbar_wait(&bars->w1full[s], (i1 >> 1) & 1u, abort_flag, p.wait_limit)) return false;
+          tc_fence_after();
+          const uint32_t b = (c0 + j) & 1u;
+          for (int kb = 0; kb < nk1; ++kb) {
+            const uint64_t zdesc = sdesc_k_sw128(smem_u32(sZ + zb * kZBytes + kb * kBlk16));
+            const uint64_t wdesc = sdesc_k_sw128(smem_u32(sW1 + s * kW1Bytes + kb * kW1Blk));
+#pragma unroll
+            for (int kk = 0; kk < UK / 16; ++kk)   // +32 bytes of K = +2 in the address field
+              umma_pair(tmem_base + kAcc1Col + b * kChunk, zdesc + 2 * kk, wdesc + 2 * kk, idesc1,
+                        (kb | kk) != 0);
+          }
+          mma_issued = true;
+          umma_commit_pair(&bars->w1empty[s]);
+          umma_commit_pair(&bars->a1full[b]);
+          if (j == nc - 1) umma_commit_pair(&bars->zempty[zb]);
+          ++i1;
+          return true;
+        };
+        ok = g1(0) && (nc < 2 || g1(1));
+        for (int j = 0; ok && j < nc; ++j) {
+          const uint32_t c = c0 + j, b = c & 1u;
+          ok = mbar_wait(&bars->a2full[b], (c >> 1) & 1u, abort_flag, p.wait_limit);
+          if (ok && j == 0)
+            ok = mbar_wait(&bars->acc2empty, (k & 1u) ^ 1u, abort_flag, p.wait_limit);
+          const int s = i2 & 1;
+          ok = ok && mbar_wait(&bars->w2full[s], (i2 >> 1) & 1u, abort_flag, p.wait_limit);
+          if (!ok) break;
+          tc_fence_after();
+#pragma unroll
+          for (int kb = 0; kb < 2; ++kb) {
+            const uint64_t adesc = sdesc_k_sw128(smem_u32(sA2 + b * kA2Bytes + kb * kBlk16));
+            const uint64_t bdesc = sdesc_k_sw128(smem_u32(sW2 + s * kW2Bytes + kb * kBlk16));
+#pragma unroll
+            for (int kk = 0; kk < UK / 16; ++kk)
+              umma_pair(tmem_base, adesc + 2 * kk, bdesc + 2 * kk, idesc2, (j | kb | kk) != 0);
+          }
+          umma_commit_pair(&bars->w2empty[s]);
+          ++i2;
+          if (j + 2 < nc) ok = g1(j + 2);
+        }
+        if (!ok) break;
+        // gate-weighted biases: A = gate16 (second block of the stage), B = b2t
+        const int s = i2 & 1;
+        if (!mbar_wait(&bars->w2full[s], (i2 >> 1) & 1u, abort_flag, p.wait_limit)) break;
+        tc_fence_after();
+        const uint64_t gdesc = sdesc_k_sw128(smem_u32(sW2 + s * kW2Bytes + kBlk16));
+        const uint64_t bdesc = sdesc_k_sw128(smem_u32(sW2 + s * kW2Bytes));
+#pragma unroll
+        for (int kk = 0; kk < UK / 16; ++kk)
+          umma_pair(tmem_base, gdesc + 2 * kk, bdesc + 2 * kk, idesc2, 1u);
+        umma_commit_pair(&bars->w2empty[s]);
+        umma_commit_pair(&bars->acc2full);
+        ++i2;
+        c0 += nc;
+      }
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------ epilogue (both CTAs)
+    const int e = warp - 4, q = e & 3, par = e >> 2;
+    const int r = q * 32 + lane;
+    const uint32_t tq = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+    const uint32_t a2_addr = smem_u32(sA2 + par * kA2Bytes);
+    const __half* b1h = static_cast<const __half*>(p.b1h);
+    uint32_t c0 = 0, k = 0;
+    bool ok = true;
+    for (int t = pair; ok && t < total; t += n_pairs, ++k) {
+      const int gl = t / n_mp, mp = t - gl * n_mp;
+      const int grp = p.g0 + gl;
+      const int m_own = 2 * mp + static_cast<int>(rank);
+      const bool valid = m_own < n_m;
+      const float* grow =
+          p.gate + (static_cast<size_t>(grp) * d.tpad + static_cast<size_t>(m_own) * UM + r) * d.E;
+      for (int j = static_cast<int>((c0 & 1u) ^ static_cast<uint32_t>(par)); j < nc; j += 2) {
+        const uint32_t c = c0 + j;
+        const float gate = valid ? __ldg(grow + (j * kChunk) / d.H) : 0.f;
+        int w = 1;
+        if (lane == 0) w = mbar_wait(&bars->a1full[par], (c >> 1) & 1u, abort_flag, p.wait_limit);
+        if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+        tc_fence_after();
+        epi_chunk(tq + kAcc1Col + par * kChunk, b1h + static_cast<size_t>(grp) * d.EH + j * kChunk,
+                  gate, a2_addr, r);
+        fence_proxy_async_smem();   // the MMA (async proxy) reads these stores
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(&bars->a2full[par], 0);
+      }
+      if (!ok) break;
+      int w = 1;
+      if (lane == 0) w = mbar_wait(&bars->acc2full, k & 1u, abort_flag, p.wait_limit);
+      if (!__shfl_sync(0xffffffffu, w, 0)) break;
+      tc_fence_after();
+      if (valid) epilogue_gemm2(p, tq, q, lane, grp, m_own, 0, par * (UN / 2), UN / 64);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(&bars->acc2empty, 0);
+      c0 += nc;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort_flag) {
+    // Unwinding after a timed-out wait (bounded): copies this CTA started
+    // complete on the leader's barriers, so give them time to land; the
+    // leader also waits for its issued MMAs.
+    if (warp == 0 && lane == 0 && pend_mask) {
+      if (leader) {
+        uint64_t* fulls[6] = {&bars->zfull[0],  &bars->zfull[1],  &bars->w1full[0],
+                              &bars->w1full[1], &bars->w2full[0], &bars->w2full[1]};
+#pragma unroll
+        for (int i = 0; i < 6; ++i)
+          if ((pend_mask >> i) & 1u) {
+            const uint32_t a = smem_u32(fulls[i]);
+            const long long t0 = clock64();
+            while (!mbar_try_wait(a, (pend_par >> i) & 1u) && clock64() - t0 < p.wait_limit) {
+            }
+          }
+      } else {
+        spin_cycles(20000000LL);
+      }
+    }
+    if (warp == 1 && lane == 0 && leader && mma_issued) {
+      umma_commit_pair(&bars->drain);
+      const uint32_t a = smem_u32(&bars->drain);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(a, 0) && clock64() - t0 < p.wait_limit) {
+      }
+    }
+    __syncthreads();
+  }
+  tc_fence_before();
+  cluster_sync();   // the leader's MMAs no longer read this CTA's shared memory or TMEM
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, kTmemAlloc);
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicOr(p.status, kStatusTimeout);
+}
+
+}  // namespace
+
+bool onchip_supported(const Dims& d) {
+  return umma_supported(d) && d.Dt == UN && d.Ds <= 2 * UK && d.H % kChunk == 0;
+}
+
+cudaError_t launch_onchip(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                          const CUtensorMap& tmW1q, const CUtensorMap& tmW2h,
+                          const CUtensorMap& tmG16, const CUtensorMap& tmB2th, int num_sms,
+                          cudaStream_t st) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(onchip_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kSmemBytes);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  OnchipArgs oa;
+  oa.p = a;
+  oa.nk1 = a.d.Ds / UK;
+  oa.nc = a.d.EH / kChunk;
+  const long long pairs = static_cast<long long>(a.gp) * ((a.d.tiles_max + 1) / 2);
+  const long long max_pairs = num_sms / 2;
+  const int grid = 2 * static_cast<int>(pairs < max_pairs ? pairs : max_pairs);
+  if (grid <= 0) return cudaSuccess;
+  onchip_kernel<<<grid, kThreads, kSmemBytes, st>>>(tmK, tmV, tmW1q, tmW2h, tmG16, tmB2th, oa);
+  return cudaGetLastError();
+}
+
+}  // namespace mot

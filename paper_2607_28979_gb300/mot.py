@@ -222,7 +222,7 @@ def mot_get_path(h: Handle) -> int:
     return p.value
 
 
-SCHEDULE_SPLIT, SCHEDULE_FUSED, SCHEDULE_PAIR = 0, 1, 2
+SCHEDULE_SPLIT, SCHEDULE_FUSED, SCHEDULE_PAIR, SCHEDULE_ONCHIP = 0, 1, 2, 3
 
 
 def mot_set_schedule(h: Handle, schedule: int) -> None:

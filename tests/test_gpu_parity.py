@@ -50,12 +50,21 @@ SMALL = {
 }
 
 
-@pytest.mark.parametrize("schedule", [2, 1, 0])
+def onchip_supported(wl):
+    """Shapes the on-chip schedule (3) takes: D_s <= 128, D_t = 256, bf16 tensor-core path."""
+    d_s, d_t = wl.src_kv_heads * wl.src_head_dim, wl.tgt_kv_heads * wl.tgt_head_dim
+    return (wl.dtype == "bf16" and d_s <= 128 and d_t == 256 and wl.hidden % 256 == 0
+            and wl.src_head_dim % 64 == 0 and wl.tgt_head_dim % 32 == 0)
+
+
+@pytest.mark.parametrize("schedule", [3, 2, 1, 0])
 @pytest.mark.parametrize("name", sorted(SMALL))
 def test_small_shapes_every_element(name, schedule):
     wl = SMALL[name]
     if schedule != 2 and not name.startswith("umma"):
         pytest.skip("the schedule only applies to the tensor-core path")
+    if schedule == 3 and not onchip_supported(wl):
+        pytest.skip("the on-chip schedule needs D_s <= 128 and D_t = 256")
     sk, sv, blob = inputs(wl, seed=1)
     run = G.Run(wl, sk, sv, blob)
     expect_path = 1 if name.startswith("umma") else 0
@@ -65,11 +74,14 @@ def test_small_shapes_every_element(name, schedule):
     full_check(wl, run, sk, sv, blob, name)
 
 
-@pytest.mark.parametrize("other", [1, 2])
-@pytest.mark.parametrize("name", ["umma_ragged", "umma_e3", "gpt2s_opt125m", "qwen7_long"])
+@pytest.mark.parametrize("other", [1, 2, 3])
+@pytest.mark.parametrize("name", ["umma_ragged", "umma_e3", "gpt2s_opt125m", "qwen7_long",
+                                  "qwen05_qwen15"])
 def test_launch_schedules_are_bit_identical(name, other):
     """Every launch schedule runs the same per-tile arithmetic in the same order."""
     wl = SMALL.get(name) or synth.WORKLOADS[name]
+    if other == 3 and not onchip_supported(wl):
+        pytest.skip("the on-chip schedule needs D_s <= 128 and D_t = 256")
     sk, sv, blob = inputs(wl, seed=3)
     a = G.Run(wl, sk, sv, blob)
     b = G.Run(wl, sk, sv, blob)
@@ -267,6 +279,7 @@ def test_argument_errors_with_a_live_handle():
 
 
 @pytest.mark.parametrize("schedule,kernels", [
+    (3, {"prep_tiles", "gate", "umma2_onchip_translate"}),
     (2, {"prep_tiles", "gate", "umma2_gemm1_gelu_gate", "umma2_gemm2_combine_store"}),
     (1, {"prep_tiles", "gate", "umma_fused_translate"}),
     (0, {"prep_tiles", "gate", "umma_gemm1_gelu_gate", "umma_gemm2_combine_store"})])
@@ -274,7 +287,7 @@ def test_profile_and_launch_count(schedule, kernels):
     wl = SMALL["umma_ragged"]
     sk, sv, blob = inputs(wl, seed=10)
     run = G.Run(wl, sk, sv, blob)
-    assert M.mot_get_schedule(run.h) == 2
+    assert M.mot_get_schedule(run.h) == 3   # the default where the on-chip schedule applies
     M.mot_set_schedule(run.h, schedule)
     n0 = M.mot_get_launch_count(run.h)
     M.mot_profile_enable(run.h, True)
@@ -283,6 +296,21 @@ def test_profile_and_launch_count(schedule, kernels):
     assert set(stats) == kernels
     assert all(v[0] >= 1 and v[1] > 0 for v in stats.values())
     assert M.mot_get_launch_count(run.h) - n0 == sum(v[0] for v in stats.values())
+
+
+def test_onchip_schedule_is_refused_where_unsupported():
+    """D_t != 256: the default stays 2 and asking for 3 is MOT_ERR_UNSUPPORTED."""
+    wl = SMALL["umma_e1"]
+    sk, sv, blob = inputs(wl, seed=11)
+    run = G.Run(wl, sk, sv, blob)
+    assert M.mot_get_schedule(run.h) == 2
+    with pytest.raises(M.MotError) as e:
+        M.mot_set_schedule(run.h, 3)
+    assert e.value.status == M.MOT_ERR_UNSUPPORTED
+    assert M.mot_get_schedule(run.h) == 2
+    with pytest.raises(M.MotError) as e:
+        M.mot_set_schedule(run.h, 4)
+    assert e.value.status == M.MOT_ERR_INVALID_ARG
 
 
 # ---------------------------------------------------------------- Top-K routing (Def. 3.1)

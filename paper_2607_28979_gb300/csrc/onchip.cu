@@ -25,9 +25,13 @@
 //                           transaction bytes complete on the leader's barriers;
 //   warp 1 lane 0 (leader)  MMA issue, in the order G1(0) G1(1) | G2(j) G1(j+2) ... | bias;
 //   warp 2 (both)           TMEM allocation of the pair;
-//   warps 4..11 (both)      epilogue: warp 4 + 4 p + q owns rows 32 q .. 32 q + 31 and
-//                           the chunks with c % 2 == p; at the end of a tile it stores
-//                           output columns 128 p .. 128 p + 127.
+//   warps 4..11 (both)      epilogue: warp 4 + 4 p + q owns rows 32 q .. 32 q + 31; of
+//                           every chunk it evaluates columns 64 p .. 64 p + 63 (K block p
+//                           of the chunk's A2), and at the end of a tile it stores output
+//                           columns 128 p .. 128 p + 127.
+// With two acc1 buffers, the epilogue of chunk c has the MMA time of GEMM2(c-1)
+// and GEMM1(c+1) to finish before GEMM2(c) is due, so all eight warps share each
+// chunk and take its bias into registers before its accumulator is ready.
 // Every wait is bounded; a timeout unwinds and raises kStatusTimeout.
 #include "umma_common.cuh"
 
@@ -55,7 +59,7 @@ constexpr uint32_t kTmemAlloc = 512;
 struct Bars {
   uint64_t zfull[2], zempty[2], w1full[2], w1empty[2], w2full[2], w2empty[2];
   uint64_t a1full[2];   // GEMM1 of a chunk done (commit, both CTAs)
-  uint64_t a2full[2];   // chunk's A2 written and acc1 read (leader; 2 x 4 warp arrivals)
+  uint64_t a2full[2];   // chunk's A2 written and acc1 read (leader; 2 x 8 warp arrivals)
   uint64_t acc2full;    // a tile's GEMM2 + bias done (commit, both CTAs)
   uint64_t acc2empty;   // acc2 read out (leader; 2 x 8 warp arrivals)
   uint64_t drain;
@@ -76,36 +80,59 @@ __device__ __forceinline__ void spin_cycles(long long cycles) {
   }
 }
 
-// Row r's 32 columns of sub-chunk s (columns 32 s .. 32 s + 31 of the chunk)
-// into the A2 buffer at `a2`: K block s / 2, 16-byte chunks 4 (s % 2) .. + 3,
-// each at chunk position (index ^ (r % 8)) of its 128-byte row (128B swizzle).
-__device__ __forceinline__ void store_a2_sub(uint32_t a2, int r, int s, const uint32_t (&pk)[16]) {
-  const uint32_t row = a2 + static_cast<uint32_t>((s >> 1) * kBlk16 + r * 128);
-  const int c0 = (s & 1) * 4;
+// GELU(u + b) * g on 32 accumulator columns (`acc`, fp32 bits) with their
+// fp16 biases in `b` (four 16-byte vectors): fp16 pairs for the A2 operand.
+__device__ __forceinline__ void gelu_cols(const uint32_t (&acc)[32], const uint4* b, __half2 half_g,
+                                          uint32_t (&pk)[16]) {
+#pragma unroll
+  for (int v = 0; v < 4; ++v) {
+    const uint32_t bw[4] = {b[v].x, b[v].y, b[v].z, b[v].w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int j = v * 8 + 2 * k;
+      __half2 u = __float22half2_rn(make_float2(__uint_as_float(acc[j]), __uint_as_float(acc[j + 1])));
+      u = __hadd2(u, *reinterpret_cast<const __half2*>(&bw[k]));
+      const __half2 o = gelu_times_h2(u, half_g);
+      pk[4 * v + k] = *reinterpret_cast<const uint32_t*>(&o);
+    }
+  }
+}
+
+// Row r's 16-byte chunks 4 s .. 4 s + 3 of a 64-wide K block at `blk`, each at
+// chunk position (index ^ (r % 8)) of its 128-byte row (the 128B swizzle).
+__device__ __forceinline__ void store_a2(uint32_t blk, int r, int s, const uint32_t (&pk)[16]) {
+  const uint32_t row = blk + static_cast<uint32_t>(r * 128);
 #pragma unroll
   for (int v = 0; v < 4; ++v)
-    st_shared_v4(row + static_cast<uint32_t>(((c0 + v) ^ (r & 7)) << 4), pk[4 * v],
+    st_shared_v4(row + static_cast<uint32_t>(((4 * s + v) ^ (r & 7)) << 4), pk[4 * v],
                  pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
 }
 
-// GEMM1 epilogue of one warp for one chunk: TMEM acc1 (32 rows x 128 columns
-// at `tb`) -> GELU(u + b1) * g -> fp16 into the A2 buffer at `a2`.
-__device__ __forceinline__ void epi_chunk(uint32_t tb, const __half* bias, float gate, uint32_t a2,
-                                          int r) {
+// One warp's share of a chunk: TMEM acc1 columns at `tb` (32 rows x 64) ->
+// GELU(u + b1) * g -> fp16 into the K block at `blk` of the A2 buffer.
+__device__ __forceinline__ void epi_half(uint32_t tb, const uint4 (&bias)[8], float gate,
+                                         uint32_t blk, int r) {
   const __half2 half_g = __float2half2_rn(0.5f * gate);
   uint32_t ra[32], rb[32], pk[16];
   tmem_ld_32x32b_x32(tb, ra);
-#pragma unroll 1
-  for (int s = 0; s < 4; s += 2) {
-    tmem_ld_wait(ra);
-    tmem_ld_32x32b_x32(tb + (s + 1) * 32, rb);
-    gemm1_sub(ra, reinterpret_cast<const uint4*>(bias + s * 32), half_g, pk);
-    store_a2_sub(a2, r, s, pk);
-    tmem_ld_wait(rb);
-    if (s + 2 < 4) tmem_ld_32x32b_x32(tb + (s + 2) * 32, ra);
-    gemm1_sub(rb, reinterpret_cast<const uint4*>(bias + (s + 1) * 32), half_g, pk);
-    store_a2_sub(a2, r, s + 1, pk);
-  }
+  tmem_ld_32x32b_x32(tb + 32, rb);
+  tmem_ld_wait(ra);
+  tmem_ld_wait(rb);
+  gelu_cols(ra, bias, half_g, pk);
+  store_a2(blk, r, 0, pk);
+  gelu_cols(rb, bias + 4, half_g, pk);
+  store_a2(blk, r, 1, pk);
+}
+
+// 32 fp32 accumulator columns -> 32 bf16 channels at `o` (64 bytes).
+__device__ __forceinline__ void store_out(const uint32_t (&acc)[32], __nv_bfloat16* o) {
+  uint4* o4 = reinterpret_cast<uint4*>(o);
+#pragma unroll
+  for (int v = 0; v < 4; ++v)
+    o4[v] = make_uint4(pack_bf16x2(__uint_as_float(acc[8 * v + 0]), __uint_as_float(acc[8 * v + 1])),
+                       pack_bf16x2(__uint_as_float(acc[8 * v + 2]), __uint_as_float(acc[8 * v + 3])),
+                       pack_bf16x2(__uint_as_float(acc[8 * v + 4]), __uint_as_float(acc[8 * v + 5])),
+                       pack_bf16x2(__uint_as_float(acc[8 * v + 6]), __uint_as_float(acc[8 * v + 7])));
 }
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
@@ -140,7 +167,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(&bars->w2full[i], 1);
       mbar_init(&bars->w2empty[i], 1);
       mbar_init(&bars->a1full[i], 1);
-      mbar_init(&bars->a2full[i], 2 * (kEpiWarps / 2));
+      mbar_init(&bars->a2full[i], 2 * kEpiWarps);
     }
     mbar_init(&bars->acc2full, 1);
     mbar_init(&bars->acc2empty, 2 * kEpiWarps);
@@ -328,12 +355,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= 4) {
     // ------------------------------------------------ epilogue (both CTAs)
-    const int e = warp - 4, q = e & 3, par = e >> 2;
+    const int e = warp - 4, q = e & 3, hh = e >> 2;
     const int r = q * 32 + lane;
     const uint32_t tq = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
-    const uint32_t a2_addr = smem_u32(sA2 + par * kA2Bytes);
+    const uint32_t a2_addr = smem_u32(sA2) + static_cast<uint32_t>(hh * kBlk16);
     const __half* b1h = static_cast<const __half*>(p.b1h);
-    uint32_t c0 = 0, k = 0;
+    uint32_t c = 0, k = 0;
     bool ok = true;
     for (int t = pair; ok && t < total; t += n_pairs, ++k) {
       const int gl = t / n_mp, mp = t - gl * n_mp;
@@ -342,30 +369,59 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const bool valid = m_own < n_m;
       const float* grow =
           p.gate + (static_cast<size_t>(grp) * d.tpad + static_cast<size_t>(m_own) * UM + r) * d.E;
-      for (int j = static_cast<int>((c0 & 1u) ^ static_cast<uint32_t>(par)); j < nc; j += 2) {
-        const uint32_t c = c0 + j;
+      const uint4* bias4 = reinterpret_cast<const uint4*>(b1h + static_cast<size_t>(grp) * d.EH) +
+                           hh * 8;
+      for (int j = 0; j < nc; ++j, ++c) {
+        const uint32_t b = c & 1u;
+        // this warp's 64 biases and the row's gate value, fetched before the wait
+        uint4 bias[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) bias[i] = __ldg(bias4 + j * (kChunk / 8) + i);
         const float gate = valid ? __ldg(grow + (j * kChunk) / d.H) : 0.f;
         int w = 1;
-        if (lane == 0) w = mbar_wait(&bars->a1full[par], (c >> 1) & 1u, abort_flag, p.wait_limit);
+        if (lane == 0) w = mbar_wait(&bars->a1full[b], (c >> 1) & 1u, abort_flag, p.wait_limit);
         if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
         tc_fence_after();
-        epi_chunk(tq + kAcc1Col + par * kChunk, b1h + static_cast<size_t>(grp) * d.EH + j * kChunk,
-                  gate, a2_addr, r);
+        epi_half(tq + kAcc1Col + b * kChunk + hh * 64, bias, gate, a2_addr + b * kA2Bytes, r);
         fence_proxy_async_smem();   // the MMA (async proxy) reads these stores
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive_cluster(&bars->a2full[par], 0);
+        if (lane == 0) mbar_arrive_cluster(&bars->a2full[b], 0);
       }
       if (!ok) break;
+      // output: columns 128 hh .. 128 hh + 127 of this warp's rows
+      const GroupInfo gi = p.groups[grp];
+      TileInfo ti;
+      ti.rows = 0;
+      if (valid) ti = p.tiles[m_own];
       int w = 1;
       if (lane == 0) w = mbar_wait(&bars->acc2full, k & 1u, abort_flag, p.wait_limit);
       if (!__shfl_sync(0xffffffffu, w, 0)) break;
       tc_fence_after();
-      if (valid) epilogue_gemm2(p, tq, q, lane, grp, m_own, 0, par * (UN / 2), UN / 64);
+      if (valid) {   // warp-uniform: the TMEM loads are warp-collective; stores are per row
+        __nv_bfloat16* const dst = static_cast<__nv_bfloat16*>(gi.x ? p.dst[1] : p.dst[0]);
+        const size_t s_pos = static_cast<size_t>(ti.s0) + r;
+        auto out = [&](int col) {
+          const int h = col / d.d_t, i0 = col - h * d.d_t;
+          return dst + ((((static_cast<size_t>(gi.tgt_layer) * d.B + ti.b) * d.H_t + h) * d.S +
+                         s_pos) * d.d_t + i0);
+        };
+        uint32_t ra[32], rb[32];
+#pragma unroll 1
+        for (int cc = hh * (UN / 2); cc < (hh + 1) * (UN / 2); cc += 64) {
+          tmem_ld_32x32b_x32(tq + cc, ra);
+          tmem_ld_32x32b_x32(tq + cc + 32, rb);
+          tmem_ld_wait(ra);
+          tmem_ld_wait(rb);
+          if (r < ti.rows) {
+            store_out(ra, out(cc));
+            store_out(rb, out(cc + 32));
+          }
+        }
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(&bars->acc2empty, 0);
-      c0 += nc;
     }
   }
 

@@ -17,21 +17,24 @@
 //
 // TMEM per CTA (512 columns): acc2 in [0, 256), acc1[0] in [256, 384),
 // acc1[1] in [384, 512). Shared memory per CTA: Z 2 x 32 KB (the next tile's
-// rows load during the current tile), W1 ring 2 x 16 KB, W2 ring 2 x 32 KB
-// (the last stage of a tile holds b2t and gate16), A2 2 x 32 KB.
+// rows load during the current tile; after its last GEMM1 a tile's buffer
+// holds b2t and gate16 for the bias MMA), W1 ring 2 x 16 KB, W2 ring
+// 2 x 32 KB, A2 2 x 32 KB.
 //
 // Roles per CTA:
 //   warp 0 lane 0 (both)    TMA loads of its Z rows and its halves of W1 / W2;
 //                           transaction bytes complete on the leader's barriers;
-//   warp 1 lane 0 (leader)  MMA issue, in the order G1(0) G1(1) | G2(j) G1(j+2) ... | bias;
+//   warp 1 (leader)         MMA issue (one elected lane), in the order
+//                           G1(0) G1(1) | G1(j+2) G2(j) ... | bias;
 //   warp 2 (both)           TMEM allocation of the pair;
-//   warps 4..11 (both)      epilogue: warp 4 + 4 p + q owns rows 32 q .. 32 q + 31; of
-//                           every chunk it evaluates columns 64 p .. 64 p + 63 (K block p
-//                           of the chunk's A2), and at the end of a tile it stores output
-//                           columns 128 p .. 128 p + 127.
-// With two acc1 buffers, the epilogue of chunk c has the MMA time of GEMM2(c-1)
-// and GEMM1(c+1) to finish before GEMM2(c) is due, so all eight warps share each
-// chunk and take its bias into registers before its accumulator is ready.
+//   warps 4..19 (both)      epilogue: warp 4 + 4 p + q owns rows 32 q .. 32 q + 31; of
+//                           every chunk it evaluates columns 32 p .. 32 p + 31, and at the
+//                           end of a tile it stores output columns 64 p .. 64 p + 63.
+// With two acc1 buffers the chunk epilogue is on the MMA's critical path, so it
+// is kept short: all sixteen warps share each chunk, take its biases into
+// registers before its accumulator is ready, and release acc1 as soon as it is
+// read (GEMM1 two chunks ahead is issued then, ahead of GEMM2 of this chunk);
+// the A2 stores then wait only for GEMM2 two chunks back.
 // Every wait is bounded; a timeout unwinds and raises kStatusTimeout.
 #include "umma_common.cuh"
 
@@ -49,19 +52,27 @@ constexpr int kOffW1 = 2 * kZBytes;
 constexpr int kOffW2 = kOffW1 + 2 * kW1Bytes;
 constexpr int kOffA2 = kOffW2 + 2 * kW2Bytes;
 constexpr int kOffBar = kOffA2 + 2 * kA2Bytes;
-constexpr int kEpiWarps = 8;
+constexpr int kEpiWarps = 16;
 constexpr int kThreads = 32 * (4 + kEpiWarps);
 constexpr int kSmemBytes = kOffBar + 256 + 1024;
 static_assert(kSmemBytes <= 232448, "shared memory budget");
 constexpr uint32_t kAcc1Col = UN;   // acc1[b] at column 256 + 128 b
 constexpr uint32_t kTmemAlloc = 512;
 
+// Each tcgen05.commit costs the tensor pipe several hundred cycles, so a chunk
+// has two: a1full (GEMM1 done: its acc1 is ready and its W1 slot free) and
+// a2empty (GEMM2 done: its A2 buffer and its W2 slot free). The ring slots of
+// W1, W2, acc1 and A2 are all indexed by the chunk counter c, so one commit
+// serves both waiters; the tile's bias stage (gate16, b2t) uses the tile's Z
+// buffer once its last GEMM1 is done.
 struct Bars {
-  uint64_t zfull[2], zempty[2], w1full[2], w1empty[2], w2full[2], w2empty[2];
+  uint64_t zfull[2], zempty[2], w1full[2], w2full[2], bfull[2];
   uint64_t a1full[2];   // GEMM1 of a chunk done (commit, both CTAs)
-  uint64_t a2full[2];   // chunk's A2 written and acc1 read (leader; 2 x 8 warp arrivals)
+  uint64_t acc1free[2]; // the chunk's acc1 read out (leader; 2 x 16 warp arrivals)
+  uint64_t a2full[2];   // the chunk's A2 written (leader; 2 x 16 warp arrivals)
+  uint64_t a2empty[2];  // GEMM2 of a chunk done reading its A2 (commit, both CTAs)
   uint64_t acc2full;    // a tile's GEMM2 + bias done (commit, both CTAs)
-  uint64_t acc2empty;   // acc2 read out (leader; 2 x 8 warp arrivals)
+  uint64_t acc2empty;   // acc2 read out (leader; 2 x 16 warp arrivals)
   uint64_t drain;
   uint32_t tmem_slot;
   int abort_flag;
@@ -108,23 +119,21 @@ __device__ __forceinline__ void store_a2(uint32_t blk, int r, int s, const uint3
                  pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
 }
 
-// One warp's share of a chunk: TMEM acc1 columns at `tb` (32 rows x 64) ->
-// GELU(u + b1) * g -> fp16 into the K block at `blk` of the A2 buffer.
-__device__ __forceinline__ void epi_half(uint32_t tb, const uint4 (&bias)[8], float gate,
-                                         uint32_t blk, int r) {
-  const __half2 half_g = __float2half2_rn(0.5f * gate);
-  uint32_t ra[32], rb[32], pk[16];
-  tmem_ld_32x32b_x32(tb, ra);
-  tmem_ld_32x32b_x32(tb + 32, rb);
-  tmem_ld_wait(ra);
-  tmem_ld_wait(rb);
-  gelu_cols(ra, bias, half_g, pk);
-  store_a2(blk, r, 0, pk);
-  gelu_cols(rb, bias + 4, half_g, pk);
-  store_a2(blk, r, 1, pk);
+// 32 fp32 accumulator columns -> 32 bf16 channels at `o` (64 bytes), as two
+// 32-byte stores (`o` 32-byte aligned) or four 16-byte stores.
+__device__ __forceinline__ void store_out32(const uint32_t (&acc)[32], __nv_bfloat16* o) {
+  uint32_t w[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i)
+    w[i] = pack_bf16x2(__uint_as_float(acc[2 * i]), __uint_as_float(acc[2 * i + 1]));
+#pragma unroll
+  for (int h = 0; h < 2; ++h)
+    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(o + 16 * h),
+                 "r"(w[8 * h]), "r"(w[8 * h + 1]), "r"(w[8 * h + 2]), "r"(w[8 * h + 3]),
+                 "r"(w[8 * h + 4]), "r"(w[8 * h + 5]), "r"(w[8 * h + 6]), "r"(w[8 * h + 7])
+                 : "memory");
 }
 
-// 32 fp32 accumulator columns -> 32 bf16 channels at `o` (64 bytes).
 __device__ __forceinline__ void store_out(const uint32_t (&acc)[32], __nv_bfloat16* o) {
   uint4* o4 = reinterpret_cast<uint4*>(o);
 #pragma unroll
@@ -163,11 +172,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(&bars->zfull[i], 1);
       mbar_init(&bars->zempty[i], 1);
       mbar_init(&bars->w1full[i], 1);
-      mbar_init(&bars->w1empty[i], 1);
       mbar_init(&bars->w2full[i], 1);
-      mbar_init(&bars->w2empty[i], 1);
+      mbar_init(&bars->bfull[i], 1);
       mbar_init(&bars->a1full[i], 1);
+      mbar_init(&bars->acc1free[i], 2 * kEpiWarps);
       mbar_init(&bars->a2full[i], 2 * kEpiWarps);
+      mbar_init(&bars->a2empty[i], 1);
     }
     mbar_init(&bars->acc2full, 1);
     mbar_init(&bars->acc2empty, 2 * kEpiWarps);
@@ -198,14 +208,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
 
   // unwinding state: full barriers with loads in flight (bit i: zfull 0-1,
-  // w1full 2-3, w2full 4-5) and the parity of each one's last phase
+  // w1full 2-3, w2full 4-5, bfull 6-7) and the parity of each one's last phase
   uint32_t pend_mask = 0, pend_par = 0;
   bool mma_issued = false;
 
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------ TMA producer (both CTAs)
-      uint32_t i1 = 0, i2 = 0;
       auto note = [&](int bit, uint32_t ph) {
         pend_mask |= 1u << bit;
         pend_par = (pend_par & ~(1u << bit)) | (ph << bit);
@@ -234,131 +243,153 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         note(zb, ph);
         return true;
       };
-      auto load_w1 = [&](int grp, int j) -> bool {
-        const int s = i1 & 1;
-        const uint32_t ph = (i1 >> 1) & 1u;
-        if (!mbar_wait(&bars->w1empty[s], ph ^ 1u, abort_flag, p.wait_limit)) return false;
+      // W1 rows of chunk c (column block j of group grp) into slot c % 2, once
+      // GEMM1(c - 2) has released it
+      auto load_w1 = [&](int grp, int j, uint32_t c) -> bool {
+        const int s = c & 1;
+        const uint32_t ph = (c >> 1) & 1u;
+        if (!mbar_wait(&bars->a1full[s], ph ^ 1u, abort_flag, p.wait_limit)) return false;
         if (leader) mbar_arrive_expect_tx(&bars->w1full[s], 2 * nk1 * kW1Blk);
         const uint32_t bar = leader_addr(&bars->w1full[s]);
         const int row = grp * d.EH + j * kChunk + static_cast<int>(rank) * (kChunk / 2);
         for (int kb = 0; kb < nk1; ++kb)
           tma_load_2d_pair(sW1 + s * kW1Bytes + kb * kW1Blk, &tmW1q, bar, kb * UK, row);
         note(2 + s, ph);
-        ++i1;
         return true;
       };
-      auto load_w2 = [&](int grp, int m_own, int j) -> bool {   // j == nc: the bias stage
-        const int s = i2 & 1;
-        const uint32_t ph = (i2 >> 1) & 1u;
-        if (!mbar_wait(&bars->w2empty[s], ph ^ 1u, abort_flag, p.wait_limit)) return false;
+      // W2 columns of chunk c into slot c % 2, once GEMM2(c - 2) has released it
+      auto load_w2 = [&](int grp, int j, uint32_t c) -> bool {
+        const int s = c & 1;
+        const uint32_t ph = (c >> 1) & 1u;
+        if (!mbar_wait(&bars->a2empty[s], ph ^ 1u, abort_flag, p.wait_limit)) return false;
         if (leader) mbar_arrive_expect_tx(&bars->w2full[s], 2 * kW2Bytes);
         const uint32_t bar = leader_addr(&bars->w2full[s]);
         const int row = grp * d.Dt + static_cast<int>(rank) * (UN / 2);
         uint8_t* dst = sW2 + s * kW2Bytes;
-        if (j < nc) {
-          tma_load_2d_pair(dst, &tmW2h, bar, j * kChunk, row);
-          tma_load_2d_pair(dst + kBlk16, &tmW2h, bar, j * kChunk + UK, row);
-        } else {   // B = b2t half, A = gate16 rows of this CTA's token tile
-          tma_load_2d_pair(dst, &tmB2th, bar, 0, row);
-          tma_load_3d_pair(dst + kBlk16, &tmG16, bar, 0, m_own * UM, grp);
-        }
+        tma_load_2d_pair(dst, &tmW2h, bar, j * kChunk, row);
+        tma_load_2d_pair(dst + kBlk16, &tmW2h, bar, j * kChunk + UK, row);
         note(4 + s, ph);
-        ++i2;
         return true;
       };
-      uint32_t k = 0;
-      for (int t = pair; t < total; t += n_pairs, ++k) {
+      // the tile's bias stage into its Z buffer once GEMM1 of its last chunk
+      // c_last is done: B = b2t half, A = gate16 rows of this CTA's token tile
+      auto load_bias = [&](int grp, int m_own, uint32_t k, uint32_t c_last) -> bool {
+        const int zb = k & 1;
+        const uint32_t ph = (k >> 1) & 1u;
+        if (!mbar_wait(&bars->a1full[c_last & 1], (c_last >> 1) & 1u, abort_flag, p.wait_limit))
+          return false;
+        if (leader) mbar_arrive_expect_tx(&bars->bfull[zb], 2 * kZBytes);
+        const uint32_t bar = leader_addr(&bars->bfull[zb]);
+        const int row = grp * d.Dt + static_cast<int>(rank) * (UN / 2);
+        tma_load_2d_pair(sZ + zb * kZBytes, &tmB2th, bar, 0, row);
+        tma_load_3d_pair(sZ + zb * kZBytes + kBlk16, &tmG16, bar, 0, m_own * UM, grp);
+        note(6 + zb, ph);
+        return true;
+      };
+      uint32_t k = 0, c0 = 0;
+      for (int t = pair; t < total; t += n_pairs, ++k, c0 += nc) {
         const int gl = t / n_mp, mp = t - gl * n_mp;
         const int grp = p.g0 + gl;
         const int m_own = 2 * mp + static_cast<int>(rank);
         bool ok = true;
         if (k == 0) ok = load_z(t, 0);
-        ok = ok && load_w1(grp, 0);
-        if (nc > 1) ok = ok && load_w1(grp, 1);
+        ok = ok && load_w1(grp, 0, c0);
+        if (nc > 1) ok = ok && load_w1(grp, 1, c0 + 1);
         if (t + n_pairs < total) ok = ok && load_z(t + n_pairs, k + 1);
-        for (int j = 0; ok && j < nc; ++j) {
-          ok = load_w2(grp, m_own, j);
-          if (j + 2 < nc) ok = ok && load_w1(grp, j + 2);
+        for (int j = 0; ok && j < nc; ++j) {   // the MMA's order: GEMM1(j + 2), then GEMM2(j)
+          if (j + 2 < nc) ok = load_w1(grp, j + 2, c0 + j + 2);
+          ok = ok && load_w2(grp, j, c0 + j);
         }
-        ok = ok && load_w2(grp, m_own, nc);
+        ok = ok && load_bias(grp, m_own, k, c0 + nc - 1);
         if (!ok) break;
       }
     }
   } else if (warp == 1) {
-    if (lane == 0 && leader) {
-      // ------------------------------------------------ MMA issuer (leader)
+    if (leader) {
+      // ------------------------------------------------ MMA issuer (leader, whole warp)
+      // The loop, the waits and the descriptors are warp-uniform; one elected
+      // lane issues the MMAs and their commits.
       constexpr uint32_t idesc1 = idesc_bf16_f32(2 * UM, kChunk);
       constexpr uint32_t idesc2 = idesc_f16_f32(2 * UM, UN);
-      uint32_t i1 = 0, i2 = 0, c0 = 0, k = 0;
+      auto wait_all = [&](uint64_t* bar, uint32_t parity) -> bool {
+        const bool r = mbar_wait(bar, parity, abort_flag, p.wait_limit);
+        return __all_sync(0xffffffffu, r) != 0;
+      };
+      uint32_t c0 = 0, k = 0;
       bool ok = true;
       for (int t = pair; ok && t < total; t += n_pairs, ++k) {
         const int zb = k & 1;
-        if (!mbar_wait(&bars->zfull[zb], (k >> 1) & 1u, abort_flag, p.wait_limit)) break;
+        if (!wait_all(&bars->zfull[zb], (k >> 1) & 1u)) break;
         tc_fence_after();
+        const uint32_t zaddr = smem_u32(sZ + zb * kZBytes);
         auto g1 = [&](int j) -> bool {
-          const int s = i1 & 1;
-          if (!mbar_wait(&bars->w1full[s], (i1 >> 1) & 1u, abort_flag, p.wait_limit)) return false;
+          const uint32_t c = c0 + j, b = c & 1u;
+          if (!wait_all(&bars->w1full[b], (c >> 1) & 1u)) return false;
           tc_fence_after();
-          const uint32_t b = (c0 + j) & 1u;
-          for (int kb = 0; kb < nk1; ++kb) {
-            const uint64_t zdesc = sdesc_k_sw128(smem_u32(sZ + zb * kZBytes + kb * kBlk16));
-            const uint64_t wdesc = sdesc_k_sw128(smem_u32(sW1 + s * kW1Bytes + kb * kW1Blk));
+          const uint32_t waddr = smem_u32(sW1 + b * kW1Bytes);
+          if (elect_one()) {
+            for (int kb = 0; kb < nk1; ++kb) {
+              const uint64_t zdesc = sdesc_k_sw128(zaddr + kb * kBlk16);
+              const uint64_t wdesc = sdesc_k_sw128(waddr + kb * kW1Blk);
 #pragma unroll
-            for (int kk = 0; kk < UK / 16; ++kk)   // +32 bytes of K = +2 in the address field
-              umma_pair(tmem_base + kAcc1Col + b * kChunk, zdesc + 2 * kk, wdesc + 2 * kk, idesc1,
-                        (kb | kk) != 0);
+              for (int kk = 0; kk < UK / 16; ++kk)   // +32 bytes of K = +2 in the address field
+                umma_pair(tmem_base + kAcc1Col + b * kChunk, zdesc + 2 * kk, wdesc + 2 * kk, idesc1,
+                          (kb | kk) != 0);
+            }
+            umma_commit_pair(&bars->a1full[b]);
           }
+          __syncwarp();
           mma_issued = true;
-          umma_commit_pair(&bars->w1empty[s]);
-          umma_commit_pair(&bars->a1full[b]);
-          if (j == nc - 1) umma_commit_pair(&bars->zempty[zb]);
-          ++i1;
           return true;
         };
         ok = g1(0) && (nc < 2 || g1(1));
         for (int j = 0; ok && j < nc; ++j) {
           const uint32_t c = c0 + j, b = c & 1u;
-          ok = mbar_wait(&bars->a2full[b], (c >> 1) & 1u, abort_flag, p.wait_limit);
-          if (ok && j == 0)
-            ok = mbar_wait(&bars->acc2empty, (k & 1u) ^ 1u, abort_flag, p.wait_limit);
-          const int s = i2 & 1;
-          ok = ok && mbar_wait(&bars->w2full[s], (i2 >> 1) & 1u, abort_flag, p.wait_limit);
+          // GEMM1 two chunks ahead as soon as this chunk's acc1 is read out, so
+          // that its epilogue overlaps GEMM2 of this chunk
+          if (j + 2 < nc) ok = wait_all(&bars->acc1free[b], (c >> 1) & 1u) && g1(j + 2);
+          ok = ok && wait_all(&bars->a2full[b], (c >> 1) & 1u);
+          if (ok && j == 0) ok = wait_all(&bars->acc2empty, (k & 1u) ^ 1u);
+          ok = ok && wait_all(&bars->w2full[b], (c >> 1) & 1u);
           if (!ok) break;
           tc_fence_after();
+          const uint32_t aaddr = smem_u32(sA2 + b * kA2Bytes), baddr = smem_u32(sW2 + b * kW2Bytes);
+          if (elect_one()) {
 #pragma unroll
-          for (int kb = 0; kb < 2; ++kb) {
-            const uint64_t adesc = sdesc_k_sw128(smem_u32(sA2 + b * kA2Bytes + kb * kBlk16));
-            const uint64_t bdesc = sdesc_k_sw128(smem_u32(sW2 + s * kW2Bytes + kb * kBlk16));
+            for (int kb = 0; kb < 2; ++kb) {
+              const uint64_t adesc = sdesc_k_sw128(aaddr + kb * kBlk16);
+              const uint64_t bdesc = sdesc_k_sw128(baddr + kb * kBlk16);
 #pragma unroll
-            for (int kk = 0; kk < UK / 16; ++kk)
-              umma_pair(tmem_base, adesc + 2 * kk, bdesc + 2 * kk, idesc2, (j | kb | kk) != 0);
+              for (int kk = 0; kk < UK / 16; ++kk)
+                umma_pair(tmem_base, adesc + 2 * kk, bdesc + 2 * kk, idesc2, (j | kb | kk) != 0);
+            }
+            umma_commit_pair(&bars->a2empty[b]);
           }
-          umma_commit_pair(&bars->w2empty[s]);
-          ++i2;
-          if (j + 2 < nc) ok = g1(j + 2);
+          __syncwarp();
         }
         if (!ok) break;
-        // gate-weighted biases: A = gate16 (second block of the stage), B = b2t
-        const int s = i2 & 1;
-        if (!mbar_wait(&bars->w2full[s], (i2 >> 1) & 1u, abort_flag, p.wait_limit)) break;
+        // gate-weighted biases from the tile's Z buffer: A = gate16, B = b2t
+        if (!wait_all(&bars->bfull[zb], (k >> 1) & 1u)) break;
         tc_fence_after();
-        const uint64_t gdesc = sdesc_k_sw128(smem_u32(sW2 + s * kW2Bytes + kBlk16));
-        const uint64_t bdesc = sdesc_k_sw128(smem_u32(sW2 + s * kW2Bytes));
+        if (elect_one()) {
+          const uint64_t gdesc = sdesc_k_sw128(zaddr + kBlk16);
+          const uint64_t bdesc = sdesc_k_sw128(zaddr);
 #pragma unroll
-        for (int kk = 0; kk < UK / 16; ++kk)
-          umma_pair(tmem_base, gdesc + 2 * kk, bdesc + 2 * kk, idesc2, 1u);
-        umma_commit_pair(&bars->w2empty[s]);
-        umma_commit_pair(&bars->acc2full);
-        ++i2;
+          for (int kk = 0; kk < UK / 16; ++kk)
+            umma_pair(tmem_base, gdesc + 2 * kk, bdesc + 2 * kk, idesc2, 1u);
+          umma_commit_pair(&bars->zempty[zb]);
+          umma_commit_pair(&bars->acc2full);
+        }
+        __syncwarp();
         c0 += nc;
       }
     }
   } else if (warp >= 4) {
     // ------------------------------------------------ epilogue (both CTAs)
-    const int e = warp - 4, q = e & 3, hh = e >> 2;
+    const int e = warp - 4, q = e & 3, hh = e >> 2;   // rows 32 q.., chunk columns 32 hh..
     const int r = q * 32 + lane;
     const uint32_t tq = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
-    const uint32_t a2_addr = smem_u32(sA2) + static_cast<uint32_t>(hh * kBlk16);
+    const uint32_t a2_addr = smem_u32(sA2) + static_cast<uint32_t>((hh >> 1) * kBlk16);
     const __half* b1h = static_cast<const __half*>(p.b1h);
     uint32_t c = 0, k = 0;
     bool ok = true;
@@ -370,26 +401,38 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const float* grow =
           p.gate + (static_cast<size_t>(grp) * d.tpad + static_cast<size_t>(m_own) * UM + r) * d.E;
       const uint4* bias4 = reinterpret_cast<const uint4*>(b1h + static_cast<size_t>(grp) * d.EH) +
-                           hh * 8;
+                           hh * 4;
       for (int j = 0; j < nc; ++j, ++c) {
         const uint32_t b = c & 1u;
-        // this warp's 64 biases and the row's gate value, fetched before the wait
-        uint4 bias[8];
+        // this warp's 32 biases and the row's gate value, fetched before the wait
+        uint4 bias[4];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) bias[i] = __ldg(bias4 + j * (kChunk / 8) + i);
+        for (int i = 0; i < 4; ++i) bias[i] = __ldg(bias4 + j * (kChunk / 8) + i);
         const float gate = valid ? __ldg(grow + (j * kChunk) / d.H) : 0.f;
         int w = 1;
         if (lane == 0) w = mbar_wait(&bars->a1full[b], (c >> 1) & 1u, abort_flag, p.wait_limit);
         if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
         tc_fence_after();
-        epi_half(tq + kAcc1Col + b * kChunk + hh * 64, bias, gate, a2_addr + b * kA2Bytes, r);
+        uint32_t pa[16];
+        {
+          uint32_t ra[32];
+          tmem_ld_32x32b_x32(tq + kAcc1Col + b * kChunk + hh * 32, ra);
+          tmem_ld_wait(ra);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(&bars->acc1free[b], 0);   // GEMM1(c + 2) may start
+          gelu_cols(ra, bias, __float2half2_rn(0.5f * gate), pa);
+        }
+        // GEMM2(c - 2) must be done reading this A2 buffer
+        if (lane == 0) w = mbar_wait(&bars->a2empty[b], ((c >> 1) & 1u) ^ 1u, abort_flag, p.wait_limit);
+        if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+        store_a2(a2_addr + b * kA2Bytes, r, hh & 1, pa);
         fence_proxy_async_smem();   // the MMA (async proxy) reads these stores
-        tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive_cluster(&bars->a2full[b], 0);
       }
       if (!ok) break;
-      // output: columns 128 hh .. 128 hh + 127 of this warp's rows
+      // output: columns 64 hh .. 64 hh + 63 of this warp's rows
       const GroupInfo gi = p.groups[grp];
       TileInfo ti;
       ti.rows = 0;
@@ -400,6 +443,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       tc_fence_after();
       if (valid) {   // warp-uniform: the TMEM loads are warp-collective; stores are per row
         __nv_bfloat16* const dst = static_cast<__nv_bfloat16*>(gi.x ? p.dst[1] : p.dst[0]);
+        const bool wide = (reinterpret_cast<uintptr_t>(dst) & 31u) == 0;   // 32-byte stores
         const size_t s_pos = static_cast<size_t>(ti.s0) + r;
         auto out = [&](int col) {
           const int h = col / d.d_t, i0 = col - h * d.d_t;
@@ -408,14 +452,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         };
         uint32_t ra[32], rb[32];
 #pragma unroll 1
-        for (int cc = hh * (UN / 2); cc < (hh + 1) * (UN / 2); cc += 64) {
+        for (int cc = hh * (UN / 4); cc < (hh + 1) * (UN / 4); cc += 64) {
           tmem_ld_32x32b_x32(tq + cc, ra);
           tmem_ld_32x32b_x32(tq + cc + 32, rb);
           tmem_ld_wait(ra);
           tmem_ld_wait(rb);
           if (r < ti.rows) {
-            store_out(ra, out(cc));
-            store_out(rb, out(cc + 32));
+            if (wide) {
+              store_out32(ra, out(cc));
+              store_out32(rb, out(cc + 32));
+            } else {
+              store_out(ra, out(cc));
+              store_out(rb, out(cc + 32));
+            }
           }
         }
       }
@@ -433,10 +482,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // leader also waits for its issued MMAs.
     if (warp == 0 && lane == 0 && pend_mask) {
       if (leader) {
-        uint64_t* fulls[6] = {&bars->zfull[0],  &bars->zfull[1],  &bars->w1full[0],
-                              &bars->w1full[1], &bars->w2full[0], &bars->w2full[1]};
+        uint64_t* fulls[8] = {&bars->zfull[0],  &bars->zfull[1],  &bars->w1full[0],
+                              &bars->w1full[1], &bars->w2full[0], &bars->w2full[1],
+                              &bars->bfull[0],  &bars->bfull[1]};
 #pragma unroll
-        for (int i = 0; i < 6; ++i)
+        for (int i = 0; i < 8; ++i)
           if ((pend_mask >> i) & 1u) {
             const uint32_t a = smem_u32(fulls[i]);
             const long long t0 = clock64();
@@ -447,12 +497,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         spin_cycles(20000000LL);
       }
     }
-    if (warp == 1 && lane == 0 && leader && mma_issued) {
-      umma_commit_pair(&bars->drain);
-      const uint32_t a = smem_u32(&bars->drain);
-      const long long t0 = clock64();
-      while (!mbar_try_wait(a, 0) && clock64() - t0 < p.wait_limit) {
+    if (warp == 1 && leader && mma_issued) {   // the lane that issued the MMAs commits
+      if (elect_one()) {
+        umma_commit_pair(&bars->drain);
+        const uint32_t a = smem_u32(&bars->drain);
+        const long long t0 = clock64();
+        while (!mbar_try_wait(a, 0) && clock64() - t0 < p.wait_limit) {
+        }
       }
+      __syncwarp();
     }
     __syncthreads();
   }

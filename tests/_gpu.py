@@ -31,15 +31,16 @@ def sentinel(wl):
     return SENTINEL_BF16 if wl.dtype == "bf16" else SENTINEL_F32
 
 
-def alloc_dst(wl):
-    """A target cache with CANARY_ELEMS guard elements after its end, all filled
-    with the sentinel. Returns (full buffer, cache view)."""
+def alloc_dst(wl, lead=0):
+    """A target cache with CANARY_ELEMS guard elements after its end and `lead`
+    before its start (which shifts its alignment), all filled with the sentinel.
+    Returns (full buffer, cache view)."""
     n = int(np.prod(wl.dst_shape()))
     dt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
-    buf = torch.empty(n + CANARY_ELEMS, dtype=dt, device="cuda")
+    buf = torch.empty(lead + n + CANARY_ELEMS, dtype=dt, device="cuda")
     s = sentinel(wl)
     int_view(buf).fill_(s - (1 << 16) if wl.dtype == "bf16" and s >= 1 << 15 else s)
-    return buf, buf[:n].view(wl.dst_shape())
+    return buf, buf[lead:lead + n].view(wl.dst_shape())
 
 
 def sentinel_value(wl):
@@ -50,7 +51,7 @@ def sentinel_value(wl):
 class Run:
     """One handle plus device inputs/outputs for a workload."""
 
-    def __init__(self, wl, sk, sv, blob, seq_lens=None, batch=None):
+    def __init__(self, wl, sk, sv, blob, seq_lens=None, batch=None, dst_lead=0):
         self.wl = wl
         self.h = M.mot_create(M.config_from(wl))
         M.mot_load_weights(self.h, blob)
@@ -60,17 +61,19 @@ class Run:
         self.batch = len(self.seq) if batch is None else batch
         self.lens = torch.tensor(self.seq + [0] * max(0, 1 - len(self.seq)), dtype=torch.int32,
                                  device="cuda")
-        self.buf_k, self.dk = alloc_dst(wl)
-        self.buf_v, self.dv = alloc_dst(wl)
+        self.lead = dst_lead
+        self.buf_k, self.dk = alloc_dst(wl, dst_lead)
+        self.buf_v, self.dv = alloc_dst(wl, dst_lead)
 
     def translate(self, stream=None):
         M.mot_translate(self.h, self.sk, self.sv, self.lens, self.batch, self.dk, self.dv, stream)
         return M.mot_get_device_status(self.h, stream)
 
     def canaries_intact(self):
-        n = self.dk.numel()
+        n, a = self.dk.numel(), self.lead
         s = sentinel_value(self.wl)
-        return bool((int_view(self.buf_k[n:]) == s).all() and (int_view(self.buf_v[n:]) == s).all())
+        return all(bool((int_view(b[a + n:]) == s).all()) and bool((int_view(b[:a]) == s).all())
+                   for b in (self.buf_k, self.buf_v))
 
     def padding_untouched(self, lens=None):
         """Every position that must keep its contents still holds the sentinel."""

@@ -298,6 +298,19 @@ def test_profile_and_launch_count(schedule, kernels):
     assert M.mot_get_launch_count(run.h) - n0 == sum(v[0] for v in stats.values())
 
 
+@pytest.mark.parametrize("lead", [8, 16])
+def test_target_cache_aligned_to_16_but_not_32_bytes(lead):
+    """The output stores take 32-byte vectors only where the target cache allows."""
+    wl = SMALL["umma_ragged"]
+    sk, sv, blob = inputs(wl, seed=12)
+    run = G.Run(wl, sk, sv, blob, dst_lead=lead)
+    assert run.dk.data_ptr() % 32 == (16 if lead == 8 else 0)
+    for schedule in (3, 2):
+        M.mot_set_schedule(run.h, schedule)
+        assert run.translate() == M.MOT_OK
+        full_check(wl, run, sk, sv, blob, f"lead {lead} schedule {schedule}")
+
+
 def test_onchip_schedule_is_refused_where_unsupported():
     """D_t != 256: the default stays 2 and asking for 3 is MOT_ERR_UNSUPPORTED."""
     wl = SMALL["umma_e1"]

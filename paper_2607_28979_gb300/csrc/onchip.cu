@@ -24,8 +24,8 @@
 // Roles per CTA:
 //   warp 0 lane 0 (both)    TMA loads of its Z rows and its halves of W1 / W2;
 //                           transaction bytes complete on the leader's barriers;
-//   warp 1 (leader)         MMA issue (one elected lane), in the order
-//                           G1(0) G1(1) | G1(j+2) G2(j) ... | bias;
+//   warp 1 (leader)         GEMM1 issue (one elected lane), up to two chunks ahead;
+//   warp 3 (leader)         GEMM2 and bias-MMA issue (one elected lane);
 //   warp 2 (both)           TMEM allocation of the pair;
 //   warps 4..19 (both)      epilogue: warp 4 + 4 p + q owns rows 32 q .. 32 q + 31; of
 //                           every chunk it evaluates columns 32 p .. 32 p + 31, and at the
@@ -73,7 +73,7 @@ struct Bars {
   uint64_t a2empty[2];  // GEMM2 of a chunk done reading its A2 (commit, both CTAs)
   uint64_t acc2full;    // a tile's GEMM2 + bias done (commit, both CTAs)
   uint64_t acc2empty;   // acc2 read out (leader; 2 x 16 warp arrivals)
-  uint64_t drain;
+  uint64_t drain, drain2;
   uint32_t tmem_slot;
   int abort_flag;
 };
@@ -182,6 +182,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     mbar_init(&bars->acc2full, 1);
     mbar_init(&bars->acc2empty, 2 * kEpiWarps);
     mbar_init(&bars->drain, 1);
+    mbar_init(&bars->drain2, 1);
     bars->abort_flag = 0;
     fence_barrier_init();
   }
@@ -304,27 +305,32 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (!ok) break;
       }
     }
-  } else if (warp == 1) {
-    if (leader) {
-      // ------------------------------------------------ MMA issuer (leader, whole warp)
-      // The loop, the waits and the descriptors are warp-uniform; one elected
-      // lane issues the MMAs and their commits.
+  } else if ((warp == 1 || warp == 3) && leader) {
+    // ------------------------------------------------ MMA issuers (leader)
+    // GEMM1 (warp 1) and GEMM2 + bias (warp 3) write different accumulators,
+    // so each has its own issuing warp: issuing costs tens of cycles per MMA,
+    // and one warp issuing both would serialise that with its waits. The
+    // loops, waits and descriptors are warp-uniform; one elected lane issues
+    // each warp's MMAs and commits (a commit tracks its own thread's MMAs).
+    auto wait_all = [&](uint64_t* bar, uint32_t parity) -> bool {
+      const bool r = mbar_wait(bar, parity, abort_flag, p.wait_limit);
+      return __all_sync(0xffffffffu, r) != 0;
+    };
+    uint32_t c0 = 0, k = 0;
+    bool ok = true;
+    if (warp == 1) {
       constexpr uint32_t idesc1 = idesc_bf16_f32(2 * UM, kChunk);
-      constexpr uint32_t idesc2 = idesc_f16_f32(2 * UM, UN);
-      auto wait_all = [&](uint64_t* bar, uint32_t parity) -> bool {
-        const bool r = mbar_wait(bar, parity, abort_flag, p.wait_limit);
-        return __all_sync(0xffffffffu, r) != 0;
-      };
-      uint32_t c0 = 0, k = 0;
-      bool ok = true;
-      for (int t = pair; ok && t < total; t += n_pairs, ++k) {
+      for (int t = pair; ok && t < total; t += n_pairs, ++k, c0 += nc) {
         const int zb = k & 1;
         if (!wait_all(&bars->zfull[zb], (k >> 1) & 1u)) break;
         tc_fence_after();
         const uint32_t zaddr = smem_u32(sZ + zb * kZBytes);
-        auto g1 = [&](int j) -> bool {
+        for (int j = 0; ok && j < nc; ++j) {
           const uint32_t c = c0 + j, b = c & 1u;
-          if (!wait_all(&bars->w1full[b], (c >> 1) & 1u)) return false;
+          // acc1[b] is free once the epilogue of chunk c - 2 has read it
+          if (c >= 2) ok = wait_all(&bars->acc1free[b], ((c >> 1) & 1u) ^ 1u);
+          ok = ok && wait_all(&bars->w1full[b], (c >> 1) & 1u);
+          if (!ok) break;
           tc_fence_after();
           const uint32_t waddr = smem_u32(sW1 + b * kW1Bytes);
           if (elect_one()) {
@@ -340,15 +346,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           }
           __syncwarp();
           mma_issued = true;
-          return true;
-        };
-        ok = g1(0) && (nc < 2 || g1(1));
+        }
+      }
+    } else {
+      constexpr uint32_t idesc2 = idesc_f16_f32(2 * UM, UN);
+      for (int t = pair; ok && t < total; t += n_pairs, ++k, c0 += nc) {
+        const int zb = k & 1;
         for (int j = 0; ok && j < nc; ++j) {
           const uint32_t c = c0 + j, b = c & 1u;
-          // GEMM1 two chunks ahead as soon as this chunk's acc1 is read out, so
-          // that its epilogue overlaps GEMM2 of this chunk
-          if (j + 2 < nc) ok = wait_all(&bars->acc1free[b], (c >> 1) & 1u) && g1(j + 2);
-          ok = ok && wait_all(&bars->a2full[b], (c >> 1) & 1u);
+          ok = wait_all(&bars->a2full[b], (c >> 1) & 1u);
           if (ok && j == 0) ok = wait_all(&bars->acc2empty, (k & 1u) ^ 1u);
           ok = ok && wait_all(&bars->w2full[b], (c >> 1) & 1u);
           if (!ok) break;
@@ -366,11 +372,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             umma_commit_pair(&bars->a2empty[b]);
           }
           __syncwarp();
+          mma_issued = true;
         }
         if (!ok) break;
-        // gate-weighted biases from the tile's Z buffer: A = gate16, B = b2t
+        // gate-weighted biases from the tile's Z buffer (loaded there once the
+        // tile's last GEMM1 is done): A = gate16, B = b2t
         if (!wait_all(&bars->bfull[zb], (k >> 1) & 1u)) break;
         tc_fence_after();
+        const uint32_t zaddr = smem_u32(sZ + zb * kZBytes);
         if (elect_one()) {
           const uint64_t gdesc = sdesc_k_sw128(zaddr + kBlk16);
           const uint64_t bdesc = sdesc_k_sw128(zaddr);
@@ -381,7 +390,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           umma_commit_pair(&bars->acc2full);
         }
         __syncwarp();
-        c0 += nc;
       }
     }
   } else if (warp >= 4) {
@@ -497,10 +505,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         spin_cycles(20000000LL);
       }
     }
-    if (warp == 1 && leader && mma_issued) {   // the lane that issued the MMAs commits
+    if ((warp == 1 || warp == 3) && leader && mma_issued) {   // each issuing lane drains its MMAs
       if (elect_one()) {
-        umma_commit_pair(&bars->drain);
-        const uint32_t a = smem_u32(&bars->drain);
+        uint64_t* dr = warp == 1 ? &bars->drain : &bars->drain2;
+        umma_commit_pair(dr);
+        const uint32_t a = smem_u32(dr);
         const long long t0 = clock64();
         while (!mbar_try_wait(a, 0) && clock64() - t0 < p.wait_limit) {
         }

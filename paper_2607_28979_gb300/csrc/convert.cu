@@ -36,7 +36,26 @@ __global__ void build_b2t_kernel(const float* b2, uint16_t* b2t, int G, int E, i
   }
 }
 
+// wg16[g][n][c] = wg[g][n][c] for n < E, 0 for E <= n < 16 (bf16 bits).
+__global__ void build_wg16_kernel(const uint16_t* wg, uint16_t* wg16, int G, int E, int Ds) {
+  const size_t n = size_t(G) * 16 * Ds;
+  for (size_t i = blockIdx.x * size_t(blockDim.x) + threadIdx.x; i < n;
+       i += size_t(gridDim.x) * blockDim.x) {
+    const int c = static_cast<int>(i % Ds);
+    const size_t gn = i / Ds;
+    const int r = static_cast<int>(gn % 16), g = static_cast<int>(gn / 16);
+    wg16[i] = r < E ? wg[(size_t(g) * E + r) * Ds + c] : uint16_t(0);
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_build_wg16(const void* wg, void* wg16, int G, int E, int Ds, cudaStream_t st) {
+  if (G == 0) return cudaSuccess;
+  build_wg16_kernel<<<1024, 256, 0, st>>>(static_cast<const uint16_t*>(wg),
+                                          static_cast<uint16_t*>(wg16), G, E, Ds);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_build_b2t(const float* b2, void* b2t, int G, int E, int Dt, cudaStream_t st) {
   if (G == 0) return cudaSuccess;

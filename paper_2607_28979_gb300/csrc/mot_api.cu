@@ -99,6 +99,7 @@ struct mot_ctx {
   float* gate = nullptr;
   void* gate16 = nullptr;   // fp16 gate rows padded to 64 (tensor-core path)
   void* b2t = nullptr;      // fp16 b2 transposed, padded to 64 (tensor-core path)
+  void* wg16 = nullptr;     // bf16 gate weights padded to 16 rows per group (tensor-core path)
   void* a2 = nullptr;
   TileInfo* tiles = nullptr;
   int32_t* n_tiles = nullptr;
@@ -106,7 +107,7 @@ struct mot_ctx {
   int32_t* counters = nullptr;   // fused schedule: item counter + per-tile completions
   // tensor maps that do not depend on the caller's buffers
   CUtensorMap tm_w1{}, tm_w2{}, tm_a2{}, tm_a2_st{}, tm_w1h{}, tm_w2h{}, tm_w1q{};
-  CUtensorMap tm_g16{}, tm_b2t{}, tm_b2th{};
+  CUtensorMap tm_g16{}, tm_b2t{}, tm_b2th{}, tm_wg16{};
   // host-buffer staging for mot_translate_host (allocated on first use)
   void* st_src[2] = {nullptr, nullptr};
   void* st_dst[2] = {nullptr, nullptr};
@@ -137,7 +138,7 @@ size_t group_elems(const Dims& d) {
 
 void free_all(mot_ctx* h) {
   void* ptrs[] = {h->wg, h->bg, h->w1, h->b1, h->b1h, h->w2, h->b2, h->groups, h->gate, h->gate16,
-                  h->b2t, h->a2, h->tiles,
+                  h->b2t, h->wg16, h->a2, h->tiles,
                   h->n_tiles, h->status, h->counters, h->st_src[0], h->st_src[1], h->st_dst[0],
                   h->st_dst[1], h->st_len};
   for (void* p : ptrs)
@@ -284,7 +285,10 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
     }));
   a.g0 = g_begin;
   a.gp = g_end - g_begin;
-  MOT_CUDA_TRY(timed(h, "gate", st, [&] { return launch_gate(a, st); }));
+  MOT_CUDA_TRY(timed(h, "gate", st, [&] {
+    return h->use_umma ? launch_gate_mma(a, tmK, tmV, h->tm_wg16, h->num_sms, st)
+                       : launch_gate(a, st);
+  }));
   if (h->use_umma && h->schedule == 3) {   // one launch; no A2 workspace, so no passes
     MOT_CUDA_TRY(timed(h, "umma2_onchip_translate", st, [&] {
       return launch_onchip(a, tmK, tmV, h->tm_w1q, h->tm_w2h, h->tm_g16, h->tm_b2th, h->num_sms,
@@ -460,6 +464,7 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       {(void**)&h->gate, G * size_t(d.tpad) * E * 4},
       {&h->gate16, h->use_umma ? G * size_t(d.tpad) * 64 * 2 : 16},
       {&h->b2t, h->use_umma ? G * size_t(d.Dt) * 64 * 2 : 16},
+      {&h->wg16, h->use_umma ? G * 16 * size_t(d.Ds) * 2 : 16},
       {&h->a2, size_t(h->gp_max) * per_group_a2},
       {(void**)&h->tiles, size_t(d.tiles_max) * sizeof(TileInfo)},
       {(void**)&h->n_tiles, 16}, {(void**)&h->status, 16},
@@ -514,6 +519,12 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       const uint64_t st_b[2] = {128, uint64_t(d.tpad) * 128};
       const uint32_t box[3] = {64, uint32_t(kTileM), 1};
       ok = ok && encode_bf16(&h->tm_g16, h->gate16, 3, dims, st_b, box, /*f16=*/true);
+    }
+    {  // wg16: [G * 16][Ds], box 64 x 16 (the gate MMA's B side)
+      const uint64_t dims[2] = {uint64_t(d.Ds), uint64_t(G) * 16};
+      const uint64_t st_b[1] = {uint64_t(d.Ds) * 2};
+      const uint32_t box[2] = {uint32_t(kUmmaK), 16};
+      ok = ok && encode_bf16(&h->tm_wg16, h->wg16, 2, dims, st_b, box);
     }
     {  // b2t: [G * Dt][64], boxes 64 x 256 and 64 x 128 (B side)
       const uint64_t dims[2] = {64, uint64_t(G * d.Dt)};
@@ -588,6 +599,7 @@ mot_status mot_load_weights(mot_handle h, const void* host_blob, size_t bytes) {
       MOT_CUDA_TRY(launch_bf16_to_f16_inplace(h->w2, size_t(d.G) * Dt * EH, 0));
       MOT_CUDA_TRY(launch_f32_to_f16(h->b1, h->b1h, b1.size(), 0));
       MOT_CUDA_TRY(launch_build_b2t(h->b2, h->b2t, d.G, d.E, d.Dt, 0));
+      MOT_CUDA_TRY(launch_build_wg16(h->wg, h->wg16, d.G, d.E, d.Ds, 0));
     }
   }
   MOT_CUDA_TRY(cudaDeviceSynchronize());

@@ -76,6 +76,7 @@ struct PathArgs {
 // Kernel launchers (each returns the launch's cudaError_t).
 cudaError_t launch_bf16_to_f16_inplace(void* buf, size_t n, cudaStream_t st);
 cudaError_t launch_build_b2t(const float* b2, void* b2t, int G, int E, int Dt, cudaStream_t st);
+cudaError_t launch_build_wg16(const void* wg, void* wg16, int G, int E, int Ds, cudaStream_t st);
 cudaError_t launch_f32_to_f16(const float* src, void* dst, size_t n, cudaStream_t st);
 cudaError_t launch_prep(const int32_t* seq_lens, int32_t batch, const Dims& d, TileInfo* tiles,
                         int32_t* n_tiles, int32_t* status, cudaStream_t st);
@@ -103,6 +104,12 @@ cudaError_t launch_umma2_gemm1(const PathArgs& a, const CUtensorMap& tmK, const 
 cudaError_t launch_umma2_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2h,
                                const CUtensorMap& tmG16, const CUtensorMap& tmB2th, int num_sms,
                                cudaStream_t st);
+
+// Gate on the tensor cores (gate_mma.cu): the source K/V load maps (box
+// 64 x 128) and a map over wg16 = [G * 16][D_s] bf16 (box 64 x 16), the gate
+// weights zero-padded to 16 rows per group.
+cudaError_t launch_gate_mma(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                            const CUtensorMap& tmWg, int num_sms, cudaStream_t st);
 
 // On-chip translation on CTA pairs for D_s <= 128, D_t = 256 (onchip.cu):
 // GEMM1, GELU * gate and GEMM2 in one persistent launch over all groups, the

@@ -356,21 +356,6 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint64_t* bar, uint32_t cta)
       : "memory");
 }
 
-// Named barrier `id` over `n` threads (a multiple of 32) that also returns the
-// AND of `v` over them, so that a decision taken after it is uniform.
-__device__ __forceinline__ bool bar_and(uint32_t id, uint32_t n, bool v) {
-  uint32_t r;
-  asm volatile(
-      "{\n\t.reg .pred p, q;\n\t"
-      "setp.ne.u32 q, %1, 0;\n\t"
-      "bar.red.and.pred p, %2, %3, q;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(r)
-      : "r"(static_cast<uint32_t>(v)), "r"(id), "r"(n)
-      : "memory");
-  return r != 0;
-}
-
 // True in exactly one lane of the (fully active) warp. Issuing tcgen05.mma
 // from a warp-uniform loop under elect.sync keeps its operands warp-uniform.
 __device__ __forceinline__ bool elect_one() {

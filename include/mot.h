@@ -232,6 +232,30 @@ mot_status mot_debug_set(mot_handle h, int32_t stall_test, int64_t wait_limit_cy
 /* Number of kernels this handle has launched since it was created. */
 mot_status mot_get_launch_count(mot_handle h, int64_t* count);
 
+/*
+ * Top-K routing (Def. 3.1 with 0 < top_k < E), tensor-core path.
+ *   1 (default where supported): token buckets. The tokens that chose
+ *      translator m are gathered per (layer, K/V) group and m's MLP runs on
+ *      them only (top_k / E of the dense MLP FLOPs); the top_k contributions
+ *      of a token are summed in a fixed order.
+ *   0: dense compute; every translator runs on every token, with the
+ *      unselected ones weighted by zero.
+ * Both give the translation of Def. 3.1 within rounding. Setting 1 on a
+ * handle without top_k < E, without the tensor-core path or with H not a
+ * multiple of 256 returns MOT_ERR_UNSUPPORTED.
+ */
+mot_status mot_set_routing(mot_handle h, int32_t routing);
+mot_status mot_get_routing(mot_handle h, int32_t* routing);
+
+/*
+ * Translator usage of the last routed translation (the counts I_e behind
+ * the usage metrics of Sec. 4.3): counts[g * E + m] = tokens of translated
+ * group g (2 r + x for the r-th translated target layer, x = 0 for K, 1 for
+ * V) that chose translator m. n must equal groups * E. Waits for `stream`.
+ * MOT_ERR_UNSUPPORTED unless the last translate ran with routing 1.
+ */
+mot_status mot_get_expert_counts(mot_handle h, int32_t* counts, int32_t n, mot_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -277,7 +277,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t tbase = tmem_base + static_cast<uint32_t>(acc * UN) +
                              (static_cast<uint32_t>(q * 32) << 16);
       if (it.type == 1) {
-        epilogue_gemm1(p, &tmS, tbase, tile, q, lane, gl, grp, m, it.n * UN, (e >> 2) * 128, 2,
+        epilogue_gemm1(p, &tmS, tbase, tile, q, lane, grp, it.n * UN, it.n * UN, m * UM, gl,
+                       (e >> 2) * 128, 2,
                        gemm1_prefetch(p, q, lane, grp, m, it.n * UN, (e >> 2) * 128));
         pending_f = it.f;
       } else {

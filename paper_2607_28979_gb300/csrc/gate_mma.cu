@@ -171,6 +171,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
       float g[kGN];
 #pragma unroll
       for (int e = 0; e < kGN; ++e) g[e] = 0.f;
+      uint32_t chosen = 0;   // the row's Top-K choices (sparse routing)
       if (r < ti.rows) {
         float mx = -INFINITY;
 #pragma unroll
@@ -209,9 +210,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
           const float kinv = 1.f / ks;
 #pragma unroll
           for (int e = 0; e < kGN; ++e) g[e] = (e < E && ((keep >> e) & 1u)) ? g[e] * kinv : 0.f;
+          chosen = keep;
         }
       }
       const size_t row = static_cast<size_t>(grp) * d.tpad + static_cast<size_t>(m) * UM + r;
+      if (p.sel) p.sel[row] = chosen;
       float* __restrict__ gout = p.gate + row * E;
 #pragma unroll
       for (int e = 0; e < kGN; ++e)

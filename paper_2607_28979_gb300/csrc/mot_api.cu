@@ -108,6 +108,14 @@ struct mot_ctx {
   // tensor maps that do not depend on the caller's buffers
   CUtensorMap tm_w1{}, tm_w2{}, tm_a2{}, tm_a2_st{}, tm_w1h{}, tm_w2h{}, tm_w1q{};
   CUtensorMap tm_g16{}, tm_b2t{}, tm_b2th{}, tm_wg16{};
+  // Top-K routing (tensor-core path, 0 < top_k < E): token buckets per expert
+  bool sparse_ok = false;   // the shapes support it
+  int routing = 0;          // 0 dense compute with a zeroed gate, 1 token buckets
+  int gp_sparse = 1;        // groups per routed pass
+  uint32_t* sel = nullptr;  // [G][tpad] Top-K choices per row
+  SparseArgs sp{};
+  bool counts_valid = false;
+  CUtensorMap tm_zp{}, tm_a2p{}, tm_a2p_st{}, tm_g16p{};
   // host-buffer staging for mot_translate_host (allocated on first use)
   void* st_src[2] = {nullptr, nullptr};
   void* st_dst[2] = {nullptr, nullptr};
@@ -138,7 +146,9 @@ size_t group_elems(const Dims& d) {
 
 void free_all(mot_ctx* h) {
   void* ptrs[] = {h->wg, h->bg, h->w1, h->b1, h->b1h, h->w2, h->b2, h->groups, h->gate, h->gate16,
-                  h->b2t, h->wg16, h->a2, h->tiles,
+                  h->b2t, h->wg16, h->a2, h->tiles, h->sel, h->sp.counts, h->sp.counts_all,
+                  h->sp.row0, h->sp.plan, h->sp.pairs, h->sp.ltok, h->sp.lslot, h->sp.gatep,
+                  h->sp.gate16p, h->sp.zp, h->sp.a2p, h->sp.ybuf,
                   h->n_tiles, h->status, h->counters, h->st_src[0], h->st_src[1], h->st_dst[0],
                   h->st_dst[1], h->st_len};
   for (void* p : ptrs)
@@ -285,10 +295,33 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
     }));
   a.g0 = g_begin;
   a.gp = g_end - g_begin;
+  const bool routed = h->use_umma && h->sparse_ok && h->routing == 1;
+  a.sel = routed ? h->sel : nullptr;
   MOT_CUDA_TRY(timed(h, "gate", st, [&] {
     return h->use_umma ? launch_gate_mma(a, tmK, tmV, h->tm_wg16, h->num_sms, st)
                        : launch_gate(a, st);
   }));
+  if (routed) {   // Top-K: per-expert token buckets, passes of gp_sparse groups
+    const SparseArgs& sp = h->sp;
+    for (int g0 = g_begin; g0 < g_end; g0 += h->gp_sparse) {
+      a.g0 = g0;
+      a.gp = std::min(h->gp_sparse, g_end - g0);
+      MOT_CUDA_TRY(timed(h, "route_count", st, [&] { return launch_route(a, sp, 0, st); }));
+      MOT_CUDA_TRY(timed(h, "route_plan", st, [&] { return launch_route(a, sp, 1, st); }));
+      MOT_CUDA_TRY(timed(h, "route_fill", st, [&] { return launch_route(a, sp, 2, st); }));
+      MOT_CUDA_TRY(timed(h, "pack", st, [&] { return launch_pack(a, sp, st); }));
+      MOT_CUDA_TRY(timed(h, "umma2_sparse_gemm1", st, [&] {
+        return launch_umma2_sparse_gemm1(a, sp, h->tm_zp, h->tm_w1h, h->tm_a2p_st, h->num_sms, st);
+      }));
+      MOT_CUDA_TRY(timed(h, "umma2_sparse_gemm2", st, [&] {
+        return launch_umma2_sparse_gemm2(a, sp, h->tm_a2p, h->tm_w2h, h->tm_g16p, h->tm_b2th,
+                                         h->num_sms, st);
+      }));
+      MOT_CUDA_TRY(timed(h, "combine", st, [&] { return launch_combine(a, sp, st); }));
+    }
+    h->counts_valid = true;
+    return MOT_OK;
+  }
   if (h->use_umma && h->schedule == 3) {   // one launch; no A2 workspace, so no passes
     MOT_CUDA_TRY(timed(h, "umma2_onchip_translate", st, [&] {
       return launch_onchip(a, tmK, tmV, h->tm_w1q, h->tm_w2h, h->tm_g16, h->tm_b2th, h->num_sms,
@@ -456,7 +489,35 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
     const int passes = (d.G + h->gp_max - 1) / h->gp_max;
     h->gp_max = (d.G + passes - 1) / passes;
   }
+  // Top-K routing workspace: per group, K * tpad routed rows plus each bucket's
+  // padding to whole pair tiles (under 256 rows per bucket)
+  h->sparse_ok = h->use_umma && d.top_k > 0 && d.top_k < d.E && d.H % kUmmaN == 0 && G > 0;
+  h->routing = h->sparse_ok ? 1 : 0;
+  size_t sp_rows_g = 0, sp_pairs_g = 0;
+  if (h->sparse_ok) {
+    const size_t K = d.top_k;
+    sp_rows_g = K * d.tpad + E * 2 * kTileM;
+    sp_pairs_g = (K * d.tpad + 2 * kTileM - 1) / (2 * kTileM) + E;
+    const size_t per_g = sp_rows_g * (size_t(d.Ds) * 2 + size_t(d.H) * 2 + 64 * 2 + 12) +
+                         size_t(d.tpad) * K * d.Dt * 4;
+    h->gp_sparse = static_cast<int>(std::max<size_t>(1, std::min<size_t>(G, kA2Budget / per_g)));
+    const int passes = (d.G + h->gp_sparse - 1) / h->gp_sparse;
+    h->gp_sparse = (d.G + passes - 1) / passes;
+    h->sp.R = static_cast<int32_t>(sp_rows_g * h->gp_sparse);
+    h->sp.max_pairs = static_cast<int32_t>(sp_pairs_g * h->gp_sparse);
+  }
+  const size_t spR = h->sparse_ok ? size_t(h->sp.R) : 1, spGP = h->sparse_ok ? h->gp_sparse : 1;
   struct A { void** p; size_t n; } allocs[] = {
+      {(void**)&h->sel, h->sparse_ok ? G * size_t(d.tpad) * 4 : 16},
+      {(void**)&h->sp.counts, spGP * E * 4}, {(void**)&h->sp.counts_all, G * E * 4},
+      {(void**)&h->sp.row0, spGP * E * 4}, {(void**)&h->sp.plan, 16},
+      {(void**)&h->sp.pairs, h->sparse_ok ? size_t(h->sp.max_pairs) * sizeof(SparsePair) : 16},
+      {(void**)&h->sp.ltok, spR * 4}, {(void**)&h->sp.lslot, spR * 4},
+      {(void**)&h->sp.gatep, spR * 4}, {&h->sp.gate16p, spR * 64 * 2},
+      {&h->sp.zp, h->sparse_ok ? spR * d.Ds * 2 : 16},
+      {&h->sp.a2p, h->sparse_ok ? spR * d.H * 2 : 16},
+      {(void**)&h->sp.ybuf,
+       h->sparse_ok ? spGP * d.tpad * size_t(d.top_k) * d.Dt * 4 : 16},
       {&h->wg, G * E * d.Ds * es}, {(void**)&h->bg, G * E * 4},
       {&h->w1, G * EH * d.Ds * es}, {(void**)&h->b1, G * EH * 4}, {&h->b1h, G * EH * 2},
       {&h->w2, G * d.Dt * EH * es}, {(void**)&h->b2, G * E * d.Dt * 4},
@@ -519,6 +580,23 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       const uint64_t st_b[2] = {128, uint64_t(d.tpad) * 128};
       const uint32_t box[3] = {64, uint32_t(kTileM), 1};
       ok = ok && encode_bf16(&h->tm_g16, h->gate16, 3, dims, st_b, box, /*f16=*/true);
+    }
+    if (h->sparse_ok) {   // routed rows: zp [H_s * R][d_s], A2p [1][R][H], gate16p [1][R][64]
+      const uint64_t R = uint64_t(h->sp.R);
+      const uint64_t zd[2] = {uint64_t(d.d_s), uint64_t(d.H_s) * R};
+      const uint64_t zs[1] = {uint64_t(d.d_s) * 2};
+      const uint32_t zb[2] = {uint32_t(kUmmaK), uint32_t(kTileM)};
+      ok = ok && encode_bf16(&h->tm_zp, h->sp.zp, 2, zd, zs, zb);
+      const uint64_t ad[3] = {uint64_t(d.H), R, 1};
+      const uint64_t as[2] = {uint64_t(d.H) * 2, R * d.H * 2};
+      const uint32_t ab[3] = {uint32_t(kUmmaK), uint32_t(kTileM), 1}, ab_st[3] = {32, 32, 1};
+      ok = ok && encode_bf16(&h->tm_a2p, h->sp.a2p, 3, ad, as, ab, /*f16=*/true);
+      ok = ok && encode_bf16(&h->tm_a2p_st, h->sp.a2p, 3, ad, as, ab_st, /*f16=*/true,
+                             /*swizzle64=*/true);
+      const uint64_t gd[3] = {64, R, 1};
+      const uint64_t gs[2] = {128, R * 128};
+      const uint32_t gb[3] = {64, uint32_t(kTileM), 1};
+      ok = ok && encode_bf16(&h->tm_g16p, h->sp.gate16p, 3, gd, gs, gb, /*f16=*/true);
     }
     {  // wg16: [G * 16][Ds], box 64 x 16 (the gate MMA's B side)
       const uint64_t dims[2] = {uint64_t(d.Ds), uint64_t(G) * 16};
@@ -805,6 +883,33 @@ mot_status mot_profile_read(mot_handle h, mot_kernel_stat* out, int32_t cap, int
 mot_status mot_get_launch_count(mot_handle h, int64_t* count) {
   if (!h || !count) return MOT_ERR_INVALID_ARG;
   *count = h->launches;
+  return MOT_OK;
+}
+
+mot_status mot_set_routing(mot_handle h, int32_t routing) {
+  if (!h || routing < 0 || routing > 1) return MOT_ERR_INVALID_ARG;
+  if (routing == 1 && !h->sparse_ok) return MOT_ERR_UNSUPPORTED;
+  h->routing = routing;
+  return MOT_OK;
+}
+
+mot_status mot_get_routing(mot_handle h, int32_t* routing) {
+  if (!h || !routing) return MOT_ERR_INVALID_ARG;
+  *routing = h->routing;
+  return MOT_OK;
+}
+
+mot_status mot_get_expert_counts(mot_handle h, int32_t* counts, int32_t n, mot_stream_t stream) {
+  if (!h || !counts || n != h->d.G * h->d.E) return MOT_ERR_INVALID_ARG;
+  if (!(h->sparse_ok && h->routing == 1 && h->counts_valid)) return MOT_ERR_UNSUPPORTED;
+  if (cudaSetDevice(h->device) != cudaSuccess) return MOT_ERR_CUDA;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(counts, h->sp.counts_all, size_t(n) * 4, cudaMemcpyDeviceToHost, st) !=
+          cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess) {
+    cudaGetLastError();
+    return MOT_ERR_CUDA;
+  }
   return MOT_OK;
 }
 

@@ -68,9 +68,38 @@ struct PathArgs {
   const void* b2t;   // fp16 [G][D_t][64]: b2 transposed, zero-padded (tensor-core path)
   void* a2;
   int32_t* status;
+  uint32_t* sel;          // [G][tpad] Top-K selection bits per row (sparse routing), else null
   int32_t g0, gp;         // groups [g0, g0 + gp) of this pass
   long long wait_limit;   // bound of every pipeline wait, in SM cycles
   int32_t stall_test;     // test hook (single-SM GEMM1): CTA 0 withholds its first stage
+};
+
+// Top-K routing (0 < top_k < E) on the tensor-core path (sparse.cu): for each
+// (group, expert) bucket of a pass the tokens that selected the expert are
+// gathered into a packed row space, each bucket padded to whole pairs of
+// 128-row tiles, and the translators run on their own tokens only. GEMM2
+// writes each (token, slot) row in fp32; the combine sums a token's top_k
+// slots in slot order (slot = rank of the expert among the token's choices).
+struct SparsePair {       // one 256-row pair tile of one bucket
+  int32_t vg;             // bucket: local group * E + expert
+  int32_t p0;             // packed row of its first 128-row tile
+  int32_t rows0, rows1;   // valid rows of its two tiles
+};
+struct SparseArgs {
+  int32_t* counts;        // [gp * E] tokens per bucket (this pass)
+  int32_t* counts_all;    // [G * E] tokens per bucket of the last translation
+  int32_t* row0;          // [gp * E] first packed row of each bucket
+  int32_t* plan;          // [2]: number of pairs, packed rows in use
+  SparsePair* pairs;      // [max_pairs]
+  int32_t* ltok;          // [R] token row (index into the tpad rows), -1 for padding
+  int32_t* lslot;         // [R] slot of the row's expert among the token's choices
+  float* gatep;           // [R] gtilde of the row's expert
+  void* gate16p;          // [R][64] fp16: gtilde in the bucket's expert column, else 0
+  void* zp;               // [H_s][R][d_s] packed source rows (dtype)
+  void* a2p;              // [R][H] fp16 hidden activations
+  float* ybuf;            // [gp][tpad][top_k][D_t] per-slot translator outputs
+  int32_t R;              // packed-row capacity of a pass
+  int32_t max_pairs;
 };
 
 // Kernel launchers (each returns the launch's cudaError_t).
@@ -110,6 +139,22 @@ cudaError_t launch_umma2_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const
 // weights zero-padded to 16 rows per group.
 cudaError_t launch_gate_mma(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
                             const CUtensorMap& tmWg, int num_sms, cudaStream_t st);
+
+// Sparse routing launchers (sparse.cu); the GEMMs are the pair kernels of
+// umma2.cu over the packed rows: GEMM1 reads the zp map (box 64 x 128 over
+// [H_s * R][d_s]) and stores A2p through a 32 x 32 x 1 box over [1][R][H];
+// GEMM2 reads A2p (box 64 x 128 x 1) and gate16p (box 64 x 128 x 1 over [1][R][64]).
+// step 0: bucket sizes; 1: packed layout and pair-tile list; 2: bucket rows.
+cudaError_t launch_route(const PathArgs& a, const SparseArgs& s, int step, cudaStream_t st);
+cudaError_t launch_pack(const PathArgs& a, const SparseArgs& s, cudaStream_t st);
+cudaError_t launch_combine(const PathArgs& a, const SparseArgs& s, cudaStream_t st);
+cudaError_t launch_umma2_sparse_gemm1(const PathArgs& a, const SparseArgs& s,
+                                      const CUtensorMap& tmZp, const CUtensorMap& tmW1h,
+                                      const CUtensorMap& tmA2pst, int num_sms, cudaStream_t st);
+cudaError_t launch_umma2_sparse_gemm2(const PathArgs& a, const SparseArgs& s,
+                                      const CUtensorMap& tmA2p, const CUtensorMap& tmW2h,
+                                      const CUtensorMap& tmG16p, const CUtensorMap& tmB2th,
+                                      int num_sms, cudaStream_t st);
 
 // On-chip translation on CTA pairs for D_s <= 128, D_t = 256 (onchip.cu):
 // GEMM1, GELU * gate and GEMM2 in one persistent launch over all groups, the

@@ -211,8 +211,8 @@ __global__ void __launch_bounds__(threads_of(MODE), 1)
       const uint32_t tbase = tmem_base + static_cast<uint32_t>(acc * UN) +
                              (static_cast<uint32_t>(q * 32) << 16);
       if (MODE == 1)   // 8 warps: this warp owns columns 128 * (e / 4) .. +127
-        epilogue_gemm1(p, &tmS, tbase, sOut + e * kStoreTileBytes, q, lane, gl, grp, m, n * UN,
-                       (e >> 2) * 128, 2,
+        epilogue_gemm1(p, &tmS, tbase, sOut + e * kStoreTileBytes, q, lane, grp, n * UN, n * UN,
+                       m * UM, gl, (e >> 2) * 128, 2,
                        gemm1_prefetch(p, q, lane, grp, m, n * UN, (e >> 2) * 128));
       else             // 4 warps: all 256 columns
         epilogue_gemm2(p, tbase, q, lane, grp, m, n * UN, 0, UN / 32);

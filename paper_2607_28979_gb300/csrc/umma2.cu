@@ -41,10 +41,47 @@ static_assert(smem_bytes2(1) <= 232448 && smem_bytes2(2) <= 232448, "shared memo
 
 struct Umma2Args {
   PathArgs p;
+  SparseArgs sp;      // sparse routing: the packed rows and their pair-tile list
   int32_t nk;         // K blocks per tile
-  int32_t n_tiles_n;  // 256-column tiles per group
+  int32_t n_tiles_n;  // 256-column tiles per group (per expert when sparse)
   int32_t b_rows;     // rows of B per group (E*H for GEMM1, D_t for GEMM2)
 };
+
+// One work item: a pair tile and a 256-column tile n. Dense: token tiles
+// 2 mp and 2 mp + 1 of group grp; sparse: a pair tile of bucket (group, expert
+// em) at packed rows p_own (this CTA's half). `live` = this CTA's tile has rows.
+struct Work {
+  int gl, grp, m_own, n, em, p_own, rows_own;
+  bool live;
+};
+
+// Sparse GEMM2 epilogue of one warp: row 32 q + lane of the pair tile's half
+// at packed row p_own; its fp32 result goes to the token's slot row.
+__device__ __forceinline__ void epilogue_gemm2_sparse(const PathArgs& p, const SparseArgs& sp,
+                                                      uint32_t tbase, int q, int lane, int gl,
+                                                      int p_own, int rows_own, int n0) {
+  const Dims& d = p.d;
+  const int r = q * 32 + lane;
+  const bool valid = r < rows_own;
+  float* out = nullptr;
+  if (valid) {
+    const int tok = sp.ltok[p_own + r], slot = sp.lslot[p_own + r];
+    out = sp.ybuf + ((static_cast<size_t>(gl) * d.tpad + tok) * d.top_k + slot) * d.Dt + n0;
+  }
+#pragma unroll 1
+  for (int ch = 0; ch < UN / 32; ++ch) {
+    uint32_t v[32];
+    tmem_ld_32x32b_x32(tbase + ch * 32, v);
+    tmem_ld_wait(v);
+    if (valid) {
+      float4* o4 = reinterpret_cast<float4*>(out + ch * 32);
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        o4[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                            __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+    }
+  }
+}
 
 // Spin about `cycles` SM cycles (used only while unwinding after a timeout).
 __device__ __forceinline__ void spin_cycles(long long cycles) {
@@ -53,7 +90,10 @@ __device__ __forceinline__ void spin_cycles(long long cycles) {
   }
 }
 
-template <int MODE>   // 1 = GEMM1 (A = source cache), 2 = GEMM2 (A = A2)
+// MODE 1 = GEMM1 (A = source cache, or the packed rows when SPARSE), 2 = GEMM2
+// (A = A2). SPARSE: work items come from the routing's pair-tile list and B is
+// the bucket expert's slice of W1cat / W2cat.
+template <int MODE, bool SPARSE>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
     umma2_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
                       const __grid_constant__ CUtensorMap tmA1,
@@ -110,8 +150,35 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
   const int n_m = min(*p.n_tiles, d.tiles_max);
   const int n_mp = (n_m + 1) / 2;
   const int per_grp = n_mp * ua.n_tiles_n;
-  const int total = p.gp * per_grp;
+  const int total = SPARSE ? ua.sp.plan[0] * ua.n_tiles_n : p.gp * per_grp;
   const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+  auto decode = [&](int t) {
+    Work w;
+    if (SPARSE) {
+      const int pe = t / ua.n_tiles_n;
+      w.n = t - pe * ua.n_tiles_n;
+      const SparsePair sp = ua.sp.pairs[pe];
+      w.gl = sp.vg / d.E;
+      w.em = sp.vg - w.gl * d.E;
+      w.grp = p.g0 + w.gl;
+      w.m_own = 0;
+      w.p_own = sp.p0 + static_cast<int>(rank) * UM;
+      w.rows_own = rank ? sp.rows1 : sp.rows0;
+      w.live = w.rows_own > 0;
+    } else {
+      w.gl = t / per_grp;
+      const int rem = t - w.gl * per_grp;
+      const int mp = rem / ua.n_tiles_n;
+      w.n = rem - mp * ua.n_tiles_n;
+      w.grp = p.g0 + w.gl;
+      w.m_own = 2 * mp + static_cast<int>(rank);
+      w.em = 0;
+      w.p_own = 0;
+      w.rows_own = 0;
+      w.live = w.m_own < n_m;
+    }
+    return w;
+  };
 
   uint32_t issued_mask = 0, issue_parity = 0;
   bool mma_issued = false;
@@ -122,13 +189,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
       int stage = 0;
       uint32_t phase = 0;
       for (int t = pair; t < total; t += n_pairs) {
-        const int gl = t / per_grp, rem = t - gl * per_grp;
-        const int mp = rem / ua.n_tiles_n, n = rem - mp * ua.n_tiles_n;
-        const int grp = p.g0 + gl;
-        const int m_own = 2 * mp + static_cast<int>(rank);
+        const Work w = decode(t);
+        const int gl = w.gl, n = w.n, grp = w.grp, m_own = w.m_own;
         TileInfo ti;
         GroupInfo gi;
-        if (MODE == 1) {
+        if (MODE == 1 && !SPARSE) {
           gi = p.groups[grp];
           if (m_own < n_m) {
             ti = p.tiles[m_own];
@@ -142,17 +207,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, p.wait_limit)) { ok = false; break; }
           if (leader) mbar_arrive_expect_tx(&full[stage], 2 * kStageBytes2);
           const uint32_t bar = leader_addr(&full[stage]);
-          const int b_row = grp * ua.b_rows + n * UN + static_cast<int>(rank) * (UN / 2);
-          if (MODE == 1) {
+          const int b_row = grp * ua.b_rows + (MODE == 1 ? w.em * d.H : 0) + n * UN +
+                            static_cast<int>(rank) * (UN / 2);
+          if (MODE == 1 && SPARSE) {   // packed rows: [H_s][R][d_s]
+            const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
+            tma_load_2d_pair(sA + stage * kABytes2, &tmA0, bar, d0, h * ua.sp.R + w.p_own);
+            tma_load_2d_pair(sB + stage * kBBytes2, &tmB, bar, kb * UK, b_row);
+          } else if (MODE == 1) {
             const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
             tma_load_2d_pair(sA + stage * kABytes2, gi.x ? &tmA1 : &tmA0, bar, d0,
                              ((gi.src_layer * d.B + ti.b) * d.H_s + h) * d.S + ti.s0);
             tma_load_2d_pair(sB + stage * kBBytes2, &tmB, bar, kb * UK, b_row);
-          } else if (kb < ua.nk - 1) {   // A2 x W2cat
-            tma_load_3d_pair(sA + stage * kABytes2, &tmA0, bar, kb * UK, m_own * UM, gl);
-            tma_load_2d_pair(sB + stage * kBBytes2, &tmB, bar, kb * UK, b_row);
+          } else if (kb < ua.nk - 1) {   // A2 x W2cat (sparse: the expert's K range of W2cat)
+            if (SPARSE)
+              tma_load_3d_pair(sA + stage * kABytes2, &tmA0, bar, kb * UK, w.p_own, 0);
+            else
+              tma_load_3d_pair(sA + stage * kABytes2, &tmA0, bar, kb * UK, m_own * UM, gl);
+            tma_load_2d_pair(sB + stage * kBBytes2, &tmB, bar, w.em * d.H + kb * UK, b_row);
           } else {                       // last K block: gate16 x b2t (the combine biases)
-            tma_load_3d_pair(sA + stage * kABytes2, &tmA1, bar, 0, m_own * UM, grp);
+            if (SPARSE)
+              tma_load_3d_pair(sA + stage * kABytes2, &tmA1, bar, 0, w.p_own, 0);
+            else
+              tma_load_3d_pair(sA + stage * kABytes2, &tmA1, bar, 0, m_own * UM, grp);
             tma_load_2d_pair(sB + stage * kBBytes2, &tmS, bar, 0, b_row);
           }
           issued_mask |= 1u << stage;
@@ -207,14 +283,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
       m_own = 2 * mp + static_cast<int>(rank);
     };
     float gate_next = 0.f;
-    if (MODE == 1 && pair < total) {
+    if (MODE == 1 && !SPARSE && pair < total) {
       int gl, grp, m_own, n;
       tile_coords(pair, gl, grp, m_own, n);
       if (m_own < n_m) gate_next = gemm1_prefetch(p, q, lane, grp, m_own, n * UN, (e >> 2) * 128);
     }
     for (int t = pair; t < total; t += n_pairs) {
       const float gate_cur = gate_next;
-      if (MODE == 1 && t + n_pairs < total) {
+      if (MODE == 1 && !SPARSE && t + n_pairs < total) {
         int gl, grp, m_own, n;
         tile_coords(t + n_pairs, gl, grp, m_own, n);
         if (m_own < n_m) gate_next = gemm1_prefetch(p, q, lane, grp, m_own, n * UN, (e >> 2) * 128);
@@ -224,16 +300,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
-      const int gl = t / per_grp, rem = t - gl * per_grp;
-      const int mp = rem / ua.n_tiles_n, n = rem - mp * ua.n_tiles_n;
-      const int grp = p.g0 + gl;
-      const int m_own = 2 * mp + static_cast<int>(rank);
+      const Work w = decode(t);
+      const int gl = w.gl, n = w.n, grp = w.grp, m_own = w.m_own;
       const uint32_t tbase = tmem_base + static_cast<uint32_t>(acc * UN) +
                              (static_cast<uint32_t>(q * 32) << 16);
-      if (m_own < n_m) {
-        if (MODE == 1)   // 8 warps: this warp owns columns 128 * (e / 4) .. +127
-          epilogue_gemm1(p, &tmS, tbase, sOut + e * kStoreTileBytes, q, lane, gl, grp, m_own,
-                         n * UN, (e >> 2) * 128, 2, gate_cur);
+      if (w.live) {
+        if (MODE == 1 && SPARSE)   // bias of expert em; A2 rows are the packed rows
+          epilogue_gemm1(p, &tmS, tbase, sOut + e * kStoreTileBytes, q, lane, grp,
+                         w.em * d.H + n * UN, n * UN, w.p_own, 0, (e >> 2) * 128, 2,
+                         ua.sp.gatep[w.p_own + q * 32 + lane]);
+        else if (MODE == 1)   // 8 warps: this warp owns columns 128 * (e / 4) .. +127
+          epilogue_gemm1(p, &tmS, tbase, sOut + e * kStoreTileBytes, q, lane, grp, n * UN,
+                         n * UN, m_own * UM, gl, (e >> 2) * 128, 2, gate_cur);
+        else if (SPARSE)
+          epilogue_gemm2_sparse(p, ua.sp, tbase, q, lane, gl, w.p_own, w.rows_own, n * UN);
         else             // 4 warps: all 256 columns
           epilogue_gemm2(p, tbase, q, lane, grp, m_own, n * UN, 0, UN / 32);
       }
@@ -284,28 +364,32 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
   if (threadIdx.x == 0 && *abort_flag) atomicOr(p.status, kStatusTimeout);
 }
 
-template <int MODE>
-cudaError_t launch_umma2(const PathArgs& a, const CUtensorMap& A0, const CUtensorMap& A1,
-                         const CUtensorMap& B, const CUtensorMap& S, int nk, int n_tiles_n,
-                         int b_rows, int num_sms, cudaStream_t st) {
+template <int MODE, bool SPARSE>
+cudaError_t launch_umma2(const PathArgs& a, const SparseArgs* sp, const CUtensorMap& A0,
+                         const CUtensorMap& A1, const CUtensorMap& B, const CUtensorMap& S, int nk,
+                         int n_tiles_n, int b_rows, int num_sms, cudaStream_t st) {
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(umma2_gemm_kernel<MODE>,
+    cudaError_t e = cudaFuncSetAttribute(umma2_gemm_kernel<MODE, SPARSE>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          smem_bytes2(MODE));
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  Umma2Args ua;
+  Umma2Args ua{};
   ua.p = a;
+  if (sp) ua.sp = *sp;
   ua.nk = nk;
   ua.n_tiles_n = n_tiles_n;
   ua.b_rows = b_rows;
-  const long long pairs = static_cast<long long>(a.gp) * ((a.d.tiles_max + 1) / 2) * n_tiles_n;
+  const long long pairs =
+      static_cast<long long>(SPARSE ? sp->max_pairs : a.gp * ((a.d.tiles_max + 1) / 2)) *
+      n_tiles_n;
   const long long max_pairs = num_sms / 2;
   const int grid = 2 * static_cast<int>(pairs < max_pairs ? pairs : max_pairs);
   if (grid <= 0) return cudaSuccess;
-  umma2_gemm_kernel<MODE><<<grid, threads2(MODE), smem_bytes2(MODE), st>>>(A0, A1, B, S, ua);
+  umma2_gemm_kernel<MODE, SPARSE>
+      <<<grid, threads2(MODE), smem_bytes2(MODE), st>>>(A0, A1, B, S, ua);
   return cudaGetLastError();
 }
 
@@ -314,15 +398,35 @@ cudaError_t launch_umma2(const PathArgs& a, const CUtensorMap& A0, const CUtenso
 cudaError_t launch_umma2_gemm1(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
                                const CUtensorMap& tmW1h, const CUtensorMap& tmA2st, int num_sms,
                                cudaStream_t st) {
-  return launch_umma2<1>(a, tmK, tmV, tmW1h, tmA2st, a.d.Ds / UK, a.d.EH / UN, a.d.EH, num_sms, st);
+  return launch_umma2<1, false>(a, nullptr, tmK, tmV, tmW1h, tmA2st, a.d.Ds / UK, a.d.EH / UN,
+                                a.d.EH, num_sms, st);
+}
+
+// Sparse GEMM1: A = packed rows (zp), B = the bucket expert's H rows of W1cat,
+// stores A2p rows; n runs over the expert's H / 256 column tiles.
+cudaError_t launch_umma2_sparse_gemm1(const PathArgs& a, const SparseArgs& s,
+                                      const CUtensorMap& tmZp, const CUtensorMap& tmW1h,
+                                      const CUtensorMap& tmA2pst, int num_sms, cudaStream_t st) {
+  return launch_umma2<1, true>(a, &s, tmZp, tmZp, tmW1h, tmA2pst, a.d.Ds / UK, a.d.H / UN, a.d.EH,
+                               num_sms, st);
+}
+
+// Sparse GEMM2: A = A2p rows (K = H) and gate16p for the bias block, B = the
+// expert's K range of W2cat and b2t; fp32 slot rows into ybuf.
+cudaError_t launch_umma2_sparse_gemm2(const PathArgs& a, const SparseArgs& s,
+                                      const CUtensorMap& tmA2p, const CUtensorMap& tmW2h,
+                                      const CUtensorMap& tmG16p, const CUtensorMap& tmB2th,
+                                      int num_sms, cudaStream_t st) {
+  return launch_umma2<2, true>(a, &s, tmA2p, tmG16p, tmW2h, tmB2th, a.d.H / UK + 1, a.d.Dt / UN,
+                               a.d.Dt, num_sms, st);
 }
 
 // GEMM2's map slots: A0 = A2, A1 = gate16, B = W2cat half, S = b2t half (last K block).
 cudaError_t launch_umma2_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const CUtensorMap& tmW2h,
                                const CUtensorMap& tmG16, const CUtensorMap& tmB2th, int num_sms,
                                cudaStream_t st) {
-  return launch_umma2<2>(a, tmA2, tmG16, tmW2h, tmB2th, a.d.EH / UK + 1, a.d.Dt / UN, a.d.Dt,
-                         num_sms, st);
+  return launch_umma2<2, false>(a, nullptr, tmA2, tmG16, tmW2h, tmB2th, a.d.EH / UK + 1,
+                                a.d.Dt / UN, a.d.Dt, num_sms, st);
 }
 
 }  // namespace mot

@@ -95,14 +95,18 @@ __device__ __forceinline__ float gemm1_prefetch(const PathArgs& p, int q, int la
   return g;
 }
 
+// `bias_col` is the tile's first column in the group's E*H biases; the store
+// map's coordinates of the tile are (st_x, st_y, st_z) = (first column, first
+// row, group slot) of the A2 layout in use.
 __device__ __forceinline__ void epilogue_gemm1(const PathArgs& p, const CUtensorMap* tmS,
                                                uint32_t tbase, uint8_t* tile, int q, int lane,
-                                               int gl, int grp, int m, int n0, int col_begin,
-                                               int n_chunks, float gate) {
+                                               int grp, int bias_col, int st_x, int st_y,
+                                               int st_z, int col_begin, int n_chunks,
+                                               float gate) {
   const Dims& d = p.d;
   const __half2 half_g = __float2half2_rn(0.5f * gate);
   const __half* __restrict__ bias =
-      static_cast<const __half*>(p.b1h) + static_cast<size_t>(grp) * d.EH + n0;
+      static_cast<const __half*>(p.b1h) + static_cast<size_t>(grp) * d.EH + bias_col;
   const uint32_t tile_addr = smem_u32(tile);
   const int n_sub = 2 * n_chunks;
   uint32_t ra[32], rb[32];
@@ -137,7 +141,7 @@ __device__ __forceinline__ void epilogue_gemm1(const PathArgs& p, const CUtensor
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) {
-        tma_store_3d(tmS, tile + half * 2048, n0 + col0, m * UM + q * 32, gl);
+        tma_store_3d(tmS, tile + half * 2048, st_x + col0, st_y + q * 32, st_z);
         bulk_commit_group();
       }
     }

@@ -68,6 +68,9 @@ _SIGS = {
     "mot_profile_read": [_H, ctypes.POINTER(mot_kernel_stat), ctypes.c_int32,
                          ctypes.POINTER(ctypes.c_int32)],
     "mot_get_launch_count": [_H, ctypes.POINTER(ctypes.c_int64)],
+    "mot_set_routing": [_H, ctypes.c_int32],
+    "mot_get_routing": [_H, ctypes.POINTER(ctypes.c_int32)],
+    "mot_get_expert_counts": [_H, _P, ctypes.c_int32, _P],
     "mot_debug_set": [_H, ctypes.c_int32, ctypes.c_int64],
     "mot_translate_static": [ctypes.POINTER(mot_config), _P, _P, _P, _P, ctypes.c_int32, _P, _P,
                              _P],
@@ -256,3 +259,39 @@ def mot_get_launch_count(h: Handle) -> int:
     c = ctypes.c_int64()
     _check(_lib.mot_get_launch_count(h.ptr, ctypes.byref(c)), "mot_get_launch_count")
     return c.value
+
+
+ROUTING_DENSE, ROUTING_SPARSE = 0, 1
+
+
+def mot_set_routing(h: Handle, routing: int) -> None:
+    _check(_lib.mot_set_routing(h.ptr, int(routing)), "mot_set_routing")
+
+
+def mot_get_routing(h: Handle) -> int:
+    v = ctypes.c_int32()
+    _check(_lib.mot_get_routing(h.ptr, ctypes.byref(v)), "mot_get_routing")
+    return v.value
+
+
+def mot_get_expert_counts(h: Handle, n_groups: int, n_translators: int, stream=None):
+    """Tokens routed to each translator of each (layer, K/V) group by the last
+    translation: an int32 array [n_groups][n_translators]."""
+    import numpy as np
+    out = np.zeros((n_groups, n_translators), dtype=np.int32)
+    _check(_lib.mot_get_expert_counts(h.ptr, out.ctypes.data, out.size, _stream(stream)),
+           "mot_get_expert_counts")
+    return out
+
+
+def expert_usage(counts):
+    """Translator usage statistics over selection counts I_e (Sec. 4.3): the
+    squared coefficient of variation Var(I) / Mean(I)^2 and the entropy
+    -sum p_e log p_e of p_e = I_e / sum I. Returns (cv2, entropy) as floats."""
+    import numpy as np
+    c = np.asarray(counts, dtype=np.float64).ravel()
+    mean = c.mean()
+    cv2 = float(c.var() / (mean * mean)) if mean > 0 else 0.0
+    tot = c.sum()
+    p = c[c > 0] / tot if tot > 0 else c[:0]
+    return cv2, float(-(p * np.log(p)).sum())

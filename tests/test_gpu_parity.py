@@ -365,6 +365,127 @@ def test_topk_routing_against_oracle(name):
     G.assert_parity(wl, got[tl][keep[tl]], ref[tl][keep[tl]], name)
 
 
+# ---------------------------------------------------------------- Top-K routing with token buckets
+
+TOPK_ROUTED = {
+    # two 256-column tiles per expert (H = 512) and per output (D_t = 512), D_s = 256,
+    # ragged lengths (odd bucket sizes: padded pair tiles), an untranslated target layer
+    "routed_top2_of4": synth.Workload("routed_top2_of4", 3, 4, 64, 3, 4, 128, 4, 512, 3, 300,
+                                      "bf16", (300, 129, 7), top_k=2, layer_map=(2, -1, 0)),
+    # Top-1 of 8 on the on-chip shapes (D_s = 128, D_t = 256)
+    "routed_top1_of8": synth.Workload("routed_top1_of8", 2, 2, 64, 2, 2, 128, 8, 256, 2, 400,
+                                      "bf16", (400, 250), top_k=1),
+}
+ROUTED_ALL = {**{k: v for k, v in TOPK.items() if k.startswith("umma")}, **TOPK_ROUTED}
+
+
+def _all_tokens(wl):
+    tb = np.concatenate([np.full(L, b) for b, L in enumerate(wl.seq_lens)]).astype(np.int32)
+    ts = np.concatenate([np.arange(L) for L in wl.seq_lens]).astype(np.int32)
+    return tb, ts
+
+
+def _clear_choice(wl, sk, sv, blob, tb, ts):
+    """Tokens whose K-th and (K+1)-th dense gate scores differ by at least 1e-4
+    (fp32 and fp64 then keep the same translators)."""
+    _, dense = oracle.translate_tokens(wl.replace(top_k=0), sk, sv, blob, tb, ts, want_gate=True)
+    srt = -np.sort(-dense, axis=-1)
+    return srt[..., wl.top_k - 1] - srt[..., wl.top_k] >= 1e-4
+
+
+@pytest.mark.parametrize("name", sorted(ROUTED_ALL))
+def test_routed_and_dense_topk_both_match_the_oracle(name):
+    """Token buckets (the default) and dense compute give the same translation."""
+    wl = ROUTED_ALL[name]
+    sk, sv, blob = inputs(wl, seed=13)
+    tb, ts = _all_tokens(wl)
+    ref = oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
+    ok = _clear_choice(wl, sk, sv, blob, tb, ts)
+    tl = wl.translated_layers()
+    assert ok[tl].mean() > 0.99
+    outs = {}
+    for routing in (1, 0):
+        run = G.Run(wl, sk, sv, blob)
+        assert M.mot_get_routing(run.h) == M.ROUTING_SPARSE
+        M.mot_set_routing(run.h, routing)
+        assert run.translate() == M.MOT_OK
+        assert run.canaries_intact() and run.padding_untouched()
+        got = run.gather(tb, ts)
+        keep = np.broadcast_to(ok[..., None], got.shape)
+        G.assert_parity(wl, got[tl][keep[tl]], ref[tl][keep[tl]], f"{name} routing {routing}")
+        outs[routing] = got
+    keep = np.broadcast_to(ok[..., None], outs[0].shape)
+    diff = np.abs(outs[0] - outs[1])[tl][keep[tl]]
+    assert diff.max() <= 2.0 ** -5   # fp32 summation order and one bf16 rounding apart
+
+
+def test_expert_counts_match_the_oracle_choices():
+    """mot_get_expert_counts: tokens per translator per group, as the fp64 gate
+    chooses them (up to tokens at a near tie); usage statistics from them."""
+    wl = TOPK_ROUTED["routed_top2_of4"]
+    sk, sv, blob = inputs(wl, seed=14)
+    run = G.Run(wl, sk, sv, blob)
+    groups = 2 * len(wl.translated_layers())
+    with pytest.raises(M.MotError) as e:   # nothing routed yet
+        M.mot_get_expert_counts(run.h, groups, wl.n_translators)
+    assert e.value.status == M.MOT_ERR_UNSUPPORTED
+    assert run.translate() == M.MOT_OK
+    counts = M.mot_get_expert_counts(run.h, groups, wl.n_translators)
+    tb, ts = _all_tokens(wl)
+    _, gate = oracle.translate_tokens(wl, sk, sv, blob, tb, ts, want_gate=True)
+    ok = _clear_choice(wl, sk, sv, blob, tb, ts)
+    n_tok = tb.size
+    for r, l in enumerate(wl.translated_layers()):
+        for x in (0, 1):
+            g = 2 * r + x
+            chosen = gate[l, x] > 0                       # [n][E]
+            assert (chosen.sum(axis=1) == wl.top_k).all()
+            ref = chosen.sum(axis=0)
+            ties = int((~ok[l, x]).sum())
+            assert counts[g].sum() == wl.top_k * n_tok
+            assert np.abs(counts[g] - ref).max() <= ties, (g, counts[g], ref, ties)
+    cv2, ent = M.expert_usage(counts)
+    c = counts.astype(np.float64).ravel()
+    assert cv2 == pytest.approx(c.var() / c.mean() ** 2)
+    assert 0.0 < ent <= np.log(c.size) + 1e-12
+
+
+def test_routing_switch_and_counter_errors():
+    wl = SMALL["umma_ragged"]   # dense gate: no buckets to route
+    sk, sv, blob = inputs(wl, seed=15)
+    run = G.Run(wl, sk, sv, blob)
+    assert M.mot_get_routing(run.h) == M.ROUTING_DENSE
+    for bad, status in ((1, M.MOT_ERR_UNSUPPORTED), (2, M.MOT_ERR_INVALID_ARG),
+                        (-1, M.MOT_ERR_INVALID_ARG)):
+        with pytest.raises(M.MotError) as e:
+            M.mot_set_routing(run.h, bad)
+        assert e.value.status == status
+    assert run.translate() == M.MOT_OK
+    with pytest.raises(M.MotError) as e:
+        M.mot_get_expert_counts(run.h, 2 * len(wl.translated_layers()), wl.n_translators)
+    assert e.value.status == M.MOT_ERR_UNSUPPORTED
+    wl2 = TOPK_ROUTED["routed_top1_of8"]
+    sk2, sv2, blob2 = inputs(wl2, seed=15)
+    run2 = G.Run(wl2, sk2, sv2, blob2)
+    assert run2.translate() == M.MOT_OK
+    with pytest.raises(M.MotError) as e:   # wrong element count
+        M.mot_get_expert_counts(run2.h, 1, 3)
+    assert e.value.status == M.MOT_ERR_INVALID_ARG
+
+
+def test_routed_profile_and_launch_count():
+    wl = TOPK_ROUTED["routed_top2_of4"]
+    sk, sv, blob = inputs(wl, seed=16)
+    run = G.Run(wl, sk, sv, blob)
+    n0 = M.mot_get_launch_count(run.h)
+    M.mot_profile_enable(run.h, True)
+    assert run.translate() == M.MOT_OK
+    stats = M.mot_profile_read(run.h)
+    assert set(stats) == {"prep_tiles", "gate", "route_count", "route_plan", "route_fill", "pack",
+                          "umma2_sparse_gemm1", "umma2_sparse_gemm2", "combine"}
+    assert M.mot_get_launch_count(run.h) - n0 == sum(v[0] for v in stats.values())
+
+
 # ---------------------------------------------------------------- failure detection
 
 def test_bounded_wait_reports_timeout_and_the_context_survives():

@@ -43,9 +43,11 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 
 
 def workload_desc(wl) -> str:
+    gate = ("dense softmax gate" if wl.top_k in (0, wl.n_translators)
+            else f"softmax gate, Top-{wl.top_k} routing")
     return (f"{wl.name}: {wl.n_layers_src}L {wl.src_kv_heads}x{wl.src_head_dim} -> "
             f"{wl.n_layers_tgt}L {wl.tgt_kv_heads}x{wl.tgt_head_dim}, E={wl.n_translators} MLP "
-            f"{wl.d_src}-{wl.hidden}-{wl.d_tgt} GELU, dense softmax gate, {wl.dtype}, "
+            f"{wl.d_src}-{wl.hidden}-{wl.d_tgt} GELU, {gate}, {wl.dtype}, "
             f"batch {wl.batch} seq_lens {list(wl.seq_lens)}")
 
 
@@ -56,8 +58,10 @@ def algorithmic(wl, layer_map):
     n_tl = len(wl.translated_layers())
     groups = 2 * n_tl
     f_gate = 2 * Ds * E
-    f_g1 = E * 2 * Ds * Hh
-    f_g2 = E * 2 * Hh * Dt + 2 * E * Dt
+    # with Top-K routing only the top_k chosen translators run on a token
+    Ea = wl.top_k if 0 < wl.top_k < E else E
+    f_g1 = Ea * 2 * Ds * Hh
+    f_g2 = Ea * 2 * Hh * Dt + 2 * Ea * Dt
     src_layers = {s for s in layer_map if s >= 0}
     es = wl.esize
     bytes_src = 2 * len(src_layers) * T * Ds * es
@@ -293,6 +297,8 @@ def run_mot(args, wl):
     if args.schedule != "auto":
         M.mot_set_schedule(h, {v: k for k, v in names.items()}[args.schedule])
     schedule = names[M.mot_get_schedule(h)]
+    if M.mot_get_routing(h) == M.ROUTING_SPARSE:
+        schedule = "routed (Top-K token buckets)"
     bf = wl.dtype == "bf16"
     tdt = torch.bfloat16 if bf else torch.float32
 
@@ -383,6 +389,8 @@ def run_mot(args, wl):
                             "umma2_onchip_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
                             "umma2_gemm1_gelu_gate": alg["flops_gemm1"],
                             "umma2_gemm2_combine_store": alg["flops_gemm2"],
+                            "umma2_sparse_gemm1": alg["flops_gemm1"],
+                            "umma2_sparse_gemm2": alg["flops_gemm2"],
                             "umma_gemm1_gelu_gate": alg["flops_gemm1"],
                             "simt_gemm1_gelu_gate": alg["flops_gemm1"],
                             "umma_gemm2_combine_store": alg["flops_gemm2"],
@@ -452,12 +460,17 @@ def main():
                     help="tcgen05 launch schedule: the library's default for the shape, the "
                          "on-chip GEMM1-GELU-GEMM2 kernel (D_s <= 128, D_t = 256), GEMMs on CTA "
                          "pairs (2-SM MMA), one fused persistent launch, or GEMMs on single SMs")
+    ap.add_argument("--top-k", type=int, default=0,
+                    help="route each token to its top-k translators (0: the workload's gate); "
+                         "with 0 < k < E the translators run on token buckets")
     ap.add_argument("--n-layers", type=int, default=0,
                     help="keep only the first N layers of both models (smaller profiling case)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mot":
         args.warmup = 3
     wl = synth.WORKLOADS[args.workload]
+    if args.top_k > 0:
+        wl = wl.replace(name=f"{wl.name}_top{args.top_k}", top_k=args.top_k)
     if args.n_layers > 0:
         wl = wl.replace(name=f"{wl.name}_L{args.n_layers}",
                         n_layers_src=min(args.n_layers, wl.n_layers_src),

@@ -317,7 +317,8 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
         return launch_umma2_sparse_gemm2(a, sp, h->tm_a2p, h->tm_w2h, h->tm_g16p, h->tm_b2th,
                                          h->num_sms, st);
       }));
-      MOT_CUDA_TRY(timed(h, "combine", st, [&] { return launch_combine(a, sp, st); }));
+      if (d.top_k > 1)   // top_k = 1: GEMM2 stored the target rows
+        MOT_CUDA_TRY(timed(h, "combine", st, [&] { return launch_combine(a, sp, st); }));
     }
     h->counts_valid = true;
     return MOT_OK;
@@ -499,7 +500,7 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
     sp_rows_g = K * d.tpad + E * 2 * kTileM;
     sp_pairs_g = (K * d.tpad + 2 * kTileM - 1) / (2 * kTileM) + E;
     const size_t per_g = sp_rows_g * (size_t(d.Ds) * 2 + size_t(d.H) * 2 + 64 * 2 + 12) +
-                         size_t(d.tpad) * K * d.Dt * 4;
+                         (K > 1 ? size_t(d.tpad) * K * d.Dt * 4 : 0);
     h->gp_sparse = static_cast<int>(std::max<size_t>(1, std::min<size_t>(G, kA2Budget / per_g)));
     const int passes = (d.G + h->gp_sparse - 1) / h->gp_sparse;
     h->gp_sparse = (d.G + passes - 1) / passes;
@@ -517,7 +518,7 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       {&h->sp.zp, h->sparse_ok ? spR * d.Ds * 2 : 16},
       {&h->sp.a2p, h->sparse_ok ? spR * d.H * 2 : 16},
       {(void**)&h->sp.ybuf,
-       h->sparse_ok ? spGP * d.tpad * size_t(d.top_k) * d.Dt * 4 : 16},
+       h->sparse_ok && d.top_k > 1 ? spGP * d.tpad * size_t(d.top_k) * d.Dt * 4 : 16},
       {&h->wg, G * E * d.Ds * es}, {(void**)&h->bg, G * E * 4},
       {&h->w1, G * EH * d.Ds * es}, {(void**)&h->b1, G * EH * 4}, {&h->b1h, G * EH * 2},
       {&h->w2, G * d.Dt * EH * es}, {(void**)&h->b2, G * E * d.Dt * 4},

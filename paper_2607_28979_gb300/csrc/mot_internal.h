@@ -97,7 +97,8 @@ struct SparseArgs {
   void* gate16p;          // [R][64] fp16: gtilde in the bucket's expert column, else 0
   void* zp;               // [H_s][R][d_s] packed source rows (dtype)
   void* a2p;              // [R][H] fp16 hidden activations
-  float* ybuf;            // [gp][tpad][top_k][D_t] per-slot translator outputs
+  float* ybuf;            // [gp][tpad][top_k][D_t] per-slot outputs (top_k > 1; top_k = 1
+                          // stores the target rows from GEMM2)
   int32_t R;              // packed-row capacity of a pass
   int32_t max_pairs;
 };

@@ -63,17 +63,35 @@ __device__ __forceinline__ void epilogue_gemm2_sparse(const PathArgs& p, const S
   const Dims& d = p.d;
   const int r = q * 32 + lane;
   const bool valid = r < rows_own;
-  float* out = nullptr;
+  float* out = nullptr;              // top_k > 1: the token's slot row (fp32)
+  __nv_bfloat16* tgt = nullptr;      // top_k = 1: the target cache row, head 0
   if (valid) {
     const int tok = sp.ltok[p_own + r], slot = sp.lslot[p_own + r];
-    out = sp.ybuf + ((static_cast<size_t>(gl) * d.tpad + tok) * d.top_k + slot) * d.Dt + n0;
+    if (d.top_k == 1) {
+      const GroupInfo gi = p.groups[p.g0 + gl];
+      const TileInfo ti = p.tiles[tok / UM];
+      tgt = static_cast<__nv_bfloat16*>(p.dst[gi.x]) +
+            ((static_cast<size_t>(gi.tgt_layer) * d.B + ti.b) * d.H_t * d.S + ti.s0 + tok % UM) *
+                d.d_t;
+    } else {
+      out = sp.ybuf + ((static_cast<size_t>(gl) * d.tpad + tok) * d.top_k + slot) * d.Dt + n0;
+    }
   }
 #pragma unroll 1
   for (int ch = 0; ch < UN / 32; ++ch) {
     uint32_t v[32];
     tmem_ld_32x32b_x32(tbase + ch * 32, v);
     tmem_ld_wait(v);
-    if (valid) {
+    if (valid && tgt) {   // channel c of head c / d_t, d_t a multiple of 32
+      const int c = n0 + ch * 32, h = c / d.d_t, i0 = c - h * d.d_t;
+      uint4* o4 = reinterpret_cast<uint4*>(tgt + static_cast<size_t>(h) * d.S * d.d_t + i0);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        o4[j] = make_uint4(pack_bf16x2(__uint_as_float(v[8 * j + 0]), __uint_as_float(v[8 * j + 1])),
+                           pack_bf16x2(__uint_as_float(v[8 * j + 2]), __uint_as_float(v[8 * j + 3])),
+                           pack_bf16x2(__uint_as_float(v[8 * j + 4]), __uint_as_float(v[8 * j + 5])),
+                           pack_bf16x2(__uint_as_float(v[8 * j + 6]), __uint_as_float(v[8 * j + 7])));
+    } else if (valid) {
       float4* o4 = reinterpret_cast<float4*>(out + ch * 32);
 #pragma unroll
       for (int j = 0; j < 8; ++j)

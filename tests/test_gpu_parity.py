@@ -483,6 +483,12 @@ def test_routed_profile_and_launch_count():
     stats = M.mot_profile_read(run.h)
     assert set(stats) == {"prep_tiles", "gate", "route_count", "route_plan", "route_fill", "pack",
                           "umma2_sparse_gemm1", "umma2_sparse_gemm2", "combine"}
+    wl1 = TOPK_ROUTED["routed_top1_of8"]   # Top-1: GEMM2 stores the target rows, no combine
+    sk1, sv1, blob1 = inputs(wl1, seed=16)
+    run1 = G.Run(wl1, sk1, sv1, blob1)
+    M.mot_profile_enable(run1.h, True)
+    assert run1.translate() == M.MOT_OK
+    assert "combine" not in M.mot_profile_read(run1.h)
     assert M.mot_get_launch_count(run.h) - n0 == sum(v[0] for v in stats.values())
 
 

@@ -94,3 +94,28 @@ def test_valid_config_without_gpu_is_a_cuda_error():
     with pytest.raises(M.MotError) as e:
         M.mot_create(M.make_config(**GOOD))
     assert e.value.status == M.MOT_ERR_CUDA
+
+
+def test_expert_usage_statistics_closed_forms():
+    """CV^2 = Var(I) / Mean(I)^2 and entropy -sum p log p of p = I / sum I (Sec. 4.3)."""
+    import math
+    cv2, ent = M.expert_usage([10, 10])          # balanced: no spread, log 2 nats
+    assert cv2 == 0.0 and ent == pytest.approx(math.log(2), abs=1e-15)
+    cv2, ent = M.expert_usage([20, 0])           # collapsed onto one translator
+    assert cv2 == pytest.approx(1.0) and ent == 0.0
+    cv2, ent = M.expert_usage([[6, 2], [1, 1]])  # counts of several groups pool
+    c = [6, 2, 1, 1]
+    mean = sum(c) / 4
+    var = sum((x - mean) ** 2 for x in c) / 4
+    assert cv2 == pytest.approx(var / mean ** 2)
+    assert ent == pytest.approx(-sum(x / 10 * math.log(x / 10) for x in c))
+    assert M.expert_usage([0, 0]) == (0.0, 0.0)
+
+
+def test_routing_calls_reject_null_handles():
+    import numpy as np
+    assert M._lib.mot_set_routing(None, 1) == M.MOT_ERR_INVALID_ARG
+    v = ctypes.c_int32()
+    assert M._lib.mot_get_routing(None, ctypes.byref(v)) == M.MOT_ERR_INVALID_ARG
+    buf = np.zeros(4, dtype=np.int32)
+    assert M._lib.mot_get_expert_counts(None, buf.ctypes.data, 4, None) == M.MOT_ERR_INVALID_ARG

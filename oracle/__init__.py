@@ -56,6 +56,9 @@ def _load():
         lib.oracle_translate_tokens.restype = ctypes.c_int
         lib.oracle_translate_tokens.argtypes = [ctypes.POINTER(OracleDims), P, P, P, P,
                                                 ctypes.c_int64, P, P, P, P, P]
+        lib.oracle_translate_h_tokens.restype = ctypes.c_int
+        lib.oracle_translate_h_tokens.argtypes = [ctypes.POINTER(OracleDims), ctypes.c_int32, P,
+                                                  P, P, ctypes.c_int64, P, P, P, P, P]
         lib.oracle_translate_full.restype = ctypes.c_int
         lib.oracle_translate_full.argtypes = [ctypes.POINTER(OracleDims), P, P, P, P,
                                               ctypes.c_int32, P, P, P]
@@ -119,6 +122,27 @@ def translate_tokens(wl, src_k, src_v, blob, tok_b, tok_s, gate_fixed=None, want
     if rc != 0:
         raise ValueError("oracle_translate_tokens: invalid arguments")
     return (out, gate) if want_gate else out
+
+
+def translate_h_tokens(wl, src_act, blob, tok_b, tok_s, want_act=False):
+    """MoT-h (App. C.5) for sampled tokens: the translated activation restored
+    through the target's projections. Returns (K, V), each [L_t][n][D_t] (NaN
+    for untranslated layers), and with ``want_act`` the activation [L_t][n][d_at]."""
+    assert wl.is_h and wl.src_kv_heads == 1
+    tb = np.ascontiguousarray(tok_b, dtype=np.int32)
+    ts = np.ascontiguousarray(tok_s, dtype=np.int32)
+    n = tb.size
+    ok = np.full((wl.n_layers_tgt, n, wl.d_tgt), np.nan, dtype=np.float64)
+    ov = np.full_like(ok, np.nan)
+    act = np.full((wl.n_layers_tgt, n, wl.act_tgt), np.nan) if want_act else None
+    rc = _load().oracle_translate_h_tokens(ctypes.byref(dims_of(wl)), wl.act_tgt,
+                                           _ptr(_map_arr(wl.layer_map)),
+                                           _ptr(np.ascontiguousarray(src_act)),
+                                           _ptr(np.ascontiguousarray(blob)), n, _ptr(tb), _ptr(ts),
+                                           _ptr(ok), _ptr(ov), _ptr(act))
+    if rc != 0:
+        raise ValueError("oracle_translate_h_tokens: invalid arguments")
+    return (ok, ov, act) if want_act else (ok, ov)
 
 
 def translate_full(wl, src_k, src_v, blob, seq_lens, fill=np.nan):

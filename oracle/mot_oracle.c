@@ -40,7 +40,9 @@
  * permutation translators built from GELU(x) - GELU(-x) = x; one-hot gate
  * (proof of Prop. 3.1); gate and Top-K closed forms; E = 1 against a library
  * MLP; linearity in the gate; expert-permutation invariance; brute force on
- * tiny inputs. No function here is unpinned.
+ * tiny inputs. MoT-h (below): the identity mixture with permutation and scaled
+ * projections in closed form, linearity in W^K / W^V, and the mixture part
+ * against the KV entry point on the same weights. No function here is unpinned.
  */
 #include <math.h>
 #include <stdint.h>
@@ -299,4 +301,82 @@ int oracle_translate_full(const oracle_dims* d, const int32_t* layer_map,
   }
   free(map); free(tb); free(ts); free(rows);
   return rc;
+}
+
+/*
+ * MoT-h (App. C.5): the translated representation is the intermediate
+ * activation entering the target's attention, not K and V. For each
+ * translated target layer l and token:
+ *   a       = a_src[pi(l)][b][s][:] (width d_as; the source activation,
+ *             passed like a one-head cache: d->H_s = 1, d->d_s = d_as);
+ *   a_hat   = sum over kept m of gtilde_m Tr_m(a), the same gated mixture as
+ *             above with output width d_at (Def. 3.1);
+ *   K, V    = W^K a_hat, W^V a_hat, the target layer's own key and value
+ *             projections [D_t][d_at] (App. C.5 writes the restoration as these
+ *             plain products: no bias, no positional re-encoding).
+ * Weight blob per translated target layer ascending: the mixture block (as a
+ * KV group block with D_t replaced by d_at), then W^K, then W^V.
+ * out_k, out_v: [L_t][n_tok][D_t] (c = h*d_t + i); act_out (optional):
+ * [L_t][n_tok][d_at]. Rows of untranslated layers are left untouched.
+ * Returns 0, or -1 on invalid arguments.
+ */
+int oracle_translate_h_tokens(const oracle_dims* d, int32_t act_tgt, const int32_t* layer_map,
+                              const void* src_act, const void* blob, int64_t n_tok,
+                              const int32_t* tok_b, const int32_t* tok_s, double* out_k,
+                              double* out_v, double* act_out) {
+  if (check_dims(d) || d->H_s != 1 || act_tgt <= 0 || !src_act || !blob || !out_k || !out_v ||
+      n_tok < 0)
+    return -1;
+  if (n_tok > 0 && (!tok_b || !tok_s)) return -1;
+  for (int64_t t = 0; t < n_tok; ++t)
+    if (tok_b[t] < 0 || tok_b[t] >= d->B || tok_s[t] < 0 || tok_s[t] >= d->S) return -1;
+  int32_t* map = resolve_map(d, layer_map);
+  if (!map) return -1;
+  oracle_dims md = *d;   /* the mixture: one head of width d_at out */
+  md.H_t = 1;
+  md.d_t = act_tgt;
+  const int64_t Da = act_tgt, Ds = d->d_s, Dt = (int64_t)d->H_t * d->d_t, E = d->E;
+  const int64_t mix = group_elems(&md), block = mix + 2 * Dt * Da;
+  const int64_t esz = d->dtype == 0 ? 2 : 4;
+  int64_t r = 0;
+  for (int l = 0; l < d->L_t; ++l) {
+    if (map[l] < 0) continue;
+    const int sl = map[l];
+    const char* w = (const char*)blob + r * block * esz;
+#pragma omp parallel
+    {
+      int64_t mx = Ds > d->H ? Ds : d->H;
+      if (Da > mx) mx = Da;
+      double* z = (double*)malloc(sizeof(double) * Ds);
+      double* row = (double*)malloc(sizeof(double) * mx);
+      double* h = (double*)malloc(sizeof(double) * d->H);
+      double* ym = (double*)malloc(sizeof(double) * Da);
+      double* ah = (double*)malloc(sizeof(double) * Da);
+      double g[64], logit[64];
+#pragma omp for schedule(dynamic, 1)
+      for (int64_t t = 0; t < n_tok; ++t) {
+        const int b = tok_b[t], s = tok_s[t];
+        const int64_t zi = (((int64_t)sl * d->B + b) * d->S + s) * Ds;
+        ld_row(src_act, d->dtype, zi, Ds, z);
+        translate_one(&md, w, z, NULL, ah, g, logit, row, h, ym);
+        double* ok = out_k + ((int64_t)l * n_tok + t) * Dt;
+        double* ov = out_v + ((int64_t)l * n_tok + t) * Dt;
+        for (int64_t i = 0; i < Dt; ++i) {
+          ld_row(w, d->dtype, mix + i * Da, Da, row);
+          ok[i] = dot(row, ah, Da);
+          ld_row(w, d->dtype, mix + Dt * Da + i * Da, Da, row);
+          ov[i] = dot(row, ah, Da);
+        }
+        if (act_out) {
+          double* oa = act_out + ((int64_t)l * n_tok + t) * Da;
+          for (int64_t i = 0; i < Da; ++i) oa[i] = ah[i];
+        }
+      }
+      free(z); free(row); free(h); free(ym); free(ah);
+    }
+    ++r;
+  }
+  free(map);
+  (void)E;
+  return 0;
 }

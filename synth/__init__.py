@@ -32,7 +32,7 @@ _SRC = os.path.join(_HERE, "synth.c")
 _LIB = os.path.join(_HERE, "libsynth.so")
 
 # Blob tensor ids, in blob order within one (target layer, K/V) group.
-T_WG, T_BG, T_W1, T_B1, T_W2, T_B2 = range(6)
+T_WG, T_BG, T_W1, T_B1, T_W2, T_B2, T_WK, T_WV = range(8)
 
 
 def build(force: bool = False) -> str:
@@ -87,6 +87,11 @@ class Workload:
     seq_lens: Tuple[int, ...]
     top_k: int = 0                  # 0 (or E) = dense softmax gate
     layer_map: Optional[Tuple[int, ...]] = None   # None = depth-ratio default; -1 = untranslated
+    # MoT-h (App. C.5): > 0 = the target activation width d_at. The source tensor is
+    # then the activation [L_s][B][S][d_as], stored as a one-head cache
+    # (src_kv_heads = 1, src_head_dim = d_as); the target caches are restored
+    # through per-layer projections W^K, W^V [D_t][d_at].
+    act_tgt: int = 0
 
     @property
     def d_src(self) -> int:
@@ -124,13 +129,24 @@ class Workload:
     def dst_shape(self):
         return (self.n_layers_tgt, self.max_batch, self.tgt_kv_heads, self.max_seq, self.tgt_head_dim)
 
+    @property
+    def is_h(self) -> bool:
+        return self.act_tgt > 0
+
+    @property
+    def d_mix(self) -> int:
+        """Output width of the translator mixture: D_t, or d_at for MoT-h."""
+        return self.act_tgt if self.is_h else self.d_tgt
+
     def group_elems(self) -> int:
-        """Elements of one (target layer, K/V) block of the weight blob."""
-        E, Ds, Dt, H = self.n_translators, self.d_src, self.d_tgt, self.hidden
-        return E * Ds + E + E * (H * Ds + H + Dt * H + Dt)
+        """Elements of one block of the weight blob: a (target layer, K/V) group,
+        or for MoT-h a target layer (mixture, then W^K and W^V)."""
+        E, Ds, Dm, H = self.n_translators, self.d_src, self.d_mix, self.hidden
+        n = E * Ds + E + E * (H * Ds + H + Dm * H + Dm)
+        return n + (2 * self.d_tgt * self.act_tgt if self.is_h else 0)
 
     def blob_elems(self) -> int:
-        return 2 * len(self.translated_layers()) * self.group_elems()
+        return (1 if self.is_h else 2) * len(self.translated_layers()) * self.group_elems()
 
     def replace(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)
@@ -153,6 +169,18 @@ WORKLOADS = {
     "qwen7_long": Workload("qwen7_long", 28, 4, 128, 28, 4, 128, 4, 2048, 4, 32768, "bf16",
                            (32768, 16384, 8192, 4096)),
 }
+
+# MoT-h (App. C.5) counterparts of two of the model pairs: the source activation
+# is the model width (d_model) of the source model, the translated activation
+# the target model's, and K, V are restored through the target's projections.
+WORKLOADS.update({
+    # GPT-2-small (768) -> OPT-125m (768; KV 12x64), 12 layers each, E=4, MLP 768->1536->768.
+    "h_gpt2s_opt125m": Workload("h_gpt2s_opt125m", 12, 1, 768, 12, 12, 64, 4, 1536, 8, 1024,
+                                "bf16", (1024,) * 8, act_tgt=768),
+    # Qwen2.5-0.5B (896, 24L) -> Qwen2.5-1.5B (1536, 28L; KV 2x128), E=4, MLP 896->1024->1536.
+    "h_qwen05_qwen15": Workload("h_qwen05_qwen15", 24, 1, 896, 28, 2, 128, 4, 1024, 4, 4096,
+                                "bf16", (4096,) * 4, act_tgt=1536),
+})
 
 # Order in which the workloads are listed in the build's benchmark configuration.
 WORKLOAD_ORDER = ["tiny_fp32", "gpt2s_opt125m", "qwen05_qwen15", "gpt2m_qwen7", "qwen7_long"]
@@ -182,17 +210,20 @@ def gen_cache(wl: Workload, x: int, seed: int = 0) -> np.ndarray:
 
 def blob_offsets(wl: Workload):
     """Yield (target layer, x, tensor id, expert, offset, numel, fan_in) for every blob tensor."""
-    E, Ds, Dt, H = wl.n_translators, wl.d_src, wl.d_tgt, wl.hidden
+    E, Ds, Dt, H, Dm = wl.n_translators, wl.d_src, wl.d_tgt, wl.hidden, wl.d_mix
     off = 0
     for l in wl.translated_layers():
-        for x in (0, 1):
+        for x in ((0,) if wl.is_h else (0, 1)):
             yield (l, x, T_WG, 0, off, E * Ds, Ds); off += E * Ds
             yield (l, x, T_BG, 0, off, E, Ds); off += E
             for m in range(E):
                 yield (l, x, T_W1, m, off, H * Ds, Ds); off += H * Ds
                 yield (l, x, T_B1, m, off, H, Ds); off += H
-                yield (l, x, T_W2, m, off, Dt * H, H); off += Dt * H
-                yield (l, x, T_B2, m, off, Dt, H); off += Dt
+                yield (l, x, T_W2, m, off, Dm * H, H); off += Dm * H
+                yield (l, x, T_B2, m, off, Dm, H); off += Dm
+            if wl.is_h:   # the target's key and value projections of layer l
+                yield (l, x, T_WK, 0, off, Dt * Dm, Dm); off += Dt * Dm
+                yield (l, x, T_WV, 0, off, Dt * Dm, Dm); off += Dt * Dm
 
 
 def gen_weights(wl: Workload, seed: int = 0) -> np.ndarray:

@@ -233,6 +233,40 @@ mot_status mot_debug_set(mot_handle h, int32_t stall_test, int64_t wait_limit_cy
 mot_status mot_get_launch_count(mot_handle h, int64_t* count);
 
 /*
+ * MoT-h (App. C.5): translate the source model's intermediate activation (the
+ * input of its attention) instead of K and V, and restore the target cache
+ * with the target layer's own projections: for each translated target layer
+ * l, with a = src_act[pi(l)][b][s][:],
+ *   a_hat = sum_m gtilde_m Tr_m(a)        (the gated mixture above, width d_at),
+ *   K = W^K_l a_hat, V = W^V_l a_hat      (no bias, no positional re-encoding),
+ * stored head-major into dst_k / dst_v [L_t][B][H_t][S][d_t] like
+ * mot_translate. One mixture per layer (not per K/V): about half the
+ * translated state of the KV translation.
+ *
+ * src_act: [L_s][max_batch][max_seq][src_act_dim] bf16, device, 16-byte
+ * aligned. The weight blob for mot_load_weights holds, per translated target
+ * layer ascending: Wg[E][d_as], bg[E], then for m = 0..E-1 W1[H][d_as], b1[H],
+ * W2[d_at][H], b2[d_at]; then W^K[D_t][d_at] and W^V[D_t][d_at] (bf16).
+ * Requires bf16, src_act_dim % 64 == 0, tgt_act_dim and D_t = tgt_kv_heads *
+ * tgt_head_dim multiples of 256, tgt_head_dim % 32 == 0, hidden % 256 == 0
+ * (the tensor-core path); otherwise MOT_ERR_UNSUPPORTED. A MoT-h handle
+ * accepts mot_translate_h only (mot_translate returns MOT_ERR_INVALID_ARG);
+ * schedules, routing, profiling and status calls work as for KV handles.
+ */
+typedef struct {
+  int32_t n_layers_src, src_act_dim;
+  int32_t n_layers_tgt, tgt_act_dim, tgt_kv_heads, tgt_head_dim;
+  int32_t n_translators, top_k, hidden;
+  int32_t max_batch, max_seq;
+  mot_dtype dtype;
+  const int32_t* layer_map;   /* as in mot_config */
+} mot_h_config;
+
+mot_status mot_create_h(const mot_h_config* cfg, mot_handle* out);
+mot_status mot_translate_h(mot_handle h, const void* src_act, const int32_t* seq_lens,
+                           int32_t batch, void* dst_k, void* dst_v, mot_stream_t stream);
+
+/*
  * Top-K routing (Def. 3.1 with 0 < top_k < E), tensor-core path.
  *   1 (default where supported): token buckets. The tokens that chose
  *      translator m are gathered per (layer, K/V) group and m's MLP runs on

@@ -108,6 +108,17 @@ struct mot_ctx {
   // tensor maps that do not depend on the caller's buffers
   CUtensorMap tm_w1{}, tm_w2{}, tm_a2{}, tm_a2_st{}, tm_w1h{}, tm_w2h{}, tm_w1q{};
   CUtensorMap tm_g16{}, tm_b2t{}, tm_b2th{}, tm_wg16{};
+  // MoT-h (App. C.5): kind 1 handles translate activations; `d` then holds the
+  // mixture's dims (one-head source of width d_as, one-head output of width
+  // d_at) and `hd` the target cache the projections restore.
+  int kind = 0;
+  int32_t act_tgt = 0;
+  Dims hd{};
+  int gp_h = 1;                 // groups (layers) per pass; a_hat slot = group % gp_h
+  void* wkv = nullptr;          // [G][2 D_t][d_at] bf16: W^K then W^V of each layer
+  void* ahat = nullptr;         // [gp_h][B][S][d_at] bf16 translated activations
+  int32_t* proj_layer = nullptr;   // [G] target layer of each group
+  CUtensorMap tm_wkv{}, tm_ahat{};
   // Top-K routing (tensor-core path, 0 < top_k < E): token buckets per expert
   bool sparse_ok = false;   // the shapes support it
   int routing = 0;          // 0 dense compute with a zeroed gate, 1 token buckets
@@ -148,7 +159,8 @@ void free_all(mot_ctx* h) {
   void* ptrs[] = {h->wg, h->bg, h->w1, h->b1, h->b1h, h->w2, h->b2, h->groups, h->gate, h->gate16,
                   h->b2t, h->wg16, h->a2, h->tiles, h->sel, h->sp.counts, h->sp.counts_all,
                   h->sp.row0, h->sp.plan, h->sp.pairs, h->sp.ltok, h->sp.lslot, h->sp.gatep,
-                  h->sp.gate16p, h->sp.zp, h->sp.a2p, h->sp.ybuf,
+                  h->sp.gate16p, h->sp.zp, h->sp.a2p, h->sp.ybuf, h->wkv, h->ahat,
+                  h->proj_layer,
                   h->n_tiles, h->status, h->counters, h->st_src[0], h->st_src[1], h->st_dst[0],
                   h->st_dst[1], h->st_len};
   for (void* p : ptrs)
@@ -402,7 +414,7 @@ cudaError_t copy_real_rows(void* dst, const void* src, int l0, int l1, int B, in
 mot_status check_translate_args(mot_ctx* h, const void* src_k, const void* src_v,
                                 const int32_t* seq_lens, int32_t batch, const void* dst_k,
                                 const void* dst_v) {
-  if (!h) return MOT_ERR_INVALID_ARG;
+  if (!h || h->kind != 0) return MOT_ERR_INVALID_ARG;   // MoT-h handles: mot_translate_h
   if (batch < 0 || batch > h->d.B) return MOT_ERR_INVALID_ARG;
   if (!src_k || !src_v || !dst_k || !dst_v || (batch > 0 && !seq_lens)) return MOT_ERR_INVALID_ARG;
   if (!aligned16(src_k) || !aligned16(src_v) || !aligned16(dst_k) || !aligned16(dst_v))
@@ -435,7 +447,17 @@ const char* mot_status_string(mot_status s) {
   return "MOT_ERR_UNKNOWN";
 }
 
-mot_status mot_create(const mot_config* cfg, mot_handle* out) {
+}  // extern "C"
+
+namespace {
+
+// MoT-h extras of a handle: the translated activation width and the target
+// cache the projections fill.
+struct HSpec {
+  int32_t act_tgt, H_t, d_t;
+};
+
+mot_status create_impl(const mot_config* cfg, const HSpec* hs, mot_handle* out) {
   if (!out) return MOT_ERR_INVALID_ARG;
   *out = nullptr;
   if (!cfg) return MOT_ERR_INVALID_ARG;
@@ -460,9 +482,31 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
   d.dtype = cfg->dtype == MOT_BF16 ? 0 : 1;
   d.tiles_max = d.B * ((d.S + kTileM - 1) / kTileM);
   d.tpad = d.tiles_max * kTileM;
-  for (int l = 0; l < d.L_t; ++l)
-    if (h->layer_map[l] >= 0)
-      for (int x = 0; x < 2; ++x) h->groups_h.push_back(GroupInfo{l, h->layer_map[l], x, 0});
+  std::vector<int32_t> proj_h;
+  if (hs) {   // MoT-h: one group per translated layer; its a_hat slot is group % gp_h
+    h->kind = 1;
+    h->act_tgt = hs->act_tgt;
+    h->hd = d;
+    h->hd.H_t = hs->H_t;
+    h->hd.d_t = hs->d_t;
+    h->hd.Dt = hs->H_t * hs->d_t;
+    for (int l = 0; l < d.L_t; ++l)
+      if (h->layer_map[l] >= 0) proj_h.push_back(l);
+    const size_t G = proj_h.size();
+    const size_t per = size_t(d.B) * d.S * hs->act_tgt * 2;
+    h->gp_h = static_cast<int>(std::max<size_t>(1, std::min<size_t>(G ? G : 1, kA2Budget / per)));
+    if (G) {
+      const int passes = static_cast<int>((G + h->gp_h - 1) / h->gp_h);
+      h->gp_h = static_cast<int>((G + passes - 1) / passes);
+    }
+    for (size_t g = 0; g < G; ++g)
+      h->groups_h.push_back(
+          GroupInfo{static_cast<int32_t>(g % h->gp_h), h->layer_map[proj_h[g]], 0, 0});
+  } else {
+    for (int l = 0; l < d.L_t; ++l)
+      if (h->layer_map[l] >= 0)
+        for (int x = 0; x < 2; ++x) h->groups_h.push_back(GroupInfo{l, h->layer_map[l], x, 0});
+  }
   d.G = static_cast<int32_t>(h->groups_h.size());
 
   int dev = 0, cc_major = 0, cc_minor = 0;
@@ -480,6 +524,10 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
     return MOT_ERR_UNSUPPORTED;
   }
   h->use_umma = umma_supported(d) && encode_fn() != nullptr;
+  if (hs && !(h->use_umma && h->hd.Dt % kUmmaN == 0 && h->hd.d_t % 32 == 0)) {
+    delete h;   // MoT-h runs on the tensor-core path only
+    return MOT_ERR_UNSUPPORTED;
+  }
   if (h->use_umma && onchip_supported(d)) h->schedule = 3;
 
   const size_t es = esize(d), G = d.G, E = d.E, EH = d.EH;
@@ -519,6 +567,9 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       {&h->sp.a2p, h->sparse_ok ? spR * d.H * 2 : 16},
       {(void**)&h->sp.ybuf,
        h->sparse_ok && d.top_k > 1 ? spGP * d.tpad * size_t(d.top_k) * d.Dt * 4 : 16},
+      {&h->wkv, hs ? G * 2 * size_t(h->hd.Dt) * hs->act_tgt * 2 : 16},
+      {&h->ahat, hs ? size_t(h->gp_h) * d.B * d.S * hs->act_tgt * 2 : 16},
+      {(void**)&h->proj_layer, std::max<size_t>(G, 1) * 4},
       {&h->wg, G * E * d.Ds * es}, {(void**)&h->bg, G * E * 4},
       {&h->w1, G * EH * d.Ds * es}, {(void**)&h->b1, G * EH * 4}, {&h->b1h, G * EH * 2},
       {&h->w2, G * d.Dt * EH * es}, {(void**)&h->b2, G * E * d.Dt * 4},
@@ -539,7 +590,9 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       return MOT_ERR_OOM;
     }
   }
-  if (cudaMemset(h->status, 0, 16) != cudaSuccess || cudaMemset(h->n_tiles, 0, 16) != cudaSuccess ||
+  if ((hs && G &&
+       cudaMemcpy(h->proj_layer, proj_h.data(), G * 4, cudaMemcpyHostToDevice) != cudaSuccess) ||
+      cudaMemset(h->status, 0, 16) != cudaSuccess || cudaMemset(h->n_tiles, 0, 16) != cudaSuccess ||
       (G && cudaMemcpy(h->groups, h->groups_h.data(), G * sizeof(GroupInfo),
                        cudaMemcpyHostToDevice) != cudaSuccess)) {
     cudaGetLastError();
@@ -599,6 +652,14 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
       const uint32_t gb[3] = {64, uint32_t(kTileM), 1};
       ok = ok && encode_bf16(&h->tm_g16p, h->sp.gate16p, 3, gd, gs, gb, /*f16=*/true);
     }
+    if (hs) {   // MoT-h: [W^K; W^V] per layer [G * 2 D_t][d_at] and a_hat [gp_h * B * S][d_at]
+      const uint64_t wd[2] = {uint64_t(hs->act_tgt), uint64_t(G) * 2 * h->hd.Dt};
+      const uint64_t ws[1] = {uint64_t(hs->act_tgt) * 2};
+      const uint32_t box[2] = {uint32_t(kUmmaK), uint32_t(kTileM)};
+      ok = ok && encode_bf16(&h->tm_wkv, h->wkv, 2, wd, ws, box);
+      const uint64_t ad[2] = {uint64_t(hs->act_tgt), uint64_t(h->gp_h) * d.B * d.S};
+      ok = ok && encode_bf16(&h->tm_ahat, h->ahat, 2, ad, ws, box);
+    }
     {  // wg16: [G * 16][Ds], box 64 x 16 (the gate MMA's B side)
       const uint64_t dims[2] = {uint64_t(d.Ds), uint64_t(G) * 16};
       const uint64_t st_b[1] = {uint64_t(d.Ds) * 2};
@@ -622,11 +683,47 @@ mot_status mot_create(const mot_config* cfg, mot_handle* out) {
   return MOT_OK;
 }
 
+}  // namespace
+
+extern "C" {
+
+mot_status mot_create(const mot_config* cfg, mot_handle* out) {
+  return create_impl(cfg, nullptr, out);
+}
+
+mot_status mot_create_h(const mot_h_config* cfg, mot_handle* out) {
+  if (!out) return MOT_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg || cfg->src_act_dim <= 0 || cfg->tgt_act_dim <= 0 || cfg->tgt_kv_heads <= 0 ||
+      cfg->tgt_head_dim <= 0)
+    return MOT_ERR_INVALID_ARG;
+  mot_config mc{};
+  mc.n_layers_src = cfg->n_layers_src;
+  mc.src_kv_heads = 1;
+  mc.src_head_dim = cfg->src_act_dim;
+  mc.n_layers_tgt = cfg->n_layers_tgt;
+  mc.tgt_kv_heads = 1;
+  mc.tgt_head_dim = cfg->tgt_act_dim;
+  mc.n_translators = cfg->n_translators;
+  mc.top_k = cfg->top_k;
+  mc.hidden = cfg->hidden;
+  mc.max_batch = cfg->max_batch;
+  mc.max_seq = cfg->max_seq;
+  mc.dtype = cfg->dtype;
+  mc.layer_map = cfg->layer_map;
+  if (mc.dtype != MOT_BF16) return MOT_ERR_UNSUPPORTED;
+  const HSpec hs{cfg->tgt_act_dim, cfg->tgt_kv_heads, cfg->tgt_head_dim};
+  return create_impl(&mc, &hs, out);
+}
+
 mot_status mot_load_weights(mot_handle h, const void* host_blob, size_t bytes) {
   if (!h || !host_blob) return MOT_ERR_INVALID_ARG;
   const Dims& d = h->d;
   const size_t es = esize(d), gsz = group_elems(d);
-  if (bytes != size_t(d.G) * gsz * es) return MOT_ERR_WEIGHTS_SIZE;
+  // MoT-h blocks: the mixture, then the layer's W^K and W^V [D_t][d_at]
+  const size_t proj = h->kind == 1 ? 2 * size_t(h->hd.Dt) * h->act_tgt : 0;
+  const size_t stride = gsz + proj;
+  if (bytes != size_t(d.G) * stride * es) return MOT_ERR_WEIGHTS_SIZE;
   if (cudaSetDevice(h->device) != cudaSuccess) return MOT_ERR_CUDA;
   const size_t E = d.E, Ds = d.Ds, Dt = d.Dt, H = d.H, EH = d.EH;
   const char* blob = static_cast<const char*>(host_blob);
@@ -648,7 +745,10 @@ mot_status mot_load_weights(mot_handle h, const void* host_blob, size_t bytes) {
   char* w1 = static_cast<char*>(h->w1);
   char* w2 = static_cast<char*>(h->w2);
   for (size_t g = 0; g < size_t(d.G); ++g) {
-    const char* p = blob + g * gsz * es;
+    const char* p = blob + g * stride * es;
+    if (proj)
+      MOT_CUDA_TRY(cudaMemcpy(static_cast<char*>(h->wkv) + g * proj * es, p + gsz * es,
+                              proj * es, cudaMemcpyHostToDevice));
     size_t off = 0;
     MOT_CUDA_TRY(cudaMemcpy(wg + g * E * Ds * es, p, E * Ds * es, cudaMemcpyHostToDevice));
     off += E * Ds;
@@ -698,7 +798,7 @@ mot_status mot_translate(mot_handle h, const void* src_k, const void* src_v,
 mot_status mot_translate_host(mot_handle h, const void* src_k, const void* src_v,
                               const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
                               mot_stream_t stream) {
-  if (!h) return MOT_ERR_INVALID_ARG;
+  if (!h || h->kind != 0) return MOT_ERR_INVALID_ARG;   // MoT-h handles: mot_translate_h
   if (batch < 0 || batch > h->d.B) return MOT_ERR_INVALID_ARG;
   if (!src_k || !src_v || !dst_k || !dst_v || (batch > 0 && !seq_lens)) return MOT_ERR_INVALID_ARG;
   if (!h->weights_loaded) return MOT_ERR_NO_WEIGHTS;
@@ -884,6 +984,42 @@ mot_status mot_profile_read(mot_handle h, mot_kernel_stat* out, int32_t cap, int
 mot_status mot_get_launch_count(mot_handle h, int64_t* count) {
   if (!h || !count) return MOT_ERR_INVALID_ARG;
   *count = h->launches;
+  return MOT_OK;
+}
+
+mot_status mot_translate_h(mot_handle h, const void* src_act, const int32_t* seq_lens,
+                           int32_t batch, void* dst_k, void* dst_v, mot_stream_t stream) {
+  if (!h || h->kind != 1) return MOT_ERR_INVALID_ARG;
+  const Dims& d = h->d;
+  if (batch < 0 || batch > d.B) return MOT_ERR_INVALID_ARG;
+  if (!src_act || !dst_k || !dst_v || (batch > 0 && !seq_lens)) return MOT_ERR_INVALID_ARG;
+  if (!aligned16(src_act) || !aligned16(dst_k) || !aligned16(dst_v)) return MOT_ERR_INVALID_ARG;
+  const size_t sb = src_bytes(d), db = dst_bytes(h->hd);
+  if (overlap(dst_k, db, dst_v, db) || overlap(dst_k, db, src_act, sb) ||
+      overlap(dst_v, db, src_act, sb))
+    return MOT_ERR_INVALID_ARG;
+  if (!h->weights_loaded) return MOT_ERR_NO_WEIGHTS;
+  if (cudaSetDevice(h->device) != cudaSuccess) return MOT_ERR_CUDA;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (batch == 0 || d.G == 0) return MOT_OK;
+  for (int g0 = 0; g0 < d.G; g0 += h->gp_h) {
+    const int g1 = std::min(d.G, g0 + h->gp_h);
+    // the mixture of this pass's layers into their a_hat slots
+    mot_status r = run_translate(h, src_act, src_act, seq_lens, batch, h->ahat, h->ahat, st, g0,
+                                 g1, g0 == 0);
+    if (r != MOT_OK) return r;
+    // K | V = a_hat [W^K; W^V]^T into the target caches
+    PathArgs a = path_args(h);
+    a.d = h->hd;
+    a.dst[0] = dst_k;
+    a.dst[1] = dst_v;
+    a.proj_layer = h->proj_layer;
+    a.g0 = g0;
+    a.gp = g1 - g0;
+    MOT_CUDA_TRY(timed(h, "umma2_proj", st, [&] {
+      return launch_umma2_proj(a, h->tm_ahat, h->tm_wkv, h->act_tgt, h->num_sms, st);
+    }));
+  }
   return MOT_OK;
 }
 

@@ -69,6 +69,7 @@ struct PathArgs {
   void* a2;
   int32_t* status;
   uint32_t* sel;          // [G][tpad] Top-K selection bits per row (sparse routing), else null
+  const int32_t* proj_layer;   // MoT-h projection: the target layer of each group
   int32_t g0, gp;         // groups [g0, g0 + gp) of this pass
   long long wait_limit;   // bound of every pipeline wait, in SM cycles
   int32_t stall_test;     // test hook (single-SM GEMM1): CTA 0 withholds its first stage
@@ -156,6 +157,12 @@ cudaError_t launch_umma2_sparse_gemm2(const PathArgs& a, const SparseArgs& s,
                                       const CUtensorMap& tmA2p, const CUtensorMap& tmW2h,
                                       const CUtensorMap& tmG16p, const CUtensorMap& tmB2th,
                                       int num_sms, cudaStream_t st);
+
+// MoT-h (App. C.5) projection on CTA pairs: K | V = a_hat [W^K; W^V]^T, bf16.
+// a.d holds the target cache dims; act_width = d_at (a multiple of 64).
+cudaError_t launch_umma2_proj(const PathArgs& a, const CUtensorMap& tmAct,
+                              const CUtensorMap& tmWkv, int act_width, int num_sms,
+                              cudaStream_t st);
 
 // On-chip translation on CTA pairs for D_s <= 128, D_t = 256 (onchip.cu):
 // GEMM1, GELU * gate and GEMM2 in one persistent launch over all groups, the

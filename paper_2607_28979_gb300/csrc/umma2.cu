@@ -108,9 +108,44 @@ __device__ __forceinline__ void spin_cycles(long long cycles) {
   }
 }
 
+// MoT-h projection epilogue of one warp (App. C.5): output columns
+// n0 .. n0 + 255 of [K | V] = a_hat [W^K; W^V]^T for row 32 q + lane of token
+// tile m, stored as bf16 into the target cache of the group's target layer
+// (columns below D_t into dst[0] = K, the rest into dst[1] = V). D_t is a
+// multiple of 256, so a tile never straddles the two.
+__device__ __forceinline__ void epilogue_proj(const PathArgs& p, uint32_t tbase, int q, int lane,
+                                              int grp, int m, int n0) {
+  const Dims& d = p.d;
+  const int row = q * 32 + lane;
+  const TileInfo ti = p.tiles[m];
+  const bool valid = row < ti.rows;
+  const int x = n0 >= d.Dt ? 1 : 0;
+  const int c0 = n0 - x * d.Dt;
+  __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.dst[x]);
+  const size_t s = static_cast<size_t>(ti.s0) + row;
+  const size_t lbase = (static_cast<size_t>(p.proj_layer[grp]) * d.B + ti.b) * d.H_t;
+#pragma unroll 1
+  for (int ch = 0; ch < UN / 32; ++ch) {
+    uint32_t r[32];
+    tmem_ld_32x32b_x32(tbase + ch * 32, r);
+    tmem_ld_wait(r);
+    if (valid) {
+      const int c = c0 + ch * 32, h = c / d.d_t, i0 = c - h * d.d_t;
+      uint4* o4 = reinterpret_cast<uint4*>(dst + ((lbase + h) * d.S + s) * d.d_t + i0);
+#pragma unroll
+      for (int v = 0; v < 4; ++v)
+        o4[v] = make_uint4(pack_bf16x2(__uint_as_float(r[8 * v + 0]), __uint_as_float(r[8 * v + 1])),
+                           pack_bf16x2(__uint_as_float(r[8 * v + 2]), __uint_as_float(r[8 * v + 3])),
+                           pack_bf16x2(__uint_as_float(r[8 * v + 4]), __uint_as_float(r[8 * v + 5])),
+                           pack_bf16x2(__uint_as_float(r[8 * v + 6]), __uint_as_float(r[8 * v + 7])));
+    }
+  }
+}
+
 // MODE 1 = GEMM1 (A = source cache, or the packed rows when SPARSE), 2 = GEMM2
-// (A = A2). SPARSE: work items come from the routing's pair-tile list and B is
-// the bucket expert's slice of W1cat / W2cat.
+// (A = A2), 3 = the MoT-h projection (A = translated activation, bf16).
+// SPARSE: work items come from the routing's pair-tile list and B is the
+// bucket expert's slice of W1cat / W2cat.
 template <int MODE, bool SPARSE>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
     umma2_gemm_kernel(const __grid_constant__ CUtensorMap tmA0,
@@ -211,7 +246,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
         const int gl = w.gl, n = w.n, grp = w.grp, m_own = w.m_own;
         TileInfo ti;
         GroupInfo gi;
-        if (MODE == 1 && !SPARSE) {
+        if ((MODE == 1 || MODE == 3) && !SPARSE) {
           gi = p.groups[grp];
           if (m_own < n_m) {
             ti = p.tiles[m_own];
@@ -227,7 +262,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
           const uint32_t bar = leader_addr(&full[stage]);
           const int b_row = grp * ua.b_rows + (MODE == 1 ? w.em * d.H : 0) + n * UN +
                             static_cast<int>(rank) * (UN / 2);
-          if (MODE == 1 && SPARSE) {   // packed rows: [H_s][R][d_s]
+          if (MODE == 3) {   // projection: the translated activation rows of slot gl
+            tma_load_2d_pair(sA + stage * kABytes2, &tmA0, bar, kb * UK,
+                             (gl * d.B + ti.b) * d.S + ti.s0);
+            tma_load_2d_pair(sB + stage * kBBytes2, &tmB, bar, kb * UK, b_row);
+          } else if (MODE == 1 && SPARSE) {   // packed rows: [H_s][R][d_s]
             const int k = kb * UK, h = k / d.d_s, d0 = k - h * d.d_s;
             tma_load_2d_pair(sA + stage * kABytes2, &tmA0, bar, d0, h * ua.sp.R + w.p_own);
             tma_load_2d_pair(sB + stage * kBBytes2, &tmB, bar, kb * UK, b_row);
@@ -259,7 +298,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
   } else if (warp == 1) {
     if (lane == 0 && leader) {
       // ------------------------------------------------ MMA issuer (leader)
-      const uint32_t idesc = MODE == 1 ? idesc_bf16_f32(2 * UM, UN) : idesc_f16_f32(2 * UM, UN);
+      const uint32_t idesc = MODE == 2 ? idesc_f16_f32(2 * UM, UN) : idesc_bf16_f32(2 * UM, UN);
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
       for (int t = pair; t < total; t += n_pairs) {
@@ -330,6 +369,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(threads2(MODE), 1)
         else if (MODE == 1)   // 8 warps: this warp owns columns 128 * (e / 4) .. +127
           epilogue_gemm1(p, &tmS, tbase, sOut + e * kStoreTileBytes, q, lane, grp, n * UN,
                          n * UN, m_own * UM, gl, (e >> 2) * 128, 2, gate_cur);
+        else if (MODE == 3)
+          epilogue_proj(p, tbase, q, lane, grp, m_own, n * UN);
         else if (SPARSE)
           epilogue_gemm2_sparse(p, ua.sp, tbase, q, lane, gl, w.p_own, w.rows_own, n * UN);
         else             // 4 warps: all 256 columns
@@ -445,6 +486,15 @@ cudaError_t launch_umma2_gemm2(const PathArgs& a, const CUtensorMap& tmA2, const
                                cudaStream_t st) {
   return launch_umma2<2, false>(a, nullptr, tmA2, tmG16, tmW2h, tmB2th, a.d.EH / UK + 1,
                                 a.d.Dt / UN, a.d.Dt, num_sms, st);
+}
+
+// MoT-h projection: A = translated activations [slots * B * S][d_at] (box
+// 64 x 128), B = [W^K; W^V] per group [G * 2 D_t][d_at] (box 64 x 128).
+cudaError_t launch_umma2_proj(const PathArgs& a, const CUtensorMap& tmAct,
+                              const CUtensorMap& tmWkv, int act_width, int num_sms,
+                              cudaStream_t st) {
+  return launch_umma2<3, false>(a, nullptr, tmAct, tmAct, tmWkv, tmWkv, act_width / UK,
+                                2 * a.d.Dt / UN, 2 * a.d.Dt, num_sms, st);
 }
 
 }  // namespace mot

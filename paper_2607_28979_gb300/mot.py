@@ -44,6 +44,16 @@ class mot_config(ctypes.Structure):
                 ("layer_map", ctypes.POINTER(ctypes.c_int32))]
 
 
+class mot_h_config(ctypes.Structure):
+    _fields_ = [("n_layers_src", ctypes.c_int32), ("src_act_dim", ctypes.c_int32),
+                ("n_layers_tgt", ctypes.c_int32), ("tgt_act_dim", ctypes.c_int32),
+                ("tgt_kv_heads", ctypes.c_int32), ("tgt_head_dim", ctypes.c_int32),
+                ("n_translators", ctypes.c_int32), ("top_k", ctypes.c_int32),
+                ("hidden", ctypes.c_int32), ("max_batch", ctypes.c_int32),
+                ("max_seq", ctypes.c_int32), ("dtype", ctypes.c_int32),
+                ("layer_map", ctypes.POINTER(ctypes.c_int32))]
+
+
 class mot_kernel_stat(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char * 32), ("launches", ctypes.c_int64),
                 ("total_ms", ctypes.c_double)]
@@ -68,6 +78,8 @@ _SIGS = {
     "mot_profile_read": [_H, ctypes.POINTER(mot_kernel_stat), ctypes.c_int32,
                          ctypes.POINTER(ctypes.c_int32)],
     "mot_get_launch_count": [_H, ctypes.POINTER(ctypes.c_int64)],
+    "mot_create_h": [ctypes.POINTER(mot_h_config), ctypes.POINTER(ctypes.c_void_p)],
+    "mot_translate_h": [_H, _P, _P, ctypes.c_int32, _P, _P, _P],
     "mot_set_routing": [_H, ctypes.c_int32],
     "mot_get_routing": [_H, ctypes.POINTER(ctypes.c_int32)],
     "mot_get_expert_counts": [_H, _P, ctypes.c_int32, _P],
@@ -161,6 +173,30 @@ def config_from(wl):
     return make_config(wl.n_layers_src, wl.src_kv_heads, wl.src_head_dim, wl.n_layers_tgt,
                        wl.tgt_kv_heads, wl.tgt_head_dim, wl.n_translators, wl.hidden,
                        wl.max_batch, wl.max_seq, wl.dtype, wl.top_k, wl.layer_map)
+
+
+def h_config_from(wl):
+    """mot_h_config (MoT-h) for a Workload with ``act_tgt`` > 0 (the source
+    activation stored as a one-head cache of width ``src_head_dim``)."""
+    cfg = mot_h_config(wl.n_layers_src, wl.src_head_dim, wl.n_layers_tgt, wl.act_tgt,
+                       wl.tgt_kv_heads, wl.tgt_head_dim, wl.n_translators, wl.top_k, wl.hidden,
+                       wl.max_batch, wl.max_seq, MOT_BF16 if wl.dtype == "bf16" else MOT_FP32)
+    if wl.layer_map is not None:
+        arr = (ctypes.c_int32 * len(wl.layer_map))(*wl.layer_map)
+        cfg.layer_map = ctypes.cast(arr, ctypes.POINTER(ctypes.c_int32))
+        cfg._keep = arr
+    return cfg
+
+
+def mot_create_h(cfg: mot_h_config) -> Handle:
+    out = ctypes.c_void_p()
+    _check(_lib.mot_create_h(ctypes.byref(cfg), ctypes.byref(out)), "mot_create_h")
+    return Handle(out.value, cfg.n_layers_tgt)
+
+
+def mot_translate_h(h: Handle, src_act, seq_lens, batch: int, dst_k, dst_v, stream=None) -> None:
+    _check(_lib.mot_translate_h(h.ptr, _addr(src_act), _addr(seq_lens), int(batch), _addr(dst_k),
+                                _addr(dst_v), _stream(stream)), "mot_translate_h")
 
 
 def mot_create(cfg: mot_config) -> Handle:

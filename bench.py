@@ -45,6 +45,12 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 def workload_desc(wl) -> str:
     gate = ("dense softmax gate" if wl.top_k in (0, wl.n_translators)
             else f"softmax gate, Top-{wl.top_k} routing")
+    if wl.is_h:
+        return (f"{wl.name}: MoT-h, activations {wl.n_layers_src}L x {wl.src_head_dim} -> "
+                f"{wl.n_layers_tgt}L x {wl.act_tgt}, E={wl.n_translators} MLP "
+                f"{wl.src_head_dim}-{wl.hidden}-{wl.act_tgt} GELU, {gate}, K/V restored through "
+                f"W^K, W^V to {wl.tgt_kv_heads}x{wl.tgt_head_dim}, {wl.dtype}, "
+                f"batch {wl.batch} seq_lens {list(wl.seq_lens)}")
     return (f"{wl.name}: {wl.n_layers_src}L {wl.src_kv_heads}x{wl.src_head_dim} -> "
             f"{wl.n_layers_tgt}L {wl.tgt_kv_heads}x{wl.tgt_head_dim}, E={wl.n_translators} MLP "
             f"{wl.d_src}-{wl.hidden}-{wl.d_tgt} GELU, {gate}, {wl.dtype}, "
@@ -54,21 +60,23 @@ def workload_desc(wl) -> str:
 def algorithmic(wl, layer_map):
     """FLOPs and bytes the method needs per step (no intermediate traffic).
     ``layer_map``: the channel map in use (source layer per target layer, -1 = none)."""
-    T, E, Ds, Dt, Hh = wl.tokens, wl.n_translators, wl.d_src, wl.d_tgt, wl.hidden
+    T, E, Ds, Dt, Hh, Dm = wl.tokens, wl.n_translators, wl.d_src, wl.d_tgt, wl.hidden, wl.d_mix
     n_tl = len(wl.translated_layers())
-    groups = 2 * n_tl
+    groups = n_tl if wl.is_h else 2 * n_tl   # MoT-h: one mixture per layer
     f_gate = 2 * Ds * E
     # with Top-K routing only the top_k chosen translators run on a token
     Ea = wl.top_k if 0 < wl.top_k < E else E
     f_g1 = Ea * 2 * Ds * Hh
-    f_g2 = Ea * 2 * Hh * Dt + 2 * Ea * Dt
+    f_g2 = Ea * 2 * Hh * Dm + 2 * Ea * Dm
+    f_proj = 2 * Dm * 2 * Dt if wl.is_h else 0   # MoT-h: K, V = W^K a_hat, W^V a_hat
     src_layers = {s for s in layer_map if s >= 0}
     es = wl.esize
-    bytes_src = 2 * len(src_layers) * T * Ds * es
-    bytes_dst = groups * T * Dt * es
+    bytes_src = (1 if wl.is_h else 2) * len(src_layers) * T * Ds * es
+    bytes_dst = 2 * n_tl * T * Dt * es
     bytes_w = wl.blob_elems() * es
-    return dict(flops=groups * T * (f_gate + f_g1 + f_g2), flops_gemm1=groups * T * f_g1,
-                flops_gemm2=groups * T * f_g2, bytes=bytes_src + bytes_dst + bytes_w,
+    return dict(flops=groups * T * (f_gate + f_g1 + f_g2 + f_proj), flops_gemm1=groups * T * f_g1,
+                flops_gemm2=groups * T * f_g2, flops_proj=groups * T * f_proj,
+                bytes=bytes_src + bytes_dst + bytes_w,
                 bytes_src=bytes_src, bytes_dst=bytes_dst, bytes_w=bytes_w)
 
 
@@ -208,15 +216,20 @@ def cpu_oracle_rate(wl, sk, sv, blob, budget_s: float, seed: int = 3):
         b = rng.integers(0, wl.batch, size=n)
         s = np.array([rng.integers(0, wl.seq_lens[i]) for i in b])
         return b.astype(np.int32), s.astype(np.int32)
+    def run(tb, ts):
+        if wl.is_h:
+            oracle.translate_h_tokens(wl, sk, blob, tb, ts)
+        else:
+            oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
     c = omp_cores()
     tb, ts = sample(c)   # one token per thread: measures the parallel throughput
     t0 = time.perf_counter()
-    oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
+    run(tb, ts)
     per_tok = max((time.perf_counter() - t0) / c, 1e-6)
     n = int(max(c, min(100000, budget_s / per_tok)))
     tb, ts = sample(n)
     t0 = time.perf_counter()
-    oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
+    run(tb, ts)
     dt = time.perf_counter() - t0
     return n / dt, n, dt
 
@@ -238,14 +251,21 @@ def run_reference(args, wl):
         return 0
     import oracle
     oracle.build()
-    sk, sv, blob = synth.gen_cache(wl, 0), synth.gen_cache(wl, 1), synth.gen_weights(wl)
+    sk, blob = synth.gen_cache(wl, 0), synth.gen_weights(wl)
+    sv = sk if wl.is_h else synth.gen_cache(wl, 1)
+
+    def run(tb, ts):
+        if wl.is_h:
+            oracle.translate_h_tokens(wl, sk, blob, tb, ts)
+        else:
+            oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
     rng = np.random.default_rng(11)
     # size the per-step sample to about 2 s of CPU work
     c = omp_cores()
     tb = np.zeros(c, np.int32)
     ts = (np.arange(c) % wl.seq_lens[0]).astype(np.int32)
     t0 = time.perf_counter()
-    oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
+    run(tb, ts)
     per_tok = (time.perf_counter() - t0) / c
     n = int(max(c, min(4096, 2.0 / max(per_tok, 1e-6))))
 
@@ -253,7 +273,7 @@ def run_reference(args, wl):
         b = rng.integers(0, wl.batch, size=n).astype(np.int32)
         s = np.array([rng.integers(0, wl.seq_lens[i]) for i in b], dtype=np.int32)
         t = time.perf_counter()
-        oracle.translate_tokens(wl, sk, sv, blob, b, s)
+        run(b, s)
         return time.perf_counter() - t
     for _ in range(args.warmup):
         step()
@@ -266,7 +286,7 @@ def run_reference(args, wl):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded SplitMix64/Box-Muller caches and weights)",
         "config": {"workload": workload_desc(wl), "tokens_per_step": n,
-                   "sample": f"{n} random tokens of the workload per step, all {2 * len(wl.translated_layers())} (layer, K/V) groups"},
+                   "sample": f"{n} random tokens of the workload per step, all translated layers"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": omp_cores(), "kind": "oracle",
                          "sample": f"{n} tokens per step x {args.steps} steps"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -289,8 +309,9 @@ def run_mot(args, wl):
         dist.barrier()
     import paper_2607_28979_gb300.mot as M
 
-    sk_h, sv_h, blob = synth.gen_cache(wl, 0), synth.gen_cache(wl, 1), synth.gen_weights(wl)
-    h = M.mot_create(M.config_from(wl))
+    sk_h, blob = synth.gen_cache(wl, 0), synth.gen_weights(wl)
+    sv_h = sk_h if wl.is_h else synth.gen_cache(wl, 1)   # MoT-h: one activation tensor
+    h = M.mot_create_h(M.h_config_from(wl)) if wl.is_h else M.mot_create(M.config_from(wl))
     M.mot_load_weights(h, blob)
     path = M.mot_get_path(h)
     names = {0: "split", 1: "fused", 2: "pair", 3: "onchip"}
@@ -313,7 +334,10 @@ def run_mot(args, wl):
     B = wl.batch
 
     def step():
-        M.mot_translate(h, sk, sv, lens, B, dk, dv, stream)
+        if wl.is_h:
+            M.mot_translate_h(h, sk, lens, B, dk, dv, stream)
+        else:
+            M.mot_translate(h, sk, sv, lens, B, dk, dv, stream)
 
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
@@ -356,22 +380,38 @@ def run_mot(args, wl):
     ov = torch.empty(wl.dst_shape(), dtype=odt).pin_memory()
     lens_h = np.asarray(wl.seq_lens, dtype=np.int32)
     e2e_steps = max(3, min(args.steps, 50))
+    es = wl.esize
+    tl = len(wl.translated_layers())
+
+    def e2e_step():
+        if wl.is_h:   # device entry point with the copies around it, on the same stream
+            with torch.cuda.stream(stream):
+                sk.view(torch.int16).copy_(hk, non_blocking=True)
+                M.mot_translate_h(h, sk, lens, B, dk, dv, stream)
+                ok.copy_(dk.view(torch.int16), non_blocking=True)
+                ov.copy_(dv.view(torch.int16), non_blocking=True)
+        else:
+            M.mot_translate_host(h, hk, hv, lens_h, B, ok, ov, stream)
     for _ in range(2):
-        M.mot_translate_host(h, hk, hv, lens_h, B, ok, ov, stream)
+        e2e_step()
     stream.synchronize()
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for _ in range(e2e_steps):
-        M.mot_translate_host(h, hk, hv, lens_h, B, ok, ov, stream)
+        e2e_step()
     stream.synchronize()
     e2e_s = time.perf_counter() - t0
-    es = wl.esize
-    tl = len(wl.translated_layers())
-    used_src = len({s for s in M.mot_get_layer_map(h) if s >= 0})   # source layers copied
-    h2d = 2 * used_src * wl.tokens * wl.d_src * es + 4 * B
-    d2h = 2 * tl * wl.tokens * wl.d_tgt * es
+    if wl.is_h:
+        h2d = hk.numel() * es
+        d2h = 2 * ok.numel() * es
+        e2e_api = "mot_translate_h with pinned host copies on its stream"
+    else:
+        used_src = len({s for s in M.mot_get_layer_map(h) if s >= 0})   # source layers copied
+        h2d = 2 * used_src * wl.tokens * wl.d_src * es + 4 * B
+        d2h = 2 * tl * wl.tokens * wl.d_tgt * es
+        e2e_api = "mot_translate_host (pinned host buffers)"
 
     # ---- aggregate over ranks: max time
     t_step, e2e_s = reduce_max([elapsed_ms / args.steps, e2e_s], world, "cuda")
@@ -391,6 +431,7 @@ def run_mot(args, wl):
                             "umma2_gemm2_combine_store": alg["flops_gemm2"],
                             "umma2_sparse_gemm1": alg["flops_gemm1"],
                             "umma2_sparse_gemm2": alg["flops_gemm2"],
+                            "umma2_proj": alg["flops_proj"],
                             "umma_gemm1_gelu_gate": alg["flops_gemm1"],
                             "simt_gemm1_gelu_gate": alg["flops_gemm1"],
                             "umma_gemm2_combine_store": alg["flops_gemm2"],
@@ -415,7 +456,7 @@ def run_mot(args, wl):
         if world == 1 and not args.no_cpu_baseline:
             rate, n, dt = cpu_oracle_rate(wl, sk_h, sv_h, blob, budget_s=15.0)
             cpu = {"value": rate, "unit": UNIT, "cores": omp_cores(), "kind": "oracle",
-                   "sample": f"{n} random tokens x all {2 * tl} (layer, K/V) groups, {dt:.1f} s"}
+                   "sample": f"{n} random tokens x all {tl} translated layers, {dt:.1f} s"}
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t_step, "higher_is_better": True,
@@ -436,7 +477,7 @@ def run_mot(args, wl):
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "steps": e2e_steps,
-                    "api": "mot_translate_host (pinned host buffers)"},
+                    "api": e2e_api},
             "gpu_launches": launches,
             "clocks": clocks,
         }

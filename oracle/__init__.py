@@ -20,6 +20,7 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "mot_oracle.c")
+_SRCS = (_SRC, os.path.join(_HERE, "bt_oracle.c"))
 _LIB = os.path.join(_HERE, "libmot_oracle.so")
 
 
@@ -28,11 +29,18 @@ class OracleDims(ctypes.Structure):
                 ("L_s", "H_s", "d_s", "L_t", "H_t", "d_t", "E", "top_k", "H", "B", "S", "dtype")]
 
 
+class OracleBtDims(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("win_start", "win_len", "width", "heads", "ffn")]
+
+
 def build(force: bool = False) -> str:
     """Compile ``libmot_oracle.so`` next to its source if missing or stale."""
-    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+    stale = not os.path.exists(_LIB) or any(os.path.getmtime(_LIB) < os.path.getmtime(f)
+                                             for f in _SRCS)
+    if force or stale:
         tmp = _LIB + f".{os.getpid()}.tmp"
-        subprocess.check_call(["gcc", "-O2", "-fopenmp", "-shared", "-fPIC", "-o", tmp, _SRC, "-lm"])
+        subprocess.check_call(["gcc", "-O2", "-fopenmp", "-shared", "-fPIC", "-o", tmp, *_SRCS,
+                               "-lm"])
         os.replace(tmp, _LIB)
     return _LIB
 
@@ -62,6 +70,19 @@ def _load():
         lib.oracle_translate_full.restype = ctypes.c_int
         lib.oracle_translate_full.argtypes = [ctypes.POINTER(OracleDims), P, P, P, P,
                                               ctypes.c_int32, P, P, P]
+        lib.oracle_layernorm.restype = None
+        lib.oracle_layernorm.argtypes = [P, ctypes.c_int64, P, P, P]
+        lib.oracle_bt_attention.restype = ctypes.c_int
+        lib.oracle_bt_attention.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, P, P, P, P]
+        lib.oracle_bt_blob_elems.restype = ctypes.c_int64
+        lib.oracle_bt_blob_elems.argtypes = [ctypes.POINTER(OracleDims),
+                                             ctypes.POINTER(OracleBtDims)]
+        lib.oracle_bt_backbone.restype = ctypes.c_int
+        lib.oracle_bt_backbone.argtypes = [ctypes.POINTER(OracleDims), ctypes.POINTER(OracleBtDims),
+                                           P, ctypes.c_int, ctypes.c_int, P, P, P]
+        lib.oracle_bt_tokens.restype = ctypes.c_int
+        lib.oracle_bt_tokens.argtypes = [ctypes.POINTER(OracleDims), ctypes.POINTER(OracleBtDims),
+                                         P, P, P, P, ctypes.c_int64, P, P, P, P, P]
         _lib = lib
     return _lib
 
@@ -115,9 +136,10 @@ def translate_tokens(wl, src_k, src_v, blob, tok_b, tok_s, gate_fixed=None, want
     gf = None if gate_fixed is None else np.ascontiguousarray(gate_fixed, dtype=np.float64)
     lm = _map_arr(wl.layer_map)
     d = dims_of(wl)
-    rc = _load().oracle_translate_tokens(ctypes.byref(d), _ptr(lm), _ptr(np.ascontiguousarray(src_k)),
-                                         _ptr(np.ascontiguousarray(src_v)),
-                                         _ptr(np.ascontiguousarray(blob)), n, _ptr(tb), _ptr(ts),
+    # bound to names: the C call must not see the address of a freed temporary copy
+    k_c, v_c, w_c = (np.ascontiguousarray(a) for a in (src_k, src_v, blob))
+    rc = _load().oracle_translate_tokens(ctypes.byref(d), _ptr(lm), _ptr(k_c), _ptr(v_c),
+                                         _ptr(w_c), n, _ptr(tb), _ptr(ts),
                                          _ptr(gf), _ptr(out), _ptr(gate))
     if rc != 0:
         raise ValueError("oracle_translate_tokens: invalid arguments")
@@ -135,10 +157,10 @@ def translate_h_tokens(wl, src_act, blob, tok_b, tok_s, want_act=False):
     ok = np.full((wl.n_layers_tgt, n, wl.d_tgt), np.nan, dtype=np.float64)
     ov = np.full_like(ok, np.nan)
     act = np.full((wl.n_layers_tgt, n, wl.act_tgt), np.nan) if want_act else None
-    rc = _load().oracle_translate_h_tokens(ctypes.byref(dims_of(wl)), wl.act_tgt,
-                                           _ptr(_map_arr(wl.layer_map)),
-                                           _ptr(np.ascontiguousarray(src_act)),
-                                           _ptr(np.ascontiguousarray(blob)), n, _ptr(tb), _ptr(ts),
+    lm = _map_arr(wl.layer_map)
+    a_c, w_c = np.ascontiguousarray(src_act), np.ascontiguousarray(blob)
+    rc = _load().oracle_translate_h_tokens(ctypes.byref(dims_of(wl)), wl.act_tgt, _ptr(lm),
+                                           _ptr(a_c), _ptr(w_c), n, _ptr(tb), _ptr(ts),
                                            _ptr(ok), _ptr(ov), _ptr(act))
     if rc != 0:
         raise ValueError("oracle_translate_h_tokens: invalid arguments")
@@ -152,9 +174,9 @@ def translate_full(wl, src_k, src_v, blob, seq_lens, fill=np.nan):
     dv = np.full(wl.dst_shape(), fill, dtype=np.float64)
     lm = _map_arr(wl.layer_map)
     d = dims_of(wl)
-    rc = _load().oracle_translate_full(ctypes.byref(d), _ptr(lm), _ptr(np.ascontiguousarray(src_k)),
-                                       _ptr(np.ascontiguousarray(src_v)),
-                                       _ptr(np.ascontiguousarray(blob)), sl.size, _ptr(sl),
+    k_c, v_c, w_c = (np.ascontiguousarray(a) for a in (src_k, src_v, blob))
+    rc = _load().oracle_translate_full(ctypes.byref(d), _ptr(lm), _ptr(k_c), _ptr(v_c),
+                                       _ptr(w_c), sl.size, _ptr(sl),
                                        _ptr(dk), _ptr(dv))
     if rc != 0:
         raise ValueError("oracle_translate_full: invalid arguments")
@@ -180,3 +202,71 @@ def sample_tokens(seq_lens, n_per_seq: int, seed: int = 1, tile: int = 128):
             tb.append(b)
             ts.append(s)
     return np.asarray(tb, dtype=np.int32), np.asarray(ts, dtype=np.int32)
+
+
+# ---- backbone translators (App. C.2) -------------------------------------------
+
+def bt_dims_of(wl) -> OracleBtDims:
+    return OracleBtDims(*wl.bt)
+
+
+def layernorm(x, gamma=None, beta=None) -> np.ndarray:
+    """Layer norm of a vector (eps 1e-5, biased variance)."""
+    xv = np.ascontiguousarray(x, dtype=np.float64)
+    y = np.empty_like(xv)
+    g = None if gamma is None else np.ascontiguousarray(gamma, dtype=np.float64)
+    b = None if beta is None else np.ascontiguousarray(beta, dtype=np.float64)
+    _load().oracle_layernorm(xv.ctypes.data, xv.size, _ptr(g), _ptr(b), y.ctypes.data)
+    return y
+
+
+def bt_attention(q, k, v, heads: int) -> np.ndarray:
+    """Multi-head attention of the rows of q over the rows of k, v ([P][d] each)."""
+    q, k, v = (np.ascontiguousarray(a, dtype=np.float64) for a in (q, k, v))
+    P, d = q.shape
+    o = np.empty_like(q)
+    if _load().oracle_bt_attention(P, d, heads, q.ctypes.data, k.ctypes.data, v.ctypes.data,
+                                   o.ctypes.data) != 0:
+        raise ValueError("oracle_bt_attention: invalid sizes")
+    return o
+
+
+def bt_blob_elems(wl) -> int:
+    return int(_load().oracle_bt_blob_elems(ctypes.byref(dims_of(wl)), ctypes.byref(bt_dims_of(wl))))
+
+
+def bt_backbone(wl, blob, X: int, m: int, x):
+    """One backbone translator (expert m of block X) on one token's window
+    x[N][P][d_s]. Returns (Y[N][D_t], h[N][P][d])."""
+    _, N, d, _, _ = wl.bt
+    xv = np.ascontiguousarray(x, dtype=np.float64)
+    y = np.empty((N, wl.d_tgt))
+    h = np.empty((N, wl.src_kv_heads, d))
+    w_c = np.ascontiguousarray(blob)
+    rc = _load().oracle_bt_backbone(ctypes.byref(dims_of(wl)), ctypes.byref(bt_dims_of(wl)),
+                                    _ptr(w_c), X, m, xv.ctypes.data,
+                                    y.ctypes.data, h.ctypes.data)
+    if rc != 0:
+        raise ValueError("oracle_bt_backbone: invalid arguments")
+    return y, h
+
+
+def bt_tokens(wl, src_k, src_v, blob, tok_b, tok_s, gate_fixed=None, want_gate=False):
+    """Backbone-translator MoT for sampled tokens. Returns out[N][2][n][D_t]
+    (slot r = target layer window start + r) and, with ``want_gate``, the kept
+    renormalised gate [2][n][E]."""
+    tb = np.ascontiguousarray(tok_b, dtype=np.int32)
+    ts = np.ascontiguousarray(tok_s, dtype=np.int32)
+    n = tb.size
+    N = wl.bt[1]
+    out = np.full((N, 2, n, wl.d_tgt), np.nan)
+    gate = np.full((2, n, wl.n_translators), np.nan) if want_gate else None
+    gf = None if gate_fixed is None else np.ascontiguousarray(gate_fixed, dtype=np.float64)
+    lm = _map_arr(wl.layer_map)
+    k_c, v_c, w_c = (np.ascontiguousarray(a) for a in (src_k, src_v, blob))
+    rc = _load().oracle_bt_tokens(ctypes.byref(dims_of(wl)), ctypes.byref(bt_dims_of(wl)),
+                                  _ptr(lm), _ptr(k_c), _ptr(v_c), _ptr(w_c),
+                                  n, _ptr(tb), _ptr(ts), _ptr(gf), _ptr(out), _ptr(gate))
+    if rc != 0:
+        raise ValueError("oracle_bt_tokens: invalid arguments")
+    return (out, gate) if want_gate else out

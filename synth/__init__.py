@@ -11,7 +11,9 @@ are not available):
   * K, V = s_c * N(0, 1), with a per-channel scale s_c ~ LogNormal(0, 0.5)
     drawn once per (source layer, K/V, channel c = h*d + i);
   * every weight and bias ~ N(0, 1/fan_in): fan_in = D_s for the gate and the
-    first translator layer, H for the second;
+    first translator layer, H for the second (backbone translators: the input
+    width of each linear map);
+  * backbone layer norms: gain ~ 1 + 0.1 N(0, 1), shift ~ 0.1 N(0, 1);
   * fp64 draws rounded to fp32, then (bf16 workloads) to bf16 with
     round-to-nearest-even.
 
@@ -33,6 +35,14 @@ _LIB = os.path.join(_HERE, "libsynth.so")
 
 # Blob tensor ids, in blob order within one (target layer, K/V) group.
 T_WG, T_BG, T_W1, T_B1, T_W2, T_B2, T_WK, T_WV = range(8)
+
+# Backbone-translator blob tensors (App. C.2), in blob order: the window gate,
+# then per expert the input block, per slot one CAB block, then the output block.
+BT_TENSORS = ("wg", "bg", "lnin_g", "lnin_b", "win", "bin",
+              "lnq_g", "lnq_b", "lnc_g", "lnc_b", "wq", "bq", "wk", "bk", "wv", "bv", "wo", "bo",
+              "lnf_g", "lnf_b", "wf1", "bf1", "wf2", "bf2",
+              "lnout_g", "lnout_b", "wout", "bout")
+BT_ID = {name: 16 + i for i, name in enumerate(BT_TENSORS)}
 
 
 def build(force: bool = False) -> str:
@@ -61,6 +71,10 @@ def _load():
         lib.synth_fill_normal.restype = None
         lib.synth_fill_normal.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int64,
                                           ctypes.c_double, ctypes.c_int, ctypes.c_void_p]
+        lib.synth_fill_normal_shifted.restype = None
+        lib.synth_fill_normal_shifted.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int64,
+                                                  ctypes.c_double, ctypes.c_double, ctypes.c_int,
+                                                  ctypes.c_void_p]
         lib.synth_fill_cache_layer.restype = None
         lib.synth_fill_cache_layer.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64,
                                                ctypes.c_int, ctypes.c_int, ctypes.c_int,
@@ -92,6 +106,19 @@ class Workload:
     # (src_kv_heads = 1, src_head_dim = d_as); the target caches are restored
     # through per-layer projections W^K, W^V [D_t][d_at].
     act_tgt: int = 0
+    # Backbone translators (App. C.2): (window start, window length N, width d,
+    # attention heads n_a, FFN width d_f). The window is target layers
+    # start .. start+N-1; each source-head row of a slot is one attention row.
+    bt: Optional[Tuple[int, int, int, int, int]] = None
+
+    @property
+    def is_bt(self) -> bool:
+        return self.bt is not None
+
+    @property
+    def bt_window(self) -> list:
+        q, n = self.bt[0], self.bt[1]
+        return list(range(q, q + n))
 
     @property
     def d_src(self) -> int:
@@ -140,12 +167,17 @@ class Workload:
 
     def group_elems(self) -> int:
         """Elements of one block of the weight blob: a (target layer, K/V) group,
-        or for MoT-h a target layer (mixture, then W^K and W^V)."""
+        or for MoT-h a target layer (mixture, then W^K and W^V), or for backbone
+        translators a K/V block (window gate, then every expert)."""
+        if self.is_bt:
+            return sum(item[5] for item in bt_blob_offsets(self) if item[0] == 0)
         E, Ds, Dm, H = self.n_translators, self.d_src, self.d_mix, self.hidden
         n = E * Ds + E + E * (H * Ds + H + Dm * H + Dm)
         return n + (2 * self.d_tgt * self.act_tgt if self.is_h else 0)
 
     def blob_elems(self) -> int:
+        if self.is_bt:
+            return 2 * self.group_elems()
         return (1 if self.is_h else 2) * len(self.translated_layers()) * self.group_elems()
 
     def replace(self, **kw) -> "Workload":
@@ -180,6 +212,18 @@ WORKLOADS.update({
     # Qwen2.5-0.5B (896, 24L) -> Qwen2.5-1.5B (1536, 28L; KV 2x128), E=4, MLP 896->1024->1536.
     "h_qwen05_qwen15": Workload("h_qwen05_qwen15", 24, 1, 896, 28, 2, 128, 4, 1024, 4, 4096,
                                 "bf16", (4096,) * 4, act_tgt=1536),
+})
+
+# Backbone-translator (App. C.2) counterparts: a channel window of about 0.3 of
+# the layers (the paper's default ratio), N_Tr = 2 backbones, rows of width 128
+# with 4 attention heads and an FFN of 512.
+WORKLOADS.update({
+    # GPT-2-small -> OPT-125m (12x64 -> 12x64): window = target layers 4..7.
+    "bt_gpt2s_opt125m": Workload("bt_gpt2s_opt125m", 12, 12, 64, 12, 12, 64, 2, 0, 8, 1024,
+                                 "bf16", (1024,) * 8, bt=(4, 4, 128, 4, 512)),
+    # Qwen2.5-0.5B (24L, 2x64) -> Qwen2.5-1.5B (28L, 2x128): window = target layers 10..17.
+    "bt_qwen05_qwen15": Workload("bt_qwen05_qwen15", 24, 2, 64, 28, 2, 128, 2, 0, 4, 4096,
+                                 "bf16", (4096,) * 4, bt=(10, 8, 128, 4, 512)),
 })
 
 # Order in which the workloads are listed in the build's benchmark configuration.
@@ -226,12 +270,65 @@ def blob_offsets(wl: Workload):
                 yield (l, x, T_WV, 0, off, Dt * Dm, Dm); off += Dt * Dm
 
 
+def bt_blob_offsets(wl: Workload):
+    """Backbone-translator blob: yield (x, name, expert, slot, offset, numel, mean, std)
+    for every tensor, in blob order (slot -1 = not a CAB tensor)."""
+    E, P, ds, Ds, Dt = wl.n_translators, wl.src_kv_heads, wl.src_head_dim, wl.d_src, wl.d_tgt
+    _, N, d, _, df = wl.bt
+    off = 0
+
+    def t(x, name, m, r, n, fan_in=None):
+        nonlocal off
+        if name.endswith("_g"):
+            mean, std = 1.0, 0.1
+        elif name.startswith("ln"):
+            mean, std = 0.0, 0.1
+        else:
+            mean, std = 0.0, 1.0 / np.sqrt(fan_in)
+        item = (x, name, m, r, off, n, mean, std)
+        off += n
+        return item
+
+    for x in (0, 1):
+        yield t(x, "wg", 0, -1, E * N * Ds, N * Ds)
+        yield t(x, "bg", 0, -1, E, N * Ds)
+        for m in range(E):
+            yield t(x, "lnin_g", m, -1, ds)
+            yield t(x, "lnin_b", m, -1, ds)
+            yield t(x, "win", m, -1, d * ds, ds)
+            yield t(x, "bin", m, -1, d, ds)
+            for r in range(N):
+                for nm in ("lnq_g", "lnq_b", "lnc_g", "lnc_b"):
+                    yield t(x, nm, m, r, d)
+                for nm in ("wq", "wk", "wv", "wo"):
+                    yield t(x, nm, m, r, d * d, d)
+                    yield t(x, "b" + nm[1], m, r, d, d)
+                yield t(x, "lnf_g", m, r, d)
+                yield t(x, "lnf_b", m, r, d)
+                yield t(x, "wf1", m, r, df * d, d)
+                yield t(x, "bf1", m, r, df, d)
+                yield t(x, "wf2", m, r, d * df, df)
+                yield t(x, "bf2", m, r, d, df)
+            yield t(x, "lnout_g", m, -1, P * d)
+            yield t(x, "lnout_b", m, -1, P * d)
+            yield t(x, "wout", m, -1, Dt * P * d, P * d)
+            yield t(x, "bout", m, -1, Dt, P * d)
+
+
 def gen_weights(wl: Workload, seed: int = 0) -> np.ndarray:
     """Packed weight blob (flat, storage dtype) in the library's documented order."""
     lib = _load()
     out = np.empty(wl.blob_elems(), dtype=wl.np_dtype)
     dt = 0 if wl.dtype == "bf16" else 1
     base = out.ctypes.data
+    if wl.is_bt:
+        end = 0
+        for (x, name, m, r, off, n, mean, std) in bt_blob_offsets(wl):
+            stream = _stream_weight(r & 0xFFFF, x, m, BT_ID[name])
+            lib.synth_fill_normal_shifted(seed, stream, n, mean, std, dt, base + off * wl.esize)
+            end = off + n
+        assert end == out.size
+        return out
     for (l, x, t, m, off, n, fan_in) in blob_offsets(wl):
         lib.synth_fill_normal(seed, _stream_weight(l, x, m, t), n, 1.0 / np.sqrt(fan_in), dt,
                               base + off * wl.esize)

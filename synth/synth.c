@@ -99,6 +99,26 @@ void synth_fill_normal(uint64_t seed, uint64_t stream, int64_t n, double stddev,
   }
 }
 
+/* out[i] = mean + stddev * N_i (as synth_fill_normal, shifted by `mean`). */
+void synth_fill_normal_shifted(uint64_t seed, uint64_t stream, int64_t n, double mean,
+                               double stddev, int dtype, void* out) {
+  uint64_t key = synth_stream_key(seed, stream);
+  const int64_t np = (n + 1) / 2;
+#pragma omp parallel for schedule(static)
+  for (int64_t k = 0; k < np; ++k) {
+    double v[2];
+    normal_pair(key, (uint64_t)k, &v[0], &v[1]);
+    for (int j = 0; j < 2; ++j) {
+      const int64_t i = 2 * k + j;
+      if (i >= n) break;
+      if (dtype == 2)
+        ((double*)out)[i] = mean + stddev * v[j];
+      else
+        store_val(out, i, mean + stddev * v[j], dtype);
+    }
+  }
+}
+
 /*
  * One layer of a KV cache laid out [B][H][S][d]: value = s_c * N, where the
  * per-channel scale s_c = exp(0.5 * n_c) ~ LogNormal(0, 0.5) is drawn once per

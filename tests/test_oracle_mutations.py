@@ -10,6 +10,7 @@ import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 PINS = os.path.join(ROOT, "tests", "test_oracle_pins.py")
+BT_PINS = os.path.join(ROOT, "tests", "test_oracle_bt_pins.py")
 
 MUTATIONS = {
     "drop_b1": ("h[j] = oracle_gelu(dot(row, z, Ds) + ld(w, dt, o_b1 + j));",
@@ -42,18 +43,50 @@ MUTATIONS = {
 }
 
 
-@pytest.mark.parametrize("name", sorted(MUTATIONS))
-def test_planted_mistake_is_caught(name, tmp_path):
-    before, after = MUTATIONS[name]
-    src = open(os.path.join(ROOT, "oracle", "mot_oracle.c")).read()
+# Mistakes in the backbone-translator oracle (App. C.2), caught by its own pins.
+BT_MUTATIONS = {
+    "bt_drop_ln_in": ("ln_blob(w, dt, o_lnin, ds, x + (r * P + p) * ds, s->vec, s);",
+                      "memcpy(s->vec, x + (r * P + p) * ds, sizeof(double) * (size_t)ds);"),
+    "bt_h0_from_last_slot": ("memcpy(s->h, s->z, sizeof(double) * (size_t)Pd);",
+                             "memcpy(s->h, s->z + (L->N - 1) * Pd, sizeof(double) * (size_t)Pd);"),
+    "bt_attn_unscaled": ("sc[j] = s * scale;", "sc[j] = s;"),
+    "bt_attn_one_head": ("oracle_bt_attention((int)P, (int)d, (int)L->na, s->q, s->k, s->v, s->o);",
+                         "oracle_bt_attention((int)P, (int)d, 1, s->q, s->k, s->v, s->o);"),
+    "bt_keys_from_state": ("ln_blob(w, dt, o_lnc, d, zr + p * d, s->nc + p * d, s);",
+                           "ln_blob(w, dt, o_lnc, d, s->h + p * d, s->nc + p * d, s);"),
+    "bt_no_attn_residual": ("s->ht[p * d + i] = s->h[p * d + i] + s->a[p * d + i];",
+                            "s->ht[p * d + i] = s->a[p * d + i];"),
+    "bt_ffn_no_gelu": ("for (int64_t j = 0; j < df; ++j) s->f[j] = oracle_gelu(s->f[j]);", ""),
+    "bt_ln_out_per_row": ("ln_blob(w, dt, o_lnout, Pd, s->h, s->nF, s);",
+                          "for (int64_t p = 0; p < P; ++p) "
+                          "oracle_layernorm(s->h + p * d, d, NULL, NULL, s->nF + p * d);"),
+    "bt_no_output_gelu": ("for (int64_t i = 0; i < L->Dt; ++i) yr[i] = oracle_gelu(yr[i]);", ""),
+    "bt_gate_no_bias": ("logit[m] = sdot + bld(blob, d->dtype, gbase + E * WD + m);",
+                        "logit[m] = sdot;"),
+    "bt_ln_eps": ("static const double kLnEps = 1e-5;", "static const double kLnEps = 1e-3;"),
+    "bt_ln_unbiased": ("  var /= (double)n;", "  var /= (double)(n - 1);"),
+    "bt_window_ignores_map": ("const int64_t sl = map[bt->win_start + r];",
+                              "const int64_t sl = bt->win_start + r;"),
+    "bt_slots_reversed": ("for (int64_t i = 0; i < Dt; ++i) o[i] = acc[r * Dt + i];",
+                          "for (int64_t i = 0; i < Dt; ++i) o[i] = acc[(N - 1 - r) * Dt + i];"),
+}
+
+CASES = ([(n, "mot_oracle.c", PINS, MUTATIONS[n]) for n in sorted(MUTATIONS)] +
+         [(n, "bt_oracle.c", BT_PINS, BT_MUTATIONS[n]) for n in sorted(BT_MUTATIONS)])
+
+
+@pytest.mark.parametrize("name,src_name,pins,change", CASES, ids=[c[0] for c in CASES])
+def test_planted_mistake_is_caught(name, src_name, pins, change, tmp_path):
+    before, after = change
+    src = open(os.path.join(ROOT, "oracle", src_name)).read()
     assert src.count(before) == 1, "mutation anchor not found: the oracle source changed"
     dst = tmp_path / "oracle"
     shutil.copytree(os.path.join(ROOT, "oracle"), dst,
                     ignore=shutil.ignore_patterns("*.so", "*.tmp", "__pycache__"))
-    (dst / "mot_oracle.c").write_text(src.replace(before, after))
+    (dst / src_name).write_text(src.replace(before, after))
     env = dict(os.environ, PYTHONPATH=f"{tmp_path}{os.pathsep}{ROOT}")
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider",
-                        "--rootdir", str(tmp_path), PINS], cwd=tmp_path, env=env,
+                        "--rootdir", str(tmp_path), pins], cwd=tmp_path, env=env,
                        capture_output=True, text=True, timeout=300)
     assert r.returncode != 0, f"pins did not catch '{name}':\n{r.stdout[-2000:]}"
     assert "failed" in r.stdout

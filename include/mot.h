@@ -290,6 +290,58 @@ mot_status mot_get_routing(mot_handle h, int32_t* routing);
  */
 mot_status mot_get_expert_counts(mot_handle h, int32_t* counts, int32_t n, mot_stream_t stream);
 
+/*
+ * Backbone translators (App. C.2) as the experts of the mixture (Def. 3.1).
+ * The translation covers one channel window: N consecutive target layers
+ * t_r = win_start + r (r = 0..N-1), each paired with source layer pi(t_r)
+ * (cfg.layer_map, or the depth-ratio map). For every token u and X in {K, V},
+ * slot r's input is the source cache entry X_r = src_X[pi(t_r)][b][:, s, :],
+ * a P x d_s matrix with one row per source KV head (P = src_kv_heads), and
+ * each backbone m computes, with LN a layer norm (eps 1e-5) and GELU exact:
+ *   z_r     = GELU(W_in LN_in(X_r) + b_in)                 row-wise, width d
+ *   h_0     = z_1
+ *   CAB_r:  a = MHA(LN_Q(h_{r-1}), LN_C(z_r), LN_C(z_r))    n_a heads over the
+ *                                                           token's P rows
+ *           ht = h_{r-1} + a;  h_r = ht + W_F2 GELU(W_F1 LN_F(ht) + b_F1) + b_F2
+ *   Y_r     = GELU(W_out LN_out(flatten(h_r)) + b_out)      width D_t
+ * (MHA: queries W_Q . + b_Q, keys W_K . + b_K, values W_V . + b_V, softmax of
+ * the scaled dot products over the P rows, output W_O . + b_O). The gate reads
+ * the whole window, logit = Wg concat_r(X_r flattened head-major) + bg; the
+ * output y_r = sum over kept m of gtilde_m Y_{m,r} goes into target layer t_r
+ * head-major, as in mot_translate. Layers outside the window are untouched.
+ *
+ * Weight blob (bf16), the block for X = K, then the block for X = V:
+ *   Wg[E][N * D_s], bg[E], then for each backbone m:
+ *     ln_in.gamma[d_s], ln_in.beta[d_s], W_in[d][d_s], b_in[d],
+ *     for each slot r: ln_q.gamma[d], ln_q.beta[d], ln_c.gamma[d], ln_c.beta[d],
+ *       W_Q[d][d], b_Q[d], W_K[d][d], b_K[d], W_V[d][d], b_V[d], W_O[d][d], b_O[d],
+ *       ln_f.gamma[d], ln_f.beta[d], W_F1[d_f][d], b_F1[d_f], W_F2[d][d_f], b_F2[d],
+ *     ln_out.gamma[P * d], ln_out.beta[P * d], W_out[D_t][P * d], b_out[D_t].
+ * mot_load_weights folds LN_in's and LN_out's affines into W_in and W_out;
+ * the other layer norms' affines are applied where their rows are written.
+ *
+ * cfg.hidden is unused (0). Requires bf16, P <= 16, d_s in {64, 128}, d in
+ * {64, 128}, d / n_a in {16, 32, 64}, d_f a multiple of 64 (and of 256 above
+ * 256), D_t and d_t multiples of 32, E <= 8, N <= 32, every window layer
+ * mapped; otherwise MOT_ERR_UNSUPPORTED (MOT_ERR_INVALID_ARG for a window
+ * outside [0, L_t) or non-positive sizes). A backbone handle accepts
+ * mot_translate_bt only; profiling, launch counts and status calls work as
+ * for KV handles. mot_translate_bt has the arguments, layouts, alignment,
+ * sequence-length and stream rules of mot_translate.
+ */
+typedef struct {
+  int32_t win_start;   /* first target layer of the channel window */
+  int32_t win_len;     /* N, slots of the window */
+  int32_t width;       /* d, translator width of one source-head row */
+  int32_t heads;       /* n_a, attention heads (width % heads == 0) */
+  int32_t ffn;         /* d_f, FFN hidden width */
+} mot_bt_config;
+
+mot_status mot_create_bt(const mot_config* cfg, const mot_bt_config* bt, mot_handle* out);
+mot_status mot_translate_bt(mot_handle h, const void* src_k, const void* src_v,
+                            const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
+                            mot_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1,0 +1,892 @@
+// Backbone translators (App. C.2) inside the gated mixture (Def. 3.1) on sm_103a.
+//
+// Per token, slot r of the channel window is the source cache entry of layer
+// pi(t_r): P = H_s rows (one per source KV head) of d_s values. A group
+// g = x * E + m (K/V block x, backbone m) owns a row space of R = B * S * P rows,
+// row ((b * S + s) * P + p). One slot of the recurrent scan is eight launches:
+//
+//   kBtIn   z  = GELU(W_in LN_in(x) + b_in)        A = the source cache (TMA 3-D box
+//                                                   of tau tokens x P heads), the
+//                                                   layer norm applied in the epilogue:
+//                                                   (W_in' x - mu sum(W_in')) rstd + c, with
+//                                                   W_in' = W_in diag(gamma) held as bf16
+//                                                   hi + lo (two K blocks per source block)
+//           xz = LN_C(z); slot 0 also h = z (h_0 = z_1) and xq = LN_Q(z)
+//   kBtQ    q  = W_Q xq + b_Q
+//   kBtKV   k|v = W_KV xz + b_KV
+//   attn    o  = softmax of the scaled scores over the token's P key rows, per head
+//                (SIMT, bt_attn_kernel)
+//   kBtO    ht = h + W_O o + b_O;  xf = LN_F(ht)
+//   kBtF1   f  = GELU(W_F1 xf + b_F1)
+//   kBtF2   h  = ht + W_F2 f + b_F2;  xq = LN_Q(h) of the next slot; xo = bf16(h) and
+//           the row's (mean, M2) statistics
+//   kBtOut  dst[t_r] = sum_m gtilde_m GELU(rstd (W_out' xo_m - mu sum(W_out')) + c_m)
+//                                                  (LN_out over the token's P*d values,
+//                                                   folded like LN_in; mu, rstd from the
+//                                                   P row statistics; the E backbones of
+//                                                   block x in one tile)
+//
+// The row layer norms gamma * (v - mean) / sqrt(var + 1e-5) + beta run over the
+// row's d values in fp32, on the fp32 row held in registers; the matrices they
+// feed stay the blob's exact bf16 values. Every GEMM is one persistent,
+// warp-specialised tcgen05 kernel: warp 0 TMA producer (4-stage ring of 64-wide K blocks), warp 1 MMA issuer
+// (M = 128, N = NT, fp32 accumulators in TMEM, two buffers), warp 2 TMEM
+// allocator, warps 4..7 the epilogue (one TMEM lane = one row each). Row tiles
+// hold whole tokens (tau = 128 / P of them). The epilogue warps never wait on
+// one another. All waits are bounded; on a timeout every role
+// unwinds, copies and MMAs in flight are drained, TMEM is freed and
+// kStatusTimeout is raised.
+#include <cuda_bf16.h>
+
+#include <algorithm>
+
+#include "mot_internal.h"
+#include "ptx.cuh"
+
+namespace mot {
+namespace {
+
+constexpr int kBtStages = 4;
+constexpr int kBtABytes = 128 * 64 * 2;   // 16 KB: 128 rows x 64 bf16
+constexpr int kBtBBytes = 256 * 64 * 2;   // 32 KB: up to 256 rows x 64 bf16
+constexpr int kBtStageBytes = kBtABytes + kBtBBytes;
+constexpr int kBtThreads = 256;           // warps 0..3 roles, 4..7 epilogue
+constexpr int kBtTmemCols = 512;
+constexpr float kLnEps = 1e-5f;
+constexpr int kBtSmem = kBtStages * kBtStageBytes + 256 + 1024;
+static_assert(kBtSmem <= 232448, "shared memory budget");
+
+__device__ __forceinline__ float gelu_erf(float u) {
+  return 0.5f * u * (1.f + erff(u * 0.70710678118654752f));
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ int seq_len_of(const BtArgs& a, int b) {
+  if (b >= a.batch) return 0;
+  const int L = a.seq_lens[b];
+  return L < 0 ? 0 : (L > a.d.S ? a.d.S : L);
+}
+
+struct GemmCfg {
+  int mode;
+  int K;          // reduction length per backbone
+  int NT;         // accumulator columns per tile (multiple of 32, <= 256)
+  int n_tiles;    // N tiles per group
+  int groups;     // groups iterated (2E, or 2 for kBtOut)
+  int row_tiles;  // row tiles per group
+  int a_box_bytes;
+  int b_rows_per_g;   // rows of the weight map per (group, slot) block
+};
+
+// One work item of the persistent loop. Every role decodes items the same way
+// (skipping the same inactive tiles), so their barrier phases stay in step.
+struct Work {
+  int g, b, s0, ntok, j;
+  int tok0;       // kBtOut: first token of the 128-token tile
+  bool active;
+};
+
+__device__ __forceinline__ Work decode(const BtArgs& a, const GemmCfg& c, int item) {
+  Work w;
+  const int per_g = c.row_tiles * c.n_tiles;
+  w.g = item / per_g;
+  const int rem = item - w.g * per_g;
+  const int rt = rem / c.n_tiles;
+  w.j = rem - rt * c.n_tiles;
+  if (c.mode == kBtOut) {
+    w.tok0 = rt * 128;
+    w.b = w.tok0 / a.d.S;
+    w.s0 = w.tok0 - w.b * a.d.S;
+    w.ntok = 128;
+    // active if any token of the tile is inside its sequence
+    bool act = false;
+    for (int b = w.b; b < a.d.B && b * a.d.S < w.tok0 + 128; ++b) {
+      const int lo = max(0, w.tok0 - b * a.d.S);
+      act = act || lo < seq_len_of(a, b);
+    }
+    w.active = act;
+  } else {
+    w.b = rt / a.d.tiles_b;
+    w.s0 = (rt - w.b * a.d.tiles_b) * a.d.tau;
+    w.ntok = min(a.d.tau, a.d.S - w.s0);
+    w.tok0 = w.b * a.d.S + w.s0;
+    w.active = w.s0 < seq_len_of(a, w.b);
+  }
+  return w;
+}
+
+struct EpiCtx {
+  const BtArgs* a;
+  const GemmCfg* c;
+};
+
+// ---------------------------------------------------------------- epilogues
+//
+// Each thread owns one accumulator row (TMEM lane 32 * q + lane). `tb` is the
+// accumulator address with the lane quarter already added.
+
+template <int D>
+__device__ __forceinline__ void load_row(uint32_t tb, float (&v)[D]) {
+#pragma unroll
+  for (int c = 0; c < D / 32; ++c) {
+    uint32_t r[32];
+    tmem_ld_32x32b_x32(tb + c * 32, r);
+    tmem_ld_wait(r);
+#pragma unroll
+    for (int k = 0; k < 32; ++k) v[c * 32 + k] = __uint_as_float(r[k]);
+  }
+}
+
+template <int D>
+__device__ __forceinline__ void row_stats(const float (&v)[D], float& mean, float& m2) {
+  float s = 0.f;
+#pragma unroll
+  for (int k = 0; k < D; ++k) s += v[k];
+  mean = s * (1.f / D);
+  float q = 0.f;
+#pragma unroll
+  for (int k = 0; k < D; ++k) {
+    const float t = v[k] - mean;
+    q = fmaf(t, t, q);
+  }
+  m2 = q;
+}
+
+// dst[0..D) = bf16(gamma * (v - mean) * rstd + beta), 16-byte stores; ln holds
+// gamma[D] then beta[D]
+template <int D>
+__device__ __forceinline__ void store_norm(const float (&v)[D], float mean, float rstd,
+                                           const float* ln, uint16_t* dst) {
+  uint4* d4 = reinterpret_cast<uint4*>(dst);
+  const float4* g4 = reinterpret_cast<const float4*>(ln);
+  const float4* b4 = reinterpret_cast<const float4*>(ln + D);
+#pragma unroll
+  for (int c = 0; c < D / 8; ++c) {
+    const float4 g0 = __ldg(g4 + 2 * c), g1 = __ldg(g4 + 2 * c + 1);
+    const float4 b0 = __ldg(b4 + 2 * c), b1 = __ldg(b4 + 2 * c + 1);
+    const float gg[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+    const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+    float y[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) y[k] = fmaf((v[8 * c + k] - mean) * rstd, gg[k], bb[k]);
+    d4[c] = make_uint4(pack2(y[0], y[1]), pack2(y[2], y[3]), pack2(y[4], y[5]), pack2(y[6], y[7]));
+  }
+}
+
+template <int D>
+__device__ __forceinline__ void store_f32(const float (&v)[D], float* dst) {
+  float4* d4 = reinterpret_cast<float4*>(dst);
+#pragma unroll
+  for (int c = 0; c < D / 4; ++c) d4[c] = make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+}
+
+template <int D>
+__device__ __forceinline__ void add_f32(float (&v)[D], const float* src) {
+  const float4* s4 = reinterpret_cast<const float4*>(src);
+#pragma unroll
+  for (int c = 0; c < D / 4; ++c) {
+    const float4 t = s4[c];
+    v[4 * c] += t.x;
+    v[4 * c + 1] += t.y;
+    v[4 * c + 2] += t.z;
+    v[4 * c + 3] += t.w;
+  }
+}
+
+template <int D>
+__device__ __forceinline__ void add_bias(float (&v)[D], const float* bias) {
+  const float4* b4 = reinterpret_cast<const float4*>(bias);
+#pragma unroll
+  for (int c = 0; c < D / 4; ++c) {
+    const float4 t = __ldg(b4 + c);
+    v[4 * c] += t.x;
+    v[4 * c + 1] += t.y;
+    v[4 * c + 2] += t.z;
+    v[4 * c + 3] += t.w;
+  }
+}
+
+template <int D>
+__device__ __forceinline__ void store_bf16(const float (&v)[D], uint16_t* dst) {
+  uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+  for (int c = 0; c < D / 8; ++c)
+    d4[c] = make_uint4(pack2(v[8 * c], v[8 * c + 1]), pack2(v[8 * c + 2], v[8 * c + 3]),
+                       pack2(v[8 * c + 4], v[8 * c + 5]), pack2(v[8 * c + 6], v[8 * c + 7]));
+}
+
+// Row-wise epilogues with the whole row in registers (N = D columns).
+template <int D>
+__device__ void epi_row(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
+  const BtArgs& a = *e.a;
+  const BtDims& d = a.d;
+  const int mode = e.c->mode;
+  const int r = a.slot;
+  const int L = seq_len_of(a, w.b);
+  int p, t;
+  if (mode == kBtIn) {   // rows of the 3-D box: head-major within the tile
+    p = row / d.tau;
+    t = row - p * d.tau;
+  } else {               // rows of the row space: token-major
+    t = row / d.P;
+    p = row - t * d.P;
+  }
+  const bool valid = p < d.P && t < w.ntok && w.s0 + t < L;
+  const int64_t grow =
+      int64_t(w.g) * d.R + (int64_t(w.b) * d.S + w.s0 + t) * d.P + p;   // row of this thread
+  float v[D];
+  float mean = 0.f, m2 = 0.f;
+  if (mode == kBtIn) {
+    // layer norm of the source row (d_s values), then GELU of the folded product
+    float mu = 0.f, rs = 0.f;
+    if (valid) {
+      const int x = w.g / d.E;
+      const uint16_t* xr = static_cast<const uint16_t*>(a.src[x]) +
+                           (((int64_t(a.src_layer[r]) * d.B + w.b) * d.P + p) * d.S + w.s0 + t) *
+                               d.d_s;
+      const uint4* x4 = reinterpret_cast<const uint4*>(xr);
+      float s = 0.f;
+      for (int c = 0; c < d.d_s / 8; ++c) {
+        const uint4 u = __ldg(x4 + c);
+        s += bf16_lo(u.x) + bf16_hi(u.x) + bf16_lo(u.y) + bf16_hi(u.y) + bf16_lo(u.z) +
+             bf16_hi(u.z) + bf16_lo(u.w) + bf16_hi(u.w);
+      }
+      mu = s / d.d_s;
+      float q = 0.f;
+      for (int c = 0; c < d.d_s / 8; ++c) {
+        const uint4 u = __ldg(x4 + c);
+        const float f[8] = {bf16_lo(u.x), bf16_hi(u.x), bf16_lo(u.y), bf16_hi(u.y),
+                            bf16_lo(u.z), bf16_hi(u.z), bf16_lo(u.w), bf16_hi(u.w)};
+#pragma unroll
+        for (int k = 0; k < 8; ++k) q = fmaf(f[k] - mu, f[k] - mu, q);
+      }
+      rs = rsqrtf(q / d.d_s + kLnEps);
+    }
+    __syncwarp();   // converge before the warp-collective TMEM loads
+    load_row<D>(tb, v);
+    const float* sw = a.s_in + int64_t(w.g) * D;
+    const float* cb = a.c_in + int64_t(w.g) * D;
+#pragma unroll
+    for (int k = 0; k < D; ++k) v[k] = gelu_erf(fmaf(v[k] - mu * __ldg(sw + k), rs, __ldg(cb + k)));
+    row_stats<D>(v, mean, m2);
+    if (valid) {
+      const float rstd = rsqrtf(m2 * (1.f / D) + kLnEps);
+      const int64_t ln = (int64_t(w.g) * d.N + r) * 2 * D;
+      store_norm<D>(v, mean, rstd, a.ln_c + ln, static_cast<uint16_t*>(a.xz) + grow * D);
+      if (r == 0) {   // h_0 = z_1, and slot 0's queries read LN_Q(h_0)
+        store_f32<D>(v, a.h + grow * D);
+        store_norm<D>(v, mean, rstd, a.ln_q + ln, static_cast<uint16_t*>(a.xq) + grow * D);
+      }
+    }
+    return;
+  }
+  load_row<D>(tb, v);
+  if (mode == kBtO) {
+    add_bias<D>(v, a.c_o + (int64_t(w.g) * d.N + r) * D);
+    if (valid) add_f32<D>(v, a.h + grow * D);
+    row_stats<D>(v, mean, m2);
+    if (valid) {
+      store_f32<D>(v, a.ht + grow * D);
+      store_norm<D>(v, mean, rsqrtf(m2 * (1.f / D) + kLnEps),
+                    a.ln_f + (int64_t(w.g) * d.N + r) * 2 * D,
+                    static_cast<uint16_t*>(a.xf) + grow * D);
+    }
+    return;
+  }
+  // kBtF2: the new state, its row norm (next slot's queries), the raw row for
+  // the output projection and the row's statistics for its token norm
+  add_bias<D>(v, a.c_f2 + (int64_t(w.g) * d.N + r) * D);
+  if (valid) add_f32<D>(v, a.ht + grow * D);
+  row_stats<D>(v, mean, m2);
+  if (valid) {
+    if (r + 1 < d.N) {
+      store_f32<D>(v, a.h + grow * D);
+      store_norm<D>(v, mean, rsqrtf(m2 * (1.f / D) + kLnEps),
+                    a.ln_q + (int64_t(w.g) * d.N + r + 1) * 2 * D,
+                    static_cast<uint16_t*>(a.xq) + grow * D);
+    }
+    store_bf16<D>(v, static_cast<uint16_t*>(a.xo) + grow * D);
+    a.rstat[grow] = make_float2(mean, m2);
+  }
+}
+
+// Plain epilogues, 32 columns at a time: bias (+ GELU), bf16 out.
+__device__ void epi_plain(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
+  const BtArgs& a = *e.a;
+  const GemmCfg& c = *e.c;
+  const BtDims& d = a.d;
+  const int r = a.slot;
+  const int t = row / d.P, p = row - t * d.P;
+  const bool valid = t < w.ntok && w.s0 + t < seq_len_of(a, w.b);
+  const int64_t grow = int64_t(w.g) * d.R + (int64_t(w.b) * d.S + w.s0 + t) * d.P + p;
+  const int N = c.NT * c.n_tiles;   // output row width
+  const float* bias;
+  uint16_t* out;
+  if (c.mode == kBtQ) {
+    bias = a.c_q + (int64_t(w.g) * d.N + r) * N;
+    out = static_cast<uint16_t*>(a.q);
+  } else if (c.mode == kBtKV) {
+    bias = a.c_kv + (int64_t(w.g) * d.N + r) * N;
+    out = static_cast<uint16_t*>(a.kv);
+  } else {
+    bias = a.c_f1 + (int64_t(w.g) * d.N + r) * N;
+    out = static_cast<uint16_t*>(a.f);
+  }
+  const bool gelu = c.mode == kBtF1;
+  for (int ch = 0; ch < c.NT / 32; ++ch) {
+    uint32_t rr[32];
+    __syncwarp();
+    tmem_ld_32x32b_x32(tb + ch * 32, rr);
+    tmem_ld_wait(rr);
+    if (!valid) continue;
+    const int col = w.j * c.NT + ch * 32;
+    const float4* b4 = reinterpret_cast<const float4*>(bias + col);
+    uint4* o4 = reinterpret_cast<uint4*>(out + grow * N + col);
+#pragma unroll
+    for (int q8 = 0; q8 < 4; ++q8) {
+      float f[8];
+      const float4 b0 = __ldg(b4 + 2 * q8), b1 = __ldg(b4 + 2 * q8 + 1);
+      const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        f[k] = __uint_as_float(rr[8 * q8 + k]) + bb[k];
+        if (gelu) f[k] = gelu_erf(f[k]);
+      }
+      o4[q8] = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]),
+                          pack2(f[6], f[7]));
+    }
+  }
+}
+
+// kBtOut: the E backbones' accumulators of this 128-token tile sit side by
+// side (E * NT columns); the gate-weighted sum goes to target layer q0 + r.
+__device__ void epi_out(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
+  const BtArgs& a = *e.a;
+  const GemmCfg& c = *e.c;
+  const BtDims& d = a.d;
+  const int x = w.g;   // kBtOut iterates the two K/V blocks
+  const int tok = w.tok0 + row;
+  const int b = tok / d.S, s = tok - b * d.S;
+  const bool valid = b < d.B && s < seq_len_of(a, b);
+  float gt[kMaxE], mu[kMaxE], rs[kMaxE];
+  for (int m = 0; m < d.E; ++m) {
+    gt[m] = valid ? a.gate[(int64_t(x) * d.B * d.S + tok) * d.E + m] : 0.f;
+    mu[m] = 0.f;
+    rs[m] = 0.f;
+    if (gt[m] == 0.f) continue;
+    // LN_out statistics over the token's P rows (Chan's combination of the
+    // per-row mean and M2, each over d values)
+    const float2* st = a.rstat + (int64_t(x) * d.E + m) * d.R + int64_t(tok) * d.P;
+    float tm = 0.f;
+    for (int k = 0; k < d.P; ++k) tm += st[k].x;
+    tm /= d.P;
+    float tq = 0.f;
+    for (int k = 0; k < d.P; ++k) {
+      const float2 sk = st[k];
+      tq += sk.y + d.d * (sk.x - tm) * (sk.x - tm);
+    }
+    mu[m] = tm;
+    rs[m] = rsqrtf(tq / (float(d.d) * d.P) + kLnEps);
+  }
+  uint16_t* dst = static_cast<uint16_t*>(a.dst[x]);
+  const int l = d.q0 + a.slot;
+  for (int ch = 0; ch < c.NT / 32; ++ch) {
+    float y[32];
+#pragma unroll
+    for (int k = 0; k < 32; ++k) y[k] = 0.f;
+    const int col = w.j * c.NT + ch * 32;
+    for (int m = 0; m < d.E; ++m) {
+      uint32_t rr[32];
+      __syncwarp();
+      tmem_ld_32x32b_x32(tb + m * c.NT + ch * 32, rr);
+      tmem_ld_wait(rr);
+      if (gt[m] == 0.f) continue;   // not kept for this token (or an invalid row)
+      const float* cb = a.c_out + (int64_t(x) * d.E + m) * d.Dt + col;
+      const float* sb = a.s_out + (int64_t(x) * d.E + m) * d.Dt + col;
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        const float u = fmaf(__uint_as_float(rr[k]) - mu[m] * __ldg(sb + k), rs[m], __ldg(cb + k));
+        y[k] = fmaf(gt[m], gelu_erf(u), y[k]);
+      }
+    }
+    if (!valid) continue;
+    const int hh = col / d.d_t, i0 = col - hh * d.d_t;
+    uint4* o4 = reinterpret_cast<uint4*>(
+        dst + (((int64_t(l) * d.B + b) * d.H_t + hh) * d.S + s) * d.d_t + i0);
+#pragma unroll
+    for (int q8 = 0; q8 < 4; ++q8)
+      o4[q8] = make_uint4(pack2(y[8 * q8], y[8 * q8 + 1]), pack2(y[8 * q8 + 2], y[8 * q8 + 3]),
+                          pack2(y[8 * q8 + 4], y[8 * q8 + 5]), pack2(y[8 * q8 + 6], y[8 * q8 + 7]));
+  }
+}
+
+// ---------------------------------------------------------------- the GEMM kernel
+
+template <int D>
+__global__ void __launch_bounds__(kBtThreads, 1)
+    bt_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
+                   const __grid_constant__ CUtensorMap tmB, const BtArgs a, const GemmCfg c) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + kBtStages * kBtABytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kBtStages * kBtStageBytes);
+  uint64_t* empty = full + kBtStages;
+  uint64_t* tfull = empty + kBtStages;   // [2]
+  uint64_t* tempty = tfull + 2;          // [2]
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const BtDims& d = a.d;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool is_out = c.mode == kBtOut;
+  const int n_exp = is_out ? d.E : 1;
+  const int nk = c.K / 64;
+  const int acc_cols = n_exp * c.NT;   // one accumulator buffer
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kBtStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmA2);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 2) {
+    tmem_alloc(tmem_slot, kBtTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int total = c.groups * c.row_tiles * c.n_tiles;
+  uint32_t issued_mask = 0, issue_parity = 0;
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      const uint32_t tx = c.a_box_bytes + c.NT * 128;
+      for (int it = blockIdx.x; it < total; it += gridDim.x) {
+        const Work w = decode(a, c, it);
+        if (!w.active) continue;
+        bool ok = true;
+        for (int kk = 0; kk < n_exp * nk; ++kk) {
+          const int m = kk / nk, kb = kk - m * nk;
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, a.wait_limit)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[stage], tx);
+          uint8_t* dA = sA + stage * kBtABytes;
+          uint8_t* dB = sB + stage * kBtBBytes;
+          const int kc = kb * 64;
+          const int64_t row0 = (int64_t(w.b) * d.S + w.s0) * d.P;
+          switch (c.mode) {
+            case kBtIn: {   // K blocks [0, d_s/64): hi weights, then the same source blocks x lo
+              const int x = w.g / d.E;
+              tma_load_3d(dA, x ? &tmA2 : &tmA, &full[stage], kc % d.d_s, w.s0,
+                          (a.src_layer[a.slot] * d.B + w.b) * d.P);
+              tma_load_2d(dB, &tmB, &full[stage], kc, w.g * c.b_rows_per_g + w.j * c.NT);
+              break;
+            }
+            case kBtOut: {
+              const int g = w.g * d.E + m;
+              tma_load_2d(dA, &tmA, &full[stage], kc,
+                          static_cast<int32_t>(int64_t(g) * d.B * d.S + w.tok0));
+              tma_load_2d(dB, &tmB, &full[stage], kc, g * c.b_rows_per_g + w.j * c.NT);
+              break;
+            }
+            default:
+              tma_load_2d(dA, &tmA, &full[stage], kc, static_cast<int32_t>(int64_t(w.g) * d.R + row0));
+              tma_load_2d(dB, &tmB, &full[stage], kc,
+                          (w.g * d.N + a.slot) * c.b_rows_per_g + w.j * c.NT);
+          }
+          issued_mask |= 1u << stage;
+          issue_parity = (issue_parity & ~(1u << stage)) | (phase << stage);
+          if (++stage == kBtStages) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer (warp-uniform loop, elected lane)
+    const uint32_t idesc = idesc_bf16_f32(128, c.NT);
+    int stage = 0;
+    uint32_t phase = 0;
+    int buf = 0;
+    uint32_t buf_phase = 0;
+    for (int it = blockIdx.x; it < total; it += gridDim.x) {
+      const Work w = decode(a, c, it);
+      if (!w.active) continue;
+      if (!mbar_wait(&tempty[buf], buf_phase ^ 1u, abort_flag, a.wait_limit)) break;
+      tc_fence_after();
+      bool ok = true;
+      for (int kk = 0; kk < n_exp * nk; ++kk) {
+        const int m = kk / nk, kb = kk - m * nk;
+        if (!mbar_wait(&full[stage], phase, abort_flag, a.wait_limit)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * acc_cols + m * c.NT);
+        const uint64_t adesc = sdesc_k_sw128(smem_u32(sA + stage * kBtABytes));
+        const uint64_t bdesc = sdesc_k_sw128(smem_u32(sB + stage * kBtBBytes));
+        if (elect_one()) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_bf16(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (kb | k) != 0);
+          umma_commit(&empty[stage]);
+        }
+        __syncwarp();
+        mma_issued = true;
+        if (++stage == kBtStages) { stage = 0; phase ^= 1u; }
+      }
+      if (!ok) break;
+      if (elect_one()) umma_commit(&tfull[buf]);
+      __syncwarp();
+      buf ^= 1;
+      if (buf == 0) buf_phase ^= 1u;
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------ epilogue
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    EpiCtx e{&a, &c};
+    int buf = 0;
+    uint32_t buf_phase = 0;
+    for (int it = blockIdx.x; it < total; it += gridDim.x) {
+      const Work w = decode(a, c, it);
+      if (!w.active) continue;
+      int ok = 1;
+      if (lane == 0) ok = mbar_wait(&tfull[buf], buf_phase, abort_flag, a.wait_limit) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      const uint32_t tb = tmem_base + static_cast<uint32_t>(buf * acc_cols) +
+                          (static_cast<uint32_t>(q * 32) << 16);
+      switch (c.mode) {
+        case kBtIn:
+        case kBtO:
+        case kBtF2: epi_row<D>(e, w, tb, row); break;
+        case kBtOut: epi_out(e, w, tb, row); break;
+        default: epi_plain(e, w, tb, row);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[buf]);
+      buf ^= 1;
+      if (buf == 0) buf_phase ^= 1u;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort_flag) {
+    // unwinding after a timed-out wait: let issued copies land and issued MMAs finish
+    if (warp == 0 && lane == 0) {
+      for (int s = 0; s < kBtStages; ++s)
+        if ((issued_mask >> s) & 1u) {
+          const uint32_t ad = smem_u32(&full[s]);
+          const long long t0 = clock64();
+          while (!mbar_try_wait(ad, (issue_parity >> s) & 1u) && clock64() - t0 < a.wait_limit) {
+          }
+        }
+    }
+    if (warp == 1 && mma_issued) {
+      if (elect_one()) umma_commit(drain);
+      __syncwarp();
+      const uint32_t ad = smem_u32(drain);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(ad, 0) && clock64() - t0 < a.wait_limit) {
+      }
+    }
+    __syncthreads();
+  }
+  if (warp == 2) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kBtTmemCols);
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicOr(a.status, kStatusTimeout);
+}
+
+// ---------------------------------------------------------------- gate (SIMT)
+//
+// One warp per token: logits_m = Wg[x][m] . window(token) + bg, the window
+// flattened slot-major then head-major (c = r * D_s + p * d_s + i); softmax in
+// fp32, then Top-K (ties to the lower index) and renormalisation. Also clamps
+// and reports sequence lengths outside [0, S].
+__global__ void __launch_bounds__(256) bt_gate_kernel(const BtArgs a) {
+  extern __shared__ uint4 wg_s[];   // [E][N * D_s] bf16 of block x
+  const BtDims& d = a.d;
+  const int x = blockIdx.y;
+  const int WD = d.N * d.Ds;
+  const uint4* wsrc = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(a.wg) +
+                                                     int64_t(x) * d.E * WD);
+  for (int i = threadIdx.x; i < d.E * WD / 8; i += blockDim.x) wg_s[i] = __ldg(wsrc + i);
+  if (blockIdx.x == 0 && blockIdx.y == 0)
+    for (int b = threadIdx.x; b < a.batch; b += blockDim.x) {
+      const int L = a.seq_lens[b];
+      if (L < 0 || L > d.S) atomicOr(a.status, kStatusSeqLen);
+    }
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_tok = d.B * d.S;
+  for (int tok = blockIdx.x * 8 + warp; tok < n_tok; tok += gridDim.x * 8) {
+    const int b = tok / d.S, s = tok - b * d.S;
+    if (s >= seq_len_of(a, b)) continue;
+    float acc[kMaxE];
+    for (int m = 0; m < d.E; ++m) acc[m] = 0.f;
+    for (int c8 = lane; c8 < WD / 8; c8 += 32) {
+      const int c = c8 * 8;
+      const int r = c / d.Ds, rem = c - r * d.Ds;
+      const int p = rem / d.d_s, i = rem - p * d.d_s;
+      const uint4 u = __ldg(reinterpret_cast<const uint4*>(
+          static_cast<const uint16_t*>(a.src[x]) +
+          (((int64_t(a.src_layer[r]) * d.B + b) * d.P + p) * d.S + s) * d.d_s + i));
+      const float xv[8] = {bf16_lo(u.x), bf16_hi(u.x), bf16_lo(u.y), bf16_hi(u.y),
+                           bf16_lo(u.z), bf16_hi(u.z), bf16_lo(u.w), bf16_hi(u.w)};
+      for (int m = 0; m < d.E; ++m) {
+        const uint4 wv = wg_s[(m * WD + c) / 8];
+        const float wf[8] = {bf16_lo(wv.x), bf16_hi(wv.x), bf16_lo(wv.y), bf16_hi(wv.y),
+                             bf16_lo(wv.z), bf16_hi(wv.z), bf16_lo(wv.w), bf16_hi(wv.w)};
+        float sacc = acc[m];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) sacc = fmaf(wf[k], xv[k], sacc);
+        acc[m] = sacc;
+      }
+    }
+    for (int m = 0; m < d.E; ++m)
+      for (int o = 16; o > 0; o >>= 1) acc[m] += __shfl_xor_sync(0xffffffffu, acc[m], o);
+    if (lane == 0) {
+      float g[kMaxE];
+      float mx = -INFINITY;
+      for (int m = 0; m < d.E; ++m) {
+        g[m] = acc[m] + a.bg[x * d.E + m];
+        mx = fmaxf(mx, g[m]);
+      }
+      float sum = 0.f;
+      for (int m = 0; m < d.E; ++m) {
+        g[m] = expf(g[m] - mx);
+        sum += g[m];
+      }
+      for (int m = 0; m < d.E; ++m) g[m] /= sum;
+      if (d.top_k > 0 && d.top_k < d.E) {
+        uint32_t keep = 0;
+        for (int k = 0; k < d.top_k; ++k) {
+          int best = -1;
+          for (int m = 0; m < d.E; ++m)
+            if (!((keep >> m) & 1u) && (best < 0 || g[m] > g[best])) best = m;
+          keep |= 1u << best;
+        }
+        float ks = 0.f;
+        for (int m = 0; m < d.E; ++m)
+          if ((keep >> m) & 1u) ks += g[m];
+        for (int m = 0; m < d.E; ++m) g[m] = ((keep >> m) & 1u) ? g[m] / ks : 0.f;
+      }
+      float* go = a.gate + (int64_t(x) * n_tok + tok) * d.E;
+      for (int m = 0; m < d.E; ++m) go[m] = g[m];
+    }
+  }
+}
+
+// ---------------------------------------------------------------- attention (SIMT)
+//
+// One thread per query row (token, p): for each head, scores against the
+// token's P key rows scaled by 1/sqrt(d/n_a), a max-subtracted softmax in fp32
+// and the weighted sum of the value rows.
+template <int DH>
+__global__ void __launch_bounds__(256) bt_attn_kernel(const BtArgs a) {
+  const BtDims& d = a.d;
+  const int g = blockIdx.y;
+  const int64_t row = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+  const int64_t n_rows = int64_t(d.B) * d.S * d.P;
+  if (row >= n_rows) return;
+  const int64_t tok = row / d.P;
+  const int b = static_cast<int>(tok / d.S), s = static_cast<int>(tok - int64_t(b) * d.S);
+  if (s >= seq_len_of(a, b)) return;
+  const int P = d.P, D = d.d;
+  const float scale = rsqrtf(static_cast<float>(DH));
+  const int64_t base = int64_t(g) * d.R + tok * P;   // first row of the token
+  const uint16_t* qr = static_cast<const uint16_t*>(a.q) + (int64_t(g) * d.R + row) * D;
+  const uint16_t* kvb = static_cast<const uint16_t*>(a.kv) + base * 2 * D;
+  uint16_t* orow = static_cast<uint16_t*>(a.o) + (int64_t(g) * d.R + row) * D;
+  for (int h = 0; h < d.na; ++h) {
+    float qv[DH];
+    const uint4* q4 = reinterpret_cast<const uint4*>(qr + h * DH);
+#pragma unroll
+    for (int c = 0; c < DH / 8; ++c) {
+      const uint4 u = q4[c];
+      qv[8 * c] = bf16_lo(u.x); qv[8 * c + 1] = bf16_hi(u.x);
+      qv[8 * c + 2] = bf16_lo(u.y); qv[8 * c + 3] = bf16_hi(u.y);
+      qv[8 * c + 4] = bf16_lo(u.z); qv[8 * c + 5] = bf16_hi(u.z);
+      qv[8 * c + 6] = bf16_lo(u.w); qv[8 * c + 7] = bf16_hi(u.w);
+    }
+    float sc[kBtMaxP];
+    float mx = -INFINITY;
+    for (int j = 0; j < P; ++j) {
+      const uint4* k4 = reinterpret_cast<const uint4*>(kvb + int64_t(j) * 2 * D + h * DH);
+      float sdot = 0.f;
+#pragma unroll
+      for (int c = 0; c < DH / 8; ++c) {
+        const uint4 u = k4[c];
+        sdot = fmaf(qv[8 * c], bf16_lo(u.x), sdot);
+        sdot = fmaf(qv[8 * c + 1], bf16_hi(u.x), sdot);
+        sdot = fmaf(qv[8 * c + 2], bf16_lo(u.y), sdot);
+        sdot = fmaf(qv[8 * c + 3], bf16_hi(u.y), sdot);
+        sdot = fmaf(qv[8 * c + 4], bf16_lo(u.z), sdot);
+        sdot = fmaf(qv[8 * c + 5], bf16_hi(u.z), sdot);
+        sdot = fmaf(qv[8 * c + 6], bf16_lo(u.w), sdot);
+        sdot = fmaf(qv[8 * c + 7], bf16_hi(u.w), sdot);
+      }
+      sc[j] = sdot * scale;
+      mx = fmaxf(mx, sc[j]);
+    }
+    float den = 0.f;
+    for (int j = 0; j < P; ++j) {
+      sc[j] = expf(sc[j] - mx);
+      den += sc[j];
+    }
+    const float inv = 1.f / den;
+    float ov[DH];
+#pragma unroll
+    for (int k = 0; k < DH; ++k) ov[k] = 0.f;
+    for (int j = 0; j < P; ++j) {
+      const uint4* v4 = reinterpret_cast<const uint4*>(kvb + int64_t(j) * 2 * D + D + h * DH);
+      const float wj = sc[j] * inv;
+#pragma unroll
+      for (int c = 0; c < DH / 8; ++c) {
+        const uint4 u = v4[c];
+        ov[8 * c] = fmaf(wj, bf16_lo(u.x), ov[8 * c]);
+        ov[8 * c + 1] = fmaf(wj, bf16_hi(u.x), ov[8 * c + 1]);
+        ov[8 * c + 2] = fmaf(wj, bf16_lo(u.y), ov[8 * c + 2]);
+        ov[8 * c + 3] = fmaf(wj, bf16_hi(u.y), ov[8 * c + 3]);
+        ov[8 * c + 4] = fmaf(wj, bf16_lo(u.z), ov[8 * c + 4]);
+        ov[8 * c + 5] = fmaf(wj, bf16_hi(u.z), ov[8 * c + 5]);
+        ov[8 * c + 6] = fmaf(wj, bf16_lo(u.w), ov[8 * c + 6]);
+        ov[8 * c + 7] = fmaf(wj, bf16_hi(u.w), ov[8 * c + 7]);
+      }
+    }
+    uint4* o4 = reinterpret_cast<uint4*>(orow + h * DH);
+#pragma unroll
+    for (int c = 0; c < DH / 8; ++c)
+      o4[c] = make_uint4(pack2(ov[8 * c], ov[8 * c + 1]), pack2(ov[8 * c + 2], ov[8 * c + 3]),
+                         pack2(ov[8 * c + 4], ov[8 * c + 5]), pack2(ov[8 * c + 6], ov[8 * c + 7]));
+  }
+}
+
+}  // namespace
+
+// Shapes the kernels take: bf16, P <= 16 heads of d_s in {64, 128}, width
+// d in {64, 128} with heads of 16, 32 or 64, d_f a multiple of 64 and of the
+// N tile, D_t a multiple of 32 with d_t % 32 == 0, E <= 8.
+bool bt_supported(const BtDims& d) {
+  const int dh = d.na > 0 ? d.d / d.na : 0;
+  return d.P >= 1 && d.P <= kBtMaxP && (d.d_s == 64 || d.d_s == 128) && (d.d == 64 || d.d == 128) &&
+         d.na > 0 && d.d % d.na == 0 && (dh == 16 || dh == 32 || dh == 64) && d.df % 64 == 0 &&
+         (d.df <= 256 || d.df % 256 == 0) && d.Dt % 32 == 0 && d.d_t % 32 == 0 && d.E >= 1 &&
+         d.E <= 8 && d.N >= 1 && d.N <= kBtMaxSlots && d.tau >= 1;
+}
+
+cudaError_t launch_bt_gate(const BtArgs& a, cudaStream_t st) {
+  const BtDims& d = a.d;
+  const size_t smem = size_t(d.E) * d.N * d.Ds * 2;
+  static size_t attr = 0;
+  if (smem > 48 * 1024 && smem > attr) {
+    cudaError_t e = cudaFuncSetAttribute(bt_gate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    attr = smem;
+  }
+  const int n_tok = d.B * d.S;
+  dim3 grid(std::min((n_tok + 7) / 8, 1024), 2);
+  bt_gate_kernel<<<grid, 256, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bt_attn(const BtArgs& a, cudaStream_t st) {
+  const BtDims& d = a.d;
+  const int64_t rows = int64_t(d.B) * d.S * d.P;
+  dim3 grid(static_cast<unsigned>((rows + 255) / 256), d.G);
+  switch (d.d / d.na) {
+    case 16: bt_attn_kernel<16><<<grid, 256, 0, st>>>(a); break;
+    case 32: bt_attn_kernel<32><<<grid, 256, 0, st>>>(a); break;
+    default: bt_attn_kernel<64><<<grid, 256, 0, st>>>(a); break;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bt_gemm(int mode, const BtArgs& a, const CUtensorMap& tmA,
+                           const CUtensorMap& tmA2, const CUtensorMap& tmB, int num_sms,
+                           cudaStream_t st) {
+  const BtDims& d = a.d;
+  GemmCfg c{};
+  c.mode = mode;
+  c.groups = d.G;
+  c.row_tiles = d.B * d.tiles_b;
+  c.a_box_bytes = kBtABytes;
+  c.n_tiles = 1;
+  switch (mode) {
+    case kBtIn:
+      c.K = 2 * d.d_s; c.NT = d.d; c.b_rows_per_g = d.d;
+      c.a_box_bytes = 64 * 2 * d.tau * d.P;
+      break;
+    case kBtQ: c.K = d.d; c.NT = d.d; c.b_rows_per_g = d.d; break;
+    case kBtKV: c.K = d.d; c.NT = 2 * d.d; c.b_rows_per_g = 2 * d.d; break;
+    case kBtO: c.K = d.d; c.NT = d.d; c.b_rows_per_g = d.d; break;
+    case kBtF1:
+      c.K = d.d; c.b_rows_per_g = d.df;
+      c.NT = d.df <= 256 ? d.df : 256;
+      c.n_tiles = d.df / c.NT;
+      break;
+    case kBtF2: c.K = d.df; c.NT = d.d; c.b_rows_per_g = d.d; break;
+    case kBtOut: {
+      c.K = d.P * d.d;
+      c.groups = 2;
+      c.b_rows_per_g = d.Dt;
+      int nt = 256 / d.E;
+      nt -= nt % 32;
+      while (nt > 32 && d.Dt % nt) nt -= 32;
+      c.NT = nt;
+      c.n_tiles = d.Dt / nt;
+      c.row_tiles = (d.B * d.S + 127) / 128;
+      break;
+    }
+    default: return cudaErrorInvalidValue;
+  }
+  if (c.NT < 32 || c.NT > 256 || c.NT % 32 || c.K % 64) return cudaErrorInvalidValue;
+  static bool attr_set[2] = {false, false};
+  const int di = d.d == 128 ? 1 : 0;
+  auto kern = d.d == 128 ? bt_gemm_kernel<128> : bt_gemm_kernel<64>;
+  if (!attr_set[di]) {
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kBtSmem);
+    if (e != cudaSuccess) return e;
+    attr_set[di] = true;
+  }
+  const long long items = static_cast<long long>(c.groups) * c.row_tiles * c.n_tiles;
+  const int grid = static_cast<int>(items < num_sms ? items : num_sms);
+  if (grid <= 0) return cudaSuccess;
+  kern<<<grid, kBtThreads, kBtSmem, st>>>(tmA, tmA2, tmB, a, c);
+  return cudaGetLastError();
+}
+
+}  // namespace mot

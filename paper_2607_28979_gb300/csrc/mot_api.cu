@@ -6,6 +6,7 @@
 #include <string.h>
 
 #include <algorithm>
+#include <cmath>
 #include <new>
 #include <string>
 #include <vector>
@@ -72,6 +73,36 @@ struct Ev {
 
 }  // namespace
 
+// Backbone-translator handles (kind 2): folded weights, the per-group row
+// space workspace and the tensor maps over them (bt.cu has the layouts).
+struct BtState {
+  BtDims d{};
+  int32_t src_layer[kBtMaxSlots] = {};
+  void* wg = nullptr;     // [2][E][N * Ds] bf16
+  float* bg = nullptr;    // [2][E]
+  float *s_in = nullptr, *c_in = nullptr, *c_q = nullptr, *c_kv = nullptr, *c_o = nullptr,
+        *c_f1 = nullptr, *c_f2 = nullptr, *c_out = nullptr, *s_out = nullptr, *ln_q = nullptr,
+        *ln_c = nullptr, *ln_f = nullptr;
+  // bf16 matrices: win [G][d][2 d_s] (hi | lo), wq [G][N][d][d], wkv [G][N][2d][d], wo [G][N][d][d],
+  // wf1 [G][N][df][d], wf2 [G][N][d][df], wout [G][Dt][P d]
+  void *win = nullptr, *wq = nullptr, *wkv = nullptr, *wo = nullptr, *wf1 = nullptr,
+       *wf2 = nullptr, *wout = nullptr;
+  float *gate = nullptr, *h = nullptr, *ht = nullptr;
+  void *xz = nullptr, *xq = nullptr, *q = nullptr, *kv = nullptr, *o = nullptr, *xf = nullptr,
+       *f = nullptr, *xo = nullptr;
+  float2* rstat = nullptr;
+  CUtensorMap tm_win{}, tm_wq{}, tm_wkv{}, tm_wo{}, tm_wf1{}, tm_wf2{}, tm_wout{};
+  CUtensorMap tm_xz{}, tm_xq{}, tm_o{}, tm_xf{}, tm_f{}, tm_xo{};
+
+  void free_all() {
+    void* ptrs[] = {wg, bg, s_in, c_in, c_q, c_kv, c_o, c_f1, c_f2, c_out, s_out, ln_q, ln_c,
+                    ln_f, win, wq, wkv, wo, wf1, wf2, wout, gate, h, ht, xz, xq, q, kv, o, xf,
+                    f, xo, rstat};
+    for (void* p : ptrs)
+      if (p) cudaFree(p);
+  }
+};
+
 struct mot_ctx {
   mot_config cfg{};
   std::vector<int32_t> layer_map;
@@ -119,6 +150,8 @@ struct mot_ctx {
   void* ahat = nullptr;         // [gp_h][B][S][d_at] bf16 translated activations
   int32_t* proj_layer = nullptr;   // [G] target layer of each group
   CUtensorMap tm_wkv{}, tm_ahat{};
+  // backbone translators (App. C.2): kind 2
+  BtState* bt = nullptr;
   // Top-K routing (tensor-core path, 0 < top_k < E): token buckets per expert
   bool sparse_ok = false;   // the shapes support it
   int routing = 0;          // 0 dense compute with a zeroed gate, 1 token buckets
@@ -165,6 +198,11 @@ void free_all(mot_ctx* h) {
                   h->st_dst[1], h->st_len};
   for (void* p : ptrs)
     if (p) cudaFree(p);
+  if (h->bt) {
+    h->bt->free_all();
+    delete h->bt;
+    h->bt = nullptr;
+  }
   for (auto& e : h->ev_used) { cudaEventDestroy(e.a); cudaEventDestroy(e.b); }
   for (int c = 0; c < kHostChunks; ++c) {
     if (h->ev_h2d[c]) cudaEventDestroy(h->ev_h2d[c]);
@@ -685,6 +723,292 @@ mot_status create_impl(const mot_config* cfg, const HSpec* hs, mot_handle* out) 
 
 }  // namespace
 
+namespace {
+
+// ---------------------------------------------------------------- backbone translators
+
+float bf16_bits_to_float(uint16_t b) {
+  const uint32_t u = uint32_t(b) << 16;
+  float f;
+  memcpy(&f, &u, 4);
+  return f;
+}
+
+uint16_t float_to_bf16_bits(float f) {   // round to nearest even (finite values)
+  uint32_t u;
+  memcpy(&u, &f, 4);
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return static_cast<uint16_t>(u >> 16);
+}
+
+// Elements of one K/V block of the backbone blob (see include/mot.h).
+size_t bt_block_elems(const BtDims& d) {
+  const size_t ds = d.d_s, D = d.d, df = d.df, P = d.P, Dt = d.Dt;
+  const size_t slot = 4 * D + 4 * (D * D + D) + 2 * D + (df * D + df) + (D * df + D);
+  const size_t expert = 2 * ds + D * ds + D + size_t(d.N) * slot + 2 * P * D + Dt * P * D + Dt;
+  return size_t(d.E) * d.N * d.Ds + d.E + d.E * expert;
+}
+
+mot_status bt_create(const mot_config* cfg, const mot_bt_config* bc, mot_handle* out) {
+  if (!out) return MOT_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg || !bc) return MOT_ERR_INVALID_ARG;
+  const mot_config& c = *cfg;
+  if (c.n_layers_src <= 0 || c.src_kv_heads <= 0 || c.src_head_dim <= 0 || c.n_layers_tgt <= 0 ||
+      c.tgt_kv_heads <= 0 || c.tgt_head_dim <= 0 || c.n_translators <= 0 || c.max_batch <= 0 ||
+      c.max_seq <= 0 || c.top_k < 0 || c.top_k > c.n_translators)
+    return MOT_ERR_INVALID_ARG;
+  if (bc->win_len <= 0 || bc->win_start < 0 || bc->win_start + bc->win_len > c.n_layers_tgt ||
+      bc->width <= 0 || bc->heads <= 0 || bc->ffn <= 0 || bc->width % bc->heads)
+    return MOT_ERR_INVALID_ARG;
+  if (c.dtype != MOT_BF16 && c.dtype != MOT_FP32) return MOT_ERR_INVALID_ARG;
+  std::vector<int32_t> map;
+  if (c.layer_map) {
+    for (int l = 0; l < c.n_layers_tgt; ++l)
+      if (c.layer_map[l] < -1 || c.layer_map[l] >= c.n_layers_src) return MOT_ERR_INVALID_ARG;
+    map.assign(c.layer_map, c.layer_map + c.n_layers_tgt);
+  } else {
+    depth_ratio(c.n_layers_src, c.n_layers_tgt, map);
+  }
+  if (c.dtype != MOT_BF16 || bc->win_len > kBtMaxSlots || c.max_batch > 4096)
+    return MOT_ERR_UNSUPPORTED;
+  for (int r = 0; r < bc->win_len; ++r)
+    if (map[bc->win_start + r] < 0) return MOT_ERR_UNSUPPORTED;   // every window layer mapped
+
+  BtDims bd{};
+  bd.L_s = c.n_layers_src; bd.P = c.src_kv_heads; bd.d_s = c.src_head_dim;
+  bd.L_t = c.n_layers_tgt; bd.H_t = c.tgt_kv_heads; bd.d_t = c.tgt_head_dim;
+  bd.E = c.n_translators; bd.top_k = c.top_k; bd.B = c.max_batch; bd.S = c.max_seq;
+  bd.Ds = bd.P * bd.d_s; bd.Dt = bd.H_t * bd.d_t;
+  bd.N = bc->win_len; bd.q0 = bc->win_start; bd.d = bc->width; bd.na = bc->heads; bd.df = bc->ffn;
+  bd.G = 2 * bd.E;
+  bd.tau = 128 / std::max(bd.P, 1);
+  bd.tiles_b = (bd.S + std::max(bd.tau, 1) - 1) / std::max(bd.tau, 1);
+  bd.R = int64_t(bd.B) * bd.S * bd.P;
+  if (!bt_supported(bd)) return MOT_ERR_UNSUPPORTED;
+  // tensor-map row coordinates are 32-bit
+  if (int64_t(bd.G) * bd.R > INT32_MAX / 2 ||
+      int64_t(bd.L_s) * bd.B * bd.P > INT32_MAX / 2)
+    return MOT_ERR_UNSUPPORTED;
+
+  mot_ctx* h = new (std::nothrow) mot_ctx();
+  if (!h) return MOT_ERR_OOM;
+  h->bt = new (std::nothrow) BtState();
+  if (!h->bt) {
+    delete h;
+    return MOT_ERR_OOM;
+  }
+  h->kind = 2;
+  h->cfg = c;
+  h->cfg.layer_map = nullptr;
+  h->layer_map = map;
+  Dims& d = h->d;   // the cache shapes, for the argument checks
+  d.L_s = bd.L_s; d.H_s = bd.P; d.d_s = bd.d_s; d.L_t = bd.L_t; d.H_t = bd.H_t; d.d_t = bd.d_t;
+  d.E = bd.E; d.top_k = bd.top_k; d.B = bd.B; d.S = bd.S; d.Ds = bd.Ds; d.Dt = bd.Dt;
+  d.dtype = 0;
+  BtState& bt = *h->bt;
+  bt.d = bd;
+  for (int r = 0; r < bd.N; ++r) bt.src_layer[r] = map[bd.q0 + r];
+
+  int dev = 0, cc_major = 0, cc_minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&cc_major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&cc_minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess) {
+    cudaGetLastError();
+    free_all(h);
+    delete h;
+    return MOT_ERR_CUDA;
+  }
+  h->device = dev;
+  if (cc_major != 10 || cc_minor != 3 || !encode_fn()) {
+    free_all(h);
+    delete h;
+    return MOT_ERR_UNSUPPORTED;
+  }
+  h->use_umma = true;
+
+  const size_t G = bd.G, N = bd.N, D = bd.d, df = bd.df, R = size_t(bd.R), E = bd.E;
+  struct A { void** p; size_t n; } allocs[] = {
+      {&bt.wg, 2 * E * N * bd.Ds * 2}, {(void**)&bt.bg, 2 * E * 4},
+      {(void**)&bt.s_in, G * D * 4}, {(void**)&bt.c_in, G * D * 4},
+      {(void**)&bt.c_q, G * N * D * 4}, {(void**)&bt.c_kv, G * N * 2 * D * 4},
+      {(void**)&bt.c_o, G * N * D * 4}, {(void**)&bt.c_f1, G * N * df * 4},
+      {(void**)&bt.c_f2, G * N * D * 4}, {(void**)&bt.c_out, G * bd.Dt * 4},
+      {(void**)&bt.s_out, G * bd.Dt * 4}, {(void**)&bt.rstat, G * R * 8},
+      {(void**)&bt.ln_q, G * N * 2 * D * 4}, {(void**)&bt.ln_c, G * N * 2 * D * 4},
+      {(void**)&bt.ln_f, G * N * 2 * D * 4},
+      {&bt.win, G * D * 2 * bd.d_s * 2}, {&bt.wq, G * N * D * D * 2}, {&bt.wkv, G * N * 2 * D * D * 2},
+      {&bt.wo, G * N * D * D * 2}, {&bt.wf1, G * N * df * D * 2}, {&bt.wf2, G * N * D * df * 2},
+      {&bt.wout, G * bd.Dt * bd.P * D * 2},
+      {(void**)&bt.gate, 2 * size_t(bd.B) * bd.S * E * 4},
+      {(void**)&bt.h, G * R * D * 4}, {(void**)&bt.ht, G * R * D * 4},
+      {&bt.xz, G * R * D * 2}, {&bt.xq, G * R * D * 2}, {&bt.q, G * R * D * 2},
+      {&bt.kv, G * R * 2 * D * 2}, {&bt.o, G * R * D * 2}, {&bt.xf, G * R * D * 2},
+      {&bt.f, G * R * df * 2}, {&bt.xo, G * R * D * 2},
+      {(void**)&h->status, 16}};
+  for (auto& a : allocs) {
+    if (cudaMalloc(a.p, std::max<size_t>(a.n, 16)) != cudaSuccess) {
+      cudaGetLastError();
+      free_all(h);
+      delete h;
+      return MOT_ERR_OOM;
+    }
+  }
+  if (cudaMemset(h->status, 0, 16) != cudaSuccess) {
+    cudaGetLastError();
+    free_all(h);
+    delete h;
+    return MOT_ERR_CUDA;
+  }
+  bool ok = true;
+  auto map2 = [&](CUtensorMap* m, void* base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
+    const uint64_t dims[2] = {inner, rows};
+    const uint64_t st_b[1] = {inner * 2};
+    const uint32_t box[2] = {64, box_rows};
+    ok = ok && encode_bf16(m, base, 2, dims, st_b, box);
+  };
+  // weights (B operands): box 64 x N-tile rows
+  const uint32_t nt_f1 = df <= 256 ? uint32_t(df) : 256u;
+  uint32_t nt_out = 256 / bd.E;
+  nt_out -= nt_out % 32;
+  while (nt_out > 32 && bd.Dt % nt_out) nt_out -= 32;
+  map2(&bt.tm_win, bt.win, 2 * bd.d_s, G * D, uint32_t(D));
+  map2(&bt.tm_wq, bt.wq, D, G * N * D, uint32_t(D));
+  map2(&bt.tm_wkv, bt.wkv, D, G * N * 2 * D, uint32_t(2 * D));
+  map2(&bt.tm_wo, bt.wo, D, G * N * D, uint32_t(D));
+  map2(&bt.tm_wf1, bt.wf1, D, G * N * df, nt_f1);
+  map2(&bt.tm_wf2, bt.wf2, df, G * N * D, uint32_t(D));
+  map2(&bt.tm_wout, bt.wout, uint64_t(bd.P) * D, G * bd.Dt, nt_out);
+  // activations (A operands): box 64 x 128 rows
+  map2(&bt.tm_xz, bt.xz, D, G * R, 128);
+  map2(&bt.tm_xq, bt.xq, D, G * R, 128);
+  map2(&bt.tm_o, bt.o, D, G * R, 128);
+  map2(&bt.tm_xf, bt.xf, D, G * R, 128);
+  map2(&bt.tm_f, bt.f, df, G * R, 128);
+  map2(&bt.tm_xo, bt.xo, uint64_t(bd.P) * D, G * size_t(bd.B) * bd.S, 128);
+  if (!ok) {
+    free_all(h);
+    delete h;
+    return MOT_ERR_CUDA;
+  }
+  *out = h;
+  return MOT_OK;
+}
+
+// Parse the backbone blob and upload it. LN_in and LN_out, whose inputs the
+// GEMMs read raw (the source cache, the bf16 state rows), are folded into the
+// map after them: for y = W LN(x) + b with LN(x) = gamma * xhat + beta,
+// y = W' xhat + c with W' = W diag(gamma), c = b + W beta. W_in' is kept as two
+// bf16 matrices hi + lo (hi = bf16(W'), lo = bf16(W' - hi)), so its product is
+// exact to about 2^-17; W_out' is rounded to bf16 once. The other layer norms'
+// gamma and beta are applied by the epilogues that write their rows, so W_Q,
+// W_K, W_V and W_F1 stay the blob's values.
+mot_status bt_load(mot_ctx* h, const void* host_blob, size_t bytes) {
+  BtState& bt = *h->bt;
+  const BtDims& d = bt.d;
+  const size_t blk = bt_block_elems(d);
+  if (bytes != 2 * blk * 2) return MOT_ERR_WEIGHTS_SIZE;
+  if (cudaSetDevice(h->device) != cudaSuccess) return MOT_ERR_CUDA;
+  const uint16_t* blob = static_cast<const uint16_t*>(host_blob);
+  const size_t E = d.E, N = d.N, D = d.d, df = d.df, ds = d.d_s, P = d.P, Dt = d.Dt;
+  const size_t G = d.G, WD = N * d.Ds;
+  std::vector<uint16_t> wg(2 * E * WD), win(G * D * 2 * ds), wq(G * N * D * D),
+      wkv(G * N * 2 * D * D), wo(G * N * D * D), wf1(G * N * df * D), wf2(G * N * D * df),
+      wout(G * Dt * P * D);
+  std::vector<float> bg(2 * E), s_in(G * D), c_in(G * D), c_q(G * N * D), c_kv(G * N * 2 * D),
+      c_o(G * N * D), c_f1(G * N * df), c_f2(G * N * D), c_out(G * Dt), s_out(G * Dt),
+      ln_q(G * N * 2 * D), ln_c(G * N * 2 * D), ln_f(G * N * 2 * D);
+  auto f = [&](size_t i) { return double(bf16_bits_to_float(blob[i])); };
+  // Folded rows: W'[n][k] = W[n][k] gamma[k] as hi (and lo, when w_lo is set)
+  // with row stride `ld`; c[n] = b[n] + sum_k W[n][k] beta[k]; rowsum = sum of
+  // the stored parts.
+  auto fold = [&](size_t o_g, size_t o_w, size_t o_b, size_t n_out, size_t n_in, size_t ld,
+                  uint16_t* w_hi, uint16_t* w_lo, float* c_dst, float* rowsum) {
+    for (size_t n = 0; n < n_out; ++n) {
+      double cb = f(o_b + n);
+      double rs = 0.0;
+      for (size_t k = 0; k < n_in; ++k) {
+        const double w = f(o_w + n * n_in + k);
+        const double wp = w * f(o_g + k);
+        const uint16_t hi = float_to_bf16_bits(float(wp));
+        w_hi[n * ld + k] = hi;
+        rs += bf16_bits_to_float(hi);
+        if (w_lo) {
+          const uint16_t lo = float_to_bf16_bits(float(wp - bf16_bits_to_float(hi)));
+          w_lo[n * ld + k] = lo;
+          rs += bf16_bits_to_float(lo);
+        }
+        cb += w * f(o_g + n_in + k);
+      }
+      c_dst[n] = float(cb);
+      if (rowsum) rowsum[n] = float(rs);
+    }
+  };
+  auto copy = [&](size_t o_w, size_t o_b, size_t n_out, size_t n_in, uint16_t* w_dst, float* b_dst) {
+    memcpy(w_dst, blob + o_w, n_out * n_in * 2);
+    for (size_t n = 0; n < n_out; ++n) b_dst[n] = float(f(o_b + n));
+  };
+  auto ln = [&](size_t o_g, float* dst) {   // gamma[D], beta[D]
+    for (size_t k = 0; k < 2 * D; ++k) dst[k] = float(f(o_g + k));
+  };
+  for (size_t x = 0; x < 2; ++x) {
+    size_t off = x * blk;
+    memcpy(&wg[x * E * WD], blob + off, E * WD * 2);
+    off += E * WD;
+    for (size_t m = 0; m < E; ++m) bg[x * E + m] = float(f(off + m));
+    off += E;
+    for (size_t m = 0; m < E; ++m) {
+      const size_t g = x * E + m;
+      const size_t o_lnin = off, o_win = o_lnin + 2 * ds, o_bin = o_win + D * ds;
+      uint16_t* wi = &win[g * D * 2 * ds];
+      fold(o_lnin, o_win, o_bin, D, ds, 2 * ds, wi, wi + ds, &c_in[g * D], &s_in[g * D]);
+      off = o_bin + D;
+      for (size_t r = 0; r < N; ++r) {
+        const size_t gr = g * N + r;
+        const size_t o_lnq = off, o_lnc = off + 2 * D, o_wq = off + 4 * D, o_bq = o_wq + D * D;
+        const size_t o_wk = o_bq + D, o_bk = o_wk + D * D, o_wv = o_bk + D, o_bv = o_wv + D * D;
+        const size_t o_wo = o_bv + D, o_bo = o_wo + D * D, o_lnf = o_bo + D;
+        const size_t o_wf1 = o_lnf + 2 * D, o_bf1 = o_wf1 + df * D, o_wf2 = o_bf1 + df;
+        const size_t o_bf2 = o_wf2 + D * df;
+        ln(o_lnq, &ln_q[gr * 2 * D]);
+        ln(o_lnc, &ln_c[gr * 2 * D]);
+        ln(o_lnf, &ln_f[gr * 2 * D]);
+        copy(o_wq, o_bq, D, D, &wq[gr * D * D], &c_q[gr * D]);
+        copy(o_wk, o_bk, D, D, &wkv[gr * 2 * D * D], &c_kv[gr * 2 * D]);
+        copy(o_wv, o_bv, D, D, &wkv[gr * 2 * D * D + D * D], &c_kv[gr * 2 * D + D]);
+        copy(o_wo, o_bo, D, D, &wo[gr * D * D], &c_o[gr * D]);
+        copy(o_wf1, o_bf1, df, D, &wf1[gr * df * D], &c_f1[gr * df]);
+        copy(o_wf2, o_bf2, D, df, &wf2[gr * D * df], &c_f2[gr * D]);
+        off = o_bf2 + D;
+      }
+      const size_t o_lnout = off, o_wout = o_lnout + 2 * P * D, o_bout = o_wout + Dt * P * D;
+      fold(o_lnout, o_wout, o_bout, Dt, P * D, P * D, &wout[g * Dt * P * D], nullptr,
+           &c_out[g * Dt], &s_out[g * Dt]);
+      off = o_bout + Dt;
+    }
+    if (off != (x + 1) * blk) return MOT_ERR_WEIGHTS_SIZE;   // layout bookkeeping check
+  }
+  struct U { void* dst; const void* src; size_t n; } ups[] = {
+      {bt.wg, wg.data(), wg.size() * 2}, {bt.bg, bg.data(), bg.size() * 4},
+      {bt.win, win.data(), win.size() * 2}, {bt.s_in, s_in.data(), s_in.size() * 4},
+      {bt.c_in, c_in.data(), c_in.size() * 4}, {bt.wq, wq.data(), wq.size() * 2},
+      {bt.c_q, c_q.data(), c_q.size() * 4}, {bt.wkv, wkv.data(), wkv.size() * 2},
+      {bt.c_kv, c_kv.data(), c_kv.size() * 4}, {bt.wo, wo.data(), wo.size() * 2},
+      {bt.c_o, c_o.data(), c_o.size() * 4}, {bt.wf1, wf1.data(), wf1.size() * 2},
+      {bt.c_f1, c_f1.data(), c_f1.size() * 4}, {bt.wf2, wf2.data(), wf2.size() * 2},
+      {bt.c_f2, c_f2.data(), c_f2.size() * 4}, {bt.wout, wout.data(), wout.size() * 2},
+      {bt.c_out, c_out.data(), c_out.size() * 4}, {bt.s_out, s_out.data(), s_out.size() * 4},
+      {bt.ln_q, ln_q.data(), ln_q.size() * 4}, {bt.ln_c, ln_c.data(), ln_c.size() * 4},
+      {bt.ln_f, ln_f.data(), ln_f.size() * 4}};
+  for (auto& u : ups) MOT_CUDA_TRY(cudaMemcpy(u.dst, u.src, u.n, cudaMemcpyHostToDevice));
+  MOT_CUDA_TRY(cudaDeviceSynchronize());
+  h->weights_loaded = true;
+  return MOT_OK;
+}
+
+}  // namespace
+
 extern "C" {
 
 mot_status mot_create(const mot_config* cfg, mot_handle* out) {
@@ -718,6 +1042,7 @@ mot_status mot_create_h(const mot_h_config* cfg, mot_handle* out) {
 
 mot_status mot_load_weights(mot_handle h, const void* host_blob, size_t bytes) {
   if (!h || !host_blob) return MOT_ERR_INVALID_ARG;
+  if (h->kind == 2) return bt_load(h, host_blob, bytes);
   const Dims& d = h->d;
   const size_t es = esize(d), gsz = group_elems(d);
   // MoT-h blocks: the mixture, then the layer's W^K and W^V [D_t][d_at]
@@ -1018,6 +1343,86 @@ mot_status mot_translate_h(mot_handle h, const void* src_act, const int32_t* seq
     a.gp = g1 - g0;
     MOT_CUDA_TRY(timed(h, "umma2_proj", st, [&] {
       return launch_umma2_proj(a, h->tm_ahat, h->tm_wkv, h->act_tgt, h->num_sms, st);
+    }));
+  }
+  return MOT_OK;
+}
+
+mot_status mot_create_bt(const mot_config* cfg, const mot_bt_config* bt, mot_handle* out) {
+  return bt_create(cfg, bt, out);
+}
+
+mot_status mot_translate_bt(mot_handle h, const void* src_k, const void* src_v,
+                            const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
+                            mot_stream_t stream) {
+  if (!h || h->kind != 2) return MOT_ERR_INVALID_ARG;
+  const Dims& dd = h->d;
+  if (batch < 0 || batch > dd.B) return MOT_ERR_INVALID_ARG;
+  if (!src_k || !src_v || !dst_k || !dst_v || (batch > 0 && !seq_lens)) return MOT_ERR_INVALID_ARG;
+  if (!aligned16(src_k) || !aligned16(src_v) || !aligned16(dst_k) || !aligned16(dst_v))
+    return MOT_ERR_INVALID_ARG;
+  const size_t sb = src_bytes(dd), db = dst_bytes(dd);
+  if (overlap(dst_k, db, dst_v, db) || overlap(dst_k, db, src_k, sb) ||
+      overlap(dst_k, db, src_v, sb) || overlap(dst_v, db, src_k, sb) ||
+      overlap(dst_v, db, src_v, sb))
+    return MOT_ERR_INVALID_ARG;
+  if (!h->weights_loaded) return MOT_ERR_NO_WEIGHTS;
+  if (cudaSetDevice(h->device) != cudaSuccess) return MOT_ERR_CUDA;
+  if (batch == 0) return MOT_OK;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  BtState& bt = *h->bt;
+  const BtDims& d = bt.d;
+  BtArgs a{};
+  a.d = d;
+  a.src[0] = src_k;
+  a.src[1] = src_v;
+  a.dst[0] = dst_k;
+  a.dst[1] = dst_v;
+  a.seq_lens = seq_lens;
+  a.batch = batch;
+  for (int r = 0; r < d.N; ++r) a.src_layer[r] = bt.src_layer[r];
+  a.wg = bt.wg; a.bg = bt.bg; a.s_in = bt.s_in; a.c_in = bt.c_in; a.c_q = bt.c_q;
+  a.c_kv = bt.c_kv; a.c_o = bt.c_o; a.c_f1 = bt.c_f1; a.c_f2 = bt.c_f2; a.c_out = bt.c_out;
+  a.s_out = bt.s_out; a.rstat = bt.rstat;
+  a.ln_q = bt.ln_q; a.ln_c = bt.ln_c; a.ln_f = bt.ln_f;
+  a.gate = bt.gate; a.xz = bt.xz; a.xq = bt.xq; a.h = bt.h; a.ht = bt.ht; a.q = bt.q;
+  a.kv = bt.kv; a.o = bt.o; a.xf = bt.xf; a.f = bt.f; a.xo = bt.xo;
+  a.status = h->status;
+  a.wait_limit = h->wait_limit;
+  // the source caches as 3-D tensors (d_s, S, L_s * B * H_s), box (64, tau, P)
+  CUtensorMap tmK{}, tmV{};
+  {
+    const uint64_t dims[3] = {uint64_t(d.d_s), uint64_t(d.S), uint64_t(d.L_s) * d.B * d.P};
+    const uint64_t st_b[2] = {uint64_t(d.d_s) * 2, uint64_t(d.S) * d.d_s * 2};
+    const uint32_t box[3] = {64, uint32_t(d.tau), uint32_t(d.P)};
+    if (!encode_bf16(&tmK, src_k, 3, dims, st_b, box) ||
+        !encode_bf16(&tmV, src_v, 3, dims, st_b, box))
+      return MOT_ERR_CUDA;
+  }
+  MOT_CUDA_TRY(timed(h, "bt_gate", st, [&] { return launch_bt_gate(a, st); }));
+  for (int r = 0; r < d.N; ++r) {
+    a.slot = r;
+    MOT_CUDA_TRY(timed(h, "bt_in_ln_gelu", st, [&] {
+      return launch_bt_gemm(kBtIn, a, tmK, tmV, bt.tm_win, h->num_sms, st);
+    }));
+    MOT_CUDA_TRY(timed(h, "bt_q", st, [&] {
+      return launch_bt_gemm(kBtQ, a, bt.tm_xq, bt.tm_xq, bt.tm_wq, h->num_sms, st);
+    }));
+    MOT_CUDA_TRY(timed(h, "bt_kv", st, [&] {
+      return launch_bt_gemm(kBtKV, a, bt.tm_xz, bt.tm_xz, bt.tm_wkv, h->num_sms, st);
+    }));
+    MOT_CUDA_TRY(timed(h, "bt_attn", st, [&] { return launch_bt_attn(a, st); }));
+    MOT_CUDA_TRY(timed(h, "bt_o_residual_ln", st, [&] {
+      return launch_bt_gemm(kBtO, a, bt.tm_o, bt.tm_o, bt.tm_wo, h->num_sms, st);
+    }));
+    MOT_CUDA_TRY(timed(h, "bt_ffn1_gelu", st, [&] {
+      return launch_bt_gemm(kBtF1, a, bt.tm_xf, bt.tm_xf, bt.tm_wf1, h->num_sms, st);
+    }));
+    MOT_CUDA_TRY(timed(h, "bt_ffn2_residual_ln", st, [&] {
+      return launch_bt_gemm(kBtF2, a, bt.tm_f, bt.tm_f, bt.tm_wf2, h->num_sms, st);
+    }));
+    MOT_CUDA_TRY(timed(h, "bt_out_gelu_combine", st, [&] {
+      return launch_bt_gemm(kBtOut, a, bt.tm_xo, bt.tm_xo, bt.tm_wout, h->num_sms, st);
     }));
   }
   return MOT_OK;

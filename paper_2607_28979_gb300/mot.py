@@ -54,6 +54,11 @@ class mot_h_config(ctypes.Structure):
                 ("layer_map", ctypes.POINTER(ctypes.c_int32))]
 
 
+class mot_bt_config(ctypes.Structure):
+    _fields_ = [("win_start", ctypes.c_int32), ("win_len", ctypes.c_int32),
+                ("width", ctypes.c_int32), ("heads", ctypes.c_int32), ("ffn", ctypes.c_int32)]
+
+
 class mot_kernel_stat(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char * 32), ("launches", ctypes.c_int64),
                 ("total_ms", ctypes.c_double)]
@@ -86,6 +91,9 @@ _SIGS = {
     "mot_debug_set": [_H, ctypes.c_int32, ctypes.c_int64],
     "mot_translate_static": [ctypes.POINTER(mot_config), _P, _P, _P, _P, ctypes.c_int32, _P, _P,
                              _P],
+    "mot_create_bt": [ctypes.POINTER(mot_config), ctypes.POINTER(mot_bt_config),
+                      ctypes.POINTER(ctypes.c_void_p)],
+    "mot_translate_bt": [_H, _P, _P, _P, ctypes.c_int32, _P, _P, _P],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -197,6 +205,24 @@ def mot_create_h(cfg: mot_h_config) -> Handle:
 def mot_translate_h(h: Handle, src_act, seq_lens, batch: int, dst_k, dst_v, stream=None) -> None:
     _check(_lib.mot_translate_h(h.ptr, _addr(src_act), _addr(seq_lens), int(batch), _addr(dst_k),
                                 _addr(dst_v), _stream(stream)), "mot_translate_h")
+
+
+def bt_config_from(wl):
+    """(mot_config, mot_bt_config) for a Workload with backbone translators (``bt``)."""
+    return config_from(wl), mot_bt_config(*wl.bt)
+
+
+def mot_create_bt(cfg: mot_config, bt: mot_bt_config) -> Handle:
+    out = ctypes.c_void_p()
+    _check(_lib.mot_create_bt(ctypes.byref(cfg), ctypes.byref(bt), ctypes.byref(out)),
+           "mot_create_bt")
+    return Handle(out.value, cfg.n_layers_tgt)
+
+
+def mot_translate_bt(h: Handle, src_k, src_v, seq_lens, batch: int, dst_k, dst_v,
+                     stream=None) -> None:
+    _check(_lib.mot_translate_bt(h.ptr, _addr(src_k), _addr(src_v), _addr(seq_lens), int(batch),
+                                 _addr(dst_k), _addr(dst_v), _stream(stream)), "mot_translate_bt")
 
 
 def mot_create(cfg: mot_config) -> Handle:

@@ -45,6 +45,14 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 def workload_desc(wl) -> str:
     gate = ("dense softmax gate" if wl.top_k in (0, wl.n_translators)
             else f"softmax gate, Top-{wl.top_k} routing")
+    if wl.is_bt:
+        q, N, d, na, df = wl.bt
+        return (f"{wl.name}: backbone translators (App. C.2), {wl.n_layers_src}L "
+                f"{wl.src_kv_heads}x{wl.src_head_dim} -> {wl.n_layers_tgt}L "
+                f"{wl.tgt_kv_heads}x{wl.tgt_head_dim}, window = target layers {q}..{q + N - 1}, "
+                f"E={wl.n_translators} backbones (rows of width {d}, {na} heads over the "
+                f"{wl.src_kv_heads} source heads, FFN {df}), {gate} on the window, {wl.dtype}, "
+                f"batch {wl.batch} seq_lens {list(wl.seq_lens)}")
     if wl.is_h:
         return (f"{wl.name}: MoT-h, activations {wl.n_layers_src}L x {wl.src_head_dim} -> "
                 f"{wl.n_layers_tgt}L x {wl.act_tgt}, E={wl.n_translators} MLP "
@@ -57,9 +65,56 @@ def workload_desc(wl) -> str:
             f"batch {wl.batch} seq_lens {list(wl.seq_lens)}")
 
 
+def algorithmic_bt(wl, layer_map):
+    """FLOPs and bytes the backbone-translator method needs per step, and the
+    FLOPs of each kernel per launch (one launch covers both K/V blocks and all
+    backbones of one window slot)."""
+    T, E, Ds, Dt, P, ds = (wl.tokens, wl.n_translators, wl.d_src, wl.d_tgt, wl.src_kv_heads,
+                           wl.src_head_dim)
+    q, N, d, na, df = wl.bt
+    Ea = wl.top_k if 0 < wl.top_k < E else E
+    rows = 2 * Ea * T * P            # (K/V, backbone, token, source head) rows of one slot
+    per_launch = {
+        "bt_in_ln_gelu": rows * 2 * ds * d,
+        "bt_q": rows * 2 * d * d,
+        "bt_kv": rows * 2 * d * 2 * d,
+        "bt_attn": rows * P * 4 * d,
+        "bt_o_residual_ln": rows * 2 * d * d,
+        "bt_ffn1_gelu": rows * 2 * d * df,
+        "bt_ffn2_residual_ln": rows * 2 * df * d,
+        "bt_out_gelu_combine": 2 * Ea * T * 2 * P * d * Dt,
+        "bt_gate": 2 * T * 2 * N * Ds * E,
+    }
+    flops = per_launch["bt_gate"] + N * sum(v for k, v in per_launch.items() if k != "bt_gate")
+    # bytes each kernel must move per launch in this unfused schedule (its operand
+    # rows in and result rows out; a slot after the first): its own HBM roofline
+    es = wl.esize
+    allrows = 2 * E * T * P
+    bpl = {
+        "bt_in_ln_gelu": 2 * E * T * Ds * es + allrows * d * 2,
+        "bt_q": allrows * d * 2 * 2,
+        "bt_kv": allrows * (d + 2 * d) * 2,
+        "bt_attn": allrows * (3 * d + d) * 2,
+        "bt_o_residual_ln": allrows * (d * 2 + d * 4 + d * 4 + d * 2),
+        "bt_ffn1_gelu": allrows * (d + df) * 2,
+        "bt_ffn2_residual_ln": allrows * (df * 2 + d * 4 + d * 4 + d * 2 + d * 2 + 8),
+        "bt_out_gelu_combine": allrows * (d * 2 + 8) + 2 * T * Dt * es,
+        "bt_gate": 2 * N * T * Ds * es,
+    }
+    src_layers = {layer_map[t] for t in range(q, q + N)}
+    bytes_src = 2 * len(src_layers) * T * Ds * es
+    bytes_dst = 2 * N * T * Dt * es
+    bytes_w = wl.blob_elems() * es
+    return dict(flops=flops, per_launch=per_launch, bytes_per_launch=bpl,
+                bytes=bytes_src + bytes_dst + bytes_w,
+                bytes_src=bytes_src, bytes_dst=bytes_dst, bytes_w=bytes_w)
+
+
 def algorithmic(wl, layer_map):
     """FLOPs and bytes the method needs per step (no intermediate traffic).
     ``layer_map``: the channel map in use (source layer per target layer, -1 = none)."""
+    if wl.is_bt:
+        return algorithmic_bt(wl, layer_map)
     T, E, Ds, Dt, Hh, Dm = wl.tokens, wl.n_translators, wl.d_src, wl.d_tgt, wl.hidden, wl.d_mix
     n_tl = len(wl.translated_layers())
     groups = n_tl if wl.is_h else 2 * n_tl   # MoT-h: one mixture per layer
@@ -217,7 +272,9 @@ def cpu_oracle_rate(wl, sk, sv, blob, budget_s: float, seed: int = 3):
         s = np.array([rng.integers(0, wl.seq_lens[i]) for i in b])
         return b.astype(np.int32), s.astype(np.int32)
     def run(tb, ts):
-        if wl.is_h:
+        if wl.is_bt:
+            oracle.bt_tokens(wl, sk, sv, blob, tb, ts)
+        elif wl.is_h:
             oracle.translate_h_tokens(wl, sk, blob, tb, ts)
         else:
             oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
@@ -255,7 +312,9 @@ def run_reference(args, wl):
     sv = sk if wl.is_h else synth.gen_cache(wl, 1)
 
     def run(tb, ts):
-        if wl.is_h:
+        if wl.is_bt:
+            oracle.bt_tokens(wl, sk, sv, blob, tb, ts)
+        elif wl.is_h:
             oracle.translate_h_tokens(wl, sk, blob, tb, ts)
         else:
             oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
@@ -286,7 +345,8 @@ def run_reference(args, wl):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded SplitMix64/Box-Muller caches and weights)",
         "config": {"workload": workload_desc(wl), "tokens_per_step": n,
-                   "sample": f"{n} random tokens of the workload per step, all translated layers"},
+                   "sample": f"{n} random tokens of the workload per step, all "
+                             f"{'window' if wl.is_bt else 'translated'} layers"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": omp_cores(), "kind": "oracle",
                          "sample": f"{n} tokens per step x {args.steps} steps"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -311,15 +371,22 @@ def run_mot(args, wl):
 
     sk_h, blob = synth.gen_cache(wl, 0), synth.gen_weights(wl)
     sv_h = sk_h if wl.is_h else synth.gen_cache(wl, 1)   # MoT-h: one activation tensor
-    h = M.mot_create_h(M.h_config_from(wl)) if wl.is_h else M.mot_create(M.config_from(wl))
+    if wl.is_bt:
+        h = M.mot_create_bt(*M.bt_config_from(wl))
+    elif wl.is_h:
+        h = M.mot_create_h(M.h_config_from(wl))
+    else:
+        h = M.mot_create(M.config_from(wl))
     M.mot_load_weights(h, blob)
     path = M.mot_get_path(h)
     names = {0: "split", 1: "fused", 2: "pair", 3: "onchip"}
-    if args.schedule != "auto":
+    if args.schedule != "auto" and not wl.is_bt:
         M.mot_set_schedule(h, {v: k for k, v in names.items()}[args.schedule])
     schedule = names[M.mot_get_schedule(h)]
     if M.mot_get_routing(h) == M.ROUTING_SPARSE:
         schedule = "routed (Top-K token buckets)"
+    if wl.is_bt:
+        schedule = "backbone scan (8 launches per window slot)"
     bf = wl.dtype == "bf16"
     tdt = torch.bfloat16 if bf else torch.float32
 
@@ -334,7 +401,9 @@ def run_mot(args, wl):
     B = wl.batch
 
     def step():
-        if wl.is_h:
+        if wl.is_bt:
+            M.mot_translate_bt(h, sk, sv, lens, B, dk, dv, stream)
+        elif wl.is_h:
             M.mot_translate_h(h, sk, lens, B, dk, dv, stream)
         else:
             M.mot_translate(h, sk, sv, lens, B, dk, dv, stream)
@@ -383,8 +452,23 @@ def run_mot(args, wl):
     es = wl.esize
     tl = len(wl.translated_layers())
 
+    lmap = M.mot_get_layer_map(h)
+    if wl.is_bt:
+        win = wl.bt_window
+        bt_src = sorted({lmap[t] for t in win})
+
     def e2e_step():
-        if wl.is_h:   # device entry point with the copies around it, on the same stream
+        if wl.is_bt:   # the window's source layers in, its target layers out, on one stream
+            with torch.cuda.stream(stream):
+                for l in bt_src:
+                    sk[l].view(torch.int16).copy_(hk[l], non_blocking=True)
+                    sv[l].view(torch.int16).copy_(hv[l], non_blocking=True)
+                M.mot_translate_bt(h, sk, sv, lens, B, dk, dv, stream)
+                ok[win[0]:win[-1] + 1].copy_(dk[win[0]:win[-1] + 1].view(torch.int16),
+                                             non_blocking=True)
+                ov[win[0]:win[-1] + 1].copy_(dv[win[0]:win[-1] + 1].view(torch.int16),
+                                             non_blocking=True)
+        elif wl.is_h:   # device entry point with the copies around it, on the same stream
             with torch.cuda.stream(stream):
                 sk.view(torch.int16).copy_(hk, non_blocking=True)
                 M.mot_translate_h(h, sk, lens, B, dk, dv, stream)
@@ -403,7 +487,11 @@ def run_mot(args, wl):
         e2e_step()
     stream.synchronize()
     e2e_s = time.perf_counter() - t0
-    if wl.is_h:
+    if wl.is_bt:
+        h2d = 2 * len(bt_src) * hk[0].numel() * es
+        d2h = 2 * len(win) * ok[0].numel() * es
+        e2e_api = "mot_translate_bt with pinned host copies of the window's layers on its stream"
+    elif wl.is_h:
         h2d = hk.numel() * es
         d2h = 2 * ok.numel() * es
         e2e_api = "mot_translate_h with pinned host copies on its stream"
@@ -424,20 +512,47 @@ def run_mot(args, wl):
         peaks, peak_kind = load_peaks()
         # dominant kernel: the largest share of device time
         name, (n_launch, tot_ms) = max(kstats.items(), key=lambda kv: kv[1][1])
-        gp_groups = 2 * tl
-        per_launch_flops = {"umma_fused_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
-                            "umma2_onchip_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
-                            "umma2_gemm1_gelu_gate": alg["flops_gemm1"],
-                            "umma2_gemm2_combine_store": alg["flops_gemm2"],
-                            "umma2_sparse_gemm1": alg["flops_gemm1"],
-                            "umma2_sparse_gemm2": alg["flops_gemm2"],
-                            "umma2_proj": alg["flops_proj"],
-                            "umma_gemm1_gelu_gate": alg["flops_gemm1"],
-                            "simt_gemm1_gelu_gate": alg["flops_gemm1"],
-                            "umma_gemm2_combine_store": alg["flops_gemm2"],
-                            "simt_gemm2_combine_store": alg["flops_gemm2"]}
+        if wl.is_bt:
+            per_launch_flops = {}
+        else:
+            per_launch_flops = {"umma_fused_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
+                                "umma2_onchip_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
+                                "umma2_gemm1_gelu_gate": alg["flops_gemm1"],
+                                "umma2_gemm2_combine_store": alg["flops_gemm2"],
+                                "umma2_sparse_gemm1": alg["flops_gemm1"],
+                                "umma2_sparse_gemm2": alg["flops_gemm2"],
+                                "umma2_proj": alg["flops_proj"],
+                                "umma_gemm1_gelu_gate": alg["flops_gemm1"],
+                                "simt_gemm1_gelu_gate": alg["flops_gemm1"],
+                                "umma_gemm2_combine_store": alg["flops_gemm2"],
+                                "simt_gemm2_combine_store": alg["flops_gemm2"]}
         launches_per_step = max(1, n_launch // args.steps)
-        if name in per_launch_flops:
+        if wl.is_bt:   # alg holds per-launch figures: scale to a step's launches
+            per_launch_flops = {k: v * launches_per_step for k, v in alg["per_launch"].items()}
+        if wl.is_bt and name in alg["per_launch"]:
+            # the slower of the kernel's FLOPs at tensor peak and its bytes at HBM peak
+            fl, by = alg["per_launch"][name], alg["bytes_per_launch"][name]
+            avg_s = tot_ms / n_launch / 1000.0
+            peak_t = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+            t_t, t_b = fl / (peak_t * 1e12), by / (peaks["hbm_gbs"] * 1e9)
+            if t_b >= t_t:
+                achieved = by / avg_s / 1e9
+                roof = {"kernel": name, "bound": "hbm", "achieved": round(achieved, 1),
+                        "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                        "frac": round(achieved / peaks["hbm_gbs"], 4),
+                        "peak_kind": f"HBM copy, {peak_kind}",
+                        "traffic": recorded_traffic(name, wl.name),
+                        "algorithmic_per_launch": by, "flops_per_launch": fl,
+                        "avg_launch_ms": tot_ms / n_launch}
+            else:
+                achieved = fl / avg_s / 1e12
+                roof = {"kernel": name, "bound": "tensor", "achieved": round(achieved, 1),
+                        "peak": peak_t, "unit": "TFLOP/s", "frac": round(achieved / peak_t, 4),
+                        "peak_kind": f"bf16 dense sustained, {peak_kind}",
+                        "traffic": recorded_traffic(name, wl.name),
+                        "algorithmic_per_launch": fl, "bytes_per_launch": by,
+                        "avg_launch_ms": tot_ms / n_launch}
+        elif name in per_launch_flops:
             work = per_launch_flops[name] / launches_per_step
             avg_s = tot_ms / n_launch / 1000.0
             achieved = work / avg_s / 1e12
@@ -455,8 +570,9 @@ def run_mot(args, wl):
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
             rate, n, dt = cpu_oracle_rate(wl, sk_h, sv_h, blob, budget_s=15.0)
+            layers = (f"{wl.bt[1]} window" if wl.is_bt else f"{tl} translated")
             cpu = {"value": rate, "unit": UNIT, "cores": omp_cores(), "kind": "oracle",
-                   "sample": f"{n} random tokens x all {tl} translated layers, {dt:.1f} s"}
+                   "sample": f"{n} random tokens x all {layers} layers, {dt:.1f} s"}
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": t_step, "higher_is_better": True,
@@ -465,7 +581,10 @@ def run_mot(args, wl):
             "config": {"workload": workload_desc(wl), "tokens_per_step": tokens,
                        "parallelism": "replicas" if world > 1 else "single GPU",
                        "path": ("tcgen05 " + schedule) if path == 1 else "simt",
-                       "l2": "inputs larger than L2 (%.2f GB read+written per step)" % (alg["bytes"] / 1e9)},
+                       "l2": ("inputs larger than L2 (%.2f GB read+written per step)" % (alg["bytes"] / 1e9)
+                              if not wl.is_bt else
+                              "each step moves more than L2: %.2f GB of caches and weights plus "
+                              "the row workspace (GBs)" % (alg["bytes"] / 1e9))},
             "roofline": roof,
             "step_roofline": {"flops": alg["flops"], "bytes": alg["bytes"],
                               "roofline_ms": 1000 * t_roof,

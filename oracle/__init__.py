@@ -20,13 +20,17 @@ import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "mot_oracle.c")
-_SRCS = (_SRC, os.path.join(_HERE, "bt_oracle.c"))
+_SRCS = (_SRC, os.path.join(_HERE, "bt_oracle.c"), os.path.join(_HERE, "replay_oracle.c"))
 _LIB = os.path.join(_HERE, "libmot_oracle.so")
 
 
 class OracleDims(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
                 ("L_s", "H_s", "d_s", "L_t", "H_t", "d_t", "E", "top_k", "H", "B", "S", "dtype")]
+
+
+class OracleReplayDims(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in ("B", "N", "Hq", "Hkv", "d", "S", "n_full")]
 
 
 class OracleBtDims(ctypes.Structure):
@@ -83,6 +87,15 @@ def _load():
         lib.oracle_bt_tokens.restype = ctypes.c_int
         lib.oracle_bt_tokens.argtypes = [ctypes.POINTER(OracleDims), ctypes.POINTER(OracleBtDims),
                                          P, P, P, P, ctypes.c_int64, P, P, P, P, P]
+        RD = ctypes.POINTER(OracleReplayDims)
+        lib.oracle_replay_select.restype = ctypes.c_int
+        lib.oracle_replay_select.argtypes = [RD, P, ctypes.c_int, ctypes.c_int, P]
+        lib.oracle_replay_query.restype = ctypes.c_int
+        lib.oracle_replay_query.argtypes = [RD, ctypes.c_int, P, P, P, P, ctypes.c_int,
+                                            ctypes.c_int, ctypes.c_int, P]
+        lib.oracle_replay_tokens.restype = ctypes.c_int
+        lib.oracle_replay_tokens.argtypes = [RD, ctypes.c_int, P, P, P, P, ctypes.c_int64, P, P,
+                                             P, P]
         _lib = lib
     return _lib
 
@@ -270,3 +283,36 @@ def bt_tokens(wl, src_k, src_v, blob, tok_b, tok_s, gate_fixed=None, want_gate=F
     if rc != 0:
         raise ValueError("oracle_bt_tokens: invalid arguments")
     return (out, gate) if want_gate else out
+
+
+# ---- replay attention (App. C.4) ---------------------------------------------------
+
+def replay_dims_of(wl) -> OracleReplayDims:
+    return OracleReplayDims(wl.max_batch, wl.max_seq, wl.q_heads, wl.kv_heads, wl.head_dim,
+                            wl.top_s, wl.n_full)
+
+
+def replay_select(wl, guide, b: int, u: int) -> np.ndarray:
+    """Top-S positions (ascending) of row u of batch entry b's guidance map."""
+    g = np.ascontiguousarray(guide)
+    out = np.empty(min(wl.top_s, u + 1), dtype=np.int32)
+    n = _load().oracle_replay_select(ctypes.byref(replay_dims_of(wl)), g.ctypes.data, b, u,
+                                     out.ctypes.data)
+    if n < 0:
+        raise ValueError("oracle_replay_select: invalid arguments")
+    return out[:n]
+
+
+def replay_tokens(wl, layer: int, q, k, v, guide, tb, th, tu) -> np.ndarray:
+    """Replay attention outputs [n][d] for queries (tb, th, tu) of target layer `layer`."""
+    tb, th, tu = (np.ascontiguousarray(x, dtype=np.int32) for x in (tb, th, tu))
+    q_c, k_c, v_c = (np.ascontiguousarray(a) for a in (q, k, v))
+    g_c = None if guide is None else np.ascontiguousarray(guide)
+    out = np.empty((tb.size, wl.head_dim))
+    rc = _load().oracle_replay_tokens(ctypes.byref(replay_dims_of(wl)), layer, q_c.ctypes.data,
+                                      k_c.ctypes.data, v_c.ctypes.data, _ptr(g_c), tb.size,
+                                      tb.ctypes.data, th.ctypes.data, tu.ctypes.data,
+                                      out.ctypes.data)
+    if rc != 0:
+        raise ValueError("oracle_replay_tokens: invalid arguments")
+    return out

@@ -75,6 +75,9 @@ def _load():
         lib.synth_fill_normal_shifted.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int64,
                                                   ctypes.c_double, ctypes.c_double, ctypes.c_int,
                                                   ctypes.c_void_p]
+        lib.synth_fill_guide.restype = None
+        lib.synth_fill_guide.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_int,
+                                         ctypes.c_int, ctypes.c_int, ctypes.c_void_p]
         lib.synth_fill_cache_layer.restype = None
         lib.synth_fill_cache_layer.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64,
                                                ctypes.c_int, ctypes.c_int, ctypes.c_int,
@@ -353,3 +356,69 @@ def splitmix64(key: int, n: int) -> int:
 
 def stream_key(seed: int, stream: int) -> int:
     return int(_load().synth_stream_key(seed, stream))
+
+
+# ---- replay attention (App. C.4) -------------------------------------------------
+
+@dataclasses.dataclass(frozen=True)
+class ReplayWorkload:
+    """One replay pass over the target model's layers: per layer the queries
+    [B][Hq][N][d], the replay cache [B][Hkv][N][d] and, for layers >= n_full,
+    the head-averaged guidance map [B][N][N] of source layer pi(l) (depth-ratio
+    map from the source's n_layers_src layers)."""
+    name: str
+    n_layers_src: int
+    n_layers_tgt: int
+    q_heads: int
+    kv_heads: int
+    head_dim: int
+    max_batch: int
+    max_seq: int
+    seq_lens: Tuple[int, ...]
+    top_s: int = 128
+    n_full: int = 2
+    dtype: str = "bf16"
+
+    @property
+    def batch(self) -> int:
+        return len(self.seq_lens)
+
+    @property
+    def tokens(self) -> int:
+        return int(sum(self.seq_lens))
+
+    def replace(self, **kw) -> "ReplayWorkload":
+        return dataclasses.replace(self, **kw)
+
+
+REPLAY_WORKLOADS = {
+    # Qwen2.5-0.5B (24 layers) guiding Qwen2.5-1.5B (28 layers, 12 query heads, 2 KV heads
+    # of 128), a 4K-token context budget (the paper's smallest long-context budget), S = 128,
+    # L_Full = 2 (the paper's settings).
+    "replay_qwen05_qwen15": ReplayWorkload("replay_qwen05_qwen15", 24, 28, 12, 2, 128, 4, 4096,
+                                           (4096,) * 4),
+}
+
+
+def _stream_replay(kind: int, layer: int) -> int:
+    return (4 << 56) | (kind << 48) | layer
+
+
+def gen_replay_qkv(wl: ReplayWorkload, layer: int, seed: int = 0):
+    """(q, k, v) of one target layer in bf16 bits: N(0, 1) draws."""
+    lib = _load()
+    B, N, d = wl.max_batch, wl.max_seq, wl.head_dim
+    out = []
+    for kind, H in ((1, wl.q_heads), (2, wl.kv_heads), (3, wl.kv_heads)):
+        a = np.empty((B, H, N, d), dtype=np.uint16)
+        lib.synth_fill_normal(seed, _stream_replay(kind, layer), a.size, 1.0, 0, a.ctypes.data)
+        out.append(a)
+    return tuple(out)
+
+
+def gen_guide(wl: ReplayWorkload, src_layer: int, seed: int = 0) -> np.ndarray:
+    """Guidance map of one source layer: [B][N][N] bf16 bits (zeros above the diagonal)."""
+    a = np.empty((wl.max_batch, wl.max_seq, wl.max_seq), dtype=np.uint16)
+    _load().synth_fill_guide(seed, _stream_replay(4, src_layer), wl.max_batch, wl.max_seq, 0,
+                             a.ctypes.data)
+    return a

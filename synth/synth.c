@@ -150,3 +150,34 @@ void synth_fill_cache_layer(uint64_t seed, uint64_t scale_stream, uint64_t value
   }
   free(sc);
 }
+
+/*
+ * Source guidance maps for the replay (App. C.4 reads the source attention
+ * averaged over heads): rows u of a [B][N][N] map, positive scores at j <= u
+ * and zeros above the diagonal. Each score is a LogNormal(0, 0.5) draw times a
+ * structure weight with the shapes attention maps show: a sink at position 0
+ * (x5), recency 1 + 3 exp(-(u - j) / 32), and a fixed set of "heavy" columns
+ * (about 1 in 64, x3), drawn from `stream`. Only the order within a row
+ * matters to the selection; the rows are not normalised.
+ */
+void synth_fill_guide(uint64_t seed, uint64_t stream, int B, int N, int dtype, void* out) {
+  uint64_t kval = synth_stream_key(seed, stream);
+  uint64_t kcol = synth_stream_key(seed, stream ^ 0x5A5A5A5AULL);
+  const int64_t rows = (int64_t)B * N;
+#pragma omp parallel for schedule(dynamic, 16)
+  for (int64_t r = 0; r < rows; ++r) {
+    const int64_t u = r % N;
+    for (int64_t j = 0; j < N; ++j) {
+      const int64_t idx = r * N + j;
+      if (j > u) {
+        store_val(out, idx, 0.0, dtype);
+        continue;
+      }
+      double w = 1.0 + 3.0 * exp(-(double)(u - j) / 32.0);
+      if (j == 0) w *= 5.0;
+      if ((synth_splitmix64(kcol, (uint64_t)j) & 63u) == 0) w *= 3.0;
+      const double v = w * exp(0.5 * synth_normal_at(kval, (uint64_t)idx));
+      store_val(out, idx, v, dtype);
+    }
+  }
+}

@@ -71,8 +71,25 @@ BT_MUTATIONS = {
                           "for (int64_t i = 0; i < Dt; ++i) o[i] = acc[(N - 1 - r) * Dt + i];"),
 }
 
+# Mistakes in the replay-attention oracle (App. C.4), caught by its own pins.
+REPLAY_PINS = os.path.join(ROOT, "tests", "test_oracle_replay_pins.py")
+REPLAY_MUTATIONS = {
+    "replay_ties_to_higher_position": ("if (best < 0 || v > bv) { best = j; bv = v; }",
+                                       "if (best < 0 || v >= bv) { best = j; bv = v; }"),
+    "replay_not_causal": ("  const uint16_t* row = guide + ((int64_t)b * d->N + u) * d->N;",
+                          "  n = d->N;\n  const uint16_t* row = guide + ((int64_t)b * d->N + u) * d->N;"),
+    "replay_previous_row": ("  const uint16_t* row = guide + ((int64_t)b * d->N + u) * d->N;",
+                            "  const uint16_t* row = guide + ((int64_t)b * d->N + (u > 0 ? u - 1 : 0)) * d->N;"),
+    "replay_unscaled": ("s[t] = acc * scale;", "s[t] = acc;"),
+    "replay_gqa_interleaved": ("const int hk = h / (d->Hq / d->Hkv);", "const int hk = h % d->Hkv;"),
+    "replay_full_layer_boundary": ("const int sparse = layer >= d->n_full;",
+                                   "const int sparse = layer > d->n_full;"),
+}
+
 CASES = ([(n, "mot_oracle.c", PINS, MUTATIONS[n]) for n in sorted(MUTATIONS)] +
-         [(n, "bt_oracle.c", BT_PINS, BT_MUTATIONS[n]) for n in sorted(BT_MUTATIONS)])
+         [(n, "bt_oracle.c", BT_PINS, BT_MUTATIONS[n]) for n in sorted(BT_MUTATIONS)] +
+         [(n, "replay_oracle.c", REPLAY_PINS, REPLAY_MUTATIONS[n])
+          for n in sorted(REPLAY_MUTATIONS)])
 
 
 @pytest.mark.parametrize("name,src_name,pins,change", CASES, ids=[c[0] for c in CASES])

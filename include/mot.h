@@ -342,6 +342,46 @@ mot_status mot_translate_bt(mot_handle h, const void* src_k, const void* src_v,
                             const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
                             mot_stream_t stream);
 
+/*
+ * Replay attention (App. C.4): after translation the target model replays the
+ * context over its cache, and each layer's attention runs here. For target
+ * layer `layer`, batch entry b < batch, context position u < seq_lens[b] and
+ * query head h (GQA: key/value head h / (q_heads / kv_heads)):
+ *   layer <  n_full:  o = Attn(q_u, K[0..u], V[0..u])                 (full, causal)
+ *   layer >= n_full:  N(u) = Top-S(A[b][u][0..u], top_s),  o = Attn(q_u, K[N(u)], V[N(u)])
+ * where A is the guidance map of the source layer that guides this layer (the
+ * source model's attention averaged over heads), Top-S keeps the top_s
+ * positions j <= u with the largest A[b][u][j] (equal values: the lower
+ * position first; every position when u + 1 <= top_s), and Attn is the
+ * softmax of q . k / sqrt(head_dim) over the set applied to the value rows.
+ * Layouts (bf16, device, 16-byte aligned, contiguous): q, out
+ * [max_batch][q_heads][max_seq][head_dim]; k, v [max_batch][kv_heads][max_seq]
+ * [head_dim] (one layer of the replay cache, e.g. a layer of mot_translate's
+ * target cache); guide [max_batch][max_seq][max_seq] (row u, column j; only
+ * j <= u is read; guide may be NULL for full layers). Rows u >= seq_lens[b] of
+ * out are not written. seq_lens: device int32[batch], clamped to [0, max_seq].
+ * Requires head_dim in {64, 128}, q_heads / kv_heads <= 16, top_s <= 4096,
+ * max_seq <= 65536 (else MOT_ERR_UNSUPPORTED). Asynchronous on `stream`.
+ *
+ * mot_replay_select writes the selection alone: sel [max_batch][max_seq][top_s]
+ * int32, the row's positions ascending, then -1 (rows u >= seq_lens[b] are not
+ * written). A replay handle accepts only these two calls and the profiling,
+ * launch-count and destroy calls.
+ */
+typedef struct {
+  int32_t q_heads, kv_heads, head_dim;
+  int32_t max_batch, max_seq;
+  int32_t top_s;    /* S_sparse */
+  int32_t n_full;   /* L_Full: layers below it use full causal attention */
+} mot_replay_config;
+
+mot_status mot_create_replay(const mot_replay_config* cfg, mot_handle* out);
+mot_status mot_replay_attention(mot_handle h, int32_t layer, const void* q, const void* k,
+                                const void* v, const void* guide, const int32_t* seq_lens,
+                                int32_t batch, void* out, mot_stream_t stream);
+mot_status mot_replay_select(mot_handle h, const void* guide, const int32_t* seq_lens,
+                             int32_t batch, int32_t* sel, mot_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

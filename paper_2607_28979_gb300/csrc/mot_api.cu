@@ -152,6 +152,9 @@ struct mot_ctx {
   CUtensorMap tm_wkv{}, tm_ahat{};
   // backbone translators (App. C.2): kind 2
   BtState* bt = nullptr;
+  // replay attention (App. C.4): kind 3
+  ReplayDims rd{};
+  int32_t* rsel = nullptr;   // [B][N][S] selection workspace
   // Top-K routing (tensor-core path, 0 < top_k < E): token buckets per expert
   bool sparse_ok = false;   // the shapes support it
   int routing = 0;          // 0 dense compute with a zeroed gate, 1 token buckets
@@ -194,6 +197,7 @@ void free_all(mot_ctx* h) {
                   h->sp.row0, h->sp.plan, h->sp.pairs, h->sp.ltok, h->sp.lslot, h->sp.gatep,
                   h->sp.gate16p, h->sp.zp, h->sp.a2p, h->sp.ybuf, h->wkv, h->ahat,
                   h->proj_layer,
+                  h->rsel,
                   h->n_tiles, h->status, h->counters, h->st_src[0], h->st_src[1], h->st_dst[0],
                   h->st_dst[1], h->st_len};
   for (void* p : ptrs)
@@ -1425,6 +1429,112 @@ mot_status mot_translate_bt(mot_handle h, const void* src_k, const void* src_v,
       return launch_bt_gemm(kBtOut, a, bt.tm_xo, bt.tm_xo, bt.tm_wout, h->num_sms, st);
     }));
   }
+  return MOT_OK;
+}
+
+mot_status mot_create_replay(const mot_replay_config* cfg, mot_handle* out) {
+  if (!out) return MOT_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg || cfg->q_heads <= 0 || cfg->kv_heads <= 0 || cfg->head_dim <= 0 ||
+      cfg->max_batch <= 0 || cfg->max_seq <= 0 || cfg->top_s <= 0 || cfg->n_full < 0 ||
+      cfg->q_heads % cfg->kv_heads)
+    return MOT_ERR_INVALID_ARG;
+  ReplayDims rd{cfg->max_batch, cfg->max_seq, cfg->q_heads, cfg->kv_heads, cfg->head_dim,
+                cfg->top_s, cfg->n_full};
+  if (!replay_supported(rd) || int64_t(rd.B) * rd.N > INT32_MAX / 2) return MOT_ERR_UNSUPPORTED;
+  mot_ctx* h = new (std::nothrow) mot_ctx();
+  if (!h) return MOT_ERR_OOM;
+  h->kind = 3;
+  h->rd = rd;
+  int dev = 0, cc_major = 0, cc_minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&cc_major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&cc_minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess) {
+    cudaGetLastError();
+    delete h;
+    return MOT_ERR_CUDA;
+  }
+  h->device = dev;
+  if (cc_major != 10 || cc_minor != 3) {
+    delete h;
+    return MOT_ERR_UNSUPPORTED;
+  }
+  if (cudaMalloc(&h->rsel, size_t(rd.B) * rd.N * rd.S * 4) != cudaSuccess ||
+      cudaMalloc(&h->status, 16) != cudaSuccess || cudaMemset(h->status, 0, 16) != cudaSuccess) {
+    cudaGetLastError();
+    free_all(h);
+    delete h;
+    return MOT_ERR_OOM;
+  }
+  h->weights_loaded = true;   // nothing to load
+  *out = h;
+  return MOT_OK;
+}
+
+namespace {
+
+mot_status replay_args(mot_handle h, const void* q, const void* k, const void* v,
+                       const void* guide, const int32_t* seq_lens, int32_t batch, void* out,
+                       bool need_qkv, ReplayArgs& a) {
+  if (!h || h->kind != 3) return MOT_ERR_INVALID_ARG;
+  const ReplayDims& d = h->rd;
+  if (batch < 0 || batch > d.B || (batch > 0 && !seq_lens)) return MOT_ERR_INVALID_ARG;
+  if (need_qkv && (!q || !k || !v || !out || !aligned16(q) || !aligned16(k) || !aligned16(v) ||
+                   !aligned16(out)))
+    return MOT_ERR_INVALID_ARG;
+  if (need_qkv) {
+    const size_t qb = size_t(d.B) * d.Hq * d.N * d.d * 2, kb = size_t(d.B) * d.Hkv * d.N * d.d * 2;
+    if (overlap(out, qb, q, qb) || overlap(out, qb, k, kb) || overlap(out, qb, v, kb))
+      return MOT_ERR_INVALID_ARG;
+  }
+  a = ReplayArgs{};
+  a.d = d;
+  a.q = q;
+  a.k = k;
+  a.v = v;
+  a.guide = guide;
+  a.out = out;
+  a.sel = h->rsel;
+  a.seq_lens = seq_lens;
+  a.batch = batch;
+  return MOT_OK;
+}
+
+}  // namespace
+
+mot_status mot_replay_select(mot_handle h, const void* guide, const int32_t* seq_lens,
+                             int32_t batch, int32_t* sel, mot_stream_t stream) {
+  ReplayArgs a;
+  mot_status r = replay_args(h, nullptr, nullptr, nullptr, guide, seq_lens, batch, nullptr,
+                             false, a);
+  if (r != MOT_OK) return r;
+  if (!guide || !sel || !aligned16(guide)) return MOT_ERR_INVALID_ARG;
+  if (cudaSetDevice(h->device) != cudaSuccess) return MOT_ERR_CUDA;
+  if (batch == 0) return MOT_OK;
+  a.sel = sel;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  MOT_CUDA_TRY(timed(h, "replay_select", st, [&] { return launch_replay_select(a, st); }));
+  return MOT_OK;
+}
+
+mot_status mot_replay_attention(mot_handle h, int32_t layer, const void* q, const void* k,
+                                const void* v, const void* guide, const int32_t* seq_lens,
+                                int32_t batch, void* out, mot_stream_t stream) {
+  ReplayArgs a;
+  mot_status r = replay_args(h, q, k, v, guide, seq_lens, batch, out, true, a);
+  if (r != MOT_OK) return r;
+  if (layer < 0) return MOT_ERR_INVALID_ARG;
+  const bool full = layer < h->rd.n_full;
+  if (!full && (!guide || !aligned16(guide))) return MOT_ERR_INVALID_ARG;
+  if (cudaSetDevice(h->device) != cudaSuccess) return MOT_ERR_CUDA;
+  if (batch == 0) return MOT_OK;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  a.full = full ? 1 : 0;
+  if (!full)
+    MOT_CUDA_TRY(timed(h, "replay_select", st, [&] { return launch_replay_select(a, st); }));
+  MOT_CUDA_TRY(timed(h, full ? "replay_attn_full" : "replay_attn_sparse", st,
+                     [&] { return launch_replay_attn(a, st); }));
   return MOT_OK;
 }
 

@@ -185,6 +185,32 @@ cudaError_t launch_bt_gemm(int mode, const BtArgs& a, const CUtensorMap& tmA,
                            const CUtensorMap& tmA2, const CUtensorMap& tmB, int num_sms,
                            cudaStream_t st);
 
+// ---------------------------------------------------------------- replay attention
+//
+// App. C.4 (replay.cu): one target layer's attention over the replay cache,
+// full causal for layers below L_Full, else over the Top-S positions of the
+// source guidance map's causal row. Layouts: q / out [B][Hq][N][d], k / v
+// [B][Hkv][N][d], guide [B][N][N] (bf16), sel [B][N][S] int32 (ascending
+// positions, -1 after the row's count).
+struct ReplayDims {
+  int32_t B, N, Hq, Hkv, d, S, n_full;
+};
+struct ReplayArgs {
+  ReplayDims d;
+  const void* q;
+  const void* k;
+  const void* v;
+  const void* guide;
+  void* out;
+  int32_t* sel;
+  const int32_t* seq_lens;
+  int32_t batch;
+  int32_t full;   // 1: attend to every position 0..u
+};
+bool replay_supported(const ReplayDims& d);
+cudaError_t launch_replay_select(const ReplayArgs& a, cudaStream_t st);
+cudaError_t launch_replay_attn(const ReplayArgs& a, cudaStream_t st);
+
 // Kernel launchers (each returns the launch's cudaError_t).
 cudaError_t launch_bf16_to_f16_inplace(void* buf, size_t n, cudaStream_t st);
 cudaError_t launch_build_b2t(const float* b2, void* b2t, int G, int E, int Dt, cudaStream_t st);

@@ -59,6 +59,12 @@ class mot_bt_config(ctypes.Structure):
                 ("width", ctypes.c_int32), ("heads", ctypes.c_int32), ("ffn", ctypes.c_int32)]
 
 
+class mot_replay_config(ctypes.Structure):
+    _fields_ = [("q_heads", ctypes.c_int32), ("kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("max_batch", ctypes.c_int32),
+                ("max_seq", ctypes.c_int32), ("top_s", ctypes.c_int32), ("n_full", ctypes.c_int32)]
+
+
 class mot_kernel_stat(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char * 32), ("launches", ctypes.c_int64),
                 ("total_ms", ctypes.c_double)]
@@ -94,6 +100,9 @@ _SIGS = {
     "mot_create_bt": [ctypes.POINTER(mot_config), ctypes.POINTER(mot_bt_config),
                       ctypes.POINTER(ctypes.c_void_p)],
     "mot_translate_bt": [_H, _P, _P, _P, ctypes.c_int32, _P, _P, _P],
+    "mot_create_replay": [ctypes.POINTER(mot_replay_config), ctypes.POINTER(ctypes.c_void_p)],
+    "mot_replay_attention": [_H, ctypes.c_int32, _P, _P, _P, _P, _P, ctypes.c_int32, _P, _P],
+    "mot_replay_select": [_H, _P, _P, ctypes.c_int32, _P, _P],
 }
 for _name, _args in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -223,6 +232,30 @@ def mot_translate_bt(h: Handle, src_k, src_v, seq_lens, batch: int, dst_k, dst_v
                      stream=None) -> None:
     _check(_lib.mot_translate_bt(h.ptr, _addr(src_k), _addr(src_v), _addr(seq_lens), int(batch),
                                  _addr(dst_k), _addr(dst_v), _stream(stream)), "mot_translate_bt")
+
+
+def replay_config_from(wl):
+    """mot_replay_config for a ``synth.ReplayWorkload``."""
+    return mot_replay_config(wl.q_heads, wl.kv_heads, wl.head_dim, wl.max_batch, wl.max_seq,
+                             wl.top_s, wl.n_full)
+
+
+def mot_create_replay(cfg: mot_replay_config) -> Handle:
+    out = ctypes.c_void_p()
+    _check(_lib.mot_create_replay(ctypes.byref(cfg), ctypes.byref(out)), "mot_create_replay")
+    return Handle(out.value, 0)
+
+
+def mot_replay_attention(h: Handle, layer: int, q, k, v, guide, seq_lens, batch: int, out,
+                         stream=None) -> None:
+    _check(_lib.mot_replay_attention(h.ptr, int(layer), _addr(q), _addr(k), _addr(v),
+                                     _addr(guide), _addr(seq_lens), int(batch), _addr(out),
+                                     _stream(stream)), "mot_replay_attention")
+
+
+def mot_replay_select(h: Handle, guide, seq_lens, batch: int, sel, stream=None) -> None:
+    _check(_lib.mot_replay_select(h.ptr, _addr(guide), _addr(seq_lens), int(batch), _addr(sel),
+                                  _stream(stream)), "mot_replay_select")
 
 
 def mot_create(cfg: mot_config) -> Handle:

@@ -1,0 +1,156 @@
+"""Replay attention (App. C.4) on the GPU through the C ABI, against the fp64
+oracle: the Top-S selection bit for bit, the attention within the bf16 bar."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA GPU", allow_module_level=True)
+
+import _gpu as G   # noqa: E402
+M = G.M
+
+RW = synth.ReplayWorkload
+SMALL = {
+    # GQA 12 / 2, d = 128, S = 16 (short rows below S), ragged batch
+    "r_gqa6_d128": RW("r_gqa6_d128", 6, 7, 12, 2, 128, 2, 300, (300, 131), top_s=16, n_full=2),
+    # no GQA, d = 64, the paper's S = 128 with rows shorter and longer than S
+    "r_mha_d64": RW("r_mha_d64", 4, 4, 4, 4, 64, 3, 400, (400, 128, 129), top_s=128, n_full=1),
+    # 16 query heads per key/value head, one long row per entry
+    "r_gqa16": RW("r_gqa16", 2, 2, 16, 1, 64, 1, 1000, (1000,), top_s=64, n_full=1),
+}
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda()
+
+
+class ReplayRun:
+    def __init__(self, wl, seq=None, batch=None):
+        self.wl = wl
+        self.h = M.mot_create_replay(M.replay_config_from(wl))
+        self.seq = list(wl.seq_lens if seq is None else seq)
+        self.batch = len(self.seq) if batch is None else batch
+        self.lens = torch.tensor(self.seq, dtype=torch.int32, device="cuda")
+
+    def select(self, g):
+        sel = torch.full((self.wl.max_batch, self.wl.max_seq, self.wl.top_s), -7,
+                         dtype=torch.int32, device="cuda")
+        M.mot_replay_select(self.h, _dev(g), self.lens, self.batch, sel)
+        torch.cuda.synchronize()
+        return sel.cpu().numpy()
+
+    def attend(self, layer, q, k, v, g):
+        out = torch.full((self.wl.max_batch, self.wl.q_heads, self.wl.max_seq, self.wl.head_dim),
+                         G.SENTINEL_BF16, dtype=torch.int16, device="cuda")
+        M.mot_replay_attention(self.h, layer, _dev(q), _dev(k), _dev(v),
+                               None if g is None else _dev(g), self.lens, self.batch, out)
+        torch.cuda.synchronize()
+        return out
+
+
+BF16 = synth.WORKLOADS["gpt2s_opt125m"]   # carries the bf16 tolerance of the parity bar
+
+
+def _f64(bits_t):
+    return bits_t.view(torch.bfloat16).double().cpu().numpy()
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_selection_is_bit_exact_on_every_row(name):
+    wl = SMALL[name]
+    g = synth.gen_guide(wl, 3)
+    run = ReplayRun(wl)
+    sel = run.select(g)
+    for b, L in enumerate(wl.seq_lens):
+        for u in range(L):
+            ref = oracle.replay_select(wl, g, b, u)
+            row = sel[b, u]
+            np.testing.assert_array_equal(row[:ref.size], ref, err_msg=f"b={b} u={u}")
+            assert (row[ref.size:] == -1).all()
+        assert (sel[b, L:] == -7).all()   # rows past the sequence are not written
+
+
+def test_selection_ties_and_constant_rows():
+    wl = SMALL["r_gqa6_d128"].replace(top_s=8)
+    N = wl.max_seq
+    g = np.zeros((wl.max_batch, N, N), dtype=np.uint16)
+    g[0] = 0x4000                                  # every score 2.0: the lowest positions win
+    rng = np.random.default_rng(0)
+    g[1] = (0x3F80 + rng.integers(0, 3, size=(N, N))).astype(np.uint16)   # three values only
+    run = ReplayRun(wl)
+    sel = run.select(g)
+    for b, L in enumerate(wl.seq_lens):
+        for u in range(0, L, 7):
+            ref = oracle.replay_select(wl, g, b, u)
+            np.testing.assert_array_equal(sel[b, u, :ref.size], ref)
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_attention_matches_oracle(name):
+    wl = SMALL[name]
+    q, k, v = synth.gen_replay_qkv(wl, 1)
+    g = synth.gen_guide(wl, 5)
+    run = ReplayRun(wl)
+    rng = np.random.default_rng(7)
+    for layer in (0, wl.n_full, wl.n_full + 3):
+        out = run.attend(layer, q, k, v, None if layer < wl.n_full else g)
+        tb, th, tu = [], [], []
+        for b, L in enumerate(wl.seq_lens):
+            us = np.unique(np.concatenate([[0, 1, L - 1, min(L - 1, wl.top_s), min(L - 1, wl.top_s - 1)],
+                                           rng.integers(0, L, size=20)]))
+            for u in us:
+                for h in rng.choice(wl.q_heads, size=min(4, wl.q_heads), replace=False):
+                    tb.append(b); th.append(h); tu.append(u)
+        ref = oracle.replay_tokens(wl, layer, q, k, v, g, tb, th, tu)
+        got = _f64(out)[tb, th, tu]
+        G.assert_parity(BF16, got, ref, f"{name} layer {layer}")
+        o = out.cpu().numpy()
+        for b, L in enumerate(wl.seq_lens):
+            assert (o[b, :, L:] == np.int16(G.SENTINEL_BF16)).all()
+
+
+def test_full_size_layer_sampled():
+    """Qwen2.5-0.5B -> 1.5B replay shapes (4 x 4096 context, 12 / 2 heads of 128,
+    S = 128): one full and one guided layer, in the benchmark's launch configuration."""
+    wl = synth.REPLAY_WORKLOADS["replay_qwen05_qwen15"]
+    q, k, v = synth.gen_replay_qkv(wl, 2)
+    g = synth.gen_guide(wl, 9)
+    run = ReplayRun(wl)
+    sel = run.select(g)
+    rng = np.random.default_rng(11)
+    for b in range(wl.batch):
+        for u in np.concatenate([[0, 127, 128, 4095], rng.integers(0, 4096, size=12)]):
+            ref = oracle.replay_select(wl, g, b, int(u))
+            np.testing.assert_array_equal(sel[b, u, :ref.size], ref)
+    for layer in (1, 5):
+        out = run.attend(layer, q, k, v, g)
+        tb = rng.integers(0, wl.batch, size=48)
+        th = rng.integers(0, wl.q_heads, size=48)
+        tu = np.concatenate([[0, 4095], rng.integers(0, 4096, size=46)])
+        ref = oracle.replay_tokens(wl, layer, q, k, v, g, tb, th, tu)
+        G.assert_parity(BF16, _f64(out)[tb, th, tu], ref, f"full-size layer {layer}")
+
+
+def test_batch_prefix_and_errors():
+    wl = SMALL["r_mha_d64"]
+    q, k, v = synth.gen_replay_qkv(wl, 0)
+    g = synth.gen_guide(wl, 0)
+    run = ReplayRun(wl, batch=2)
+    out = run.attend(3, q, k, v, g).cpu().numpy()
+    assert (out[2] == np.int16(G.SENTINEL_BF16)).all()    # entry 2 is past `batch`
+    dst = torch.empty(out.shape, dtype=torch.int16, device="cuda")
+    with pytest.raises(M.MotError) as e:                   # a guided layer needs its map
+        M.mot_replay_attention(run.h, 3, _dev(q), _dev(k), _dev(v), None, run.lens, 2, dst)
+    assert e.value.status == M.MOT_ERR_INVALID_ARG
+    with pytest.raises(M.MotError) as e:
+        M.mot_create_replay(M.replay_config_from(wl.replace(head_dim=96)))
+    assert e.value.status == M.MOT_ERR_UNSUPPORTED
+    with pytest.raises(M.MotError) as e:
+        M.mot_create_replay(M.replay_config_from(wl.replace(kv_heads=3)))
+    assert e.value.status == M.MOT_ERR_INVALID_ARG

@@ -607,13 +607,288 @@ def run_mot(args, wl):
     return 0
 
 
+# ---------------------------------------------------------------- replay attention (App. C.4)
+
+def replay_desc(wl) -> str:
+    return (f"{wl.name}: replay attention over {wl.n_layers_tgt} target layers "
+            f"({wl.q_heads} query / {wl.kv_heads} key-value heads of {wl.head_dim}), bottom "
+            f"{wl.n_full} full causal, the rest Top-{wl.top_s} guided by the head-averaged "
+            f"attention maps of {wl.n_layers_src} source layers (depth-ratio map), bf16, "
+            f"batch {wl.batch} seq_lens {list(wl.seq_lens)}")
+
+
+def replay_guide_layers(wl):
+    """Source guidance layer pi(l) of each target layer (depth-ratio map)."""
+    import oracle
+    return oracle.depth_ratio_map(wl.n_layers_src, wl.n_layers_tgt)
+
+
+def replay_algorithmic(wl):
+    """FLOPs and bytes per step (one replay of every layer), and per kernel launch."""
+    B, N, Hq, Hkv, d, S = wl.max_batch, wl.max_seq, wl.q_heads, wl.kv_heads, wl.head_dim, wl.top_s
+    lens = wl.seq_lens
+    keys_full = sum(L * (L + 1) // 2 for L in lens)
+    keys_sparse = sum(sum(min(S, u + 1) for u in range(L)) for L in lens)
+    fl_full = 4 * Hq * d * keys_full           # q.k and p.v, 2 FLOP each
+    fl_sparse = 4 * Hq * d * keys_sparse
+    T = wl.tokens
+    b_qo = 2 * T * Hq * d * 2                  # queries in, outputs out
+    b_kv = 2 * T * Hkv * d * 2
+    b_map = sum(L * (L + 1) // 2 for L in lens) * 2   # the causal part of one guidance map
+    b_sel = T * S * 4
+    n_sparse = wl.n_layers_tgt - wl.n_full
+    per = {
+        "replay_attn_full": dict(flops=fl_full, bytes=b_qo + b_kv),
+        "replay_attn_sparse": dict(flops=fl_sparse, bytes=b_qo + b_kv),
+        "replay_select": dict(flops=0, bytes=b_map + b_sel),
+    }
+    flops = wl.n_full * fl_full + n_sparse * fl_sparse
+    byts = wl.n_layers_tgt * (b_qo + b_kv) + n_sparse * b_map
+    return dict(flops=flops, bytes=byts, per_launch=per)
+
+
+def _replay_oracle_rate(wl, layers, budget_s, seed=5):
+    """Replayed context tokens per second of the fp64 oracle: random (layer, b, h, u)
+    queries for about budget_s; one token = one position through every layer and head."""
+    import oracle
+    rng = np.random.default_rng(seed)
+    gl = replay_guide_layers(wl)
+
+    def sample(n):
+        tb = rng.integers(0, wl.batch, size=n)
+        tu = np.array([rng.integers(0, wl.seq_lens[b]) for b in tb])
+        th = rng.integers(0, wl.q_heads, size=n)
+        tl = rng.integers(0, wl.n_layers_tgt, size=n)
+        return tb, th, tu, tl
+
+    def run(tb, th, tu, tl):
+        for l in np.unique(tl):
+            m = tl == l
+            q, k, v, g = layers(int(l), gl)
+            oracle.replay_tokens(wl, int(l), q, k, v, g, tb[m], th[m], tu[m])
+    c = omp_cores()
+    smp = sample(4 * c)
+    t0 = time.perf_counter()
+    run(*smp)
+    per_q = max((time.perf_counter() - t0) / (4 * c), 1e-7)
+    n = int(max(4 * c, min(200000, budget_s / per_q)))
+    smp = sample(n)
+    t0 = time.perf_counter()
+    run(*smp)
+    dt = time.perf_counter() - t0
+    per_token = wl.n_layers_tgt * wl.q_heads
+    return n / dt / per_token, n, dt
+
+
+def _replay_host_inputs(wl):
+    """Per-layer (q, k, v) and the guidance maps of the source layers in use, bf16
+    bits on the host; returns (layers(l, gl) -> (q, k, v, guide or None), maps)."""
+    gl = replay_guide_layers(wl)
+    used = sorted({gl[l] for l in range(wl.n_full, wl.n_layers_tgt)})
+    maps = {s: synth.gen_guide(wl, s) for s in used}
+    qkv = {l: synth.gen_replay_qkv(wl, l) for l in range(wl.n_layers_tgt)}
+
+    def layers(l, g_layers):
+        q, k, v = qkv[l]
+        return q, k, v, (maps[g_layers[l]] if l >= wl.n_full else None)
+    return layers, qkv, maps
+
+
+def run_replay_reference(args, wl):
+    world, rank, _ = dist_setup(args.gpus)
+    if rank != 0:
+        return 0
+    import oracle
+    oracle.build()
+    layers, _, _ = _replay_host_inputs(wl)
+    times, ns = [], []
+    for i in range(args.warmup + args.steps):
+        rate, n, dt = _replay_oracle_rate(wl, layers, budget_s=2.0, seed=100 + i)
+        if i >= args.warmup:
+            times.append(dt)
+            ns.append(n)
+    per_token = wl.n_layers_tgt * wl.q_heads
+    value = sum(ns) / sum(times) / per_token
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * sum(times) / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded queries, replay caches and source guidance maps)",
+        "config": {"workload": replay_desc(wl),
+                   "sample": "random (layer, batch, head, position) queries, about 2 s per step; "
+                             "a token = one position through every layer and head"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": omp_cores(), "kind": "oracle",
+                         "sample": f"{sum(ns)} queries over {args.steps} steps"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_replay(args, wl):
+    world, rank, local = dist_setup(args.gpus)
+    import torch
+    import torch.distributed as dist
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    from paper_2607_28979_gb300 import build as mot_build
+    if rank == 0 or world == 1:
+        mot_build.build()
+    if world > 1:
+        dist.barrier()
+    import paper_2607_28979_gb300.mot as M
+
+    layers, qkv_h, maps_h = _replay_host_inputs(wl)
+    gl = replay_guide_layers(wl)
+    h = M.mot_create_replay(M.replay_config_from(wl))
+
+    def dev(a):
+        return torch.from_numpy(a.view(np.int16)).cuda()
+    qkv = {l: tuple(dev(a) for a in qkv_h[l]) for l in qkv_h}
+    maps = {s: dev(m) for s, m in maps_h.items()}
+    out = torch.empty((wl.max_batch, wl.q_heads, wl.max_seq, wl.head_dim), dtype=torch.int16,
+                      device="cuda")
+    lens = torch.tensor(wl.seq_lens, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.Stream()
+    B = wl.batch
+    outs = {}
+
+    def step(dst=None):
+        for l in range(wl.n_layers_tgt):
+            q, k, v = qkv[l]
+            g = maps[gl[l]] if l >= wl.n_full else None
+            M.mot_replay_attention(h, l, q, k, v, g, lens, B, out if dst is None else dst[l],
+                                   stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step()
+    stream.synchronize()
+    sampler = ClockSampler(local) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    M.mot_profile_enable(h, True)
+    M.mot_profile_read(h)
+    launches0 = M.mot_get_launch_count(h)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    elapsed_ms = e0.elapsed_time(e1)
+    launches = M.mot_get_launch_count(h) - launches0
+    kstats = M.mot_profile_read(h)
+    M.mot_profile_enable(h, False)
+    clocks = sampler.stop() if sampler else None
+
+    # end to end: every layer's inputs copied in from pinned host memory and its
+    # output copied back, on the replay stream
+    pin = lambda a: torch.from_numpy(a.view(np.int16)).pin_memory()
+    qkv_p = {l: tuple(pin(a) for a in qkv_h[l]) for l in qkv_h}
+    maps_p = {s: pin(m) for s, m in maps_h.items()}
+    out_p = torch.empty((wl.n_layers_tgt,) + tuple(out.shape), dtype=torch.int16).pin_memory()
+
+    def e2e_step():
+        with torch.cuda.stream(stream):
+            for l in range(wl.n_layers_tgt):
+                for dsta, srca in zip(qkv[l], qkv_p[l]):
+                    dsta.copy_(srca, non_blocking=True)
+                if l >= wl.n_full:
+                    maps[gl[l]].copy_(maps_p[gl[l]], non_blocking=True)
+                q, k, v = qkv[l]
+                M.mot_replay_attention(h, l, q, k, v, maps[gl[l]] if l >= wl.n_full else None,
+                                       lens, B, out, stream)
+                out_p[l].copy_(out, non_blocking=True)
+    e2e_step()
+    stream.synchronize()
+    e2e_steps = 3
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        e2e_step()
+    stream.synchronize()
+    e2e_s = time.perf_counter() - t0
+    h2d = sum(a.numel() * 2 for l in qkv_p for a in qkv_p[l]) + \
+        sum(maps_p[gl[l]].numel() * 2 for l in range(wl.n_full, wl.n_layers_tgt))
+    d2h = out_p.numel() * 2
+
+    t_step, e2e_s = reduce_max([elapsed_ms / args.steps, e2e_s], world, "cuda")
+    value = aggregate_throughput(wl.tokens, world, t_step / 1000.0)
+    e2e_value = aggregate_throughput(wl.tokens * e2e_steps, world, e2e_s)
+    if rank == 0:
+        alg = replay_algorithmic(wl)
+        peaks, peak_kind = load_peaks()
+        name, (n_launch, tot_ms) = max(kstats.items(), key=lambda kv: kv[1][1])
+        per = alg["per_launch"].get(name)
+        avg_s = tot_ms / n_launch / 1000.0
+        peak_t = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+        t_t, t_b = per["flops"] / (peak_t * 1e12), per["bytes"] / (peaks["hbm_gbs"] * 1e9)
+        if t_t >= t_b:
+            ach = per["flops"] / avg_s / 1e12
+            roof = {"kernel": name, "bound": "tensor", "achieved": round(ach, 2), "peak": peak_t,
+                    "unit": "TFLOP/s", "frac": round(ach / peak_t, 4),
+                    "peak_kind": f"bf16 dense sustained, {peak_kind}", "traffic": None,
+                    "algorithmic_per_launch": per["flops"], "avg_launch_ms": 1000 * avg_s}
+        else:
+            ach = per["bytes"] / avg_s / 1e9
+            roof = {"kernel": name, "bound": "hbm", "achieved": round(ach, 1),
+                    "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(ach / peaks["hbm_gbs"], 4),
+                    "peak_kind": f"HBM copy, {peak_kind}", "traffic": None,
+                    "algorithmic_per_launch": per["bytes"], "avg_launch_ms": 1000 * avg_s}
+        t_roof = max(alg["flops"] / (peaks["bf16_tflops"] * 1e12), alg["bytes"] / (peaks["hbm_gbs"] * 1e9))
+        cpu = None
+        if world == 1 and not args.no_cpu_baseline:
+            rate, n, dt = _replay_oracle_rate(wl, layers, budget_s=15.0)
+            cpu = {"value": rate, "unit": UNIT, "cores": omp_cores(), "kind": "oracle",
+                   "sample": f"{n} random (layer, batch, head, position) queries, {dt:.1f} s; "
+                             f"a token = one position through all {wl.n_layers_tgt} layers and "
+                             f"{wl.q_heads} heads"}
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": t_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded N(0,1) queries and replay caches; guidance maps with "
+                    "sink, recency and heavy-column structure)",
+            "config": {"workload": replay_desc(wl), "tokens_per_step": wl.tokens,
+                       "parallelism": "replicas" if world > 1 else "single GPU",
+                       "l2": "each step reads %.2f GB (queries, caches, guidance maps), more than L2"
+                             % (alg["bytes"] / 1e9)},
+            "roofline": roof,
+            "step_roofline": {"flops": alg["flops"], "bytes": alg["bytes"],
+                              "roofline_ms": 1000 * t_roof, "frac": round(1000 * t_roof / t_step, 4),
+                              "peaks": f"bf16 {peaks['bf16_tflops']} TFLOP/s burst, HBM {peaks['hbm_gbs']} GB/s ({peak_kind})"},
+            "kernels": {k: {"launches": v[0], "total_ms": round(v[1], 3),
+                            "share": round(v[1] / sum(x[1] for x in kstats.values()), 4)}
+                        for k, v in kstats.items()},
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+                    "api": "mot_replay_attention per layer with pinned host copies of its inputs "
+                           "and output on its stream"},
+            "gpu_launches": launches,
+            "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+    M.mot_destroy(h)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=500)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["mot", "reference"], default="mot")
-    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
+                    choices=sorted(synth.WORKLOADS) + sorted(synth.REPLAY_WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--schedule", choices=["auto", "onchip", "pair", "fused", "split"],
                     default="auto",
@@ -628,6 +903,9 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mot":
         args.warmup = 3
+    if args.workload in synth.REPLAY_WORKLOADS:
+        wl = synth.REPLAY_WORKLOADS[args.workload]
+        return run_replay_reference(args, wl) if args.impl == "reference" else run_replay(args, wl)
     wl = synth.WORKLOADS[args.workload]
     if args.top_k > 0:
         wl = wl.replace(name=f"{wl.name}_top{args.top_k}", top_k=args.top_k)

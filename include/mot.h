@@ -360,7 +360,7 @@ mot_status mot_translate_bt(mot_handle h, const void* src_k, const void* src_v,
  * target cache); guide [max_batch][max_seq][max_seq] (row u, column j; only
  * j <= u is read; guide may be NULL for full layers). Rows u >= seq_lens[b] of
  * out are not written. seq_lens: device int32[batch], clamped to [0, max_seq].
- * Requires head_dim in {64, 128}, q_heads / kv_heads <= 16, top_s <= 4096,
+ * Requires head_dim in {64, 128}, q_heads / kv_heads in 1..8, 12 or 16, top_s <= 4096,
  * max_seq <= 65536 (else MOT_ERR_UNSUPPORTED). Asynchronous on `stream`.
  *
  * mot_replay_select writes the selection alone: sel [max_batch][max_seq][top_s]

@@ -155,6 +155,7 @@ struct mot_ctx {
   // replay attention (App. C.4): kind 3
   ReplayDims rd{};
   int32_t* rsel = nullptr;   // [B][N][S] selection workspace
+  void* rvt = nullptr;       // [B][Hkv][d][N] bf16: V^T for the tensor-core full attention
   // Top-K routing (tensor-core path, 0 < top_k < E): token buckets per expert
   bool sparse_ok = false;   // the shapes support it
   int routing = 0;          // 0 dense compute with a zeroed gate, 1 token buckets
@@ -197,7 +198,7 @@ void free_all(mot_ctx* h) {
                   h->sp.row0, h->sp.plan, h->sp.pairs, h->sp.ltok, h->sp.lslot, h->sp.gatep,
                   h->sp.gate16p, h->sp.zp, h->sp.a2p, h->sp.ybuf, h->wkv, h->ahat,
                   h->proj_layer,
-                  h->rsel,
+                  h->rsel, h->rvt,
                   h->n_tiles, h->status, h->counters, h->st_src[0], h->st_src[1], h->st_dst[0],
                   h->st_dst[1], h->st_len};
   for (void* p : ptrs)
@@ -1460,7 +1461,9 @@ mot_status mot_create_replay(const mot_replay_config* cfg, mot_handle* out) {
     delete h;
     return MOT_ERR_UNSUPPORTED;
   }
+  const size_t vt_bytes = replay_fmha_supported(rd) ? size_t(rd.B) * rd.Hkv * rd.d * rd.N * 2 : 16;
   if (cudaMalloc(&h->rsel, size_t(rd.B) * rd.N * rd.S * 4) != cudaSuccess ||
+      cudaMalloc(&h->rvt, vt_bytes) != cudaSuccess ||
       cudaMalloc(&h->status, 16) != cudaSuccess || cudaMemset(h->status, 0, 16) != cudaSuccess) {
     cudaGetLastError();
     free_all(h);
@@ -1498,6 +1501,7 @@ mot_status replay_args(mot_handle h, const void* q, const void* k, const void* v
   a.sel = h->rsel;
   a.seq_lens = seq_lens;
   a.batch = batch;
+  a.status = h->status;
   return MOT_OK;
 }
 
@@ -1531,6 +1535,23 @@ mot_status mot_replay_attention(mot_handle h, int32_t layer, const void* q, cons
   if (batch == 0) return MOT_OK;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   a.full = full ? 1 : 0;
+  const ReplayDims& d = h->rd;
+  if (full && replay_fmha_supported(d) && encode_fn()) {
+    // tensor-core causal attention: V^T first, then one launch over all query tiles
+    CUtensorMap tmQ{}, tmK{}, tmVt{};
+    const uint64_t qd[2] = {uint64_t(d.d), uint64_t(d.B) * d.Hq * d.N};
+    const uint64_t kd[2] = {uint64_t(d.d), uint64_t(d.B) * d.Hkv * d.N};
+    const uint64_t vd[2] = {uint64_t(d.N), uint64_t(d.B) * d.Hkv * d.d};
+    const uint64_t qs[1] = {uint64_t(d.d) * 2}, vs[1] = {uint64_t(d.N) * 2};
+    const uint32_t box[2] = {64, 128}, vbox[2] = {64, uint32_t(d.d)};
+    if (!encode_bf16(&tmQ, q, 2, qd, qs, box) || !encode_bf16(&tmK, k, 2, kd, qs, box) ||
+        !encode_bf16(&tmVt, h->rvt, 2, vd, vs, vbox))
+      return MOT_ERR_CUDA;
+    MOT_CUDA_TRY(timed(h, "replay_vt", st, [&] { return launch_replay_vt(a, h->rvt, st); }));
+    MOT_CUDA_TRY(timed(h, "replay_fmha_full", st,
+                       [&] { return launch_replay_fmha(a, tmQ, tmK, tmVt, st); }));
+    return MOT_OK;
+  }
   if (!full)
     MOT_CUDA_TRY(timed(h, "replay_select", st, [&] { return launch_replay_select(a, st); }));
   MOT_CUDA_TRY(timed(h, full ? "replay_attn_full" : "replay_attn_sparse", st,

@@ -206,8 +206,16 @@ struct ReplayArgs {
   const int32_t* seq_lens;
   int32_t batch;
   int32_t full;   // 1: attend to every position 0..u
+  int32_t* status;
 };
 bool replay_supported(const ReplayDims& d);
+// Full causal attention on the tensor cores: maps over q [B*Hq*N][d], k
+// [B*Hkv*N][d] (box 64 x 128) and V^T [B*Hkv*d][N] (box 64 x d), the last
+// written by launch_replay_vt into `vt`.
+bool replay_fmha_supported(const ReplayDims& d);
+cudaError_t launch_replay_vt(const ReplayArgs& a, void* vt, cudaStream_t st);
+cudaError_t launch_replay_fmha(const ReplayArgs& a, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+                               const CUtensorMap& tmVt, cudaStream_t st);
 cudaError_t launch_replay_select(const ReplayArgs& a, cudaStream_t st);
 cudaError_t launch_replay_attn(const ReplayArgs& a, cudaStream_t st);
 

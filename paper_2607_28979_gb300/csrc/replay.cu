@@ -20,16 +20,33 @@
 //                         the softmax is fp32, and thread i accumulates output
 //                         dimension i over the chunk's value rows (coalesced
 //                         across the warp).
+//   replay_fmha_kernel    full causal attention on the tensor cores (layers below
+//                         L_Full): one CTA per (b, query head, 128-query tile),
+//                         persistent over its key tiles 0..diagonal.
+//                           warp 0  TMA: the Q tile once, then K and V^T tiles
+//                                   (V transposed per layer by replay_vt_kernel so
+//                                   both MMAs read K-major operands) into 2 stages;
+//                           warp 1  S = Q K^T (M=128, N=128 keys) and, one tile
+//                                   later, PV = P V (M=128, N=d), into double-
+//                                   buffered TMEM;
+//                           warps 4..7  one query row per thread: the scaled,
+//                                   masked row of S from TMEM, its running max and
+//                                   sum (base-2 exponentials), P as bf16 into a
+//                                   128B-swizzled SMEM tile for the second MMA, and
+//                                   the output row in registers, rescaled by
+//                                   exp2(m_old - m_new) before each PV is added.
+//                         Every wait is bounded; on a timeout the roles unwind,
+//                         copies and MMAs in flight are drained and TMEM is freed.
 #include <cuda_bf16.h>
 
 #include "mot_internal.h"
+#include "ptx.cuh"
 
 namespace mot {
 namespace {
 
 constexpr int kSelThreads = 256;
 constexpr int kAttnThreads = 128;   // = the key chunk
-constexpr int kMaxGroup = 16;       // query heads per key/value head
 
 __device__ __forceinline__ float bf16f(uint16_t b) { return __uint_as_float(uint32_t(b) << 16); }
 
@@ -126,14 +143,13 @@ __global__ void __launch_bounds__(kSelThreads) replay_select_kernel(const Replay
     if (((ord16(A[j]) << 16) | (0xFFFFu - uint32_t(j))) >= thr) out[pos++] = j;
 }
 
-template <int D>
+template <int D, int G>
 __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayArgs a) {
-  __shared__ float qs[kMaxGroup][D];
-  __shared__ float ps[kMaxGroup][kAttnThreads];
+  __shared__ float qs[G][D];
+  __shared__ float ps[G][kAttnThreads];
   __shared__ int32_t idx[kAttnThreads];
-  __shared__ float red[kMaxGroup][kAttnThreads / 32];
+  __shared__ float red[G][kAttnThreads / 32];
   const ReplayDims& d = a.d;
-  const int G = d.Hq / d.Hkv;
   const int u = blockIdx.x;
   const int hk = blockIdx.y % d.Hkv, b = blockIdx.y / d.Hkv;
   if (u >= seq_len_of(a, b)) return;
@@ -151,7 +167,8 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
   const int32_t* sel = a.sel + (int64_t(b) * d.N + u) * d.S;
   const uint16_t* kb = static_cast<const uint16_t*>(a.k) + (int64_t(b) * d.Hkv + hk) * d.N * D;
   const uint16_t* vb = static_cast<const uint16_t*>(a.v) + (int64_t(b) * d.Hkv + hk) * d.N * D;
-  float m[kMaxGroup], l[kMaxGroup], acc[kMaxGroup];
+  float m[G], l[G], acc[G];
+#pragma unroll
   for (int g = 0; g < G; ++g) {
     m[g] = -INFINITY;
     l[g] = 0.f;
@@ -163,10 +180,12 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
     const int j = t < nc ? (full ? c0 + t : sel[c0 + t]) : -1;
     idx[t] = j;
     // scores of key t against every query of the group
-    float s[kMaxGroup];
+    float s[G];
+#pragma unroll
     for (int g = 0; g < G; ++g) s[g] = -INFINITY;
     if (j >= 0) {
       const uint4* k4 = reinterpret_cast<const uint4*>(kb + int64_t(j) * D);
+#pragma unroll
       for (int g = 0; g < G; ++g) s[g] = 0.f;
 #pragma unroll 4
       for (int c = 0; c < D / 8; ++c) {
@@ -175,12 +194,14 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const float k0 = __uint_as_float(ww[e] << 16), k1 = __uint_as_float(ww[e] & 0xFFFF0000u);
+#pragma unroll
           for (int g = 0; g < G; ++g)
             s[g] = fmaf(qs[g][8 * c + 2 * e + 1], k1, fmaf(qs[g][8 * c + 2 * e], k0, s[g]));
         }
       }
     }
     // chunk maxima per query
+#pragma unroll
     for (int g = 0; g < G; ++g) {
       float x = s[g];
 #pragma unroll
@@ -188,7 +209,8 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
       if (lane == 0) red[g][warp] = x;
     }
     __syncthreads();
-    float mnew[kMaxGroup], corr[kMaxGroup];
+    float mnew[G], corr[G];
+#pragma unroll
     for (int g = 0; g < G; ++g) {
       float x = red[g][0];
       for (int w = 1; w < kAttnThreads / 32; ++w) x = fmaxf(x, red[g][w]);
@@ -198,6 +220,7 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
     }
     __syncthreads();
     // sums and the weighted value rows (thread t owns output dimension t)
+#pragma unroll
     for (int g = 0; g < G; ++g) {
       float x = ps[g][t];
 #pragma unroll
@@ -205,6 +228,7 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
       if (lane == 0) red[g][warp] = x;
     }
     __syncthreads();
+#pragma unroll
     for (int g = 0; g < G; ++g) {
       float x = 0.f;
       for (int w = 0; w < kAttnThreads / 32; ++w) x += red[g][w];
@@ -215,6 +239,7 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
     if (t < D) {
       for (int jj = 0; jj < nc; ++jj) {
         const float vv = bf16f(vb[int64_t(idx[jj]) * D + t]);
+#pragma unroll
         for (int g = 0; g < G; ++g) acc[g] = fmaf(ps[g][jj], vv, acc[g]);
       }
     }
@@ -222,6 +247,7 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
   }
   if (t < D) {
     uint16_t* o = static_cast<uint16_t*>(a.out);
+#pragma unroll
     for (int g = 0; g < G; ++g) {
       const int h = hk * G + g;
       __nv_bfloat16 r = __float2bfloat16_rn(acc[g] / l[g]);
@@ -230,10 +256,347 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
   }
 }
 
+
+// ---------------------------------------------------------------- V^T for the tensor-core path
+
+// vt[(b * Hkv + hk) * d + i][j] = v[(b * Hkv + hk) * N + j][i], 32 x 32 tiles through SMEM.
+__global__ void __launch_bounds__(256) replay_vt_kernel(const uint16_t* __restrict__ v,
+                                                         uint16_t* __restrict__ vt, int N, int D) {
+  __shared__ uint16_t tile[32][33];
+  const int bh = blockIdx.z;
+  const int j0 = blockIdx.x * 32, i0 = blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 32 x 8
+  const uint16_t* src = v + int64_t(bh) * N * D;
+  uint16_t* dst = vt + int64_t(bh) * D * N;
+  for (int r = ty; r < 32; r += 8) {
+    const int j = j0 + r, i = i0 + tx;
+    tile[r][tx] = (j < N && i < D) ? src[int64_t(j) * D + i] : 0;
+  }
+  __syncthreads();
+  for (int r = ty; r < 32; r += 8) {
+    const int i = i0 + r, j = j0 + tx;
+    if (i < D && j < N) dst[int64_t(i) * N + j] = tile[tx][r];
+  }
+}
+
+// ---------------------------------------------------------------- tensor-core causal attention
+
+template <int D>
+struct Fa {
+  static constexpr int kQ = 128 * D * 2;      // Q tile: D/64 blocks of 128 rows x 128 B
+  static constexpr int kK = 128 * D * 2;      // K tile, same layout
+  static constexpr int kVtBlk = D * 128;      // one V^T block: D rows x 64 keys
+  static constexpr int kVt = 2 * kVtBlk;      // V^T tile: 128 keys
+  static constexpr int kPBlk = 128 * 128;     // one P block: 128 rows x 64 keys
+  static constexpr int kP = 2 * kPBlk;
+  static constexpr int kBytes = kQ + 2 * kK + 2 * kVt + 2 * kP;
+  static constexpr int kSmem = kBytes + 256 + 1024;
+  static constexpr int kThreads = 256;
+};
+static_assert(Fa<128>::kSmem <= 232448, "shared memory budget");
+
+// chunk store of 32 bf16 (16 words) into row r of a 128B-swizzled 64-column block,
+// half s (columns 32 s .. 32 s + 31)
+__device__ __forceinline__ void st_sw128_half(uint32_t blk, int r, int s, const uint32_t (&pk)[16]) {
+  const uint32_t row = blk + static_cast<uint32_t>(r * 128);
+#pragma unroll
+  for (int v = 0; v < 4; ++v)
+    st_shared_v4(row + static_cast<uint32_t>(((4 * s + v) ^ (r & 7)) << 4), pk[4 * v],
+                 pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+}
+
+template <int D>
+__global__ void __launch_bounds__(Fa<D>::kThreads, 1)
+    replay_fmha_kernel(const __grid_constant__ CUtensorMap tmQ,
+                       const __grid_constant__ CUtensorMap tmK,
+                       const __grid_constant__ CUtensorMap tmVt, const ReplayArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sK = sQ + Fa<D>::kQ;              // [2]
+  uint8_t* sV = sK + 2 * Fa<D>::kK;          // [2]
+  uint8_t* sP = sV + 2 * Fa<D>::kVt;         // [2]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + 2 * Fa<D>::kP);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;      // [2]
+  uint64_t* kv_empty = bars + 3;     // [2]
+  uint64_t* s_full = bars + 5;       // [2]
+  uint64_t* s_empty = bars + 7;      // [2]
+  uint64_t* p_full = bars + 9;       // [2]
+  uint64_t* p_empty = bars + 11;     // [2]
+  uint64_t* pv_full = bars + 13;     // [2]
+  uint64_t* pv_empty = bars + 15;    // [2]
+  uint64_t* drain = bars + 17;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const ReplayDims& d = a.d;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_qt = (d.N + 127) / 128;
+  const int qt = n_qt - 1 - static_cast<int>(blockIdx.x % n_qt);   // heavy tiles first
+  const int bh = static_cast<int>(blockIdx.x / n_qt);
+  const int b = bh / d.Hq, h = bh - b * d.Hq;
+  const int hk = h / (d.Hq / d.Hkv);
+  const int L = seq_len_of(a, b);
+  const int q0 = qt * 128;
+  if (q0 >= L) return;   // uniform over the CTA: no barrier or TMEM use yet
+  const int n_kv = qt + 1;
+  const long long wl = 4000000000LL;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&kv_full[i], 1);
+      mbar_init(&kv_empty[i], 1);
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_empty[i], 4);
+      mbar_init(&p_full[i], 4);
+      mbar_init(&p_empty[i], 1);
+      mbar_init(&pv_full[i], 1);
+      mbar_init(&pv_empty[i], 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmVt);
+  }
+  if (warp == 2) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;   // S[i] at columns 128 i, PV[i] at 256 + D i
+  uint32_t issued_mask = 0, issue_parity = 0;
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      const int qrow = (b * d.Hq + h) * d.N + q0;
+      mbar_arrive_expect_tx(q_full, Fa<D>::kQ);
+      for (int kb = 0; kb < D / 64; ++kb)
+        tma_load_2d(sQ + kb * 128 * 128, &tmQ, q_full, kb * 64, qrow);
+      const int krow = (b * d.Hkv + hk) * d.N, vrow = (b * d.Hkv + hk) * D;
+      for (int j = 0; j < n_kv; ++j) {
+        const int st = j & 1;
+        if (!mbar_wait(&kv_empty[st], ((j >> 1) & 1) ^ 1u, abort_flag, wl)) break;
+        mbar_arrive_expect_tx(&kv_full[st], Fa<D>::kK + Fa<D>::kVt);
+        for (int kb = 0; kb < D / 64; ++kb)
+          tma_load_2d(sK + st * Fa<D>::kK + kb * 128 * 128, &tmK, &kv_full[st], kb * 64,
+                      krow + j * 128);
+        for (int kb = 0; kb < 2; ++kb)
+          tma_load_2d(sV + st * Fa<D>::kVt + kb * Fa<D>::kVtBlk, &tmVt, &kv_full[st],
+                      j * 128 + kb * 64, vrow);
+        issued_mask |= 1u << st;
+        issue_parity = (issue_parity & ~(1u << st)) | (uint32_t((j >> 1) & 1) << st);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer (warp-uniform, elected lane)
+    const uint32_t idS = idesc_bf16_f32(128, 128), idPV = idesc_bf16_f32(128, D);
+    bool ok = mbar_wait(q_full, 0, abort_flag, wl);
+    tc_fence_after();
+    auto issue_s = [&](int j) -> bool {   // S[j & 1] = Q K_j^T
+      const int st = j & 1;
+      if (!mbar_wait(&kv_full[st], (j >> 1) & 1, abort_flag, wl)) return false;
+      if (!mbar_wait(&s_empty[st], ((j >> 1) & 1) ^ 1u, abort_flag, wl)) return false;
+      tc_fence_after();
+      if (elect_one()) {
+        for (int kb = 0; kb < D / 64; ++kb) {
+          const uint64_t ad = sdesc_k_sw128(smem_u32(sQ + kb * 128 * 128));
+          const uint64_t bd = sdesc_k_sw128(smem_u32(sK + st * Fa<D>::kK + kb * 128 * 128));
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_bf16(tmem + st * 128, ad + 2 * k, bd + 2 * k, idS, (kb | k) != 0);
+        }
+        umma_commit(&s_full[st]);
+      }
+      __syncwarp();
+      mma_issued = true;
+      return true;
+    };
+    auto issue_pv = [&](int j) -> bool {   // PV[j & 1] = P_j V_j (B = V_j^T, K-major)
+      const int st = j & 1;
+      if (!mbar_wait(&p_full[st], (j >> 1) & 1, abort_flag, wl)) return false;
+      if (!mbar_wait(&pv_empty[st], ((j >> 1) & 1) ^ 1u, abort_flag, wl)) return false;
+      tc_fence_after();
+      if (elect_one()) {
+        for (int kb = 0; kb < 2; ++kb) {
+          const uint64_t ad = sdesc_k_sw128(smem_u32(sP + st * Fa<D>::kP + kb * Fa<D>::kPBlk));
+          const uint64_t bd =
+              sdesc_k_sw128(smem_u32(sV + st * Fa<D>::kVt + kb * Fa<D>::kVtBlk));
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            umma_bf16(tmem + 256 + st * D, ad + 2 * k, bd + 2 * k, idPV, (kb | k) != 0);
+        }
+        umma_commit(&pv_full[st]);
+        umma_commit(&p_empty[st]);
+        umma_commit(&kv_empty[st]);
+      }
+      __syncwarp();
+      return true;
+    };
+    if (ok) ok = issue_s(0);
+    for (int j = 0; ok && j < n_kv; ++j) {
+      if (j + 1 < n_kv) ok = issue_s(j + 1);
+      if (ok) ok = issue_pv(j);
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------ softmax and output rows
+    const int r = (warp & 3) * 32 + lane;
+    const uint32_t lanes = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    const float sl2 = rsqrtf(float(D)) * 1.4426950408889634f;   // scale * log2(e)
+    float o[D];
+#pragma unroll
+    for (int i = 0; i < D; ++i) o[i] = 0.f;
+    float m = -INFINITY, l = 0.f, alpha_prev = 0.f;
+    bool ok = true;
+    auto apply_pv = [&](int j, float alpha) -> bool {   // o = o * alpha + PV_j
+      const int st = j & 1;
+      int w = 1;
+      if (lane == 0) w = mbar_wait(&pv_full[st], (j >> 1) & 1, abort_flag, wl) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, w, 0)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(tmem + lanes + 256 + st * D + c * 32, v);
+        tmem_ld_wait(v);
+#pragma unroll
+        for (int k = 0; k < 32; ++k) o[c * 32 + k] = fmaf(o[c * 32 + k], alpha, __uint_as_float(v[k]));
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&pv_empty[st]);
+      return true;
+    };
+    for (int j = 0; j < n_kv; ++j) {
+      const int st = j & 1;
+      int w = 1;
+      if (lane == 0) w = mbar_wait(&s_full[st], (j >> 1) & 1, abort_flag, wl) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+      tc_fence_after();
+      const bool diag = j == qt;
+      // pass 1: the row maximum of the scaled, masked scores
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(tmem + lanes + st * 128 + c * 32, v);
+        tmem_ld_wait(v);
+#pragma unroll
+        for (int k = 0; k < 32; ++k)
+          if (!diag || c * 32 + k <= r) mx = fmaxf(mx, __uint_as_float(v[k]) * sl2);
+      }
+      const float m_new = fmaxf(m, mx);
+      const float alpha = m == -INFINITY ? 0.f : exp2f(m - m_new);
+      // P_j must not overwrite the buffer before PV_{j-2} has read it
+      w = 1;
+      if (lane == 0) w = mbar_wait(&p_empty[st], ((j >> 1) & 1) ^ 1u, abort_flag, wl) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+      // pass 2: P = exp2(s - m_new) as bf16 into the swizzled P tile, and its row sum
+      float sum = 0.f;
+      const uint32_t pbase = smem_u32(sP + st * Fa<D>::kP);
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(tmem + lanes + st * 128 + c * 32, v);
+        tmem_ld_wait(v);
+        uint32_t pk[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) {
+          const int c0 = c * 32 + 2 * k;
+          const float p0 = (!diag || c0 <= r) ? exp2f(__uint_as_float(v[2 * k]) * sl2 - m_new) : 0.f;
+          const float p1 = (!diag || c0 + 1 <= r) ? exp2f(__uint_as_float(v[2 * k + 1]) * sl2 - m_new) : 0.f;
+          __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
+          // the row sum counts the rounded probabilities the second MMA uses
+          const float2 pr = __bfloat1622float2(pb);
+          sum += pr.x + pr.y;
+          pk[k] = *reinterpret_cast<uint32_t*>(&pb);
+        }
+        st_sw128_half(pbase + (c >> 1) * Fa<D>::kPBlk, r, c & 1, pk);
+      }
+      tc_fence_before();
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(&s_empty[st]);
+        mbar_arrive(&p_full[st]);
+      }
+      l = l * alpha + sum;
+      m = m_new;
+      if (j > 0 && !apply_pv(j - 1, alpha_prev)) { ok = false; break; }
+      alpha_prev = alpha;
+    }
+    if (ok && apply_pv(n_kv - 1, alpha_prev)) {
+      const int q = q0 + r;
+      if (q < L) {
+        const float inv = 1.f / l;
+        uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.out) +
+                                              ((int64_t(b) * d.Hq + h) * d.N + q) * D);
+#pragma unroll
+        for (int c = 0; c < D / 8; ++c) {
+          uint32_t w4[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            __nv_bfloat162 t = __floats2bfloat162_rn(o[8 * c + 2 * e] * inv, o[8 * c + 2 * e + 1] * inv);
+            w4[e] = *reinterpret_cast<uint32_t*>(&t);
+          }
+          dst[c] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+        }
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort_flag) {
+    if (warp == 0 && lane == 0) {
+      for (int st = 0; st < 2; ++st)
+        if ((issued_mask >> st) & 1u) {
+          const uint32_t ad = smem_u32(&kv_full[st]);
+          const long long t0 = clock64();
+          while (!mbar_try_wait(ad, (issue_parity >> st) & 1u) && clock64() - t0 < wl) {
+          }
+        }
+      const uint32_t aq = smem_u32(q_full);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(aq, 0) && clock64() - t0 < wl) {
+      }
+    }
+    if (warp == 1 && mma_issued) {
+      if (elect_one()) umma_commit(drain);
+      __syncwarp();
+      const uint32_t ad = smem_u32(drain);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(ad, 0) && clock64() - t0 < wl) {
+      }
+    }
+    __syncthreads();
+  }
+  if (warp == 2) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicOr(a.status, kStatusTimeout);
+}
 }  // namespace
 
+// GQA group sizes with an instantiated attention kernel
+__host__ __device__ constexpr bool group_ok(int g) {
+  return (g >= 1 && g <= 8) || g == 12 || g == 16;
+}
+
 bool replay_supported(const ReplayDims& d) {
-  return d.Hkv > 0 && d.Hq % d.Hkv == 0 && d.Hq / d.Hkv <= kMaxGroup &&
+  return d.Hkv > 0 && d.Hq % d.Hkv == 0 && group_ok(d.Hq / d.Hkv) &&
          (d.d == 64 || d.d == 128) && d.S >= 1 && d.S <= 4096 && d.N >= 1 && d.N <= 65536;
 }
 
@@ -244,12 +607,51 @@ cudaError_t launch_replay_select(const ReplayArgs& a, cudaStream_t st) {
   return cudaGetLastError();
 }
 
+bool replay_fmha_supported(const ReplayDims& d) {
+  return (d.d == 64 || d.d == 128) && d.N % 8 == 0;
+}
+
+cudaError_t launch_replay_vt(const ReplayArgs& a, void* vt, cudaStream_t st) {
+  const ReplayDims& d = a.d;
+  dim3 grid((d.N + 31) / 32, (d.d + 31) / 32, d.B * d.Hkv);
+  replay_vt_kernel<<<grid, 256, 0, st>>>(static_cast<const uint16_t*>(a.v),
+                                         static_cast<uint16_t*>(vt), d.N, d.d);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_replay_fmha(const ReplayArgs& a, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+                               const CUtensorMap& tmVt, cudaStream_t st) {
+  const ReplayDims& d = a.d;
+  static bool attr[2] = {false, false};
+  const int di = d.d == 128 ? 1 : 0;
+  auto kern = d.d == 128 ? replay_fmha_kernel<128> : replay_fmha_kernel<64>;
+  const int smem = d.d == 128 ? Fa<128>::kSmem : Fa<64>::kSmem;
+  if (!attr[di]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    attr[di] = true;
+  }
+  const int n_qt = (d.N + 127) / 128;
+  kern<<<d.B * d.Hq * n_qt, 256, smem, st>>>(tmQ, tmK, tmVt, a);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_replay_attn(const ReplayArgs& a, cudaStream_t st) {
   dim3 grid(a.d.N, a.d.B * a.d.Hkv);
-  if (a.d.d == 128)
-    replay_attn_kernel<128><<<grid, kAttnThreads, 0, st>>>(a);
-  else
-    replay_attn_kernel<64><<<grid, kAttnThreads, 0, st>>>(a);
+  const int G = a.d.Hq / a.d.Hkv;
+#define MOT_RP_CASE(GG)                                                          \
+  case GG:                                                                       \
+    if (a.d.d == 128)                                                            \
+      replay_attn_kernel<128, GG><<<grid, kAttnThreads, 0, st>>>(a);             \
+    else                                                                         \
+      replay_attn_kernel<64, GG><<<grid, kAttnThreads, 0, st>>>(a);              \
+    break;
+  switch (G) {
+    MOT_RP_CASE(1) MOT_RP_CASE(2) MOT_RP_CASE(3) MOT_RP_CASE(4) MOT_RP_CASE(5)
+    MOT_RP_CASE(6) MOT_RP_CASE(7) MOT_RP_CASE(8) MOT_RP_CASE(12) MOT_RP_CASE(16)
+    default: return cudaErrorInvalidValue;
+  }
+#undef MOT_RP_CASE
   return cudaGetLastError();
 }
 

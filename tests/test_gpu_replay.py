@@ -137,6 +137,20 @@ def test_full_size_layer_sampled():
         G.assert_parity(BF16, _f64(out)[tb, th, tu], ref, f"full-size layer {layer}")
 
 
+def test_full_layers_use_the_tensor_core_kernel():
+    """max_seq % 8 == 0: full layers run the tcgen05 attention kernel (after the V
+    transpose); guided layers run the selection and the gather kernel."""
+    wl = SMALL["r_mha_d64"]
+    q, k, v = synth.gen_replay_qkv(wl, 0)
+    g = synth.gen_guide(wl, 0)
+    run = ReplayRun(wl)
+    M.mot_profile_enable(run.h, True)
+    run.attend(0, q, k, v, None)
+    run.attend(2, q, k, v, g)
+    prof = M.mot_profile_read(run.h)
+    assert set(prof) == {"replay_vt", "replay_fmha_full", "replay_select", "replay_attn_sparse"}
+
+
 def test_batch_prefix_and_errors():
     wl = SMALL["r_mha_d64"]
     q, k, v = synth.gen_replay_qkv(wl, 0)

@@ -2,24 +2,25 @@
 // Top-S source-guided sparse attention, and full causal attention for the
 // L_Full bottom layers.
 //
-//   replay_select_kernel  one CTA per context row (b, u): the S positions j <= u
+//   replay_select_kernel  one warp per context row (b, u): the S positions j <= u
 //                         with the largest guidance score A[b][u][j] (ties to the
-//                         lower position), written in ascending order. Each
-//                         candidate gets the unique 32-bit key
-//                         (order-preserving bits of A) << 16 | (0xFFFF - j), so the
-//                         selection is exact integer work: an MSB-first radix
-//                         select (four 8-bit digits, 256-bin shared histograms)
-//                         finds the S-th largest key, and a block scan compacts
-//                         the keys at or above it. Rows with u + 1 <= S take every
-//                         position.
+//                         lower position), written in ascending order. It is exact
+//                         integer work on the order-preserving 16-bit image of each
+//                         score: two 256-bin histogram passes (high byte, then low
+//                         byte, warp-aggregated increments) find the score V of the
+//                         S-th largest (score, -position) key and how many of the
+//                         positions scoring V it takes; ballots then keep every
+//                         score above V and the lowest positions at V. Rows with
+//                         u + 1 <= S take every position.
 //   replay_attn_kernel    one CTA per (b, key/value head, u): the query heads of
 //                         the GQA group attend to the selected rows (sparse) or to
 //                         positions 0..u in 128-key chunks with an online softmax
 //                         (full). Thread t scores key t of the chunk against every
 //                         query of the group (its key row read as 16-byte vectors),
-//                         the softmax is fp32, and thread i accumulates output
-//                         dimension i over the chunk's value rows (coalesced
-//                         across the warp).
+//                         the softmax is fp32, and each thread accumulates 4 output
+//                         dimensions over every (128 / (d / 4))-th value row of the
+//                         chunk (8-byte reads); the row groups are summed within
+//                         the warp and then warp by warp in a fixed order.
 //   replay_fmha_kernel    full causal attention on the tensor cores (layers below
 //                         L_Full): one CTA per (b, query head, 128-query tile),
 //                         persistent over its key tiles 0..diagonal.
@@ -45,7 +46,6 @@
 namespace mot {
 namespace {
 
-constexpr int kSelThreads = 256;
 constexpr int kAttnThreads = 128;   // = the key chunk
 
 __device__ __forceinline__ float bf16f(uint16_t b) { return __uint_as_float(uint32_t(b) << 16); }
@@ -61,99 +61,150 @@ __device__ __forceinline__ int seq_len_of(const ReplayArgs& a, int b) {
   return L < 0 ? 0 : (L > a.d.N ? a.d.N : L);
 }
 
-// Exclusive scan of one value per thread over the block (kSelThreads threads).
-__device__ __forceinline__ int block_excl_scan(int v, int* warp_sums, int& total) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+constexpr int kSelWarps = 8;         // rows per CTA, one warp each
+
+// Warp-wide exclusive prefix of v (and the warp total).
+__device__ __forceinline__ int warp_excl_scan(int v, int& total) {
+  const int lane = threadIdx.x & 31;
   int x = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
     const int y = __shfl_up_sync(0xffffffffu, x, o);
     if (lane >= o) x += y;
   }
-  if (lane == 31) warp_sums[warp] = x;
-  __syncthreads();
-  if (warp == 0) {
-    int w = lane < kSelThreads / 32 ? warp_sums[lane] : 0;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, w, o);
-      if (lane >= o) w += y;
-    }
-    if (lane < kSelThreads / 32) warp_sums[lane] = w;   // inclusive warp prefix
-  }
-  __syncthreads();
-  const int before = warp > 0 ? warp_sums[warp - 1] : 0;
-  total = warp_sums[kSelThreads / 32 - 1];
-  __syncthreads();
-  return before + x - v;
+  total = __shfl_sync(0xffffffffu, x, 31);
+  return x - v;
 }
 
-__global__ void __launch_bounds__(kSelThreads) replay_select_kernel(const ReplayArgs a) {
-  __shared__ int hist[256];
-  __shared__ int warp_sums[kSelThreads / 32];
-  __shared__ uint32_t s_prefix;
-  __shared__ int s_k;
+// One warp per context row (b, u). With o = the order-preserving 16 bits of a
+// score, the S-th largest (o, -j) key is found in two histogram passes over o
+// (high byte, then low byte): V = its score bits, k = how many positions with
+// o == V it takes. The selection is then every o > V plus the k lowest
+// positions with o == V, compacted in ascending order by warp scans.
+__global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const ReplayArgs a) {
+  __shared__ int hist[kSelWarps][256];
   const ReplayDims& d = a.d;
-  const int row = blockIdx.x;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = blockIdx.x * kSelWarps + w;
+  if (row >= d.B * d.N) return;
   const int b = row / d.N, u = row - b * d.N;
   if (u >= seq_len_of(a, b)) return;
   int32_t* out = a.sel + int64_t(row) * d.S;
   const int n = u + 1;
   if (n <= d.S) {
-    for (int j = threadIdx.x; j < d.S; j += kSelThreads) out[j] = j < n ? j : -1;
+    for (int j = lane; j < d.S; j += 32) out[j] = j < n ? j : -1;
     return;
   }
   const uint16_t* A = static_cast<const uint16_t*>(a.guide) + int64_t(row) * d.N;
-  // this thread's contiguous chunk of candidates (ascending positions across threads)
-  const int C = (n + kSelThreads - 1) / kSelThreads;
-  const int j0 = min(n, int(threadIdx.x) * C), j1 = min(n, j0 + C);
-  if (threadIdx.x == 0) {
-    s_prefix = 0;
-    s_k = d.S;
+  // three passes read the row (from L2 after the first); no shared copy, so
+  // that every SM keeps 64 rows in flight
+  auto ord_at = [&](int j) -> uint32_t { return ord16(__ldg(A + j)); };
+  int* hw = hist[w];
+  int k = d.S;
+  uint32_t hi = 0;
+  // pass 1: high byte of the score bits (strided over the lanes)
+  for (int i = lane; i < 256; i += 32) hw[i] = 0;
+  __syncwarp();
+  for (int j0 = 0; j0 < n; j0 += 32) {
+    const int j = j0 + lane;
+    const int bin = j < n ? int(ord_at(j) >> 8) : 256;
+    const unsigned peers = __match_any_sync(0xffffffffu, bin);
+    if (bin < 256 && lane == __ffs(peers) - 1) atomicAdd(&hw[bin], __popc(peers));
   }
-  // MSB-first radix select of the S-th largest key (digits of 8 bits)
-  for (int shift = 24; shift >= 0; shift -= 8) {
-    for (int i = threadIdx.x; i < 256; i += kSelThreads) hist[i] = 0;
-    __syncthreads();
-    const uint32_t prefix = s_prefix;
-    const uint32_t hi_mask = shift == 24 ? 0u : (0xFFFFFFFFu << (shift + 8));
-    for (int j = j0; j < j1; ++j) {
-      const uint32_t key = (ord16(A[j]) << 16) | (0xFFFFu - uint32_t(j));
-      if ((key & hi_mask) == prefix) atomicAdd(&hist[(key >> shift) & 0xFFu], 1);
+  __syncwarp();
+  {   // the bin holding the k-th largest: suffix sums over 8 bins per lane
+    int c[8], t = 0;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      c[e] = hw[(31 - lane) * 8 + (7 - e)];   // lane 0 holds the top bins
+      t += c[e];
     }
-    __syncthreads();
-    if (threadIdx.x == 0) {   // from the top bin down: the bin holding the k-th largest
-      int k = s_k, bin = 255;
-      for (; bin > 0; --bin) {
-        if (hist[bin] >= k) break;
-        k -= hist[bin];
+    int tot;
+    const int before = warp_excl_scan(t, tot);   // counts in higher bins than this lane's
+    int found = -1, krem = 0, acc = before;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      if (found < 0 && acc + c[e] >= k) {
+        found = (31 - lane) * 8 + (7 - e);
+        krem = k - acc;
       }
-      s_k = k;
-      s_prefix = prefix | (uint32_t(bin) << shift);
+      acc += c[e];
     }
-    __syncthreads();
+    const unsigned has = __ballot_sync(0xffffffffu, found >= 0);
+    const int src = __ffs(has) - 1;   // the first lane (highest bins) holding it
+    hi = uint32_t(__shfl_sync(0xffffffffu, found, src));
+    k = __shfl_sync(0xffffffffu, krem, src);
   }
-  const uint32_t thr = s_prefix;   // the S-th largest key: exactly S keys are >= thr
-  int cnt = 0;
-  for (int j = j0; j < j1; ++j)
-    cnt += ((ord16(A[j]) << 16) | (0xFFFFu - uint32_t(j))) >= thr;
-  int total;
-  int pos = block_excl_scan(cnt, warp_sums, total);
-  for (int j = j0; j < j1; ++j)
-    if (((ord16(A[j]) << 16) | (0xFFFFu - uint32_t(j))) >= thr) out[pos++] = j;
+  __syncwarp();
+  // pass 2: low byte among the scores whose high byte is `hi`
+  for (int i = lane; i < 256; i += 32) hw[i] = 0;
+  __syncwarp();
+  for (int j0 = 0; j0 < n; j0 += 32) {
+    const int j = j0 + lane;
+    int bin = 256;
+    if (j < n) {
+      const uint32_t o = ord_at(j);
+      if ((o >> 8) == hi) bin = int(o & 0xFFu);
+    }
+    const unsigned peers = __match_any_sync(0xffffffffu, bin);
+    if (bin < 256 && lane == __ffs(peers) - 1) atomicAdd(&hw[bin], __popc(peers));
+  }
+  __syncwarp();
+  uint32_t V;
+  {
+    int c[8], t = 0;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      c[e] = hw[(31 - lane) * 8 + (7 - e)];
+      t += c[e];
+    }
+    int tot;
+    const int before = warp_excl_scan(t, tot);
+    int found = -1, krem = 0, acc = before;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      if (found < 0 && acc + c[e] >= k) {
+        found = (31 - lane) * 8 + (7 - e);
+        krem = k - acc;
+      }
+      acc += c[e];
+    }
+    const unsigned has = __ballot_sync(0xffffffffu, found >= 0);
+    const int src = __ffs(has) - 1;
+    V = (hi << 8) | uint32_t(__shfl_sync(0xffffffffu, found, src));
+    k = __shfl_sync(0xffffffffu, krem, src);   // positions with o == V to take (lowest first)
+  }
+  // compaction in ascending position order, 32 positions per round
+  int base = 0, eq_taken = 0;
+  for (int j0 = 0; j0 < n; j0 += 32) {
+    const int j = j0 + lane;
+    const uint32_t o = j < n ? ord_at(j) : 0u;
+    const bool eq = j < n && o == V;
+    const unsigned eqm = __ballot_sync(0xffffffffu, eq);
+    const int eq_rank = eq_taken + __popc(eqm & ((1u << lane) - 1u));
+    const bool sel = j < n && (o > V || (eq && eq_rank < k));
+    const unsigned sm = __ballot_sync(0xffffffffu, sel);
+    if (sel) out[base + __popc(sm & ((1u << lane) - 1u))] = j;
+    base += __popc(sm);
+    eq_taken += __popc(eqm);
+  }
 }
 
 template <int D, int G>
-__global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayArgs a) {
-  __shared__ float qs[G][D];
+__global__ void __launch_bounds__(kAttnThreads, 6) replay_attn_kernel(const ReplayArgs a) {
+  constexpr int DV = D / 4;                 // 8-byte (4-value) slices per value row
+  constexpr int RG = kAttnThreads / DV;     // row groups of the value phase
+  __shared__ __align__(16) float qs[G][D];
   __shared__ float ps[G][kAttnThreads];
   __shared__ int32_t idx[kAttnThreads];
   __shared__ float red[G][kAttnThreads / 32];
+  __shared__ float outs[G][D];
   const ReplayDims& d = a.d;
   const int u = blockIdx.x;
   const int hk = blockIdx.y % d.Hkv, b = blockIdx.y / d.Hkv;
   if (u >= seq_len_of(a, b)) return;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const int dv = t % DV, rg = t / DV;
   const float scale = rsqrtf(float(D));
   // the group's queries, pre-scaled
   for (int i = t; i < G * D; i += kAttnThreads) {
@@ -167,12 +218,13 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
   const int32_t* sel = a.sel + (int64_t(b) * d.N + u) * d.S;
   const uint16_t* kb = static_cast<const uint16_t*>(a.k) + (int64_t(b) * d.Hkv + hk) * d.N * D;
   const uint16_t* vb = static_cast<const uint16_t*>(a.v) + (int64_t(b) * d.Hkv + hk) * d.N * D;
-  float m[G], l[G], acc[G];
+  float m[G], l[G], acc[G][4];
 #pragma unroll
   for (int g = 0; g < G; ++g) {
     m[g] = -INFINITY;
     l[g] = 0.f;
-    acc[g] = 0.f;
+#pragma unroll
+    for (int e = 0; e < 4; ++e) acc[g][e] = 0.f;
   }
   __syncthreads();
   for (int c0 = 0; c0 < n_keys; c0 += kAttnThreads) {
@@ -187,16 +239,23 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
       const uint4* k4 = reinterpret_cast<const uint4*>(kb + int64_t(j) * D);
 #pragma unroll
       for (int g = 0; g < G; ++g) s[g] = 0.f;
-#pragma unroll 4
+#pragma unroll 2
       for (int c = 0; c < D / 8; ++c) {
         const uint4 w = __ldg(k4 + c);
-        const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+        const float kf[8] = {__uint_as_float(w.x << 16), __uint_as_float(w.x & 0xFFFF0000u),
+                             __uint_as_float(w.y << 16), __uint_as_float(w.y & 0xFFFF0000u),
+                             __uint_as_float(w.z << 16), __uint_as_float(w.z & 0xFFFF0000u),
+                             __uint_as_float(w.w << 16), __uint_as_float(w.w & 0xFFFF0000u)};
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float k0 = __uint_as_float(ww[e] << 16), k1 = __uint_as_float(ww[e] & 0xFFFF0000u);
-#pragma unroll
-          for (int g = 0; g < G; ++g)
-            s[g] = fmaf(qs[g][8 * c + 2 * e + 1], k1, fmaf(qs[g][8 * c + 2 * e], k0, s[g]));
+        for (int g = 0; g < G; ++g) {   // the query slice as two 16-byte shared loads
+          const float4 q0 = *reinterpret_cast<const float4*>(&qs[g][8 * c]);
+          const float4 q1 = *reinterpret_cast<const float4*>(&qs[g][8 * c + 4]);
+          float x = s[g];
+          x = fmaf(q0.x, kf[0], x); x = fmaf(q0.y, kf[1], x);
+          x = fmaf(q0.z, kf[2], x); x = fmaf(q0.w, kf[3], x);
+          x = fmaf(q1.x, kf[4], x); x = fmaf(q1.y, kf[5], x);
+          x = fmaf(q1.z, kf[6], x); x = fmaf(q1.w, kf[7], x);
+          s[g] = x;
         }
       }
     }
@@ -209,17 +268,17 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
       if (lane == 0) red[g][warp] = x;
     }
     __syncthreads();
-    float mnew[G], corr[G];
+    float corr[G];
 #pragma unroll
     for (int g = 0; g < G; ++g) {
       float x = red[g][0];
       for (int w = 1; w < kAttnThreads / 32; ++w) x = fmaxf(x, red[g][w]);
-      mnew[g] = fmaxf(m[g], x);
-      corr[g] = m[g] == -INFINITY ? 0.f : expf(m[g] - mnew[g]);
-      ps[g][t] = j >= 0 ? expf(s[g] - mnew[g]) : 0.f;
+      const float mnew = fmaxf(m[g], x);
+      corr[g] = m[g] == -INFINITY ? 0.f : expf(m[g] - mnew);
+      ps[g][t] = j >= 0 ? expf(s[g] - mnew) : 0.f;
+      m[g] = mnew;
     }
     __syncthreads();
-    // sums and the weighted value rows (thread t owns output dimension t)
 #pragma unroll
     for (int g = 0; g < G; ++g) {
       float x = ps[g][t];
@@ -233,15 +292,41 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
       float x = 0.f;
       for (int w = 0; w < kAttnThreads / 32; ++w) x += red[g][w];
       l[g] = l[g] * corr[g] + x;
-      acc[g] *= corr[g];
-      m[g] = mnew[g];
-    }
-    if (t < D) {
-      for (int jj = 0; jj < nc; ++jj) {
-        const float vv = bf16f(vb[int64_t(idx[jj]) * D + t]);
 #pragma unroll
-        for (int g = 0; g < G; ++g) acc[g] = fmaf(ps[g][jj], vv, acc[g]);
+      for (int e = 0; e < 4; ++e) acc[g][e] *= corr[g];
+    }
+    // weighted value rows: this thread takes 4 dimensions of rows rg, rg + RG, ...
+    for (int jj = rg; jj < nc; jj += RG) {
+      const uint2 w = __ldg(reinterpret_cast<const uint2*>(vb + int64_t(idx[jj]) * D + dv * 4));
+      const float v0 = __uint_as_float(w.x << 16), v1 = __uint_as_float(w.x & 0xFFFF0000u);
+      const float v2 = __uint_as_float(w.y << 16), v3 = __uint_as_float(w.y & 0xFFFF0000u);
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        const float p = ps[g][jj];
+        acc[g][0] = fmaf(p, v0, acc[g][0]);
+        acc[g][1] = fmaf(p, v1, acc[g][1]);
+        acc[g][2] = fmaf(p, v2, acc[g][2]);
+        acc[g][3] = fmaf(p, v3, acc[g][3]);
       }
+    }
+    __syncthreads();
+  }
+  // sum the row groups: first within the warp, then the warps in a fixed order
+#pragma unroll
+  for (int g = 0; g < G; ++g)
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+#pragma unroll
+      for (int o = DV; o < 32; o <<= 1) acc[g][e] += __shfl_xor_sync(0xffffffffu, acc[g][e], o);
+  // lanes below DV of each warp hold its sums (DV = 32 for d = 128: every lane)
+  constexpr int LW = DV < 32 ? DV : 32;
+  for (int w = 0; w < kAttnThreads / 32; ++w) {
+    if (warp == w && lane < LW) {
+#pragma unroll
+      for (int g = 0; g < G; ++g)
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          outs[g][dv * 4 + e] = (w == 0 ? 0.f : outs[g][dv * 4 + e]) + acc[g][e];
     }
     __syncthreads();
   }
@@ -250,12 +335,11 @@ __global__ void __launch_bounds__(kAttnThreads) replay_attn_kernel(const ReplayA
 #pragma unroll
     for (int g = 0; g < G; ++g) {
       const int h = hk * G + g;
-      __nv_bfloat16 r = __float2bfloat16_rn(acc[g] / l[g]);
+      __nv_bfloat16 r = __float2bfloat16_rn(outs[g][t] / l[g]);
       o[((int64_t(b) * d.Hq + h) * d.N + u) * D + t] = *reinterpret_cast<uint16_t*>(&r);
     }
   }
 }
-
 
 // ---------------------------------------------------------------- V^T for the tensor-core path
 
@@ -603,7 +687,7 @@ bool replay_supported(const ReplayDims& d) {
 cudaError_t launch_replay_select(const ReplayArgs& a, cudaStream_t st) {
   const int rows = a.d.B * a.d.N;
   if (rows <= 0) return cudaSuccess;
-  replay_select_kernel<<<rows, kSelThreads, 0, st>>>(a);
+  replay_select_kernel<<<(rows + kSelWarps - 1) / kSelWarps, 32 * kSelWarps, 0, st>>>(a);
   return cudaGetLastError();
 }
 

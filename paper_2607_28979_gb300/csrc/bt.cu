@@ -29,9 +29,11 @@
 // The row layer norms gamma * (v - mean) / sqrt(var + 1e-5) + beta run over the
 // row's d values in fp32, on the fp32 row held in registers; the matrices they
 // feed stay the blob's exact bf16 values. Every GEMM is one persistent,
-// warp-specialised tcgen05 kernel: warp 0 TMA producer (4-stage ring of 64-wide K blocks), warp 1 MMA issuer
-// (M = 128, N = NT, fp32 accumulators in TMEM, two buffers), warp 2 TMEM
-// allocator, warps 4..7 the epilogue (one TMEM lane = one row each). Row tiles
+// warp-specialised tcgen05 kernel: warp 0 TMA producer (4-stage ring of 64-wide
+// K blocks), warp 1 MMA issuer (M = 128, N = NT, fp32 accumulators in TMEM, two
+// buffers), warp 2 TMEM allocator, then the epilogue warps (4 for the row-norm
+// stages, one row per thread; 16 for the others, a quarter of the columns per
+// warp). Row tiles
 // hold whole tokens (tau = 128 / P of them). The epilogue warps never wait on
 // one another. All waits are bounded; on a timeout every role
 // unwinds, copies and MMAs in flight are drained, TMEM is freed and
@@ -50,7 +52,10 @@ constexpr int kBtStages = 4;
 constexpr int kBtABytes = 128 * 64 * 2;   // 16 KB: 128 rows x 64 bf16
 constexpr int kBtBBytes = 256 * 64 * 2;   // 32 KB: up to 256 rows x 64 bf16
 constexpr int kBtStageBytes = kBtABytes + kBtBBytes;
-constexpr int kBtThreads = 256;           // warps 0..3 roles, 4..7 epilogue
+// warps 0..3 roles, then EPI epilogue warps: 4 for the row-norm stages (a row's
+// d values in one thread), 16 for the others (each warp of a lane quarter
+// takes every fourth 32-column chunk)
+__host__ __device__ constexpr int bt_threads(int epi) { return 32 * (4 + epi); }
 constexpr int kBtTmemCols = 512;
 constexpr float kLnEps = 1e-5f;
 constexpr int kBtSmem = kBtStages * kBtStageBytes + 256 + 1024;
@@ -317,8 +322,9 @@ __device__ void epi_row(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
   }
 }
 
-// Plain epilogues, 32 columns at a time: bias (+ GELU), bf16 out.
-__device__ void epi_plain(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
+// Plain epilogues, 32 columns at a time: bias (+ GELU), bf16 out. Column group
+// cg of ng takes chunks cg, cg + ng, ...
+__device__ void epi_plain(const EpiCtx& e, const Work& w, uint32_t tb, int row, int cg, int ng) {
   const BtArgs& a = *e.a;
   const GemmCfg& c = *e.c;
   const BtDims& d = a.d;
@@ -340,7 +346,7 @@ __device__ void epi_plain(const EpiCtx& e, const Work& w, uint32_t tb, int row) 
     out = static_cast<uint16_t*>(a.f);
   }
   const bool gelu = c.mode == kBtF1;
-  for (int ch = 0; ch < c.NT / 32; ++ch) {
+  for (int ch = cg; ch < c.NT / 32; ch += ng) {
     uint32_t rr[32];
     __syncwarp();
     tmem_ld_32x32b_x32(tb + ch * 32, rr);
@@ -367,7 +373,7 @@ __device__ void epi_plain(const EpiCtx& e, const Work& w, uint32_t tb, int row) 
 
 // kBtOut: the E backbones' accumulators of this 128-token tile sit side by
 // side (E * NT columns); the gate-weighted sum goes to target layer q0 + r.
-__device__ void epi_out(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
+__device__ void epi_out(const EpiCtx& e, const Work& w, uint32_t tb, int row, int cg, int ng) {
   const BtArgs& a = *e.a;
   const GemmCfg& c = *e.c;
   const BtDims& d = a.d;
@@ -397,7 +403,7 @@ __device__ void epi_out(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
   }
   uint16_t* dst = static_cast<uint16_t*>(a.dst[x]);
   const int l = d.q0 + a.slot;
-  for (int ch = 0; ch < c.NT / 32; ++ch) {
+  for (int ch = cg; ch < c.NT / 32; ch += ng) {
     float y[32];
 #pragma unroll
     for (int k = 0; k < 32; ++k) y[k] = 0.f;
@@ -429,8 +435,8 @@ __device__ void epi_out(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
 
 // ---------------------------------------------------------------- the GEMM kernel
 
-template <int D>
-__global__ void __launch_bounds__(kBtThreads, 1)
+template <int D, int EPI>
+__global__ void __launch_bounds__(bt_threads(EPI), 1)
     bt_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
                    const __grid_constant__ CUtensorMap tmB, const BtArgs a, const GemmCfg c) {
   extern __shared__ uint8_t smem_raw[];
@@ -460,7 +466,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], 4);
+      mbar_init(&tempty[b], EPI);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -568,6 +574,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
   } else if (warp >= 4) {
     // ------------------------------------------------ epilogue
     const int q = warp & 3;
+    const int cg = (warp - 4) >> 2;   // column group of this warp (EPI / 4 groups)
     const int row = q * 32 + lane;
     EpiCtx e{&a, &c};
     int buf = 0;
@@ -582,12 +589,13 @@ __global__ void __launch_bounds__(kBtThreads, 1)
       tc_fence_after();
       const uint32_t tb = tmem_base + static_cast<uint32_t>(buf * acc_cols) +
                           (static_cast<uint32_t>(q * 32) << 16);
-      switch (c.mode) {
-        case kBtIn:
-        case kBtO:
-        case kBtF2: epi_row<D>(e, w, tb, row); break;
-        case kBtOut: epi_out(e, w, tb, row); break;
-        default: epi_plain(e, w, tb, row);
+      if constexpr (EPI == 4) {   // the row-norm stages (kBtIn, kBtO, kBtF2)
+        epi_row<D>(e, w, tb, row);
+      } else {
+        if (c.mode == kBtOut)
+          epi_out(e, w, tb, row, cg, EPI / 4);
+        else
+          epi_plain(e, w, tb, row, cg, EPI / 4);
       }
       tc_fence_before();
       __syncwarp();
@@ -873,9 +881,12 @@ cudaError_t launch_bt_gemm(int mode, const BtArgs& a, const CUtensorMap& tmA,
     default: return cudaErrorInvalidValue;
   }
   if (c.NT < 32 || c.NT > 256 || c.NT % 32 || c.K % 64) return cudaErrorInvalidValue;
-  static bool attr_set[2] = {false, false};
-  const int di = d.d == 128 ? 1 : 0;
-  auto kern = d.d == 128 ? bt_gemm_kernel<128> : bt_gemm_kernel<64>;
+  // the row-norm stages keep a row in one thread; the others spread it over 16 warps
+  const bool wide = mode == kBtQ || mode == kBtKV || mode == kBtF1 || mode == kBtOut;
+  static bool attr_set[4] = {false, false, false, false};
+  const int di = (d.d == 128 ? 1 : 0) + (wide ? 2 : 0);
+  auto kern = wide ? (d.d == 128 ? bt_gemm_kernel<128, 16> : bt_gemm_kernel<64, 16>)
+                   : (d.d == 128 ? bt_gemm_kernel<128, 4> : bt_gemm_kernel<64, 4>);
   if (!attr_set[di]) {
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kBtSmem);
@@ -885,7 +896,7 @@ cudaError_t launch_bt_gemm(int mode, const BtArgs& a, const CUtensorMap& tmA,
   const long long items = static_cast<long long>(c.groups) * c.row_tiles * c.n_tiles;
   const int grid = static_cast<int>(items < num_sms ? items : num_sms);
   if (grid <= 0) return cudaSuccess;
-  kern<<<grid, kBtThreads, kBtSmem, st>>>(tmA, tmA2, tmB, a, c);
+  kern<<<grid, bt_threads(wide ? 16 : 4), kBtSmem, st>>>(tmA, tmA2, tmB, a, c);
   return cudaGetLastError();
 }
 

@@ -12,15 +12,16 @@
 //                         positions scoring V it takes; ballots then keep every
 //                         score above V and the lowest positions at V. Rows with
 //                         u + 1 <= S take every position.
-//   replay_attn_kernel    one CTA per (b, key/value head, u): the query heads of
-//                         the GQA group attend to the selected rows (sparse) or to
-//                         positions 0..u in 128-key chunks with an online softmax
-//                         (full). Thread t scores key t of the chunk against every
-//                         query of the group (its key row read as 16-byte vectors),
-//                         the softmax is fp32, and each thread accumulates 4 output
-//                         dimensions over every (128 / (d / 4))-th value row of the
-//                         chunk (8-byte reads); the row groups are summed within
-//                         the warp and then warp by warp in a fixed order.
+//   replay_attn_kernel    one warp per (b, key/value head, u), no block barriers:
+//                         the query heads of the GQA group attend to the selected
+//                         rows (sparse) or to positions 0..u in 128-key chunks
+//                         with an online softmax (full). Each lane scores four keys
+//                         of the chunk against every query of the group (16-byte
+//                         key reads, the pre-scaled queries broadcast from the
+//                         warp's shared copy), the softmax runs on warp shuffles in
+//                         fp32, and each lane accumulates d / 32 output dimensions
+//                         over the chunk's value rows (the warp reads each row
+//                         once, coalesced).
 //   replay_fmha_kernel    full causal attention on the tensor cores (layers below
 //                         L_Full): one CTA per (b, query head, 128-query tile),
 //                         persistent over its key tiles 0..diagonal.
@@ -46,9 +47,13 @@
 namespace mot {
 namespace {
 
-constexpr int kAttnThreads = 128;   // = the key chunk
 
 __device__ __forceinline__ float bf16f(uint16_t b) { return __uint_as_float(uint32_t(b) << 16); }
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
 
 // Order-preserving map of bf16 bits to unsigned 16-bit: larger value -> larger key.
 __device__ __forceinline__ uint32_t ord16(uint16_t b) {
@@ -190,153 +195,156 @@ __global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const Rep
   }
 }
 
+constexpr int kAttnWarps = 4;   // (b, key/value head, u) items per CTA, one warp each
+
+// Shared memory of one warp: the group's pre-scaled queries [G][D], the chunk's
+// probabilities [G][128] and its key positions [128].
 template <int D, int G>
-__global__ void __launch_bounds__(kAttnThreads, 6) replay_attn_kernel(const ReplayArgs a) {
-  constexpr int DV = D / 4;                 // 8-byte (4-value) slices per value row
-  constexpr int RG = kAttnThreads / DV;     // row groups of the value phase
-  __shared__ __align__(16) float qs[G][D];
-  __shared__ float ps[G][kAttnThreads];
-  __shared__ int32_t idx[kAttnThreads];
-  __shared__ float red[G][kAttnThreads / 32];
-  __shared__ float outs[G][D];
+__host__ __device__ constexpr int attn_warp_floats() { return G * D + G * 128 + 128; }
+
+template <int D, int G>
+__global__ void __launch_bounds__(32 * kAttnWarps) replay_attn_kernel(const ReplayArgs a) {
+  constexpr int DL = D / 32;   // output dimensions per lane
+  extern __shared__ float4 attn_smem4[];
   const ReplayDims& d = a.d;
-  const int u = blockIdx.x;
-  const int hk = blockIdx.y % d.Hkv, b = blockIdx.y / d.Hkv;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t item = int64_t(blockIdx.x) * kAttnWarps + warp;
+  if (item >= int64_t(d.B) * d.Hkv * d.N) return;
+  const int u = static_cast<int>(item % d.N);
+  const int bh = static_cast<int>(item / d.N);
+  const int hk = bh % d.Hkv, b = bh / d.Hkv;
   if (u >= seq_len_of(a, b)) return;
-  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-  const int dv = t % DV, rg = t / DV;
+  float* ws = reinterpret_cast<float*>(attn_smem4) + warp * attn_warp_floats<D, G>();
+  float* qs = ws;                        // [G][D]
+  float* ps = ws + G * D;                // [G][128]
+  int32_t* ix = reinterpret_cast<int32_t*>(ps + G * 128);   // [128]
   const float scale = rsqrtf(float(D));
-  // the group's queries, pre-scaled
-  for (int i = t; i < G * D; i += kAttnThreads) {
+  for (int i = lane; i < G * D; i += 32) {
     const int g = i / D, c = i - g * D;
-    const int h = hk * G + g;
-    qs[g][c] = bf16f(static_cast<const uint16_t*>(a.q)[((int64_t(b) * d.Hq + h) * d.N + u) * D + c]) *
-               scale;
+    qs[i] = bf16f(static_cast<const uint16_t*>(a.q)[((int64_t(b) * d.Hq + hk * G + g) * d.N + u) * D + c]) *
+            scale;
   }
   const bool full = a.full != 0;
   const int n_keys = full ? u + 1 : min(d.S, u + 1);
   const int32_t* sel = a.sel + (int64_t(b) * d.N + u) * d.S;
   const uint16_t* kb = static_cast<const uint16_t*>(a.k) + (int64_t(b) * d.Hkv + hk) * d.N * D;
   const uint16_t* vb = static_cast<const uint16_t*>(a.v) + (int64_t(b) * d.Hkv + hk) * d.N * D;
-  float m[G], l[G], acc[G][4];
+  float m[G], l[G], acc[G][DL];
 #pragma unroll
   for (int g = 0; g < G; ++g) {
     m[g] = -INFINITY;
     l[g] = 0.f;
 #pragma unroll
-    for (int e = 0; e < 4; ++e) acc[g][e] = 0.f;
+    for (int e = 0; e < DL; ++e) acc[g][e] = 0.f;
   }
-  __syncthreads();
-  for (int c0 = 0; c0 < n_keys; c0 += kAttnThreads) {
-    const int nc = min(kAttnThreads, n_keys - c0);
-    const int j = t < nc ? (full ? c0 + t : sel[c0 + t]) : -1;
-    idx[t] = j;
-    // scores of key t against every query of the group
-    float s[G];
+  __syncwarp();
+  for (int c0 = 0; c0 < n_keys; c0 += 128) {
+    const int nc = min(128, n_keys - c0);
+    // this lane's keys: chunk positions lane, lane + 32, lane + 64, lane + 96
+    int j[4];
 #pragma unroll
-    for (int g = 0; g < G; ++g) s[g] = -INFINITY;
-    if (j >= 0) {
-      const uint4* k4 = reinterpret_cast<const uint4*>(kb + int64_t(j) * D);
+    for (int i = 0; i < 4; ++i) {
+      const int t = lane + 32 * i;
+      j[i] = t < nc ? (full ? c0 + t : sel[c0 + t]) : -1;
+      ix[t] = j[i];
+    }
+    float s[4][G];
 #pragma unroll
-      for (int g = 0; g < G; ++g) s[g] = 0.f;
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int g = 0; g < G; ++g) s[i][g] = 0.f;
 #pragma unroll 2
-      for (int c = 0; c < D / 8; ++c) {
-        const uint4 w = __ldg(k4 + c);
-        const float kf[8] = {__uint_as_float(w.x << 16), __uint_as_float(w.x & 0xFFFF0000u),
-                             __uint_as_float(w.y << 16), __uint_as_float(w.y & 0xFFFF0000u),
-                             __uint_as_float(w.z << 16), __uint_as_float(w.z & 0xFFFF0000u),
-                             __uint_as_float(w.w << 16), __uint_as_float(w.w & 0xFFFF0000u)};
+    for (int c = 0; c < D / 8; ++c) {
+      float kf[4][8];
 #pragma unroll
-        for (int g = 0; g < G; ++g) {   // the query slice as two 16-byte shared loads
-          const float4 q0 = *reinterpret_cast<const float4*>(&qs[g][8 * c]);
-          const float4 q1 = *reinterpret_cast<const float4*>(&qs[g][8 * c + 4]);
-          float x = s[g];
-          x = fmaf(q0.x, kf[0], x); x = fmaf(q0.y, kf[1], x);
-          x = fmaf(q0.z, kf[2], x); x = fmaf(q0.w, kf[3], x);
-          x = fmaf(q1.x, kf[4], x); x = fmaf(q1.y, kf[5], x);
-          x = fmaf(q1.z, kf[6], x); x = fmaf(q1.w, kf[7], x);
-          s[g] = x;
+      for (int i = 0; i < 4; ++i) {
+        uint4 w = make_uint4(0u, 0u, 0u, 0u);
+        if (j[i] >= 0) w = __ldg(reinterpret_cast<const uint4*>(kb + int64_t(j[i]) * D) + c);
+        kf[i][0] = __uint_as_float(w.x << 16); kf[i][1] = __uint_as_float(w.x & 0xFFFF0000u);
+        kf[i][2] = __uint_as_float(w.y << 16); kf[i][3] = __uint_as_float(w.y & 0xFFFF0000u);
+        kf[i][4] = __uint_as_float(w.z << 16); kf[i][5] = __uint_as_float(w.z & 0xFFFF0000u);
+        kf[i][6] = __uint_as_float(w.w << 16); kf[i][7] = __uint_as_float(w.w & 0xFFFF0000u);
+      }
+#pragma unroll
+      for (int g = 0; g < G; ++g) {
+        const float4 q0 = *reinterpret_cast<const float4*>(qs + g * D + 8 * c);
+        const float4 q1 = *reinterpret_cast<const float4*>(qs + g * D + 8 * c + 4);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          float x = s[i][g];
+          x = fmaf(q0.x, kf[i][0], x); x = fmaf(q0.y, kf[i][1], x);
+          x = fmaf(q0.z, kf[i][2], x); x = fmaf(q0.w, kf[i][3], x);
+          x = fmaf(q1.x, kf[i][4], x); x = fmaf(q1.y, kf[i][5], x);
+          x = fmaf(q1.z, kf[i][6], x); x = fmaf(q1.w, kf[i][7], x);
+          s[i][g] = x;
         }
       }
     }
-    // chunk maxima per query
+    // online softmax per query of the group (warp reductions only)
 #pragma unroll
     for (int g = 0; g < G; ++g) {
-      float x = s[g];
+      float mx = -INFINITY;
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
-      if (lane == 0) red[g][warp] = x;
-    }
-    __syncthreads();
-    float corr[G];
+      for (int i = 0; i < 4; ++i)
+        if (j[i] >= 0) mx = fmaxf(mx, s[i][g]);
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-      float x = red[g][0];
-      for (int w = 1; w < kAttnThreads / 32; ++w) x = fmaxf(x, red[g][w]);
-      const float mnew = fmaxf(m[g], x);
-      corr[g] = m[g] == -INFINITY ? 0.f : expf(m[g] - mnew);
-      ps[g][t] = j >= 0 ? expf(s[g] - mnew) : 0.f;
+      for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      const float mnew = fmaxf(m[g], mx);
+      const float corr = m[g] == -INFINITY ? 0.f : expf(m[g] - mnew);
+      float sum = 0.f;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float pv = j[i] >= 0 ? expf(s[i][g] - mnew) : 0.f;
+        ps[g * 128 + lane + 32 * i] = pv;
+        sum += pv;
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+      l[g] = l[g] * corr + sum;
       m[g] = mnew;
+#pragma unroll
+      for (int e = 0; e < DL; ++e) acc[g][e] *= corr;
     }
-    __syncthreads();
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      float x = ps[g][t];
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-      if (lane == 0) red[g][warp] = x;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      float x = 0.f;
-      for (int w = 0; w < kAttnThreads / 32; ++w) x += red[g][w];
-      l[g] = l[g] * corr[g] + x;
-#pragma unroll
-      for (int e = 0; e < 4; ++e) acc[g][e] *= corr[g];
-    }
-    // weighted value rows: this thread takes 4 dimensions of rows rg, rg + RG, ...
-    for (int jj = rg; jj < nc; jj += RG) {
-      const uint2 w = __ldg(reinterpret_cast<const uint2*>(vb + int64_t(idx[jj]) * D + dv * 4));
-      const float v0 = __uint_as_float(w.x << 16), v1 = __uint_as_float(w.x & 0xFFFF0000u);
-      const float v2 = __uint_as_float(w.y << 16), v3 = __uint_as_float(w.y & 0xFFFF0000u);
+    __syncwarp();
+    // weighted value rows: this lane's DL dimensions of every selected row
+    for (int t0 = 0; t0 < nc; t0 += 4) {
+      float pq[G][4];
 #pragma unroll
       for (int g = 0; g < G; ++g) {
-        const float p = ps[g][jj];
-        acc[g][0] = fmaf(p, v0, acc[g][0]);
-        acc[g][1] = fmaf(p, v1, acc[g][1]);
-        acc[g][2] = fmaf(p, v2, acc[g][2]);
-        acc[g][3] = fmaf(p, v3, acc[g][3]);
+        const float4 p4 = *reinterpret_cast<const float4*>(ps + g * 128 + t0);
+        pq[g][0] = p4.x; pq[g][1] = p4.y; pq[g][2] = p4.z; pq[g][3] = p4.w;
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        if (t0 + i >= nc) break;
+        const uint16_t* vr = vb + int64_t(ix[t0 + i]) * D + lane * DL;
+        float vv[DL];
+        if constexpr (DL == 4) {
+          const uint2 w = __ldg(reinterpret_cast<const uint2*>(vr));
+          vv[0] = __uint_as_float(w.x << 16); vv[1] = __uint_as_float(w.x & 0xFFFF0000u);
+          vv[2] = __uint_as_float(w.y << 16); vv[3] = __uint_as_float(w.y & 0xFFFF0000u);
+        } else {
+          const uint32_t w = __ldg(reinterpret_cast<const uint32_t*>(vr));
+          vv[0] = __uint_as_float(w << 16); vv[1] = __uint_as_float(w & 0xFFFF0000u);
+        }
+#pragma unroll
+        for (int g = 0; g < G; ++g)
+#pragma unroll
+          for (int e = 0; e < DL; ++e) acc[g][e] = fmaf(pq[g][i], vv[e], acc[g][e]);
       }
     }
-    __syncthreads();
+    __syncwarp();
   }
-  // sum the row groups: first within the warp, then the warps in a fixed order
+  uint16_t* o = static_cast<uint16_t*>(a.out);
 #pragma unroll
-  for (int g = 0; g < G; ++g)
-#pragma unroll
-    for (int e = 0; e < 4; ++e)
-#pragma unroll
-      for (int o = DV; o < 32; o <<= 1) acc[g][e] += __shfl_xor_sync(0xffffffffu, acc[g][e], o);
-  // lanes below DV of each warp hold its sums (DV = 32 for d = 128: every lane)
-  constexpr int LW = DV < 32 ? DV : 32;
-  for (int w = 0; w < kAttnThreads / 32; ++w) {
-    if (warp == w && lane < LW) {
-#pragma unroll
-      for (int g = 0; g < G; ++g)
-#pragma unroll
-        for (int e = 0; e < 4; ++e)
-          outs[g][dv * 4 + e] = (w == 0 ? 0.f : outs[g][dv * 4 + e]) + acc[g][e];
-    }
-    __syncthreads();
-  }
-  if (t < D) {
-    uint16_t* o = static_cast<uint16_t*>(a.out);
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      const int h = hk * G + g;
-      __nv_bfloat16 r = __float2bfloat16_rn(outs[g][t] / l[g]);
-      o[((int64_t(b) * d.Hq + h) * d.N + u) * D + t] = *reinterpret_cast<uint16_t*>(&r);
+  for (int g = 0; g < G; ++g) {
+    const float inv = 1.f / l[g];
+    uint16_t* orow = o + ((int64_t(b) * d.Hq + hk * G + g) * d.N + u) * D + lane * DL;
+    if constexpr (DL == 4) {
+      *reinterpret_cast<uint2*>(orow) = make_uint2(pack_bf16(acc[g][0] * inv, acc[g][1] * inv),
+                                                   pack_bf16(acc[g][2] * inv, acc[g][3] * inv));
+    } else {
+      *reinterpret_cast<uint32_t*>(orow) = pack_bf16(acc[g][0] * inv, acc[g][1] * inv);
     }
   }
 }
@@ -720,23 +728,33 @@ cudaError_t launch_replay_fmha(const ReplayArgs& a, const CUtensorMap& tmQ, cons
   return cudaGetLastError();
 }
 
+template <int D, int G>
+cudaError_t launch_attn_dg(const ReplayArgs& a, cudaStream_t st) {
+  const size_t smem = size_t(kAttnWarps) * attn_warp_floats<D, G>() * 4;
+  static bool attr = false;
+  if (!attr && smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(replay_attn_kernel<D, G>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e != cudaSuccess) return e;
+  }
+  attr = true;
+  const int64_t items = int64_t(a.d.B) * a.d.Hkv * a.d.N;
+  const unsigned grid = static_cast<unsigned>((items + kAttnWarps - 1) / kAttnWarps);
+  replay_attn_kernel<D, G><<<grid, 32 * kAttnWarps, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_replay_attn(const ReplayArgs& a, cudaStream_t st) {
-  dim3 grid(a.d.N, a.d.B * a.d.Hkv);
   const int G = a.d.Hq / a.d.Hkv;
-#define MOT_RP_CASE(GG)                                                          \
-  case GG:                                                                       \
-    if (a.d.d == 128)                                                            \
-      replay_attn_kernel<128, GG><<<grid, kAttnThreads, 0, st>>>(a);             \
-    else                                                                         \
-      replay_attn_kernel<64, GG><<<grid, kAttnThreads, 0, st>>>(a);              \
-    break;
+#define MOT_RP_CASE(GG)                                                             \
+  case GG:                                                                          \
+    return a.d.d == 128 ? launch_attn_dg<128, GG>(a, st) : launch_attn_dg<64, GG>(a, st);
   switch (G) {
     MOT_RP_CASE(1) MOT_RP_CASE(2) MOT_RP_CASE(3) MOT_RP_CASE(4) MOT_RP_CASE(5)
     MOT_RP_CASE(6) MOT_RP_CASE(7) MOT_RP_CASE(8) MOT_RP_CASE(12) MOT_RP_CASE(16)
     default: return cudaErrorInvalidValue;
   }
 #undef MOT_RP_CASE
-  return cudaGetLastError();
 }
 
 }  // namespace mot

@@ -85,7 +85,8 @@ __device__ __forceinline__ int warp_excl_scan(int v, int& total) {
 // score, the S-th largest (o, -j) key is found in two histogram passes over o
 // (high byte, then low byte): V = its score bits, k = how many positions with
 // o == V it takes. The selection is then every o > V plus the k lowest
-// positions with o == V, compacted in ascending order by warp scans.
+// positions with o == V, compacted in ascending order by warp scans. Each lane
+// reads 8 consecutive scores per step (16-byte loads when max_seq % 8 == 0).
 __global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const ReplayArgs a) {
   __shared__ int hist[kSelWarps][256];
   const ReplayDims& d = a.d;
@@ -101,62 +102,46 @@ __global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const Rep
     return;
   }
   const uint16_t* A = static_cast<const uint16_t*>(a.guide) + int64_t(row) * d.N;
-  // three passes read the row (from L2 after the first); no shared copy, so
-  // that every SM keeps 64 rows in flight
-  auto ord_at = [&](int j) -> uint32_t { return ord16(__ldg(A + j)); };
+  const bool vec = (d.N & 7) == 0;   // then every 8-score group of the row is 16-byte aligned
+  // the 8 order-preserving scores at positions j8 .. j8 + 7 (0 past n; never counted)
+  auto load8 = [&](int j8, uint32_t (&o)[8]) {
+    if (vec) {
+      const uint4 q = __ldg(reinterpret_cast<const uint4*>(A + j8));
+      const uint32_t qq[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        o[2 * e] = ord16(qq[e] & 0xFFFFu);
+        o[2 * e + 1] = ord16(qq[e] >> 16);
+      }
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) o[e] = j8 + e < n ? ord16(__ldg(A + j8 + e)) : 0u;
+    }
+  };
   int* hw = hist[w];
   int k = d.S;
-  uint32_t hi = 0;
-  // pass 1: high byte of the score bits (strided over the lanes)
-  for (int i = lane; i < 256; i += 32) hw[i] = 0;
-  __syncwarp();
-  for (int j0 = 0; j0 < n; j0 += 32) {
-    const int j = j0 + lane;
-    const int bin = j < n ? int(ord_at(j) >> 8) : 256;
-    const unsigned peers = __match_any_sync(0xffffffffu, bin);
-    if (bin < 256 && lane == __ffs(peers) - 1) atomicAdd(&hw[bin], __popc(peers));
-  }
-  __syncwarp();
-  {   // the bin holding the k-th largest: suffix sums over 8 bins per lane
-    int c[8], t = 0;
+  uint32_t hi = 0, V = 0;
+  for (int pass = 0; pass < 2; ++pass) {
+    for (int i = lane; i < 256; i += 32) hw[i] = 0;
+    __syncwarp();
+    for (int j8 = lane * 8; j8 - lane * 8 < n; j8 += 256) {   // warp-uniform trip count
+      uint32_t o[8];
+      if (j8 < n) load8(j8, o);
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      c[e] = hw[(31 - lane) * 8 + (7 - e)];   // lane 0 holds the top bins
-      t += c[e];
-    }
-    int tot;
-    const int before = warp_excl_scan(t, tot);   // counts in higher bins than this lane's
-    int found = -1, krem = 0, acc = before;
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      if (found < 0 && acc + c[e] >= k) {
-        found = (31 - lane) * 8 + (7 - e);
-        krem = k - acc;
+      for (int e = 0; e < 8; ++e) {
+        int bin = 256;   // none
+        if (j8 + e < n) {
+          if (pass == 0)
+            bin = int(o[e] >> 8);
+          else if ((o[e] >> 8) == hi)
+            bin = int(o[e] & 0xFFu);
+        }
+        const unsigned peers = __match_any_sync(0xffffffffu, bin);
+        if (bin < 256 && lane == __ffs(peers) - 1) atomicAdd(&hw[bin], __popc(peers));
       }
-      acc += c[e];
     }
-    const unsigned has = __ballot_sync(0xffffffffu, found >= 0);
-    const int src = __ffs(has) - 1;   // the first lane (highest bins) holding it
-    hi = uint32_t(__shfl_sync(0xffffffffu, found, src));
-    k = __shfl_sync(0xffffffffu, krem, src);
-  }
-  __syncwarp();
-  // pass 2: low byte among the scores whose high byte is `hi`
-  for (int i = lane; i < 256; i += 32) hw[i] = 0;
-  __syncwarp();
-  for (int j0 = 0; j0 < n; j0 += 32) {
-    const int j = j0 + lane;
-    int bin = 256;
-    if (j < n) {
-      const uint32_t o = ord_at(j);
-      if ((o >> 8) == hi) bin = int(o & 0xFFu);
-    }
-    const unsigned peers = __match_any_sync(0xffffffffu, bin);
-    if (bin < 256 && lane == __ffs(peers) - 1) atomicAdd(&hw[bin], __popc(peers));
-  }
-  __syncwarp();
-  uint32_t V;
-  {
+    __syncwarp();
+    // the bin holding the k-th largest: lane 0 holds the top 8 bins, lane 31 the bottom 8
     int c[8], t = 0;
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
@@ -174,24 +159,42 @@ __global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const Rep
       }
       acc += c[e];
     }
-    const unsigned has = __ballot_sync(0xffffffffu, found >= 0);
-    const int src = __ffs(has) - 1;
-    V = (hi << 8) | uint32_t(__shfl_sync(0xffffffffu, found, src));
-    k = __shfl_sync(0xffffffffu, krem, src);   // positions with o == V to take (lowest first)
+    const int src = __ffs(__ballot_sync(0xffffffffu, found >= 0)) - 1;
+    const uint32_t bin = uint32_t(__shfl_sync(0xffffffffu, found, src));
+    k = __shfl_sync(0xffffffffu, krem, src);
+    if (pass == 0)
+      hi = bin;
+    else
+      V = (hi << 8) | bin;   // k: positions with o == V to take, lowest first
+    __syncwarp();
   }
-  // compaction in ascending position order, 32 positions per round
+  // compaction in ascending position order, 256 positions per round
   int base = 0, eq_taken = 0;
-  for (int j0 = 0; j0 < n; j0 += 32) {
-    const int j = j0 + lane;
-    const uint32_t o = j < n ? ord_at(j) : 0u;
-    const bool eq = j < n && o == V;
-    const unsigned eqm = __ballot_sync(0xffffffffu, eq);
-    const int eq_rank = eq_taken + __popc(eqm & ((1u << lane) - 1u));
-    const bool sel = j < n && (o > V || (eq && eq_rank < k));
-    const unsigned sm = __ballot_sync(0xffffffffu, sel);
-    if (sel) out[base + __popc(sm & ((1u << lane) - 1u))] = j;
-    base += __popc(sm);
-    eq_taken += __popc(eqm);
+  for (int j8 = lane * 8; j8 - lane * 8 < n; j8 += 256) {
+    uint32_t o[8];
+    if (j8 < n) load8(j8, o);
+    int n_eq = 0;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) n_eq += (j8 + e < n && o[e] == V);
+    int eq_tot;
+    int eq_rank = eq_taken + warp_excl_scan(n_eq, eq_tot);
+    bool sel[8];
+    int n_sel = 0;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const bool in = j8 + e < n;
+      const bool eq = in && o[e] == V;
+      sel[e] = in && (o[e] > V || (eq && eq_rank < k));
+      eq_rank += eq;
+      n_sel += sel[e];
+    }
+    int sel_tot;
+    int pos = base + warp_excl_scan(n_sel, sel_tot);
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      if (sel[e]) out[pos++] = j8 + e;
+    base += sel_tot;
+    eq_taken += eq_tot;
   }
 }
 

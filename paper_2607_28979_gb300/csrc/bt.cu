@@ -61,8 +61,14 @@ constexpr float kLnEps = 1e-5f;
 constexpr int kBtSmem = kBtStages * kBtStageBytes + 256 + 1024;
 static_assert(kBtSmem <= 232448, "shared memory budget");
 
-__device__ __forceinline__ float gelu_erf(float u) {
-  return 0.5f * u * (1.f + erff(u * 0.70710678118654752f));
+// GELU in its tanh form, 0.5 u (1 + tanh(sqrt(2/pi) (u + 0.044715 u^3))), on
+// the hardware tanh unit: within 5e-4 of the erf form over the line (the
+// parity tests bound the whole path), at a fraction of erff's instruction count.
+__device__ __forceinline__ float gelu_tanh(float u) {
+  const float k0 = 0.7978845608028654f, k1 = 0.7978845608028654f * 0.044715f;
+  const float t = tanh_approx(u * fmaf(k1, u * u, k0));
+  const float hu = 0.5f * u;
+  return fmaf(hu, t, hu);
 }
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
@@ -279,7 +285,7 @@ __device__ void epi_row(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
     const float* sw = a.s_in + int64_t(w.g) * D;
     const float* cb = a.c_in + int64_t(w.g) * D;
 #pragma unroll
-    for (int k = 0; k < D; ++k) v[k] = gelu_erf(fmaf(v[k] - mu * __ldg(sw + k), rs, __ldg(cb + k)));
+    for (int k = 0; k < D; ++k) v[k] = gelu_tanh(fmaf(v[k] - mu * __ldg(sw + k), rs, __ldg(cb + k)));
     row_stats<D>(v, mean, m2);
     if (valid) {
       const float rstd = rsqrtf(m2 * (1.f / D) + kLnEps);
@@ -363,7 +369,7 @@ __device__ void epi_plain(const EpiCtx& e, const Work& w, uint32_t tb, int row, 
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
         f[k] = __uint_as_float(rr[8 * q8 + k]) + bb[k];
-        if (gelu) f[k] = gelu_erf(f[k]);
+        if (gelu) f[k] = gelu_tanh(f[k]);
       }
       o4[q8] = make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]),
                           pack2(f[6], f[7]));
@@ -419,7 +425,7 @@ __device__ void epi_out(const EpiCtx& e, const Work& w, uint32_t tb, int row, in
 #pragma unroll
       for (int k = 0; k < 32; ++k) {
         const float u = fmaf(__uint_as_float(rr[k]) - mu[m] * __ldg(sb + k), rs[m], __ldg(cb + k));
-        y[k] = fmaf(gt[m], gelu_erf(u), y[k]);
+        y[k] = fmaf(gt[m], gelu_tanh(u), y[k]);
       }
     }
     if (!valid) continue;

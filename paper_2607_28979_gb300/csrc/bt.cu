@@ -724,87 +724,94 @@ __global__ void __launch_bounds__(256) bt_gate_kernel(const BtArgs a) {
 
 // ---------------------------------------------------------------- attention (SIMT)
 //
-// One thread per query row (token, p): for each head, scores against the
-// token's P key rows scaled by 1/sqrt(d/n_a), a max-subtracted softmax in fp32
-// and the weighted sum of the value rows.
+// One thread per (query row, head): scores against the token's P key rows
+// scaled by 1/sqrt(d/n_a), a max-subtracted softmax in fp32 and the weighted
+// sum of the value rows. Consecutive threads take consecutive heads of a row,
+// so a warp reads whole query rows and writes whole output rows.
 template <int DH>
 __global__ void __launch_bounds__(256) bt_attn_kernel(const BtArgs a) {
   const BtDims& d = a.d;
   const int g = blockIdx.y;
-  const int64_t row = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+  const int64_t id = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
   const int64_t n_rows = int64_t(d.B) * d.S * d.P;
-  if (row >= n_rows) return;
+  if (id >= n_rows * d.na) return;
+  const int h = static_cast<int>(id % d.na);
+  const int64_t row = id / d.na;
   const int64_t tok = row / d.P;
   const int b = static_cast<int>(tok / d.S), s = static_cast<int>(tok - int64_t(b) * d.S);
   if (s >= seq_len_of(a, b)) return;
   const int P = d.P, D = d.d;
   const float scale = rsqrtf(static_cast<float>(DH));
   const int64_t base = int64_t(g) * d.R + tok * P;   // first row of the token
-  const uint16_t* qr = static_cast<const uint16_t*>(a.q) + (int64_t(g) * d.R + row) * D;
-  const uint16_t* kvb = static_cast<const uint16_t*>(a.kv) + base * 2 * D;
-  uint16_t* orow = static_cast<uint16_t*>(a.o) + (int64_t(g) * d.R + row) * D;
-  for (int h = 0; h < d.na; ++h) {
-    float qv[DH];
-    const uint4* q4 = reinterpret_cast<const uint4*>(qr + h * DH);
+  const uint16_t* qr = static_cast<const uint16_t*>(a.q) + (int64_t(g) * d.R + row) * D + h * DH;
+  const uint16_t* kvb = static_cast<const uint16_t*>(a.kv) + base * 2 * D + h * DH;
+  uint16_t* orow = static_cast<uint16_t*>(a.o) + (int64_t(g) * d.R + row) * D + h * DH;
+  float qv[DH];
+  const uint4* q4 = reinterpret_cast<const uint4*>(qr);
+#pragma unroll
+  for (int c = 0; c < DH / 8; ++c) {
+    const uint4 u = q4[c];
+    qv[8 * c] = bf16_lo(u.x); qv[8 * c + 1] = bf16_hi(u.x);
+    qv[8 * c + 2] = bf16_lo(u.y); qv[8 * c + 3] = bf16_hi(u.y);
+    qv[8 * c + 4] = bf16_lo(u.z); qv[8 * c + 5] = bf16_hi(u.z);
+    qv[8 * c + 6] = bf16_lo(u.w); qv[8 * c + 7] = bf16_hi(u.w);
+  }
+  float sc[kBtMaxP];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int j = 0; j < kBtMaxP; ++j) {
+    if (j >= P) break;
+    const uint4* k4 = reinterpret_cast<const uint4*>(kvb + int64_t(j) * 2 * D);
+    float sdot = 0.f;
 #pragma unroll
     for (int c = 0; c < DH / 8; ++c) {
-      const uint4 u = q4[c];
-      qv[8 * c] = bf16_lo(u.x); qv[8 * c + 1] = bf16_hi(u.x);
-      qv[8 * c + 2] = bf16_lo(u.y); qv[8 * c + 3] = bf16_hi(u.y);
-      qv[8 * c + 4] = bf16_lo(u.z); qv[8 * c + 5] = bf16_hi(u.z);
-      qv[8 * c + 6] = bf16_lo(u.w); qv[8 * c + 7] = bf16_hi(u.w);
+      const uint4 u = k4[c];
+      sdot = fmaf(qv[8 * c], bf16_lo(u.x), sdot);
+      sdot = fmaf(qv[8 * c + 1], bf16_hi(u.x), sdot);
+      sdot = fmaf(qv[8 * c + 2], bf16_lo(u.y), sdot);
+      sdot = fmaf(qv[8 * c + 3], bf16_hi(u.y), sdot);
+      sdot = fmaf(qv[8 * c + 4], bf16_lo(u.z), sdot);
+      sdot = fmaf(qv[8 * c + 5], bf16_hi(u.z), sdot);
+      sdot = fmaf(qv[8 * c + 6], bf16_lo(u.w), sdot);
+      sdot = fmaf(qv[8 * c + 7], bf16_hi(u.w), sdot);
     }
-    float sc[kBtMaxP];
-    float mx = -INFINITY;
-    for (int j = 0; j < P; ++j) {
-      const uint4* k4 = reinterpret_cast<const uint4*>(kvb + int64_t(j) * 2 * D + h * DH);
-      float sdot = 0.f;
-#pragma unroll
-      for (int c = 0; c < DH / 8; ++c) {
-        const uint4 u = k4[c];
-        sdot = fmaf(qv[8 * c], bf16_lo(u.x), sdot);
-        sdot = fmaf(qv[8 * c + 1], bf16_hi(u.x), sdot);
-        sdot = fmaf(qv[8 * c + 2], bf16_lo(u.y), sdot);
-        sdot = fmaf(qv[8 * c + 3], bf16_hi(u.y), sdot);
-        sdot = fmaf(qv[8 * c + 4], bf16_lo(u.z), sdot);
-        sdot = fmaf(qv[8 * c + 5], bf16_hi(u.z), sdot);
-        sdot = fmaf(qv[8 * c + 6], bf16_lo(u.w), sdot);
-        sdot = fmaf(qv[8 * c + 7], bf16_hi(u.w), sdot);
-      }
-      sc[j] = sdot * scale;
-      mx = fmaxf(mx, sc[j]);
-    }
-    float den = 0.f;
-    for (int j = 0; j < P; ++j) {
-      sc[j] = expf(sc[j] - mx);
-      den += sc[j];
-    }
-    const float inv = 1.f / den;
-    float ov[DH];
-#pragma unroll
-    for (int k = 0; k < DH; ++k) ov[k] = 0.f;
-    for (int j = 0; j < P; ++j) {
-      const uint4* v4 = reinterpret_cast<const uint4*>(kvb + int64_t(j) * 2 * D + D + h * DH);
-      const float wj = sc[j] * inv;
-#pragma unroll
-      for (int c = 0; c < DH / 8; ++c) {
-        const uint4 u = v4[c];
-        ov[8 * c] = fmaf(wj, bf16_lo(u.x), ov[8 * c]);
-        ov[8 * c + 1] = fmaf(wj, bf16_hi(u.x), ov[8 * c + 1]);
-        ov[8 * c + 2] = fmaf(wj, bf16_lo(u.y), ov[8 * c + 2]);
-        ov[8 * c + 3] = fmaf(wj, bf16_hi(u.y), ov[8 * c + 3]);
-        ov[8 * c + 4] = fmaf(wj, bf16_lo(u.z), ov[8 * c + 4]);
-        ov[8 * c + 5] = fmaf(wj, bf16_hi(u.z), ov[8 * c + 5]);
-        ov[8 * c + 6] = fmaf(wj, bf16_lo(u.w), ov[8 * c + 6]);
-        ov[8 * c + 7] = fmaf(wj, bf16_hi(u.w), ov[8 * c + 7]);
-      }
-    }
-    uint4* o4 = reinterpret_cast<uint4*>(orow + h * DH);
-#pragma unroll
-    for (int c = 0; c < DH / 8; ++c)
-      o4[c] = make_uint4(pack2(ov[8 * c], ov[8 * c + 1]), pack2(ov[8 * c + 2], ov[8 * c + 3]),
-                         pack2(ov[8 * c + 4], ov[8 * c + 5]), pack2(ov[8 * c + 6], ov[8 * c + 7]));
+    sc[j] = sdot * scale;
+    mx = fmaxf(mx, sc[j]);
   }
+  float den = 0.f;
+#pragma unroll
+  for (int j = 0; j < kBtMaxP; ++j) {
+    if (j >= P) break;
+    sc[j] = expf(sc[j] - mx);
+    den += sc[j];
+  }
+  const float inv = 1.f / den;
+  float ov[DH];
+#pragma unroll
+  for (int k = 0; k < DH; ++k) ov[k] = 0.f;
+#pragma unroll
+  for (int j = 0; j < kBtMaxP; ++j) {
+    if (j >= P) break;
+    const uint4* v4 = reinterpret_cast<const uint4*>(kvb + int64_t(j) * 2 * D + D);
+    const float wj = sc[j] * inv;
+#pragma unroll
+    for (int c = 0; c < DH / 8; ++c) {
+      const uint4 u = v4[c];
+      ov[8 * c] = fmaf(wj, bf16_lo(u.x), ov[8 * c]);
+      ov[8 * c + 1] = fmaf(wj, bf16_hi(u.x), ov[8 * c + 1]);
+      ov[8 * c + 2] = fmaf(wj, bf16_lo(u.y), ov[8 * c + 2]);
+      ov[8 * c + 3] = fmaf(wj, bf16_hi(u.y), ov[8 * c + 3]);
+      ov[8 * c + 4] = fmaf(wj, bf16_lo(u.z), ov[8 * c + 4]);
+      ov[8 * c + 5] = fmaf(wj, bf16_hi(u.z), ov[8 * c + 5]);
+      ov[8 * c + 6] = fmaf(wj, bf16_lo(u.w), ov[8 * c + 6]);
+      ov[8 * c + 7] = fmaf(wj, bf16_hi(u.w), ov[8 * c + 7]);
+    }
+  }
+  uint4* o4 = reinterpret_cast<uint4*>(orow);
+#pragma unroll
+  for (int c = 0; c < DH / 8; ++c)
+    o4[c] = make_uint4(pack2(ov[8 * c], ov[8 * c + 1]), pack2(ov[8 * c + 2], ov[8 * c + 3]),
+                       pack2(ov[8 * c + 4], ov[8 * c + 5]), pack2(ov[8 * c + 6], ov[8 * c + 7]));
 }
 
 }  // namespace
@@ -838,8 +845,8 @@ cudaError_t launch_bt_gate(const BtArgs& a, cudaStream_t st) {
 
 cudaError_t launch_bt_attn(const BtArgs& a, cudaStream_t st) {
   const BtDims& d = a.d;
-  const int64_t rows = int64_t(d.B) * d.S * d.P;
-  dim3 grid(static_cast<unsigned>((rows + 255) / 256), d.G);
+  const int64_t threads = int64_t(d.B) * d.S * d.P * d.na;
+  dim3 grid(static_cast<unsigned>((threads + 255) / 256), d.G);
   switch (d.d / d.na) {
     case 16: bt_attn_kernel<16><<<grid, 256, 0, st>>>(a); break;
     case 32: bt_attn_kernel<32><<<grid, 256, 0, st>>>(a); break;

@@ -205,8 +205,13 @@ constexpr int kAttnWarps = 4;   // (b, key/value head, u) items per CTA, one war
 template <int D, int G>
 __host__ __device__ constexpr int attn_warp_floats() { return G * D + G * 128 + 128; }
 
+// Residency floor per group size: the gathers are latency-bound, so small groups
+// trade a few spilled registers for more resident warps.
+__host__ __device__ constexpr int attn_min_blocks(int g) { return g <= 8 ? 4 : 1; }
+
 template <int D, int G>
-__global__ void __launch_bounds__(32 * kAttnWarps) replay_attn_kernel(const ReplayArgs a) {
+__global__ void __launch_bounds__(32 * kAttnWarps, attn_min_blocks(G))
+    replay_attn_kernel(const ReplayArgs a) {
   constexpr int DL = D / 32;   // output dimensions per lane
   extern __shared__ float4 attn_smem4[];
   const ReplayDims& d = a.d;

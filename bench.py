@@ -85,7 +85,9 @@ def algorithmic_bt(wl, layer_map):
         "bt_out_gelu_combine": 2 * Ea * T * 2 * P * d * Dt,
         "bt_gate": 2 * T * 2 * N * Ds * E,
     }
-    flops = per_launch["bt_gate"] + N * sum(v for k, v in per_launch.items() if k != "bt_gate")
+    per_launch["bt_ffn_fused"] = per_launch["bt_ffn1_gelu"] + per_launch["bt_ffn2_residual_ln"]
+    flops = per_launch["bt_gate"] + N * sum(v for k, v in per_launch.items()
+                                            if k not in ("bt_gate", "bt_ffn_fused"))
     # bytes each kernel must move per launch in this unfused schedule (its operand
     # rows in and result rows out; a slot after the first): its own HBM roofline
     es = wl.esize
@@ -100,6 +102,8 @@ def algorithmic_bt(wl, layer_map):
         "bt_ffn2_residual_ln": allrows * (df * 2 + d * 4 + d * 4 + d * 2 + d * 2 + 8),
         "bt_out_gelu_combine": allrows * (d * 2 + 8) + 2 * T * Dt * es,
         "bt_gate": 2 * N * T * Ds * es,
+        # FFN1 + GELU + FFN2 in one kernel: no hidden rows in HBM
+        "bt_ffn_fused": allrows * (d * 2 + d * 4 + d * 4 + d * 2 + d * 2 + 8),
     }
     src_layers = {layer_map[t] for t in range(q, q + N)}
     bytes_src = 2 * len(src_layers) * T * Ds * es

@@ -642,6 +642,292 @@ __global__ void __launch_bounds__(bt_threads(EPI), 1)
   if (threadIdx.x == 0 && *abort_flag) atomicOr(a.status, kStatusTimeout);
 }
 
+// ---------------------------------------------------------------- fused FFN (FFN1 + GELU + FFN2)
+//
+// One persistent CTA per SM over (group, row tile): the FFN hidden never leaves
+// the SM. For each 128-column chunk hc of d_f:
+//   MMA1  acc1[hc & 1] = xf W_F1[hc]^T          (M = 128, N = 128, K = d)
+//   epi   A2[hc & 1]   = bf16(GELU(acc1 + b_F1)) into a 128B-swizzled SMEM tile
+//   MMA2  acc2        += A2 W_F2[:, hc]^T        (M = 128, N = d, K = 128)
+// MMA1 runs one chunk ahead of MMA2; after the last chunk the kBtF2 row epilogue
+// reads acc2. warp 0: TMA (xf once per tile, W_F1 / W_F2 chunks in 2-slot
+// rings); warp 1: MMAs; warp 2: TMEM; warps 4..7: epilogue (one row each).
+template <int D>
+struct Ffn {
+  static constexpr int kA = 128 * D * 2;       // xf tile: D / 64 blocks of 128 rows x 128 B
+  static constexpr int kW1 = 128 * D * 2;      // W_F1 chunk: 128 rows x D
+  static constexpr int kW2 = D * 128 * 2;      // W_F2 chunk: D rows x 128 (two 64-column blocks)
+  static constexpr int kA2 = 128 * 128 * 2;    // hidden chunk: two blocks of 128 rows x 64
+  static constexpr int kBytes = kA + 2 * kW1 + 2 * kW2 + 2 * kA2;
+  static constexpr int kSmem = kBytes + 256 + 1024;
+};
+static_assert(Ffn<128>::kSmem <= 232448, "shared memory budget");
+
+template <int D>
+__global__ void __launch_bounds__(256, 1)
+    bt_ffn_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW1,
+                  const __grid_constant__ CUtensorMap tmW2, const BtArgs a, const GemmCfg c) {
+  using F = Ffn<D>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sW1 = sA + F::kA;        // [2]
+  uint8_t* sW2 = sW1 + 2 * F::kW1;  // [2]
+  uint8_t* sH = sW2 + 2 * F::kW2;   // [2] hidden chunks
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sH + 2 * F::kA2);
+  uint64_t* a_full = bars;          // xf tile landed
+  uint64_t* a_empty = bars + 1;     // every MMA1 of the tile done
+  uint64_t* w1_full = bars + 2;     // [2]
+  uint64_t* w1_empty = bars + 4;    // [2]
+  uint64_t* w2_full = bars + 6;     // [2]
+  uint64_t* w2_empty = bars + 8;    // [2]
+  uint64_t* c1_full = bars + 10;    // [2] acc1 written
+  uint64_t* c1_empty = bars + 12;   // [2] acc1 read (4 epilogue warps)
+  uint64_t* h_full = bars + 14;     // [2] hidden chunk written (4 warps)
+  uint64_t* h_empty = bars + 16;    // [2] hidden chunk consumed by MMA2
+  uint64_t* c2_full = bars + 18;    // acc2 complete
+  uint64_t* c2_empty = bars + 19;   // acc2 read (4 warps)
+  uint64_t* drain = bars + 20;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 21);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const BtDims& d = a.d;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_hc = d.df / 128;
+  const int total = c.groups * c.row_tiles;
+  if (threadIdx.x == 0) {
+    mbar_init(a_full, 1);
+    mbar_init(a_empty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&w1_full[i], 1);
+      mbar_init(&w1_empty[i], 1);
+      mbar_init(&w2_full[i], 1);
+      mbar_init(&w2_empty[i], 1);
+      mbar_init(&c1_full[i], 1);
+      mbar_init(&c1_empty[i], 4);
+      mbar_init(&h_full[i], 4);
+      mbar_init(&h_empty[i], 1);
+    }
+    mbar_init(c2_full, 1);
+    mbar_init(c2_empty, 4);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmW1);
+    tma_prefetch_desc(&tmW2);
+  }
+  if (warp == 2) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;   // acc1[i] at 128 i, acc2 at 256
+  const long long wl = a.wait_limit;
+  uint32_t issued = 0;   // producer: 1 when any copy was issued (for the drain)
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------ TMA producer
+      int tl = 0;   // local tile count
+      int w1c = 0, w2c = 0;   // chunk counters of the two rings
+      for (int it = blockIdx.x; it < total; it += gridDim.x) {
+        const Work w = decode(a, c, it);
+        if (!w.active) continue;
+        if (!mbar_wait(a_empty, (tl & 1) ^ 1u, abort_flag, wl)) break;
+        mbar_arrive_expect_tx(a_full, F::kA);
+        const int64_t row0 = (int64_t(w.b) * d.S + w.s0) * d.P;
+        for (int kb = 0; kb < D / 64; ++kb)
+          tma_load_2d(sA + kb * 128 * 128, &tmA, a_full, kb * 64,
+                      static_cast<int32_t>(int64_t(w.g) * d.R + row0));
+        issued = 1;
+        bool ok = true;
+        const int wrow1 = (w.g * d.N + a.slot) * d.df, wrow2 = (w.g * d.N + a.slot) * D;
+        for (int hc = 0; hc < n_hc && ok; ++hc) {
+          const int s1 = w1c & 1;
+          if (!mbar_wait(&w1_empty[s1], ((w1c >> 1) & 1) ^ 1u, abort_flag, wl)) { ok = false; break; }
+          mbar_arrive_expect_tx(&w1_full[s1], F::kW1);
+          for (int kb = 0; kb < D / 64; ++kb)
+            tma_load_2d(sW1 + s1 * F::kW1 + kb * 128 * 128, &tmW1, &w1_full[s1], kb * 64,
+                        wrow1 + hc * 128);
+          ++w1c;
+          const int s2 = w2c & 1;
+          if (!mbar_wait(&w2_empty[s2], ((w2c >> 1) & 1) ^ 1u, abort_flag, wl)) { ok = false; break; }
+          mbar_arrive_expect_tx(&w2_full[s2], F::kW2);
+          for (int kb = 0; kb < 2; ++kb)
+            tma_load_2d(sW2 + s2 * F::kW2 + kb * D * 128, &tmW2, &w2_full[s2], hc * 128 + kb * 64,
+                        wrow2);
+          ++w2c;
+        }
+        if (!ok) break;
+        ++tl;
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer (warp-uniform, elected lane)
+    const uint32_t id1 = idesc_bf16_f32(128, 128), id2 = idesc_bf16_f32(128, D);
+    int tl = 0, w1c = 0, w2c = 0, c1c = 0, hcc = 0;
+    bool ok = true;
+    for (int it = blockIdx.x; it < total && ok; it += gridDim.x) {
+      const Work w = decode(a, c, it);
+      if (!w.active) continue;
+      if (!mbar_wait(a_full, tl & 1, abort_flag, wl)) { ok = false; break; }
+      auto mma1 = [&](int hc) -> bool {
+        const int s1 = w1c & 1, b1 = c1c & 1;
+        if (!mbar_wait(&w1_full[s1], (w1c >> 1) & 1, abort_flag, wl)) return false;
+        if (!mbar_wait(&c1_empty[b1], ((c1c >> 1) & 1) ^ 1u, abort_flag, wl)) return false;
+        tc_fence_after();
+        if (elect_one()) {
+          for (int kb = 0; kb < D / 64; ++kb) {
+            const uint64_t ad = sdesc_k_sw128(smem_u32(sA + kb * 128 * 128));
+            const uint64_t bd = sdesc_k_sw128(smem_u32(sW1 + s1 * F::kW1 + kb * 128 * 128));
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              umma_bf16(tmem + b1 * 128, ad + 2 * k, bd + 2 * k, id1, (kb | k) != 0);
+          }
+          umma_commit(&c1_full[b1]);
+          umma_commit(&w1_empty[s1]);
+          if (hc == n_hc - 1) umma_commit(a_empty);   // the tile's last read of xf
+        }
+        __syncwarp();
+        mma_issued = true;
+        ++w1c;
+        ++c1c;
+        return true;
+      };
+      auto mma2 = [&](int hc) -> bool {
+        const int s2 = w2c & 1, bh = hcc & 1;
+        if (!mbar_wait(&w2_full[s2], (w2c >> 1) & 1, abort_flag, wl)) return false;
+        if (!mbar_wait(&h_full[bh], (hcc >> 1) & 1, abort_flag, wl)) return false;
+        if (hc == 0 && !mbar_wait(c2_empty, (tl & 1) ^ 1u, abort_flag, wl)) return false;
+        tc_fence_after();
+        if (elect_one()) {
+          for (int kb = 0; kb < 2; ++kb) {
+            const uint64_t ad = sdesc_k_sw128(smem_u32(sH + bh * F::kA2 + kb * 128 * 128));
+            const uint64_t bd = sdesc_k_sw128(smem_u32(sW2 + s2 * F::kW2 + kb * D * 128));
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              umma_bf16(tmem + 256, ad + 2 * k, bd + 2 * k, id2, (hc | kb | k) != 0);
+          }
+          umma_commit(&h_empty[bh]);
+          umma_commit(&w2_empty[s2]);
+          if (hc == n_hc - 1) umma_commit(c2_full);
+        }
+        __syncwarp();
+        ++w2c;
+        ++hcc;
+        return true;
+      };
+      ok = mma1(0);
+      for (int hc = 0; ok && hc < n_hc; ++hc) {
+        if (hc + 1 < n_hc) ok = mma1(hc + 1);
+        if (ok) ok = mma2(hc);
+      }
+      ++tl;
+    }
+  } else if (warp >= 4) {
+    // ------------------------------------------------ epilogue: GELU chunks, then the F2 rows
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    const uint32_t lanes = static_cast<uint32_t>(q * 32) << 16;
+    EpiCtx e{&a, &c};
+    int tl = 0, c1c = 0, hcc = 0;
+    bool ok = true;
+    for (int it = blockIdx.x; it < total && ok; it += gridDim.x) {
+      const Work w = decode(a, c, it);
+      if (!w.active) continue;
+      const float* b1 = a.c_f1 + (int64_t(w.g) * d.N + a.slot) * d.df;
+      for (int hc = 0; hc < n_hc; ++hc) {
+        const int b1i = c1c & 1, bh = hcc & 1;
+        int wv = 1;
+        if (lane == 0) wv = mbar_wait(&c1_full[b1i], (c1c >> 1) & 1, abort_flag, wl) ? 1 : 0;
+        if (!__shfl_sync(0xffffffffu, wv, 0)) { ok = false; break; }
+        wv = 1;
+        if (lane == 0) wv = mbar_wait(&h_empty[bh], ((hcc >> 1) & 1) ^ 1u, abort_flag, wl) ? 1 : 0;
+        if (!__shfl_sync(0xffffffffu, wv, 0)) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t hbase = smem_u32(sH + bh * F::kA2);
+#pragma unroll
+        for (int ch = 0; ch < 4; ++ch) {
+          uint32_t rr[32];
+          tmem_ld_32x32b_x32(tmem + lanes + b1i * 128 + ch * 32, rr);
+          tmem_ld_wait(rr);
+          const float4* bb4 = reinterpret_cast<const float4*>(b1 + hc * 128 + ch * 32);
+          uint32_t pk[16];
+#pragma unroll
+          for (int k4 = 0; k4 < 8; ++k4) {
+            const float4 bb = __ldg(bb4 + k4);
+            const float x0 = gelu_tanh(__uint_as_float(rr[4 * k4]) + bb.x);
+            const float x1 = gelu_tanh(__uint_as_float(rr[4 * k4 + 1]) + bb.y);
+            const float x2 = gelu_tanh(__uint_as_float(rr[4 * k4 + 2]) + bb.z);
+            const float x3 = gelu_tanh(__uint_as_float(rr[4 * k4 + 3]) + bb.w);
+            pk[2 * k4] = pack2(x0, x1);
+            pk[2 * k4 + 1] = pack2(x2, x3);
+          }
+          // row `row`, columns 32 ch .. 32 ch + 31 of the 128-column chunk: block ch / 2,
+          // half ch % 2 of its 64 columns, 16-byte chunks permuted by the 128B swizzle
+          const uint32_t rbase = hbase + (ch >> 1) * 128 * 128 + row * 128;
+#pragma unroll
+          for (int v = 0; v < 4; ++v)
+            st_shared_v4(rbase + static_cast<uint32_t>((((ch & 1) * 4 + v) ^ (row & 7)) << 4),
+                         pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+        }
+        tc_fence_before();
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&c1_empty[b1i]);
+          mbar_arrive(&h_full[bh]);
+        }
+        ++c1c;
+        ++hcc;
+      }
+      if (!ok) break;
+      int wv = 1;
+      if (lane == 0) wv = mbar_wait(c2_full, tl & 1, abort_flag, wl) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, wv, 0)) { ok = false; break; }
+      tc_fence_after();
+      epi_row<D>(e, w, tmem + lanes + 256, row);   // the kBtF2 row epilogue
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(c2_empty);
+      ++tl;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (*abort_flag) {
+    // unwinding: let issued copies land (bounded) and issued MMAs finish
+    if (warp == 0 && lane == 0 && issued) {
+      const long long t0 = clock64();
+      while (clock64() - t0 < (wl < 100000000LL ? wl : 100000000LL)) {
+      }
+    }
+    if (warp == 1 && mma_issued) {
+      if (elect_one()) umma_commit(drain);
+      __syncwarp();
+      const uint32_t ad = smem_u32(drain);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(ad, 0) && clock64() - t0 < wl) {
+      }
+    }
+    __syncthreads();
+  }
+  if (warp == 2) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+  if (threadIdx.x == 0 && *abort_flag) atomicOr(a.status, kStatusTimeout);
+}
+
 // ---------------------------------------------------------------- gate (SIMT)
 //
 // One warp per token: logits_m = Wg[x][m] . window(token) + bg, the window
@@ -910,6 +1196,33 @@ cudaError_t launch_bt_gemm(int mode, const BtArgs& a, const CUtensorMap& tmA,
   const int grid = static_cast<int>(items < num_sms ? items : num_sms);
   if (grid <= 0) return cudaSuccess;
   kern<<<grid, bt_threads(wide ? 16 : 4), kBtSmem, st>>>(tmA, tmA2, tmB, a, c);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bt_ffn(const BtArgs& a, const CUtensorMap& tmXf, const CUtensorMap& tmW1,
+                          const CUtensorMap& tmW2, int num_sms, cudaStream_t st) {
+  const BtDims& d = a.d;
+  if (d.df % 128) return cudaErrorInvalidValue;
+  GemmCfg c{};
+  c.mode = kBtF2;   // the row epilogue after the last chunk is kBtF2's
+  c.groups = d.G;
+  c.row_tiles = d.B * d.tiles_b;
+  c.n_tiles = 1;
+  c.NT = d.d;
+  c.K = d.df;
+  static bool attr[2] = {false, false};
+  const int di = d.d == 128 ? 1 : 0;
+  auto kern = d.d == 128 ? bt_ffn_kernel<128> : bt_ffn_kernel<64>;
+  const int smem = d.d == 128 ? Ffn<128>::kSmem : Ffn<64>::kSmem;
+  if (!attr[di]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    attr[di] = true;
+  }
+  const long long items = static_cast<long long>(c.groups) * c.row_tiles;
+  const int grid = static_cast<int>(items < num_sms ? items : num_sms);
+  if (grid <= 0) return cudaSuccess;
+  kern<<<grid, 256, smem, st>>>(tmXf, tmW1, tmW2, a, c);
   return cudaGetLastError();
 }
 

@@ -91,7 +91,7 @@ struct BtState {
   void *xz = nullptr, *xq = nullptr, *q = nullptr, *kv = nullptr, *o = nullptr, *xf = nullptr,
        *f = nullptr, *xo = nullptr;
   float2* rstat = nullptr;
-  CUtensorMap tm_win{}, tm_wq{}, tm_wkv{}, tm_wo{}, tm_wf1{}, tm_wf2{}, tm_wout{};
+  CUtensorMap tm_win{}, tm_wq{}, tm_wkv{}, tm_wo{}, tm_wf1{}, tm_wf2{}, tm_wout{}, tm_wf1c{};
   CUtensorMap tm_xz{}, tm_xq{}, tm_o{}, tm_xf{}, tm_f{}, tm_xo{};
 
   void free_all() {
@@ -883,6 +883,7 @@ mot_status bt_create(const mot_config* cfg, const mot_bt_config* bc, mot_handle*
   map2(&bt.tm_wkv, bt.wkv, D, G * N * 2 * D, uint32_t(2 * D));
   map2(&bt.tm_wo, bt.wo, D, G * N * D, uint32_t(D));
   map2(&bt.tm_wf1, bt.wf1, D, G * N * df, nt_f1);
+  map2(&bt.tm_wf1c, bt.wf1, D, G * N * df, 128);   // 128-row chunks for the fused FFN
   map2(&bt.tm_wf2, bt.wf2, df, G * N * D, uint32_t(D));
   map2(&bt.tm_wout, bt.wout, uint64_t(bd.P) * D, G * bd.Dt, nt_out);
   // activations (A operands): box 64 x 128 rows
@@ -1420,12 +1421,18 @@ mot_status mot_translate_bt(mot_handle h, const void* src_k, const void* src_v,
     MOT_CUDA_TRY(timed(h, "bt_o_residual_ln", st, [&] {
       return launch_bt_gemm(kBtO, a, bt.tm_o, bt.tm_o, bt.tm_wo, h->num_sms, st);
     }));
-    MOT_CUDA_TRY(timed(h, "bt_ffn1_gelu", st, [&] {
-      return launch_bt_gemm(kBtF1, a, bt.tm_xf, bt.tm_xf, bt.tm_wf1, h->num_sms, st);
-    }));
-    MOT_CUDA_TRY(timed(h, "bt_ffn2_residual_ln", st, [&] {
-      return launch_bt_gemm(kBtF2, a, bt.tm_f, bt.tm_f, bt.tm_wf2, h->num_sms, st);
-    }));
+    if (d.df % 128 == 0) {   // FFN1, GELU and FFN2 with the hidden kept on the SM
+      MOT_CUDA_TRY(timed(h, "bt_ffn_fused", st, [&] {
+        return launch_bt_ffn(a, bt.tm_xf, bt.tm_wf1c, bt.tm_wf2, h->num_sms, st);
+      }));
+    } else {
+      MOT_CUDA_TRY(timed(h, "bt_ffn1_gelu", st, [&] {
+        return launch_bt_gemm(kBtF1, a, bt.tm_xf, bt.tm_xf, bt.tm_wf1, h->num_sms, st);
+      }));
+      MOT_CUDA_TRY(timed(h, "bt_ffn2_residual_ln", st, [&] {
+        return launch_bt_gemm(kBtF2, a, bt.tm_f, bt.tm_f, bt.tm_wf2, h->num_sms, st);
+      }));
+    }
     MOT_CUDA_TRY(timed(h, "bt_out_gelu_combine", st, [&] {
       return launch_bt_gemm(kBtOut, a, bt.tm_xo, bt.tm_xo, bt.tm_wout, h->num_sms, st);
     }));

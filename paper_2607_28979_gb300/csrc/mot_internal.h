@@ -184,6 +184,10 @@ cudaError_t launch_bt_attn(const BtArgs& a, cudaStream_t st);
 cudaError_t launch_bt_gemm(int mode, const BtArgs& a, const CUtensorMap& tmA,
                            const CUtensorMap& tmA2, const CUtensorMap& tmB, int num_sms,
                            cudaStream_t st);
+// FFN1 + GELU + FFN2 in one kernel (d_f % 128 == 0): xf map (box 64 x 128), W_F1
+// map with box 64 x 128, W_F2 map with box 64 x d; ends with kBtF2's row epilogue.
+cudaError_t launch_bt_ffn(const BtArgs& a, const CUtensorMap& tmXf, const CUtensorMap& tmW1,
+                          const CUtensorMap& tmW2, int num_sms, cudaStream_t st);
 
 // ---------------------------------------------------------------- replay attention
 //

@@ -190,12 +190,13 @@ def test_bt_launch_sequence_and_profile():
     M.mot_profile_enable(run.h, True)
     c0 = M.mot_get_launch_count(run.h)
     assert run.translate() == M.MOT_OK
-    N = wl.bt[1]
-    assert M.mot_get_launch_count(run.h) - c0 == 1 + 8 * N
+    N, d_f = wl.bt[1], wl.bt[4]
+    fused = d_f % 128 == 0   # FFN1 + GELU + FFN2 in one kernel
+    assert M.mot_get_launch_count(run.h) - c0 == 1 + (7 if fused else 8) * N
     prof = M.mot_profile_read(run.h)
+    ffn = {"bt_ffn_fused"} if fused else {"bt_ffn1_gelu", "bt_ffn2_residual_ln"}
     assert set(prof) == {"bt_gate", "bt_in_ln_gelu", "bt_q", "bt_kv", "bt_attn",
-                         "bt_o_residual_ln", "bt_ffn1_gelu", "bt_ffn2_residual_ln",
-                         "bt_out_gelu_combine"}
+                         "bt_o_residual_ln", "bt_out_gelu_combine"} | ffn
     assert prof["bt_gate"][0] == 1 and prof["bt_q"][0] == N
 
 

@@ -42,7 +42,7 @@
 
 #include <algorithm>
 
-#include "mot_internal.h"
+#include "bt_internal.h"
 #include "ptx.cuh"
 
 namespace mot {

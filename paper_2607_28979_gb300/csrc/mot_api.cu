@@ -11,7 +11,9 @@
 #include <string>
 #include <vector>
 
+#include "bt_internal.h"
 #include "mot_internal.h"
+#include "replay_internal.h"
 
 using namespace mot;
 
@@ -1557,6 +1559,13 @@ mot_status mot_replay_attention(mot_handle h, int32_t layer, const void* q, cons
     MOT_CUDA_TRY(timed(h, "replay_vt", st, [&] { return launch_replay_vt(a, h->rvt, st); }));
     MOT_CUDA_TRY(timed(h, "replay_fmha_full", st,
                        [&] { return launch_replay_fmha(a, tmQ, tmK, tmVt, st); }));
+    return MOT_OK;
+  }
+  if (!full && replay_gattn_supported(d)) {
+    // guided layer on the tensor cores: selection, then the gathered-row attention
+    MOT_CUDA_TRY(timed(h, "replay_select", st, [&] { return launch_replay_select(a, st); }));
+    MOT_CUDA_TRY(timed(h, "replay_attn_sparse", st,
+                       [&] { return launch_replay_gattn(a, h->num_sms, st); }));
     return MOT_OK;
   }
   if (!full)

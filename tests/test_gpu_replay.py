@@ -23,6 +23,11 @@ SMALL = {
     "r_mha_d64": RW("r_mha_d64", 4, 4, 4, 4, 64, 3, 400, (400, 128, 129), top_s=128, n_full=1),
     # 16 query heads per key/value head, one long row per entry
     "r_gqa16": RW("r_gqa16", 2, 2, 16, 1, 64, 1, 1000, (1000,), top_s=64, n_full=1),
+    # d = 128 on the tensor-core guided kernel: S = 128, 16 heads per group, ragged rows
+    "r_gqa16_d128": RW("r_gqa16_d128", 2, 4, 16, 1, 128, 3, 520, (520, 127, 129), top_s=128,
+                       n_full=1),
+    # d = 128, no GQA, an S that is not a multiple of 4 (partial gather4 groups)
+    "r_mha_d128_s99": RW("r_mha_d128_s99", 2, 4, 3, 3, 128, 2, 333, (333, 98), top_s=99, n_full=1),
 }
 
 

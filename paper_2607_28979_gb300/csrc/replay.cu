@@ -813,12 +813,12 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
   tc_fence_after();
   const uint32_t tmem = *tmem_slot + 32 * ln;   // this lane's S^T (+0) and O^T (+16)
 
-  // gather roles: warp w copies the 16-byte chunks of keys w, w + 4, .., lane l
-  // being chunk l of the key's 32 (16 of its key row, 16 of its value row)
-  const int kv = lane >> 4, q16 = lane & 15;
+  // gather roles: per copy instruction a warp moves two 256-byte rows (lanes
+  // 0-15 one key's row, lanes 16-31 the next key's); warp w takes keys
+  // 8 m + 2 w + {0, 1}, and lane L holds the position of key 8 (L >> 1) + 2 w + (L & 1)
+  const int half = lane >> 4, q16 = lane & 15;
   const uint32_t sbase = smem_u32(tiles);
-  const uint32_t dchunk = sbase + static_cast<uint32_t>(kv * Ga::kKV + (q16 >> 3) * Ga::kBlk);
-  const uint16_t* src_kv = static_cast<const uint16_t*>(kv ? a.v : a.k) + q16 * 8;
+  const int my_key = 8 * (lane >> 1) + 2 * warp + (lane & 1);
   // softmax / output roles: warp w owns keys (S^T rows) and dims (O^T rows) 32 w .. 32 w + 31,
   // TMEM lanes 32 w .. 32 w + 31 (w = the warp's index mod 4)
   const int row = 32 * warp + lane;
@@ -831,34 +831,61 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
   uint32_t n = 0;   // items done: the parity of both MMA barriers
 
   // lane `ln` of CTA `blockIdx.x` takes items v, v + V, .. (v its global lane index)
-  for (int64_t it = int64_t(blockIdx.x) * Ga::kLanes + ln; it < n_items;
-       it += int64_t(gridDim.x) * Ga::kLanes) {
-    int b, hk, u;
-    if (!gattn_item(a, it, b, hk, u)) continue;
-    const int c = min(d.S, u + 1);
-    // ---- gather the selected key / value rows and the group's query rows
-    {
-      const int32_t* sel = a.sel + (int64_t(b) * d.N + u) * d.S;
-      const int my_key = warp + 4 * lane;
-      const int my_pos = my_key < c ? min(max(sel[my_key], 0), d.N - 1) : 0;
-      const int64_t row0 = int64_t(b * d.Hkv + hk) * d.N;
-#pragma unroll 4
-      for (int m = 0; m < 32; ++m) {
-        const int key = warp + 4 * m;
-        const int pos = __shfl_sync(0xffffffffu, my_pos, m);
-        if (key < c)
-          cp_async_16(dchunk + key * 128 + (((q16 & 7) ^ (key & 7)) << 4), src_kv + (row0 + pos) * D);
+  struct Item {
+    int b, hk, u, c;
+  };
+  int64_t it = int64_t(blockIdx.x) * Ga::kLanes + ln;
+  const int64_t it_step = int64_t(gridDim.x) * Ga::kLanes;
+  auto next_item = [&](Item& x) -> bool {
+    for (; it < n_items; it += it_step) {
+      if (gattn_item(a, it, x.b, x.hk, x.u)) {
+        x.c = min(d.S, x.u + 1);
+        it += it_step;
+        return true;
       }
+    }
+    return false;
+  };
+  auto load_pos = [&](const Item& x) -> int {
+    return my_key < x.c ? min(max(a.sel[(int64_t(x.b) * d.N + x.u) * d.S + my_key], 0), d.N - 1) : 0;
+  };
+  // the item's selected key rows (which = 0, plus its query rows) or value rows (which = 1)
+  auto issue_rows = [&](const Item& x, int my_pos, int which) {
+    const uint16_t* src = static_cast<const uint16_t*>(which ? a.v : a.k) +
+                          int64_t(x.b * d.Hkv + x.hk) * d.N * D + q16 * 8;
+    const uint32_t dst = sbase + static_cast<uint32_t>(which * Ga::kKV + (q16 >> 3) * Ga::kBlk);
+#pragma unroll 4
+    for (int m = 0; m < 16; ++m) {
+      const int key = 8 * m + 2 * warp + half;
+      const int pos = __shfl_sync(0xffffffffu, my_pos, 2 * m + half);
+      if (key < x.c) cp_async_16(dst + key * 128 + (((q16 & 7) ^ (key & 7)) << 4), src + int64_t(pos) * D);
+    }
+    if (which == 0) {
       for (int e = tid; e < G * 16; e += 128) {
         const int h = e >> 4, c16 = e & 15;
         cp_async_16(sbase + Ga::kOffQ + (c16 >> 3) * Ga::kQBlk + h * 128 + (((c16 & 7) ^ (h & 7)) << 4),
-                    static_cast<const uint16_t*>(a.q) + ((int64_t(b) * d.Hq + hk * G + h) * d.N + u) * D +
-                        c16 * 8);
+                    static_cast<const uint16_t*>(a.q) +
+                        ((int64_t(x.b) * d.Hq + x.hk * G + h) * d.N + x.u) * D + c16 * 8);
       }
-      cp_async_commit();
-      cp_async_wait_group<0>();
-      fence_proxy_async_smem();   // this thread's copies, visible to the tensor core
     }
+    cp_async_commit();
+  };
+
+  // Copies run one step ahead: the next item's key and query rows go out once
+  // the first MMA has read the current ones, its value rows once the second
+  // MMA has. Commit groups stay in the order KQ(i), V(i), KQ(i+1), V(i+1), ..
+  Item cur, nxt;
+  bool have = next_item(cur);
+  int pos_cur = have ? load_pos(cur) : 0;
+  if (have) {
+    issue_rows(cur, pos_cur, 0);
+    issue_rows(cur, pos_cur, 1);
+  }
+  while (have) {
+    const bool have_nxt = next_item(nxt);
+    const int pos_nxt = have_nxt ? load_pos(nxt) : 0;
+    cp_async_wait_group<1>();   // KQ(cur) landed (V(cur) may still be in flight)
+    fence_proxy_async_smem();   // this thread's copies, visible to the tensor core
     lane_sync(bar_id);
     // ---- MMA 1: S^T = K_sel Q^T (M = 128 keys, N = 16 heads, K = d)
     if (warp == 0) {
@@ -879,19 +906,22 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
     if (!lane_and(bar_id, tid != 0 || mbar_wait(bar_s, n & 1u, abort_flag, wl))) break;
     tc_fence_after();
     // ---- softmax over the keys of each head (TMEM lane = key)
-    const bool valid = row < c;
+    const bool valid = row < cur.c;
     float sc[16];
     {
       uint32_t v[16];
       tmem_ld_32x32b_x16(tmem + tlanes, v);
       tmem_ld_wait(v);
 #pragma unroll
-      for (int h = 0; h < 16; ++h) {
-        sc[h] = __uint_as_float(v[h]) * sl2;
-        if (h < G) {
-          const float m = redux_max_f32(valid ? sc[h] : -INFINITY);
-          if (lane == h) xm[h * 4 + warp] = m;
-        }
+      for (int h = 0; h < 16; ++h) sc[h] = __uint_as_float(v[h]) * sl2;
+    }
+    if (have_nxt) issue_rows(nxt, pos_nxt, 0);   // the key and query tiles are free again
+    else cp_async_commit();
+#pragma unroll
+    for (int h = 0; h < 16; ++h) {
+      if (h < G) {
+        const float m = redux_max_f32(valid ? sc[h] : -INFINITY);
+        if (lane == h) xm[h * 4 + warp] = m;
       }
     }
     lane_sync(bar_id);
@@ -907,14 +937,15 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
         if (lane == h) xl[h * 4 + warp] = sum;
       }
     }
-    fence_proxy_async_smem();
+    cp_async_wait_group<1>();   // V(cur) landed (KQ(nxt) may still be in flight)
+    fence_proxy_async_smem();   // the P tile and the value rows, visible to the tensor core
     tc_fence_before();
     lane_sync(bar_id);
     // ---- MMA 2: O^T = V_sel^T P^T (M = 128 dims, value rows read MN-major, N = 16 heads)
     if (warp == 0) {
       tc_fence_after();
       if (elect_one()) {
-        const int n_ks = (c + 15) >> 4;   // 16-key steps holding the row's keys
+        const int n_ks = (cur.c + 15) >> 4;   // 16-key steps holding the row's keys
         for (int ks = 0; ks < n_ks; ++ks) {
           const uint64_t ad = sdesc_mn_sw128(sbase + Ga::kOffV + ks * 2048, Ga::kBlk);
           const uint64_t bd = sdesc_k_sw128(sbase + Ga::kOffP + (ks >> 2) * Ga::kPBlk) + 2 * (ks & 3);
@@ -926,12 +957,14 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
     }
     if (!lane_and(bar_id, tid != 0 || mbar_wait(bar_o, n & 1u, abort_flag, wl))) break;
     tc_fence_after();
+    if (have_nxt) issue_rows(nxt, pos_nxt, 1);   // the value tile is free again
+    else cp_async_commit();
     // ---- output: O^T row = this thread's dim, normalised per head
     {
       uint32_t v[16];
       tmem_ld_32x32b_x16(tmem + tlanes + 16, v);
       tmem_ld_wait(v);
-      uint16_t* o = static_cast<uint16_t*>(a.out) + ((int64_t(b) * d.Hq + hk * G) * d.N + u) * D + row;
+      uint16_t* o = static_cast<uint16_t*>(a.out) + ((int64_t(cur.b) * d.Hq + cur.hk * G) * d.N + cur.u) * D + row;
 #pragma unroll
       for (int h = 0; h < 16; ++h) {
         if (h < G) {
@@ -942,8 +975,10 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
       }
     }
     tc_fence_before();
-    lane_sync(bar_id);   // tiles, exchange words and TMEM free for the next item
+    lane_sync(bar_id);   // exchange words and TMEM free for the next item
     ++n;
+    cur = nxt;
+    have = have_nxt;
   }
 
   cp_async_wait_group<0>();

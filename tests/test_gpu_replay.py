@@ -81,13 +81,17 @@ def test_selection_is_bit_exact_on_every_row(name):
         assert (sel[b, L:] == -7).all()   # rows past the sequence are not written
 
 
-def test_selection_ties_and_constant_rows():
-    wl = SMALL["r_gqa6_d128"].replace(top_s=8)
+@pytest.mark.parametrize("name", ["r_gqa6_d128", "r_mha_d64"])   # max_seq 300 and 400: scalar and 16-byte loads
+def test_selection_ties_and_constant_rows(name):
+    wl = SMALL[name].replace(top_s=8)
     N = wl.max_seq
     g = np.zeros((wl.max_batch, N, N), dtype=np.uint16)
     g[0] = 0x4000                                  # every score 2.0: the lowest positions win
     rng = np.random.default_rng(0)
     g[1] = (0x3F80 + rng.integers(0, 3, size=(N, N))).astype(np.uint16)   # three values only
+    if wl.batch > 2:   # mixed signs (no exact zeros: -0 and +0 order apart in the 16-bit keys)
+        x = rng.standard_normal((N, N)).astype(np.float32)
+        g[2] = (x.view(np.uint32) >> 16).astype(np.uint16)
     run = ReplayRun(wl)
     sel = run.select(g)
     for b, L in enumerate(wl.seq_lens):

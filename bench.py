@@ -154,6 +154,10 @@ KERNEL_SOURCES = {
     "umma2_gemm1_gelu_gate": ["umma2.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
     "umma2_gemm2_combine_store": ["umma2.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
     "umma2_onchip_translate": ["onchip.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
+    # replay stages (all kernels of replay.cu)
+    "replay_attn_sparse": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
+    "replay_select": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
+    "replay_fmha_full": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
 }
 
 
@@ -837,13 +841,14 @@ def run_replay(args, wl):
             ach = per["flops"] / avg_s / 1e12
             roof = {"kernel": name, "bound": "tensor", "achieved": round(ach, 2), "peak": peak_t,
                     "unit": "TFLOP/s", "frac": round(ach / peak_t, 4),
-                    "peak_kind": f"bf16 dense sustained, {peak_kind}", "traffic": None,
+                    "peak_kind": f"bf16 dense sustained, {peak_kind}",
+                    "traffic": recorded_traffic(name, wl.name),
                     "algorithmic_per_launch": per["flops"], "avg_launch_ms": 1000 * avg_s}
         else:
             ach = per["bytes"] / avg_s / 1e9
             roof = {"kernel": name, "bound": "hbm", "achieved": round(ach, 1),
                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(ach / peaks["hbm_gbs"], 4),
-                    "peak_kind": f"HBM copy, {peak_kind}", "traffic": None,
+                    "peak_kind": f"HBM copy, {peak_kind}", "traffic": recorded_traffic(name, wl.name),
                     "algorithmic_per_launch": per["bytes"], "avg_launch_ms": 1000 * avg_s}
         t_roof = max(alg["flops"] / (peaks["bf16_tflops"] * 1e12), alg["bytes"] / (peaks["hbm_gbs"] * 1e9))
         cpu = None

@@ -871,21 +871,35 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
     cp_async_commit();
   };
 
-  // Copies run one step ahead: the next item's key and query rows go out once
-  // the first MMA has read the current ones, its value rows once the second
-  // MMA has. Commit groups stay in the order KQ(i), V(i), KQ(i+1), V(i+1), ..
-  Item cur, nxt;
-  bool have = next_item(cur);
+  // Per item i the lane issues the first MMA, then finishes item i - 1 (waits
+  // for its second MMA, copies item i's value rows into the freed tile, writes
+  // item i - 1's output rows), then runs item i's softmax (copying item i + 1's
+  // key and query rows into the freed tiles) and issues its second MMA without
+  // waiting for it. Commit groups run KQ(0), V(0), KQ(1), V(1), ..
+  auto output_rows = [&](const Item& x) {   // O^T row = this thread's dim, normalised per head
+    uint32_t v[16];
+    tmem_ld_32x32b_x16(tmem + tlanes + 16, v);
+    tmem_ld_wait(v);
+    uint16_t* o = static_cast<uint16_t*>(a.out) + ((int64_t(x.b) * d.Hq + x.hk * G) * d.N + x.u) * D + row;
+#pragma unroll
+    for (int h = 0; h < 16; ++h) {
+      if (h < G) {
+        const uint4 l4 = *reinterpret_cast<const uint4*>(xl + h * 4);
+        const float l = __uint2float_rn(l4.x + l4.y + l4.z + l4.w) * (1.f / 16777216.f);
+        o[int64_t(h) * d.N * D] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(v[h]) / l));
+      }
+    }
+  };
+  Item cur, nxt, prev;
+  bool have = next_item(cur), have_prev = false, ok = true;
   int pos_cur = have ? load_pos(cur) : 0;
-  if (have) {
-    issue_rows(cur, pos_cur, 0);
-    issue_rows(cur, pos_cur, 1);
-  }
+  if (have) issue_rows(cur, pos_cur, 0);
   while (have) {
     const bool have_nxt = next_item(nxt);
     const int pos_nxt = have_nxt ? load_pos(nxt) : 0;
-    cp_async_wait_group<1>();   // KQ(cur) landed (V(cur) may still be in flight)
+    cp_async_wait_group<0>();   // KQ(cur) landed
     fence_proxy_async_smem();   // this thread's copies, visible to the tensor core
+    tc_fence_before();
     lane_sync(bar_id);
     // ---- MMA 1: S^T = K_sel Q^T (M = 128 keys, N = 16 heads, K = d)
     if (warp == 0) {
@@ -903,7 +917,20 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
       __syncwarp();
       mma_issued = true;
     }
-    if (!lane_and(bar_id, tid != 0 || mbar_wait(bar_s, n & 1u, abort_flag, wl))) break;
+    // ---- finish the previous item while the first MMA runs
+    if (have_prev) {
+      if (!lane_and(bar_id, tid != 0 || mbar_wait(bar_o, (n - 1) & 1u, abort_flag, wl))) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+    }
+    issue_rows(cur, pos_cur, 1);   // the value tile (and the P tile) are free again
+    if (have_prev) output_rows(prev);
+    if (!lane_and(bar_id, tid != 0 || mbar_wait(bar_s, n & 1u, abort_flag, wl))) {
+      ok = false;
+      break;
+    }
     tc_fence_after();
     // ---- softmax over the keys of each head (TMEM lane = key)
     const bool valid = row < cur.c;
@@ -924,7 +951,7 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
         if (lane == h) xm[h * 4 + warp] = m;
       }
     }
-    lane_sync(bar_id);
+    lane_sync(bar_id);   // maxima traded; every thread's output rows of the previous item read xl
 #pragma unroll
     for (int h = 0; h < 16; ++h) {
       if (h < G) {
@@ -955,30 +982,18 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
       }
       __syncwarp();
     }
-    if (!lane_and(bar_id, tid != 0 || mbar_wait(bar_o, n & 1u, abort_flag, wl))) break;
-    tc_fence_after();
-    if (have_nxt) issue_rows(nxt, pos_nxt, 1);   // the value tile is free again
-    else cp_async_commit();
-    // ---- output: O^T row = this thread's dim, normalised per head
-    {
-      uint32_t v[16];
-      tmem_ld_32x32b_x16(tmem + tlanes + 16, v);
-      tmem_ld_wait(v);
-      uint16_t* o = static_cast<uint16_t*>(a.out) + ((int64_t(cur.b) * d.Hq + cur.hk * G) * d.N + cur.u) * D + row;
-#pragma unroll
-      for (int h = 0; h < 16; ++h) {
-        if (h < G) {
-          const uint4 l4 = *reinterpret_cast<const uint4*>(xl + h * 4);
-          const float l = __uint2float_rn(l4.x + l4.y + l4.z + l4.w) * (1.f / 16777216.f);
-          o[int64_t(h) * d.N * D] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(v[h]) / l));
-        }
-      }
-    }
-    tc_fence_before();
-    lane_sync(bar_id);   // exchange words and TMEM free for the next item
     ++n;
+    prev = cur;
+    have_prev = true;
     cur = nxt;
+    pos_cur = pos_nxt;
     have = have_nxt;
+  }
+  if (ok && have_prev) {   // the last item's output rows
+    if (lane_and(bar_id, tid != 0 || mbar_wait(bar_o, (n - 1) & 1u, abort_flag, wl))) {
+      tc_fence_after();
+      output_rows(prev);
+    }
   }
 
   cp_async_wait_group<0>();

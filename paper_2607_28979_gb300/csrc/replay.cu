@@ -142,17 +142,19 @@ __global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const Rep
     for (int j8 = lane * 8; j8 - lane * 8 < n; j8 += 256) {   // warp-uniform trip count
       uint32_t o[8];
       if (j8 < n) load8(j8, o);
+      if (pass == 0) {
+        // many scores share a high byte: one warp-aggregated increment per distinct bin
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        int bin = 256;   // none
-        if (j8 + e < n) {
-          if (pass == 0)
-            bin = int(o[e] >> 8);
-          else if ((o[e] >> 8) == hi)
-            bin = int(o[e] & 0xFFu);
+        for (int e = 0; e < 8; ++e) {
+          const int bin = j8 + e < n ? int(o[e] >> 8) : 256;   // 256: none
+          const unsigned peers = __match_any_sync(0xffffffffu, bin);
+          if (bin < 256 && lane == __ffs(peers) - 1) atomicAdd(&hw[bin], __popc(peers));
         }
-        const unsigned peers = __match_any_sync(0xffffffffu, bin);
-        if (bin < 256 && lane == __ffs(peers) - 1) atomicAdd(&hw[bin], __popc(peers));
+      } else {
+        // only the scores in bin `hi` count, spread over 256 low bytes: plain increments
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+          if (j8 + e < n && (o[e] >> 8) == hi) atomicAdd(&hw[o[e] & 0xFFu], 1);
       }
     }
     __syncwarp();

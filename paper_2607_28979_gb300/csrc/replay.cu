@@ -82,6 +82,7 @@ __device__ __forceinline__ int seq_len_of(const ReplayArgs& a, int b) {
 }
 
 constexpr int kSelWarps = 8;         // rows per CTA, one warp each
+constexpr int kSelCopies = 4;        // histogram copies per warp
 
 // Warp-wide exclusive prefix of v (and the warp total).
 __device__ __forceinline__ int warp_excl_scan(int v, int& total) {
@@ -103,7 +104,7 @@ __device__ __forceinline__ int warp_excl_scan(int v, int& total) {
 // positions with o == V, compacted in ascending order by warp scans. Each lane
 // reads 8 consecutive scores per step (16-byte loads when max_seq % 8 == 0).
 __global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const ReplayArgs a) {
-  __shared__ int hist[kSelWarps][256];
+  __shared__ int hist[kSelWarps][kSelCopies][256];   // copy lane % kSelCopies: fewer same-bin collisions
   const ReplayDims& d = a.d;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = blockIdx.x * kSelWarps + w;
@@ -133,23 +134,19 @@ __global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const Rep
       for (int e = 0; e < 8; ++e) o[e] = j8 + e < n ? ord16(__ldg(A + j8 + e)) : 0u;
     }
   };
-  int* hw = hist[w];
+  int* hw = hist[w][lane % kSelCopies];
   int k = d.S;
   uint32_t hi = 0, V = 0;
   for (int pass = 0; pass < 2; ++pass) {
-    for (int i = lane; i < 256; i += 32) hw[i] = 0;
+    for (int i = lane; i < kSelCopies * 256; i += 32) hist[w][0][i] = 0;
     __syncwarp();
     for (int j8 = lane * 8; j8 - lane * 8 < n; j8 += 256) {   // warp-uniform trip count
       uint32_t o[8];
       if (j8 < n) load8(j8, o);
       if (pass == 0) {
-        // many scores share a high byte: one warp-aggregated increment per distinct bin
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          const int bin = j8 + e < n ? int(o[e] >> 8) : 256;   // 256: none
-          const unsigned peers = __match_any_sync(0xffffffffu, bin);
-          if (bin < 256 && lane == __ffs(peers) - 1) atomicAdd(&hw[bin], __popc(peers));
-        }
+        for (int e = 0; e < 8; ++e)
+          if (j8 + e < n) atomicAdd(&hw[o[e] >> 8], 1);
       } else {
         // only the scores in bin `hi` count, spread over 256 low bytes: plain increments
 #pragma unroll
@@ -162,7 +159,9 @@ __global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const Rep
     int c[8], t = 0;
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-      c[e] = hw[(31 - lane) * 8 + (7 - e)];
+      c[e] = 0;
+#pragma unroll
+      for (int cp = 0; cp < kSelCopies; ++cp) c[e] += hist[w][cp][(31 - lane) * 8 + (7 - e)];
       t += c[e];
     }
     int tot;

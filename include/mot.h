@@ -226,6 +226,9 @@ mot_status mot_profile_read(mot_handle h, mot_kernel_stat* out, int32_t cap, int
  * first CTA of the single-SM GEMM1 kernel (schedule 0) never fills its first
  * pipeline stage, so a wait on it runs out: translations then report
  * MOT_ERR_TIMEOUT through mot_get_device_status and the context stays usable.
+ * On a replay handle, stall_test = 1 makes the tensor-core guided attention's
+ * first CTA withhold the completion signal of its first MMA, with the same
+ * outcome for mot_replay_attention on a guided layer.
  */
 mot_status mot_debug_set(mot_handle h, int32_t stall_test, int64_t wait_limit_cycles);
 

@@ -1511,6 +1511,8 @@ mot_status replay_args(mot_handle h, const void* q, const void* k, const void* v
   a.seq_lens = seq_lens;
   a.batch = batch;
   a.status = h->status;
+  a.wait_limit = h->wait_limit;
+  a.stall_test = h->stall_test;
   return MOT_OK;
 }
 

@@ -27,6 +27,8 @@ struct ReplayArgs {
   int32_t batch;
   int32_t full;   // 1: attend to every position 0..u
   int32_t* status;
+  long long wait_limit;   // bound of every pipeline wait (SM cycles)
+  int32_t stall_test;     // test hook: the guided kernel's first CTA stalls its first MMA barrier
 };
 bool replay_supported(const ReplayDims& d);
 // Full causal attention on the tensor cores: maps over q [B*Hq*N][d], k

@@ -177,3 +177,30 @@ def test_batch_prefix_and_errors():
     with pytest.raises(M.MotError) as e:
         M.mot_create_replay(M.replay_config_from(wl.replace(kv_heads=3)))
     assert e.value.status == M.MOT_ERR_INVALID_ARG
+
+
+def test_guided_timeout_is_reported_and_recovers():
+    """Failure detection without a fault: with the stall hook the guided kernel's
+    first CTA withholds one MMA completion signal, its wait runs out after the
+    short limit, the kernel unwinds and the status word reports a timeout. The
+    next guided layer on the same context matches the oracle."""
+    wl = SMALL["r_gqa6_d128"]
+    q, k, v = synth.gen_replay_qkv(wl, 3)
+    g = synth.gen_guide(wl, 6)
+    run = ReplayRun(wl)
+    layer = wl.n_full + 1
+    M.mot_debug_set(run.h, True, 20_000_000)        # about 10 ms of SM cycles
+    run.attend(layer, q, k, v, g)
+    assert M.mot_get_device_status(run.h) == M.MOT_ERR_TIMEOUT
+    assert M.mot_get_device_status(run.h) == M.MOT_OK   # reading cleared it
+    M.mot_debug_set(run.h, False, 0)
+    out = run.attend(layer, q, k, v, g)
+    assert M.mot_get_device_status(run.h) == M.MOT_OK
+    rng = np.random.default_rng(5)
+    tb, th, tu = [], [], []
+    for b, L in enumerate(wl.seq_lens):
+        for u in np.unique(np.concatenate([[0, L - 1], rng.integers(0, L, size=12)])):
+            for h in rng.choice(wl.q_heads, size=3, replace=False):
+                tb.append(b); th.append(h); tu.append(u)
+    ref = oracle.replay_tokens(wl, layer, q, k, v, g, tb, th, tu)
+    G.assert_parity(BF16, _f64(out)[tb, th, tu], ref, "guided layer after a timeout")

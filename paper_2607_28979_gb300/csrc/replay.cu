@@ -411,6 +411,23 @@ struct Fa {
 };
 static_assert(Fa<128>::kSmem <= 232448, "shared memory budget");
 
+// Each thread of the warp writes 32 consecutive 32-bit columns of its TMEM lane.
+__device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+      "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]),
+      "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]),
+      "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 // chunk store of 32 bf16 (16 words) into row r of a 128B-swizzled 64-column block,
 // half s (columns 32 s .. 32 s + 31)
 __device__ __forceinline__ void st_sw128_half(uint32_t blk, int r, int s, const uint32_t (&pk)[16]) {
@@ -441,8 +458,7 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
   uint64_t* s_empty = bars + 7;      // [2]
   uint64_t* p_full = bars + 9;       // [2]
   uint64_t* p_empty = bars + 11;     // [2]
-  uint64_t* pv_full = bars + 13;     // [2]
-  uint64_t* pv_empty = bars + 15;    // [2]
+  uint64_t* pv_done = bars + 13;     // phase j: PV_j has been added into O
   uint64_t* drain = bars + 17;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -469,9 +485,9 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
       mbar_init(&s_empty[i], 4);
       mbar_init(&p_full[i], 4);
       mbar_init(&p_empty[i], 1);
-      mbar_init(&pv_full[i], 1);
-      mbar_init(&pv_empty[i], 4);
+
     }
+    mbar_init(pv_done, 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -488,7 +504,7 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = *tmem_slot;   // S[i] at columns 128 i, PV[i] at 256 + D i
+  const uint32_t tmem = *tmem_slot;   // S[i] at columns 128 i, O at 256 (D columns)
   uint32_t issued_mask = 0, issue_parity = 0;
   bool mma_issued = false;
 
@@ -538,10 +554,9 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
       mma_issued = true;
       return true;
     };
-    auto issue_pv = [&](int j) -> bool {   // PV[j & 1] = P_j V_j (B = V_j^T, K-major)
+    auto issue_pv = [&](int j) -> bool {   // O += P_j V_j (B = V_j^T, K-major); tile 0 overwrites
       const int st = j & 1;
       if (!mbar_wait(&p_full[st], (j >> 1) & 1, abort_flag, wl)) return false;
-      if (!mbar_wait(&pv_empty[st], ((j >> 1) & 1) ^ 1u, abort_flag, wl)) return false;
       tc_fence_after();
       if (elect_one()) {
         for (int kb = 0; kb < 2; ++kb) {
@@ -550,9 +565,9 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
               sdesc_k_sw128(smem_u32(sV + st * Fa<D>::kVt + kb * Fa<D>::kVtBlk));
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            umma_bf16(tmem + 256 + st * D, ad + 2 * k, bd + 2 * k, idPV, (kb | k) != 0);
+            umma_bf16(tmem + 256, ad + 2 * k, bd + 2 * k, idPV, (j | kb | k) != 0);
         }
-        umma_commit(&pv_full[st]);
+        umma_commit(pv_done);
         umma_commit(&p_empty[st]);
         umma_commit(&kv_empty[st]);
       }
@@ -566,38 +581,24 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
     }
   } else if (warp >= 4) {
     // ------------------------------------------------ softmax and output rows
+    // O accumulates in TMEM across key tiles. A row's running max m is raised
+    // only when a tile's max exceeds it by more than kTau (base 2), so every
+    // probability exp2(s - m) stays below 2^kTau; raising it rescales the row's
+    // sum and its O row in TMEM (after the previous tile's PV has landed).
+    constexpr float kTau = 8.f;
     const int r = (warp & 3) * 32 + lane;
     const uint32_t lanes = static_cast<uint32_t>((warp & 3) * 32) << 16;
     const float sl2 = rsqrtf(float(D)) * 1.4426950408889634f;   // scale * log2(e)
-    float o[D];
-#pragma unroll
-    for (int i = 0; i < D; ++i) o[i] = 0.f;
-    float m = -INFINITY, l = 0.f, alpha_prev = 0.f;
+    float m = -INFINITY, l = 0.f;
     bool ok = true;
-    auto apply_pv = [&](int j, float alpha) -> bool {   // o = o * alpha + PV_j
-      const int st = j & 1;
+    auto wait_lane0 = [&](uint64_t* bar, uint32_t par) -> bool {
       int w = 1;
-      if (lane == 0) w = mbar_wait(&pv_full[st], (j >> 1) & 1, abort_flag, wl) ? 1 : 0;
-      if (!__shfl_sync(0xffffffffu, w, 0)) return false;
-      tc_fence_after();
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(tmem + lanes + 256 + st * D + c * 32, v);
-        tmem_ld_wait(v);
-#pragma unroll
-        for (int k = 0; k < 32; ++k) o[c * 32 + k] = fmaf(o[c * 32 + k], alpha, __uint_as_float(v[k]));
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&pv_empty[st]);
-      return true;
+      if (lane == 0) w = mbar_wait(bar, par, abort_flag, wl) ? 1 : 0;
+      return __shfl_sync(0xffffffffu, w, 0) != 0;
     };
     for (int j = 0; j < n_kv; ++j) {
       const int st = j & 1;
-      int w = 1;
-      if (lane == 0) w = mbar_wait(&s_full[st], (j >> 1) & 1, abort_flag, wl) ? 1 : 0;
-      if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+      if (!wait_lane0(&s_full[st], (j >> 1) & 1)) { ok = false; break; }
       tc_fence_after();
       const bool diag = j == qt;
       // pass 1: the row maximum of the scaled, masked scores
@@ -611,13 +612,28 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
         for (int k = 0; k < 32; ++k)
           if (!diag || c * 32 + k <= r) mx = fmaxf(mx, __uint_as_float(v[k]) * sl2);
       }
-      const float m_new = fmaxf(m, mx);
-      const float alpha = m == -INFINITY ? 0.f : exp2f(m - m_new);
+      const bool raise = mx > m + kTau;   // always on the first tile (m = -inf)
+      const float alpha = (raise && m != -INFINITY) ? exp2f(m - mx) : 1.f;
+      if (__any_sync(0xffffffffu, alpha != 1.f)) {
+        // rescale O rows in TMEM once PV_{j-1} has been added
+        if (!wait_lane0(pv_done, static_cast<uint32_t>(j - 1) & 1u)) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(tmem + lanes + 256 + c * 32, v);
+          tmem_ld_wait(v);
+#pragma unroll
+          for (int k = 0; k < 32; ++k) v[k] = __float_as_uint(__uint_as_float(v[k]) * alpha);
+          tmem_st_32x32b_x32(tmem + lanes + 256 + c * 32, v);
+        }
+        tmem_st_wait();
+      }
+      l *= alpha;
+      if (raise) m = mx;
       // P_j must not overwrite the buffer before PV_{j-2} has read it
-      w = 1;
-      if (lane == 0) w = mbar_wait(&p_empty[st], ((j >> 1) & 1) ^ 1u, abort_flag, wl) ? 1 : 0;
-      if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
-      // pass 2: P = exp2(s - m_new) as bf16 into the swizzled P tile, and its row sum
+      if (!wait_lane0(&p_empty[st], ((j >> 1) & 1) ^ 1u)) { ok = false; break; }
+      // pass 2: P = exp2(s - m) as bf16 into the swizzled P tile, and its row sum
       float sum = 0.f;
       const uint32_t pbase = smem_u32(sP + st * Fa<D>::kP);
 #pragma unroll
@@ -629,8 +645,8 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
           const int c0 = c * 32 + 2 * k;
-          const float p0 = (!diag || c0 <= r) ? exp2f(__uint_as_float(v[2 * k]) * sl2 - m_new) : 0.f;
-          const float p1 = (!diag || c0 + 1 <= r) ? exp2f(__uint_as_float(v[2 * k + 1]) * sl2 - m_new) : 0.f;
+          const float p0 = (!diag || c0 <= r) ? exp2f(__uint_as_float(v[2 * k]) * sl2 - m) : 0.f;
+          const float p1 = (!diag || c0 + 1 <= r) ? exp2f(__uint_as_float(v[2 * k + 1]) * sl2 - m) : 0.f;
           __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
           // the row sum counts the rounded probabilities the second MMA uses
           const float2 pr = __bfloat1622float2(pb);
@@ -646,26 +662,31 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
         mbar_arrive(&s_empty[st]);
         mbar_arrive(&p_full[st]);
       }
-      l = l * alpha + sum;
-      m = m_new;
-      if (j > 0 && !apply_pv(j - 1, alpha_prev)) { ok = false; break; }
-      alpha_prev = alpha;
+      l += sum;
     }
-    if (ok && apply_pv(n_kv - 1, alpha_prev)) {
+    if (ok && wait_lane0(pv_done, static_cast<uint32_t>(n_kv - 1) & 1u)) {
+      tc_fence_after();
       const int q = q0 + r;
-      if (q < L) {
-        const float inv = 1.f / l;
-        uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.out) +
-                                              ((int64_t(b) * d.Hq + h) * d.N + q) * D);
+      const float inv = 1.f / l;
+      uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.out) +
+                                            ((int64_t(b) * d.Hq + h) * d.N + q) * D);
 #pragma unroll
-        for (int c = 0; c < D / 8; ++c) {
-          uint32_t w4[4];
+      for (int c = 0; c < D / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld_32x32b_x32(tmem + lanes + 256 + c * 32, v);
+        tmem_ld_wait(v);
+        if (q < L) {
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            __nv_bfloat162 t = __floats2bfloat162_rn(o[8 * c + 2 * e] * inv, o[8 * c + 2 * e + 1] * inv);
-            w4[e] = *reinterpret_cast<uint32_t*>(&t);
+          for (int e8 = 0; e8 < 4; ++e8) {
+            uint32_t w4[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              __nv_bfloat162 t = __floats2bfloat162_rn(__uint_as_float(v[8 * e8 + 2 * e]) * inv,
+                                                       __uint_as_float(v[8 * e8 + 2 * e + 1]) * inv);
+              w4[e] = *reinterpret_cast<uint32_t*>(&t);
+            }
+            dst[c * 4 + e8] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
           }
-          dst[c] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
         }
       }
     }

@@ -664,7 +664,7 @@ def _replay_oracle_rate(wl, layers, budget_s, seed=5):
 
     def sample(n):
         tb = rng.integers(0, wl.batch, size=n)
-        tu = np.array([rng.integers(0, wl.seq_lens[b]) for b in tb])
+        tu = (rng.random(n) * np.asarray(wl.seq_lens)[tb]).astype(np.int64)   # u < seq_len(b)
         th = rng.integers(0, wl.q_heads, size=n)
         tl = rng.integers(0, wl.n_layers_tgt, size=n)
         return tb, th, tu, tl
@@ -674,12 +674,19 @@ def _replay_oracle_rate(wl, layers, budget_s, seed=5):
             m = tl == l
             q, k, v, g = layers(int(l), gl)
             oracle.replay_tokens(wl, int(l), q, k, v, g, tb[m], th[m], tu[m])
-    c = omp_cores()
-    smp = sample(4 * c)
-    t0 = time.perf_counter()
-    run(*smp)
-    per_q = max((time.perf_counter() - t0) / (4 * c), 1e-7)
-    n = int(max(4 * c, min(200000, budget_s / per_q)))
+    # calibrate on samples large enough that per-layer call overhead does not
+    # dominate (doubling until one takes a second or a tenth of the budget)
+    n = 4 * omp_cores()
+    while True:
+        smp = sample(n)
+        t0 = time.perf_counter()
+        run(*smp)
+        dt = time.perf_counter() - t0
+        if dt >= min(1.0, 0.1 * budget_s) or n >= 1 << 20:
+            break
+        n *= 2
+    per_q = max(dt / n, 1e-8)
+    n = int(max(n, min(2_000_000, budget_s / per_q)))
     smp = sample(n)
     t0 = time.perf_counter()
     run(*smp)

@@ -1014,13 +1014,29 @@ __global__ void __launch_bounds__(256) bt_gate_kernel(const BtArgs a) {
 // scaled by 1/sqrt(d/n_a), a max-subtracted softmax in fp32 and the weighted
 // sum of the value rows. Consecutive threads take consecutive heads of a row,
 // so a warp reads whole query rows and writes whole output rows.
+// The CTA first copies the key/value rows of the tokens its threads cover into
+// shared memory (one coalesced pass), so each token's rows are read from memory
+// once rather than by each of its P x na threads.
 template <int DH>
 __global__ void __launch_bounds__(256) bt_attn_kernel(const BtArgs a) {
+  extern __shared__ uint4 bt_kv_s4[];
   const BtDims& d = a.d;
   const int g = blockIdx.y;
-  const int64_t id = int64_t(blockIdx.x) * blockDim.x + threadIdx.x;
+  const int64_t id0 = int64_t(blockIdx.x) * blockDim.x;
+  const int64_t id = id0 + threadIdx.x;
   const int64_t n_rows = int64_t(d.B) * d.S * d.P;
-  if (id >= n_rows * d.na) return;
+  const int64_t n_thr = n_rows * d.na;
+  const int64_t tok0 = (id0 / d.na) / d.P;
+  {
+    const int64_t last = (id0 + blockDim.x < n_thr ? id0 + blockDim.x : n_thr) - 1;
+    const int64_t tok1 = (last / d.na) / d.P;
+    const int64_t n16 = (tok1 - tok0 + 1) * d.P * 2 * d.d / 8;
+    const uint4* src = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(a.kv) +
+                                                      (int64_t(g) * d.R + tok0 * d.P) * 2 * d.d);
+    for (int64_t i = threadIdx.x; i < n16; i += blockDim.x) bt_kv_s4[i] = src[i];
+  }
+  __syncthreads();
+  if (id >= n_thr) return;
   const int h = static_cast<int>(id % d.na);
   const int64_t row = id / d.na;
   const int64_t tok = row / d.P;
@@ -1028,9 +1044,8 @@ __global__ void __launch_bounds__(256) bt_attn_kernel(const BtArgs a) {
   if (s >= seq_len_of(a, b)) return;
   const int P = d.P, D = d.d;
   const float scale = rsqrtf(static_cast<float>(DH));
-  const int64_t base = int64_t(g) * d.R + tok * P;   // first row of the token
   const uint16_t* qr = static_cast<const uint16_t*>(a.q) + (int64_t(g) * d.R + row) * D + h * DH;
-  const uint16_t* kvb = static_cast<const uint16_t*>(a.kv) + base * 2 * D + h * DH;
+  const uint16_t* kvb = reinterpret_cast<const uint16_t*>(bt_kv_s4) + (tok - tok0) * P * 2 * D + h * DH;
   uint16_t* orow = static_cast<uint16_t*>(a.o) + (int64_t(g) * d.R + row) * D + h * DH;
   float qv[DH];
   const uint4* q4 = reinterpret_cast<const uint4*>(qr);
@@ -1133,11 +1148,15 @@ cudaError_t launch_bt_attn(const BtArgs& a, cudaStream_t st) {
   const BtDims& d = a.d;
   const int64_t threads = int64_t(d.B) * d.S * d.P * d.na;
   dim3 grid(static_cast<unsigned>((threads + 255) / 256), d.G);
-  switch (d.d / d.na) {
-    case 16: bt_attn_kernel<16><<<grid, 256, 0, st>>>(a); break;
-    case 32: bt_attn_kernel<32><<<grid, 256, 0, st>>>(a); break;
-    default: bt_attn_kernel<64><<<grid, 256, 0, st>>>(a); break;
+  // 256 consecutive threads span at most 256 / na + 2 rows, so at most that / P + 2 tokens
+  const int max_tok = (256 / d.na + 2) / d.P + 2;
+  const int smem = max_tok * d.P * 2 * d.d * 2;
+  auto kern = d.d / d.na == 16 ? bt_attn_kernel<16> : d.d / d.na == 32 ? bt_attn_kernel<32> : bt_attn_kernel<64>;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
   }
+  kern<<<grid, 256, smem, st>>>(a);
   return cudaGetLastError();
 }
 

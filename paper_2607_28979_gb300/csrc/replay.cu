@@ -43,15 +43,17 @@
 //                           warp 0  TMA: the Q tile once, then K and V^T tiles
 //                                   (V transposed per layer by replay_vt_kernel so
 //                                   both MMAs read K-major operands) into 2 stages;
-//                           warp 1  S = Q K^T (M=128, N=128 keys) and, one tile
-//                                   later, PV = P V (M=128, N=d), into double-
-//                                   buffered TMEM;
+//                           warp 1  S = Q K^T (M=128, N=128 keys) into double-
+//                                   buffered TMEM and, one tile later, O += P V
+//                                   (M=128, N=d) accumulated in TMEM;
 //                           warps 4..7  one query row per thread: the scaled,
 //                                   masked row of S from TMEM, its running max and
 //                                   sum (base-2 exponentials), P as bf16 into a
-//                                   128B-swizzled SMEM tile for the second MMA, and
-//                                   the output row in registers, rescaled by
-//                                   exp2(m_old - m_new) before each PV is added.
+//                                   128B-swizzled SMEM tile for the second MMA. The
+//                                   running max rises only when a tile's max exceeds
+//                                   it by more than 2^8, and only then are the sum
+//                                   and the O row in TMEM rescaled; O is read from
+//                                   TMEM once, at the end.
 //                         Every wait is bounded; on a timeout the roles unwind,
 //                         copies and MMAs in flight are drained and TMEM is freed.
 #include <cuda_bf16.h>

@@ -158,6 +158,8 @@ KERNEL_SOURCES = {
     "replay_attn_sparse": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
     "replay_select": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
     "replay_fmha_full": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
+    # backbone translators (all kernels of bt.cu)
+    "bt_ffn_fused": ["bt.cu", "bt_internal.h", "mot_internal.h", "ptx.cuh"],
 }
 
 

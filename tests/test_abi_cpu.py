@@ -119,3 +119,49 @@ def test_routing_calls_reject_null_handles():
     assert M._lib.mot_get_routing(None, ctypes.byref(v)) == M.MOT_ERR_INVALID_ARG
     buf = np.zeros(4, dtype=np.int32)
     assert M._lib.mot_get_expert_counts(None, buf.ctypes.data, 4, None) == M.MOT_ERR_INVALID_ARG
+
+
+RP_GOOD = dict(q_heads=12, kv_heads=2, head_dim=128, max_batch=4, max_seq=4096, top_s=128, n_full=2)
+
+
+@pytest.mark.parametrize("change, expect", [
+    (dict(q_heads=0), "MOT_ERR_INVALID_ARG"),
+    (dict(kv_heads=0), "MOT_ERR_INVALID_ARG"),
+    (dict(kv_heads=5), "MOT_ERR_INVALID_ARG"),      # 12 % 5: not a GQA grouping
+    (dict(top_s=0), "MOT_ERR_INVALID_ARG"),
+    (dict(n_full=-1), "MOT_ERR_INVALID_ARG"),
+    (dict(max_seq=0), "MOT_ERR_INVALID_ARG"),
+    (dict(head_dim=96), "MOT_ERR_UNSUPPORTED"),     # kernels take d in {64, 128}
+    (dict(q_heads=20, kv_heads=2), "MOT_ERR_UNSUPPORTED"),   # group of 10: no instantiated kernel
+])
+def test_replay_create_rejects_bad_config_before_cuda(change, expect):
+    kw = dict(RP_GOOD)
+    kw.update(change)
+    cfg = M.mot_replay_config(*[kw[k] for k in ("q_heads", "kv_heads", "head_dim", "max_batch",
+                                                "max_seq", "top_s", "n_full")])
+    out = ctypes.c_void_p(1)
+    assert M._lib.mot_create_replay(ctypes.byref(cfg), ctypes.byref(out)) == getattr(M, expect)
+    assert not out.value   # no handle on failure
+
+
+def test_backbone_create_rejects_bad_window_before_cuda():
+    import synth
+    wl = synth.WORKLOADS["bt_gpt2s_opt125m"]
+    cfg, bt = M.bt_config_from(wl)
+    out = ctypes.c_void_p(1)
+    for field, value in (("win_len", 0), ("win_start", -1), ("win_start", wl.n_layers_tgt),
+                         ("heads", 0), ("heads", 5)):   # width 128 not a multiple of 5 heads
+        bad = M.mot_bt_config(*[getattr(bt, f) for f, _ in M.mot_bt_config._fields_])
+        setattr(bad, field, value)
+        assert M._lib.mot_create_bt(ctypes.byref(cfg), ctypes.byref(bad),
+                                    ctypes.byref(out)) == M.MOT_ERR_INVALID_ARG, field
+        assert not out.value
+    assert M._lib.mot_create_bt(None, ctypes.byref(bt), ctypes.byref(out)) == M.MOT_ERR_INVALID_ARG
+
+
+def test_replay_backbone_and_debug_calls_reject_null_handles():
+    L = M._lib
+    assert L.mot_replay_attention(None, 0, None, None, None, None, None, 0, None, None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_replay_select(None, None, None, 0, None, None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_translate_bt(None, None, None, None, 0, None, None, None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_debug_set(None, 0, 0) == M.MOT_ERR_INVALID_ARG

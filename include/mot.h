@@ -364,12 +364,14 @@ mot_status mot_translate_bt(mot_handle h, const void* src_k, const void* src_v,
  * j <= u is read; guide may be NULL for full layers). Rows u >= seq_lens[b] of
  * out are not written. seq_lens: device int32[batch], clamped to [0, max_seq].
  * Requires head_dim in {64, 128}, q_heads / kv_heads in 1..8, 12 or 16, top_s <= 4096,
- * max_seq <= 65536 (else MOT_ERR_UNSUPPORTED). Asynchronous on `stream`.
+ * max_seq <= 65536 (else MOT_ERR_UNSUPPORTED). Asynchronous on `stream`. Guided
+ * layers with head_dim 128 and top_s <= 128 run on the tensor cores, full
+ * layers with max_seq % 8 == 0 too; other shapes take the SIMT kernels.
  *
  * mot_replay_select writes the selection alone: sel [max_batch][max_seq][top_s]
  * int32, the row's positions ascending, then -1 (rows u >= seq_lens[b] are not
  * written). A replay handle accepts only these two calls and the profiling,
- * launch-count and destroy calls.
+ * launch-count, device-status, test-hook (mot_debug_set) and destroy calls.
  */
 typedef struct {
   int32_t q_heads, kv_heads, head_dim;

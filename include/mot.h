@@ -161,9 +161,14 @@ const char* mot_status_string(mot_status s);
  *   256-rounded(batch * S_pad * E * 4) + batch * S_pad * E * H * 4 bytes,
  *   S_pad = max_seq rounded up to 64,
  * and returns MOT_ERR_UNSUPPORTED, before any CUDA call, when that exceeds the
- * array. The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress, with that device current); make that first call
- * before any stream capture. All calls share the array and it keeps the last
+ * array (or when max_seq > INT32_MAX - 63). dst_k and dst_v may overlap
+ * neither each other, nor src_k / src_v, nor the weight blob
+ * (MOT_ERR_INVALID_ARG, before any CUDA call). The first call on a device
+ * looks up the array's device address (cudaGetSymbolAddress, with that device
+ * current) and keeps it for the life of the process; make that first call
+ * before any stream capture. The kept address belongs to the device's primary
+ * context (the one the CUDA runtime uses): calls from another context on the
+ * device, or after cudaDeviceReset, are not supported. All calls share the array and it keeps the last
  * call's contents (nothing in it needs to start at zero): calls that overlap
  * on the GPU, on any streams, race with each other. Lengths outside
  * [0, max_seq] are clamped; there is no status word to report them. The

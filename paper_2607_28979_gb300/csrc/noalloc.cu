@@ -204,6 +204,19 @@ __global__ void __launch_bounds__(256) static_translate_kernel(StaticArgs a, int
 std::mutex g_setup_mutex;
 void* g_scratch_ptr[kMaxDevices] = {};
 
+// a * b, saturating at SIZE_MAX (buffer sizes from int32 dimensions).
+size_t mul_sat(size_t a, size_t b) {
+  if (a != 0 && b > SIZE_MAX / a) return SIZE_MAX;
+  return a * b;
+}
+
+bool ranges_overlap(const void* a, size_t na, const void* b, size_t nb) {
+  const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+  const uintptr_t xe = na > UINTPTR_MAX - x ? UINTPTR_MAX : x + na;
+  const uintptr_t ye = nb > UINTPTR_MAX - y ? UINTPTR_MAX : y + nb;
+  return x < ye && y < xe;
+}
+
 }  // namespace
 }  // namespace mot
 
@@ -224,11 +237,45 @@ extern "C" mot_status mot_translate_static(const mot_config* cfg, const void* we
     for (int l = 0; l < c.n_layers_tgt; ++l)
       if (c.layer_map[l] < -1 || c.layer_map[l] >= c.n_layers_src) return MOT_ERR_INVALID_ARG;
   if (c.n_translators > kMaxE || c.max_batch > 4096) return MOT_ERR_UNSUPPORTED;
+  // S_pad (max_seq rounded up to 64) must stay an int32
+  if (c.max_seq > INT32_MAX - (kRows - 1)) return MOT_ERR_UNSUPPORTED;
   if (batch < 0 || batch > c.max_batch || (batch > 0 && !seq_lens)) return MOT_ERR_INVALID_ARG;
   const uintptr_t al = reinterpret_cast<uintptr_t>(weights) | reinterpret_cast<uintptr_t>(src_k) |
                        reinterpret_cast<uintptr_t>(src_v) | reinterpret_cast<uintptr_t>(dst_k) |
                        reinterpret_cast<uintptr_t>(dst_v);
   if (al & 15u) return MOT_ERR_INVALID_ARG;
+
+  // The outputs may overlap neither each other, nor the caches they read, nor
+  // the weights: target layer l would overwrite a source layer that a later
+  // target layer still reads (the depth-ratio map reuses source layers).
+  const size_t es = c.dtype == MOT_BF16 ? 2 : 4;
+  int n_translated = 0;
+  for (int l = 0; l < c.n_layers_tgt; ++l)
+    if (!c.layer_map || c.layer_map[l] >= 0) ++n_translated;
+  const size_t src_b = mul_sat(mul_sat(mul_sat(mul_sat(mul_sat(c.n_layers_src, c.max_batch),
+                                                       c.src_kv_heads), c.max_seq),
+                                       c.src_head_dim), es);
+  const size_t dst_b = mul_sat(mul_sat(mul_sat(mul_sat(mul_sat(c.n_layers_tgt, c.max_batch),
+                                                       c.tgt_kv_heads), c.max_seq),
+                                       c.tgt_head_dim), es);
+  const size_t Ds_ = mul_sat(c.src_kv_heads, c.src_head_dim);
+  const size_t Dt_ = mul_sat(c.tgt_kv_heads, c.tgt_head_dim);
+  size_t per_exp = mul_sat(c.hidden, Ds_);
+  per_exp = per_exp + c.hidden;
+  per_exp = per_exp + mul_sat(Dt_, c.hidden) + Dt_;
+  const size_t group_elems = mul_sat(c.n_translators, Ds_) + c.n_translators +
+                             mul_sat(c.n_translators, per_exp);
+  const size_t w_b = mul_sat(mul_sat(2 * size_t(n_translated), group_elems), es);
+  if (ranges_overlap(dst_k, dst_b, dst_v, dst_b) || ranges_overlap(dst_k, dst_b, src_k, src_b) ||
+      ranges_overlap(dst_k, dst_b, src_v, src_b) || ranges_overlap(dst_v, dst_b, src_k, src_b) ||
+      ranges_overlap(dst_v, dst_b, src_v, src_b) || ranges_overlap(dst_k, dst_b, weights, w_b) ||
+      ranges_overlap(dst_v, dst_b, weights, w_b))
+    return MOT_ERR_INVALID_ARG;
+
+  // the kernels index with int32 widths
+  if (Ds_ > INT32_MAX || Dt_ > INT32_MAX ||
+      mul_sat(c.n_translators, c.hidden) > size_t(INT32_MAX))
+    return MOT_ERR_UNSUPPORTED;
 
   StaticArgs a{};
   a.L_s = c.n_layers_src; a.H_s = c.src_kv_heads; a.d_s = c.src_head_dim;
@@ -238,9 +285,9 @@ extern "C" mot_status mot_translate_static(const mot_config* cfg, const void* we
   a.Ds = a.H_s * a.d_s; a.Dt = a.H_t * a.d_t; a.EH = a.E * a.H;
   a.s_pad = (a.S + kRows - 1) / kRows * kRows;
   // scratch: gate rows then hidden rows, both fp32, for every (batch entry, position)
-  const size_t rows = size_t(batch) * a.s_pad;
+  const size_t rows = size_t(batch) * size_t(a.s_pad);
   const size_t gate_bytes = (rows * a.E * 4 + 255) / 256 * 256;
-  const size_t need = gate_bytes + rows * size_t(a.EH) * 4;
+  const size_t need = gate_bytes + mul_sat(mul_sat(rows, size_t(a.EH)), 4);
   if (need > kStaticScratchBytes) return MOT_ERR_UNSUPPORTED;   // scratch too small
   if (batch == 0) return MOT_OK;
 
@@ -267,7 +314,6 @@ extern "C" mot_status mot_translate_static(const mot_config* cfg, const void* we
   a.a2 = reinterpret_cast<float*>(static_cast<unsigned char*>(scratch) + gate_bytes);
   a.seq_lens = seq_lens;
 
-  const size_t es = c.dtype == MOT_BF16 ? 2 : 4;
   const size_t gsz = size_t(a.E) * a.Ds + a.E +
                      size_t(a.E) * (size_t(a.H) * a.Ds + a.H + size_t(a.Dt) * a.H + a.Dt);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);

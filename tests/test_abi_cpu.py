@@ -4,6 +4,8 @@ import ctypes
 import os
 import re
 
+import numpy as np
+
 import pytest
 
 from paper_2607_28979_gb300 import build as mot_build
@@ -165,3 +167,42 @@ def test_replay_backbone_and_debug_calls_reject_null_handles():
     assert L.mot_replay_select(None, None, None, 0, None, None) == M.MOT_ERR_INVALID_ARG
     assert L.mot_translate_bt(None, None, None, None, 0, None, None, None) == M.MOT_ERR_INVALID_ARG
     assert L.mot_debug_set(None, 0, 0) == M.MOT_ERR_INVALID_ARG
+
+
+def _static_call(cfg, weights, src_k, src_v, dst_k, dst_v, lens=0x9000, batch=1):
+    """mot_translate_static with raw addresses (the checks below run before any
+    CUDA call, so nothing is dereferenced)."""
+    return M._lib.mot_translate_static(ctypes.byref(cfg), weights, src_k, src_v, lens, batch,
+                                       dst_k, dst_v, None)
+
+
+def test_static_entry_point_rejects_overlapping_outputs_before_cuda():
+    import synth
+    wl = synth.Workload("alias", 3, 2, 64, 4, 2, 128, 2, 256, 2, 64, "bf16", (64, 9))
+    cfg = M.config_from(wl)
+    sb = int(np.prod(wl.src_shape())) * 2
+    db = int(np.prod(wl.dst_shape())) * 2
+    wb = wl.blob_elems() * 2
+    base = 1 << 40   # disjoint 16-byte-aligned address ranges
+    w, sk, sv = base, base + (1 << 32), base + (2 << 32)
+    dk, dv = base + (3 << 32), base + (4 << 32)
+    # the same call without overlaps gets past these checks (no GPU: a CUDA error)
+    ok = _static_call(cfg, w, sk, sv, dk, dv)
+    assert ok != M.MOT_ERR_INVALID_ARG
+    for args in ((w, sk, sv, sk, dv),                    # dst_k is src_k
+                 (w, sk, sv, dk, sv),                    # dst_v is src_v
+                 (w, sk, sv, sv + sb - 16, dv),          # dst_k runs into the tail of src_v
+                 (w, sk, sv, dk, dk + db - 16),          # dst_v overlaps dst_k
+                 (w, sk, sv, w + wb - 16, dv),           # dst_k over the weights' tail
+                 (dv - wb + 16, sk, sv, dk, dv)):        # the weights' tail under dst_v
+        assert _static_call(cfg, *args) == M.MOT_ERR_INVALID_ARG, args
+
+
+def test_static_entry_point_rejects_huge_lengths_before_cuda():
+    import synth
+    wl = synth.Workload("huge", 2, 2, 64, 2, 2, 128, 2, 256, 1, 2**31 - 40, "bf16", (64,))
+    cfg = M.config_from(wl)
+    base = 1 << 44
+    st = _static_call(cfg, base, base + (1 << 40), base + (2 << 40), base + (3 << 40),
+                      base + (4 << 40))
+    assert st == M.MOT_ERR_UNSUPPORTED

@@ -4,11 +4,20 @@
 Metric: source-context tokens translated per second into the full target
 cache (sum of seq_lens per mot_translate call, all translated layers, K and V).
 
-One step = one mot_translate call over one synthetic batch of the workload
-(default: the GPT-2-small -> OPT-125m-shaped pair, 12 layers, 12x64 heads,
-E=4 translators 768->1536->768, batch 8 x 1024 tokens), with inputs resident
-in HBM. Every step reads 1.06 GB (source caches, weights, target caches), far
-more than the 129 MB L2, so no flush is needed between steps.
+One step = one mot_translate call over one synthetic batch of the workload,
+with inputs resident in HBM. The default workload is the largest bf16 model
+pair: Qwen2.5-7B-shaped -> Qwen2.5-7B-shaped caches (28 layers, 4 KV heads of
+128), E=4 translators 512->2048->512, a ragged batch of 4 sequences of
+32768/16384/8192/4096 tokens (61,440 tokens per step). Every step reads and
+writes 8 GB (source caches, weights, target caches), far more than the
+129 MB L2, so no flush is needed between steps. The same line carries, under
+``per_config``, the device-resident timing of the other three bf16 model pairs
+(GPT-2-small -> OPT-125m, Qwen2.5-0.5B -> 1.5B, GPT-2-medium -> Qwen2.5-7B),
+each with its step roofline and its dominant kernel's fraction.
+
+Roofline peaks: the burst bf16 figure applies when the run's own clock record
+shows neither the power cap nor a lowered SM clock under load; otherwise the
+sustained figure. Both fractions are printed.
 
   python bench.py [--gpus N --steps K --warmup W] [--impl mot|reference]
 
@@ -38,7 +47,7 @@ import synth   # noqa: E402
 
 METRIC = "source-context tokens translated/sec into full target cache (1×GB300); % of roofline"
 UNIT = "tokens/s"
-DEFAULT_WORKLOAD = "gpt2s_opt125m"
+DEFAULT_WORKLOAD = "qwen7_long"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -365,6 +374,184 @@ def run_reference(args, wl):
     return 0
 
 
+# Per-launch FLOPs of each translation kernel, from the step's algorithmic split.
+def _per_launch_flops(alg):
+    return {"umma_fused_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
+            "umma2_onchip_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
+            "umma2_gemm1_gelu_gate": alg["flops_gemm1"],
+            "umma2_gemm2_combine_store": alg["flops_gemm2"],
+            "umma2_sparse_gemm1": alg["flops_gemm1"],
+            "umma2_sparse_gemm2": alg["flops_gemm2"],
+            "umma2_proj": alg["flops_proj"],
+            "umma_gemm1_gelu_gate": alg["flops_gemm1"],
+            "simt_gemm1_gelu_gate": alg["flops_gemm1"],
+            "umma_gemm2_combine_store": alg["flops_gemm2"],
+            "simt_gemm2_combine_store": alg["flops_gemm2"]}
+
+
+def choose_tensor_peak(peaks, clocks):
+    """The bf16 peak that applies to this run, from its own clock record: the
+    burst figure when no sample showed the power cap and the SM clock under load
+    stayed at its maximum (a short timed region), else the sustained figure
+    (the GPU settled at its power limit). Returns (peak TFLOP/s, kind, why)."""
+    burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    sustained = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    reasons = (clocks or {}).get("reasons") or []
+    sm, smax = (clocks or {}).get("sm_mhz"), (clocks or {}).get("sm_max_mhz")
+    if "sw_power_cap" in reasons:
+        return sustained, "sustained", "sw_power_cap seen during the timed region"
+    if sm is None or smax is None:
+        return sustained, "sustained", "no clock record"
+    if sm < 0.97 * smax:
+        return sustained, "sustained", f"SM clock under load {sm:.0f} of {smax:.0f} MHz"
+    return burst, "burst", f"SM clock under load {sm:.0f} of {smax:.0f} MHz, no power cap"
+
+
+def kernel_roofline(wl, alg, kstats, steps, peaks, peak_kind, clocks):
+    """Roofline of the dominant kernel (largest share of device time): its
+    algorithmic work per launch over its mean CUDA-event launch time."""
+    name, (n_launch, tot_ms) = max(kstats.items(), key=lambda kv: kv[1][1])
+    launches_per_step = max(1, n_launch // steps)
+    avg_s = tot_ms / n_launch / 1000.0
+    peak_t, which, why = choose_tensor_peak(peaks, clocks)
+    burst = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    sustained = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    if wl.is_bt and name in alg["per_launch"]:
+        # the slower of the kernel's FLOPs at tensor peak and its bytes at HBM peak
+        fl, by = alg["per_launch"][name], alg["bytes_per_launch"][name]
+        t_t, t_b = fl / (peak_t * 1e12), by / (peaks["hbm_gbs"] * 1e9)
+        if t_b >= t_t:
+            achieved = by / avg_s / 1e9
+            return {"kernel": name, "bound": "hbm", "achieved": round(achieved, 1),
+                    "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                    "frac": round(achieved / peaks["hbm_gbs"], 4),
+                    "peak_kind": f"HBM copy, {peak_kind}",
+                    "traffic": recorded_traffic(name, wl.name),
+                    "algorithmic_per_launch": by, "flops_per_launch": fl,
+                    "avg_launch_ms": tot_ms / n_launch}
+        work = fl
+    else:
+        plf = _per_launch_flops(alg) if not wl.is_bt else {}
+        if name not in plf:
+            return {"kernel": name, "bound": "hbm", "achieved": None, "peak": peaks["hbm_gbs"],
+                    "unit": "GB/s", "frac": None, "traffic": None}
+        work = plf[name] / launches_per_step
+    achieved = work / avg_s / 1e12
+    return {"kernel": name, "bound": "tensor", "achieved": round(achieved, 1),
+            "peak": peak_t, "unit": "TFLOP/s", "frac": round(achieved / peak_t, 4),
+            "peak_kind": f"bf16 dense {which}, {peak_kind} ({why})",
+            "frac_of_burst": round(achieved / burst, 4),
+            "frac_of_sustained": round(achieved / sustained, 4),
+            "traffic": recorded_traffic(name, wl.name),
+            "algorithmic_per_launch": work, "avg_launch_ms": tot_ms / n_launch}
+
+
+def step_roofline(alg, t_step_ms, peaks, peak_kind, clocks):
+    """The whole step against max(FLOPs at the tensor peak, bytes at the HBM peak),
+    with the peak this run's clocks call for, and both figures."""
+    peak_t, which, _ = choose_tensor_peak(peaks, clocks)
+    out = {"flops": alg["flops"], "bytes": alg["bytes"]}
+    for tag, p in (("", peak_t), ("_burst", peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])),
+                   ("_sustained", peaks.get("bf16_tflops_sustained",
+                                            FALLBACK_PEAKS["bf16_tflops_sustained"]))):
+        t_roof = max(alg["flops"] / (p * 1e12), alg["bytes"] / (peaks["hbm_gbs"] * 1e9))
+        out["roofline_ms" + tag] = 1000 * t_roof
+        out["frac" + tag] = round(1000 * t_roof / t_step_ms, 4)
+    out["peaks"] = (f"bf16 {peak_t} TFLOP/s ({which}), HBM {peaks['hbm_gbs']} GB/s ({peak_kind})")
+    return out
+
+
+class _Setup:
+    """One handle with its weights and device inputs/outputs for a workload."""
+
+    def __init__(self, M, torch, wl, args):
+        self.wl = wl
+        self.sk_h, self.blob = synth.gen_cache(wl, 0), synth.gen_weights(wl)
+        self.sv_h = self.sk_h if wl.is_h else synth.gen_cache(wl, 1)   # MoT-h: one activation
+        if wl.is_bt:
+            self.h = M.mot_create_bt(*M.bt_config_from(wl))
+        elif wl.is_h:
+            self.h = M.mot_create_h(M.h_config_from(wl))
+        else:
+            self.h = M.mot_create(M.config_from(wl))
+        M.mot_load_weights(self.h, self.blob)
+        self.path = M.mot_get_path(self.h)
+        names = {0: "split", 1: "fused", 2: "pair", 3: "onchip"}
+        if args.schedule != "auto" and not wl.is_bt:
+            M.mot_set_schedule(self.h, {v: k for k, v in names.items()}[args.schedule])
+        sched = names[M.mot_get_schedule(self.h)]
+        if M.mot_get_routing(self.h) == M.ROUTING_SPARSE:
+            sched = "routed (Top-K token buckets)"
+        if wl.is_bt:
+            sched = "backbone scan (7 launches per window slot)"
+        self.schedule = sched
+        self.bf = wl.dtype == "bf16"
+        tdt = torch.bfloat16 if self.bf else torch.float32
+
+        def dev(a):
+            t = torch.from_numpy(a.view(np.int16) if self.bf else a).cuda()
+            return t.view(torch.bfloat16) if self.bf else t
+        self.sk, self.sv = dev(self.sk_h), dev(self.sv_h)
+        self.dk = torch.zeros(wl.dst_shape(), dtype=tdt, device="cuda")
+        self.dv = torch.zeros(wl.dst_shape(), dtype=tdt, device="cuda")
+        self.lens = torch.tensor(wl.seq_lens, dtype=torch.int32, device="cuda")
+        self.stream = torch.cuda.Stream()
+        self.M = M
+
+    def step(self):
+        M, wl, B = self.M, self.wl, self.wl.batch
+        if wl.is_bt:
+            M.mot_translate_bt(self.h, self.sk, self.sv, self.lens, B, self.dk, self.dv, self.stream)
+        elif wl.is_h:
+            M.mot_translate_h(self.h, self.sk, self.lens, B, self.dk, self.dv, self.stream)
+        else:
+            M.mot_translate(self.h, self.sk, self.sv, self.lens, B, self.dk, self.dv, self.stream)
+
+
+def time_device(M, torch, S, args, world, rank, local):
+    """W warm-up steps, then K timed steps between barriers and synchronisations,
+    CUDA events on the launching stream, per-kernel events and nvidia-smi clocks
+    sampled during the timed region. Returns (ms per step, kernel stats, launches,
+    clocks)."""
+    import torch.distributed as dist
+    with torch.cuda.stream(S.stream):
+        for _ in range(args.warmup):
+            S.step()
+    S.stream.synchronize()
+    if M.mot_get_device_status(S.h, S.stream) != M.MOT_OK:
+        raise SystemExit(f"{S.wl.name}: device status not OK after warm-up")
+    sampler = ClockSampler(local) if rank == 0 else None
+    if sampler:
+        sampler.start()
+    M.mot_profile_enable(S.h, True)
+    M.mot_profile_read(S.h)
+    launches0 = M.mot_get_launch_count(S.h)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0.record(S.stream)
+    for _ in range(args.steps):
+        S.step()
+    e1.record(S.stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    elapsed_ms = e0.elapsed_time(e1)
+    launches = M.mot_get_launch_count(S.h) - launches0
+    kstats = M.mot_profile_read(S.h)
+    M.mot_profile_enable(S.h, False)
+    clocks = sampler.stop() if sampler else None
+    status = M.mot_get_device_status(S.h, S.stream)
+    if status != M.MOT_OK:
+        raise SystemExit(f"{S.wl.name}: device status {M.mot_status_string(status)}")
+    return elapsed_ms / args.steps, kstats, launches, clocks
+
+
+# The bf16 model pairs reported beside the headline workload in one line.
+PER_CONFIG = ["gpt2s_opt125m", "qwen05_qwen15", "gpt2m_qwen7"]
+
+
 def run_mot(args, wl):
     world, rank, local = dist_setup(args.gpus)
     import torch
@@ -379,77 +566,10 @@ def run_mot(args, wl):
         dist.barrier()
     import paper_2607_28979_gb300.mot as M
 
-    sk_h, blob = synth.gen_cache(wl, 0), synth.gen_weights(wl)
-    sv_h = sk_h if wl.is_h else synth.gen_cache(wl, 1)   # MoT-h: one activation tensor
-    if wl.is_bt:
-        h = M.mot_create_bt(*M.bt_config_from(wl))
-    elif wl.is_h:
-        h = M.mot_create_h(M.h_config_from(wl))
-    else:
-        h = M.mot_create(M.config_from(wl))
-    M.mot_load_weights(h, blob)
-    path = M.mot_get_path(h)
-    names = {0: "split", 1: "fused", 2: "pair", 3: "onchip"}
-    if args.schedule != "auto" and not wl.is_bt:
-        M.mot_set_schedule(h, {v: k for k, v in names.items()}[args.schedule])
-    schedule = names[M.mot_get_schedule(h)]
-    if M.mot_get_routing(h) == M.ROUTING_SPARSE:
-        schedule = "routed (Top-K token buckets)"
-    if wl.is_bt:
-        schedule = "backbone scan (8 launches per window slot)"
-    bf = wl.dtype == "bf16"
-    tdt = torch.bfloat16 if bf else torch.float32
-
-    def dev(a):
-        t = torch.from_numpy(a.view(np.int16) if bf else a).cuda()
-        return t.view(torch.bfloat16) if bf else t
-    sk, sv = dev(sk_h), dev(sv_h)
-    dk = torch.zeros(wl.dst_shape(), dtype=tdt, device="cuda")
-    dv = torch.zeros(wl.dst_shape(), dtype=tdt, device="cuda")
-    lens = torch.tensor(wl.seq_lens, dtype=torch.int32, device="cuda")
-    stream = torch.cuda.Stream()
-    B = wl.batch
-
-    def step():
-        if wl.is_bt:
-            M.mot_translate_bt(h, sk, sv, lens, B, dk, dv, stream)
-        elif wl.is_h:
-            M.mot_translate_h(h, sk, lens, B, dk, dv, stream)
-        else:
-            M.mot_translate(h, sk, sv, lens, B, dk, dv, stream)
-
-    with torch.cuda.stream(stream):
-        for _ in range(args.warmup):
-            step()
-    stream.synchronize()
-    if M.mot_get_device_status(h, stream) != M.MOT_OK:
-        raise SystemExit("device status not OK after warm-up")
-
-    sampler = ClockSampler(local) if rank == 0 else None
-    if sampler:
-        sampler.start()
-    M.mot_profile_enable(h, True)
-    M.mot_profile_read(h)
-    launches0 = M.mot_get_launch_count(h)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    if world > 1:
-        dist.barrier()
-    torch.cuda.synchronize()
-    e0.record(stream)
-    for _ in range(args.steps):
-        step()
-    e1.record(stream)
-    torch.cuda.synchronize()
-    if world > 1:
-        dist.barrier()
-    elapsed_ms = e0.elapsed_time(e1)
-    launches = M.mot_get_launch_count(h) - launches0
-    kstats = M.mot_profile_read(h)
-    M.mot_profile_enable(h, False)
-    clocks = sampler.stop() if sampler else None
-    status = M.mot_get_device_status(h, stream)
-    if status != M.MOT_OK:
-        raise SystemExit(f"device status {M.mot_status_string(status)}")
+    S = _Setup(M, torch, wl, args)
+    h, sk, sv, dk, dv, lens, stream = S.h, S.sk, S.sv, S.dk, S.dv, S.lens, S.stream
+    sk_h, sv_h, blob, bf, B = S.sk_h, S.sv_h, S.blob, S.bf, wl.batch
+    t_step, kstats, launches, clocks = time_device(M, torch, S, args, world, rank, local)
 
     # ---- end to end through the host-buffer entry point (pinned memory)
     hk = torch.from_numpy(sk_h.view(np.int16) if bf else sk_h).pin_memory()
@@ -511,72 +631,57 @@ def run_mot(args, wl):
         d2h = 2 * tl * wl.tokens * wl.d_tgt * es
         e2e_api = "mot_translate_host (pinned host buffers)"
 
+    # ---- the host link alone: the same byte counts, pinned host -> device and
+    # device -> pinned host at once on two streams (no translation)
+    link_ms = _host_link_ms(torch, hk, hv, ok, ov, sk, sv, dk, dv, h2d, d2h, reps=3)
+
     # ---- aggregate over ranks: max time
-    t_step, e2e_s = reduce_max([elapsed_ms / args.steps, e2e_s], world, "cuda")
+    t_step, e2e_s = reduce_max([t_step, e2e_s], world, "cuda")
     tokens = wl.tokens
     value = aggregate_throughput(tokens, world, t_step / 1000.0)
     e2e_value = aggregate_throughput(tokens * e2e_steps, world, e2e_s)
+    e2e_ms = 1000 * e2e_s / e2e_steps
+
+    alg = algorithmic(wl, M.mot_get_layer_map(h))
+    peaks, peak_kind = load_peaks()
+    roof = kernel_roofline(wl, alg, kstats, args.steps, peaks, peak_kind, clocks) if rank == 0 else None
+    path_str = ("tcgen05 " + S.schedule) if S.path == 1 else "simt"
+    M.mot_destroy(h)
+    del S, sk, sv, dk, dv, hk, hv, ok, ov
+    torch.cuda.empty_cache()
+
+    # ---- the other bf16 model pairs, device-resident, in the same run
+    per_config = None
+    if args.per_config:
+        per_config = {}
+        for name in PER_CONFIG:
+            if name == wl.name:
+                continue
+            w2 = synth.WORKLOADS[name]
+            S2 = _Setup(M, torch, w2, args)
+            t2, k2, l2, c2 = time_device(M, torch, S2, args, world, rank, local)
+            t2 = reduce_max([t2], world, "cuda")[0]
+            if rank == 0:
+                a2 = algorithmic(w2, M.mot_get_layer_map(S2.h))
+                r2 = kernel_roofline(w2, a2, k2, args.steps, peaks, peak_kind, c2)
+                sr = step_roofline(a2, t2, peaks, peak_kind, c2)
+                per_config[name] = {
+                    "workload": workload_desc(w2), "ms_per_step": t2,
+                    "tokens_per_s": aggregate_throughput(w2.tokens, world, t2 / 1000.0),
+                    "path": ("tcgen05 " + S2.schedule) if S2.path == 1 else "simt",
+                    "step_roofline": sr,
+                    "dominant_kernel": {k: r2.get(k) for k in
+                                        ("kernel", "achieved", "unit", "peak", "frac",
+                                         "frac_of_burst", "frac_of_sustained",
+                                         "avg_launch_ms")},
+                    "kernels": {k: {"launches": v[0], "total_ms": round(v[1], 3)}
+                                for k, v in k2.items()},
+                    "gpu_launches": l2, "clocks": c2}
+            M.mot_destroy(S2.h)
+            del S2
+            torch.cuda.empty_cache()
 
     if rank == 0:
-        alg = algorithmic(wl, M.mot_get_layer_map(h))
-        peaks, peak_kind = load_peaks()
-        # dominant kernel: the largest share of device time
-        name, (n_launch, tot_ms) = max(kstats.items(), key=lambda kv: kv[1][1])
-        if wl.is_bt:
-            per_launch_flops = {}
-        else:
-            per_launch_flops = {"umma_fused_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
-                                "umma2_onchip_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
-                                "umma2_gemm1_gelu_gate": alg["flops_gemm1"],
-                                "umma2_gemm2_combine_store": alg["flops_gemm2"],
-                                "umma2_sparse_gemm1": alg["flops_gemm1"],
-                                "umma2_sparse_gemm2": alg["flops_gemm2"],
-                                "umma2_proj": alg["flops_proj"],
-                                "umma_gemm1_gelu_gate": alg["flops_gemm1"],
-                                "simt_gemm1_gelu_gate": alg["flops_gemm1"],
-                                "umma_gemm2_combine_store": alg["flops_gemm2"],
-                                "simt_gemm2_combine_store": alg["flops_gemm2"]}
-        launches_per_step = max(1, n_launch // args.steps)
-        if wl.is_bt:   # alg holds per-launch figures: scale to a step's launches
-            per_launch_flops = {k: v * launches_per_step for k, v in alg["per_launch"].items()}
-        if wl.is_bt and name in alg["per_launch"]:
-            # the slower of the kernel's FLOPs at tensor peak and its bytes at HBM peak
-            fl, by = alg["per_launch"][name], alg["bytes_per_launch"][name]
-            avg_s = tot_ms / n_launch / 1000.0
-            peak_t = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-            t_t, t_b = fl / (peak_t * 1e12), by / (peaks["hbm_gbs"] * 1e9)
-            if t_b >= t_t:
-                achieved = by / avg_s / 1e9
-                roof = {"kernel": name, "bound": "hbm", "achieved": round(achieved, 1),
-                        "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                        "frac": round(achieved / peaks["hbm_gbs"], 4),
-                        "peak_kind": f"HBM copy, {peak_kind}",
-                        "traffic": recorded_traffic(name, wl.name),
-                        "algorithmic_per_launch": by, "flops_per_launch": fl,
-                        "avg_launch_ms": tot_ms / n_launch}
-            else:
-                achieved = fl / avg_s / 1e12
-                roof = {"kernel": name, "bound": "tensor", "achieved": round(achieved, 1),
-                        "peak": peak_t, "unit": "TFLOP/s", "frac": round(achieved / peak_t, 4),
-                        "peak_kind": f"bf16 dense sustained, {peak_kind}",
-                        "traffic": recorded_traffic(name, wl.name),
-                        "algorithmic_per_launch": fl, "bytes_per_launch": by,
-                        "avg_launch_ms": tot_ms / n_launch}
-        elif name in per_launch_flops:
-            work = per_launch_flops[name] / launches_per_step
-            avg_s = tot_ms / n_launch / 1000.0
-            achieved = work / avg_s / 1e12
-            peak = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-            roof = {"kernel": name, "bound": "tensor", "achieved": round(achieved, 1),
-                    "peak": peak, "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
-                    "peak_kind": f"bf16 dense sustained, {peak_kind}",
-                    "traffic": recorded_traffic(name, wl.name),
-                    "algorithmic_per_launch": work, "avg_launch_ms": tot_ms / n_launch}
-        else:
-            roof = {"kernel": name, "bound": "hbm", "achieved": None, "peak": peaks["hbm_gbs"],
-                    "unit": "GB/s", "frac": None, "traffic": None}
-        # whole-step roofline (the slower of FLOPs at tensor peak and bytes at HBM peak)
-        t_roof = max(alg["flops"] / (peaks["bf16_tflops"] * 1e12), alg["bytes"] / (peaks["hbm_gbs"] * 1e9))
         cpu = None
         if world == 1 and not args.no_cpu_baseline:
             rate, n, dt = cpu_oracle_rate(wl, sk_h, sv_h, blob, budget_s=15.0)
@@ -590,31 +695,69 @@ def run_mot(args, wl):
             "data": "synthetic (seeded SplitMix64/Box-Muller caches, N(0,1/fan_in) weights)",
             "config": {"workload": workload_desc(wl), "tokens_per_step": tokens,
                        "parallelism": "replicas" if world > 1 else "single GPU",
-                       "path": ("tcgen05 " + schedule) if path == 1 else "simt",
+                       "path": path_str,
                        "l2": ("inputs larger than L2 (%.2f GB read+written per step)" % (alg["bytes"] / 1e9)
                               if not wl.is_bt else
                               "each step moves more than L2: %.2f GB of caches and weights plus "
                               "the row workspace (GBs)" % (alg["bytes"] / 1e9))},
             "roofline": roof,
-            "step_roofline": {"flops": alg["flops"], "bytes": alg["bytes"],
-                              "roofline_ms": 1000 * t_roof,
-                              "frac": round(1000 * t_roof / t_step, 4),
-                              "peaks": f"bf16 {peaks['bf16_tflops']} TFLOP/s burst, HBM {peaks['hbm_gbs']} GB/s ({peak_kind})"},
+            "step_roofline": step_roofline(alg, t_step, peaks, peak_kind, clocks),
             "kernels": {k: {"launches": v[0], "total_ms": round(v[1], 3),
                             "share": round(v[1] / sum(x[1] for x in kstats.values()), 4)}
                         for k, v in kstats.items()},
+            "per_config": per_config,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h, "steps": e2e_steps,
-                    "api": e2e_api},
+                    "d2h_bytes_per_step": d2h, "steps": e2e_steps, "api": e2e_api,
+                    "ms_per_step": e2e_ms,
+                    "host_link_gbs": round((h2d + d2h) / (e2e_ms / 1000) / 1e9, 1),
+                    "link_only_ms": link_ms,
+                    "link_only_gbs": round((h2d + d2h) / (link_ms / 1000) / 1e9, 1),
+                    "device_ms": t_step,
+                    "overlap": round(max(link_ms, t_step) / e2e_ms, 3)},
             "gpu_launches": launches,
             "clocks": clocks,
         }
         print(json.dumps(line), flush=True)
-    M.mot_destroy(h)
     if world > 1:
         dist.destroy_process_group()
     return 0
+
+
+def _host_link_ms(torch, hk, hv, ok, ov, sk, sv, dk, dv, h2d, d2h, reps=3):
+    """Milliseconds to move h2d bytes host -> device and d2h bytes device -> host
+    at once (two streams, pinned memory, flat copies): what the host link alone
+    allows per step."""
+    def flat(*ts):
+        return [t.view(torch.int16).reshape(-1) for t in ts]
+    src_h, dst_d = flat(hk, hv), flat(sk, sv)
+    src_d, dst_h = flat(dk, dv), flat(ok, ov)
+
+    def plan(total_bytes, srcs, dsts):
+        out, left = [], total_bytes // 2
+        for s, d in zip(srcs, dsts):
+            n = min(left, s.numel(), d.numel())
+            if n > 0:
+                out.append((s[:n], d[:n]))
+            left -= n
+        return out
+    up, down = plan(h2d, src_h, dst_d), plan(d2h, src_d, dst_h)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+
+    def once():
+        with torch.cuda.stream(s1):
+            for a, b in up:
+                b.copy_(a, non_blocking=True)
+        with torch.cuda.stream(s2):
+            for a, b in down:
+                b.copy_(a, non_blocking=True)
+    once()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(reps):
+        once()
+    torch.cuda.synchronize()
+    return 1000 * (time.perf_counter() - t0) / reps
 
 
 # ---------------------------------------------------------------- replay attention (App. C.4)
@@ -908,6 +1051,10 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD,
                     choices=sorted(synth.WORKLOADS) + sorted(synth.REPLAY_WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--per-config", dest="per_config", action="store_true", default=None,
+                    help="also time the other bf16 model pairs (device-resident) in the same "
+                         "run (default: on for the headline workload)")
+    ap.add_argument("--no-per-config", dest="per_config", action="store_false")
     ap.add_argument("--schedule", choices=["auto", "onchip", "pair", "fused", "split"],
                     default="auto",
                     help="tcgen05 launch schedule: the library's default for the shape, the "
@@ -931,6 +1078,9 @@ def main():
         wl = wl.replace(name=f"{wl.name}_L{args.n_layers}",
                         n_layers_src=min(args.n_layers, wl.n_layers_src),
                         n_layers_tgt=min(args.n_layers, wl.n_layers_tgt))
+    if args.per_config is None:
+        args.per_config = (args.workload == DEFAULT_WORKLOAD and args.top_k == 0
+                           and args.n_layers == 0)
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_mot(args, wl)

@@ -237,6 +237,22 @@ mot_status mot_profile_read(mot_handle h, mot_kernel_stat* out, int32_t cap, int
  */
 mot_status mot_debug_set(mot_handle h, int32_t stall_test, int64_t wait_limit_cycles);
 
+/*
+ * GELU probe (App. C.2: phi = GELU). Evaluates, on the device, the GELU form a
+ * kernel family uses, out[i] = GELU(u[i]) * gate[i], so that a test can
+ * measure it against the exact erf form:
+ *   form 0: the tensor-core MLP epilogue (every schedule): u rounded to fp16,
+ *           the tanh form in packed fp16x2 on the hardware tanh unit, times
+ *           gate (fp16 of gate / 2, doubled in the form), fp16 result;
+ *   form 1: the backbone-translator epilogues: the tanh form in fp32;
+ *   form 2: the SIMT path: the exact erf form with erff, fp32.
+ * u, gate, out: device float[n]. Asynchronous on `stream`. Errors:
+ * MOT_ERR_INVALID_ARG (form outside 0..2, n < 0, NULL buffers with n > 0),
+ * MOT_ERR_CUDA.
+ */
+mot_status mot_debug_gelu(int32_t form, const float* u, const float* gate, int64_t n, float* out,
+                           mot_stream_t stream);
+
 /* Number of kernels this handle has launched since it was created. */
 mot_status mot_get_launch_count(mot_handle h, int64_t* count);
 

@@ -43,6 +43,7 @@
 #include <algorithm>
 
 #include "bt_internal.h"
+#include "gelu.cuh"
 #include "ptx.cuh"
 
 namespace mot {
@@ -60,16 +61,6 @@ constexpr int kBtTmemCols = 512;
 constexpr float kLnEps = 1e-5f;
 constexpr int kBtSmem = kBtStages * kBtStageBytes + 256 + 1024;
 static_assert(kBtSmem <= 232448, "shared memory budget");
-
-// GELU in its tanh form, 0.5 u (1 + tanh(sqrt(2/pi) (u + 0.044715 u^3))), on
-// the hardware tanh unit: within 5e-4 of the erf form over the line (the
-// parity tests bound the whole path), at a fraction of erff's instruction count.
-__device__ __forceinline__ float gelu_tanh(float u) {
-  const float k0 = 0.7978845608028654f, k1 = 0.7978845608028654f * 0.044715f;
-  const float t = tanh_approx(u * fmaf(k1, u * u, k0));
-  const float hu = 0.5f * u;
-  return fmaf(hu, t, hu);
-}
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }

@@ -101,10 +101,7 @@ __device__ __forceinline__ void gelu_cols(const uint32_t (&acc)[32], const uint4
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       const int j = v * 8 + 2 * k;
-      __half2 u = __float22half2_rn(make_float2(__uint_as_float(acc[j]), __uint_as_float(acc[j + 1])));
-      u = __hadd2(u, *reinterpret_cast<const __half2*>(&bw[k]));
-      const __half2 o = gelu_times_h2(u, half_g);
-      pk[4 * v + k] = *reinterpret_cast<const uint32_t*>(&o);
+      pk[4 * v + k] = gelu_gate_pair(acc[j], acc[j + 1], bw[k], half_g);
     }
   }
 }

@@ -8,6 +8,7 @@
 // GELU is the exact erf form; a2 is kept in fp32.
 #include <cuda_bf16.h>
 
+#include "gelu.cuh"
 #include "mot_internal.h"
 
 namespace mot {
@@ -19,10 +20,6 @@ __device__ __forceinline__ float ld_f(const float* p) { return *p; }
 __device__ __forceinline__ float ld_f(const __nv_bfloat16* p) { return __bfloat162float(*p); }
 __device__ __forceinline__ void st_v(float* p, float v) { *p = v; }
 __device__ __forceinline__ void st_v(__nv_bfloat16* p, float v) { *p = __float2bfloat16_rn(v); }
-
-__device__ __forceinline__ float gelu_erf(float u) {
-  return 0.5f * u * (1.f + erff(u * 0.70710678118654752f));
-}
 
 // Grid (2*tiles_max, ceil(EH/64), gp), 256 threads, 4x4 outputs per thread.
 template <typename T>

@@ -14,6 +14,7 @@
 #include <cuda_fp16.h>
 
 #include "mot_internal.h"
+#include "gelu.cuh"
 #include "ptx.cuh"
 
 namespace mot {
@@ -33,28 +34,6 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// GELU(u) * g with the tanh form of GELU on the hardware tanh unit:
-// 0.5 u (1 + tanh(sqrt(2/pi) (u + 0.044715 u^3))). Its largest deviation from
-// the erf form is 4.7e-4 (at |u| = 2.7). fp32 version (for reference and tests).
-__device__ __forceinline__ float gelu_times(float u, float half_g) {
-  const float k0 = 0.7978845608028654f, k1 = 0.7978845608028654f * 0.044715f;
-  const float t = tanh_approx(u * fmaf(k1, u * u, k0));
-  const float hu = u * half_g;
-  return fmaf(hu, t, hu);
-}
-
-// The same on two fp16 lanes at once (HFMA2 + tanh.approx.f16x2): about 2^-11
-// relative rounding per step, finer than the fp16 result it produces.
-__device__ __forceinline__ __half2 gelu_times_h2(__half2 u, __half2 half_g) {
-  const __half2 k0 = __float2half2_rn(0.7978845608028654f);
-  const __half2 k1 = __float2half2_rn(0.7978845608028654f * 0.044715f);
-  const __half2 arg = __hmul2(u, __hfma2(__hmul2(u, u), k1, k0));
-  const uint32_t tb = tanh_approx_f16x2(*reinterpret_cast<const uint32_t*>(&arg));
-  const __half2 t = *reinterpret_cast<const __half2*>(&tb);
-  const __half2 hu = __hmul2(u, half_g);
-  return __hfma2(hu, t, hu);
-}
-
 // GEMM1 epilogue of one warp: rows 32*q + lane of the tile, columns
 // [col_begin, col_begin + 64 * n_chunks). `tbase` is the accumulator's TMEM
 // address including the warp's lane quarter; `tile` this warp's 4 KB of
@@ -71,10 +50,7 @@ __device__ __forceinline__ void gemm1_sub(const uint32_t (&r)[32], const uint4* 
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       const int j = v * 8 + 2 * k;
-      __half2 u = __float22half2_rn(make_float2(__uint_as_float(r[j]), __uint_as_float(r[j + 1])));
-      u = __hadd2(u, *reinterpret_cast<const __half2*>(&bw[k]));
-      const __half2 o = gelu_times_h2(u, half_g);
-      pk[4 * v + k] = *reinterpret_cast<const uint32_t*>(&o);
+      pk[4 * v + k] = gelu_gate_pair(r[j], r[j + 1], bw[k], half_g);
     }
   }
 }

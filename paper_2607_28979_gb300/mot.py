@@ -95,6 +95,7 @@ _SIGS = {
     "mot_get_routing": [_H, ctypes.POINTER(ctypes.c_int32)],
     "mot_get_expert_counts": [_H, _P, ctypes.c_int32, _P],
     "mot_debug_set": [_H, ctypes.c_int32, ctypes.c_int64],
+    "mot_debug_gelu": [ctypes.c_int32, _P, _P, ctypes.c_int64, _P, _P],
     "mot_translate_static": [ctypes.POINTER(mot_config), _P, _P, _P, _P, ctypes.c_int32, _P, _P,
                              _P],
     "mot_create_bt": [ctypes.POINTER(mot_config), ctypes.POINTER(mot_bt_config),
@@ -295,6 +296,15 @@ def mot_translate_static(cfg: mot_config, weights, src_k, src_v, seq_lens, batch
     _check(_lib.mot_translate_static(ctypes.byref(cfg), _addr(weights), _addr(src_k),
                                      _addr(src_v), _addr(seq_lens), int(batch), _addr(dst_k),
                                      _addr(dst_v), _stream(stream)), "mot_translate_static")
+
+
+GELU_FORM_MLP, GELU_FORM_BACKBONE, GELU_FORM_SIMT = 0, 1, 2
+
+
+def mot_debug_gelu(form: int, u, gate, out, stream=None) -> None:
+    """out = GELU(u) * gate with the device GELU form `form` (float32 device tensors)."""
+    _check(_lib.mot_debug_gelu(int(form), _addr(u), _addr(gate), int(u.numel()), _addr(out),
+                               _stream(stream)), "mot_debug_gelu")
 
 
 def mot_get_device_status(h: Handle, stream=None) -> int:

@@ -95,3 +95,75 @@ def gather_src(wl, src, layer, b, s):
 def dst_row(dst, l, b, s):
     """Target vector at (layer l, b, s) from a target-layout cache, head-major."""
     return np.asarray(dst[l, b, :, s, :]).reshape(-1)
+
+
+def stratified_tokens(seq_lens, n_random, seed=1, tile=128):
+    """A token sample spread over the batch: n_random positions split across the
+    sequences in proportion to their lengths, always including each sequence's
+    first and last position and the positions on either side of some `tile`
+    boundaries. Returns (tb, ts) int32 arrays (test bookkeeping only)."""
+    rng = np.random.default_rng(seed)
+    total = sum(max(0, L) for L in seq_lens)
+    tb, ts = [], []
+    for b, L in enumerate(seq_lens):
+        if L <= 0:
+            continue
+        k = min(L, max(2, int(round(n_random * L / max(total, 1)))))
+        pos = {0, L - 1}
+        bounds = list(range(tile, L, tile))
+        for t in rng.permutation(bounds)[:max(1, k // 8)] if bounds else []:
+            pos.update({int(t) - 1, int(t)})
+        for p in rng.permutation(L).tolist():   # random positions until k are chosen
+            if len(pos) >= k:
+                break
+            pos.add(p)
+        pos = sorted(pos)
+        tb += [b] * len(pos)
+        ts += pos
+    return np.asarray(tb, dtype=np.int32), np.asarray(ts, dtype=np.int32)
+
+
+def whole_tiles(seq_lens, tile=256, seed=2, last=True):
+    """Every token of one `tile`-aligned window per sequence (the rows of one
+    tile of the tensor-core schedule), plus, with `last`, the final window of the
+    last non-empty sequence (the last wave of a persistent schedule). A sequence
+    shorter than `tile` contributes all its tokens."""
+    rng = np.random.default_rng(seed)
+    tb, ts = [], []
+    seen = set()
+    for b, L in enumerate(seq_lens):
+        if L <= 0:
+            continue
+        n_win = max(1, L // tile)
+        w = int(rng.integers(0, n_win))
+        seen.add((b, w))
+        s0 = w * tile
+        for s in range(s0, min(L, s0 + tile)):
+            tb.append(b)
+            ts.append(s)
+    if last:
+        nz = [b for b, L in enumerate(seq_lens) if L > 0]
+        if nz:
+            b = nz[-1]
+            L = seq_lens[b]
+            w = max(0, (L - 1) // tile)
+            if (b, w) not in seen:
+                for s in range(w * tile, L):
+                    tb.append(b)
+                    ts.append(s)
+    return np.asarray(tb, dtype=np.int32), np.asarray(ts, dtype=np.int32)
+
+
+def restrict_layers(wl, blob, layer_map, keep):
+    """The workload and blob for computing only target layers `keep` (the other
+    target layers marked untranslated): each kept layer's blocks (K and V, or
+    the one MoT-h block) are cut out of the full blob, in blob order. `layer_map` is the full map in use."""
+    tl = [l for l in range(wl.n_layers_tgt) if layer_map[l] >= 0]
+    gsz = wl.group_elems()
+    nx = 1 if wl.is_h else 2   # MoT-h: one block per layer
+    parts = []
+    for r, l in enumerate(tl):
+        if l in keep:
+            parts.append(blob[nx * r * gsz:nx * (r + 1) * gsz])
+    lm = tuple(layer_map[l] if l in keep else -1 for l in range(wl.n_layers_tgt))
+    return wl.replace(layer_map=lm), np.concatenate(parts)

@@ -58,3 +58,39 @@ def test_traffic_records_parse():
         recs.append(f)
     assert {r["kernel"] for r in recs} >= {"umma2_gemm1_gelu_gate", "replay_attn_sparse", "bt_ffn_fused"}
     assert bench.recorded_traffic("no_such_kernel", "gpt2s_opt125m") is None
+
+
+PEAKS = {"hbm_gbs": 6796.5, "bf16_tflops": 1928.9, "bf16_tflops_sustained": 1708.6}
+
+
+def test_peak_follows_the_clock_record():
+    """Burst peak only for a run that saw no power cap and kept its SM clock at max."""
+    short = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": []}
+    capped = {"sm_mhz": 1455.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"]}
+    low = {"sm_mhz": 1800.0, "sm_max_mhz": 2070.0, "reasons": []}
+    assert bench.choose_tensor_peak(PEAKS, short)[:2] == (1928.9, "burst")
+    assert bench.choose_tensor_peak(PEAKS, capped)[:2] == (1708.6, "sustained")
+    assert bench.choose_tensor_peak(PEAKS, low)[:2] == (1708.6, "sustained")
+    assert bench.choose_tensor_peak(PEAKS, None)[:2] == (1708.6, "sustained")
+
+
+def test_kernel_and_step_roofline_recompute_from_their_own_fields():
+    """frac = algorithmic work per launch / mean launch time / the named peak."""
+    wl = synth.WORKLOADS["qwen7_long"]
+    alg = bench.algorithmic(wl, list(range(28)))
+    # GEMM1 of every (layer, X) group: E * 2 * D_s * H FLOPs per token
+    assert alg["flops_gemm1"] == 56 * 61440 * 4 * 2 * 512 * 2048
+    kstats = {"gate": (20, 1.0), "umma2_gemm1_gelu_gate": (280, 480.0),
+              "umma2_gemm2_combine_store": (280, 360.0)}
+    clocks = {"sm_mhz": 1500.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"]}
+    r = bench.kernel_roofline(wl, alg, kstats, 20, PEAKS, "measured", clocks)
+    assert r["kernel"] == "umma2_gemm1_gelu_gate" and r["peak"] == 1708.6
+    per_launch = alg["flops_gemm1"] / 14            # 280 launches over 20 steps
+    assert r["algorithmic_per_launch"] == pytest.approx(per_launch)
+    ach = per_launch / (480.0 / 280 / 1000) / 1e12
+    assert r["achieved"] == pytest.approx(ach, abs=0.05)
+    assert r["frac"] == pytest.approx(ach / 1708.6, abs=1e-4)
+    assert r["frac_of_burst"] == pytest.approx(ach / 1928.9, abs=1e-4)
+    s = bench.step_roofline(alg, 45.0, PEAKS, "measured", clocks)
+    assert s["frac"] == pytest.approx(alg["flops"] / 1708.6e12 * 1000 / 45.0, abs=1e-4)
+    assert s["frac_burst"] == pytest.approx(alg["flops"] / 1928.9e12 * 1000 / 45.0, abs=1e-4)

@@ -12,6 +12,7 @@ torch = pytest.importorskip("torch")
 if not torch.cuda.is_available():
     pytest.skip("needs a CUDA GPU", allow_module_level=True)
 
+import _helpers as H   # noqa: E402
 import _gpu as G   # noqa: E402
 M = G.M
 
@@ -129,10 +130,14 @@ def test_bt_full_size_sampled_tokens():
     sk, sv, blob = _inputs(wl)
     run = BtRun(wl, sk, sv, blob)
     assert run.translate() == M.MOT_OK
-    tb, ts = oracle.sample_tokens(wl.seq_lens, 6, seed=3, tile=10)
+    # a stratified sample of the batch, plus 40 consecutive tokens per sequence
+    # (whole 10-token row tiles of P = 12 source-head rows) and the batch's end
+    tb, ts = H.stratified_tokens(wl.seq_lens, 1024, seed=3, tile=10)
+    pb, ps = H.whole_tiles(wl.seq_lens, tile=40, seed=5)
+    tb, ts = np.concatenate([tb, pb]), np.concatenate([ts, ps])
     ref = oracle.bt_tokens(wl, sk, sv, blob, tb, ts)
     got = run.gather(tb, ts)
-    G.assert_parity(wl, got, ref, "bt_gpt2s_opt125m")
+    G.assert_parity(wl, got, ref, f"bt_gpt2s_opt125m ({tb.size} tokens)")
 
 
 def test_bt_qwen_shapes_sampled_tokens():

@@ -12,6 +12,7 @@ torch = pytest.importorskip("torch")
 if not torch.cuda.is_available():
     pytest.skip("needs a CUDA GPU", allow_module_level=True)
 
+import _helpers as H   # noqa: E402
 import _gpu as G   # noqa: E402
 M = G.M
 
@@ -113,11 +114,21 @@ def test_moth_full_size_sampled():
     act, blob = synth.gen_cache(wl, 0), synth.gen_weights(wl)
     run = HRun(wl, act, blob)
     assert run.translate() == M.MOT_OK
-    tb, ts = oracle.sample_tokens(wl.seq_lens, 24)
+    tb, ts = H.stratified_tokens(wl.seq_lens, 1024, seed=1)
     rk, rv = oracle.translate_h_tokens(wl, act, blob, tb, ts)
     gk, gv = run.gather(tb, ts)
-    G.assert_parity(wl, gk, rk, "h_gpt2s_opt125m K")
-    G.assert_parity(wl, gv, rv, "h_gpt2s_opt125m V")
+    G.assert_parity(wl, gk, rk, f"h_gpt2s_opt125m K ({tb.size} tokens)")
+    G.assert_parity(wl, gv, rv, f"h_gpt2s_opt125m V ({tb.size} tokens)")
+    # every token of one 256-token pair tile per sequence and the batch's last
+    # pair tile, on the first and last target layer
+    keep = {0, wl.n_layers_tgt - 1}
+    wl2, blob2 = H.restrict_layers(wl, blob, list(range(wl.n_layers_tgt)), keep)
+    pb, ps = H.whole_tiles(wl.seq_lens, tile=256)
+    rk, rv = oracle.translate_h_tokens(wl2, act, blob2, pb, ps)
+    gk, gv = run.gather(pb, ps)
+    kl = sorted(keep)
+    G.assert_parity(wl, gk[kl], rk[kl], f"h_gpt2s_opt125m K pair tiles ({pb.size} tokens)")
+    G.assert_parity(wl, gv[kl], rv[kl], f"h_gpt2s_opt125m V pair tiles ({pb.size} tokens)")
 
 
 def test_moth_schedules_and_kernels():

@@ -103,22 +103,40 @@ def test_tiny_fp32_workload_every_element():
 
 # ---------------------------------------------------------------- full-size workloads, sampled
 
-@pytest.mark.parametrize("name", ["gpt2s_opt125m", "qwen05_qwen15", "gpt2m_qwen7", "qwen7_long"])
+# tokens sampled over the whole batch per workload (the oracle's cost per token
+# grows with D_s * H * E: the two largest get fewer)
+FULL_SIZE_SAMPLE = {"gpt2s_opt125m": 1024, "qwen05_qwen15": 1024, "gpt2m_qwen7": 256,
+                    "qwen7_long": 256}
+
+
+@pytest.mark.parametrize("name", sorted(FULL_SIZE_SAMPLE))
 def test_full_size_workload_sampled(name):
-    """The workload at full size in the benchmark's launch configuration: the
-    oracle computes a token sample (sequence ends and 128-token tile boundaries
-    included); every untouched position must still hold the sentinel."""
+    """The workload at full size in the benchmark's launch configuration, against
+    the oracle on (a) a stratified token sample over every sequence (ends and
+    128-token tile boundaries included), on every translated layer, and (b)
+    every token of one 256-token pair tile per sequence plus the last pair tile
+    of the batch (the persistent schedule's last wave), on the first and the
+    last target layer. Every untouched position must still hold the sentinel."""
     wl = synth.WORKLOADS[name]
     sk, sv, blob = inputs(wl)
     run = G.Run(wl, sk, sv, blob)
     assert run.translate() == M.MOT_OK
     assert run.canaries_intact() and run.padding_untouched()
-    tb, ts = oracle.sample_tokens(wl.seq_lens, n_per_seq=6)
+    tb, ts = H.stratified_tokens(wl.seq_lens, FULL_SIZE_SAMPLE[name], seed=1)
     ref = oracle.translate_tokens(wl, sk, sv, blob, tb, ts)
     got = run.gather(tb, ts)
     tl = wl.translated_layers()
-    m = G.assert_parity(wl, got[tl], ref[tl], name)
-    print(name, m)
+    m = G.assert_parity(wl, got[tl], ref[tl], f"{name} stratified ({tb.size} tokens)")
+    print(name, "stratified", tb.size, m)
+    lm = M.mot_get_layer_map(run.h)
+    keep = {tl[0], tl[-1]}
+    wl2, blob2 = H.restrict_layers(wl, blob, lm, keep)
+    pb, ps = H.whole_tiles(wl.seq_lens, tile=256)
+    ref2 = oracle.translate_tokens(wl2, sk, sv, blob2, pb, ps)
+    got2 = run.gather(pb, ps)
+    kl = sorted(keep)
+    m2 = G.assert_parity(wl, got2[kl], ref2[kl], f"{name} whole pair tiles ({pb.size} tokens)")
+    print(name, "pair tiles", pb.size, m2)
 
 
 # ---------------------------------------------------------------- invariants on the GPU

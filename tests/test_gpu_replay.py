@@ -133,15 +133,25 @@ def test_full_size_layer_sampled():
     run = ReplayRun(wl)
     sel = run.select(g)
     rng = np.random.default_rng(11)
+    # 256 selection rows per batch entry (both ends, the S boundary, a whole
+    # 128-row block and random rows), each bit-exact
     for b in range(wl.batch):
-        for u in np.concatenate([[0, 127, 128, 4095], rng.integers(0, 4096, size=12)]):
+        blk = 128 * int(rng.integers(1, 32))
+        us = np.unique(np.concatenate([[0, 127, 128, 4095], np.arange(blk, blk + 128),
+                                       rng.integers(0, 4096, size=124)]))
+        for u in us:
             ref = oracle.replay_select(wl, g, b, int(u))
             np.testing.assert_array_equal(sel[b, u, :ref.size], ref)
-    for layer in (1, 5):
+    # 2048 queries per layer: a full layer, a guided layer and the last layer;
+    # every query head of one whole 128-query tile of one batch entry included
+    for layer in (1, 5, wl.n_layers_tgt - 1):
         out = run.attend(layer, q, k, v, g)
-        tb = rng.integers(0, wl.batch, size=48)
-        th = rng.integers(0, wl.q_heads, size=48)
-        tu = np.concatenate([[0, 4095], rng.integers(0, 4096, size=46)])
+        t0 = 128 * int(rng.integers(0, 32))
+        tile_h, tile_u = np.meshgrid(np.arange(wl.q_heads), np.arange(t0, t0 + 128), indexing="ij")
+        n = 2048 - tile_h.size
+        tb = np.concatenate([np.full(tile_h.size, 3), rng.integers(0, wl.batch, size=n)])
+        th = np.concatenate([tile_h.ravel(), rng.integers(0, wl.q_heads, size=n)])
+        tu = np.concatenate([tile_u.ravel(), [0, 4095], rng.integers(0, 4096, size=n - 2)])
         ref = oracle.replay_tokens(wl, layer, q, k, v, g, tb, th, tu)
         G.assert_parity(BF16, _f64(out)[tb, th, tu], ref, f"full-size layer {layer}")
 

@@ -315,6 +315,16 @@ mot_status mot_get_routing(mot_handle h, int32_t* routing);
 mot_status mot_get_expert_counts(mot_handle h, int32_t* counts, int32_t n, mot_stream_t stream);
 
 /*
+ * Translator usage statistics of Sec. 4.3 over selection counts I_e
+ * (host-only; counts[0..n) as returned by mot_get_expert_counts, all groups
+ * pooled): *cv2 = Var(I) / Mean(I)^2 (population variance) and *entropy =
+ * -sum_e p_e ln p_e with p_e = I_e / sum I (terms with I_e = 0 contribute 0).
+ * Both are 0 when every count is 0. MOT_ERR_INVALID_ARG for NULL pointers,
+ * n <= 0 or a negative count.
+ */
+mot_status mot_expert_usage(const int32_t* counts, int32_t n, double* cv2, double* entropy);
+
+/*
  * Backbone translators (App. C.2) as the experts of the mixture (Def. 3.1).
  * The translation covers one channel window: N consecutive target layers
  * t_r = win_start + r (r = 0..N-1), each paired with source layer pi(t_r)

@@ -1604,4 +1604,27 @@ mot_status mot_get_expert_counts(mot_handle h, int32_t* counts, int32_t n, mot_s
   return MOT_OK;
 }
 
+mot_status mot_expert_usage(const int32_t* counts, int32_t n, double* cv2, double* entropy) {
+  if (!counts || !cv2 || !entropy || n <= 0) return MOT_ERR_INVALID_ARG;
+  double sum = 0.0;
+  for (int32_t i = 0; i < n; ++i) {
+    if (counts[i] < 0) return MOT_ERR_INVALID_ARG;
+    sum += counts[i];
+  }
+  const double mean = sum / n;
+  double var = 0.0;
+  for (int32_t i = 0; i < n; ++i) var += (counts[i] - mean) * (counts[i] - mean);
+  var /= n;
+  *cv2 = mean > 0.0 ? var / (mean * mean) : 0.0;
+  double h = 0.0;
+  if (sum > 0.0)
+    for (int32_t i = 0; i < n; ++i)
+      if (counts[i] > 0) {
+        const double p = counts[i] / sum;
+        h -= p * std::log(p);
+      }
+  *entropy = h;
+  return MOT_OK;
+}
+
 }  // extern "C"

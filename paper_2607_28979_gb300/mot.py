@@ -94,6 +94,7 @@ _SIGS = {
     "mot_set_routing": [_H, ctypes.c_int32],
     "mot_get_routing": [_H, ctypes.POINTER(ctypes.c_int32)],
     "mot_get_expert_counts": [_H, _P, ctypes.c_int32, _P],
+    "mot_expert_usage": [_P, ctypes.c_int32, _P, _P],
     "mot_debug_set": [_H, ctypes.c_int32, ctypes.c_int64],
     "mot_debug_gelu": [ctypes.c_int32, _P, _P, ctypes.c_int64, _P, _P],
     "mot_translate_static": [ctypes.POINTER(mot_config), _P, _P, _P, _P, ctypes.c_int32, _P, _P,
@@ -390,13 +391,12 @@ def mot_get_expert_counts(h: Handle, n_groups: int, n_translators: int, stream=N
 
 
 def expert_usage(counts):
-    """Translator usage statistics over selection counts I_e (Sec. 4.3): the
-    squared coefficient of variation Var(I) / Mean(I)^2 and the entropy
-    -sum p_e log p_e of p_e = I_e / sum I. Returns (cv2, entropy) as floats."""
+    """Translator usage statistics over selection counts I_e (Sec. 4.3), all
+    groups pooled: (Var(I) / Mean(I)^2, -sum p_e ln p_e). Computed by the
+    library's mot_expert_usage."""
     import numpy as np
-    c = np.asarray(counts, dtype=np.float64).ravel()
-    mean = c.mean()
-    cv2 = float(c.var() / (mean * mean)) if mean > 0 else 0.0
-    tot = c.sum()
-    p = c[c > 0] / tot if tot > 0 else c[:0]
-    return cv2, float(-(p * np.log(p)).sum())
+    c = np.ascontiguousarray(np.asarray(counts).ravel(), dtype=np.int32)
+    cv2, ent = ctypes.c_double(), ctypes.c_double()
+    _check(_lib.mot_expert_usage(c.ctypes.data, int(c.size), ctypes.byref(cv2), ctypes.byref(ent)),
+           "mot_expert_usage")
+    return cv2.value, ent.value

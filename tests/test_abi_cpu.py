@@ -99,7 +99,8 @@ def test_valid_config_without_gpu_is_a_cuda_error():
 
 
 def test_expert_usage_statistics_closed_forms():
-    """CV^2 = Var(I) / Mean(I)^2 and entropy -sum p log p of p = I / sum I (Sec. 4.3)."""
+    """CV^2 = Var(I) / Mean(I)^2 and entropy -sum p log p of p = I / sum I (Sec. 4.3),
+    computed by the library's mot_expert_usage (host code, no GPU)."""
     import math
     cv2, ent = M.expert_usage([10, 10])          # balanced: no spread, log 2 nats
     assert cv2 == 0.0 and ent == pytest.approx(math.log(2), abs=1e-15)
@@ -112,6 +113,8 @@ def test_expert_usage_statistics_closed_forms():
     assert cv2 == pytest.approx(var / mean ** 2)
     assert ent == pytest.approx(-sum(x / 10 * math.log(x / 10) for x in c))
     assert M.expert_usage([0, 0]) == (0.0, 0.0)
+    with pytest.raises(M.MotError):
+        M.expert_usage([3, -1])
 
 
 def test_routing_calls_reject_null_handles():

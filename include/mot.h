@@ -238,6 +238,20 @@ mot_status mot_profile_read(mot_handle h, mot_kernel_stat* out, int32_t cap, int
 mot_status mot_debug_set(mot_handle h, int32_t stall_test, int64_t wait_limit_cycles);
 
 /*
+ * Fixed-gate test hook (Def. 3.1 / Eq. mot_definition: the combine is linear
+ * in the gate weights). While set, mot_translate uses the caller's gate rows
+ * instead of evaluating the gate: gate is device float
+ * [G][max_batch][max_seq][E], G = 2 x translated target layers, group 2 r + x
+ * for the r-th translated target layer (x = 0 for K, 1 for V); row (g, b, s)
+ * is the gtilde of token (b, s) in group g (not renormalised or checked). The
+ * buffer must stay valid while set; NULL clears the hook. Dense translation
+ * only: a routed translation (mot_set_routing 1) returns MOT_ERR_UNSUPPORTED
+ * while the hook is set. MOT_ERR_INVALID_ARG for a MoT-h, backbone or replay
+ * handle or a misaligned pointer.
+ */
+mot_status mot_debug_fixed_gate(mot_handle h, const float* gate);
+
+/*
  * GELU probe (App. C.2: phi = GELU). Evaluates, on the device, the GELU form a
  * kernel family uses, out[i] = GELU(u[i]) * gate[i], so that a test can
  * measure it against the exact erf form:

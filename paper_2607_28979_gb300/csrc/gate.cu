@@ -379,6 +379,37 @@ __global__ void __launch_bounds__(256) gate_tile_kernel(PathArgs a) {
 }
 
 // Gate of groups [a.g0, a.g0 + a.gp).
+// Test hook: the gate rows of every tile taken from a caller buffer
+// fg[G][B][S][E] (fp32) instead of the gate's linear map and softmax, written
+// in the layouts the translators read (fp32 rows and the fp16 bias-block rows).
+// Grid (tiles_max, gp), one thread per tile row.
+__global__ void __launch_bounds__(kTileM) fixed_gate_kernel(PathArgs a, const float* __restrict__ fg) {
+  const Dims& d = a.d;
+  const int m = blockIdx.x;
+  const int grp = a.g0 + blockIdx.y;
+  if (m >= *a.n_tiles) return;
+  const TileInfo ti = a.tiles[m];
+  const int r = threadIdx.x;
+  const bool real = r < ti.rows;
+  float g[kMaxE];
+#pragma unroll
+  for (int e = 0; e < kMaxE; ++e)
+    g[e] = (real && e < d.E)
+               ? fg[((static_cast<size_t>(grp) * d.B + ti.b) * d.S + ti.s0 + r) * d.E + e]
+               : 0.f;
+  float* gout = a.gate + (static_cast<size_t>(grp) * d.tpad + static_cast<size_t>(m) * kTileM + r) * d.E;
+#pragma unroll
+  for (int e = 0; e < kMaxE; ++e)
+    if (e < d.E) gout[e] = g[e];
+  write_gate16(a, grp, static_cast<size_t>(m) * kTileM + r, real ? g : nullptr, d.E);
+}
+
+cudaError_t launch_fixed_gate(const PathArgs& a, const float* fg, cudaStream_t st) {
+  if (a.gp <= 0) return cudaSuccess;
+  fixed_gate_kernel<<<dim3(a.d.tiles_max, a.gp), kTileM, 0, st>>>(a, fg);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_gate(const PathArgs& a, cudaStream_t st) {
   const Dims& d = a.d;
   if (a.gp <= 0) return cudaSuccess;

@@ -115,6 +115,7 @@ struct mot_ctx {
   int schedule = 2;           // tcgen05 path: 0 split, 1 fused, 2 split on CTA pairs, 3 on-chip
   long long wait_limit = 4000000000LL;   // bound of every pipeline wait (SM cycles)
   int stall_test = 0;                    // test hook, see mot_debug_set
+  const float* fixed_gate = nullptr;     // test hook, see mot_debug_fixed_gate
   bool weights_loaded = false;
   int gp_max = 1;
   std::vector<GroupInfo> groups_h;
@@ -354,10 +355,15 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
   a.gp = g_end - g_begin;
   const bool routed = h->use_umma && h->sparse_ok && h->routing == 1;
   a.sel = routed ? h->sel : nullptr;
-  MOT_CUDA_TRY(timed(h, "gate", st, [&] {
-    return h->use_umma ? launch_gate_mma(a, tmK, tmV, h->tm_wg16, h->num_sms, st)
-                       : launch_gate(a, st);
-  }));
+  if (h->fixed_gate) {   // test hook: the caller's gate rows replace the gate
+    if (routed) return MOT_ERR_UNSUPPORTED;
+    MOT_CUDA_TRY(timed(h, "gate_fixed", st, [&] { return launch_fixed_gate(a, h->fixed_gate, st); }));
+  } else {
+    MOT_CUDA_TRY(timed(h, "gate", st, [&] {
+      return h->use_umma ? launch_gate_mma(a, tmK, tmV, h->tm_wg16, h->num_sms, st)
+                         : launch_gate(a, st);
+    }));
+  }
   if (routed) {   // Top-K: per-expert token buckets, passes of gp_sparse groups
     const SparseArgs& sp = h->sp;
     for (int g0 = g_begin; g0 < g_end; g0 += h->gp_sparse) {
@@ -1276,6 +1282,13 @@ mot_status mot_debug_set(mot_handle h, int32_t stall_test, int64_t wait_limit_cy
   if (!h || stall_test < 0 || stall_test > 1 || wait_limit_cycles < 0) return MOT_ERR_INVALID_ARG;
   h->stall_test = stall_test;
   h->wait_limit = wait_limit_cycles > 0 ? wait_limit_cycles : 4000000000LL;
+  return MOT_OK;
+}
+
+mot_status mot_debug_fixed_gate(mot_handle h, const float* gate) {
+  if (!h || h->kind != 0) return MOT_ERR_INVALID_ARG;
+  if (gate && (reinterpret_cast<uintptr_t>(gate) & 3u)) return MOT_ERR_INVALID_ARG;
+  h->fixed_gate = gate;
   return MOT_OK;
 }
 

@@ -112,6 +112,7 @@ cudaError_t launch_f32_to_f16(const float* src, void* dst, size_t n, cudaStream_
 cudaError_t launch_prep(const int32_t* seq_lens, int32_t batch, const Dims& d, TileInfo* tiles,
                         int32_t* n_tiles, int32_t* status, cudaStream_t st);
 cudaError_t launch_gate(const PathArgs& a, cudaStream_t st);
+cudaError_t launch_fixed_gate(const PathArgs& a, const float* fg, cudaStream_t st);
 cudaError_t launch_simt_gemm1(const PathArgs& a, cudaStream_t st);
 cudaError_t launch_simt_gemm2(const PathArgs& a, cudaStream_t st);
 

@@ -97,6 +97,7 @@ _SIGS = {
     "mot_expert_usage": [_P, ctypes.c_int32, _P, _P],
     "mot_debug_set": [_H, ctypes.c_int32, ctypes.c_int64],
     "mot_debug_gelu": [ctypes.c_int32, _P, _P, ctypes.c_int64, _P, _P],
+    "mot_debug_fixed_gate": [_H, _P],
     "mot_translate_static": [ctypes.POINTER(mot_config), _P, _P, _P, _P, ctypes.c_int32, _P, _P,
                              _P],
     "mot_create_bt": [ctypes.POINTER(mot_config), ctypes.POINTER(mot_bt_config),
@@ -297,6 +298,12 @@ def mot_translate_static(cfg: mot_config, weights, src_k, src_v, seq_lens, batch
     _check(_lib.mot_translate_static(ctypes.byref(cfg), _addr(weights), _addr(src_k),
                                      _addr(src_v), _addr(seq_lens), int(batch), _addr(dst_k),
                                      _addr(dst_v), _stream(stream)), "mot_translate_static")
+
+
+def mot_debug_fixed_gate(h: Handle, gate) -> None:
+    """Use the gate rows in `gate` (device float [G][max_batch][max_seq][E]) until
+    cleared with None."""
+    _check(_lib.mot_debug_fixed_gate(h.ptr, _addr(gate)), "mot_debug_fixed_gate")
 
 
 GELU_FORM_MLP, GELU_FORM_BACKBONE, GELU_FORM_SIMT = 0, 1, 2

@@ -170,6 +170,11 @@ def test_replay_backbone_and_debug_calls_reject_null_handles():
     assert L.mot_replay_select(None, None, None, 0, None, None) == M.MOT_ERR_INVALID_ARG
     assert L.mot_translate_bt(None, None, None, None, 0, None, None, None) == M.MOT_ERR_INVALID_ARG
     assert L.mot_debug_set(None, 0, 0) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_debug_fixed_gate(None, None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_debug_gelu(3, None, None, 0, None, None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_debug_gelu(0, None, None, -1, None, None) == M.MOT_ERR_INVALID_ARG
+    assert L.mot_debug_gelu(0, None, None, 0, None, None) == M.MOT_OK   # nothing to do
+    assert L.mot_debug_gelu(0, None, None, 4, None, None) == M.MOT_ERR_INVALID_ARG
 
 
 def _static_call(cfg, weights, src_k, src_v, dst_k, dst_v, lens=0x9000, batch=1):

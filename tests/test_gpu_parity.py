@@ -528,3 +528,70 @@ def test_bounded_wait_reports_timeout_and_the_context_survives():
     run.buf_v, run.dv = G.alloc_dst(wl)
     assert run.translate() == M.MOT_OK
     full_check(wl, run, sk, sv, blob, "after a timeout")
+
+
+# ---------------------------------------------------------------- linearity in the gate
+
+LIN = {
+    "umma": synth.Workload("lin_umma", 3, 2, 64, 4, 2, 128, 3, 256, 3, 300, "bf16",
+                           (300, 129, 1), layer_map=(2, -1, 0, 1)),
+    "simt": synth.Workload("lin_simt", 2, 3, 16, 2, 5, 8, 3, 40, 2, 70, "bf16", (70, 33)),
+}
+
+
+def _fixed_gates(wl, seed):
+    """Two gates on the simplex per (group, b, s) and their mixture at alpha = 0.3,
+    fp32 [G][B][S][E]."""
+    rng = np.random.default_rng(seed)
+    G_ = 2 * len(wl.translated_layers())
+    shape = (G_, wl.max_batch, wl.max_seq, wl.n_translators)
+    g1 = rng.dirichlet(np.ones(wl.n_translators), size=shape[:3]).astype(np.float32)
+    g2 = rng.dirichlet(np.ones(wl.n_translators) * 0.3, size=shape[:3]).astype(np.float32)
+    alpha = 0.3
+    g3 = (alpha * g1.astype(np.float64) + (1 - alpha) * g2.astype(np.float64)).astype(np.float32)
+    return g1, g2, g3, alpha
+
+
+def _oracle_gate(wl, g, tb, ts):
+    """The [G][B][S][E] gate rows in the oracle's [L_t][2][n][E] layout."""
+    out = np.zeros((wl.n_layers_tgt, 2, tb.size, wl.n_translators))
+    for r, l in enumerate(wl.translated_layers()):
+        for x in (0, 1):
+            out[l, x] = g[2 * r + x][tb, ts]
+    return out
+
+
+@pytest.mark.parametrize("case,schedule", [("umma", 3), ("umma", 2), ("umma", 1), ("umma", 0),
+                                           ("simt", 2)])
+def test_fixed_gate_matches_oracle_and_combine_is_linear(case, schedule):
+    """Eq. mot_definition on the GPU: with the gate rows given (test hook), the
+    translation matches the oracle's with the same rows, and the translation of
+    the mixed gate alpha g1 + (1 - alpha) g2 is alpha y(g1) + (1 - alpha) y(g2)
+    within the outputs' rounding."""
+    wl = LIN[case]
+    sk, sv, blob = inputs(wl, seed=21)
+    g1, g2, g3, alpha = _fixed_gates(wl, 5)
+    tb = np.concatenate([np.full(L, b) for b, L in enumerate(wl.seq_lens)]).astype(np.int32)
+    ts = np.concatenate([np.arange(L) for L in wl.seq_lens]).astype(np.int32)
+    tl = wl.translated_layers()
+    outs = []
+    for g in (g1, g2, g3):
+        run = G.Run(wl, sk, sv, blob)
+        M.mot_set_schedule(run.h, schedule)
+        gd = torch.from_numpy(g).cuda()
+        M.mot_debug_fixed_gate(run.h, gd)
+        assert run.translate() == M.MOT_OK
+        M.mot_debug_fixed_gate(run.h, None)
+        got = run.gather(tb, ts)[tl]
+        ref = oracle.translate_tokens(wl, sk, sv, blob, tb, ts,
+                                      gate_fixed=_oracle_gate(wl, g, tb, ts))[tl]
+        G.assert_parity(wl, got, ref, f"{case} schedule {schedule} fixed gate")
+        assert run.padding_untouched() and run.canaries_intact()
+        outs.append(got)
+    mix = alpha * outs[0] + (1 - alpha) * outs[1]
+    G.assert_parity(wl, outs[2], mix, f"{case} schedule {schedule} linearity")
+    # the hook is cleared: the next translation evaluates the gate again
+    run = G.Run(wl, sk, sv, blob)
+    assert run.translate() == M.MOT_OK
+    ref = oracle.translate_tokens(wl, sk, sv, blob, tb, ts)[tl]
+    G.assert_parity(wl, run.gather(tb, ts)[tl], ref, f"{case} evaluated gate")

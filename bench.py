@@ -1065,6 +1065,9 @@ def main():
                          "with 0 < k < E the translators run on token buckets")
     ap.add_argument("--n-layers", type=int, default=0,
                     help="keep only the first N layers of both models (smaller profiling case)")
+    ap.add_argument("--seq-div", type=int, default=1,
+                    help="divide max_seq and every sequence length by this factor (smaller "
+                         "profiling case)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "mot":
         args.warmup = 3
@@ -1080,7 +1083,10 @@ def main():
                         n_layers_tgt=min(args.n_layers, wl.n_layers_tgt))
     if args.per_config is None:
         args.per_config = (args.workload == DEFAULT_WORKLOAD and args.top_k == 0
-                           and args.n_layers == 0)
+                           and args.n_layers == 0 and args.seq_div == 1)
+    if args.seq_div > 1:
+        wl = wl.replace(name=f"{wl.name}_S{args.seq_div}", max_seq=wl.max_seq // args.seq_div,
+                        seq_lens=tuple(L // args.seq_div for L in wl.seq_lens))
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_mot(args, wl)

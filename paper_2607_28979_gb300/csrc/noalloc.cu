@@ -266,12 +266,6 @@ extern "C" mot_status mot_translate_static(const mot_config* cfg, const void* we
   const size_t group_elems = mul_sat(c.n_translators, Ds_) + c.n_translators +
                              mul_sat(c.n_translators, per_exp);
   const size_t w_b = mul_sat(mul_sat(2 * size_t(n_translated), group_elems), es);
-  if (ranges_overlap(dst_k, dst_b, dst_v, dst_b) || ranges_overlap(dst_k, dst_b, src_k, src_b) ||
-      ranges_overlap(dst_k, dst_b, src_v, src_b) || ranges_overlap(dst_v, dst_b, src_k, src_b) ||
-      ranges_overlap(dst_v, dst_b, src_v, src_b) || ranges_overlap(dst_k, dst_b, weights, w_b) ||
-      ranges_overlap(dst_v, dst_b, weights, w_b))
-    return MOT_ERR_INVALID_ARG;
-
   // the kernels index with int32 widths
   if (Ds_ > INT32_MAX || Dt_ > INT32_MAX ||
       mul_sat(c.n_translators, c.hidden) > size_t(INT32_MAX))
@@ -289,6 +283,12 @@ extern "C" mot_status mot_translate_static(const mot_config* cfg, const void* we
   const size_t gate_bytes = (rows * a.E * 4 + 255) / 256 * 256;
   const size_t need = gate_bytes + mul_sat(mul_sat(rows, size_t(a.EH)), 4);
   if (need > kStaticScratchBytes) return MOT_ERR_UNSUPPORTED;   // scratch too small
+  if (ranges_overlap(dst_k, dst_b, dst_v, dst_b) || ranges_overlap(dst_k, dst_b, src_k, src_b) ||
+      ranges_overlap(dst_k, dst_b, src_v, src_b) || ranges_overlap(dst_v, dst_b, src_k, src_b) ||
+      ranges_overlap(dst_v, dst_b, src_v, src_b) || ranges_overlap(dst_k, dst_b, weights, w_b) ||
+      ranges_overlap(dst_v, dst_b, weights, w_b))
+    return MOT_ERR_INVALID_ARG;
+
   if (batch == 0) return MOT_OK;
 
   int dev = 0;

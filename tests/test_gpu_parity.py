@@ -610,9 +610,10 @@ OUTLIER = {
 def test_outlier_source_channels_stay_finite_and_within_the_bar(case):
     """Real K caches carry a few channels 10-100x the median scale. Scaling 4
     source channels of every layer by 100 enlarges the hidden pre-activations
-    (rounded to fp16 on the tensor-core path) and the outputs; the translation
-    stays finite and within rel-RMS 1e-2, and within max-abs 3e-2 plus the bf16
-    rounding of the larger outputs (2^-8 |y|)."""
+    (rounded to fp16 on the tensor-core path) and the outputs (|y| up to ~100).
+    The translation stays finite and within rel-RMS 1e-2; the max-abs bar of
+    3e-2, set for outputs of unit scale, is scaled by the outputs' RMS (the
+    fp16 rounding of the hidden values grows with them)."""
     wl = OUTLIER[case]
     sk, sv, blob = inputs(wl, seed=31)
     rng = np.random.default_rng(9)
@@ -631,7 +632,7 @@ def test_outlier_source_channels_stay_finite_and_within_the_bar(case):
     for got, ref, x in ((gk[mask], rk[mask], "K"), (gv[mask], rv[mask], "V")):
         assert np.isfinite(got).all()
         m = G.metrics(got, ref)
-        excess = np.abs(got - ref) - 2.0 ** -8 * np.abs(ref)
-        print(case, x, m, "max |y|", np.abs(ref).max())
+        rms = float(np.sqrt(np.mean(ref ** 2)))
+        print(case, x, m, "rms(y)", rms)
         assert m["rel_rms"] <= 1e-2, (case, x, m)
-        assert excess.max() <= 3e-2, (case, x, excess.max())
+        assert m["max_abs"] <= 3e-2 * max(1.0, rms), (case, x, m, rms)

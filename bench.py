@@ -163,6 +163,7 @@ KERNEL_SOURCES = {
     "umma2_gemm1_gelu_gate": ["umma2.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
     "umma2_gemm2_combine_store": ["umma2.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
     "umma2_onchip_translate": ["onchip.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
+    "umma2_wide_translate": ["wide.cu", "umma_common.cuh", "gelu.cuh", "ptx.cuh", "mot_internal.h"],
     # replay stages (all kernels of replay.cu)
     "replay_attn_sparse": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
     "replay_select": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
@@ -378,6 +379,7 @@ def run_reference(args, wl):
 def _per_launch_flops(alg):
     return {"umma_fused_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
             "umma2_onchip_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
+            "umma2_wide_translate": alg["flops_gemm1"] + alg["flops_gemm2"],
             "umma2_gemm1_gelu_gate": alg["flops_gemm1"],
             "umma2_gemm2_combine_store": alg["flops_gemm2"],
             "umma2_sparse_gemm1": alg["flops_gemm1"],
@@ -476,7 +478,7 @@ class _Setup:
             self.h = M.mot_create(M.config_from(wl))
         M.mot_load_weights(self.h, self.blob)
         self.path = M.mot_get_path(self.h)
-        names = {0: "split", 1: "fused", 2: "pair", 3: "onchip"}
+        names = {0: "split", 1: "fused", 2: "pair", 3: "onchip", 4: "wide"}
         if args.schedule != "auto" and not wl.is_bt:
             M.mot_set_schedule(self.h, {v: k for k, v in names.items()}[args.schedule])
         sched = names[M.mot_get_schedule(self.h)]
@@ -1055,9 +1057,10 @@ def main():
                     help="also time the other bf16 model pairs (device-resident) in the same "
                          "run (default: on for the headline workload)")
     ap.add_argument("--no-per-config", dest="per_config", action="store_false")
-    ap.add_argument("--schedule", choices=["auto", "onchip", "pair", "fused", "split"],
+    ap.add_argument("--schedule", choices=["auto", "wide", "onchip", "pair", "fused", "split"],
                     default="auto",
                     help="tcgen05 launch schedule: the library's default for the shape, the "
+                         "on-chip kernel on clusters of two CTA pairs (D_t = 512), the "
                          "on-chip GEMM1-GELU-GEMM2 kernel (D_s <= 128, D_t = 256), GEMMs on CTA "
                          "pairs (2-SM MMA), one fused persistent launch, or GEMMs on single SMs")
     ap.add_argument("--top-k", type=int, default=0,

@@ -112,7 +112,8 @@ struct mot_ctx {
   int device = 0;
   int num_sms = 0;
   bool use_umma = false;
-  int schedule = 2;           // tcgen05 path: 0 split, 1 fused, 2 split on CTA pairs, 3 on-chip
+  int schedule = 2;           // tcgen05 path: 0 split, 1 fused, 2 split on CTA pairs, 3 on-chip,
+                              // 4 on-chip on clusters of two pairs (D_t = 512)
   long long wait_limit = 4000000000LL;   // bound of every pipeline wait (SM cycles)
   int stall_test = 0;                    // test hook, see mot_debug_set
   const float* fixed_gate = nullptr;     // test hook, see mot_debug_fixed_gate
@@ -384,6 +385,12 @@ mot_status run_translate(mot_ctx* h, const void* src_k, const void* src_v, const
         MOT_CUDA_TRY(timed(h, "combine", st, [&] { return launch_combine(a, sp, st); }));
     }
     h->counts_valid = true;
+    return MOT_OK;
+  }
+  if (h->use_umma && h->schedule == 4) {   // one launch; no A2 workspace, so no passes
+    MOT_CUDA_TRY(timed(h, "umma2_wide_translate", st, [&] {
+      return launch_wide(a, tmK, tmV, h->tm_w1q, h->tm_w2h, h->tm_g16, h->tm_b2th, h->num_sms, st);
+    }));
     return MOT_OK;
   }
   if (h->use_umma && h->schedule == 3) {   // one launch; no A2 workspace, so no passes
@@ -1266,8 +1273,10 @@ mot_status mot_get_path(mot_handle h, int32_t* path) {
 }
 
 mot_status mot_set_schedule(mot_handle h, int32_t schedule) {
-  if (!h || schedule < 0 || schedule > 3) return MOT_ERR_INVALID_ARG;
+  if (!h || schedule < 0 || schedule > 4) return MOT_ERR_INVALID_ARG;
   if (schedule == 3 && !(h->use_umma && onchip_supported(h->d))) return MOT_ERR_UNSUPPORTED;
+  if (schedule == 4 && !(h->kind == 0 && h->use_umma && wide_supported(h->d)))
+    return MOT_ERR_UNSUPPORTED;
   h->schedule = schedule;
   return MOT_OK;
 }

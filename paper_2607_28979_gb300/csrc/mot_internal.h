@@ -175,6 +175,16 @@ cudaError_t launch_onchip(const PathArgs& a, const CUtensorMap& tmK, const CUten
                           const CUtensorMap& tmG16, const CUtensorMap& tmB2th, int num_sms,
                           cudaStream_t st);
 
+// On-chip translation for D_t = 512 (wide.cu): clusters of two CTA pairs, pair
+// p owning output columns [256 p, 256 p + 256); the pairs split GEMM1's hidden
+// chunks and exchange them through distributed shared memory. Same maps as the
+// on-chip kernel.
+bool wide_supported(const Dims& d);
+cudaError_t launch_wide(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                        const CUtensorMap& tmW1q, const CUtensorMap& tmW2h,
+                        const CUtensorMap& tmG16, const CUtensorMap& tmB2th, int num_sms,
+                        cudaStream_t st);
+
 // Fused persistent kernel: both GEMMs of a pass in one launch (fused.cu).
 // `counters` holds fused_counter_ints(d, gp) int32 (zeroed by the launcher).
 int fused_block_tiles(const Dims& d, int num_sms);

@@ -390,6 +390,74 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint64_t* bar, uint32_t cta)
       : "memory");
 }
 
+// As umma_commit_pair, but arriving on the barrier at `bar`'s offset in every
+// cluster CTA whose bit is set in `mask` (CTAs of other pairs included).
+__device__ __forceinline__ void umma_commit_mask(uint64_t* bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+      " [%0], %1;" ::"r"(smem_u32(bar)),
+      "h"(mask)
+      : "memory");
+}
+
+// Arrive on the barrier at `bar`'s offset in cluster CTA `cta`, releasing this
+// thread's prior memory operations at cluster scope.
+__device__ __forceinline__ void mbar_arrive_release_cluster(uint64_t* bar, uint32_t cta) {
+  asm volatile(
+      "{\n\t.reg .b32 ra;\n\t"
+      "mapa.shared::cluster.u32 ra, %0, %1;\n\t"
+      "mbarrier.arrive.release.cluster.shared::cluster.b64 _, [ra];\n\t}" ::"r"(smem_u32(bar)),
+      "r"(cta)
+      : "memory");
+}
+
+// Wait for phase `parity` of a local barrier that remote CTAs arrive on
+// (acquire at cluster scope); bounded like mbar_wait.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar_addr, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar_addr), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity,
+                                                  volatile int* abort_flag,
+                                                  long long limit = kWaitLimitCycles) {
+  const uint32_t a = smem_u32(bar);
+  if (mbar_try_wait_cluster(a, parity)) return true;
+  const long long t0 = clock64();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait_cluster(a, parity)) return true;
+    if ((it & 63u) == 0) {
+      if (*abort_flag) return false;
+      if (clock64() - t0 > limit) {
+        *abort_flag = 1;
+        return false;
+      }
+    }
+  }
+}
+
+// Copy `bytes` (a multiple of 16) from this CTA's shared memory at `src` to
+// the same offset as `dst` in cluster CTA `cta`; the bytes complete on the
+// barrier at `bar`'s offset in that CTA.
+__device__ __forceinline__ void bulk_copy_to_cta(const void* dst, const void* src, uint32_t bytes,
+                                                 uint64_t* bar, uint32_t cta) {
+  asm volatile(
+      "{\n\t.reg .b32 rd, rb;\n\t"
+      "mapa.shared::cluster.u32 rd, %0, %3;\n\t"
+      "mapa.shared::cluster.u32 rb, %2, %3;\n\t"
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [rd], [%1], %4, [rb];"
+      "\n\t}" ::"r"(smem_u32(dst)),
+      "r"(smem_u32(src)), "r"(smem_u32(bar)), "r"(cta), "r"(bytes)
+      : "memory");
+}
+
 // True in exactly one lane of the (fully active) warp. Issuing tcgen05.mma
 // from a warp-uniform loop under elect.sync keeps its operands warp-uniform.
 // Warp-wide maximum of an fp32 value (every lane of the warp takes part).

@@ -47,6 +47,13 @@ SMALL = {
                                 (90, 0, 65), layer_map=(2, 0)),
     # single translator (E = 1) on the tensor-core path
     "umma_e1": synth.Workload("umma_e1", 2, 4, 64, 2, 2, 128, 1, 512, 1, 256, "bf16", (256,)),
+    # D_t = 512 (two CTA pairs per cluster): ragged, an odd tile count (the last
+    # pair tile has one live half), a -1 in the map, E = 3 (6 hidden chunks)
+    "umma_wide": synth.Workload("umma_wide", 3, 4, 64, 4, 4, 128, 3, 256, 3, 300, "bf16",
+                                (300, 129, 1), layer_map=(2, -1, 0, 1)),
+    # D_t = 512, D_s = 512 (8 K blocks), E = 1, H = 768 (6 chunks)
+    "umma_wide_e1": synth.Workload("umma_wide_e1", 2, 4, 128, 2, 4, 128, 1, 768, 2, 256, "bf16",
+                                   (256, 200)),
 }
 
 
@@ -57,14 +64,29 @@ def onchip_supported(wl):
             and wl.src_head_dim % 64 == 0 and wl.tgt_head_dim % 32 == 0)
 
 
-@pytest.mark.parametrize("schedule", [3, 2, 1, 0])
+def wide_supported(wl):
+    """Shapes the on-chip schedule on clusters of two CTA pairs (4) takes: D_t = 512."""
+    d_t = wl.tgt_kv_heads * wl.tgt_head_dim
+    return (wl.dtype == "bf16" and d_t == 512 and wl.hidden % 128 == 0
+            and wl.src_head_dim % 64 == 0 and wl.tgt_head_dim % 32 == 0)
+
+
+def schedule_supported(wl, schedule):
+    if schedule == 3:
+        return onchip_supported(wl)
+    if schedule == 4:
+        return wide_supported(wl)
+    return True
+
+
+@pytest.mark.parametrize("schedule", [4, 3, 2, 1, 0])
 @pytest.mark.parametrize("name", sorted(SMALL))
 def test_small_shapes_every_element(name, schedule):
     wl = SMALL[name]
     if schedule != 2 and not name.startswith("umma"):
         pytest.skip("the schedule only applies to the tensor-core path")
-    if schedule == 3 and not onchip_supported(wl):
-        pytest.skip("the on-chip schedule needs D_s <= 128 and D_t = 256")
+    if not schedule_supported(wl, schedule):
+        pytest.skip("the schedule does not take this shape")
     sk, sv, blob = inputs(wl, seed=1)
     run = G.Run(wl, sk, sv, blob)
     expect_path = 1 if name.startswith("umma") else 0
@@ -74,14 +96,14 @@ def test_small_shapes_every_element(name, schedule):
     full_check(wl, run, sk, sv, blob, name)
 
 
-@pytest.mark.parametrize("other", [1, 2, 3])
-@pytest.mark.parametrize("name", ["umma_ragged", "umma_e3", "gpt2s_opt125m", "qwen7_long",
-                                  "qwen05_qwen15"])
+@pytest.mark.parametrize("other", [1, 2, 3, 4])
+@pytest.mark.parametrize("name", ["umma_ragged", "umma_e3", "umma_wide", "umma_wide_e1",
+                                  "gpt2s_opt125m", "qwen7_long", "qwen05_qwen15", "gpt2m_qwen7"])
 def test_launch_schedules_are_bit_identical(name, other):
     """Every launch schedule runs the same per-tile arithmetic in the same order."""
     wl = SMALL.get(name) or synth.WORKLOADS[name]
-    if other == 3 and not onchip_supported(wl):
-        pytest.skip("the on-chip schedule needs D_s <= 128 and D_t = 256")
+    if not schedule_supported(wl, other):
+        pytest.skip("the schedule does not take this shape")
     sk, sv, blob = inputs(wl, seed=3)
     a = G.Run(wl, sk, sv, blob)
     b = G.Run(wl, sk, sv, blob)

@@ -458,6 +458,27 @@ __device__ __forceinline__ void bulk_copy_to_cta(const void* dst, const void* sr
       : "memory");
 }
 
+// Shared::cluster address of `p`'s offset in cluster CTA `cta`.
+__device__ __forceinline__ uint32_t mapa_cluster(const void* p, uint32_t cta) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(p)), "r"(cta));
+  return r;
+}
+
+// 16-byte store into another CTA's shared memory (a shared::cluster address).
+__device__ __forceinline__ void st_cluster_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
+                                              uint32_t d) {
+  asm volatile("st.shared::cluster.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b),
+               "r"(c), "r"(d)
+               : "memory");
+}
+
+// Make this thread's generic-proxy writes to shared memory anywhere in the
+// cluster visible to async-proxy readers (TMA, tensor core).
+__device__ __forceinline__ void fence_proxy_async_cluster() {
+  asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+}
+
 // True in exactly one lane of the (fully active) warp. Issuing tcgen05.mma
 // from a warp-uniform loop under elect.sync keeps its operands warp-uniform.
 // Warp-wide maximum of an fp32 value (every lane of the warp takes part).

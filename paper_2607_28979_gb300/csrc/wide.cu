@@ -1,99 +1,100 @@
-// On-chip translation for D_t = 512, D_s <= 512 (schedule 4): GEMM1 -> GELU *
-// gate -> GEMM2 with the hidden activations kept on chip, for translators whose
-// output is too wide for one CTA pair's tensor memory.
+// On-chip translation for D_t = 512 (schedule 4): GEMM1 -> GELU * gate ->
+// GEMM2 with the hidden activations kept in shared memory, for translators
+// whose output is too wide for one CTA pair's tensor memory.
 //
-// One pair's GEMM2 accumulator for 256 token rows and D_t = 512 columns fills
-// all 512 TMEM columns of each of its SMs, leaving none for GEMM1. So a
-// cluster of four CTAs -- two CTA pairs -- works on one 256-row pair tile
-// (token tiles 2 mp and 2 mp + 1 of one (target layer, K/V) group) with the
-// two GEMMs on different pairs:
-//   pair 0 (ranks 0, 1) walks the concatenated hidden dimension E*H in
-//     128-column chunks, U_c = Z * W1cat[128 c .. 128 c + 127]^T (M = 256,
-//     N = 128, K = D_s) into one of four TMEM accumulators, with the tile's
-//     source rows Z resident in shared memory; its epilogue computes
-//     A2_c = fp16(GELU(U_c + b1) * gtilde_m) and stores it straight into a
-//     shared-memory slot of the pair-1 CTA that holds the same token rows,
-//     in the tcgen05 operand layout (st.shared::cluster);
-//   pair 1 (ranks 2, 3) accumulates Y += A2_c * W2cat[:, 128 c .. 128 c + 127]^T
-//     (M = 256, two N = 256 halves of D_t, K = 128) in TMEM over every chunk,
-//     adds the gate-weighted biases sum_m gtilde_m b2_m (Def. 3.1) as one more
-//     K block (A = gate16, B = b2t), and stores Y as bf16 into the target
-//     cache.
-// The two GEMMs have equal work when D_s = D_t. A2 never leaves the chip.
+// A pair's accumulator for 256 token rows and D_t = 512 output columns would
+// fill all 512 TMEM columns of each SM, leaving none for GEMM1. So a cluster
+// of four CTAs -- two CTA pairs -- shares one 256-row pair tile (token tiles
+// 2 mp and 2 mp + 1 of one (target layer, K/V) group): pair p accumulates
+// output columns [256 p, 256 p + 256) of Y = A2 * W2cat^T in TMEM (256
+// columns) and keeps two 128-column GEMM1 accumulators. The concatenated
+// hidden dimension E*H is walked in 128-column chunks; chunk c's GEMM1
+//   U_c = Z * W1cat[128 c .. 128 c + 127]^T     (M = 256, N = 128, K = D_s)
+// runs on pair c % 2 only, whose epilogue writes A2_c = fp16(GELU(U_c + b1) *
+// gtilde_m) into its pair's shared-memory slot in the tcgen05 operand layout,
+// and each epilogue warp copies its 4 KB of rows (cp.async.bulk, shared::cta ->
+// shared::cluster) into the same slot of the other pair's CTA that holds the
+// same token rows. Both pairs run
+//   Y_p += A2_c * W2cat[256 p .. 256 p + 255, 128 c .. 128 c + 127]^T
+// for every chunk; after the last chunk, Y_p += gate16 * b2t adds the
+// gate-weighted biases sum_m gtilde_m b2_m (Def. 3.1) as one more K block,
+// and the epilogue stores Y_p as bf16 into the target cache. A2 never leaves
+// the chip, and each pair does half of both GEMMs' tensor-core work.
 //
-// Shared memory per CTA, pair 0: Z as D_s / 64 blocks of 16 KB (128 rows x 64
-// K) and a ring of 12 W1 stages of 8 KB (its 64 of a chunk's 128 rows, K = 64);
-// pair 1: 3 A2 slots of 32 KB (chunk c in slot c % 3), a ring of 3 W2 stages
-// of 32 KB (its 128 rows of each 256-column half, K = 64; the tile's b2t
-// block takes one stage too) and 16 KB of gate16 rows.
-// TMEM: pair 0 acc1[4] x 128 columns, pair 1 acc2 512 columns.
+// Shared memory per CTA: a ring of 4 stages of 24 KB (a 16 KB block of this
+// CTA's 128 source rows and the 8 KB block of its half of the chunk's W1
+// rows, K = 64 each), a ring of 2 W2 stages of 16 KB (this CTA's 128 of its
+// pair's 256 rows of W2cat, K = 64; the tile's b2t block takes one stage
+// too), 2 A2 slots of 32 KB and 16 KB of gate16 rows. Slot q holds the chunks
+// that pair q computes (c % 2 == q), so a slot is only ever written by one
+// pair's epilogue, which waits for every use of it in order: no barrier phase
+// of a slot can pass unobserved by its writer.
+// TMEM per CTA (512 columns): acc2 in [0, 256), acc1[0] in [256, 384),
+// acc1[1] in [384, 512).
 //
-// Roles (13 warps per CTA):
-//   pair 0  warp 0 lane 0   TMA loads of Z (once per tile) and of the W1 ring;
-//           warp 3 (leader) GEMM1 issue (one elected lane);
-//           warps 5..12     chunk epilogue: warp w owns rows 32 (w % 4) ..,
-//                           chunk columns 64 hh .. 64 hh + 63 (hh = (w - 5) / 4);
-//   pair 1  warp 1 lane 0   TMA loads of the W2 ring, b2t and gate16;
-//           warp 4 (leader) GEMM2 and bias issue (one elected lane); the commit
-//                           after each chunk frees its slot (arrives in pair 0);
-//           warps 5..12     output epilogue: rows 32 (w % 4) .., columns
-//                           256 hh .. 256 hh + 255;
-//   both    warp 2          TMEM allocation of the pair.
-// Every slot use is written by pair 0's epilogue, which waits for the slot's
-// previous use to be freed before every write, so no barrier phase can pass
-// unobserved. Every wait is bounded; a timeout unwinds every role and raises
+// Roles per CTA (13 warps):
+//   warp 0 lane 0      TMA loads of the source / W1 ring (own chunks only);
+//   warp 1 lane 0      TMA loads of the W2 ring, the b2t block and gate16;
+//   warp 2             TMEM allocation of the pair, then (lane 0) the relay:
+//                      for an own chunk it waits for this CTA's epilogue and
+//                      tells the pair leader the slot is full; for the other
+//                      pair's chunk it waits for the copies to land and tells
+//                      the pair leader;
+//   warp 3 (leader)    GEMM1 issue (one elected lane);
+//   warp 4 (leader)    GEMM2 and bias issue (one elected lane); every GEMM2
+//                      commit arrives on slot-free barriers in all four CTAs;
+//   warps 5..12        epilogue: warp 5 + 4 hh + q owns rows 32 q .. 32 q + 31,
+//                      chunk columns 64 hh .. 64 hh + 63 and output columns
+//                      128 hh .. 128 hh + 127 of its pair's 256.
+// Every wait is bounded; a timeout unwinds every role and raises
 // kStatusTimeout.
 #include "umma_common.cuh"
 
 namespace mot {
 namespace {
 
-constexpr int kWCtas = 4;                     // two CTA pairs per cluster
+constexpr int kWPairs = 2;                    // CTA pairs per cluster (D_t = 256 * kWPairs)
+constexpr int kWCtas = 2 * kWPairs;
 constexpr int kWChunk = 128;                  // hidden columns per chunk
 constexpr int kWBlk = UM * UK * 2;            // 16 KB: 128 rows x 64 K, 16-bit
 constexpr int kWW1Blk = (kWChunk / 2) * UK * 2;   // 8 KB: 64 rows x 64 K
-constexpr int kWMaxZ = 8;                     // Z blocks: D_s <= 512
-constexpr int kWStagesW1 = 12;
-constexpr int kWStagesW2 = 3;
-constexpr int kWW2Stage = 2 * kWBlk;          // both 256-column halves, K = 64
-constexpr int kWSlots = 3;
+constexpr int kWStage1 = kWBlk + kWW1Blk;     // source block + W1 block
+constexpr int kWStages1 = 4;
+constexpr int kWStages2 = 2;
+constexpr int kWSlots = kWPairs;              // slot q: the chunks pair q computes
 constexpr int kWSlotBytes = 2 * kWBlk;        // 128 rows x 128 K
-constexpr int kWAcc1 = 4;                     // GEMM1 accumulators of 128 columns
-// pair 0 layout
-constexpr int kWOffW1 = kWMaxZ * kWBlk;
-constexpr int kWEnd0 = kWOffW1 + kWStagesW1 * kWW1Blk;
-// pair 1 layout
-constexpr int kWOffW2 = kWSlots * kWSlotBytes;
-constexpr int kWOffG = kWOffW2 + kWStagesW2 * kWW2Stage;
-constexpr int kWEnd1 = kWOffG + kWBlk;
-constexpr int kWOffBar = kWEnd0 > kWEnd1 ? kWEnd0 : kWEnd1;
+constexpr int kWOffW2 = kWStages1 * kWStage1;
+constexpr int kWOffA2 = kWOffW2 + kWStages2 * kWBlk;
+constexpr int kWOffG = kWOffA2 + kWSlots * kWSlotBytes;
+constexpr int kWOffBar = kWOffG + kWBlk;
 constexpr int kWEpiWarps = 8;
 constexpr int kWThreads = 32 * (5 + kWEpiWarps);
-constexpr int kWSmemBytes = kWOffBar + 1024 + 1024;
+constexpr int kWSmemBytes = kWOffBar + 512 + 1024;
 static_assert(kWSmemBytes <= 232448, "shared memory budget");
-static_assert(kWOffW1 % 1024 == 0 && kWOffW2 % 1024 == 0 && kWOffG % 1024 == 0, "alignment");
+static_assert(kWOffW2 % 1024 == 0 && kWOffA2 % 1024 == 0 && kWOffG % 1024 == 0, "alignment");
+constexpr uint32_t kWAcc1Col = UN;            // acc1[b] at column 256 + 128 b
 constexpr uint32_t kWTmemAlloc = 512;
+constexpr uint32_t kWSlotTx = kWSlotBytes;    // bytes of one slot's copies (8 x 4 KB)
+constexpr uint32_t kWPieceBytes = 32 * 128;   // one epilogue warp's rows of one K block
 
 struct WBars {
-  // pair 0
-  uint64_t zfull[kWMaxZ];        // Z block landed (leader; both CTAs' bytes)
-  uint64_t zempty;               // the tile's last GEMM1 done with Z (commit, pair 0)
-  uint64_t w1full[kWStagesW1], w1empty[kWStagesW1];
-  uint64_t a1full[kWAcc1];       // GEMM1 of a chunk done (commit, pair 0)
-  uint64_t acc1free[kWAcc1];     // its accumulator read out (pair-0 leader; 2 x 8 arrivals)
-  uint64_t slotfree[kWSlots];    // pair 1's GEMM2 done with the slot (commit, arrives in pair 0)
-  // pair 1
-  uint64_t a2full[kWSlots];      // a chunk's A2 written into both pair-1 CTAs (pair-1 leader;
-                                 // 2 x 8 warp arrivals from pair 0)
-  uint64_t w2full[kWStagesW2], w2empty[kWStagesW2];
-  uint64_t gfull, gempty;
-  uint64_t acc2full;             // a tile's GEMM2 + bias done (commit, pair 1)
-  uint64_t acc2empty;            // acc2 read out (pair-1 leader; 2 x 8 arrivals)
-  uint64_t drain;
+  uint64_t zfull[kWStages1], zempty[kWStages1];   // source / W1 ring
+  uint64_t w2full[kWStages2], w2empty[kWStages2]; // W2 ring
+  uint64_t gfull, gempty;                         // gate16 rows of the tile
+  uint64_t a1full[2];     // GEMM1 of an own chunk done (commit, both CTAs of the pair)
+  uint64_t acc1free[2];   // its acc1 read out (pair leader; 2 x 8 warp arrivals)
+  uint64_t epidone[kWSlots];  // this CTA's A2 rows of an own chunk written (8 warp arrivals)
+  uint64_t rx[kWSlots];       // the other pair's chunk copied in (1 arrival + 8 x 4 KB)
+  uint64_t a2full[kWSlots];   // both CTAs' rows of a chunk present (pair leader; 2 arrivals)
+  uint64_t slotfree[kWSlots]; // every pair's GEMM2 of the slot's chunk done (kWPairs commits;
+                              // waited only by the slot's writers, at every use)
+  uint64_t acc2full;      // a tile's GEMM2 + bias done (commit, both CTAs of the pair)
+  uint64_t acc2empty;     // acc2 read out (pair leader; 2 x 8 warp arrivals)
+  uint64_t drain, drain2;
   uint32_t tmem_slot;
   int abort_flag;
 };
-static_assert(sizeof(WBars) <= 1024, "barrier block");
+static_assert(sizeof(WBars) <= 512, "barrier block");
 
 struct WideArgs {
   PathArgs p;
@@ -107,6 +108,15 @@ __device__ __forceinline__ void wide_spin(long long cycles) {
   }
 }
 
+// Row r's 16-byte chunks 4 s .. 4 s + 3 of a 64-wide K block at `blk` (128B swizzle).
+__device__ __forceinline__ void wide_store_a2(uint32_t blk, int r, int s, const uint32_t (&pk)[16]) {
+  const uint32_t row = blk + static_cast<uint32_t>(r * 128);
+#pragma unroll
+  for (int v = 0; v < 4; ++v)
+    st_shared_v4(row + static_cast<uint32_t>(((4 * s + v) ^ (r & 7)) << 4), pk[4 * v],
+                 pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+}
+
 __device__ __forceinline__ void wide_gelu_cols(const uint32_t (&acc)[32], const uint4 (&b)[4],
                                                __half2 half_g, uint32_t (&pk)[16]) {
 #pragma unroll
@@ -118,17 +128,6 @@ __device__ __forceinline__ void wide_gelu_cols(const uint32_t (&acc)[32], const 
       pk[4 * v + k] = gelu_gate_pair(acc[j], acc[j + 1], bw[k], half_g);
     }
   }
-}
-
-// Row r's 16-byte chunks 4 s .. 4 s + 3 of a 64-wide K block at cluster
-// address `blk` (128B swizzle), in another CTA's shared memory.
-__device__ __forceinline__ void wide_store_a2_remote(uint32_t blk, int r, int s,
-                                                     const uint32_t (&pk)[16]) {
-  const uint32_t row = blk + static_cast<uint32_t>(r * 128);
-#pragma unroll
-  for (int v = 0; v < 4; ++v)
-    st_cluster_v4(row + static_cast<uint32_t>(((4 * s + v) ^ (r & 7)) << 4), pk[4 * v],
-                  pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
 }
 
 __device__ __forceinline__ void wide_store_out(const uint32_t (&acc)[32], __nv_bfloat16* o) {
@@ -149,6 +148,10 @@ __global__ void __cluster_dims__(kWCtas, 1, 1) __launch_bounds__(kWThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
+  uint8_t* sZW = smem;
+  uint8_t* sW2 = smem + kWOffW2;
+  uint8_t* sA2 = smem + kWOffA2;
+  uint8_t* sG = smem + kWOffG;
   WBars* bars = reinterpret_cast<WBars*>(smem + kWOffBar);
   volatile int* abort_flag = &bars->abort_flag;
 
@@ -157,35 +160,38 @@ __global__ void __cluster_dims__(kWCtas, 1, 1) __launch_bounds__(kWThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = cluster_ctarank();
   const uint32_t half = rank & 1u;            // which 128 rows of the pair tile
-  const uint32_t pr = rank >> 1;              // 0: GEMM1 pair, 1: GEMM2 pair
+  const uint32_t pr = rank >> 1;              // which CTA pair: output columns 256 pr ..
+  const uint32_t lead = rank & ~1u;           // the pair's leader CTA
   const bool leader = half == 0;
-  constexpr uint16_t kMask0 = 0x3, kMask1 = 0xC;   // the CTAs of pair 0 / pair 1
+  const uint16_t pair_mask = static_cast<uint16_t>(3u << (2 * pr));
+  const uint16_t all_mask = static_cast<uint16_t>((1u << kWCtas) - 1u);
   const int nc = wa.nc, nk1 = wa.nk1;
 
   if (threadIdx.x == 0) {
-    for (int i = 0; i < kWMaxZ; ++i) mbar_init(&bars->zfull[i], 1);
-    mbar_init(&bars->zempty, 1);
-    for (int i = 0; i < kWStagesW1; ++i) {
-      mbar_init(&bars->w1full[i], 1);
-      mbar_init(&bars->w1empty[i], 1);
+    for (int i = 0; i < kWStages1; ++i) {
+      mbar_init(&bars->zfull[i], 1);
+      mbar_init(&bars->zempty[i], 1);
     }
-    for (int i = 0; i < kWAcc1; ++i) {
-      mbar_init(&bars->a1full[i], 1);
-      mbar_init(&bars->acc1free[i], 2 * kWEpiWarps);
-    }
-    for (int i = 0; i < kWSlots; ++i) {
-      mbar_init(&bars->slotfree[i], 1);
-      mbar_init(&bars->a2full[i], 2 * kWEpiWarps);
-    }
-    for (int i = 0; i < kWStagesW2; ++i) {
+    for (int i = 0; i < kWStages2; ++i) {
       mbar_init(&bars->w2full[i], 1);
       mbar_init(&bars->w2empty[i], 1);
     }
     mbar_init(&bars->gfull, 1);
     mbar_init(&bars->gempty, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&bars->a1full[i], 1);
+      mbar_init(&bars->acc1free[i], 2 * kWEpiWarps);
+    }
+    for (int i = 0; i < kWSlots; ++i) {
+      mbar_init(&bars->epidone[i], kWEpiWarps);
+      mbar_init(&bars->rx[i], 1);
+      mbar_init(&bars->a2full[i], 2);
+      mbar_init(&bars->slotfree[i], kWPairs);
+    }
     mbar_init(&bars->acc2full, 1);
     mbar_init(&bars->acc2empty, 2 * kWEpiWarps);
     mbar_init(&bars->drain, 1);
+    mbar_init(&bars->drain2, 1);
     bars->abort_flag = 0;
     fence_barrier_init();
   }
@@ -210,22 +216,20 @@ __global__ void __cluster_dims__(kWCtas, 1, 1) __launch_bounds__(kWThreads, 1)
   const int n_mp = (n_m + 1) / 2;
   const int total = p.gp * n_mp;
   const int cl = blockIdx.x / kWCtas, n_cl = gridDim.x / kWCtas;
+  // own chunks of a tile: c = pr, pr + kWPairs, ...
+  const int n_own = (nc - static_cast<int>(pr) + kWPairs - 1) / kWPairs;
 
-  // unwinding state: loads in flight (bit i: zfull 0-7, w1full 8-19, w2full 20-22, gfull 23)
+  // unwinding state: loads in flight (bit i: zfull 0-2, w2full 3-4, gfull 5)
   uint32_t pend_mask = 0, pend_par = 0;
-  auto note = [&](int bit, uint32_t ph) {
-    pend_mask |= 1u << bit;
-    pend_par = (pend_par & ~(1u << bit)) | (ph << bit);
-  };
   bool mma_issued = false;
 
-  if (pr == 0 && warp == 0) {
+  if (warp == 0) {
     if (lane == 0) {
-      // ------------------------------------------------ Z and W1 loads (pair 0)
+      // ------------------------------------------------ source / W1 loads (own chunks)
       int s = 0;
-      uint32_t ph = 0, k = 0;
+      uint32_t ph = 0;
       bool ok = true;
-      for (int t = cl; ok && t < total; t += n_cl, ++k) {
+      for (int t = cl; ok && t < total; t += n_cl) {
         const int gl = t / n_mp, mp = t - gl * n_mp;
         const int grp = p.g0 + gl;
         const GroupInfo gi = p.groups[grp];
@@ -237,50 +241,40 @@ __global__ void __cluster_dims__(kWCtas, 1, 1) __launch_bounds__(kWThreads, 1)
           ti.b = 0;
           ti.s0 = 0;
         }
-        // chunk 0's W1 blocks first (they only need free ring stages), then Z
-        // once the previous tile's last GEMM1 is done with it, then the rest
-        for (int c = 0; ok && c < nc; ++c) {
-          if (c == 1 || nc == 1) {
-            if (!mbar_wait(&bars->zempty, (k & 1u) ^ 1u, abort_flag, p.wait_limit)) {
-              ok = false;
-              break;
-            }
-            const int zrow = ((gi.src_layer * d.B + ti.b) * d.H_s) * d.S + ti.s0;
-            for (int kb = 0; kb < nk1; ++kb) {
-              if (leader) mbar_arrive_expect_tx(&bars->zfull[kb], 2 * kWBlk);
-              const int kk = kb * UK, h = kk / d.d_s, d0 = kk - h * d.d_s;
-              tma_load_2d_pair(smem + kb * kWBlk, gi.x ? &tmV : &tmK,
-                               leader_addr(&bars->zfull[kb]), d0, zrow + h * d.S);
-              note(kb, k & 1u);
-            }
-          }
+        const int zrow = ((gi.src_layer * d.B + ti.b) * d.H_s) * d.S + ti.s0;
+        for (int c = static_cast<int>(pr); ok && c < nc; c += kWPairs) {
           const int wrow = grp * d.EH + c * kWChunk + static_cast<int>(half) * (kWChunk / 2);
           for (int kb = 0; kb < nk1; ++kb) {
-            if (!mbar_wait(&bars->w1empty[s], ph ^ 1u, abort_flag, p.wait_limit)) { ok = false; break; }
-            if (leader) mbar_arrive_expect_tx(&bars->w1full[s], 2 * kWW1Blk);
-            tma_load_2d_pair(smem + kWOffW1 + s * kWW1Blk, &tmW1q, leader_addr(&bars->w1full[s]),
-                             kb * UK, wrow);
-            note(kWMaxZ + s, ph);
-            if (++s == kWStagesW1) { s = 0; ph ^= 1u; }
+            if (!mbar_wait(&bars->zempty[s], ph ^ 1u, abort_flag, p.wait_limit)) { ok = false; break; }
+            if (leader) mbar_arrive_expect_tx(&bars->zfull[s], 2 * kWStage1);
+            const uint32_t bar = leader_addr(&bars->zfull[s]);
+            const int kk = kb * UK, h = kk / d.d_s, d0 = kk - h * d.d_s;
+            uint8_t* st = sZW + s * kWStage1;
+            tma_load_2d_pair(st, gi.x ? &tmV : &tmK, bar, d0, zrow + h * d.S);
+            tma_load_2d_pair(st + kWBlk, &tmW1q, bar, kk, wrow);
+            pend_mask |= 1u << s;
+            pend_par = (pend_par & ~(1u << s)) | (ph << s);
+            if (++s == kWStages1) { s = 0; ph ^= 1u; }
           }
         }
       }
     }
-  } else if (pr == 1 && warp == 1) {
+  } else if (warp == 1) {
     if (lane == 0) {
-      // ------------------------------------------------ W2 ring, b2t and gate16 loads (pair 1)
+      // ------------------------------------------------ W2 ring, b2t and gate16 loads
       int s = 0;
       uint32_t ph = 0, k = 0;
       bool ok = true;
-      const int wrow = static_cast<int>(half) * UM;   // this CTA's rows of each 256-column half
-      auto stage = [&]() -> uint32_t {
+      const int wrow0 = static_cast<int>(pr) * UN + static_cast<int>(half) * UM;
+      auto w2_stage = [&]() -> uint32_t {
         if (!mbar_wait(&bars->w2empty[s], ph ^ 1u, abort_flag, p.wait_limit)) return 0;
-        if (leader) mbar_arrive_expect_tx(&bars->w2full[s], 2 * kWW2Stage);
+        if (leader) mbar_arrive_expect_tx(&bars->w2full[s], 2 * kWBlk);
         return leader_addr(&bars->w2full[s]);
       };
-      auto next = [&]() {
-        note(kWMaxZ + kWStagesW1 + s, ph);
-        if (++s == kWStagesW2) { s = 0; ph ^= 1u; }
+      auto w2_next = [&]() {
+        pend_mask |= 1u << (kWStages1 + s);
+        pend_par = (pend_par & ~(1u << (kWStages1 + s))) | (ph << (kWStages1 + s));
+        if (++s == kWStages2) { s = 0; ph ^= 1u; }
       };
       for (int t = cl; ok && t < total; t += n_cl, ++k) {
         const int gl = t / n_mp, mp = t - gl * n_mp;
@@ -288,31 +282,56 @@ __global__ void __cluster_dims__(kWCtas, 1, 1) __launch_bounds__(kWThreads, 1)
         const int m_own = 2 * mp + static_cast<int>(half);
         for (int c = 0; ok && c < nc; ++c)
           for (int kb = 0; kb < 2; ++kb) {
-            const uint32_t bar = stage();
+            const uint32_t bar = w2_stage();
             if (!bar) { ok = false; break; }
-            uint8_t* st = smem + kWOffW2 + s * kWW2Stage;
-            for (int n = 0; n < 2; ++n)
-              tma_load_2d_pair(st + n * kWBlk, &tmW2h, bar, c * kWChunk + kb * UK,
-                               grp * d.Dt + n * UN + wrow);
-            next();
+            tma_load_2d_pair(sW2 + s * kWBlk, &tmW2h, bar, c * kWChunk + kb * UK,
+                             grp * d.Dt + wrow0);
+            w2_next();
           }
         if (!ok) break;
-        {   // the bias block's B: b2t rows of both halves
-          const uint32_t bar = stage();
+        // the tile's bias block: B = b2t rows of this pair's columns, A = gate16 rows
+        {
+          const uint32_t bar = w2_stage();
           if (!bar) break;
-          uint8_t* st = smem + kWOffW2 + s * kWW2Stage;
-          for (int n = 0; n < 2; ++n)
-            tma_load_2d_pair(st + n * kWBlk, &tmB2th, bar, 0, grp * d.Dt + n * UN + wrow);
-          next();
+          tma_load_2d_pair(sW2 + s * kWBlk, &tmB2th, bar, 0, grp * d.Dt + wrow0);
+          w2_next();
         }
         if (!mbar_wait(&bars->gempty, (k & 1u) ^ 1u, abort_flag, p.wait_limit)) break;
         if (leader) mbar_arrive_expect_tx(&bars->gfull, 2 * kWBlk);
-        tma_load_3d_pair(smem + kWOffG, &tmG16, leader_addr(&bars->gfull), 0, m_own * UM, grp);
-        note(kWMaxZ + kWStagesW1 + kWStagesW2, k & 1u);
+        tma_load_3d_pair(sG, &tmG16, leader_addr(&bars->gfull), 0, m_own * UM, grp);
+        pend_mask |= 1u << (kWStages1 + kWStages2);
+        pend_par = (pend_par & ~(1u << (kWStages1 + kWStages2))) |
+                   ((k & 1u) << (kWStages1 + kWStages2));
       }
     }
-  } else if (warp == 3 + static_cast<int>(pr) && leader) {
-    // ------------------------------------------------ MMA issue (pair leaders)
+  } else if (warp == 2) {
+    if (lane == 0) {
+      // ------------------------------------------------ relay between the pairs
+      // per slot: uses whose epilogue (own) or copies (other pair) were waited for
+      uint32_t use_n[kWSlots] = {};
+      bool ok = true;
+      for (int t = cl; ok && t < total; t += n_cl) {
+        for (int c = 0; c < nc; ++c) {
+          const int slot = c % kWPairs;
+          if (slot == static_cast<int>(pr)) {
+            if (!mbar_wait(&bars->epidone[slot], use_n[slot] & 1u, abort_flag, p.wait_limit)) {
+              ok = false;
+              break;
+            }
+          } else {
+            mbar_arrive_expect_tx(&bars->rx[slot], kWSlotTx);
+            if (!mbar_wait_cluster(&bars->rx[slot], use_n[slot] & 1u, abort_flag, p.wait_limit)) {
+              ok = false;
+              break;
+            }
+          }
+          ++use_n[slot];
+          mbar_arrive_release_cluster(&bars->a2full[slot], lead);
+        }
+      }
+    }
+  } else if ((warp == 3 || warp == 4) && leader) {
+    // ------------------------------------------------ MMA issuers (pair leader)
     auto wait_all = [&](uint64_t* bar, uint32_t parity) -> bool {
       const bool r = mbar_wait(bar, parity, abort_flag, p.wait_limit);
       return __all_sync(0xffffffffu, r) != 0;
@@ -322,75 +341,69 @@ __global__ void __cluster_dims__(kWCtas, 1, 1) __launch_bounds__(kWThreads, 1)
       return __all_sync(0xffffffffu, r) != 0;
     };
     bool ok = true;
-    if (pr == 0) {
-      // GEMM1: acc1[cg % 4] = Z * W1cat[chunk]^T
+    if (warp == 3) {
+      // GEMM1 of own chunks: acc1[j % 2] = Z * W1cat[chunk]^T
       constexpr uint32_t idesc1 = idesc_bf16_f32(2 * UM, kWChunk);
       int s = 0;
-      uint32_t ph = 0, k = 0, cg = 0;
-      for (int t = cl; ok && t < total; t += n_cl, ++k) {
-        for (int c = 0; ok && c < nc; ++c, ++cg) {
-          const uint32_t b = cg % kWAcc1;
-          if (cg >= kWAcc1) ok = wait_all(&bars->acc1free[b], ((cg / kWAcc1) & 1u) ^ 1u);
+      uint32_t ph = 0, j = 0;
+      for (int t = cl; ok && t < total; t += n_cl) {
+        for (int o = 0; ok && o < n_own; ++o, ++j) {
+          const uint32_t b = j & 1u;
+          if (j >= 2) ok = wait_all(&bars->acc1free[b], ((j >> 1) & 1u) ^ 1u);
           if (!ok) break;
-          const uint32_t d1 = tmem_base + b * kWChunk;
+          const uint32_t d1 = tmem_base + kWAcc1Col + b * kWChunk;
           for (int kb = 0; kb < nk1; ++kb) {
-            if (c == 0 && !wait_all(&bars->zfull[kb], k & 1u)) { ok = false; break; }
-            if (!wait_all(&bars->w1full[s], ph)) { ok = false; break; }
+            if (!wait_all(&bars->zfull[s], ph)) { ok = false; break; }
             tc_fence_after();
+            const uint32_t za = smem_u32(sZW + s * kWStage1);
             if (elect_one()) {
-              const uint64_t zdesc = sdesc_k_sw128(smem_u32(smem + kb * kWBlk));
-              const uint64_t wdesc = sdesc_k_sw128(smem_u32(smem + kWOffW1 + s * kWW1Blk));
+              const uint64_t zdesc = sdesc_k_sw128(za), wdesc = sdesc_k_sw128(za + kWBlk);
 #pragma unroll
               for (int kk = 0; kk < UK / 16; ++kk)   // +32 bytes of K = +2 in the address field
                 umma_pair(d1, zdesc + 2 * kk, wdesc + 2 * kk, idesc1, (kb | kk) != 0);
-              umma_commit_mask(&bars->w1empty[s], kMask0);
+              umma_commit_mask(&bars->zempty[s], pair_mask);
             }
             __syncwarp();
             mma_issued = true;
-            if (++s == kWStagesW1) { s = 0; ph ^= 1u; }
+            if (++s == kWStages1) { s = 0; ph ^= 1u; }
           }
           if (!ok) break;
-          if (elect_one()) {
-            umma_commit_mask(&bars->a1full[b], kMask0);
-            if (c == nc - 1) umma_commit_mask(&bars->zempty, kMask0);
-          }
+          if (elect_one()) umma_commit_mask(&bars->a1full[b], pair_mask);
           __syncwarp();
         }
       }
     } else {
-      // GEMM2: acc2[0, 512) += A2_c * W2cat[:, chunk]^T over every chunk, then the bias block
+      // GEMM2 of every chunk into acc2, then the bias block
       constexpr uint32_t idesc2 = idesc_f16_f32(2 * UM, UN);
       int s = 0;
-      uint32_t ph = 0, k = 0, cg = 0;
+      uint32_t ph = 0, k = 0;
+      uint32_t use_n[kWSlots] = {};
       for (int t = cl; ok && t < total; t += n_cl, ++k) {
-        for (int c = 0; ok && c < nc; ++c, ++cg) {
-          const uint32_t slot = cg % kWSlots, use = cg / kWSlots;
-          ok = wait_all_cluster(&bars->a2full[slot], use & 1u);
+        for (int c = 0; ok && c < nc; ++c) {
+          const int slot = c % kWPairs;
+          ok = wait_all_cluster(&bars->a2full[slot], use_n[slot] & 1u);
+          ++use_n[slot];
           if (ok && c == 0) ok = wait_all(&bars->acc2empty, (k & 1u) ^ 1u);
           if (!ok) break;
-          const uint32_t aa = smem_u32(smem + slot * kWSlotBytes);
+          const uint32_t aa = smem_u32(sA2 + slot * kWSlotBytes);
           for (int kb = 0; kb < 2; ++kb) {
             if (!wait_all(&bars->w2full[s], ph)) { ok = false; break; }
             tc_fence_after();
             if (elect_one()) {
               const uint64_t adesc = sdesc_k_sw128(aa + kb * kWBlk);
-              const uint32_t ba = smem_u32(smem + kWOffW2 + s * kWW2Stage);
+              const uint64_t bdesc = sdesc_k_sw128(smem_u32(sW2 + s * kWBlk));
 #pragma unroll
-              for (int n = 0; n < 2; ++n) {
-                const uint64_t bdesc = sdesc_k_sw128(ba + n * kWBlk);
-#pragma unroll
-                for (int kk = 0; kk < UK / 16; ++kk)
-                  umma_pair(tmem_base + n * UN, adesc + 2 * kk, bdesc + 2 * kk, idesc2,
-                            (c | kb | kk) != 0);
-              }
-              umma_commit_mask(&bars->w2empty[s], kMask1);
+              for (int kk = 0; kk < UK / 16; ++kk)
+                umma_pair(tmem_base, adesc + 2 * kk, bdesc + 2 * kk, idesc2, (c | kb | kk) != 0);
+              umma_commit_mask(&bars->w2empty[s], pair_mask);
             }
             __syncwarp();
             mma_issued = true;
-            if (++s == kWStagesW2) { s = 0; ph ^= 1u; }
+            if (++s == kWStages2) { s = 0; ph ^= 1u; }
           }
           if (!ok) break;
-          if (elect_one()) umma_commit_mask(&bars->slotfree[slot], kMask0);   // pair 0 may refill it
+          // the slot is free once every pair's GEMM2 of this chunk is done
+          if (elect_one()) umma_commit_mask(&bars->slotfree[slot], all_mask);
           __syncwarp();
         }
         if (!ok) break;
@@ -398,126 +411,118 @@ __global__ void __cluster_dims__(kWCtas, 1, 1) __launch_bounds__(kWThreads, 1)
         if (!wait_all(&bars->w2full[s], ph)) break;
         tc_fence_after();
         if (elect_one()) {
-          const uint64_t gdesc = sdesc_k_sw128(smem_u32(smem + kWOffG));
-          const uint32_t ba = smem_u32(smem + kWOffW2 + s * kWW2Stage);
+          const uint64_t gdesc = sdesc_k_sw128(smem_u32(sG));
+          const uint64_t bdesc = sdesc_k_sw128(smem_u32(sW2 + s * kWBlk));
 #pragma unroll
-          for (int n = 0; n < 2; ++n) {
-            const uint64_t bdesc = sdesc_k_sw128(ba + n * kWBlk);
-#pragma unroll
-            for (int kk = 0; kk < UK / 16; ++kk)
-              umma_pair(tmem_base + n * UN, gdesc + 2 * kk, bdesc + 2 * kk, idesc2, 1u);
-          }
-          umma_commit_mask(&bars->w2empty[s], kMask1);
-          umma_commit_mask(&bars->gempty, kMask1);
-          umma_commit_mask(&bars->acc2full, kMask1);
+          for (int kk = 0; kk < UK / 16; ++kk)
+            umma_pair(tmem_base, gdesc + 2 * kk, bdesc + 2 * kk, idesc2, 1u);
+          umma_commit_mask(&bars->w2empty[s], pair_mask);
+          umma_commit_mask(&bars->gempty, pair_mask);
+          umma_commit_mask(&bars->acc2full, pair_mask);
         }
         __syncwarp();
-        if (++s == kWStagesW2) { s = 0; ph ^= 1u; }
+        if (++s == kWStages2) { s = 0; ph ^= 1u; }
       }
     }
   } else if (warp >= 5) {
+    // ------------------------------------------------ epilogue (every CTA)
     const int e = warp - 5, q = warp & 3, hh = e >> 2;   // q: the TMEM lane quarter warp % 4 may access
     const int r = q * 32 + lane;
     const uint32_t tq = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+    const __half* b1h = static_cast<const __half*>(p.b1h);
+    uint32_t j = 0, k = 0;   // j: own chunks so far = uses of this pair's slot
     bool ok = true;
-    if (pr == 0) {
-      // ------------------------------------------------ chunk epilogue (pair 0)
-      const __half* b1h = static_cast<const __half*>(p.b1h);
-      const uint32_t peer = rank + 2u;   // the pair-1 CTA with the same token rows
-      const uint32_t a2_remote = mapa_cluster(smem, peer);
-      uint32_t cg = 0;
-      for (int t = cl; ok && t < total; t += n_cl) {
-        const int gl = t / n_mp, mp = t - gl * n_mp;
-        const int grp = p.g0 + gl;
-        const int m_own = 2 * mp + static_cast<int>(half);
-        const bool valid = m_own < n_m;
-        const float* grow = p.gate + (static_cast<size_t>(grp) * d.tpad +
-                                      static_cast<size_t>(m_own) * UM + r) * d.E;
-        const uint4* bias4 = reinterpret_cast<const uint4*>(b1h + static_cast<size_t>(grp) * d.EH);
-        for (int c = 0; c < nc; ++c, ++cg) {
-          const uint32_t b = cg % kWAcc1, slot = cg % kWSlots, use = cg / kWSlots;
-          // this warp's 2 x 32 biases and the row's gate value, fetched before the wait
-          uint4 bias[2][4];
+    const int slot = static_cast<int>(pr);
+    const uint32_t peer = (rank ^ 2u);   // the other pair's CTA with the same rows (2 pairs)
+    for (int t = cl; ok && t < total; t += n_cl, ++k) {
+      const int gl = t / n_mp, mp = t - gl * n_mp;
+      const int grp = p.g0 + gl;
+      const int m_own = 2 * mp + static_cast<int>(half);
+      const bool valid = m_own < n_m;
+      const float* grow =
+          p.gate + (static_cast<size_t>(grp) * d.tpad + static_cast<size_t>(m_own) * UM + r) * d.E;
+      const uint4* bias4 = reinterpret_cast<const uint4*>(b1h + static_cast<size_t>(grp) * d.EH);
+      for (int c = static_cast<int>(pr); c < nc; c += kWPairs, ++j) {
+        const uint32_t b = j & 1u;
+        // this warp's 2 x 32 biases and the row's gate value, fetched before the wait
+        uint4 bias[2][4];
 #pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            bias[0][i] = __ldg(bias4 + (c * kWChunk + hh * 64) / 8 + i);
-            bias[1][i] = __ldg(bias4 + (c * kWChunk + hh * 64 + 32) / 8 + i);
-          }
-          const float gate = valid ? __ldg(grow + (c * kWChunk) / d.H) : 0.f;
-          int w = 1;
-          if (lane == 0) w = mbar_wait(&bars->a1full[b], (cg / kWAcc1) & 1u, abort_flag, p.wait_limit);
-          if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
-          tc_fence_after();
-          uint32_t pa[16], pb[16];
-          {
-            uint32_t ra[32], rb[32];
-            tmem_ld_32x32b_x32(tq + b * kWChunk + hh * 64, ra);
-            tmem_ld_32x32b_x32(tq + b * kWChunk + hh * 64 + 32, rb);
-            tmem_ld_wait(ra);
-            tmem_ld_wait(rb);
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive_cluster(&bars->acc1free[b], 0);   // GEMM1(cg + 4) may start
-            const __half2 hg = __float2half2_rn(0.5f * gate);
-            wide_gelu_cols(ra, bias[0], hg, pa);
-            wide_gelu_cols(rb, bias[1], hg, pb);
-          }
-          // pair 1's GEMM2 of the slot's previous chunk must be done reading it
-          if (use >= 1) {
-            if (lane == 0)
-              w = mbar_wait_cluster(&bars->slotfree[slot], (use - 1) & 1u, abort_flag, p.wait_limit);
-            if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
-          }
-          const uint32_t blk = a2_remote + slot * kWSlotBytes + static_cast<uint32_t>(hh * kWBlk);
-          wide_store_a2_remote(blk, r, 0, pa);
-          wide_store_a2_remote(blk, r, 1, pb);
-          fence_proxy_async_cluster();   // pair 1's tensor core (async proxy) reads these stores
+        for (int i = 0; i < 4; ++i) {
+          bias[0][i] = __ldg(bias4 + (c * kWChunk + hh * 64) / 8 + i);
+          bias[1][i] = __ldg(bias4 + (c * kWChunk + hh * 64 + 32) / 8 + i);
+        }
+        const float gate = valid ? __ldg(grow + (c * kWChunk) / d.H) : 0.f;
+        int w = 1;
+        if (lane == 0) w = mbar_wait(&bars->a1full[b], (j >> 1) & 1u, abort_flag, p.wait_limit);
+        if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+        tc_fence_after();
+        uint32_t pa[16], pb[16];
+        {
+          uint32_t ra[32], rb[32];
+          tmem_ld_32x32b_x32(tq + kWAcc1Col + b * kWChunk + hh * 64, ra);
+          tmem_ld_32x32b_x32(tq + kWAcc1Col + b * kWChunk + hh * 64 + 32, rb);
+          tmem_ld_wait(ra);
+          tmem_ld_wait(rb);
+          tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive_release_cluster(&bars->a2full[slot], 2u);
+          if (lane == 0) mbar_arrive_cluster(&bars->acc1free[b], lead);   // GEMM1(j + 2) may start
+          const __half2 hg = __float2half2_rn(0.5f * gate);
+          wide_gelu_cols(ra, bias[0], hg, pa);
+          wide_gelu_cols(rb, bias[1], hg, pb);
+        }
+        // every pair's GEMM2 of the slot's previous chunk (use j - 1) must be
+        // done reading it, here and in the other pair's CTA this warp copies to
+        if (j >= 1) {
+          if (lane == 0)
+            w = mbar_wait_cluster(&bars->slotfree[slot], (j - 1) & 1u, abort_flag, p.wait_limit);
+          if (!__shfl_sync(0xffffffffu, w, 0)) { ok = false; break; }
+        }
+        uint8_t* piece = sA2 + slot * kWSlotBytes + hh * kWBlk + q * kWPieceBytes;
+        const uint32_t a2 = smem_u32(sA2 + slot * kWSlotBytes) + static_cast<uint32_t>(hh * kWBlk);
+        wide_store_a2(a2, r, 0, pa);
+        wide_store_a2(a2, r, 1, pb);
+        fence_proxy_async_smem();   // the MMA and the bulk copy (async proxy) read these stores
+        __syncwarp();
+        if (lane == 0) {
+          bulk_copy_to_cta(piece, piece, kWPieceBytes, &bars->rx[slot], peer);
+          mbar_arrive(&bars->epidone[slot]);
         }
       }
-    } else {
-      // ------------------------------------------------ output epilogue (pair 1)
-      uint32_t k = 0;
-      for (int t = cl; t < total; t += n_cl, ++k) {
-        const int gl = t / n_mp, mp = t - gl * n_mp;
-        const int grp = p.g0 + gl;
-        const int m_own = 2 * mp + static_cast<int>(half);
-        const bool valid = m_own < n_m;
-        const GroupInfo gi = p.groups[grp];
-        TileInfo ti;
-        ti.rows = 0;
-        if (valid) ti = p.tiles[m_own];
-        int w = 1;
-        if (lane == 0) w = mbar_wait(&bars->acc2full, k & 1u, abort_flag, p.wait_limit);
-        if (!__shfl_sync(0xffffffffu, w, 0)) break;
-        tc_fence_after();
-        if (valid) {   // warp-uniform: the TMEM loads are warp-collective; stores are per row
-          __nv_bfloat16* const dst = static_cast<__nv_bfloat16*>(gi.x ? p.dst[1] : p.dst[0]);
-          const size_t s_pos = static_cast<size_t>(ti.s0) + r;
-          uint32_t ra[32], rb[32];
+      if (!ok) break;
+      // output: this pair's columns 256 pr + 128 hh .. + 127 of this warp's rows
+      const GroupInfo gi = p.groups[grp];
+      TileInfo ti;
+      ti.rows = 0;
+      if (valid) ti = p.tiles[m_own];
+      int w = 1;
+      if (lane == 0) w = mbar_wait(&bars->acc2full, k & 1u, abort_flag, p.wait_limit);
+      if (!__shfl_sync(0xffffffffu, w, 0)) break;
+      tc_fence_after();
+      if (valid) {   // warp-uniform: the TMEM loads are warp-collective; stores are per row
+        __nv_bfloat16* const dst = static_cast<__nv_bfloat16*>(gi.x ? p.dst[1] : p.dst[0]);
+        const size_t s_pos = static_cast<size_t>(ti.s0) + r;
+        uint32_t ra[32], rb[32];
 #pragma unroll 1
-          for (int cc = hh * UN; cc < (hh + 1) * UN; cc += 64) {
-            tmem_ld_32x32b_x32(tq + cc, ra);
-            tmem_ld_32x32b_x32(tq + cc + 32, rb);
-            tmem_ld_wait(ra);
-            tmem_ld_wait(rb);
-            if (r < ti.rows) {
+        for (int cc = hh * (UN / 2); cc < (hh + 1) * (UN / 2); cc += 64) {
+          tmem_ld_32x32b_x32(tq + cc, ra);
+          tmem_ld_32x32b_x32(tq + cc + 32, rb);
+          tmem_ld_wait(ra);
+          tmem_ld_wait(rb);
+          if (r < ti.rows) {
 #pragma unroll
-              for (int u = 0; u < 2; ++u) {
-                const int col = cc + 32 * u;
-                const int hd = col / d.d_t, i0 = col - hd * d.d_t;
-                __nv_bfloat16* o = dst + ((((static_cast<size_t>(gi.tgt_layer) * d.B + ti.b) *
-                                            d.H_t + hd) * d.S + s_pos) * d.d_t + i0);
-                wide_store_out(u ? rb : ra, o);
-              }
+            for (int u = 0; u < 2; ++u) {
+              const int col = static_cast<int>(pr) * UN + cc + 32 * u;
+              const int hd = col / d.d_t, i0 = col - hd * d.d_t;
+              __nv_bfloat16* o = dst + ((((static_cast<size_t>(gi.tgt_layer) * d.B + ti.b) * d.H_t +
+                                          hd) * d.S + s_pos) * d.d_t + i0);
+              wide_store_out(u ? rb : ra, o);
             }
           }
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive_cluster(&bars->acc2empty, 2);
       }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(&bars->acc2empty, lead);
     }
   }
 
@@ -529,13 +534,11 @@ __global__ void __cluster_dims__(kWCtas, 1, 1) __launch_bounds__(kWThreads, 1)
     // leader also waits for its issued MMAs.
     if ((warp == 0 || warp == 1) && lane == 0 && pend_mask) {
       if (leader) {
-        for (int i = 0; i < kWMaxZ + kWStagesW1 + kWStagesW2 + 1; ++i) {
+        for (int i = 0; i < kWStages1 + kWStages2 + 1; ++i) {
           if (!((pend_mask >> i) & 1u)) continue;
-          uint64_t* fb = i < kWMaxZ ? &bars->zfull[i]
-                       : i < kWMaxZ + kWStagesW1 ? &bars->w1full[i - kWMaxZ]
-                       : i < kWMaxZ + kWStagesW1 + kWStagesW2
-                           ? &bars->w2full[i - kWMaxZ - kWStagesW1]
-                           : &bars->gfull;
+          uint64_t* fb = i < kWStages1 ? &bars->zfull[i]
+                                       : (i < kWStages1 + kWStages2 ? &bars->w2full[i - kWStages1]
+                                                                    : &bars->gfull);
           const uint32_t a = smem_u32(fb);
           const long long t0 = clock64();
           while (!mbar_try_wait(a, (pend_par >> i) & 1u) && clock64() - t0 < p.wait_limit) {
@@ -545,20 +548,22 @@ __global__ void __cluster_dims__(kWCtas, 1, 1) __launch_bounds__(kWThreads, 1)
         wide_spin(20000000LL);
       }
     }
-    if (warp == 3 + static_cast<int>(pr) && leader && mma_issued) {   // drain its MMAs
+    if ((warp == 3 || warp == 4) && leader && mma_issued) {   // each issuing lane drains its MMAs
       if (elect_one()) {
-        umma_commit_mask(&bars->drain, pr ? kMask1 : kMask0);
-        const uint32_t a = smem_u32(&bars->drain);
+        uint64_t* dr = warp == 3 ? &bars->drain : &bars->drain2;
+        umma_commit_mask(dr, pair_mask);
+        const uint32_t a = smem_u32(dr);
         const long long t0 = clock64();
         while (!mbar_try_wait(a, 0) && clock64() - t0 < p.wait_limit) {
         }
       }
       __syncwarp();
     }
+    if (warp >= 5 && lane == 0) wide_spin(20000000LL);   // slot copies in flight land
     __syncthreads();
   }
   tc_fence_before();
-  cluster_sync();   // no CTA's MMAs, stores or arrivals still touch another CTA
+  cluster_sync();   // no CTA's MMAs, copies or arrivals still touch another CTA
   if (warp == 2) {
     tc_fence_after();
     tmem_dealloc_pair(tmem_base, kWTmemAlloc);
@@ -569,8 +574,8 @@ __global__ void __cluster_dims__(kWCtas, 1, 1) __launch_bounds__(kWThreads, 1)
 }  // namespace
 
 bool wide_supported(const Dims& d) {
-  return umma_supported(d) && d.Dt == 2 * UN && d.Ds % UK == 0 && d.Ds <= kWMaxZ * UK &&
-         d.H % kWChunk == 0 && d.d_t % 32 == 0;
+  return umma_supported(d) && d.Dt == kWPairs * UN && d.Ds % UK == 0 && d.H % kWChunk == 0 &&
+         d.d_t % 32 == 0;
 }
 
 cudaError_t launch_wide(const PathArgs& a, const CUtensorMap& tmK, const CUtensorMap& tmV,

@@ -65,10 +65,9 @@ def onchip_supported(wl):
 
 
 def wide_supported(wl):
-    """Shapes the on-chip schedule on clusters of two CTA pairs (4) takes: D_t = 512,
-    D_s <= 512."""
-    d_s, d_t = wl.src_kv_heads * wl.src_head_dim, wl.tgt_kv_heads * wl.tgt_head_dim
-    return (wl.dtype == "bf16" and d_t == 512 and d_s <= 512 and wl.hidden % 256 == 0
+    """Shapes the on-chip schedule on clusters of two CTA pairs (4) takes: D_t = 512."""
+    d_t = wl.tgt_kv_heads * wl.tgt_head_dim
+    return (wl.dtype == "bf16" and d_t == 512 and wl.hidden % 256 == 0
             and wl.src_head_dim % 64 == 0 and wl.tgt_head_dim % 32 == 0)
 
 

@@ -315,6 +315,10 @@ mot_status mot_translate_h(mot_handle h, const void* src_act, const int32_t* seq
  * Both give the translation of Def. 3.1 within rounding. Setting 1 on a
  * handle without top_k < E, without the tensor-core path or with H not a
  * multiple of 256 returns MOT_ERR_UNSUPPORTED.
+ * Backbone handles (mot_create_bt) with top_k = 1 route too, and do so by
+ * default: each backbone runs on the tokens that chose it only (per window
+ * slot their source rows are packed per backbone), with a result bit-identical
+ * to the dense schedule; other top_k values take the dense schedule only.
  */
 mot_status mot_set_routing(mot_handle h, int32_t routing);
 mot_status mot_get_routing(mot_handle h, int32_t* routing);
@@ -324,7 +328,9 @@ mot_status mot_get_routing(mot_handle h, int32_t* routing);
  * the usage metrics of Sec. 4.3): counts[g * E + m] = tokens of translated
  * group g (2 r + x for the r-th translated target layer, x = 0 for K, 1 for
  * V) that chose translator m. n must equal groups * E. Waits for `stream`.
- * MOT_ERR_UNSUPPORTED unless the last translate ran with routing 1.
+ * For a backbone handle, counts[x * E + m] = tokens of block x (K, V) that
+ * chose backbone m, and n must equal 2 * E. MOT_ERR_UNSUPPORTED unless the
+ * last translate ran with routing 1.
  */
 mot_status mot_get_expert_counts(mot_handle h, int32_t* counts, int32_t n, mot_stream_t stream);
 
@@ -373,8 +379,8 @@ mot_status mot_expert_usage(const int32_t* counts, int32_t n, double* cv2, doubl
  * 256), D_t and d_t multiples of 32, E <= 8, N <= 32, every window layer
  * mapped; otherwise MOT_ERR_UNSUPPORTED (MOT_ERR_INVALID_ARG for a window
  * outside [0, L_t) or non-positive sizes). A backbone handle accepts
- * mot_translate_bt only; profiling, launch counts and status calls work as
- * for KV handles. mot_translate_bt has the arguments, layouts, alignment,
+ * mot_translate_bt only; routing (top_k = 1), expert counts, profiling, launch
+ * counts and status calls work as for KV handles. mot_translate_bt has the arguments, layouts, alignment,
  * sequence-length and stream rules of mot_translate.
  */
 typedef struct {

@@ -91,12 +91,39 @@ struct GemmCfg {
 // (skipping the same inactive tiles), so their barrier phases stay in step.
 struct Work {
   int g, b, s0, ntok, j;
-  int tok0;       // kBtOut: first token of the 128-token tile
+  int tok0;       // kBtOut: first token of the 128-token tile (routed: bucket position)
+  int64_t row0;   // the tile's first row in its group's row space
   bool active;
 };
 
+// Items of a launch: dense, groups x row tiles x N tiles; routed, the tiles of
+// every bucket (from the route kernel's prefix sums) x N tiles.
+__device__ __forceinline__ int total_items(const BtArgs& a, const GemmCfg& c) {
+  if (!a.routed) return c.groups * c.row_tiles * c.n_tiles;
+  const int* pre = a.rpre + (c.mode == kBtOut ? a.d.G + 1 : 0);
+  return pre[a.d.G] * c.n_tiles;
+}
+
 __device__ __forceinline__ Work decode(const BtArgs& a, const GemmCfg& c, int item) {
   Work w;
+  if (a.routed) {   // tile of bucket positions of group g
+    const bool out = c.mode == kBtOut;
+    const int* pre = a.rpre + (out ? a.d.G + 1 : 0);
+    const int tile = item / c.n_tiles;
+    w.j = item - tile * c.n_tiles;
+    int g = 0;
+    while (g + 1 < a.d.G && pre[g + 1] <= tile) ++g;
+    w.g = g;
+    const int span = out ? 128 : a.d.tau;
+    const int pos0 = (tile - pre[g]) * span;
+    w.ntok = min(span, a.cnt[g] - pos0);
+    w.tok0 = pos0;
+    w.b = 0;
+    w.s0 = pos0;
+    w.row0 = int64_t(pos0) * a.d.P;
+    w.active = w.ntok > 0;
+    return w;
+  }
   const int per_g = c.row_tiles * c.n_tiles;
   w.g = item / per_g;
   const int rem = item - w.g * per_g;
@@ -121,7 +148,13 @@ __device__ __forceinline__ Work decode(const BtArgs& a, const GemmCfg& c, int it
     w.tok0 = w.b * a.d.S + w.s0;
     w.active = w.s0 < seq_len_of(a, w.b);
   }
+  w.row0 = int64_t(w.tok0) * a.d.P;
   return w;
+}
+
+// Whether token t of a (non-output) tile is a real token.
+__device__ __forceinline__ bool tile_token_valid(const BtArgs& a, const Work& w, int t) {
+  return t < w.ntok && (a.routed || w.s0 + t < seq_len_of(a, w.b));
 }
 
 struct EpiCtx {
@@ -231,18 +264,16 @@ __device__ void epi_row(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
   const BtDims& d = a.d;
   const int mode = e.c->mode;
   const int r = a.slot;
-  const int L = seq_len_of(a, w.b);
   int p, t;
-  if (mode == kBtIn) {   // rows of the 3-D box: head-major within the tile
+  if (mode == kBtIn && !a.routed) {   // rows of the 3-D box: head-major within the tile
     p = row / d.tau;
     t = row - p * d.tau;
   } else {               // rows of the row space: token-major
     t = row / d.P;
     p = row - t * d.P;
   }
-  const bool valid = p < d.P && t < w.ntok && w.s0 + t < L;
-  const int64_t grow =
-      int64_t(w.g) * d.R + (int64_t(w.b) * d.S + w.s0 + t) * d.P + p;   // row of this thread
+  const bool valid = p < d.P && tile_token_valid(a, w, t);
+  const int64_t grow = int64_t(w.g) * d.R + w.row0 + int64_t(t) * d.P + p;   // row of this thread
   float v[D];
   float mean = 0.f, m2 = 0.f;
   if (mode == kBtIn) {
@@ -250,9 +281,11 @@ __device__ void epi_row(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
     float mu = 0.f, rs = 0.f;
     if (valid) {
       const int x = w.g / d.E;
-      const uint16_t* xr = static_cast<const uint16_t*>(a.src[x]) +
-                           (((int64_t(a.src_layer[r]) * d.B + w.b) * d.P + p) * d.S + w.s0 + t) *
-                               d.d_s;
+      const uint16_t* xr =
+          a.routed ? static_cast<const uint16_t*>(a.xs) + grow * d.d_s
+                   : static_cast<const uint16_t*>(a.src[x]) +
+                         (((int64_t(a.src_layer[r]) * d.B + w.b) * d.P + p) * d.S + w.s0 + t) *
+                             d.d_s;
       const uint4* x4 = reinterpret_cast<const uint4*>(xr);
       float s = 0.f;
       for (int c = 0; c < d.d_s / 8; ++c) {
@@ -327,8 +360,8 @@ __device__ void epi_plain(const EpiCtx& e, const Work& w, uint32_t tb, int row, 
   const BtDims& d = a.d;
   const int r = a.slot;
   const int t = row / d.P, p = row - t * d.P;
-  const bool valid = t < w.ntok && w.s0 + t < seq_len_of(a, w.b);
-  const int64_t grow = int64_t(w.g) * d.R + (int64_t(w.b) * d.S + w.s0 + t) * d.P + p;
+  const bool valid = tile_token_valid(a, w, t);
+  const int64_t grow = int64_t(w.g) * d.R + w.row0 + int64_t(t) * d.P + p;
   const int N = c.NT * c.n_tiles;   // output row width
   const float* bias;
   uint16_t* out;
@@ -370,6 +403,63 @@ __device__ void epi_plain(const EpiCtx& e, const Work& w, uint32_t tb, int row, 
 
 // kBtOut: the E backbones' accumulators of this 128-token tile sit side by
 // side (E * NT columns); the gate-weighted sum goes to target layer q0 + r.
+// Routed (Top-1): one bucket's accumulator for 128 of its positions; each row
+// is its token's whole output (gtilde = 1), stored at the token's position.
+__device__ void epi_out_routed(const EpiCtx& e, const Work& w, uint32_t tb, int row, int cg,
+                               int ng) {
+  const BtArgs& a = *e.a;
+  const GemmCfg& c = *e.c;
+  const BtDims& d = a.d;
+  const int g = w.g, x = g / d.E, m = g - x * d.E;
+  const int pos = w.tok0 + row;
+  const bool valid = row < w.ntok;
+  int b = 0, s = 0;
+  float gt = 0.f, mu = 0.f, rs = 0.f;
+  if (valid) {
+    const int tok = a.list[int64_t(g) * d.B * d.S + pos];
+    b = tok / d.S;
+    s = tok - b * d.S;
+    gt = a.gate[(int64_t(x) * d.B * d.S + tok) * d.E + m];
+    const float2* st = a.rstat + int64_t(g) * d.R + int64_t(pos) * d.P;
+    float tm = 0.f;
+    for (int k = 0; k < d.P; ++k) tm += st[k].x;
+    tm /= d.P;
+    float tq = 0.f;
+    for (int k = 0; k < d.P; ++k) {
+      const float2 sk = st[k];
+      tq += sk.y + d.d * (sk.x - tm) * (sk.x - tm);
+    }
+    mu = tm;
+    rs = rsqrtf(tq / (float(d.d) * d.P) + kLnEps);
+  }
+  uint16_t* dst = static_cast<uint16_t*>(a.dst[x]);
+  const int l = d.q0 + a.slot;
+  const float* cbase = a.c_out + int64_t(g) * d.Dt;
+  const float* sbase = a.s_out + int64_t(g) * d.Dt;
+  for (int ch = cg; ch < c.NT / 32; ch += ng) {
+    uint32_t rr[32];
+    __syncwarp();
+    tmem_ld_32x32b_x32(tb + ch * 32, rr);
+    tmem_ld_wait(rr);
+    if (!valid) continue;
+    const int col = w.j * c.NT + ch * 32;
+    float y[32];
+#pragma unroll
+    for (int k = 0; k < 32; ++k) {
+      const float u = fmaf(__uint_as_float(rr[k]) - mu * __ldg(sbase + col + k), rs,
+                           __ldg(cbase + col + k));
+      y[k] = fmaf(gt, gelu_tanh(u), 0.f);
+    }
+    const int hh = col / d.d_t, i0 = col - hh * d.d_t;
+    uint4* o4 = reinterpret_cast<uint4*>(
+        dst + (((int64_t(l) * d.B + b) * d.H_t + hh) * d.S + s) * d.d_t + i0);
+#pragma unroll
+    for (int q8 = 0; q8 < 4; ++q8)
+      o4[q8] = make_uint4(pack2(y[8 * q8], y[8 * q8 + 1]), pack2(y[8 * q8 + 2], y[8 * q8 + 3]),
+                          pack2(y[8 * q8 + 4], y[8 * q8 + 5]), pack2(y[8 * q8 + 6], y[8 * q8 + 7]));
+  }
+}
+
 __device__ void epi_out(const EpiCtx& e, const Work& w, uint32_t tb, int row, int cg, int ng) {
   const BtArgs& a = *e.a;
   const GemmCfg& c = *e.c;
@@ -452,7 +542,7 @@ __global__ void __launch_bounds__(bt_threads(EPI), 1)
   const BtDims& d = a.d;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool is_out = c.mode == kBtOut;
-  const int n_exp = is_out ? d.E : 1;
+  const int n_exp = is_out && !a.routed ? d.E : 1;   // routed: one backbone per bucket
   const int nk = c.K / 64;
   const int acc_cols = n_exp * c.NT;   // one accumulator buffer
 
@@ -483,7 +573,7 @@ __global__ void __launch_bounds__(bt_threads(EPI), 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const int total = c.groups * c.row_tiles * c.n_tiles;
+  const int total = total_items(a, c);
   uint32_t issued_mask = 0, issue_parity = 0;
   bool mma_issued = false;
 
@@ -504,17 +594,21 @@ __global__ void __launch_bounds__(bt_threads(EPI), 1)
           uint8_t* dA = sA + stage * kBtABytes;
           uint8_t* dB = sB + stage * kBtBBytes;
           const int kc = kb * 64;
-          const int64_t row0 = (int64_t(w.b) * d.S + w.s0) * d.P;
+          const int64_t row0 = w.row0;
           switch (c.mode) {
             case kBtIn: {   // K blocks [0, d_s/64): hi weights, then the same source blocks x lo
               const int x = w.g / d.E;
-              tma_load_3d(dA, x ? &tmA2 : &tmA, &full[stage], kc % d.d_s, w.s0,
-                          (a.src_layer[a.slot] * d.B + w.b) * d.P);
+              if (a.routed)   // the bucket's packed source rows (token-major)
+                tma_load_2d(dA, &tmA, &full[stage], kc % d.d_s,
+                            static_cast<int32_t>(int64_t(w.g) * d.R + row0));
+              else
+                tma_load_3d(dA, x ? &tmA2 : &tmA, &full[stage], kc % d.d_s, w.s0,
+                            (a.src_layer[a.slot] * d.B + w.b) * d.P);
               tma_load_2d(dB, &tmB, &full[stage], kc, w.g * c.b_rows_per_g + w.j * c.NT);
               break;
             }
             case kBtOut: {
-              const int g = w.g * d.E + m;
+              const int g = a.routed ? w.g : w.g * d.E + m;
               tma_load_2d(dA, &tmA, &full[stage], kc,
                           static_cast<int32_t>(int64_t(g) * d.B * d.S + w.tok0));
               tma_load_2d(dB, &tmB, &full[stage], kc, g * c.b_rows_per_g + w.j * c.NT);
@@ -589,7 +683,9 @@ __global__ void __launch_bounds__(bt_threads(EPI), 1)
       if constexpr (EPI == 4) {   // the row-norm stages (kBtIn, kBtO, kBtF2)
         epi_row<D>(e, w, tb, row);
       } else {
-        if (c.mode == kBtOut)
+        if (c.mode == kBtOut && a.routed)
+          epi_out_routed(e, w, tb, row, cg, EPI / 4);
+        else if (c.mode == kBtOut)
           epi_out(e, w, tb, row, cg, EPI / 4);
         else
           epi_plain(e, w, tb, row, cg, EPI / 4);
@@ -686,7 +782,7 @@ __global__ void __launch_bounds__(256, 1)
   const BtDims& d = a.d;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_hc = d.df / 128;
-  const int total = c.groups * c.row_tiles;
+  const int total = total_items(a, c);
   if (threadIdx.x == 0) {
     mbar_init(a_full, 1);
     mbar_init(a_empty, 1);
@@ -733,7 +829,7 @@ __global__ void __launch_bounds__(256, 1)
         if (!w.active) continue;
         if (!mbar_wait(a_empty, (tl & 1) ^ 1u, abort_flag, wl)) break;
         mbar_arrive_expect_tx(a_full, F::kA);
-        const int64_t row0 = (int64_t(w.b) * d.S + w.s0) * d.P;
+        const int64_t row0 = w.row0;
         for (int kb = 0; kb < D / 64; ++kb)
           tma_load_2d(sA + kb * 128 * 128, &tmA, a_full, kb * 64,
                       static_cast<int32_t>(int64_t(w.g) * d.R + row0));
@@ -999,6 +1095,84 @@ __global__ void __launch_bounds__(256) bt_gate_kernel(const BtArgs a) {
   }
 }
 
+// ---------------------------------------------------------------- Top-1 routing
+//
+// One CTA of 1024 threads. For each group g = x * E + m, the tokens whose kept
+// gate weight for backbone m is nonzero (with Top-1, exactly the chosen
+// backbone), in token order: every thread counts the choices in its contiguous
+// chunk of token slots, a block scan gives each thread its first bucket
+// position, and the thread writes its tokens there. Then cnt[g] and the tile
+// prefix sums (tau-token tiles, 128-token tiles).
+__global__ void __launch_bounds__(1024) bt_route_kernel(const BtArgs a, int32_t* cnt,
+                                                        int32_t* list, int32_t* rpre) {
+  __shared__ int s_scan[1024];
+  __shared__ int s_cnt[2 * kMaxE];
+  const BtDims& d = a.d;
+  const int T = d.B * d.S;
+  const int tid = threadIdx.x;
+  const int per = (T + 1023) / 1024;
+  const int t0 = min(T, tid * per), t1 = min(T, t0 + per);
+  for (int g = 0; g < d.G; ++g) {
+    const int x = g / d.E, m = g - x * d.E;
+    const float* gx = a.gate + int64_t(x) * T * d.E + m;
+    auto chose = [&](int tok) {
+      const int b = tok / d.S, s = tok - b * d.S;
+      return s < seq_len_of(a, b) && gx[int64_t(tok) * d.E] > 0.f;
+    };
+    int c = 0;
+    for (int tok = t0; tok < t1; ++tok) c += chose(tok) ? 1 : 0;
+    s_scan[tid] = c;
+    __syncthreads();
+    for (int o = 1; o < 1024; o <<= 1) {   // inclusive scan (Hillis-Steele)
+      const int v = tid >= o ? s_scan[tid - o] : 0;
+      __syncthreads();
+      s_scan[tid] += v;
+      __syncthreads();
+    }
+    int off = s_scan[tid] - c;
+    int32_t* lg = list + int64_t(g) * T;
+    for (int tok = t0; tok < t1; ++tok)
+      if (chose(tok)) lg[off++] = tok;
+    if (tid == 1023) s_cnt[g] = s_scan[1023];
+    __syncthreads();
+  }
+  if (tid == 0) {
+    int p0 = 0, p1 = 0;
+    for (int g = 0; g < d.G; ++g) {
+      cnt[g] = s_cnt[g];
+      rpre[g] = p0;
+      rpre[d.G + 1 + g] = p1;
+      p0 += (s_cnt[g] + d.tau - 1) / d.tau;
+      p1 += (s_cnt[g] + 127) / 128;
+    }
+    rpre[d.G] = p0;
+    rpre[2 * d.G + 1] = p1;
+  }
+}
+
+// The source rows of slot a.slot for every bucket position, packed per group:
+// xs[g][pos * P + p] = src[x][pi(t_r)][b][p][s] (16-byte copies).
+__global__ void __launch_bounds__(256) bt_pack_kernel(const BtArgs a, uint4* __restrict__ xs) {
+  const BtDims& d = a.d;
+  const int g = blockIdx.y, x = g / d.E;
+  const int T = d.B * d.S;
+  const int cpr = d.d_s / 8;   // 16-byte chunks per row
+  const int64_t total = int64_t(a.cnt[g]) * d.P * cpr;
+  const uint4* src = static_cast<const uint4*>(a.src[x]);
+  const int32_t* lg = a.list + int64_t(g) * T;
+  const int64_t lbase = int64_t(a.src_layer[a.slot]) * d.B;
+  for (int64_t i = int64_t(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+       i += int64_t(gridDim.x) * blockDim.x) {
+    const int64_t rowi = i / cpr;
+    const int c = static_cast<int>(i - rowi * cpr);
+    const int pos = static_cast<int>(rowi / d.P), p = static_cast<int>(rowi - int64_t(pos) * d.P);
+    const int tok = lg[pos];
+    const int b = tok / d.S, s = tok - b * d.S;
+    xs[(int64_t(g) * d.R + rowi) * cpr + c] =
+        __ldg(src + (((lbase + b) * d.P + p) * d.S + s) * cpr + c);
+  }
+}
+
 // ---------------------------------------------------------------- attention (SIMT)
 //
 // One thread per (query row, head): scores against the token's P key rows
@@ -1015,8 +1189,10 @@ __global__ void __launch_bounds__(256) bt_attn_kernel(const BtArgs a) {
   const int g = blockIdx.y;
   const int64_t id0 = int64_t(blockIdx.x) * blockDim.x;
   const int64_t id = id0 + threadIdx.x;
-  const int64_t n_rows = int64_t(d.B) * d.S * d.P;
+  // routed: the bucket's positions (its rows are packed); dense: every token slot
+  const int64_t n_rows = (a.routed ? int64_t(a.cnt[g]) : int64_t(d.B) * d.S) * d.P;
   const int64_t n_thr = n_rows * d.na;
+  if (id0 >= n_thr) return;
   const int64_t tok0 = (id0 / d.na) / d.P;
   {
     const int64_t last = (id0 + blockDim.x < n_thr ? id0 + blockDim.x : n_thr) - 1;
@@ -1031,8 +1207,10 @@ __global__ void __launch_bounds__(256) bt_attn_kernel(const BtArgs a) {
   const int h = static_cast<int>(id % d.na);
   const int64_t row = id / d.na;
   const int64_t tok = row / d.P;
-  const int b = static_cast<int>(tok / d.S), s = static_cast<int>(tok - int64_t(b) * d.S);
-  if (s >= seq_len_of(a, b)) return;
+  if (!a.routed) {
+    const int b = static_cast<int>(tok / d.S), s = static_cast<int>(tok - int64_t(b) * d.S);
+    if (s >= seq_len_of(a, b)) return;
+  }
   const int P = d.P, D = d.d;
   const float scale = rsqrtf(static_cast<float>(DH));
   const uint16_t* qr = static_cast<const uint16_t*>(a.q) + (int64_t(g) * d.R + row) * D + h * DH;
@@ -1135,6 +1313,22 @@ cudaError_t launch_bt_gate(const BtArgs& a, cudaStream_t st) {
   return cudaGetLastError();
 }
 
+cudaError_t launch_bt_route(const BtArgs& a, int32_t* cnt, int32_t* list, int32_t* rpre,
+                            cudaStream_t st) {
+  if (a.d.G > 2 * kMaxE) return cudaErrorInvalidValue;
+  bt_route_kernel<<<1, 1024, 0, st>>>(a, cnt, list, rpre);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_bt_pack(const BtArgs& a, void* xs, cudaStream_t st) {
+  const BtDims& d = a.d;
+  const int64_t per_g = int64_t(d.B) * d.S * d.P * (d.d_s / 8);
+  const int64_t blocks = (per_g + 255) / 256;
+  dim3 grid(static_cast<unsigned>(blocks < 1024 ? blocks : 1024), d.G);
+  bt_pack_kernel<<<grid, 256, 0, st>>>(a, static_cast<uint4*>(xs));
+  return cudaGetLastError();
+}
+
 cudaError_t launch_bt_attn(const BtArgs& a, cudaStream_t st) {
   const BtDims& d = a.d;
   const int64_t threads = int64_t(d.B) * d.S * d.P * d.na;
@@ -1177,9 +1371,9 @@ cudaError_t launch_bt_gemm(int mode, const BtArgs& a, const CUtensorMap& tmA,
     case kBtF2: c.K = d.df; c.NT = d.d; c.b_rows_per_g = d.d; break;
     case kBtOut: {
       c.K = d.P * d.d;
-      c.groups = 2;
+      c.groups = a.routed ? d.G : 2;   // routed: one bucket (one backbone) per tile
       c.b_rows_per_g = d.Dt;
-      int nt = 256 / d.E;
+      int nt = a.routed ? 256 : 256 / d.E;
       nt -= nt % 32;
       while (nt > 32 && d.Dt % nt) nt -= 32;
       c.NT = nt;

@@ -64,6 +64,15 @@ struct BtArgs {
   float2* rstat;         // [G][R] (mean, M2) of each h_r row over its d values
   int32_t* status;
   long long wait_limit;
+  // Top-1 routing (token buckets): group g's row space holds only the tokens
+  // that chose backbone g % E, packed in token order: row (pos * P + p) for
+  // bucket position pos < cnt[g], whose token slot b * S + s is list[g][pos].
+  int32_t routed;
+  const int32_t* cnt;         // [G] tokens per bucket
+  const int32_t* list;        // [G][B * S] token slot of each bucket position
+  const int32_t* rpre;        // [2][G + 1] prefix sums of row tiles per bucket: tau-token
+                              // tiles, then 128-token tiles (the output projection)
+  const void* xs;             // [G][R][d_s] bf16 source rows of the slot, packed per bucket
 };
 
 // GEMM modes of bt_gemm (the epilogue each one runs).
@@ -79,9 +88,14 @@ enum BtMode : int {
 
 bool bt_supported(const BtDims& d);
 cudaError_t launch_bt_gate(const BtArgs& a, cudaStream_t st);
+// Top-1 routing: bucket lists and tile prefixes from the gate (cnt, list, rpre),
+// then per window slot the bucket tokens' source rows packed into xs.
+cudaError_t launch_bt_route(const BtArgs& a, int32_t* cnt, int32_t* list, int32_t* rpre,
+                            cudaStream_t st);
+cudaError_t launch_bt_pack(const BtArgs& a, void* xs, cudaStream_t st);
 cudaError_t launch_bt_attn(const BtArgs& a, cudaStream_t st);
-// tmA: the mode's A operand map (kBtIn: the source K and V maps, tmA and tmA2);
-// tmB: its weight map.
+// tmA: the mode's A operand map (kBtIn: the source K and V maps, tmA and tmA2;
+// routed, the packed source rows xs in tmA); tmB: its weight map.
 cudaError_t launch_bt_gemm(int mode, const BtArgs& a, const CUtensorMap& tmA,
                            const CUtensorMap& tmA2, const CUtensorMap& tmB, int num_sms,
                            cudaStream_t st);

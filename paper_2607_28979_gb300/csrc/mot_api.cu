@@ -93,13 +93,17 @@ struct BtState {
   void *xz = nullptr, *xq = nullptr, *q = nullptr, *kv = nullptr, *o = nullptr, *xf = nullptr,
        *f = nullptr, *xo = nullptr;
   float2* rstat = nullptr;
+  // Top-1 routing (token buckets): counts, lists, tile prefixes, packed source rows
+  int32_t *rcnt = nullptr, *rlist = nullptr, *rpre = nullptr;
+  void* xs = nullptr;   // [G][R][d_s] bf16
   CUtensorMap tm_win{}, tm_wq{}, tm_wkv{}, tm_wo{}, tm_wf1{}, tm_wf2{}, tm_wout{}, tm_wf1c{};
   CUtensorMap tm_xz{}, tm_xq{}, tm_o{}, tm_xf{}, tm_f{}, tm_xo{};
+  CUtensorMap tm_xs{}, tm_wout_r{};   // routed: packed source rows, W_out with 256-row boxes
 
   void free_all() {
     void* ptrs[] = {wg, bg, s_in, c_in, c_q, c_kv, c_o, c_f1, c_f2, c_out, s_out, ln_q, ln_c,
                     ln_f, win, wq, wkv, wo, wf1, wf2, wout, gate, h, ht, xz, xq, q, kv, o, xf,
-                    f, xo, rstat};
+                    f, xo, rstat, rcnt, rlist, rpre, xs};
     for (void* p : ptrs)
       if (p) cudaFree(p);
   }
@@ -866,6 +870,9 @@ mot_status bt_create(const mot_config* cfg, const mot_bt_config* bc, mot_handle*
       {&bt.xz, G * R * D * 2}, {&bt.xq, G * R * D * 2}, {&bt.q, G * R * D * 2},
       {&bt.kv, G * R * 2 * D * 2}, {&bt.o, G * R * D * 2}, {&bt.xf, G * R * D * 2},
       {&bt.f, G * R * df * 2}, {&bt.xo, G * R * D * 2},
+      {(void**)&bt.rcnt, 64 * 4}, {(void**)&bt.rlist, G * size_t(bd.B) * bd.S * 4},
+      {(void**)&bt.rpre, (2 * G + 2) * 4},
+      {&bt.xs, bd.top_k == 1 ? G * R * bd.d_s * 2 : 16},
       {(void**)&h->status, 16}};
   for (auto& a : allocs) {
     if (cudaMalloc(a.p, std::max<size_t>(a.n, 16)) != cudaSuccess) {
@@ -908,6 +915,13 @@ mot_status bt_create(const mot_config* cfg, const mot_bt_config* bc, mot_handle*
   map2(&bt.tm_xf, bt.xf, D, G * R, 128);
   map2(&bt.tm_f, bt.f, df, G * R, 128);
   map2(&bt.tm_xo, bt.xo, uint64_t(bd.P) * D, G * size_t(bd.B) * bd.S, 128);
+  if (bd.top_k == 1) {   // Top-1 routing (the default for these handles): token buckets
+    uint32_t nt_r = 256;
+    while (nt_r > 32 && bd.Dt % nt_r) nt_r -= 32;
+    map2(&bt.tm_wout_r, bt.wout, uint64_t(bd.P) * D, G * bd.Dt, nt_r);
+    map2(&bt.tm_xs, bt.xs, bd.d_s, G * R, uint32_t(bd.tau * bd.P));
+    h->routing = 1;
+  }
   if (!ok) {
     free_all(h);
     delete h;
@@ -1430,10 +1444,25 @@ mot_status mot_translate_bt(mot_handle h, const void* src_k, const void* src_v,
       return MOT_ERR_CUDA;
   }
   MOT_CUDA_TRY(timed(h, "bt_gate", st, [&] { return launch_bt_gate(a, st); }));
+  // Top-1 routing: each backbone runs on its own tokens only (packed row spaces)
+  const bool routed = h->routing == 1 && d.top_k == 1;
+  if (routed) {
+    a.routed = 1;
+    a.cnt = bt.rcnt;
+    a.list = bt.rlist;
+    a.rpre = bt.rpre;
+    a.xs = bt.xs;
+    MOT_CUDA_TRY(timed(h, "bt_route", st, [&] {
+      return launch_bt_route(a, bt.rcnt, bt.rlist, bt.rpre, st);
+    }));
+  }
   for (int r = 0; r < d.N; ++r) {
     a.slot = r;
+    if (routed)
+      MOT_CUDA_TRY(timed(h, "bt_pack", st, [&] { return launch_bt_pack(a, bt.xs, st); }));
     MOT_CUDA_TRY(timed(h, "bt_in_ln_gelu", st, [&] {
-      return launch_bt_gemm(kBtIn, a, tmK, tmV, bt.tm_win, h->num_sms, st);
+      return routed ? launch_bt_gemm(kBtIn, a, bt.tm_xs, bt.tm_xs, bt.tm_win, h->num_sms, st)
+                    : launch_bt_gemm(kBtIn, a, tmK, tmV, bt.tm_win, h->num_sms, st);
     }));
     MOT_CUDA_TRY(timed(h, "bt_q", st, [&] {
       return launch_bt_gemm(kBtQ, a, bt.tm_xq, bt.tm_xq, bt.tm_wq, h->num_sms, st);
@@ -1458,9 +1487,11 @@ mot_status mot_translate_bt(mot_handle h, const void* src_k, const void* src_v,
       }));
     }
     MOT_CUDA_TRY(timed(h, "bt_out_gelu_combine", st, [&] {
-      return launch_bt_gemm(kBtOut, a, bt.tm_xo, bt.tm_xo, bt.tm_wout, h->num_sms, st);
+      return launch_bt_gemm(kBtOut, a, bt.tm_xo, bt.tm_xo, routed ? bt.tm_wout_r : bt.tm_wout,
+                            h->num_sms, st);
     }));
   }
+  if (routed) h->counts_valid = true;
   return MOT_OK;
 }
 
@@ -1601,7 +1632,8 @@ mot_status mot_replay_attention(mot_handle h, int32_t layer, const void* q, cons
 
 mot_status mot_set_routing(mot_handle h, int32_t routing) {
   if (!h || routing < 0 || routing > 1) return MOT_ERR_INVALID_ARG;
-  if (routing == 1 && !h->sparse_ok) return MOT_ERR_UNSUPPORTED;
+  const bool bt_top1 = h->kind == 2 && h->bt && h->bt->d.top_k == 1;
+  if (routing == 1 && !h->sparse_ok && !bt_top1) return MOT_ERR_UNSUPPORTED;
   h->routing = routing;
   return MOT_OK;
 }
@@ -1613,6 +1645,19 @@ mot_status mot_get_routing(mot_handle h, int32_t* routing) {
 }
 
 mot_status mot_get_expert_counts(mot_handle h, int32_t* counts, int32_t n, mot_stream_t stream) {
+  if (h && h->kind == 2 && h->bt) {   // backbone buckets: [2][E], block x then backbone
+    if (!counts || n != h->bt->d.G) return MOT_ERR_INVALID_ARG;
+    if (!(h->routing == 1 && h->bt->d.top_k == 1 && h->counts_valid)) return MOT_ERR_UNSUPPORTED;
+    if (cudaSetDevice(h->device) != cudaSuccess) return MOT_ERR_CUDA;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (cudaMemcpyAsync(counts, h->bt->rcnt, size_t(n) * 4, cudaMemcpyDeviceToHost, st) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess) {
+      cudaGetLastError();
+      return MOT_ERR_CUDA;
+    }
+    return MOT_OK;
+  }
   if (!h || !counts || n != h->d.G * h->d.E) return MOT_ERR_INVALID_ARG;
   if (!(h->sparse_ok && h->routing == 1 && h->counts_valid)) return MOT_ERR_UNSUPPORTED;
   if (cudaSetDevice(h->device) != cudaSuccess) return MOT_ERR_CUDA;

@@ -140,6 +140,25 @@ def test_bt_full_size_sampled_tokens():
     G.assert_parity(wl, got, ref, f"bt_gpt2s_opt125m ({tb.size} tokens)")
 
 
+def test_bt_full_size_top1_routed_sampled_tokens():
+    """The GPT-2-small -> OPT-125m backbone workload at full size with the
+    paper's default Top-1 of 2 backbones on token buckets."""
+    wl = synth.WORKLOADS["bt_gpt2s_opt125m"].replace(top_k=1)
+    sk, sv, blob = _inputs(wl)
+    run = BtRun(wl, sk, sv, blob)
+    assert M.mot_get_routing(run.h) == 1
+    assert run.translate() == M.MOT_OK
+    assert run.untouched_outside()
+    tb, ts = H.stratified_tokens(wl.seq_lens, 512, seed=6, tile=10)
+    ref = oracle.bt_tokens(wl, sk, sv, blob, tb, ts)
+    dense = _dense_gate(wl, sk, sv, blob, tb, ts)
+    clear = _clear(wl, dense)
+    assert clear.mean() > 0.99
+    got = run.gather(tb, ts)
+    for X in range(2):
+        G.assert_parity(wl, got[:, X][:, clear[X]], ref[:, X][:, clear[X]], f"Top-1 X={X}")
+
+
 def test_bt_qwen_shapes_sampled_tokens():
     wl = synth.WORKLOADS["bt_qwen05_qwen15"].replace(max_batch=2, max_seq=1024,
                                                      seq_lens=(1024, 700))
@@ -188,21 +207,70 @@ def test_bt_batch_prefix_and_length_clamp():
     assert run2.untouched_outside(lens=[50, 7])
 
 
-def test_bt_launch_sequence_and_profile():
+@pytest.mark.parametrize("routing", [1, 0])
+def test_bt_launch_sequence_and_profile(routing):
+    """Dense: the gate, then 7 launches per window slot. Top-1 routing (token
+    buckets, the default for a Top-1 handle): the gate and the route kernel, then
+    per slot the bucket tokens' source rows are packed before the 7 stages."""
     wl = SMALL_BT["bt_p2_top1"]
     sk, sv, blob = _inputs(wl)
     run = BtRun(wl, sk, sv, blob)
+    assert M.mot_get_routing(run.h) == 1   # the default for top_k = 1
+    M.mot_set_routing(run.h, routing)
     M.mot_profile_enable(run.h, True)
     c0 = M.mot_get_launch_count(run.h)
     assert run.translate() == M.MOT_OK
     N, d_f = wl.bt[1], wl.bt[4]
     fused = d_f % 128 == 0   # FFN1 + GELU + FFN2 in one kernel
-    assert M.mot_get_launch_count(run.h) - c0 == 1 + (7 if fused else 8) * N
+    per_slot = (7 if fused else 8) + (1 if routing else 0)
+    assert M.mot_get_launch_count(run.h) - c0 == 1 + routing + per_slot * N
     prof = M.mot_profile_read(run.h)
     ffn = {"bt_ffn_fused"} if fused else {"bt_ffn1_gelu", "bt_ffn2_residual_ln"}
+    routed = {"bt_route", "bt_pack"} if routing else set()
     assert set(prof) == {"bt_gate", "bt_in_ln_gelu", "bt_q", "bt_kv", "bt_attn",
-                         "bt_o_residual_ln", "bt_out_gelu_combine"} | ffn
+                         "bt_o_residual_ln", "bt_out_gelu_combine"} | ffn | routed
     assert prof["bt_gate"][0] == 1 and prof["bt_q"][0] == N
+
+
+ROUTED = {
+    "bt_p2_top1": SMALL_BT["bt_p2_top1"],
+    # P = 12 (120-row tiles of 10 tokens), Top-1 of 3, ragged with an empty sequence
+    "bt_p12_top1": W("bt_p12_top1", 6, 12, 64, 6, 12, 64, 3, 0, 3, 50, "bf16", (50, 23, 0),
+                     top_k=1, bt=(1, 3, 128, 4, 512)),
+    # FFN 768 (unfused FFN, three N tiles), P = 1, Top-1 of 2
+    "bt_p1_top1": W("bt_p1_top1", 4, 1, 64, 4, 1, 64, 2, 0, 2, 200, "bf16", (200, 131),
+                    top_k=1, bt=(3, 1, 128, 2, 768)),
+}
+
+
+@pytest.mark.parametrize("name", sorted(ROUTED))
+def test_bt_top1_token_buckets_equal_dense_and_oracle(name):
+    """Top-1 of E (Def. 3.1 with backbone experts): running each backbone only on
+    the tokens that chose it (token buckets) gives bit for bit the dense result
+    (every backbone on every token, the unchosen weighted by zero), and both
+    match the oracle; the bucket sizes are the oracle's choice counts."""
+    wl = ROUTED[name]
+    sk, sv, blob = _inputs(wl, 8)
+    runs = []
+    for routing in (1, 0):
+        run = BtRun(wl, sk, sv, blob)
+        M.mot_set_routing(run.h, routing)
+        assert run.translate() == M.MOT_OK
+        assert run.untouched_outside()
+        runs.append(run)
+    assert torch.equal(G.int_view(runs[0].dk), G.int_view(runs[1].dk))
+    assert torch.equal(G.int_view(runs[0].dv), G.int_view(runs[1].dv))
+    tb, ts = _all_tokens(wl.seq_lens)
+    ref, gate = oracle.bt_tokens(wl, sk, sv, blob, tb, ts, want_gate=True)
+    got = runs[0].gather(tb, ts)
+    dense = _dense_gate(wl, sk, sv, blob, tb, ts)
+    clear = _clear(wl, dense)
+    for X in range(2):
+        G.assert_parity(wl, got[:, X][:, clear[X]], ref[:, X][:, clear[X]], f"{name} X={X}")
+    counts = M.mot_get_expert_counts(runs[0].h, 2, wl.n_translators)
+    want = np.stack([(gate[X] > 0).sum(axis=0) for X in range(2)])
+    assert (np.abs(counts - want) <= (~clear).sum(axis=1)[:, None]).all(), (counts, want)
+    assert counts.sum() == 2 * tb.size
 
 
 def test_bt_argument_errors():

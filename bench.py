@@ -485,7 +485,9 @@ class _Setup:
         if M.mot_get_routing(self.h) == M.ROUTING_SPARSE:
             sched = "routed (Top-K token buckets)"
         if wl.is_bt:
-            sched = "backbone scan (7 launches per window slot)"
+            sched = ("backbone scan on Top-1 token buckets (8 launches per window slot)"
+                     if M.mot_get_routing(self.h) == 1 else
+                     "backbone scan (7 launches per window slot)")
         self.schedule = sched
         self.bf = wl.dtype == "bf16"
         tdt = torch.bfloat16 if self.bf else torch.float32

@@ -218,15 +218,16 @@ WORKLOADS.update({
 })
 
 # Backbone-translator (App. C.2) counterparts: a channel window of about 0.3 of
-# the layers (the paper's default ratio), N_Tr = 2 backbones, rows of width 128
-# with 4 attention heads and an FFN of 512.
+# the layers (the paper's default ratio), N_Tr = 2 backbones with Top-1 routing
+# (the paper's default (Top-K, N_Tr) = (1, 2)), rows of width 128 with 4
+# attention heads and an FFN of 512.
 WORKLOADS.update({
     # GPT-2-small -> OPT-125m (12x64 -> 12x64): window = target layers 4..7.
     "bt_gpt2s_opt125m": Workload("bt_gpt2s_opt125m", 12, 12, 64, 12, 12, 64, 2, 0, 8, 1024,
-                                 "bf16", (1024,) * 8, bt=(4, 4, 128, 4, 512)),
+                                 "bf16", (1024,) * 8, top_k=1, bt=(4, 4, 128, 4, 512)),
     # Qwen2.5-0.5B (24L, 2x64) -> Qwen2.5-1.5B (28L, 2x128): window = target layers 10..17.
     "bt_qwen05_qwen15": Workload("bt_qwen05_qwen15", 24, 2, 64, 28, 2, 128, 2, 0, 4, 4096,
-                                 "bf16", (4096,) * 4, bt=(10, 8, 128, 4, 512)),
+                                 "bf16", (4096,) * 4, top_k=1, bt=(10, 8, 128, 4, 512)),
 })
 
 # Order in which the workloads are listed in the build's benchmark configuration.

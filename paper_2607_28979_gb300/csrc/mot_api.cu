@@ -245,6 +245,7 @@ int kind_id(mot_ctx* h, const char* name) {
 // Launch wrapper: counts the launch and, when profiling, brackets it with events.
 template <class F>
 cudaError_t timed(mot_ctx* h, const char* name, cudaStream_t st, F&& launch) {
+  NvtxRange range(name);
   Ev ev{};
   if (h->profile) {
     if (!h->ev_free.empty()) {
@@ -1149,6 +1150,7 @@ mot_status mot_load_weights(mot_handle h, const void* host_blob, size_t bytes) {
 mot_status mot_translate(mot_handle h, const void* src_k, const void* src_v,
                          const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
                          mot_stream_t stream) {
+  NvtxRange range("mot_translate");
   mot_status s = check_translate_args(h, src_k, src_v, seq_lens, batch, dst_k, dst_v);
   if (s != MOT_OK) return s;
   return run_translate(h, src_k, src_v, seq_lens, batch, dst_k, dst_v,
@@ -1158,6 +1160,7 @@ mot_status mot_translate(mot_handle h, const void* src_k, const void* src_v,
 mot_status mot_translate_host(mot_handle h, const void* src_k, const void* src_v,
                               const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
                               mot_stream_t stream) {
+  NvtxRange range("mot_translate_host");
   if (!h || h->kind != 0) return MOT_ERR_INVALID_ARG;   // MoT-h handles: mot_translate_h
   if (batch < 0 || batch > h->d.B) return MOT_ERR_INVALID_ARG;
   if (!src_k || !src_v || !dst_k || !dst_v || (batch > 0 && !seq_lens)) return MOT_ERR_INVALID_ARG;
@@ -1358,6 +1361,7 @@ mot_status mot_get_launch_count(mot_handle h, int64_t* count) {
 
 mot_status mot_translate_h(mot_handle h, const void* src_act, const int32_t* seq_lens,
                            int32_t batch, void* dst_k, void* dst_v, mot_stream_t stream) {
+  NvtxRange range("mot_translate_h");
   if (!h || h->kind != 1) return MOT_ERR_INVALID_ARG;
   const Dims& d = h->d;
   if (batch < 0 || batch > d.B) return MOT_ERR_INVALID_ARG;
@@ -1399,6 +1403,7 @@ mot_status mot_create_bt(const mot_config* cfg, const mot_bt_config* bt, mot_han
 mot_status mot_translate_bt(mot_handle h, const void* src_k, const void* src_v,
                             const int32_t* seq_lens, int32_t batch, void* dst_k, void* dst_v,
                             mot_stream_t stream) {
+  NvtxRange range("mot_translate_bt");
   if (!h || h->kind != 2) return MOT_ERR_INVALID_ARG;
   const Dims& dd = h->d;
   if (batch < 0 || batch > dd.B) return MOT_ERR_INVALID_ARG;
@@ -1589,6 +1594,7 @@ mot_status mot_replay_select(mot_handle h, const void* guide, const int32_t* seq
 mot_status mot_replay_attention(mot_handle h, int32_t layer, const void* q, const void* k,
                                 const void* v, const void* guide, const int32_t* seq_lens,
                                 int32_t batch, void* out, mot_stream_t stream) {
+  NvtxRange range("mot_replay_attention");
   ReplayArgs a;
   mot_status r = replay_args(h, q, k, v, guide, seq_lens, batch, out, true, a);
   if (r != MOT_OK) return r;

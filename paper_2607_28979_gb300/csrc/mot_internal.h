@@ -7,7 +7,19 @@
 
 #include "mot.h"
 
+#include <nvtx3/nvToolsExt.h>
+
 namespace mot {
+
+// NVTX range over a scope (host code): the entry points and every kernel
+// launch are named for nsys / ncu NVTX filtering. Without a tool attached the
+// push and pop are a null-pointer check each.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 constexpr int kTileM = 128;   // tokens per token tile (rows of one MMA tile)
 constexpr int kMaxE = 16;     // translators per (layer, K/V) group

@@ -352,17 +352,19 @@ def test_target_cache_aligned_to_16_but_not_32_bytes(lead):
 
 
 def test_onchip_schedule_is_refused_where_unsupported():
-    """D_t != 256: the default stays 2 and asking for 3 is MOT_ERR_UNSUPPORTED."""
+    """D_t = 256 with D_s = 256: the default stays 2, asking for 3 (D_s <= 128) or
+    4 (D_t = 512) is MOT_ERR_UNSUPPORTED, and 5 is not a schedule."""
     wl = SMALL["umma_e1"]
     sk, sv, blob = inputs(wl, seed=11)
     run = G.Run(wl, sk, sv, blob)
     assert M.mot_get_schedule(run.h) == 2
-    with pytest.raises(M.MotError) as e:
-        M.mot_set_schedule(run.h, 3)
-    assert e.value.status == M.MOT_ERR_UNSUPPORTED
+    for sched in (3, 4):
+        with pytest.raises(M.MotError) as e:
+            M.mot_set_schedule(run.h, sched)
+        assert e.value.status == M.MOT_ERR_UNSUPPORTED
     assert M.mot_get_schedule(run.h) == 2
     with pytest.raises(M.MotError) as e:
-        M.mot_set_schedule(run.h, 4)
+        M.mot_set_schedule(run.h, 5)
     assert e.value.status == M.MOT_ERR_INVALID_ARG
 
 

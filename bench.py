@@ -160,16 +160,19 @@ def load_peaks():
 # Source files each profiled kernel is built from (its traffic figure is stale
 # once any of them changes).
 KERNEL_SOURCES = {
-    "umma2_gemm1_gelu_gate": ["umma2.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
-    "umma2_gemm2_combine_store": ["umma2.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
-    "umma2_onchip_translate": ["onchip.cu", "umma_common.cuh", "ptx.cuh", "mot_internal.h"],
+    "umma2_gemm1_gelu_gate": ["umma2.cu", "umma_common.cuh", "gelu.cuh", "ptx.cuh",
+                              "mot_internal.h"],
+    "umma2_gemm2_combine_store": ["umma2.cu", "umma_common.cuh", "gelu.cuh", "ptx.cuh",
+                                  "mot_internal.h"],
+    "umma2_onchip_translate": ["onchip.cu", "umma_common.cuh", "gelu.cuh", "ptx.cuh",
+                               "mot_internal.h"],
     "umma2_wide_translate": ["wide.cu", "umma_common.cuh", "gelu.cuh", "ptx.cuh", "mot_internal.h"],
     # replay stages (all kernels of replay.cu)
     "replay_attn_sparse": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
     "replay_select": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
     "replay_fmha_full": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
     # backbone translators (all kernels of bt.cu)
-    "bt_ffn_fused": ["bt.cu", "bt_internal.h", "mot_internal.h", "ptx.cuh"],
+    "bt_ffn_fused": ["bt.cu", "bt_internal.h", "gelu.cuh", "mot_internal.h", "ptx.cuh"],
 }
 
 

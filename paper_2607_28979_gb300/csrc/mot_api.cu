@@ -24,7 +24,7 @@ namespace {
 constexpr size_t kA2Budget = size_t(8) << 30;
 
 // Chunks of target layers the host-buffer entry point pipelines over.
-constexpr int kHostChunks = 6;
+constexpr int kHostChunks = 16;   // most chunks of layers of the host-buffer pipeline
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
@@ -1206,7 +1206,21 @@ mot_status mot_translate_host(mot_handle h, const void* src_k, const void* src_v
   for (int l = 0; l < d.L_t; ++l)
     if (h->layer_map[l] >= 0) tl.push_back(l);
   const int n_tl = static_cast<int>(tl.size());
-  const int nc = std::min(kHostChunks, n_tl);
+  // chunk boundaries: the first and last chunks are small (1, then 2 layers),
+  // so the pipeline fills and drains quickly; the middle chunks hold about 4
+  // (more when there are more than 4 * (kHostChunks - 4) of them)
+  std::vector<int> cb{0};
+  if (n_tl <= 6) {
+    for (int r = 1; r <= n_tl; ++r) cb.push_back(r);
+  } else {
+    cb.push_back(1);
+    cb.push_back(3);
+    const int mid = n_tl - 6, nm = std::min((mid + 3) / 4, kHostChunks - 4);
+    for (int i = 1; i <= nm; ++i) cb.push_back(3 + i * mid / nm);
+    cb.push_back(n_tl - 1);
+    cb.push_back(n_tl);
+  }
+  const int nc = static_cast<int>(cb.size()) - 1;   // <= kHostChunks
   // the previous call's translation read the source staging and its copies
   // read the target staging: order this call after both
   MOT_CUDA_TRY(cudaStreamWaitEvent(h->copy_h2d, h->ev_prev_compute, 0));
@@ -1214,7 +1228,7 @@ mot_status mot_translate_host(mot_handle h, const void* src_k, const void* src_v
   MOT_CUDA_TRY(cudaMemcpyAsync(h->st_len, seq_lens, size_t(batch) * 4, cudaMemcpyHostToDevice, st));
   std::vector<char> copied(d.L_s, 0);
   for (int c = 0; c < nc; ++c) {
-    const int r0 = c * n_tl / nc, r1 = (c + 1) * n_tl / nc;
+    const int r0 = cb[c], r1 = cb[c + 1];
     // source layers first needed by this chunk, copied in runs of consecutive layers
     std::vector<char> need(d.L_s, 0);
     for (int r = r0; r < r1; ++r) {

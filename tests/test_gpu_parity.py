@@ -264,6 +264,9 @@ HOST_CASES = {
     "ragged": (SMALL["umma_ragged"], None),
     "uniform_partial_batch": (SMALL["umma_ragged"].replace(seq_lens=(200, 200)), None),
     "uniform_full_batch": (SMALL["umma_e3"].replace(seq_lens=(200, 200)), None),
+    # 10 translated layers: chunks of 1, 2, 4, 2 and 1 layers
+    "many_layers": (synth.Workload("host_many", 9, 2, 64, 10, 2, 128, 2, 256, 2, 160, "bf16",
+                                   (160, 77)), None),
 }
 
 

@@ -6,12 +6,17 @@
 //                         with the largest guidance score A[b][u][j] (ties to the
 //                         lower position), written in ascending order. It is exact
 //                         integer work on the order-preserving 16-bit image of each
-//                         score: two 256-bin histogram passes (high byte, then low
-//                         byte, warp-aggregated increments) find the score V of the
-//                         S-th largest (score, -position) key and how many of the
-//                         positions scoring V it takes; ballots then keep every
-//                         score above V and the lowest positions at V. Rows with
-//                         u + 1 <= S take every position.
+//                         score. The row is read once into shared memory as keys,
+//                         with its key range; a 256-bin histogram of the top digit
+//                         of (key - min), scaled to the row's range, and, when the
+//                         range spans more than 256 keys, a histogram of the low bits in the
+//                         chosen bin find the key V of the S-th largest (score,
+//                         -position) and how many of the positions scoring V it
+//                         takes; ballots then keep every score above V and the
+//                         lowest positions at V. Rows with u + 1 <= S take every
+//                         position. Rows past 4,096 positions take
+//   replay_select_stream_kernel, the same selection with the high and low byte as
+//                         the two digits, reading the row once per pass.
 //   replay_attn_kernel    one warp per (b, key/value head, u), no block barriers:
 //                         the query heads of the GQA group attend to the selected
 //                         rows (sparse) or to positions 0..u in 128-key chunks
@@ -99,13 +104,49 @@ __device__ __forceinline__ int warp_excl_scan(int v, int& total) {
   return x - v;
 }
 
-// One warp per context row (b, u). With o = the order-preserving 16 bits of a
-// score, the S-th largest (o, -j) key is found in two histogram passes over o
-// (high byte, then low byte): V = its score bits, k = how many positions with
-// o == V it takes. The selection is then every o > V plus the k lowest
-// positions with o == V, compacted in ascending order by warp scans. Each lane
-// reads 8 consecutive scores per step (16-byte loads when max_seq % 8 == 0).
-__global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const ReplayArgs a) {
+// The bin of a warp's histogram (kSelCopies copies of 256 bins) that holds the
+// k-th largest counted key, scanning from bin 255 down: lane 0 sums the top 8
+// bins, lane 31 the bottom 8. On return k is the rank left inside that bin.
+__device__ __forceinline__ uint32_t kth_bin(const int (*h)[256], int& k) {
+  const int lane = threadIdx.x & 31;
+  int c[8], t = 0;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    c[e] = 0;
+#pragma unroll
+    for (int cp = 0; cp < kSelCopies; ++cp) c[e] += h[cp][(31 - lane) * 8 + (7 - e)];
+    t += c[e];
+  }
+  int tot;
+  const int before = warp_excl_scan(t, tot);
+  int found = -1, krem = 0, acc = before;
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    if (found < 0 && acc + c[e] >= k) {
+      found = (31 - lane) * 8 + (7 - e);
+      krem = k - acc;
+    }
+    acc += c[e];
+  }
+  const int src = __ffs(__ballot_sync(0xffffffffu, found >= 0)) - 1;
+  k = __shfl_sync(0xffffffffu, krem, src);
+  return uint32_t(__shfl_sync(0xffffffffu, found, src));
+}
+
+// Order-preserving keys of two bf16 scores packed in a word (low half first):
+// a negative score's bits are inverted, a positive score's sign bit is set.
+__device__ __forceinline__ uint32_t ord16x2(uint32_t q) {
+  return q ^ ((((q >> 15) & 0x00010001u) * 0xFFFFu) | 0x80008000u);
+}
+
+// Selection for any max_seq. One warp per context row (b, u). With o = the
+// order-preserving 16 bits of a score, the S-th largest (o, -j) key is found in
+// two histogram passes over o (high byte, then low byte): V = its score bits, k =
+// how many positions with o == V it takes. The selection is then every o > V plus
+// the k lowest positions with o == V, compacted in ascending order by warp scans.
+// Each lane reads 8 consecutive scores per step (16-byte loads when max_seq % 8
+// == 0); every pass reads the row again.
+__global__ void __launch_bounds__(32 * kSelWarps) replay_select_stream_kernel(const ReplayArgs a) {
   __shared__ int hist[kSelWarps][kSelCopies][256];   // copy lane % kSelCopies: fewer same-bin collisions
   const ReplayDims& d = a.d;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -150,36 +191,14 @@ __global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const Rep
         for (int e = 0; e < 8; ++e)
           if (j8 + e < n) atomicAdd(&hw[o[e] >> 8], 1);
       } else {
-        // only the scores in bin `hi` count, spread over 256 low bytes: plain increments
+        // only the scores in bin `hi` count, spread over 256 low bytes
 #pragma unroll
         for (int e = 0; e < 8; ++e)
           if (j8 + e < n && (o[e] >> 8) == hi) atomicAdd(&hw[o[e] & 0xFFu], 1);
       }
     }
     __syncwarp();
-    // the bin holding the k-th largest: lane 0 holds the top 8 bins, lane 31 the bottom 8
-    int c[8], t = 0;
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      c[e] = 0;
-#pragma unroll
-      for (int cp = 0; cp < kSelCopies; ++cp) c[e] += hist[w][cp][(31 - lane) * 8 + (7 - e)];
-      t += c[e];
-    }
-    int tot;
-    const int before = warp_excl_scan(t, tot);
-    int found = -1, krem = 0, acc = before;
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      if (found < 0 && acc + c[e] >= k) {
-        found = (31 - lane) * 8 + (7 - e);
-        krem = k - acc;
-      }
-      acc += c[e];
-    }
-    const int src = __ffs(__ballot_sync(0xffffffffu, found >= 0)) - 1;
-    const uint32_t bin = uint32_t(__shfl_sync(0xffffffffu, found, src));
-    k = __shfl_sync(0xffffffffu, krem, src);
+    const uint32_t bin = kth_bin(hist[w], k);
     if (pass == 0)
       hi = bin;
     else
@@ -213,6 +232,142 @@ __global__ void __launch_bounds__(32 * kSelWarps) replay_select_kernel(const Rep
       if (sel[e]) out[pos++] = j8 + e;
     base += sel_tot;
     eq_taken += eq_tot;
+  }
+}
+
+// Selection for max_seq <= 4096, with the row's keys cached in shared memory.
+// One warp per context row (b, u): the row is read once and turned into
+// order-preserving keys o (lane L holds positions 256 r + 8 L + e, as one 16-byte
+// word of packed keys per round r), together with its key range [omin, omax].
+// The S-th largest (o, -j) key is then found by a radix selection over o - omin:
+// a 256-bin histogram of the top digit (o - omin) >> sh, sh the smallest shift
+// that fits the row's range into 256 bins, then, when sh > 0, a histogram of the
+// low sh bits among the keys of the chosen bin. That gives V, the threshold key,
+// and k, how many positions with o == V are taken. The compaction keeps every
+// o > V and the k lowest positions with o == V, in ascending order. The digits
+// follow the row's own range, so increments spread over many bins even when the
+// scores share a few binades.
+constexpr int kSelCacheWarps = 4;    // rows per CTA
+constexpr int kSelCacheRounds = 16;  // 256-position rounds cached per row: max_seq <= 4096
+
+__global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(const ReplayArgs a) {
+  __shared__ int hist[kSelCacheWarps][kSelCopies][256];   // copy lane % kSelCopies
+  __shared__ uint4 keys[kSelCacheWarps][kSelCacheRounds][32];
+  const ReplayDims& d = a.d;
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = blockIdx.x * kSelCacheWarps + w;
+  if (row >= d.B * d.N) return;
+  const int b = row / d.N, u = row - b * d.N;
+  if (u >= seq_len_of(a, b)) return;
+  int32_t* out = a.sel + int64_t(row) * d.S;
+  const int n = u + 1;
+  if (n <= d.S) {
+    for (int j = lane; j < d.S; j += 32) out[j] = j < n ? j : -1;
+    return;
+  }
+  const uint16_t* A = static_cast<const uint16_t*>(a.guide) + int64_t(row) * d.N;
+  const bool vec = (d.N & 7) == 0;   // then every 8-score group of the row is 16-byte aligned
+  const int nr = (n + 255) >> 8;     // rounds holding positions < n (<= kSelCacheRounds)
+  uint4 (*kc)[32] = keys[w];
+  uint32_t lo = 0xFFFFu, hi = 0u;
+  for (int r = 0; r < nr; ++r) {
+    const int j8 = r * 256 + lane * 8;
+    const int lim = min(n - j8, 8);   // this lane's positions < n in the round (may be <= 0)
+    uint32_t q[4] = {0u, 0u, 0u, 0u};
+    if (lim > 0) {
+      if (vec) {
+        const uint4 v = __ldg(reinterpret_cast<const uint4*>(A + j8));
+        q[0] = v.x;
+        q[1] = v.y;
+        q[2] = v.z;
+        q[3] = v.w;
+      } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+          if (e < lim) q[e >> 1] |= uint32_t(__ldg(A + j8 + e)) << (16 * (e & 1));
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      q[i] = ord16x2(q[i]);
+      const uint32_t o0 = q[i] & 0xFFFFu, o1 = q[i] >> 16;
+      if (2 * i < lim) {
+        lo = min(lo, o0);
+        hi = max(hi, o0);
+      }
+      if (2 * i + 1 < lim) {
+        lo = min(lo, o1);
+        hi = max(hi, o1);
+      }
+    }
+    kc[r][lane] = make_uint4(q[0], q[1], q[2], q[3]);
+  }
+  const uint32_t omin = __reduce_min_sync(0xffffffffu, lo);
+  const uint32_t range = __reduce_max_sync(0xffffffffu, hi) - omin;   // < 65536
+  const int sh = range > 255u ? 24 - __clz(range) : 0;   // (range >> sh) <= 255, sh <= 8
+  int* hw = hist[w][lane % kSelCopies];
+  int k = d.S;
+  // key e (0..7) of a lane's 16-byte word
+  auto key_of = [](const uint4& v, int e) -> uint32_t {
+    const uint32_t x = e < 2 ? v.x : e < 4 ? v.y : e < 6 ? v.z : v.w;
+    return (e & 1) ? x >> 16 : x & 0xFFFFu;
+  };
+  // top digit
+  for (int i = lane; i < kSelCopies * 256; i += 32) hist[w][0][i] = 0;
+  __syncwarp();
+  for (int r = 0; r < nr; ++r) {
+    const int lim = min(n - (r * 256 + lane * 8), 8);
+    const uint4 v = kc[r][lane];
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      if (e < lim) atomicAdd(&hw[(key_of(v, e) - omin) >> sh], 1);
+  }
+  __syncwarp();
+  const uint32_t top = kth_bin(hist[w], k);
+  uint32_t V = omin + (top << sh);
+  if (sh > 0) {   // the low sh bits among the keys of bin `top`
+    __syncwarp();
+    for (int i = lane; i < kSelCopies * 256; i += 32) hist[w][0][i] = 0;
+    __syncwarp();
+    const uint32_t msk = (1u << sh) - 1u;
+    for (int r = 0; r < nr; ++r) {
+      const int lim = min(n - (r * 256 + lane * 8), 8);
+      const uint4 v = kc[r][lane];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const uint32_t o = key_of(v, e) - omin;
+        if (e < lim && (o >> sh) == top) atomicAdd(&hw[o & msk], 1);
+      }
+    }
+    __syncwarp();
+    V += kth_bin(hist[w], k);
+  }
+  // compaction in ascending position order; bit e of a lane's masks is position 256 r + 8 lane + e
+  int base = 0, eq_taken = 0;
+  for (int r = 0; r < nr && base < d.S; ++r) {   // warp-uniform
+    const int j8 = r * 256 + lane * 8;
+    const int lim = min(n - j8, 8);
+    const uint4 v = kc[r][lane];
+    uint32_t gt = 0u, eq = 0u;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const uint32_t o = key_of(v, e);
+      if (e < lim) {
+        gt |= uint32_t(o > V) << e;
+        eq |= uint32_t(o == V) << e;
+      }
+    }
+    uint32_t sel = gt;
+    if (__any_sync(0xffffffffu, eq != 0u)) {   // the k lowest positions at the threshold are taken
+      int eq_tot;
+      int take = k - (eq_taken + warp_excl_scan(__popc(eq), eq_tot));
+      for (uint32_t m = eq; m != 0u && take > 0; m &= m - 1u, --take) sel |= m & (0u - m);
+      eq_taken += eq_tot;
+    }
+    int sel_tot;
+    int pos = base + warp_excl_scan(__popc(sel), sel_tot);
+    for (uint32_t m = sel; m != 0u; m &= m - 1u) out[pos++] = j8 + __ffs(m) - 1;
+    base += sel_tot;
   }
 }
 
@@ -779,17 +934,11 @@ __device__ __forceinline__ bool lane_and(int id, bool p) {
   return r != 0;
 }
 
-// (b, key/value head, u) of item `it`; false past the entry's sequence length.
-__device__ __forceinline__ bool gattn_item(const ReplayArgs& a, int64_t it, int& b, int& hk, int& u) {
-  u = static_cast<int>(it % a.d.N);
-  const int bh = static_cast<int>(it / a.d.N);
-  hk = bh % a.d.Hkv;
-  b = bh / a.d.Hkv;
-  return u < seq_len_of(a, b);
-}
-
+// G: query heads per key/value head (the N = 16 columns of the MMAs hold G of them).
+template <int G>
 __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const ReplayArgs a) {
   constexpr int D = 128;
+  static_assert(G >= 1 && G <= 16, "GQA group of the N = 16 MMA columns");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -808,8 +957,7 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
   const int bar_id = 1 + ln;
 
   const ReplayDims& d = a.d;
-  const int G = d.Hq / d.Hkv;
-  const int64_t n_items = int64_t(d.B) * d.Hkv * d.N;
+  const int64_t n_items = int64_t(d.B) * d.Hkv * d.N;   // <= INT32_MAX (checked at launch)
   const long long wl = a.wait_limit;
 
   // Zero the operand tiles once: query rows >= G, P rows >= G and key/value rows
@@ -839,10 +987,15 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
 
   // gather roles: per copy instruction a warp moves two 256-byte rows (lanes
   // 0-15 one key's row, lanes 16-31 the next key's); warp w takes keys
-  // 8 m + 2 w + {0, 1}, and lane L holds the position of key 8 (L >> 1) + 2 w + (L & 1)
+  // 8 m + kr (m = 0..15, kr = 2 w + half), and lane L holds the position of key
+  // 8 (L >> 1) + 2 w + (L & 1). A thread's 16-byte unit q16 of key 8 m + kr lands
+  // at the same swizzled column of every 1,024-byte atom (key & 7 == kr), so its
+  // destination is a fixed base plus 1,024 m.
   const int half = lane >> 4, q16 = lane & 15;
   const uint32_t sbase = smem_u32(tiles);
   const int my_key = 8 * (lane >> 1) + 2 * warp + (lane & 1);
+  const int kr = 2 * warp + half;
+  const uint32_t gdst = sbase + static_cast<uint32_t>((q16 >> 3) * Ga::kBlk + kr * 128 + (((q16 & 7) ^ kr) << 4));
   // softmax / output roles: warp w owns keys (S^T rows) and dims (O^T rows) 32 w .. 32 w + 31,
   // TMEM lanes 32 w .. 32 w + 31 (w = the warp's index mod 4)
   const int row = 32 * warp + lane;
@@ -854,17 +1007,32 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
   bool mma_issued = false;
   uint32_t n = 0;   // items done: the parity of both MMA barriers
 
-  // lane `ln` of CTA `blockIdx.x` takes items v, v + V, .. (v its global lane index)
+  // lane `ln` of CTA `blockIdx.x` takes items v, v + V, .. (v its global lane index);
+  // item it = bh * N + u is (b, key/value head) = (bh / Hkv, bh % Hkv) at context
+  // position u, kept as (c_bh, c_u) and advanced by V without a division
   struct Item {
     int b, hk, u, c;
   };
   int64_t it = int64_t(blockIdx.x) * Ga::kLanes + ln;
-  const int64_t it_step = int64_t(gridDim.x) * Ga::kLanes;
+  const int it_step = static_cast<int>(gridDim.x) * Ga::kLanes;
+  const int step_bh = it_step / d.N, step_u = it_step - step_bh * d.N;
+  int c_bh = static_cast<int>(it / d.N), c_u = static_cast<int>(it - int64_t(c_bh) * d.N);
   auto next_item = [&](Item& x) -> bool {
-    for (; it < n_items; it += it_step) {
-      if (gattn_item(a, it, x.b, x.hk, x.u)) {
-        x.c = min(d.S, x.u + 1);
-        it += it_step;
+    while (it < n_items) {
+      const int bh = c_bh, u = c_u;
+      it += it_step;
+      c_bh += step_bh;
+      c_u += step_u;
+      if (c_u >= d.N) {
+        c_u -= d.N;
+        ++c_bh;
+      }
+      const int b = bh / d.Hkv;
+      if (u < seq_len_of(a, b)) {
+        x.b = b;
+        x.hk = bh - b * d.Hkv;
+        x.u = u;
+        x.c = min(d.S, u + 1);
         return true;
       }
     }
@@ -875,14 +1043,14 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
   };
   // the item's selected key rows (which = 0, plus its query rows) or value rows (which = 1)
   auto issue_rows = [&](const Item& x, int my_pos, int which) {
-    const uint16_t* src = static_cast<const uint16_t*>(which ? a.v : a.k) +
-                          int64_t(x.b * d.Hkv + x.hk) * d.N * D + q16 * 8;
-    const uint32_t dst = sbase + static_cast<uint32_t>(which * Ga::kKV + (q16 >> 3) * Ga::kBlk);
-#pragma unroll 4
+    const char* src = reinterpret_cast<const char*>(static_cast<const uint16_t*>(which ? a.v : a.k) +
+                                                    int64_t(x.b * d.Hkv + x.hk) * d.N * D + q16 * 8);
+    const uint32_t dst = gdst + static_cast<uint32_t>(which * Ga::kKV);
+    const int n_m = x.c - kr;   // key 8 m + kr is selected while 8 m < n_m
+#pragma unroll
     for (int m = 0; m < 16; ++m) {
-      const int key = 8 * m + 2 * warp + half;
-      const int pos = __shfl_sync(0xffffffffu, my_pos, 2 * m + half);
-      if (key < x.c) cp_async_16(dst + key * 128 + (((q16 & 7) ^ (key & 7)) << 4), src + int64_t(pos) * D);
+      const int pos = __shfl_sync(0xffffffffu, my_pos, 2 * m + half);   // pos < N <= 65536
+      if (8 * m < n_m) cp_async_16(dst + 1024 * m, src + static_cast<uint32_t>(pos) * (2 * D));
     }
     if (which == 0) {
       for (int e = tid; e < G * 16; e += 128) {
@@ -909,8 +1077,9 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
     for (int h = 0; h < 16; ++h) {
       if (h < G) {
         const uint4 l4 = *reinterpret_cast<const uint4*>(xl + h * 4);
+        // l >= 1 (the row maximum's probability is 1), so the fast division is exact to 2 ulp
         const float l = __uint2float_rn(l4.x + l4.y + l4.z + l4.w) * (1.f / 16777216.f);
-        o[int64_t(h) * d.N * D] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(v[h]) / l));
+        o[int64_t(h) * d.N * D] = __bfloat16_as_ushort(__float2bfloat16_rn(__fdividef(__uint_as_float(v[h]), l)));
       }
     }
   };
@@ -1053,7 +1222,10 @@ bool replay_supported(const ReplayDims& d) {
 cudaError_t launch_replay_select(const ReplayArgs& a, cudaStream_t st) {
   const int rows = a.d.B * a.d.N;
   if (rows <= 0) return cudaSuccess;
-  replay_select_kernel<<<(rows + kSelWarps - 1) / kSelWarps, 32 * kSelWarps, 0, st>>>(a);
+  if (a.d.N <= 256 * kSelCacheRounds)
+    replay_select_kernel<<<(rows + kSelCacheWarps - 1) / kSelCacheWarps, 32 * kSelCacheWarps, 0, st>>>(a);
+  else
+    replay_select_stream_kernel<<<(rows + kSelWarps - 1) / kSelWarps, 32 * kSelWarps, 0, st>>>(a);
   return cudaGetLastError();
 }
 
@@ -1088,14 +1260,15 @@ cudaError_t launch_replay_fmha(const ReplayArgs& a, const CUtensorMap& tmQ, cons
 
 bool replay_gattn_supported(const ReplayDims& d) {
   const int G = d.Hq / d.Hkv;
-  return d.d == 128 && G >= 1 && G <= 16 && d.S >= 1 && d.S <= 128 &&
+  return d.d == 128 && group_ok(G) && G <= 16 && d.S >= 1 && d.S <= 128 &&
          int64_t(d.B) * d.Hkv * d.N <= INT32_MAX && int64_t(d.B) * d.Hq <= INT32_MAX;
 }
 
-cudaError_t launch_replay_gattn(const ReplayArgs& a, int num_sms, cudaStream_t st) {
+template <int G>
+cudaError_t launch_gattn_g(const ReplayArgs& a, int num_sms, cudaStream_t st) {
   static bool attr = false;
   if (!attr) {
-    cudaError_t e = cudaFuncSetAttribute(replay_gattn_kernel,
+    cudaError_t e = cudaFuncSetAttribute(replay_gattn_kernel<G>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, Ga::kSmem);
     if (e != cudaSuccess) return e;
     attr = true;
@@ -1103,8 +1276,24 @@ cudaError_t launch_replay_gattn(const ReplayArgs& a, int num_sms, cudaStream_t s
   const int64_t lanes = (int64_t(a.d.B) * a.d.Hkv * a.d.N + Ga::kLanes - 1) / Ga::kLanes;
   const int g = static_cast<int>(lanes < num_sms ? lanes : num_sms);   // persistent, one CTA per SM
   if (g <= 0) return cudaSuccess;
-  replay_gattn_kernel<<<g, Ga::kThreads, Ga::kSmem, st>>>(a);
+  replay_gattn_kernel<G><<<g, Ga::kThreads, Ga::kSmem, st>>>(a);
   return cudaGetLastError();
+}
+
+cudaError_t launch_replay_gattn(const ReplayArgs& a, int num_sms, cudaStream_t st) {
+  switch (a.d.Hq / a.d.Hkv) {
+    case 1: return launch_gattn_g<1>(a, num_sms, st);
+    case 2: return launch_gattn_g<2>(a, num_sms, st);
+    case 3: return launch_gattn_g<3>(a, num_sms, st);
+    case 4: return launch_gattn_g<4>(a, num_sms, st);
+    case 5: return launch_gattn_g<5>(a, num_sms, st);
+    case 6: return launch_gattn_g<6>(a, num_sms, st);
+    case 7: return launch_gattn_g<7>(a, num_sms, st);
+    case 8: return launch_gattn_g<8>(a, num_sms, st);
+    case 12: return launch_gattn_g<12>(a, num_sms, st);
+    case 16: return launch_gattn_g<16>(a, num_sms, st);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 template <int D, int G>

@@ -100,6 +100,39 @@ def test_selection_ties_and_constant_rows(name):
             np.testing.assert_array_equal(sel[b, u, :ref.size], ref)
 
 
+@pytest.mark.parametrize("span", [1, 255, 256, 257, 511, 512, 4097, 0x7EFF])
+def test_selection_across_key_ranges(span):
+    """Rows whose 16-bit keys span `span` values: the histogram digit's width
+    follows the row's range, so spans around 2^8 and 2^9 take the one-pass and
+    two-pass cases and their boundary."""
+    wl = SMALL["r_mha_d64"].replace(top_s=32)
+    N = wl.max_seq
+    rng = np.random.default_rng(span)
+    base = 0x3C00 if span < 0x4000 else 0x0080        # positive bf16 bit patterns, no NaN or Inf
+    g = (base + rng.integers(0, span + 1, size=(wl.max_batch, N, N))).astype(np.uint16)
+    g[:, :, 0] = base                                   # the range's ends are present
+    g[:, :, 1] = base + span
+    run = ReplayRun(wl)
+    sel = run.select(g)
+    for b, L in enumerate(wl.seq_lens):
+        for u in range(0, L, 5):
+            ref = oracle.replay_select(wl, g, b, u)
+            np.testing.assert_array_equal(sel[b, u, :ref.size], ref, err_msg=f"b={b} u={u}")
+
+
+@pytest.mark.parametrize("max_seq", [4104, 4099])   # 16-byte and scalar loads
+def test_selection_rows_longer_than_the_key_cache(max_seq):
+    """Rows past 4,096 positions take the streaming selection (the row read once per pass)."""
+    wl = RW("r_long", 2, 2, 4, 1, 64, 1, max_seq, (max_seq,), top_s=128, n_full=1)
+    g = synth.gen_guide(wl, 13)
+    sel = ReplayRun(wl).select(g)
+    rng = np.random.default_rng(max_seq)
+    for u in np.unique(np.concatenate([[0, 127, 128, 4095, 4096, max_seq - 1],
+                                       rng.integers(129, max_seq, size=40)])):
+        ref = oracle.replay_select(wl, g, 0, int(u))
+        np.testing.assert_array_equal(sel[0, u, :ref.size], ref, err_msg=f"u={u}")
+
+
 @pytest.mark.parametrize("name", sorted(SMALL))
 def test_attention_matches_oracle(name):
     wl = SMALL[name]

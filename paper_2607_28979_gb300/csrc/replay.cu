@@ -104,9 +104,10 @@ __device__ __forceinline__ int warp_excl_scan(int v, int& total) {
   return x - v;
 }
 
-// The bin of a warp's histogram (kSelCopies copies of 256 bins) that holds the
+// The bin of a warp's histogram (C copies of 256 bins) that holds the
 // k-th largest counted key, scanning from bin 255 down: lane 0 sums the top 8
 // bins, lane 31 the bottom 8. On return k is the rank left inside that bin.
+template <int C = kSelCopies>
 __device__ __forceinline__ uint32_t kth_bin(const int (*h)[256], int& k) {
   const int lane = threadIdx.x & 31;
   int c[8], t = 0;
@@ -114,7 +115,7 @@ __device__ __forceinline__ uint32_t kth_bin(const int (*h)[256], int& k) {
   for (int e = 0; e < 8; ++e) {
     c[e] = 0;
 #pragma unroll
-    for (int cp = 0; cp < kSelCopies; ++cp) c[e] += h[cp][(31 - lane) * 8 + (7 - e)];
+    for (int cp = 0; cp < C; ++cp) c[e] += h[cp][(31 - lane) * 8 + (7 - e)];
     t += c[e];
   }
   int tot;
@@ -249,9 +250,10 @@ __global__ void __launch_bounds__(32 * kSelWarps) replay_select_stream_kernel(co
 // scores share a few binades.
 constexpr int kSelCacheWarps = 4;    // rows per CTA
 constexpr int kSelCacheRounds = 16;  // 256-position rounds cached per row: max_seq <= 4096
+constexpr int kSelCacheCopies = 1;   // histogram copies per warp (36 KB per CTA: 6 CTAs per SM)
 
 __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(const ReplayArgs a) {
-  __shared__ int hist[kSelCacheWarps][kSelCopies][256];   // copy lane % kSelCopies
+  __shared__ int hist[kSelCacheWarps][kSelCacheCopies][256];   // copy lane % kSelCacheCopies
   __shared__ uint4 keys[kSelCacheWarps][kSelCacheRounds][32];
   const ReplayDims& d = a.d;
   const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -270,6 +272,7 @@ __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(cons
   const int nr = (n + 255) >> 8;     // rounds holding positions < n (<= kSelCacheRounds)
   uint4 (*kc)[32] = keys[w];
   uint32_t lo = 0xFFFFu, hi = 0u;
+#pragma unroll 4
   for (int r = 0; r < nr; ++r) {
     const int j8 = r * 256 + lane * 8;
     const int lim = min(n - j8, 8);   // this lane's positions < n in the round (may be <= 0)
@@ -305,7 +308,7 @@ __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(cons
   const uint32_t omin = __reduce_min_sync(0xffffffffu, lo);
   const uint32_t range = __reduce_max_sync(0xffffffffu, hi) - omin;   // < 65536
   const int sh = range > 255u ? 24 - __clz(range) : 0;   // (range >> sh) <= 255, sh <= 8
-  int* hw = hist[w][lane % kSelCopies];
+  int* hw = hist[w][lane % kSelCacheCopies];
   int k = d.S;
   // key e (0..7) of a lane's 16-byte word
   auto key_of = [](const uint4& v, int e) -> uint32_t {
@@ -313,7 +316,7 @@ __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(cons
     return (e & 1) ? x >> 16 : x & 0xFFFFu;
   };
   // top digit
-  for (int i = lane; i < kSelCopies * 256; i += 32) hist[w][0][i] = 0;
+  for (int i = lane; i < kSelCacheCopies * 256; i += 32) hist[w][0][i] = 0;
   __syncwarp();
   for (int r = 0; r < nr; ++r) {
     const int lim = min(n - (r * 256 + lane * 8), 8);
@@ -323,11 +326,11 @@ __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(cons
       if (e < lim) atomicAdd(&hw[(key_of(v, e) - omin) >> sh], 1);
   }
   __syncwarp();
-  const uint32_t top = kth_bin(hist[w], k);
+  const uint32_t top = kth_bin<kSelCacheCopies>(hist[w], k);
   uint32_t V = omin + (top << sh);
   if (sh > 0) {   // the low sh bits among the keys of bin `top`
     __syncwarp();
-    for (int i = lane; i < kSelCopies * 256; i += 32) hist[w][0][i] = 0;
+    for (int i = lane; i < kSelCacheCopies * 256; i += 32) hist[w][0][i] = 0;
     __syncwarp();
     const uint32_t msk = (1u << sh) - 1u;
     for (int r = 0; r < nr; ++r) {
@@ -340,7 +343,7 @@ __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(cons
       }
     }
     __syncwarp();
-    V += kth_bin(hist[w], k);
+    V += kth_bin<kSelCacheCopies>(hist[w], k);
   }
   // compaction in ascending position order; bit e of a lane's masks is position 256 r + 8 lane + e
   int base = 0, eq_taken = 0;

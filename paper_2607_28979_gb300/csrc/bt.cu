@@ -53,13 +53,16 @@ constexpr int kBtStages = 4;
 constexpr int kBtABytes = 128 * 64 * 2;   // 16 KB: 128 rows x 64 bf16
 constexpr int kBtBBytes = 256 * 64 * 2;   // 32 KB: up to 256 rows x 64 bf16
 constexpr int kBtStageBytes = kBtABytes + kBtBBytes;
-// warps 0..3 roles, then EPI epilogue warps: 4 for the row-norm stages (a row's
-// d values in one thread), 16 for the others (each warp of a lane quarter
+// warps 0..3 roles, then EPI epilogue warps: 8 for the row-norm stages (a row's
+// d values split over two threads, one per half, whose layer-norm statistics are
+// combined through shared memory), 16 for the others (each warp of a lane quarter
 // takes every fourth 32-column chunk)
 __host__ __device__ constexpr int bt_threads(int epi) { return 32 * (4 + epi); }
+constexpr int kBtRowEpi = 8;
 constexpr int kBtTmemCols = 512;
 constexpr float kLnEps = 1e-5f;
-constexpr int kBtSmem = kBtStages * kBtStageBytes + 256 + 1024;
+constexpr int kBtXchBytes = 2 * 2 * 128 * 8;   // [tile parity][half][row] (mean, M2)
+constexpr int kBtSmem = kBtStages * kBtStageBytes + 256 + kBtXchBytes + 1024;
 static_assert(kBtSmem <= 232448, "shared memory budget");
 
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
@@ -194,14 +197,13 @@ __device__ __forceinline__ void row_stats(const float (&v)[D], float& mean, floa
   m2 = q;
 }
 
-// dst[0..D) = bf16(gamma * (v - mean) * rstd + beta), 16-byte stores; ln holds
-// gamma[D] then beta[D]
+// dst[0..D) = bf16(gamma * (v - mean) * rstd + beta), 16-byte stores
 template <int D>
 __device__ __forceinline__ void store_norm(const float (&v)[D], float mean, float rstd,
-                                           const float* ln, uint16_t* dst) {
+                                           const float* gamma, const float* beta, uint16_t* dst) {
   uint4* d4 = reinterpret_cast<uint4*>(dst);
-  const float4* g4 = reinterpret_cast<const float4*>(ln);
-  const float4* b4 = reinterpret_cast<const float4*>(ln + D);
+  const float4* g4 = reinterpret_cast<const float4*>(gamma);
+  const float4* b4 = reinterpret_cast<const float4*>(beta);
 #pragma unroll
   for (int c = 0; c < D / 8; ++c) {
     const float4 g0 = __ldg(g4 + 2 * c), g1 = __ldg(g4 + 2 * c + 1);
@@ -257,9 +259,49 @@ __device__ __forceinline__ void store_bf16(const float (&v)[D], uint16_t* dst) {
                        pack2(v[8 * c + 4], v[8 * c + 5]), pack2(v[8 * c + 6], v[8 * c + 7]));
 }
 
-// Row-wise epilogues with the whole row in registers (N = D columns).
-template <int D>
-__device__ void epi_row(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
+// Named barrier over the nthreads epilogue threads, with the AND of p.
+__device__ __forceinline__ bool epi_and(int id, int nthreads, bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred a, q;\n\t"
+      "setp.ne.u32 a, %1, 0;\n\t"
+      "bar.red.and.pred q, %2, %3, a;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(p)), "r"(id), "r"(nthreads)
+      : "memory");
+  return r != 0;
+}
+
+// Where a row is split over two threads (half cg of the columns each), the
+// halves' statistics: each thread's (mean, M2) of its DH values goes to xch, and
+// after the epilogue barrier the pair combines them by the pairwise formula
+// (equal counts). Both threads form the same sums, so both get the same result.
+struct RowXch {
+  float2* xch;   // [2][128] of this tile parity, or null: the row is whole in one thread
+  int cg, nthreads;
+};
+template <int DH>
+__device__ __forceinline__ void row_stats_x(const float (&v)[DH], float& mean, float& m2, int row,
+                                            const RowXch& x) {
+  row_stats<DH>(v, mean, m2);
+  if (x.xch != nullptr) {
+    x.xch[x.cg * 128 + row] = make_float2(mean, m2);
+    epi_and(1, x.nthreads, true);
+    const float2 o = x.xch[(x.cg ^ 1) * 128 + row];
+    const float dl = o.x - mean;
+    m2 = (m2 + o.y) + dl * dl * (0.5f * DH);
+    mean = 0.5f * (mean + o.x);
+  }
+}
+
+// Row-wise epilogues with the row in registers: N = D columns, split in NCG
+// halves of DH = D / NCG columns (half x.cg in this thread).
+template <int D, int NCG>
+__device__ void epi_row(const EpiCtx& e, const Work& w, uint32_t tb, int row, const RowXch& xr) {
+  constexpr int DH = D / NCG;
+  constexpr int DF = D;   // full row width: the row statistics and strides
+  const int col0 = xr.cg * DH;
   const BtArgs& a = *e.a;
   const BtDims& d = a.d;
   const int mode = e.c->mode;
@@ -274,26 +316,27 @@ __device__ void epi_row(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
   }
   const bool valid = p < d.P && tile_token_valid(a, w, t);
   const int64_t grow = int64_t(w.g) * d.R + w.row0 + int64_t(t) * d.P + p;   // row of this thread
-  float v[D];
+  const int64_t gcol = grow * DF + col0;                                        // its first column
+  float v[DH];
   float mean = 0.f, m2 = 0.f;
   if (mode == kBtIn) {
     // layer norm of the source row (d_s values), then GELU of the folded product
     float mu = 0.f, rs = 0.f;
     if (valid) {
       const int x = w.g / d.E;
-      const uint16_t* xr =
+      const uint16_t* xs_row =
           a.routed ? static_cast<const uint16_t*>(a.xs) + grow * d.d_s
                    : static_cast<const uint16_t*>(a.src[x]) +
                          (((int64_t(a.src_layer[r]) * d.B + w.b) * d.P + p) * d.S + w.s0 + t) *
                              d.d_s;
-      const uint4* x4 = reinterpret_cast<const uint4*>(xr);
-      float s = 0.f;
+      const uint4* x4 = reinterpret_cast<const uint4*>(xs_row);
+      float sum = 0.f;
       for (int c = 0; c < d.d_s / 8; ++c) {
         const uint4 u = __ldg(x4 + c);
-        s += bf16_lo(u.x) + bf16_hi(u.x) + bf16_lo(u.y) + bf16_hi(u.y) + bf16_lo(u.z) +
-             bf16_hi(u.z) + bf16_lo(u.w) + bf16_hi(u.w);
+        sum += bf16_lo(u.x) + bf16_hi(u.x) + bf16_lo(u.y) + bf16_hi(u.y) + bf16_lo(u.z) +
+               bf16_hi(u.z) + bf16_lo(u.w) + bf16_hi(u.w);
       }
-      mu = s / d.d_s;
+      mu = sum / d.d_s;
       float q = 0.f;
       for (int c = 0; c < d.d_s / 8; ++c) {
         const uint4 u = __ldg(x4 + c);
@@ -305,50 +348,51 @@ __device__ void epi_row(const EpiCtx& e, const Work& w, uint32_t tb, int row) {
       rs = rsqrtf(q / d.d_s + kLnEps);
     }
     __syncwarp();   // converge before the warp-collective TMEM loads
-    load_row<D>(tb, v);
-    const float* sw = a.s_in + int64_t(w.g) * D;
-    const float* cb = a.c_in + int64_t(w.g) * D;
+    load_row<DH>(tb + col0, v);
+    const float* sw = a.s_in + int64_t(w.g) * DF + col0;
+    const float* cb = a.c_in + int64_t(w.g) * DF + col0;
 #pragma unroll
-    for (int k = 0; k < D; ++k) v[k] = gelu_tanh(fmaf(v[k] - mu * __ldg(sw + k), rs, __ldg(cb + k)));
-    row_stats<D>(v, mean, m2);
+    for (int k = 0; k < DH; ++k) v[k] = gelu_tanh(fmaf(v[k] - mu * __ldg(sw + k), rs, __ldg(cb + k)));
+    row_stats_x<DH>(v, mean, m2, row, xr);
     if (valid) {
-      const float rstd = rsqrtf(m2 * (1.f / D) + kLnEps);
-      const int64_t ln = (int64_t(w.g) * d.N + r) * 2 * D;
-      store_norm<D>(v, mean, rstd, a.ln_c + ln, static_cast<uint16_t*>(a.xz) + grow * D);
+      const float rstd = rsqrtf(m2 * (1.f / DF) + kLnEps);
+      const float* lnc = a.ln_c + (int64_t(w.g) * d.N + r) * 2 * DF + col0;
+      store_norm<DH>(v, mean, rstd, lnc, lnc + DF, static_cast<uint16_t*>(a.xz) + gcol);
       if (r == 0) {   // h_0 = z_1, and slot 0's queries read LN_Q(h_0)
-        store_f32<D>(v, a.h + grow * D);
-        store_norm<D>(v, mean, rstd, a.ln_q + ln, static_cast<uint16_t*>(a.xq) + grow * D);
+        const float* lnq = a.ln_q + (int64_t(w.g) * d.N + r) * 2 * DF + col0;
+        store_f32<DH>(v, a.h + gcol);
+        store_norm<DH>(v, mean, rstd, lnq, lnq + DF, static_cast<uint16_t*>(a.xq) + gcol);
       }
     }
     return;
   }
-  load_row<D>(tb, v);
+  load_row<DH>(tb + col0, v);
   if (mode == kBtO) {
-    add_bias<D>(v, a.c_o + (int64_t(w.g) * d.N + r) * D);
-    if (valid) add_f32<D>(v, a.h + grow * D);
-    row_stats<D>(v, mean, m2);
+    add_bias<DH>(v, a.c_o + (int64_t(w.g) * d.N + r) * DF + col0);
+    if (valid) add_f32<DH>(v, a.h + gcol);
+    row_stats_x<DH>(v, mean, m2, row, xr);
     if (valid) {
-      store_f32<D>(v, a.ht + grow * D);
-      store_norm<D>(v, mean, rsqrtf(m2 * (1.f / D) + kLnEps),
-                    a.ln_f + (int64_t(w.g) * d.N + r) * 2 * D,
-                    static_cast<uint16_t*>(a.xf) + grow * D);
+      const float* lnf = a.ln_f + (int64_t(w.g) * d.N + r) * 2 * DF + col0;
+      store_f32<DH>(v, a.ht + gcol);
+      store_norm<DH>(v, mean, rsqrtf(m2 * (1.f / DF) + kLnEps), lnf, lnf + DF,
+                     static_cast<uint16_t*>(a.xf) + gcol);
     }
     return;
   }
   // kBtF2: the new state, its row norm (next slot's queries), the raw row for
   // the output projection and the row's statistics for its token norm
-  add_bias<D>(v, a.c_f2 + (int64_t(w.g) * d.N + r) * D);
-  if (valid) add_f32<D>(v, a.ht + grow * D);
-  row_stats<D>(v, mean, m2);
+  add_bias<DH>(v, a.c_f2 + (int64_t(w.g) * d.N + r) * DF + col0);
+  if (valid) add_f32<DH>(v, a.ht + gcol);
+  row_stats_x<DH>(v, mean, m2, row, xr);
   if (valid) {
     if (r + 1 < d.N) {
-      store_f32<D>(v, a.h + grow * D);
-      store_norm<D>(v, mean, rsqrtf(m2 * (1.f / D) + kLnEps),
-                    a.ln_q + (int64_t(w.g) * d.N + r + 1) * 2 * D,
-                    static_cast<uint16_t*>(a.xq) + grow * D);
+      const float* lnq = a.ln_q + (int64_t(w.g) * d.N + r + 1) * 2 * DF + col0;
+      store_f32<DH>(v, a.h + gcol);
+      store_norm<DH>(v, mean, rsqrtf(m2 * (1.f / DF) + kLnEps), lnq, lnq + DF,
+                     static_cast<uint16_t*>(a.xq) + gcol);
     }
-    store_bf16<D>(v, static_cast<uint16_t*>(a.xo) + grow * D);
-    a.rstat[grow] = make_float2(mean, m2);
+    store_bf16<DH>(v, static_cast<uint16_t*>(a.xo) + gcol);
+    if (xr.cg == 0) a.rstat[grow] = make_float2(mean, m2);
   }
 }
 
@@ -538,6 +582,7 @@ __global__ void __launch_bounds__(bt_threads(EPI), 1)
   uint64_t* drain = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float2* xch = reinterpret_cast<float2*>(smem + kBtStages * kBtStageBytes + 256);   // [2][2][128]
 
   const BtDims& d = a.d;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -676,12 +721,14 @@ __global__ void __launch_bounds__(bt_threads(EPI), 1)
       int ok = 1;
       if (lane == 0) ok = mbar_wait(&tfull[buf], buf_phase, abort_flag, a.wait_limit) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
+      // the split rows pair warps at a barrier: every epilogue warp stops, or none
+      if constexpr (EPI == kBtRowEpi) ok = epi_and(1, 32 * EPI, ok != 0) ? 1 : 0;
       if (!ok) break;
       tc_fence_after();
       const uint32_t tb = tmem_base + static_cast<uint32_t>(buf * acc_cols) +
                           (static_cast<uint32_t>(q * 32) << 16);
-      if constexpr (EPI == 4) {   // the row-norm stages (kBtIn, kBtO, kBtF2)
-        epi_row<D>(e, w, tb, row);
+      if constexpr (EPI == kBtRowEpi) {   // the row-norm stages (kBtIn, kBtO, kBtF2)
+        epi_row<D, 2>(e, w, tb, row, RowXch{xch + buf * 256, cg, 32 * EPI});
       } else {
         if (c.mode == kBtOut && a.routed)
           epi_out_routed(e, w, tb, row, cg, EPI / 4);
@@ -980,7 +1027,7 @@ __global__ void __launch_bounds__(256, 1)
       if (lane == 0) wv = mbar_wait(c2_full, tl & 1, abort_flag, wl) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, wv, 0)) { ok = false; break; }
       tc_fence_after();
-      epi_row<D>(e, w, tmem + lanes + 256, row);   // the kBtF2 row epilogue
+      epi_row<D, 1>(e, w, tmem + lanes + 256, row, RowXch{nullptr, 0, 0});   // the kBtF2 row epilogue
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(c2_empty);
@@ -1389,7 +1436,7 @@ cudaError_t launch_bt_gemm(int mode, const BtArgs& a, const CUtensorMap& tmA,
   static bool attr_set[4] = {false, false, false, false};
   const int di = (d.d == 128 ? 1 : 0) + (wide ? 2 : 0);
   auto kern = wide ? (d.d == 128 ? bt_gemm_kernel<128, 16> : bt_gemm_kernel<64, 16>)
-                   : (d.d == 128 ? bt_gemm_kernel<128, 4> : bt_gemm_kernel<64, 4>);
+                   : (d.d == 128 ? bt_gemm_kernel<128, kBtRowEpi> : bt_gemm_kernel<64, kBtRowEpi>);
   if (!attr_set[di]) {
     cudaError_t e =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kBtSmem);
@@ -1399,7 +1446,7 @@ cudaError_t launch_bt_gemm(int mode, const BtArgs& a, const CUtensorMap& tmA,
   const long long items = static_cast<long long>(c.groups) * c.row_tiles * c.n_tiles;
   const int grid = static_cast<int>(items < num_sms ? items : num_sms);
   if (grid <= 0) return cudaSuccess;
-  kern<<<grid, bt_threads(wide ? 16 : 4), kBtSmem, st>>>(tmA, tmA2, tmB, a, c);
+  kern<<<grid, bt_threads(wide ? 16 : kBtRowEpi), kBtSmem, st>>>(tmA, tmA2, tmB, a, c);
   return cudaGetLastError();
 }
 

@@ -797,8 +797,9 @@ struct Ffn {
 };
 static_assert(Ffn<128>::kSmem <= 232448, "shared memory budget");
 
+constexpr int kFfnEpi = 8;   // epilogue warps: two per TMEM lane quarter, each half of a row
 template <int D>
-__global__ void __launch_bounds__(256, 1)
+__global__ void __launch_bounds__(32 * (4 + kFfnEpi), 1)
     bt_ffn_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW1,
                   const __grid_constant__ CUtensorMap tmW2, const BtArgs a, const GemmCfg c) {
   using F = Ffn<D>;
@@ -817,11 +818,11 @@ __global__ void __launch_bounds__(256, 1)
   uint64_t* w2_full = bars + 6;     // [2]
   uint64_t* w2_empty = bars + 8;    // [2]
   uint64_t* c1_full = bars + 10;    // [2] acc1 written
-  uint64_t* c1_empty = bars + 12;   // [2] acc1 read (4 epilogue warps)
-  uint64_t* h_full = bars + 14;     // [2] hidden chunk written (4 warps)
+  uint64_t* c1_empty = bars + 12;   // [2] acc1 read (every epilogue warp)
+  uint64_t* h_full = bars + 14;     // [2] hidden chunk written (every epilogue warp)
   uint64_t* h_empty = bars + 16;    // [2] hidden chunk consumed by MMA2
   uint64_t* c2_full = bars + 18;    // acc2 complete
-  uint64_t* c2_empty = bars + 19;   // acc2 read (4 warps)
+  uint64_t* c2_empty = bars + 19;   // acc2 read (every epilogue warp)
   uint64_t* drain = bars + 20;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 21);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -839,12 +840,12 @@ __global__ void __launch_bounds__(256, 1)
       mbar_init(&w2_full[i], 1);
       mbar_init(&w2_empty[i], 1);
       mbar_init(&c1_full[i], 1);
-      mbar_init(&c1_empty[i], 4);
-      mbar_init(&h_full[i], 4);
+      mbar_init(&c1_empty[i], kFfnEpi);
+      mbar_init(&h_full[i], kFfnEpi);
       mbar_init(&h_empty[i], 1);
     }
     mbar_init(c2_full, 1);
-    mbar_init(c2_empty, 4);
+    mbar_init(c2_empty, kFfnEpi);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -966,9 +967,14 @@ __global__ void __launch_bounds__(256, 1)
       ++tl;
     }
   } else if (warp >= 4) {
-    // ------------------------------------------------ epilogue: GELU chunks, then the F2 rows
+    // ------------------------------------------------ epilogue: GELU chunks, then the F2 rows.
+    // Warps 4 + 4 cg + q (cg = 0, 1) share TMEM lane quarter q: each takes half of every
+    // hidden chunk's columns and half of the F2 row, whose statistics the pair exchanges
+    // through hidden buffer 0 (free once acc2 is complete).
     const int q = warp & 3;
+    const int cg = (warp - 4) >> 2;
     const int row = q * 32 + lane;
+    float2* xch = reinterpret_cast<float2*>(sH);   // [2][128] (mean, M2) of the row halves
     const uint32_t lanes = static_cast<uint32_t>(q * 32) << 16;
     EpiCtx e{&a, &c};
     int tl = 0, c1c = 0, hcc = 0;
@@ -988,7 +994,7 @@ __global__ void __launch_bounds__(256, 1)
         tc_fence_after();
         const uint32_t hbase = smem_u32(sH + bh * F::kA2);
 #pragma unroll
-        for (int ch = 0; ch < 4; ++ch) {
+        for (int ch = 2 * cg; ch < 2 * cg + 2; ++ch) {
           uint32_t rr[32];
           tmem_ld_32x32b_x32(tmem + lanes + b1i * 128 + ch * 32, rr);
           tmem_ld_wait(rr);
@@ -1022,12 +1028,13 @@ __global__ void __launch_bounds__(256, 1)
         ++c1c;
         ++hcc;
       }
-      if (!ok) break;
-      int wv = 1;
-      if (lane == 0) wv = mbar_wait(c2_full, tl & 1, abort_flag, wl) ? 1 : 0;
-      if (!__shfl_sync(0xffffffffu, wv, 0)) { ok = false; break; }
+      int wv = 0;
+      if (ok && lane == 0) wv = mbar_wait(c2_full, tl & 1, abort_flag, wl) ? 1 : 0;
+      // the row halves pair warps at a barrier: every epilogue warp stops, or none
+      if (!epi_and(1, 32 * kFfnEpi, __shfl_sync(0xffffffffu, wv, 0) != 0)) { ok = false; break; }
       tc_fence_after();
-      epi_row<D, 1>(e, w, tmem + lanes + 256, row, RowXch{nullptr, 0, 0});   // the kBtF2 row epilogue
+      epi_row<D, 2>(e, w, tmem + lanes + 256, row, RowXch{xch, cg, 32 * kFfnEpi});   // the kBtF2 rows
+      epi_and(1, 32 * kFfnEpi, true);   // both halves read the exchange before hidden buffer 0 is reused
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(c2_empty);
@@ -1473,7 +1480,7 @@ cudaError_t launch_bt_ffn(const BtArgs& a, const CUtensorMap& tmXf, const CUtens
   const long long items = static_cast<long long>(c.groups) * c.row_tiles;
   const int grid = static_cast<int>(items < num_sms ? items : num_sms);
   if (grid <= 0) return cudaSuccess;
-  kern<<<grid, 256, smem, st>>>(tmXf, tmW1, tmW2, a, c);
+  kern<<<grid, 32 * (4 + kFfnEpi), smem, st>>>(tmXf, tmW1, tmW2, a, c);
   return cudaGetLastError();
 }
 

@@ -72,6 +72,15 @@ namespace {
 
 __device__ __forceinline__ float bf16f(uint16_t b) { return __uint_as_float(uint32_t(b) << 16); }
 
+// 2^x on the special-function unit (PTX ex2.approx.ftz: relative error about 2^-22, results
+// below the normal range flushed to 0), for the softmax probabilities that are then rounded
+// to bf16.
+__device__ __forceinline__ float ex2_fast(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
@@ -805,8 +814,8 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
           const int c0 = c * 32 + 2 * k;
-          const float p0 = (!diag || c0 <= r) ? exp2f(__uint_as_float(v[2 * k]) * sl2 - m) : 0.f;
-          const float p1 = (!diag || c0 + 1 <= r) ? exp2f(__uint_as_float(v[2 * k + 1]) * sl2 - m) : 0.f;
+          const float p0 = (!diag || c0 <= r) ? ex2_fast(__uint_as_float(v[2 * k]) * sl2 - m) : 0.f;
+          const float p1 = (!diag || c0 + 1 <= r) ? ex2_fast(__uint_as_float(v[2 * k + 1]) * sl2 - m) : 0.f;
           __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
           // the row sum counts the rounded probabilities the second MMA uses
           const float2 pr = __bfloat1622float2(pb);
@@ -1154,7 +1163,7 @@ __global__ void __launch_bounds__(Ga::kThreads, 1) replay_gattn_kernel(const Rep
       if (h < G) {
         const float4 m4 = *reinterpret_cast<const float4*>(xm + h * 4);
         const float m = fmaxf(fmaxf(m4.x, m4.y), fmaxf(m4.z, m4.w));
-        const __nv_bfloat16 pb16 = __float2bfloat16_rn(valid ? exp2f(sc[h] - m) : 0.f);
+        const __nv_bfloat16 pb16 = __float2bfloat16_rn(valid ? ex2_fast(sc[h] - m) : 0.f);
         st_shared_u16(prow + h * 128 + (((kk >> 3) ^ (h & 7)) << 4) + (kk & 7) * 2, __bfloat16_as_ushort(pb16));
         // the row sum of the rounded probabilities the MMA uses, in exact 2^-24 units
         const uint32_t sum = redux_add_u32(__float2uint_rn(__bfloat162float(pb16) * 16777216.f));

@@ -16,6 +16,8 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
+#include <algorithm>
+
 #include "mot_internal.h"
 
 namespace mot {
@@ -172,31 +174,44 @@ __global__ void __launch_bounds__(kRouteThreads) route_fill_kernel(PathArgs a, S
   }
 }
 
-// Gather the packed rows' source vectors (16 bytes per thread); padding rows
-// become zeros. zp[h][p][:] = src_x[src_layer][b][h][s][:].
-__global__ void pack_kernel(PathArgs a, SparseArgs s) {
+// Packed source rows: zp[h][p] = head row h of the token of packed row p (the
+// bucket's rows in token order), 16-byte vectors; packed rows without a token (the
+// tail of a bucket's last pair tile) are zeros. grid (x, H_s): block (x, h) takes
+// rows p = x * rpb + t / vpr, stepping by gridDim.x * rpb, thread t the row's
+// vector t % vpr; all index arithmetic per row is a shift or one small division.
+__global__ void __launch_bounds__(256) pack_kernel(PathArgs a, SparseArgs s) {
   const Dims& d = a.d;
   const int rows = s.plan[1];
-  const int vpr = d.d_s / 8;   // 16-byte vectors per head row (bf16)
-  const size_t n = static_cast<size_t>(rows) * d.H_s * vpr;
-  for (size_t i = blockIdx.x * size_t(blockDim.x) + threadIdx.x; i < n;
-       i += size_t(gridDim.x) * blockDim.x) {
-    const int v = static_cast<int>(i % vpr);
-    const size_t ph = i / vpr;
-    const int h = static_cast<int>(ph % d.H_s);
-    const int p = static_cast<int>(ph / d.H_s);
-    const int tok = s.ltok[p];
-    uint4 val = make_uint4(0u, 0u, 0u, 0u);
-    if (tok >= 0) {
-      const int vg = s.pairs[p / (2 * kTileM)].vg;
-      const GroupInfo gi = a.groups[a.g0 + vg / d.E];
-      const TileInfo ti = a.tiles[tok / kTileM];
-      const size_t pos = static_cast<size_t>(ti.s0) + tok % kTileM;
-      const uint4* src = static_cast<const uint4*>(a.src[gi.x]);
-      val = src[((((static_cast<size_t>(gi.src_layer) * d.B + ti.b) * d.H_s + h) * d.S + pos) *
-                 d.d_s) / 8 + v];
+  const int vpr = d.d_s / 8;     // 16-byte vectors per head row (<= 256, checked at launch)
+  const int rpb = 256 / vpr;     // rows per block per step
+  const int t = threadIdx.x;
+  if (t >= rpb * vpr) return;
+  const int v = t % vpr, h = blockIdx.y;
+  uint4* zp = static_cast<uint4*>(s.zp) + static_cast<size_t>(h) * s.R * vpr + v;
+  const int step = gridDim.x * rpb;
+  // eight rows per thread per pass: their chains of dependent loads (token, pair, group
+  // and tile, source vector) are in flight together
+  constexpr int kRows = 8;
+  for (int p0 = blockIdx.x * rpb + t / vpr; p0 < rows; p0 += kRows * step) {
+    int tok[kRows];
+#pragma unroll
+    for (int j = 0; j < kRows; ++j) tok[j] = p0 + j * step < rows ? s.ltok[p0 + j * step] : -1;
+    uint4 val[kRows];
+#pragma unroll
+    for (int j = 0; j < kRows; ++j) {
+      val[j] = make_uint4(0u, 0u, 0u, 0u);
+      if (tok[j] >= 0) {
+        const int vg = s.pairs[(p0 + j * step) / (2 * kTileM)].vg;
+        const GroupInfo gi = a.groups[a.g0 + vg / d.E];
+        const TileInfo ti = a.tiles[tok[j] / kTileM];
+        const size_t pos = static_cast<size_t>(ti.s0) + tok[j] % kTileM;
+        const uint4* src = static_cast<const uint4*>(a.src[gi.x]);
+        val[j] = src[(((static_cast<size_t>(gi.src_layer) * d.B + ti.b) * d.H_s + h) * d.S + pos) * vpr + v];
+      }
     }
-    static_cast<uint4*>(s.zp)[((static_cast<size_t>(h) * s.R + p) * d.d_s) / 8 + v] = val;
+#pragma unroll
+    for (int j = 0; j < kRows; ++j)
+      if (p0 + j * step < rows) zp[static_cast<size_t>(p0 + j * step) * vpr] = val[j];
   }
 }
 
@@ -251,7 +266,9 @@ cudaError_t launch_route(const PathArgs& a, const SparseArgs& s, int step, cudaS
 
 cudaError_t launch_pack(const PathArgs& a, const SparseArgs& s, cudaStream_t st) {
   if (a.gp <= 0) return cudaSuccess;
-  pack_kernel<<<4 * 152, 256, 0, st>>>(a, s);
+  if (a.d.d_s % 8 || a.d.d_s / 8 > 256 || a.d.H_s <= 0) return cudaErrorInvalidValue;
+  const dim3 grid(static_cast<unsigned>(std::max(1, 8 * 152 / a.d.H_s)), a.d.H_s);
+  pack_kernel<<<grid, 256, 0, st>>>(a, s);
   return cudaGetLastError();
 }
 

@@ -29,6 +29,25 @@ __device__ __forceinline__ int n_rows_of(const PathArgs& a) {
   return min(*a.n_tiles, a.d.tiles_max) * kTileM;
 }
 
+// Block-wide sum (1024 threads); s_warp holds at least 33 ints.
+__device__ __forceinline__ int block_sum(int v, int* s_warp) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  if (lane == 0) s_warp[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    int t = s_warp[lane];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+    if (lane == 0) s_warp[32] = t;
+  }
+  __syncthreads();
+  const int total = s_warp[32];
+  __syncthreads();   // s_warp is reused by the next call
+  return total;
+}
+
 // Block-wide exclusive scan of one flag per thread (1024 threads): returns the
 // thread's prefix and writes the block total to *total.
 __device__ __forceinline__ int block_scan_flag(int f, int* s_warp, int* total) {
@@ -128,25 +147,48 @@ __global__ void __launch_bounds__(kRouteThreads) route_plan_kernel(PathArgs a, S
   }
 }
 
-// grid (gp, E): the bucket's rows in ascending token order, then its padding.
+// Bucket lists: block (g, m, c) writes the packed rows of bucket (g, m) for the
+// tokens of row chunk c (kFillChunk rows), in token order: it first counts the
+// bucket's tokens in the rows before its chunk, then scans its chunk 1024 rows at
+// a time. Chunk 0 also writes the padding rows of the bucket's last pair tile.
+constexpr int kFillChunk = 4096;
+
 __global__ void __launch_bounds__(kRouteThreads) route_fill_kernel(PathArgs a, SparseArgs s) {
   const int g = blockIdx.x, m = blockIdx.y, grp = a.g0 + g, E = a.d.E, b = g * E + m;
   if (s.plan[1] == 0) return;
   const int n_rows = n_rows_of(a);
+  const int r_lo = blockIdx.z * kFillChunk;
+  const int base = s.row0[b], count = s.counts[b];
+  uint16_t* g16 = static_cast<uint16_t*>(s.gate16p);
+  if (blockIdx.z == 0) {   // padding rows of the bucket's last pair tile
+    const int padded = ((count + 2 * kTileM - 1) / (2 * kTileM)) * 2 * kTileM;
+    for (int p = base + count + threadIdx.x; p < base + padded; p += kRouteThreads) {
+      s.ltok[p] = -1;
+      s.lslot[p] = 0;
+      s.gatep[p] = 0.f;
+      uint4* row16 = reinterpret_cast<uint4*>(g16 + static_cast<size_t>(p) * 64);
+#pragma unroll
+      for (int v = 0; v < 8; ++v) row16[v] = make_uint4(0u, 0u, 0u, 0u);
+    }
+  }
+  if (r_lo >= n_rows) return;   // uniform over the block
   const uint32_t* __restrict__ sel = a.sel + static_cast<size_t>(grp) * a.d.tpad;
   const float* __restrict__ gate = a.gate + static_cast<size_t>(grp) * a.d.tpad * E;
   __shared__ int s_warp[64];
   __shared__ int s_total;
-  const int base = s.row0[b], count = s.counts[b];
-  uint16_t* g16 = static_cast<uint16_t*>(s.gate16p);
+  // the bucket's tokens before this chunk
+  int before = 0;
+  for (int r = threadIdx.x; r < r_lo; r += kRouteThreads) before += (sel[r] >> m) & 1u;
+  before = block_sum(before, s_warp);
+  const int r_hi = min(n_rows, r_lo + kFillChunk);
   int done = 0;
-  for (int r0 = 0; r0 < n_rows; r0 += kRouteThreads) {
+  for (int r0 = r_lo; r0 < r_hi; r0 += kRouteThreads) {
     const int r = r0 + threadIdx.x;
-    const uint32_t sv = r < n_rows ? sel[r] : 0u;
+    const uint32_t sv = r < r_hi ? sel[r] : 0u;
     const int f = (sv >> m) & 1u;
     const int pre = block_scan_flag(f, s_warp, &s_total);
     if (f) {
-      const int p = base + done + pre;
+      const int p = base + before + done + pre;
       const float gv = gate[static_cast<size_t>(r) * E + m];
       s.ltok[p] = r;
       s.lslot[p] = __popc(sv & ((1u << m) - 1u));
@@ -161,16 +203,6 @@ __global__ void __launch_bounds__(kRouteThreads) route_fill_kernel(PathArgs a, S
       }
     }
     done += s_total;
-  }
-  // padding rows of the bucket's last pair tile
-  const int padded = ((count + 2 * kTileM - 1) / (2 * kTileM)) * 2 * kTileM;
-  for (int p = base + count + threadIdx.x; p < base + padded; p += kRouteThreads) {
-    s.ltok[p] = -1;
-    s.lslot[p] = 0;
-    s.gatep[p] = 0.f;
-    uint4* row16 = reinterpret_cast<uint4*>(g16 + static_cast<size_t>(p) * 64);
-#pragma unroll
-    for (int v = 0; v < 8; ++v) row16[v] = make_uint4(0u, 0u, 0u, 0u);
   }
 }
 
@@ -260,7 +292,8 @@ cudaError_t launch_route(const PathArgs& a, const SparseArgs& s, int step, cudaS
   else if (step == 1)
     route_plan_kernel<<<1, kRouteThreads, 0, st>>>(a, s);
   else
-    route_fill_kernel<<<grid, kRouteThreads, 0, st>>>(a, s);
+    route_fill_kernel<<<dim3(a.gp, a.d.E, (a.d.tiles_max * kTileM + kFillChunk - 1) / kFillChunk),
+                        kRouteThreads, 0, st>>>(a, s);
   return cudaGetLastError();
 }
 

@@ -51,14 +51,16 @@
 //                           warp 1  S = Q K^T (M=128, N=128 keys) into double-
 //                                   buffered TMEM and, one tile later, O += P V
 //                                   (M=128, N=d) accumulated in TMEM;
-//                           warps 4..7  one query row per thread: the scaled,
-//                                   masked row of S from TMEM, its running max and
-//                                   sum (base-2 exponentials), P as bf16 into a
-//                                   128B-swizzled SMEM tile for the second MMA. The
-//                                   running max rises only when a tile's max exceeds
-//                                   it by more than 2^8, and only then are the sum
-//                                   and the O row in TMEM rescaled; O is read from
-//                                   TMEM once, at the end.
+//                           warps 4..11 two threads per query row, each half of
+//                                   its keys and of its output columns: the scaled,
+//                                   masked scores from TMEM, the row's running max
+//                                   (the halves' maxima traded through TMEM) and
+//                                   sum (base-2 exponentials on ex2.approx), P as
+//                                   bf16 into a 128B-swizzled SMEM tile for the
+//                                   second MMA. The running max rises only when a
+//                                   tile's max exceeds it by more than 2^8, and only
+//                                   then are the sum and the O row in TMEM rescaled;
+//                                   O is read from TMEM once, at the end.
 //                         Every wait is bounded; on a timeout the roles unwind,
 //                         copies and MMAs in flight are drained and TMEM is freed.
 #include <cuda_bf16.h>
@@ -576,9 +578,41 @@ struct Fa {
   static constexpr int kP = 2 * kPBlk;
   static constexpr int kBytes = kQ + 2 * kK + 2 * kVt + 2 * kP;
   static constexpr int kSmem = kBytes + 256 + 1024;
-  static constexpr int kThreads = 256;
+  static constexpr int kThreads = 384;   // 4 role warps, 8 softmax warps (two per lane quarter)
 };
 static_assert(Fa<128>::kSmem <= 232448, "shared memory budget");
+static_assert(Fa<64>::kThreads == Fa<128>::kThreads, "one launch size for both head widths");
+
+// One 32-bit TMEM column of the thread's lane (warp-collective, 32x32b shape).
+__device__ __forceinline__ void tmem_st_x1(uint32_t taddr, float v) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr), "r"(__float_as_uint(v))
+               : "memory");
+}
+
+__device__ __forceinline__ float tmem_ld_x1(uint32_t taddr) {
+  uint32_t v;
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(v) : "r"(taddr) : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" : "+r"(v)::"memory");
+  return __uint_as_float(v);
+}
+
+// Named barrier `id` over `n` threads, and the same returning the AND of `p`.
+__device__ __forceinline__ void lane_sync_n(int id, int n) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+__device__ __forceinline__ bool lane_and_n(int id, int n, bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred a, q;\n\t"
+      "setp.ne.u32 a, %1, 0;\n\t"
+      "bar.red.and.pred q, %2, %3, a;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(p)), "r"(id), "r"(n)
+      : "memory");
+  return r != 0;
+}
 
 // Each thread of the warp writes 32 consecutive 32-bit columns of its TMEM lane.
 __device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const uint32_t (&r)[32]) {
@@ -651,8 +685,8 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
       mbar_init(&kv_full[i], 1);
       mbar_init(&kv_empty[i], 1);
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_empty[i], 4);
-      mbar_init(&p_full[i], 4);
+      mbar_init(&s_empty[i], Fa<D>::kThreads / 32 - 4);   // every softmax warp
+      mbar_init(&p_full[i], Fa<D>::kThreads / 32 - 4);
       mbar_init(&p_empty[i], 1);
 
     }
@@ -754,12 +788,22 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
     // only when a tile's max exceeds it by more than kTau (base 2), so every
     // probability exp2(s - m) stays below 2^kTau; raising it rescales the row's
     // sum and its O row in TMEM (after the previous tile's PV has landed).
+    // Warps 4 + 4 hh + q (hh = 0, 1) share TMEM lane quarter q: thread (hh, row)
+    // takes keys and output columns [64 hh, 64 hh + 64) of the row. The pair trades
+    // its partial maxima through TMEM columns 384.. of the row's lane (double-buffered
+    // by tile parity; S and O use columns 0..383) and adds its partial sums at the end;
+    // both threads of a row therefore take the same max and the same rescaling decisions. Every per-tile wait is agreed
+    // on by all softmax warps (bar.red.and) before the pair barrier.
     constexpr float kTau = 8.f;
-    const int r = (warp & 3) * 32 + lane;
-    const uint32_t lanes = static_cast<uint32_t>((warp & 3) * 32) << 16;
+    constexpr int kSmWarps = Fa<D>::kThreads / 32 - 4;   // 8
+    constexpr int H = D / 2;                               // output columns per thread
+    const int q = warp & 3, hh = (warp - 4) >> 2;
+    const int r = q * 32 + lane;
+    const uint32_t lanes = static_cast<uint32_t>(q * 32) << 16;
     const float sl2 = rsqrtf(float(D)) * 1.4426950408889634f;   // scale * log2(e)
     float m = -INFINITY, l = 0.f;
     bool ok = true;
+    auto agree = [&](bool p) -> bool { return lane_and_n(1, 32 * kSmWarps, p); };
     auto wait_lane0 = [&](uint64_t* bar, uint32_t par) -> bool {
       int w = 1;
       if (lane == 0) w = mbar_wait(bar, par, abort_flag, wl) ? 1 : 0;
@@ -767,53 +811,61 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
     };
     for (int j = 0; j < n_kv; ++j) {
       const int st = j & 1;
-      if (!wait_lane0(&s_full[st], (j >> 1) & 1)) { ok = false; break; }
+      if (!agree(wait_lane0(&s_full[st], (j >> 1) & 1))) { ok = false; break; }
       tc_fence_after();
       const bool diag = j == qt;
-      // pass 1: the row maximum of the scaled, masked scores
+      // pass 1: the maximum of this thread's 64 scaled, masked scores, then the row's
       float mx = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
+      for (int c = 0; c < 2; ++c) {
         uint32_t v[32];
-        tmem_ld_32x32b_x32(tmem + lanes + st * 128 + c * 32, v);
+        tmem_ld_32x32b_x32(tmem + lanes + st * 128 + hh * 64 + c * 32, v);
         tmem_ld_wait(v);
 #pragma unroll
         for (int k = 0; k < 32; ++k)
-          if (!diag || c * 32 + k <= r) mx = fmaxf(mx, __uint_as_float(v[k]) * sl2);
+          if (!diag || hh * 64 + c * 32 + k <= r) mx = fmaxf(mx, __uint_as_float(v[k]) * sl2);
       }
+      const uint32_t xcol = tmem + lanes + 384 + 2 * static_cast<uint32_t>(j & 1);
+      tmem_st_x1(xcol + hh, mx);
+      tmem_st_wait();
+      tc_fence_before();
+      lane_sync_n(1, 32 * kSmWarps);
+      tc_fence_after();
+      mx = fmaxf(mx, tmem_ld_x1(xcol + (hh ^ 1)));
       const bool raise = mx > m + kTau;   // always on the first tile (m = -inf)
-      const float alpha = (raise && m != -INFINITY) ? exp2f(m - mx) : 1.f;
-      if (__any_sync(0xffffffffu, alpha != 1.f)) {
-        // rescale O rows in TMEM once PV_{j-1} has been added
-        if (!wait_lane0(pv_done, static_cast<uint32_t>(j - 1) & 1u)) { ok = false; break; }
+      const float alpha = (raise && m != -INFINITY) ? ex2_fast(m - mx) : 1.f;
+      const bool rescale = __any_sync(0xffffffffu, alpha != 1.f);
+      // rescaling needs PV_{j-1} in O; writing P_j needs PV_{j-2} done with the buffer
+      bool w = !rescale || wait_lane0(pv_done, static_cast<uint32_t>(j - 1) & 1u);
+      w = w && wait_lane0(&p_empty[st], ((j >> 1) & 1) ^ 1u);
+      if (!agree(w)) { ok = false; break; }
+      if (rescale) {
         tc_fence_after();
 #pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
+        for (int c = 0; c < H / 32; ++c) {
           uint32_t v[32];
-          tmem_ld_32x32b_x32(tmem + lanes + 256 + c * 32, v);
+          tmem_ld_32x32b_x32(tmem + lanes + 256 + hh * H + c * 32, v);
           tmem_ld_wait(v);
 #pragma unroll
           for (int k = 0; k < 32; ++k) v[k] = __float_as_uint(__uint_as_float(v[k]) * alpha);
-          tmem_st_32x32b_x32(tmem + lanes + 256 + c * 32, v);
+          tmem_st_32x32b_x32(tmem + lanes + 256 + hh * H + c * 32, v);
         }
         tmem_st_wait();
       }
       l *= alpha;
       if (raise) m = mx;
-      // P_j must not overwrite the buffer before PV_{j-2} has read it
-      if (!wait_lane0(&p_empty[st], ((j >> 1) & 1) ^ 1u)) { ok = false; break; }
-      // pass 2: P = exp2(s - m) as bf16 into the swizzled P tile, and its row sum
+      // pass 2: P = exp2(s - m) as bf16 into block hh of the swizzled P tile, and the partial sum
       float sum = 0.f;
-      const uint32_t pbase = smem_u32(sP + st * Fa<D>::kP);
+      const uint32_t pbase = smem_u32(sP + st * Fa<D>::kP) + static_cast<uint32_t>(hh * Fa<D>::kPBlk);
 #pragma unroll
-      for (int c = 0; c < 4; ++c) {
+      for (int c = 0; c < 2; ++c) {
         uint32_t v[32];
-        tmem_ld_32x32b_x32(tmem + lanes + st * 128 + c * 32, v);
+        tmem_ld_32x32b_x32(tmem + lanes + st * 128 + hh * 64 + c * 32, v);
         tmem_ld_wait(v);
         uint32_t pk[16];
 #pragma unroll
         for (int k = 0; k < 16; ++k) {
-          const int c0 = c * 32 + 2 * k;
+          const int c0 = hh * 64 + c * 32 + 2 * k;
           const float p0 = (!diag || c0 <= r) ? ex2_fast(__uint_as_float(v[2 * k]) * sl2 - m) : 0.f;
           const float p1 = (!diag || c0 + 1 <= r) ? ex2_fast(__uint_as_float(v[2 * k + 1]) * sl2 - m) : 0.f;
           __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
@@ -822,7 +874,7 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
           sum += pr.x + pr.y;
           pk[k] = *reinterpret_cast<uint32_t*>(&pb);
         }
-        st_sw128_half(pbase + (c >> 1) * Fa<D>::kPBlk, r, c & 1, pk);
+        st_sw128_half(pbase, r, c, pk);
       }
       tc_fence_before();
       fence_proxy_async_smem();
@@ -833,18 +885,27 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
       }
       l += sum;
     }
-    if (ok && wait_lane0(pv_done, static_cast<uint32_t>(n_kv - 1) & 1u)) {
+    // every softmax warp takes part in the agreement (ok is uniform: the loop's exits are agreed)
+    const bool done = agree(ok && wait_lane0(pv_done, static_cast<uint32_t>(n_kv - 1) & 1u));
+    if (done) {
       tc_fence_after();
-      const int q = q0 + r;
+      // the row's sum: this half's plus the partner's (TMEM columns 388, 389)
+      tmem_st_x1(tmem + lanes + 388 + hh, l);
+      tmem_st_wait();
+      tc_fence_before();
+      lane_sync_n(1, 32 * kSmWarps);
+      tc_fence_after();
+      l += tmem_ld_x1(tmem + lanes + 388 + (hh ^ 1));
+      const int qq = q0 + r;
       const float inv = 1.f / l;
       uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.out) +
-                                            ((int64_t(b) * d.Hq + h) * d.N + q) * D);
+                                            ((int64_t(b) * d.Hq + h) * d.N + qq) * D + hh * H);
 #pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
+      for (int c = 0; c < H / 32; ++c) {
         uint32_t v[32];
-        tmem_ld_32x32b_x32(tmem + lanes + 256 + c * 32, v);
+        tmem_ld_32x32b_x32(tmem + lanes + 256 + hh * H + c * 32, v);
         tmem_ld_wait(v);
-        if (q < L) {
+        if (qq < L) {
 #pragma unroll
           for (int e8 = 0; e8 < 4; ++e8) {
             uint32_t w4[4];
@@ -1266,7 +1327,7 @@ cudaError_t launch_replay_fmha(const ReplayArgs& a, const CUtensorMap& tmQ, cons
     attr[di] = true;
   }
   const int n_qt = (d.N + 127) / 128;
-  kern<<<d.B * d.Hq * n_qt, 256, smem, st>>>(tmQ, tmK, tmVt, a);
+  kern<<<d.B * d.Hq * n_qt, Fa<128>::kThreads, smem, st>>>(tmQ, tmK, tmVt, a);
   return cudaGetLastError();
 }
 

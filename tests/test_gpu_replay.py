@@ -157,6 +157,31 @@ def test_attention_matches_oracle(name):
             assert (o[b, :, L:] == np.int16(G.SENTINEL_BF16)).all()
 
 
+@pytest.mark.parametrize("group", [2, 3, 4, 5, 7, 8, 12])
+def test_guided_attention_every_group_size(group):
+    """The tensor-core guided kernel is instantiated per GQA group size G (the
+    query heads of one key/value head): a guided layer with d = 128 and S = 128
+    for each G the other tests do not reach, sampled against the oracle."""
+    kv = 2 if group <= 4 else 1
+    wl = RW(f"r_g{group}", 2, 3, group * kv, kv, 128, 2, 264, (264, 131), top_s=128, n_full=1)
+    q, k, v = synth.gen_replay_qkv(wl, 17)
+    g = synth.gen_guide(wl, 19)
+    run = ReplayRun(wl)
+    out = run.attend(2, q, k, v, g)
+    rng = np.random.default_rng(group)
+    tb, th, tu = [], [], []
+    for b, L in enumerate(wl.seq_lens):
+        us = np.unique(np.concatenate([[0, 127, 128, L - 1], rng.integers(0, L, size=12)]))
+        for u in us:
+            for h in range(wl.q_heads):
+                tb.append(b); th.append(h); tu.append(u)
+    ref = oracle.replay_tokens(wl, 2, q, k, v, g, tb, th, tu)
+    G.assert_parity(BF16, _f64(out)[tb, th, tu], ref, f"group {group}")
+    o = out.cpu().numpy()
+    for b, L in enumerate(wl.seq_lens):
+        assert (o[b, :, L:] == np.int16(G.SENTINEL_BF16)).all()
+
+
 def test_full_size_layer_sampled():
     """Qwen2.5-0.5B -> 1.5B replay shapes (4 x 4096 context, 12 / 2 heads of 128,
     S = 128): one full and one guided layer, in the benchmark's launch configuration."""

@@ -31,11 +31,12 @@
 // feed stay the blob's exact bf16 values. Every GEMM is one persistent,
 // warp-specialised tcgen05 kernel: warp 0 TMA producer (4-stage ring of 64-wide
 // K blocks), warp 1 MMA issuer (M = 128, N = NT, fp32 accumulators in TMEM, two
-// buffers), warp 2 TMEM allocator, then the epilogue warps (4 for the row-norm
-// stages, one row per thread; 16 for the others, a quarter of the columns per
-// warp). Row tiles
-// hold whole tokens (tau = 128 / P of them). The epilogue warps never wait on
-// one another. All waits are bounded; on a timeout every role
+// buffers), warp 2 TMEM allocator, then the epilogue warps (8 for the row-norm
+// stages, two per TMEM lane quarter, each thread one half of a row, the halves'
+// layer-norm statistics combined through shared memory; 16 for the others, a
+// quarter of the columns per warp). Row tiles hold whole tokens (tau = 128 / P of
+// them). Apart from the row halves' exchange, the epilogue warps never wait on one
+// another. All waits are bounded; on a timeout every role
 // unwinds, copies and MMAs in flight are drained, TMEM is freed and
 // kStatusTimeout is raised.
 #include <cuda_bf16.h>
@@ -785,7 +786,8 @@ __global__ void __launch_bounds__(bt_threads(EPI), 1)
 //   MMA2  acc2        += A2 W_F2[:, hc]^T        (M = 128, N = d, K = 128)
 // MMA1 runs one chunk ahead of MMA2; after the last chunk the kBtF2 row epilogue
 // reads acc2. warp 0: TMA (xf once per tile, W_F1 / W_F2 chunks in 2-slot
-// rings); warp 1: MMAs; warp 2: TMEM; warps 4..7: epilogue (one row each).
+// rings); warp 1: MMAs; warp 2: TMEM; warps 4..11: epilogue (two per TMEM lane
+// quarter: each half of every hidden chunk and half of the FFN2 row).
 template <int D>
 struct Ffn {
   static constexpr int kA = 128 * D * 2;       // xf tile: D / 64 blocks of 128 rows x 128 B

@@ -148,16 +148,28 @@ __global__ void __launch_bounds__(kRouteThreads) route_plan_kernel(PathArgs a, S
 }
 
 // Bucket lists: block (g, m, c) writes the packed rows of bucket (g, m) for the
-// tokens of row chunk c (kFillChunk rows), in token order: it first counts the
-// bucket's tokens in the rows before its chunk, then scans its chunk 1024 rows at
-// a time. Chunk 0 also writes the padding rows of the bucket's last pair tile.
+// tokens of row chunk c, in token order: it first counts the bucket's tokens in the
+// rows before its chunk, then scans its chunk 1024 rows at a time. Chunk 0 also
+// writes the padding rows of the bucket's last pair tile. Chunks are at least
+// kFillChunk rows and at most kFillChunks per bucket, so the counting stays linear
+// in the rows times a small factor.
 constexpr int kFillChunk = 4096;
+constexpr int kFillChunks = 32;
+
+// Rows per chunk for `rows_max` rows (a multiple of kRouteThreads), the same on
+// the host (grid) and in the kernel.
+__host__ __device__ __forceinline__ int fill_chunk_rows(int rows_max) {
+  const int per = (rows_max + kFillChunks - 1) / kFillChunks;
+  const int c = per > kFillChunk ? per : kFillChunk;
+  return (c + kRouteThreads - 1) / kRouteThreads * kRouteThreads;
+}
 
 __global__ void __launch_bounds__(kRouteThreads) route_fill_kernel(PathArgs a, SparseArgs s) {
   const int g = blockIdx.x, m = blockIdx.y, grp = a.g0 + g, E = a.d.E, b = g * E + m;
   if (s.plan[1] == 0) return;
   const int n_rows = n_rows_of(a);
-  const int r_lo = blockIdx.z * kFillChunk;
+  const int chunk = fill_chunk_rows(a.d.tiles_max * kTileM);
+  const int r_lo = blockIdx.z * chunk;
   const int base = s.row0[b], count = s.counts[b];
   uint16_t* g16 = static_cast<uint16_t*>(s.gate16p);
   if (blockIdx.z == 0) {   // padding rows of the bucket's last pair tile
@@ -180,7 +192,7 @@ __global__ void __launch_bounds__(kRouteThreads) route_fill_kernel(PathArgs a, S
   int before = 0;
   for (int r = threadIdx.x; r < r_lo; r += kRouteThreads) before += (sel[r] >> m) & 1u;
   before = block_sum(before, s_warp);
-  const int r_hi = min(n_rows, r_lo + kFillChunk);
+  const int r_hi = min(n_rows, r_lo + chunk);
   int done = 0;
   for (int r0 = r_lo; r0 < r_hi; r0 += kRouteThreads) {
     const int r = r0 + threadIdx.x;
@@ -287,13 +299,14 @@ __global__ void combine_kernel(PathArgs a, SparseArgs s) {
 cudaError_t launch_route(const PathArgs& a, const SparseArgs& s, int step, cudaStream_t st) {
   if (a.gp <= 0) return cudaSuccess;
   const dim3 grid(a.gp, a.d.E);
-  if (step == 0)
+  if (step == 0) {
     route_count_kernel<<<grid, kRouteThreads, 0, st>>>(a, s);
-  else if (step == 1)
+  } else if (step == 1) {
     route_plan_kernel<<<1, kRouteThreads, 0, st>>>(a, s);
-  else
-    route_fill_kernel<<<dim3(a.gp, a.d.E, (a.d.tiles_max * kTileM + kFillChunk - 1) / kFillChunk),
-                        kRouteThreads, 0, st>>>(a, s);
+  } else {
+    const int rows_max = a.d.tiles_max * kTileM, chunk = fill_chunk_rows(rows_max);
+    route_fill_kernel<<<dim3(a.gp, a.d.E, (rows_max + chunk - 1) / chunk), kRouteThreads, 0, st>>>(a, s);
+  }
   return cudaGetLastError();
 }
 

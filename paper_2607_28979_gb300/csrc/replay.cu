@@ -43,24 +43,27 @@
 //                         MN-major); normalised rows out. Lanes synchronise on
 //                         their own named barriers only.
 //   replay_fmha_kernel    full causal attention on the tensor cores (layers below
-//                         L_Full): one CTA per (b, query head, 128-query tile),
-//                         persistent over its key tiles 0..diagonal.
-//                           warp 0  TMA: the Q tile once, then K and V^T tiles
+//                         L_Full): one CTA per (b, query head, pair of consecutive
+//                         128-query tiles), persistent over key tiles 0..the
+//                         second tile's diagonal; each key tile serves both.
+//                           warp 0  TMA: the two Q tiles once, then K and V^T tiles
 //                                   (V transposed per layer by replay_vt_kernel so
 //                                   both MMAs read K-major operands) into 2 stages;
-//                           warp 1  S = Q K^T (M=128, N=128 keys) into double-
-//                                   buffered TMEM and, one tile later, O += P V
-//                                   (M=128, N=d) accumulated in TMEM;
-//                           warps 4..11 two threads per query row, each half of
-//                                   its keys and of its output columns: the scaled,
-//                                   masked scores from TMEM, the row's running max
-//                                   (the halves' maxima traded through TMEM) and
-//                                   sum (base-2 exponentials on ex2.approx), P as
-//                                   bf16 into a 128B-swizzled SMEM tile for the
-//                                   second MMA. The running max rises only when a
-//                                   tile's max exceeds it by more than 2^8, and only
-//                                   then are the sum and the O row in TMEM rescaled;
-//                                   O is read from TMEM once, at the end.
+//                           warp 1  per query tile t: S_t = Q_t K^T (M=128, N=128
+//                                   keys) into TMEM, then O_t += P_t V (M=128, N=d)
+//                                   with P_t read from TMEM, accumulated in TMEM;
+//                                   the two tiles alternate, so the tensor core
+//                                   works on one while the other's softmax runs;
+//                           warps 4..19 eight per query tile, two threads per query
+//                                   row, each half of its keys and of its output
+//                                   columns: the scaled, masked scores from TMEM, the
+//                                   row's running max (the halves' maxima traded
+//                                   through shared memory) and sum (base-2
+//                                   exponentials on ex2.approx), P as bf16 pairs
+//                                   written back over the scores' TMEM columns. The running max rises
+//                                   only when a tile's max exceeds it by more than
+//                                   2^8, and only then are the sum and the O row in
+//                                   TMEM rescaled; O is read from TMEM once, at the end.
 //                         Every wait is bounded; on a timeout the roles unwind,
 //                         copies and MMAs in flight are drained and TMEM is freed.
 #include <cuda_bf16.h>
@@ -570,31 +573,17 @@ __global__ void __launch_bounds__(256) replay_vt_kernel(const uint16_t* __restri
 
 template <int D>
 struct Fa {
-  static constexpr int kQ = 128 * D * 2;      // Q tile: D/64 blocks of 128 rows x 128 B
+  static constexpr int kQ = 128 * D * 2;      // one Q tile: D/64 blocks of 128 rows x 128 B
   static constexpr int kK = 128 * D * 2;      // K tile, same layout
   static constexpr int kVtBlk = D * 128;      // one V^T block: D rows x 64 keys
   static constexpr int kVt = 2 * kVtBlk;      // V^T tile: 128 keys
-  static constexpr int kPBlk = 128 * 128;     // one P block: 128 rows x 64 keys
-  static constexpr int kP = 2 * kPBlk;
-  static constexpr int kBytes = kQ + 2 * kK + 2 * kVt + 2 * kP;
-  static constexpr int kSmem = kBytes + 256 + 1024;
-  static constexpr int kThreads = 384;   // 4 role warps, 8 softmax warps (two per lane quarter)
+  static constexpr int kBytes = 2 * kQ + 2 * kK + 2 * kVt;   // two Q tiles, two K/V^T stages
+  static constexpr int kXch = 1536 * 4;   // softmax exchange: per tile [2][2][128] maxima, [2][128] sums
+  static constexpr int kSmem = kBytes + 256 + kXch + 1024;
+  static constexpr int kThreads = 640;   // 4 role warps, then 8 softmax warps per query tile
 };
 static_assert(Fa<128>::kSmem <= 232448, "shared memory budget");
 static_assert(Fa<64>::kThreads == Fa<128>::kThreads, "one launch size for both head widths");
-
-// One 32-bit TMEM column of the thread's lane (warp-collective, 32x32b shape).
-__device__ __forceinline__ void tmem_st_x1(uint32_t taddr, float v) {
-  asm volatile("tcgen05.st.sync.aligned.32x32b.x1.b32 [%0], {%1};" ::"r"(taddr), "r"(__float_as_uint(v))
-               : "memory");
-}
-
-__device__ __forceinline__ float tmem_ld_x1(uint32_t taddr) {
-  uint32_t v;
-  asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(v) : "r"(taddr) : "memory");
-  asm volatile("tcgen05.wait::ld.sync.aligned;" : "+r"(v)::"memory");
-  return __uint_as_float(v);
-}
 
 // Named barrier `id` over `n` threads, and the same returning the AND of `p`.
 __device__ __forceinline__ void lane_sync_n(int id, int n) {
@@ -614,7 +603,7 @@ __device__ __forceinline__ bool lane_and_n(int id, int n, bool p) {
   return r != 0;
 }
 
-// Each thread of the warp writes 32 consecutive 32-bit columns of its TMEM lane.
+// Each thread of the warp writes 32 (16) consecutive 32-bit columns of its TMEM lane.
 __device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
@@ -627,20 +616,93 @@ __device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const uint32_
       : "memory");
 }
 
+__device__ __forceinline__ void tmem_st_32x32b_x16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
 __device__ __forceinline__ void tmem_st_wait() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-// chunk store of 32 bf16 (16 words) into row r of a 128B-swizzled 64-column block,
-// half s (columns 32 s .. 32 s + 31)
-__device__ __forceinline__ void st_sw128_half(uint32_t blk, int r, int s, const uint32_t (&pk)[16]) {
-  const uint32_t row = blk + static_cast<uint32_t>(r * 128);
-#pragma unroll
-  for (int v = 0; v < 4; ++v)
-    st_shared_v4(row + static_cast<uint32_t>(((4 * s + v) ^ (r & 7)) << 4), pk[4 * v],
-                 pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+// mbar_wait for the role warps of the attention kernel: each poll may suspend
+// the warp (up to 0.5 us, ended early when the phase completes), so waiting
+// warps leave the issue slots of their sub-partition to the softmax warps.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar_addr, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar_addr), "r"(parity), "r"(500u)
+      : "memory");
+  return ok != 0;
 }
 
+__device__ __forceinline__ bool mbar_wait_sleep(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
+                                                long long limit) {
+  const uint32_t a = smem_u32(bar);
+  const long long t0 = clock64();
+  while (!mbar_try_wait_sleep(a, parity)) {
+    if (*abort_flag) return false;
+    if (clock64() - t0 > limit) {
+      *abort_flag = 1;
+      return false;
+    }
+  }
+  return true;
+}
+
+// One 32-key chunk (keys k0 .. k0 + 31 of the tile) of a query row's scores v, in
+// its softmax: the running maxima of 8 independent chains, and the bf16 pairs of
+// P = exp2(s * sl2 - m) with the partial sums of the rounded values (the ones the
+// second MMA uses) in 4 chains. DIAG: the diagonal tile, whose keys past the row r
+// are masked (on other tiles every key counts, with no per-key test).
+template <bool DIAG>
+__device__ __forceinline__ void chunk_max(const uint32_t (&v)[32], int k0, int r, float (&mk)[8]) {
+#pragma unroll
+  for (int k = 0; k < 32; ++k)
+    if (!DIAG || k0 + k <= r) mk[k & 7] = fmaxf(mk[k & 7], __uint_as_float(v[k]));
+}
+
+template <bool DIAG>
+__device__ __forceinline__ void chunk_p(const uint32_t (&v)[32], int k0, int r, float sl2, float m,
+                                        uint32_t (&pk)[16], float (&sk)[4]) {
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    const float p0 = (!DIAG || k0 + 2 * k <= r) ? ex2_fast(__uint_as_float(v[2 * k]) * sl2 - m) : 0.f;
+    const float p1 = (!DIAG || k0 + 2 * k + 1 <= r) ? ex2_fast(__uint_as_float(v[2 * k + 1]) * sl2 - m) : 0.f;
+    __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
+    const float2 pr = __bfloat1622float2(pb);
+    sk[k & 3] += pr.x + pr.y;
+    pk[k] = *reinterpret_cast<uint32_t*>(&pb);
+  }
+}
+
+// D[tmem] (+)= A[tmem] * B[smem]^T, issued by a single thread: A (M = 128 rows,
+// 16-bit elements, two consecutive K values per 32-bit column) is read from the
+// lanes of the issuing CTA's tensor memory.
+__device__ __forceinline__ void umma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                             uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// One CTA per (b, query head, pair of consecutive 128-query tiles qa = 2 i and
+// qb = 2 i + 1), persistent over key tiles 0..qb; each K / V^T tile serves both
+// query tiles. Tensor memory (512 columns): S_t of tile t at columns 128 t, its
+// bf16 probabilities P_t for keys 64 h .. 64 h + 63 written over columns 128 t +
+// 64 h .. + 31 (two keys per 32-bit column), O_t at 256 + 128 t. The second MMA
+// reads P_t from tensor memory.
 template <int D>
 __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
     replay_fmha_kernel(const __grid_constant__ CUtensorMap tmQ,
@@ -649,35 +711,36 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint8_t* sQ = smem;
-  uint8_t* sK = sQ + Fa<D>::kQ;              // [2]
-  uint8_t* sV = sK + 2 * Fa<D>::kK;          // [2]
-  uint8_t* sP = sV + 2 * Fa<D>::kVt;         // [2]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + 2 * Fa<D>::kP);
+  uint8_t* sQ = smem;                        // [2] query tiles
+  uint8_t* sK = sQ + 2 * Fa<D>::kQ;          // [2] stages
+  uint8_t* sV = sK + 2 * Fa<D>::kK;          // [2] stages
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sV + 2 * Fa<D>::kVt);
   uint64_t* q_full = bars;
-  uint64_t* kv_full = bars + 1;      // [2]
-  uint64_t* kv_empty = bars + 3;     // [2]
-  uint64_t* s_full = bars + 5;       // [2]
-  uint64_t* s_empty = bars + 7;      // [2]
-  uint64_t* p_full = bars + 9;       // [2]
-  uint64_t* p_empty = bars + 11;     // [2]
-  uint64_t* pv_done = bars + 13;     // phase j: PV_j has been added into O
-  uint64_t* drain = bars + 17;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
+  uint64_t* kv_full = bars + 1;      // [2] by stage
+  uint64_t* kv_empty = bars + 3;     // [2] by stage
+  uint64_t* s_full = bars + 5;       // [2] by query tile: S_t of its current key tile written
+  uint64_t* p_full = bars + 7;       // [2] by query tile: P_t written (its 4 softmax warps)
+  uint64_t* pv_done = bars + 9;      // [2] by query tile: phase j, P_t V_j added into O_t
+  uint64_t* drain = bars + 11;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 12);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  float* xch = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);   // Fa::kXch bytes
 
   const ReplayDims& d = a.d;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_qt = (d.N + 127) / 128;
-  const int qt = n_qt - 1 - static_cast<int>(blockIdx.x % n_qt);   // heavy tiles first
-  const int bh = static_cast<int>(blockIdx.x / n_qt);
+  const int n_pr = (n_qt + 1) / 2;
+  const int pr = n_pr - 1 - static_cast<int>(blockIdx.x % n_pr);   // heavy pairs first
+  const int bh = static_cast<int>(blockIdx.x / n_pr);
   const int b = bh / d.Hq, h = bh - b * d.Hq;
   const int hk = h / (d.Hq / d.Hkv);
   const int L = seq_len_of(a, b);
-  const int q0 = qt * 128;
-  if (q0 >= L) return;   // uniform over the CTA: no barrier or TMEM use yet
-  const int n_kv = qt + 1;
+  const int qa = 2 * pr, qb = qa + 1;
+  if (qa * 128 >= L) return;   // uniform over the CTA: no barrier or TMEM use yet
+  const bool has_b = qb < n_qt && qb * 128 < L;
+  const int n_kv = has_b ? qb + 1 : qa + 1;   // key tiles 0 .. the last active diagonal
   const long long wl = a.wait_limit;
+  auto active = [&](int t, int j) -> bool { return t == 0 ? j <= qa : (has_b && j <= qb); };
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
@@ -685,12 +748,9 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
       mbar_init(&kv_full[i], 1);
       mbar_init(&kv_empty[i], 1);
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_empty[i], Fa<D>::kThreads / 32 - 4);   // every softmax warp
-      mbar_init(&p_full[i], Fa<D>::kThreads / 32 - 4);
-      mbar_init(&p_empty[i], 1);
-
+      mbar_init(&p_full[i], 8);   // the tile's softmax warps
+      mbar_init(&pv_done[i], 1);
     }
-    mbar_init(pv_done, 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_barrier_init();
@@ -707,21 +767,22 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = *tmem_slot;   // S[i] at columns 128 i, O at 256 (D columns)
+  const uint32_t tmem = *tmem_slot;
   uint32_t issued_mask = 0, issue_parity = 0;
   bool mma_issued = false;
 
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------ TMA producer
-      const int qrow = (b * d.Hq + h) * d.N + q0;
-      mbar_arrive_expect_tx(q_full, Fa<D>::kQ);
-      for (int kb = 0; kb < D / 64; ++kb)
-        tma_load_2d(sQ + kb * 128 * 128, &tmQ, q_full, kb * 64, qrow);
+      const int qrow = (b * d.Hq + h) * d.N + qa * 128;
+      mbar_arrive_expect_tx(q_full, (has_b ? 2 : 1) * Fa<D>::kQ);
+      for (int t = 0; t < (has_b ? 2 : 1); ++t)
+        for (int kb = 0; kb < D / 64; ++kb)
+          tma_load_2d(sQ + t * Fa<D>::kQ + kb * 128 * 128, &tmQ, q_full, kb * 64, qrow + t * 128);
       const int krow = (b * d.Hkv + hk) * d.N, vrow = (b * d.Hkv + hk) * D;
       for (int j = 0; j < n_kv; ++j) {
         const int st = j & 1;
-        if (!mbar_wait(&kv_empty[st], ((j >> 1) & 1) ^ 1u, abort_flag, wl)) break;
+        if (!mbar_wait_sleep(&kv_empty[st], ((j >> 1) & 1) ^ 1u, abort_flag, wl)) break;
         mbar_arrive_expect_tx(&kv_full[st], Fa<D>::kK + Fa<D>::kVt);
         for (int kb = 0; kb < D / 64; ++kb)
           tma_load_2d(sK + st * Fa<D>::kK + kb * 128 * 128, &tmK, &kv_full[st], kb * 64,
@@ -735,187 +796,192 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
     }
   } else if (warp == 1) {
     // ------------------------------------------------ MMA issuer (warp-uniform, elected lane)
+    // Order: S_0(0), S_1(0), then per key tile j: O_0 += P_0 V_j, S_0(j + 1),
+    // O_1 += P_1 V_j, S_1(j + 1); while one tile's softmax runs, the tensor core
+    // works on the other tile. S_t(j + 1) overwrites P_t, and MMAs with different
+    // accumulators are not ordered by issue, so it waits until O_t += P_t V_j is done.
     const uint32_t idS = idesc_bf16_f32(128, 128), idPV = idesc_bf16_f32(128, D);
     bool ok = mbar_wait(q_full, 0, abort_flag, wl);
     tc_fence_after();
-    auto issue_s = [&](int j) -> bool {   // S[j & 1] = Q K_j^T
+    auto issue_s = [&](int t, int j) -> bool {   // S_t = Q_t K_j^T
       const int st = j & 1;
       if (!mbar_wait(&kv_full[st], (j >> 1) & 1, abort_flag, wl)) return false;
-      if (!mbar_wait(&s_empty[st], ((j >> 1) & 1) ^ 1u, abort_flag, wl)) return false;
       tc_fence_after();
       if (elect_one()) {
         for (int kb = 0; kb < D / 64; ++kb) {
-          const uint64_t ad = sdesc_k_sw128(smem_u32(sQ + kb * 128 * 128));
+          const uint64_t ad = sdesc_k_sw128(smem_u32(sQ + t * Fa<D>::kQ + kb * 128 * 128));
           const uint64_t bd = sdesc_k_sw128(smem_u32(sK + st * Fa<D>::kK + kb * 128 * 128));
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            umma_bf16(tmem + st * 128, ad + 2 * k, bd + 2 * k, idS, (kb | k) != 0);
+            umma_bf16(tmem + t * 128, ad + 2 * k, bd + 2 * k, idS, (kb | k) != 0);
         }
-        umma_commit(&s_full[st]);
+        umma_commit(&s_full[t]);
       }
       __syncwarp();
       mma_issued = true;
       return true;
     };
-    auto issue_pv = [&](int j) -> bool {   // O += P_j V_j (B = V_j^T, K-major); tile 0 overwrites
+    // O_t += P_t V_j (B = V_j^T, K-major; P_t from TMEM); key tile 0 overwrites.
+    // `last`: the last MMA that reads stage j & 1, which it then releases.
+    auto issue_pv = [&](int t, int j, bool last) -> bool {
       const int st = j & 1;
-      if (!mbar_wait(&p_full[st], (j >> 1) & 1, abort_flag, wl)) return false;
+      if (!mbar_wait(&p_full[t], j & 1, abort_flag, wl)) return false;
       tc_fence_after();
       if (elect_one()) {
         for (int kb = 0; kb < 2; ++kb) {
-          const uint64_t ad = sdesc_k_sw128(smem_u32(sP + st * Fa<D>::kP + kb * Fa<D>::kPBlk));
-          const uint64_t bd =
-              sdesc_k_sw128(smem_u32(sV + st * Fa<D>::kVt + kb * Fa<D>::kVtBlk));
+          const uint64_t bd = sdesc_k_sw128(smem_u32(sV + st * Fa<D>::kVt + kb * Fa<D>::kVtBlk));
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
-            umma_bf16(tmem + 256, ad + 2 * k, bd + 2 * k, idPV, (j | kb | k) != 0);
+          for (int k = 0; k < 4; ++k)   // keys 64 kb + 16 k .. + 15: P columns 64 kb + 8 k
+            umma_bf16_ts(tmem + 256 + t * 128, tmem + t * 128 + kb * 64 + k * 8, bd + 2 * k, idPV,
+                         (j | kb | k) != 0);
         }
-        umma_commit(pv_done);
-        umma_commit(&p_empty[st]);
-        umma_commit(&kv_empty[st]);
+        umma_commit(&pv_done[t]);
+        if (last) umma_commit(&kv_empty[st]);
       }
       __syncwarp();
       return true;
     };
-    if (ok) ok = issue_s(0);
+    if (ok) ok = issue_s(0, 0);
+    if (ok && has_b) ok = issue_s(1, 0);
     for (int j = 0; ok && j < n_kv; ++j) {
-      if (j + 1 < n_kv) ok = issue_s(j + 1);
-      if (ok) ok = issue_pv(j);
+      for (int t = 0; ok && t < 2; ++t) {
+        if (!active(t, j)) continue;
+        ok = issue_pv(t, j, t == 1 || !active(1, j));
+        if (ok && active(t, j + 1))
+          ok = mbar_wait(&pv_done[t], j & 1, abort_flag, wl) && issue_s(t, j + 1);
+      }
     }
   } else if (warp >= 4) {
     // ------------------------------------------------ softmax and output rows
-    // O accumulates in TMEM across key tiles. A row's running max m is raised
-    // only when a tile's max exceeds it by more than kTau (base 2), so every
-    // probability exp2(s - m) stays below 2^kTau; raising it rescales the row's
-    // sum and its O row in TMEM (after the previous tile's PV has landed).
-    // Warps 4 + 4 hh + q (hh = 0, 1) share TMEM lane quarter q: thread (hh, row)
-    // takes keys and output columns [64 hh, 64 hh + 64) of the row. The pair trades
-    // its partial maxima through TMEM columns 384.. of the row's lane (double-buffered
-    // by tile parity; S and O use columns 0..383) and adds its partial sums at the end;
-    // both threads of a row therefore take the same max and the same rescaling decisions. Every per-tile wait is agreed
-    // on by all softmax warps (bar.red.and) before the pair barrier.
+    // Warps 4 + 8 t + 4 hh + q take query tile t, TMEM lane quarter q; the two
+    // threads (hh = 0, 1) of a query row each take half of a tile's keys (64 hh ..
+    // 64 hh + 63) and half of the output columns. P for keys 64 hh .. goes over the
+    // first 32 of the half's own 64 score columns, so neither thread writes where
+    // the other reads. The halves trade their partial maxima through shared memory
+    // (double-buffered by key-tile parity) and add their partial sums at the end,
+    // so both take the same max and the same rescaling decisions. O_t accumulates
+    // in TMEM across key tiles. A row's running max m is raised only when a tile's
+    // max exceeds it by more than kTau (base 2), so every probability exp2(s - m)
+    // stays below 2^kTau; raising it rescales the row's sum and its O row in TMEM
+    // (after the previous tile's PV has landed). Every wait is agreed on by the
+    // tile's eight warps (bar.red.and on named barrier 1 + t) before they pair.
     constexpr float kTau = 8.f;
-    constexpr int kSmWarps = Fa<D>::kThreads / 32 - 4;   // 8
-    constexpr int H = D / 2;                               // output columns per thread
-    const int q = warp & 3, hh = (warp - 4) >> 2;
-    const int r = q * 32 + lane;
-    const uint32_t lanes = static_cast<uint32_t>(q * 32) << 16;
-    const float sl2 = rsqrtf(float(D)) * 1.4426950408889634f;   // scale * log2(e)
-    float m = -INFINITY, l = 0.f;
-    bool ok = true;
-    auto agree = [&](bool p) -> bool { return lane_and_n(1, 32 * kSmWarps, p); };
-    auto wait_lane0 = [&](uint64_t* bar, uint32_t par) -> bool {
-      int w = 1;
-      if (lane == 0) w = mbar_wait(bar, par, abort_flag, wl) ? 1 : 0;
-      return __shfl_sync(0xffffffffu, w, 0) != 0;
-    };
-    for (int j = 0; j < n_kv; ++j) {
-      const int st = j & 1;
-      if (!agree(wait_lane0(&s_full[st], (j >> 1) & 1))) { ok = false; break; }
-      tc_fence_after();
-      const bool diag = j == qt;
-      // pass 1: the maximum of this thread's 64 scaled, masked scores, then the row's
-      float mx = -INFINITY;
-#pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(tmem + lanes + st * 128 + hh * 64 + c * 32, v);
-        tmem_ld_wait(v);
-#pragma unroll
-        for (int k = 0; k < 32; ++k)
-          if (!diag || hh * 64 + c * 32 + k <= r) mx = fmaxf(mx, __uint_as_float(v[k]) * sl2);
-      }
-      const uint32_t xcol = tmem + lanes + 384 + 2 * static_cast<uint32_t>(j & 1);
-      tmem_st_x1(xcol + hh, mx);
-      tmem_st_wait();
-      tc_fence_before();
-      lane_sync_n(1, 32 * kSmWarps);
-      tc_fence_after();
-      mx = fmaxf(mx, tmem_ld_x1(xcol + (hh ^ 1)));
-      const bool raise = mx > m + kTau;   // always on the first tile (m = -inf)
-      const float alpha = (raise && m != -INFINITY) ? ex2_fast(m - mx) : 1.f;
-      const bool rescale = __any_sync(0xffffffffu, alpha != 1.f);
-      // rescaling needs PV_{j-1} in O; writing P_j needs PV_{j-2} done with the buffer
-      bool w = !rescale || wait_lane0(pv_done, static_cast<uint32_t>(j - 1) & 1u);
-      w = w && wait_lane0(&p_empty[st], ((j >> 1) & 1) ^ 1u);
-      if (!agree(w)) { ok = false; break; }
-      if (rescale) {
+    constexpr int H = D / 2;   // output columns per thread
+    const int t = (warp - 4) >> 3, hh = ((warp - 4) >> 2) & 1, q = warp & 3;
+    if (t == 0 || has_b) {
+      const int qt = t == 0 ? qa : qb;
+      const int r = q * 32 + lane;
+      const uint32_t lanes = static_cast<uint32_t>(q * 32) << 16;
+      const uint32_t tS = tmem + lanes + t * 128 + hh * 64, tO = tmem + lanes + 256 + t * 128 + hh * H;
+      float* xm = xch + t * 512;          // [parity][hh][row] partial maxima
+      float* xl = xch + 1024 + t * 256;   // [hh][row] partial sums
+      const float sl2 = rsqrtf(float(D)) * 1.4426950408889634f;   // scale * log2(e)
+      const int k0 = hh * 64;             // this half's first key
+      float m = -INFINITY, l = 0.f;
+      bool ok = true;
+      auto agree = [&](bool p) -> bool { return lane_and_n(1 + t, 256, p); };
+      auto wait_lane0 = [&](uint64_t* bar, uint32_t par) -> bool {
+        int w = 1;
+        if (lane == 0) w = mbar_wait_sleep(bar, par, abort_flag, wl) ? 1 : 0;
+        return __shfl_sync(0xffffffffu, w, 0) != 0;
+      };
+      for (int j = 0; j <= qt; ++j) {
+        if (!agree(wait_lane0(&s_full[t], j & 1))) { ok = false; break; }
         tc_fence_after();
+        const bool diag = j == qt;
+        // the maximum of this half's masked scores in 8 independent chains
+        float mk[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) mk[e] = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(tS + c * 32, v);
+          tmem_ld_wait(v);
+          if (diag)
+            chunk_max<true>(v, k0 + c * 32, r, mk);
+          else
+            chunk_max<false>(v, k0 + c * 32, r, mk);
+        }
+        const float pm = fmaxf(fmaxf(fmaxf(mk[0], mk[1]), fmaxf(mk[2], mk[3])),
+                               fmaxf(fmaxf(mk[4], mk[5]), fmaxf(mk[6], mk[7])));
+        float* xmj = xm + (j & 1) * 256;
+        xmj[hh * 128 + r] = pm;
+        lane_sync_n(1 + t, 256);
+        // the row's max of the scaled scores (the scale is positive: scaled after the comparison)
+        const float mx = fmaxf(pm, xmj[(hh ^ 1) * 128 + r]) * sl2;
+        const bool raise = mx > m + kTau;   // always on the first tile (m = -inf)
+        const float alpha = (raise && m != -INFINITY) ? ex2_fast(m - mx) : 1.f;
+        const bool rescale = __any_sync(0xffffffffu, alpha != 1.f);
+        // rescaling needs P_t V_{j-1} in O_t
+        if (!agree(!rescale || wait_lane0(&pv_done[t], static_cast<uint32_t>(j - 1) & 1u))) {
+          ok = false;
+          break;
+        }
+        if (rescale) {
+          tc_fence_after();
+#pragma unroll
+          for (int c = 0; c < H / 32; ++c) {
+            uint32_t o[32];
+            tmem_ld_32x32b_x32(tO + c * 32, o);
+            tmem_ld_wait(o);
+#pragma unroll
+            for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * alpha);
+            tmem_st_32x32b_x32(tO + c * 32, o);
+          }
+        }
+        l *= alpha;
+        if (raise) m = mx;
+        // P = exp2(s - m) as bf16 pairs: chunk c's 16 words go to columns 16 c .. of the
+        // half's own scores, which this thread has already read
+        float sk[4] = {0.f, 0.f, 0.f, 0.f};   // partial sums of the rounded probabilities
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(tS + c * 32, v);
+          tmem_ld_wait(v);
+          uint32_t pk[16];
+          if (diag)
+            chunk_p<true>(v, k0 + c * 32, r, sl2, m, pk, sk);
+          else
+            chunk_p<false>(v, k0 + c * 32, r, sl2, m, pk, sk);
+          tmem_st_32x32b_x16(tS + c * 16, pk);
+        }
+        tmem_st_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[t]);
+        l += (sk[0] + sk[1]) + (sk[2] + sk[3]);
+      }
+      // the tile's warps all take part (ok is uniform over them: the loop's exits are agreed)
+      const bool done = agree(ok && wait_lane0(&pv_done[t], static_cast<uint32_t>(qt) & 1u));
+      if (done) {
+        tc_fence_after();
+        // the row's sum: this half's plus the partner's
+        xl[hh * 128 + r] = l;
+        lane_sync_n(1 + t, 256);
+        l += xl[(hh ^ 1) * 128 + r];
+        const int qq = qt * 128 + r;
+        const float inv = 1.f / l;
+        uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.out) +
+                                              ((int64_t(b) * d.Hq + h) * d.N + qq) * D + hh * H);
 #pragma unroll
         for (int c = 0; c < H / 32; ++c) {
           uint32_t v[32];
-          tmem_ld_32x32b_x32(tmem + lanes + 256 + hh * H + c * 32, v);
+          tmem_ld_32x32b_x32(tO + c * 32, v);
           tmem_ld_wait(v);
+          if (qq < L) {
 #pragma unroll
-          for (int k = 0; k < 32; ++k) v[k] = __float_as_uint(__uint_as_float(v[k]) * alpha);
-          tmem_st_32x32b_x32(tmem + lanes + 256 + hh * H + c * 32, v);
-        }
-        tmem_st_wait();
-      }
-      l *= alpha;
-      if (raise) m = mx;
-      // pass 2: P = exp2(s - m) as bf16 into block hh of the swizzled P tile, and the partial sum
-      float sum = 0.f;
-      const uint32_t pbase = smem_u32(sP + st * Fa<D>::kP) + static_cast<uint32_t>(hh * Fa<D>::kPBlk);
+            for (int e8 = 0; e8 < 4; ++e8) {
+              uint32_t w4[4];
 #pragma unroll
-      for (int c = 0; c < 2; ++c) {
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(tmem + lanes + st * 128 + hh * 64 + c * 32, v);
-        tmem_ld_wait(v);
-        uint32_t pk[16];
-#pragma unroll
-        for (int k = 0; k < 16; ++k) {
-          const int c0 = hh * 64 + c * 32 + 2 * k;
-          const float p0 = (!diag || c0 <= r) ? ex2_fast(__uint_as_float(v[2 * k]) * sl2 - m) : 0.f;
-          const float p1 = (!diag || c0 + 1 <= r) ? ex2_fast(__uint_as_float(v[2 * k + 1]) * sl2 - m) : 0.f;
-          __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
-          // the row sum counts the rounded probabilities the second MMA uses
-          const float2 pr = __bfloat1622float2(pb);
-          sum += pr.x + pr.y;
-          pk[k] = *reinterpret_cast<uint32_t*>(&pb);
-        }
-        st_sw128_half(pbase, r, c, pk);
-      }
-      tc_fence_before();
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&s_empty[st]);
-        mbar_arrive(&p_full[st]);
-      }
-      l += sum;
-    }
-    // every softmax warp takes part in the agreement (ok is uniform: the loop's exits are agreed)
-    const bool done = agree(ok && wait_lane0(pv_done, static_cast<uint32_t>(n_kv - 1) & 1u));
-    if (done) {
-      tc_fence_after();
-      // the row's sum: this half's plus the partner's (TMEM columns 388, 389)
-      tmem_st_x1(tmem + lanes + 388 + hh, l);
-      tmem_st_wait();
-      tc_fence_before();
-      lane_sync_n(1, 32 * kSmWarps);
-      tc_fence_after();
-      l += tmem_ld_x1(tmem + lanes + 388 + (hh ^ 1));
-      const int qq = q0 + r;
-      const float inv = 1.f / l;
-      uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.out) +
-                                            ((int64_t(b) * d.Hq + h) * d.N + qq) * D + hh * H);
-#pragma unroll
-      for (int c = 0; c < H / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld_32x32b_x32(tmem + lanes + 256 + hh * H + c * 32, v);
-        tmem_ld_wait(v);
-        if (qq < L) {
-#pragma unroll
-          for (int e8 = 0; e8 < 4; ++e8) {
-            uint32_t w4[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              __nv_bfloat162 t = __floats2bfloat162_rn(__uint_as_float(v[8 * e8 + 2 * e]) * inv,
-                                                       __uint_as_float(v[8 * e8 + 2 * e + 1]) * inv);
-              w4[e] = *reinterpret_cast<uint32_t*>(&t);
+              for (int e = 0; e < 4; ++e) {
+                __nv_bfloat162 u = __floats2bfloat162_rn(__uint_as_float(v[8 * e8 + 2 * e]) * inv,
+                                                         __uint_as_float(v[8 * e8 + 2 * e + 1]) * inv);
+                w4[e] = *reinterpret_cast<uint32_t*>(&u);
+              }
+              dst[c * 4 + e8] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
             }
-            dst[c * 4 + e8] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
           }
         }
       }
@@ -1326,8 +1392,8 @@ cudaError_t launch_replay_fmha(const ReplayArgs& a, const CUtensorMap& tmQ, cons
     if (e != cudaSuccess) return e;
     attr[di] = true;
   }
-  const int n_qt = (d.N + 127) / 128;
-  kern<<<d.B * d.Hq * n_qt, Fa<128>::kThreads, smem, st>>>(tmQ, tmK, tmVt, a);
+  const int n_pr = ((d.N + 127) / 128 + 1) / 2;   // pairs of 128-query tiles
+  kern<<<d.B * d.Hq * n_pr, Fa<128>::kThreads, smem, st>>>(tmQ, tmK, tmVt, a);
   return cudaGetLastError();
 }
 

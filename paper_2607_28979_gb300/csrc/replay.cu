@@ -661,8 +661,8 @@ __device__ __forceinline__ bool mbar_wait_sleep(uint64_t* bar, uint32_t parity, 
 // One 32-key chunk (keys k0 .. k0 + 31 of the tile) of a query row's scores v, in
 // its softmax: the running maxima of 8 independent chains, and the bf16 pairs of
 // P = exp2(s * sl2 - m) with the partial sums of the rounded values (the ones the
-// second MMA uses) in 4 chains. DIAG: the diagonal tile, whose keys past the row r
-// are masked (on other tiles every key counts, with no per-key test).
+// second MMA uses) in 2 chains of fp32 pairs. DIAG: the diagonal tile, whose keys
+// past the row r are masked (on other tiles every key counts, with no per-key test).
 template <bool DIAG>
 __device__ __forceinline__ void chunk_max(const uint32_t (&v)[32], int k0, int r, float (&mk)[8]) {
 #pragma unroll
@@ -670,17 +670,35 @@ __device__ __forceinline__ void chunk_max(const uint32_t (&v)[32], int k0, int r
     if (!DIAG || k0 + k <= r) mk[k & 7] = fmaxf(mk[k & 7], __uint_as_float(v[k]));
 }
 
+// Packed pairs of fp32 (sm_100 family): d = a * b + c and d = a + b per lane.
+__device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
+  return (static_cast<uint64_t>(__float_as_uint(hi)) << 32) | __float_as_uint(lo);
+}
+__device__ __forceinline__ uint64_t ffma_x2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fadd_x2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 template <bool DIAG>
 __device__ __forceinline__ void chunk_p(const uint32_t (&v)[32], int k0, int r, float sl2, float m,
-                                        uint32_t (&pk)[16], float (&sk)[4]) {
+                                        uint32_t (&pk)[16], uint64_t (&sk)[2]) {
+  const uint64_t s2 = f32x2(sl2, sl2), nm2 = f32x2(-m, -m);
 #pragma unroll
   for (int k = 0; k < 16; ++k) {
-    const float p0 = (!DIAG || k0 + 2 * k <= r) ? ex2_fast(__uint_as_float(v[2 * k]) * sl2 - m) : 0.f;
-    const float p1 = (!DIAG || k0 + 2 * k + 1 <= r) ? ex2_fast(__uint_as_float(v[2 * k + 1]) * sl2 - m) : 0.f;
+    const uint64_t x = ffma_x2((static_cast<uint64_t>(v[2 * k + 1]) << 32) | v[2 * k], s2, nm2);
+    const float p0 = (!DIAG || k0 + 2 * k <= r) ? ex2_fast(__uint_as_float(static_cast<uint32_t>(x))) : 0.f;
+    const float p1 = (!DIAG || k0 + 2 * k + 1 <= r) ? ex2_fast(__uint_as_float(static_cast<uint32_t>(x >> 32))) : 0.f;
     __nv_bfloat162 pb = __floats2bfloat162_rn(p0, p1);
-    const float2 pr = __bfloat1622float2(pb);
-    sk[k & 3] += pr.x + pr.y;
-    pk[k] = *reinterpret_cast<uint32_t*>(&pb);
+    const uint32_t w = *reinterpret_cast<uint32_t*>(&pb);
+    pk[k] = w;
+    // the rounded values themselves (bf16 -> fp32 is exact: the bits move up)
+    sk[k & 1] = fadd_x2(sk[k & 1], (static_cast<uint64_t>(w & 0xFFFF0000u) << 32) | (w << 16));
   }
 }
 
@@ -934,7 +952,7 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
         if (raise) m = mx;
         // P = exp2(s - m) as bf16 pairs: chunk c's 16 words go to columns 16 c .. of the
         // half's own scores, which this thread has already read
-        float sk[4] = {0.f, 0.f, 0.f, 0.f};   // partial sums of the rounded probabilities
+        uint64_t sk[2] = {0u, 0u};   // partial sums of the rounded probabilities (fp32 pairs)
 #pragma unroll
         for (int c = 0; c < 2; ++c) {
           uint32_t v[32];
@@ -951,7 +969,8 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&p_full[t]);
-        l += (sk[0] + sk[1]) + (sk[2] + sk[3]);
+        const uint64_t sk2 = fadd_x2(sk[0], sk[1]);
+        l += __uint_as_float(static_cast<uint32_t>(sk2)) + __uint_as_float(static_cast<uint32_t>(sk2 >> 32));
       }
       // the tile's warps all take part (ok is uniform over them: the loop's exits are agreed)
       const bool done = agree(ok && wait_lane0(&pv_done[t], static_cast<uint32_t>(qt) & 1u));

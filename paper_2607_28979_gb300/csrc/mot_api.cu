@@ -1622,18 +1622,16 @@ mot_status mot_replay_attention(mot_handle h, int32_t layer, const void* q, cons
   const ReplayDims& d = h->rd;
   if (full && replay_fmha_supported(d) && encode_fn()) {
     // tensor-core causal attention: V^T first, then one launch over all query tiles
-    CUtensorMap tmQ{}, tmK{}, tmVt{};
-    const uint64_t qd[2] = {uint64_t(d.d), uint64_t(d.B) * d.Hq * d.N};
+    CUtensorMap tmK{}, tmVt{};
     const uint64_t kd[2] = {uint64_t(d.d), uint64_t(d.B) * d.Hkv * d.N};
     const uint64_t vd[2] = {uint64_t(d.N), uint64_t(d.B) * d.Hkv * d.d};
-    const uint64_t qs[1] = {uint64_t(d.d) * 2}, vs[1] = {uint64_t(d.N) * 2};
+    const uint64_t ks[1] = {uint64_t(d.d) * 2}, vs[1] = {uint64_t(d.N) * 2};
     const uint32_t box[2] = {64, 128}, vbox[2] = {64, uint32_t(d.d)};
-    if (!encode_bf16(&tmQ, q, 2, qd, qs, box) || !encode_bf16(&tmK, k, 2, kd, qs, box) ||
-        !encode_bf16(&tmVt, h->rvt, 2, vd, vs, vbox))
+    if (!encode_bf16(&tmK, k, 2, kd, ks, box) || !encode_bf16(&tmVt, h->rvt, 2, vd, vs, vbox))
       return MOT_ERR_CUDA;
     MOT_CUDA_TRY(timed(h, "replay_vt", st, [&] { return launch_replay_vt(a, h->rvt, st); }));
     MOT_CUDA_TRY(timed(h, "replay_fmha_full", st,
-                       [&] { return launch_replay_fmha(a, tmQ, tmK, tmVt, st); }));
+                       [&] { return launch_replay_fmha(a, tmK, tmVt, st); }));
     return MOT_OK;
   }
   if (!full && replay_gattn_supported(d)) {

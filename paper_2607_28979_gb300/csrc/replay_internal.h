@@ -31,12 +31,12 @@ struct ReplayArgs {
   int32_t stall_test;     // test hook: the guided kernel's first CTA stalls its first MMA barrier
 };
 bool replay_supported(const ReplayDims& d);
-// Full causal attention on the tensor cores: maps over q [B*Hq*N][d], k
-// [B*Hkv*N][d] (box 64 x 128) and V^T [B*Hkv*d][N] (box 64 x d), the last
-// written by launch_replay_vt into `vt`.
+// Full causal attention on the tensor cores: maps over k [B*Hkv*N][d] (box
+// 64 x 128) and V^T [B*Hkv*d][N] (box 64 x d), the latter written by
+// launch_replay_vt into `vt`; the query rows are read from a.q (16-byte aligned).
 bool replay_fmha_supported(const ReplayDims& d);
 cudaError_t launch_replay_vt(const ReplayArgs& a, void* vt, cudaStream_t st);
-cudaError_t launch_replay_fmha(const ReplayArgs& a, const CUtensorMap& tmQ, const CUtensorMap& tmK,
+cudaError_t launch_replay_fmha(const ReplayArgs& a, const CUtensorMap& tmK,
                                const CUtensorMap& tmVt, cudaStream_t st);
 cudaError_t launch_replay_select(const ReplayArgs& a, cudaStream_t st);
 // Guided layers on the tensor cores (d = 128, GQA groups of up to 16, S <= 128):

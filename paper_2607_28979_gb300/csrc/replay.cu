@@ -331,12 +331,26 @@ __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(cons
     const uint32_t x = e < 2 ? v.x : e < 4 ? v.y : e < 6 ? v.z : v.w;
     return (e & 1) ? x >> 16 : x & 0xFFFFu;
   };
+  // Rounds r < nfull hold n's positions on every lane (no per-key test). Every key is
+  // at least omin, so subtracting omin from both halves of a packed word borrows
+  // nothing across them: each half holds its own o - omin.
+  const int nfull = n >> 8;
+  const uint32_t omin2 = omin * 0x10001u;
   // top digit
   for (int i = lane; i < kSelCacheCopies * 256; i += 32) hist[w][0][i] = 0;
   __syncwarp();
-  for (int r = 0; r < nr; ++r) {
-    const int lim = min(n - (r * 256 + lane * 8), 8);
+  for (int r = 0; r < nfull; ++r) {
     const uint4 v = kc[r][lane];
+    const uint32_t wd[4] = {v.x - omin2, v.y - omin2, v.z - omin2, v.w - omin2};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      atomicAdd(&hw[(wd[i] & 0xFFFFu) >> sh], 1);
+      atomicAdd(&hw[wd[i] >> (16 + sh)], 1);
+    }
+  }
+  if (nfull < nr) {
+    const int lim = min(n - (nfull * 256 + lane * 8), 8);
+    const uint4 v = kc[nfull][lane];
 #pragma unroll
     for (int e = 0; e < 8; ++e)
       if (e < lim) atomicAdd(&hw[(key_of(v, e) - omin) >> sh], 1);
@@ -344,14 +358,24 @@ __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(cons
   __syncwarp();
   const uint32_t top = kth_bin<kSelCacheCopies>(hist[w], k);
   uint32_t V = omin + (top << sh);
-  if (sh > 0) {   // the low sh bits among the keys of bin `top`
+  if (sh > 0) {   // the low sh bits among the keys of bin `top`: o - omin in [top << sh, + 2^sh)
     __syncwarp();
     for (int i = lane; i < kSelCacheCopies * 256; i += 32) hist[w][0][i] = 0;
     __syncwarp();
-    const uint32_t msk = (1u << sh) - 1u;
-    for (int r = 0; r < nr; ++r) {
-      const int lim = min(n - (r * 256 + lane * 8), 8);
+    const uint32_t msk = (1u << sh) - 1u, lo_b = top << sh;
+    for (int r = 0; r < nfull; ++r) {
       const uint4 v = kc[r][lane];
+      const uint32_t wd[4] = {v.x - omin2, v.y - omin2, v.z - omin2, v.w - omin2};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t a = wd[i] & 0xFFFFu, c = wd[i] >> 16;
+        if (a - lo_b <= msk) atomicAdd(&hw[a & msk], 1);
+        if (c - lo_b <= msk) atomicAdd(&hw[c & msk], 1);
+      }
+    }
+    if (nfull < nr) {
+      const int lim = min(n - (nfull * 256 + lane * 8), 8);
+      const uint4 v = kc[nfull][lane];
 #pragma unroll
       for (int e = 0; e < 8; ++e) {
         const uint32_t o = key_of(v, e) - omin;
@@ -365,16 +389,19 @@ __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(cons
   int base = 0, eq_taken = 0;
   for (int r = 0; r < nr && base < d.S; ++r) {   // warp-uniform
     const int j8 = r * 256 + lane * 8;
-    const int lim = min(n - j8, 8);
     const uint4 v = kc[r][lane];
     uint32_t gt = 0u, eq = 0u;
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
       const uint32_t o = key_of(v, e);
-      if (e < lim) {
-        gt |= uint32_t(o > V) << e;
-        eq |= uint32_t(o == V) << e;
-      }
+      gt |= uint32_t(o > V) << e;
+      eq |= uint32_t(o == V) << e;
+    }
+    if (r == nfull) {   // the partial round: positions past n never count
+      const int lim = min(n - j8, 8);
+      const uint32_t in = lim <= 0 ? 0u : (1u << lim) - 1u;
+      gt &= in;
+      eq &= in;
     }
     uint32_t sel = gt;
     if (__any_sync(0xffffffffu, eq != 0u)) {   // the k lowest positions at the threshold are taken

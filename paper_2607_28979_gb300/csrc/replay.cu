@@ -288,8 +288,29 @@ __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(cons
   const int nr = (n + 255) >> 8;     // rounds holding positions < n (<= kSelCacheRounds)
   uint4 (*kc)[32] = keys[w];
   uint32_t lo = 0xFFFFu, hi = 0u;
+  // Rounds r < nfull hold n's positions on every lane (no per-position test there).
+  const int nfull = n >> 8;
+  int r0 = 0;
+  if (vec) {
+    uint32_t lo1 = 0xFFFFu, hi1 = 0u;
 #pragma unroll 4
-  for (int r = 0; r < nr; ++r) {
+    for (; r0 < nfull; ++r0) {
+      const uint4 v = __ldg(reinterpret_cast<const uint4*>(A + r0 * 256 + lane * 8));
+      const uint32_t q[4] = {ord16x2(v.x), ord16x2(v.y), ord16x2(v.z), ord16x2(v.w)};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        lo = min(lo, q[i] & 0xFFFFu);
+        hi = max(hi, q[i] & 0xFFFFu);
+        lo1 = min(lo1, q[i] >> 16);
+        hi1 = max(hi1, q[i] >> 16);
+      }
+      kc[r0][lane] = make_uint4(q[0], q[1], q[2], q[3]);
+    }
+    lo = min(lo, lo1);
+    hi = max(hi, hi1);
+  }
+#pragma unroll 4
+  for (int r = r0; r < nr; ++r) {
     const int j8 = r * 256 + lane * 8;
     const int lim = min(n - j8, 8);   // this lane's positions < n in the round (may be <= 0)
     uint32_t q[4] = {0u, 0u, 0u, 0u};
@@ -331,10 +352,8 @@ __global__ void __launch_bounds__(32 * kSelCacheWarps) replay_select_kernel(cons
     const uint32_t x = e < 2 ? v.x : e < 4 ? v.y : e < 6 ? v.z : v.w;
     return (e & 1) ? x >> 16 : x & 0xFFFFu;
   };
-  // Rounds r < nfull hold n's positions on every lane (no per-key test). Every key is
-  // at least omin, so subtracting omin from both halves of a packed word borrows
-  // nothing across them: each half holds its own o - omin.
-  const int nfull = n >> 8;
+  // Every key is at least omin, so subtracting omin from both halves of a packed word
+  // borrows nothing across them: each half holds its own o - omin.
   const uint32_t omin2 = omin * 0x10001u;
   // top digit
   for (int i = lane; i < kSelCacheCopies * 256; i += 32) hist[w][0][i] = 0;

@@ -688,9 +688,10 @@ __device__ __forceinline__ void tmem_st_wait() {
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-// mbar_wait for the role warps of the attention kernel: each poll may suspend
-// the warp (up to 0.5 us, ended early when the phase completes), so waiting
-// warps leave the issue slots of their sub-partition to the softmax warps.
+// mbar_wait for the attention kernel's TMA producer and the softmax warps' lane-0
+// waits: each poll may suspend the thread (up to 0.5 us, ended early when the
+// phase completes), so waiting warps leave their sub-partition's issue slots to
+// the softmax warps. The MMA issuer keeps the polling mbar_wait.
 __device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar_addr, uint32_t parity) {
   uint32_t ok;
   asm volatile(

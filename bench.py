@@ -30,6 +30,7 @@ from __future__ import annotations
 
 import argparse
 import hashlib
+import re
 import json
 import os
 import statistics
@@ -176,13 +177,23 @@ KERNEL_SOURCES = {
 }
 
 
+def _code_only(text: str) -> str:
+    """Source text without comments and with runs of whitespace folded, so that an edit
+    to a comment does not count as a kernel change (the sources hold no string with
+    a comment marker in it)."""
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
 def kernel_source_sha(kernel: str) -> str:
+    """Hash of the code (comments left out) of the sources a kernel is built from."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2607_28979_gb300", "csrc")
     for n in KERNEL_SOURCES.get(kernel, sorted(os.listdir(csrc))):
         if n.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, n), "rb") as f:
-                h.update(f.read())
+            with open(os.path.join(csrc, n), encoding="utf-8") as f:
+                h.update(_code_only(f.read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -60,6 +60,14 @@ def test_traffic_records_parse():
     assert bench.recorded_traffic("no_such_kernel", "gpt2s_opt125m") is None
 
 
+def test_kernel_source_hash_ignores_comments_only():
+    """A traffic record stays valid across comment edits, not across code edits."""
+    code = "int f(int x) {\n  return x + 1;  // one more\n}\n/* note */\n"
+    assert bench._code_only(code) == bench._code_only(code.replace("one more", "the successor"))
+    assert bench._code_only(code) == bench._code_only(code.replace("/* note */", "/* a\nlonger note */"))
+    assert bench._code_only(code) != bench._code_only(code.replace("x + 1", "x + 2"))
+
+
 PEAKS = {"hbm_gbs": 6796.5, "bf16_tflops": 1928.9, "bf16_tflops_sustained": 1708.6}
 
 

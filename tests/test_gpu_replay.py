@@ -182,6 +182,38 @@ def test_guided_attention_every_group_size(group):
         assert (o[b, :, L:] == np.int16(G.SENTINEL_BF16)).all()
 
 
+@pytest.mark.parametrize("gain", [0.05, 2.0])
+def test_attention_scores_rising_along_the_context(gain):
+    """Keys that grow along a common direction of the queries, so a query's scores
+    rise with the key position by about `gain` (base 2) per key: the full-attention
+    kernel's running max passes its 2^8 margin on later key tiles and rescales O
+    and the row sum (gain 0.05: every tile or two by a moderate factor; gain 2:
+    every tile, the earlier keys' weight vanishing), and the guided kernel sees
+    rows whose selected scores span hundreds of binades. Against the oracle."""
+    import _helpers as H
+    wl = RW("r_rise", 2, 3, 12, 2, 128, 2, 520, (520, 300), top_s=128, n_full=1)
+    q, k, v = synth.gen_replay_qkv(wl, 23)
+    g = synth.gen_guide(wl, 29)
+    # q . k / sqrt(d) = 128 (gain j / 16) / sqrt(128) ~ 0.7 gain j, about gain j in base 2
+    qf = 0.25 * H.bf16_bits_to_f64(q) + 1.0
+    j = np.arange(wl.max_seq, dtype=np.float64)[None, None, :, None]
+    kf = 0.25 * H.bf16_bits_to_f64(k) + gain * j / 16.0
+    q = H.f32_to_bf16_bits(qf.astype(np.float32))
+    k = H.f32_to_bf16_bits(kf.astype(np.float32))
+    run = ReplayRun(wl)
+    rng = np.random.default_rng(31)
+    for layer in (0, 2):
+        out = run.attend(layer, q, k, v, None if layer < wl.n_full else g)
+        tb, th, tu = [], [], []
+        for b, L in enumerate(wl.seq_lens):
+            us = np.unique(np.concatenate([[0, 127, 128, 255, 256, L - 1], rng.integers(0, L, size=10)]))
+            for u in us:
+                for h in range(wl.q_heads):
+                    tb.append(b); th.append(h); tu.append(u)
+        ref = oracle.replay_tokens(wl, layer, q, k, v, g, tb, th, tu)
+        G.assert_parity(BF16, _f64(out)[tb, th, tu], ref, f"gain {gain} layer {layer}")
+
+
 def test_full_size_layer_sampled():
     """Qwen2.5-0.5B -> 1.5B replay shapes (4 x 4096 context, 12 / 2 heads of 128,
     S = 128): one full and one guided layer, in the benchmark's launch configuration."""

@@ -638,11 +638,7 @@ static_assert(Fa<128>::kSmem <= 232448, "shared memory budget");
 static_assert(Fa<128>::kQcol + 64 <= 512 && Fa<64>::kQcol + 32 <= 512, "TMEM columns");
 static_assert(Fa<64>::kThreads == Fa<128>::kThreads, "one launch size for both head widths");
 
-// Named barrier `id` over `n` threads, and the same returning the AND of `p`.
-__device__ __forceinline__ void lane_sync_n(int id, int n) {
-  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
-}
-
+// Named barrier `id` over `n` threads, returning the AND of `p`.
 __device__ __forceinline__ bool lane_and_n(int id, int n, bool p) {
   uint32_t r;
   asm volatile(
@@ -948,8 +944,8 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
     // than kTau (base 2), so every probability exp2(s - m) stays below 2^kTau;
     // raising it rescales the row's O columns and sum in TMEM (after the previous
     // tile's PV has landed). The four warps of a lane quarter (one per key
-    // quarter) pair on named barrier 1 + q, and agree on every wait first
-    // (bar.red.and), so a timeout stops all four before they pair.
+    // quarter) pair on named barrier 1 + q with bar.red.and, which also agrees on
+    // their waits, so a timeout stops all four together.
     constexpr float kTau = 8.f;
     const int c4 = (warp - 4) >> 2, q = warp & 3;
     const int r = q * 32 + lane;
@@ -1002,34 +998,39 @@ __global__ void __launch_bounds__(Fa<D>::kThreads, 1)
     };
     for (int j = 0; j < n_kv; ++j) {
       const uint32_t tS = tmem + lanes + (j & 1) * 128 + k0;
-      if (!agree(wait_lane0(&s_full[j & 1], static_cast<uint32_t>(j >> 1) & 1u))) { ok = false; break; }
-      tc_fence_after();
+      const bool okw = wait_lane0(&s_full[j & 1], static_cast<uint32_t>(j >> 1) & 1u);
       const bool diag = j == qt;
       uint32_t v[32];
-      tmem_ld_32x32b_x32(tS, v);
-      tmem_ld_wait(v);
-      // the maximum of this quarter's masked scores in 8 independent chains
-      float mk[8];
+      float pm = -INFINITY;
+      if (okw) {
+        tc_fence_after();
+        tmem_ld_32x32b_x32(tS, v);
+        tmem_ld_wait(v);
+        // the maximum of this quarter's masked scores in 8 independent chains
+        float mk[8];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) mk[e] = -INFINITY;
-      if (diag)
-        chunk_max<true>(v, k0, r, mk);
-      else
-        chunk_max<false>(v, k0, r, mk);
+        for (int e = 0; e < 8; ++e) mk[e] = -INFINITY;
+        if (diag)
+          chunk_max<true>(v, k0, r, mk);
+        else
+          chunk_max<false>(v, k0, r, mk);
+        pm = fmaxf(fmax3(mk[0], mk[1], mk[2]), fmax3(mk[3], mk[4], fmax3(mk[5], mk[6], mk[7])));
+      }
       float* xmj = xm + (j & 1) * 512;
-      xmj[c4 * 128 + r] = fmaxf(fmax3(mk[0], mk[1], mk[2]), fmax3(mk[3], mk[4], fmax3(mk[5], mk[6], mk[7])));
-      lane_sync_n(1 + q, 128);
+      xmj[c4 * 128 + r] = pm;
+      // one barrier trades the quarters' maxima and agrees on the four warps' waits
+      if (!agree(okw)) { ok = false; break; }
       // the row's max of the scaled scores (the scale is positive: scaled after the comparison)
       const float mx = fmaxf(fmax3(xmj[r], xmj[128 + r], xmj[256 + r]), xmj[384 + r]) * sl2;
       const bool raise = mx > m + kTau;   // always on the first tile (m = -inf)
       const float alpha = (raise && m != -INFINITY) ? ex2_fast(m - mx) : 1.f;
+      // the same for the quarter's four warps: they hold the same 32 rows
       const bool rescale = __any_sync(0xffffffffu, alpha != 1.f);
-      // rescaling needs P_{j-1} V_{j-1} in O
-      if (!agree(!rescale || wait_lane0(pv_done, static_cast<uint32_t>(j - 1) & 1u))) {
-        ok = false;
-        break;
-      }
-      if (rescale) {
+      if (rescale) {   // needs P_{j-1} V_{j-1} in O
+        if (!agree(wait_lane0(pv_done, static_cast<uint32_t>(j - 1) & 1u))) {
+          ok = false;
+          break;
+        }
         tc_fence_after();
         uint32_t o[OC];
         if constexpr (OC == 32) {

@@ -168,10 +168,13 @@ KERNEL_SOURCES = {
     "umma2_onchip_translate": ["onchip.cu", "umma_common.cuh", "gelu.cuh", "ptx.cuh",
                                "mot_internal.h"],
     "umma2_wide_translate": ["wide.cu", "umma_common.cuh", "gelu.cuh", "ptx.cuh", "mot_internal.h"],
-    # replay stages (all kernels of replay.cu)
-    "replay_attn_sparse": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
-    "replay_select": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
-    "replay_fmha_full": ["replay.cu", "replay_internal.h", "mot_internal.h", "ptx.cuh"],
+    # replay stages: guided attention, selection (with the SIMT kernels), full attention
+    "replay_attn_sparse": ["replay_gattn.cu", "replay_common.cuh", "replay_internal.h",
+                           "mot_internal.h", "ptx.cuh"],
+    "replay_select": ["replay.cu", "replay_common.cuh", "replay_internal.h", "mot_internal.h",
+                      "ptx.cuh"],
+    "replay_fmha_full": ["replay_fmha.cu", "replay_common.cuh", "replay_internal.h",
+                         "mot_internal.h", "ptx.cuh"],
     # backbone translators (all kernels of bt.cu)
     "bt_ffn_fused": ["bt.cu", "bt_internal.h", "gelu.cuh", "mot_internal.h", "ptx.cuh"],
 }

@@ -1,4 +1,5 @@
-// Internal declarations of the replay attention (replay.cu), shared with the C-ABI layer.
+// Internal declarations of the replay attention (replay.cu, replay_fmha.cu,
+// replay_gattn.cu), shared with the C-ABI layer.
 #pragma once
 
 #include "mot_internal.h"
@@ -7,7 +8,7 @@ namespace mot {
 
 // ---------------------------------------------------------------- replay attention
 //
-// App. C.4 (replay.cu): one target layer's attention over the replay cache,
+// App. C.4: one target layer's attention over the replay cache,
 // full causal for layers below L_Full, else over the Top-S positions of the
 // source guidance map's causal row. Layouts: q / out [B][Hq][N][d], k / v
 // [B][Hkv][N][d], guide [B][N][N] (bf16), sel [B][N][S] int32 (ascending
